@@ -1,0 +1,114 @@
+/*
+ * CPU oracle for block-wise diffusion-LLM (LLaDA-style) decoding, as
+ * described in "Efficient On-Device Diffusion LLM Inference with Mobile NPU"
+ * (arXiv 2606.13740), Sec. 2.1 (block-wise decoding, prefix KV reuse) and
+ * Sec. 3.2-3.3 (decoding window, draft tokens, staged stabilisation).
+ *
+ * TEST INFRASTRUCTURE ONLY.  This library is a plain, slow, obviously
+ * correct restatement of what the GPU path computes.  Only the test suite,
+ * the smoke check and the benchmark's CPU-baseline leg may load it.  It
+ * shares no source with the CUDA library and includes none of its headers.
+ *
+ * Arithmetic: fp32 storage, fp64 accumulation in every dot product, softmax
+ * sum and norm.  Weights are bf16 bit patterns widened exactly to fp32.
+ */
+#ifndef DLLM_ORACLE_H
+#define DLLM_ORACLE_H
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Token states (Sec. 3.3 "Staged Token Stabilization" plus the draft flag
+ * of Sec. 3.2).  COMMITTED = visible but revisable; STABLE = long-term. */
+enum { ORC_FIXED = 0, ORC_MASKED = 1, ORC_COMMITTED = 2, ORC_STABLE = 3, ORC_DRAFT = 4 };
+
+/* Tensor ids used by the counter-based weight generator. */
+enum { ORC_T_EMBED = 1, ORC_T_HEAD = 2 };
+enum { ORC_W_Q = 0, ORC_W_K = 1, ORC_W_V = 2, ORC_W_O = 3, ORC_W_GATE = 4, ORC_W_UP = 5, ORC_W_DOWN = 6 };
+#define ORC_LAYER_TENSOR(l, w) (16ull + 8ull * (uint64_t)(l) + (uint64_t)(w))
+#define ORC_KV_TENSOR(b, l, c, L) (0x100000000ull + ((uint64_t)(b) * (uint64_t)(L) + (uint64_t)(l)) * 2ull + (uint64_t)(c))
+
+typedef struct {
+    int n_layers, d_model, n_heads, head_dim, ffn, vocab, mask_id;
+    double rope_base, rms_eps;
+    uint64_t weight_seed;
+} orc_config;
+
+typedef struct {
+    int steps_per_block;   /* S */
+    int block_len;         /* 32 */
+    float theta_remask;    /* 0 disables the revision pass */
+    float theta_stable;    /* promotion to STABLE */
+    int remask_max;        /* R_max re-masks per step */
+    int spec_trigger;      /* lookahead when masked count <= trigger */
+    int spec_blocks;       /* future blocks added to the window; 0 = off */
+    int use_prefix_cache;  /* 0 = vanilla full-sequence decoding */
+} orc_sched;
+
+typedef struct {
+    int n_committed, n_remasked, n_stable, n_drafts, block_done, masked_after;
+} orc_step_out;
+
+/* ---- counter-based generator (SplitMix64, Steele/Lea/Flood 2014) ---- */
+uint64_t orc_splitmix_at(uint64_t key, uint64_t n);
+void orc_gen_f32(uint64_t seed, uint64_t tensor_id, uint64_t first, uint64_t n, double sigma, float* out);
+void orc_gen_bf16(uint64_t seed, uint64_t tensor_id, uint64_t first, uint64_t n, double sigma, uint16_t* out);
+uint16_t orc_f32_to_bf16(float f);
+float orc_bf16_to_f32(uint16_t h);
+
+/* ---- model ---- */
+typedef struct orc_model orc_model;
+/* gen_layers < 0: all layers; gen_head: generate the LM head. */
+orc_model* orc_model_new(const orc_config* c, int gen_layers, int gen_head);
+orc_model* orc_model_new_zero(const orc_config* c);
+/* Direct access to a weight (bf16 bits, logical row-major [out][in]).
+ * layer = -1: which = ORC_T_EMBED / ORC_T_HEAD. */
+uint16_t* orc_model_weight(orc_model* m, int layer, int which, size_t* n_elems);
+float* orc_model_norm(orc_model* m, int layer, int which /*0 attn,1 ffn; layer -1: final*/);
+void orc_model_free(orc_model* m);
+
+/* ---- single ops (Sec. 2.1 transformer step), exposed for pins ---- */
+void orc_rmsnorm(int n, const float* x, const float* gamma, double eps, float* out);
+void orc_rope(int hd, double base, int pos, float* vec /* [hd], in place */);
+/* logits -> decision (argmax excluding mask, max-softmax confidence). */
+void orc_decide(int V, int mask_id, const float* logits, int32_t cur_tok,
+                int32_t* x0, float* conf, float* tokconf, float* margin);
+
+/* Forward over a window of T tokens at absolute positions pos[], against a
+ * prefix of P cached keys/values per layer (prefix_k/v: [L][P][d], NULL if
+ * P == 0).  group (nullable): window key j is visible to window query i iff
+ * group[j] <= group[i].  out_k/out_v (nullable): window K/V [L][T][d].
+ * logits (nullable): [T][V]; head skipped when NULL.  Returns 0. */
+int orc_forward(const orc_model* m, int T, const int32_t* tok, const int32_t* pos,
+                int P, const float* prefix_k, const float* prefix_v, const int32_t* group,
+                float* out_k, float* out_v, float* logits, int n_layers_run);
+
+/* One commit / re-mask / draft pass (C5-C9 of the scope table) over a
+ * single sequence's state arrays (length n_pos).  Pure function. */
+int orc_commit(const orc_sched* s, int mask_id, int n_pos, int32_t* tok, uint8_t* st,
+               int w0, int T, int c0, int c1, int step, const int32_t* x0, const float* conf,
+               const float* tokconf, orc_step_out* out);
+
+/* ---- stateful session (one sequence) ---- */
+typedef struct orc_session orc_session;
+orc_session* orc_session_new(const orc_model* m, const orc_sched* s, int Lp, const int32_t* prompt, int gen_len);
+void orc_session_free(orc_session* x);
+int orc_prefill(orc_session* x);
+/* 0: started a block; 1: generation finished (last block appended). */
+int orc_begin_block(orc_session* x);
+int orc_denoise_step(orc_session* x, orc_step_out* out, int keep_logits);
+int orc_window(const orc_session* x, int32_t* info /* w0, T, c0, c1, step, kv_len, spec_on */);
+int orc_step_decisions(const orc_session* x, int32_t* x0, float* conf, float* tokconf, float* margin, float* logits);
+int orc_get_state(const orc_session* x, int32_t* tok, uint8_t* st, int32_t* kv_len);
+int orc_set_state(orc_session* x, const int32_t* tok, const uint8_t* st);
+/* prefix K/V of layer l: [kv_len][d] (pointer into the session). */
+const float* orc_prefix_kv(const orc_session* x, int layer, int which);
+int orc_n_pos(const orc_session* x);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

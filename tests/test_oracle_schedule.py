@@ -1,0 +1,258 @@
+"""Pins of the oracle's decoding loop: the commit schedule, top-k selection,
+re-masking, drafts, prefix-KV bookkeeping, and equivalence with a separately
+written vanilla LLaDA sampler (Sec. 2.1, Sec. 3.2, Sec. 3.3 of the paper).
+"""
+import numpy as np
+import pytest
+
+import dllm_inputs as I
+import oracle as O
+
+TINY = O.OracleConfig()  # 2 layers, d 256, 4x64 heads, ffn 688, vocab 1024, mask 1023
+
+
+@pytest.fixture(scope="module")
+def tiny_model(oracle_lib):
+    return O.Model(TINY)
+
+
+def _llada_schedule(m0, S):
+    """LLaDA's front-loaded per-step transfer counts (closed form)."""
+    base, rem = divmod(m0, S)
+    return [base + (1 if s < rem else 0) for s in range(S)]
+
+
+# ------------------------------------------------------------ commit pass
+@pytest.mark.parametrize("m0,S", [(32, 8), (32, 32), (24, 32), (5, 4), (1, 3), (31, 7)])
+def test_commit_counts_follow_llada_closed_form(oracle_lib, m0, S):
+    n = 40
+    tok = np.full(n, TINY.mask_id, np.int32)
+    st = np.full(n, O.MASKED, np.uint8)
+    c0, c1 = 4, 4 + 32
+    st[:c0] = O.FIXED
+    st[c0:c1][m0:] = O.COMMITTED  # 32 - m0 already committed
+    tok[:c0] = 5
+    tok[c0:c1][m0:] = 6
+    sched = O.OracleSched(steps_per_block=S, block_len=32)
+    got = []
+    for s in range(S):
+        conf = I.scripted_confidences(n, seed=100 + s)
+        x0 = np.arange(n, dtype=np.int32) % 1000
+        tok, st, out = O.commit(sched, TINY.mask_id, tok, st, 0, n, c0, c1, s, x0, conf, np.zeros(n, np.float32))
+        got.append(out["n_committed"])
+        assert out["masked_after"] == int((st[c0:c1] == O.MASKED).sum())
+    assert got == _llada_schedule(m0, S)
+    assert sum(got) == m0
+    assert not (st[c0:c1] == O.MASKED).any()
+    assert not (tok[c0:c1] == TINY.mask_id).any()
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_commit_selects_top_k_by_confidence_then_position(oracle_lib, seed):
+    n, c0, c1 = 48, 8, 40
+    rng = np.random.default_rng(seed)
+    st = np.where(rng.random(n) < 0.6, O.MASKED, O.COMMITTED).astype(np.uint8)
+    tok = np.where(st == O.MASKED, TINY.mask_id, 1).astype(np.int32)
+    conf = I.scripted_confidences(n, seed=seed, ties=True)
+    x0 = rng.integers(0, 1000, n).astype(np.int32)
+    S, s = 8, 3
+    sched = O.OracleSched(steps_per_block=S)
+    tok2, st2, out = O.commit(sched, TINY.mask_id, tok, st, 0, n, c0, c1, s, x0, conf, np.zeros(n, np.float32))
+    masked = [p for p in range(c0, c1) if st[p] == O.MASKED]
+    k = -(-len(masked) // (S - s)) if masked else 0
+    want = sorted(masked, key=lambda p: (-conf[p], p))[:k]
+    got = [p for p in range(n) if st2[p] != st[p]]
+    assert sorted(want) == got
+    assert out["n_committed"] == k
+    assert all(tok2[p] == x0[p] and st2[p] == O.COMMITTED for p in want)
+    outside = [p for p in range(n) if not (c0 <= p < c1)]
+    assert np.array_equal(tok2[outside], tok[outside])
+
+
+def test_remask_lowest_confidence_and_stable_promotion(oracle_lib):
+    n, c0, c1 = 32, 0, 32
+    st = np.full(n, O.COMMITTED, np.uint8)
+    st[20:] = O.MASKED
+    tok = np.where(st == O.MASKED, TINY.mask_id, 3).astype(np.int32)
+    tokconf = np.full(n, 0.6, np.float32)
+    tokconf[[2, 5, 9]] = [0.3, 0.1, 0.1]  # below 0.5: 5 and 9 tie, 5 wins
+    tokconf[[1, 4]] = [0.95, 0.9]  # at or above theta_stable
+    conf = I.scripted_confidences(n, seed=7)
+    x0 = np.full(n, 11, np.int32)
+    sched = O.OracleSched(steps_per_block=16, theta_remask=0.5, theta_stable=0.9, remask_max=1)
+    tok2, st2, out = O.commit(sched, TINY.mask_id, tok, st, 0, n, c0, c1, 2, x0, conf, tokconf)
+    assert out["n_remasked"] == 1 and out["n_stable"] == 2
+    assert st2[1] == O.STABLE and st2[4] == O.STABLE
+    # position 5 was re-masked; it competes with the other masked positions
+    masked_before_commit = sorted([5] + list(range(20, 32)))
+    k = -(-len(masked_before_commit) // (16 - 2))
+    chosen = sorted(masked_before_commit, key=lambda p: (-conf[p], p))[:k]
+    for p in masked_before_commit:
+        if p in chosen:
+            assert st2[p] == O.COMMITTED and tok2[p] == 11
+        else:
+            assert st2[p] == O.MASKED and tok2[p] == TINY.mask_id
+    assert st2[9] == O.COMMITTED and tok2[9] == 3 and st2[2] == O.COMMITTED
+    # two re-masks allowed: both ties at 0.1 go
+    sched2 = O.OracleSched(steps_per_block=16, theta_remask=0.5, remask_max=2)
+    conf2 = np.ones(n, np.float32)
+    conf2[[5, 9]] = 0.0  # the re-masked positions lose the commit pass
+    _, st3, out3 = O.commit(sched2, TINY.mask_id, tok, st, 0, n, c0, c1, 2, x0, conf2, tokconf)
+    assert out3["n_remasked"] == 2 and st3[5] == O.MASKED and st3[9] == O.MASKED and st3[2] == O.COMMITTED
+
+
+def test_revision_disabled_on_last_step_and_at_zero_threshold(oracle_lib):
+    n = 32
+    st = np.full(n, O.COMMITTED, np.uint8)
+    st[-1] = O.MASKED
+    tok = np.where(st == O.MASKED, TINY.mask_id, 3).astype(np.int32)
+    tokconf = np.full(n, 0.01, np.float32)
+    x0 = np.full(n, 4, np.int32)
+    conf = np.ones(n, np.float32)
+    last = O.OracleSched(steps_per_block=8, theta_remask=0.5)
+    _, st2, out = O.commit(last, TINY.mask_id, tok, st, 0, n, 0, n, 7, x0, conf, tokconf)
+    assert out["n_remasked"] == 0 and out["block_done"] == 1
+    off = O.OracleSched(steps_per_block=8, theta_remask=0.0)
+    _, _, out = O.commit(off, TINY.mask_id, tok, st, 0, n, 0, n, 2, x0, conf, tokconf)
+    assert out["n_remasked"] == 0 and out["n_stable"] == 0
+
+
+def test_drafts_one_per_speculative_block(oracle_lib):
+    n, bl = 128, 32
+    c0, c1 = 32, 64
+    st = np.full(n, O.MASKED, np.uint8)
+    st[:c0] = O.FIXED
+    st[c0:c0 + 28] = O.COMMITTED
+    st[64 + 3] = O.DRAFT
+    tok = np.where(st == O.MASKED, TINY.mask_id, 2).astype(np.int32)
+    conf = I.scripted_confidences(n, seed=9, ties=True)
+    x0 = (np.arange(n) % 900).astype(np.int32)
+    sched = O.OracleSched(steps_per_block=32, spec_blocks=2, spec_trigger=8, use_prefix_cache=1)
+    w0, T = c0, 96  # decisions are indexed by window offset
+    tok2, st2, out = O.commit(sched, TINY.mask_id, tok, st, w0, T, c0, c1, 5, x0[w0:w0 + T], conf[w0:w0 + T],
+                              np.zeros(T, np.float32))
+    assert out["n_drafts"] == 2
+    for b0, b1 in ((64, 96), (96, 128)):
+        new = [p for p in range(b0, b1) if st2[p] == O.DRAFT and st[p] != O.DRAFT]
+        cand = [p for p in range(b0, b1) if st[p] == O.MASKED]
+        assert new == [sorted(cand, key=lambda p: (-conf[p], p))[0]]
+        assert tok2[new[0]] == x0[new[0]]
+
+
+# ------------------------------------------------------------ sessions
+def _vanilla_llada(model, prompt, gen_len, block_len, steps_per_block):
+    """Separately written LLaDA sampler: full sequence every step, the
+    front-loaded per-block transfer schedule, top-k by confidence."""
+    cfg = model.cfg
+    Lp = prompt.size
+    x = np.concatenate([prompt, np.full(gen_len, cfg.mask_id, np.int32)])
+    pos = np.arange(x.size, dtype=np.int32)
+    for b in range(gen_len // block_len):
+        lo, hi = Lp + b * block_len, Lp + (b + 1) * block_len
+        counts = _llada_schedule(int((x[lo:hi] == cfg.mask_id).sum()), steps_per_block)
+        for s in range(steps_per_block):
+            logits = O.forward(model, x, pos)["logits"]
+            dec = [O.decide(logits[p], cfg.mask_id, x[p]) for p in range(x.size)]
+            masked = [p for p in range(lo, hi) if x[p] == cfg.mask_id]
+            chosen = sorted(masked, key=lambda p: (-dec[p][1], p))[:counts[s]]
+            for p in chosen:
+                x[p] = dec[p][0]
+    return x[Lp:]
+
+
+def test_vanilla_equivalence(tiny_model):
+    """Cache off and one block spanning the whole generation equals the
+    vanilla full-sequence sampler."""
+    prompt = I.uniform_prompt(16, TINY.vocab, TINY.mask_id, seed=11)
+    gen = 32
+    want = _vanilla_llada(tiny_model, prompt, gen, gen, 8)
+    sess = O.Session(tiny_model, O.OracleSched(steps_per_block=8, block_len=gen, use_prefix_cache=0), prompt, gen)
+    got = sess.generate()
+    assert np.array_equal(got, want)
+
+
+def test_cache_off_blockwise_equals_semi_autoregressive_llada(tiny_model):
+    prompt = I.uniform_prompt(8, TINY.vocab, TINY.mask_id, seed=12)
+    want = _vanilla_llada(tiny_model, prompt, 64, 32, 4)
+    sess = O.Session(tiny_model, O.OracleSched(steps_per_block=4, block_len=32, use_prefix_cache=0), prompt, 64)
+    assert np.array_equal(sess.generate(), want)
+
+
+def test_incremental_prefix_kv_equals_block_causal_recompute(tiny_model):
+    prompt = I.uniform_prompt(40, TINY.vocab, TINY.mask_id, seed=13)
+    sess = O.Session(tiny_model, O.OracleSched(steps_per_block=8), prompt, 64)
+    gen = sess.generate()
+    tok, st, kv_len = sess.state()
+    assert kv_len == 40 + 64
+    assert (st[40:] == O.COMMITTED).all() and np.array_equal(tok[40:], gen)
+    group = np.array([0] * 40 + [1] * 32 + [2] * 32, np.int32)
+    full = O.forward(tiny_model, tok, np.arange(tok.size), group=group, want_kv=True, logits=False)
+    for layer in range(TINY.n_layers):
+        assert np.array_equal(sess.prefix_kv(layer, 0), full["k"][layer])
+        assert np.array_equal(sess.prefix_kv(layer, 1), full["v"][layer])
+
+
+def test_session_schedule_and_mask_invariants(tiny_model):
+    prompt = I.uniform_prompt(64, TINY.vocab, TINY.mask_id)
+    sess = O.Session(tiny_model, O.OracleSched(steps_per_block=8), prompt, 64)
+    sess.prefill()
+    blocks = 0
+    while sess.begin_block():
+        counts = []
+        while True:
+            w = sess.window()
+            out = sess.step()
+            counts.append(out["n_committed"])
+            assert sess.window()["T"] == 32 and sess.window()["w0"] == 64 + 32 * blocks
+            if out["block_done"]:
+                break
+        assert counts == [4] * 8
+        assert sess.state()[2] == 64 + 32 * blocks
+        blocks += 1
+    tok, st, kv = sess.state()
+    assert blocks == 2 and kv == 128
+    assert not (tok[64:] == TINY.mask_id).any()
+
+
+def test_speculation_trigger_off_equals_plain_blocks(tiny_model):
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=21)
+    plain = O.Session(tiny_model, O.OracleSched(steps_per_block=16), prompt, 96).generate()
+    never = O.Session(tiny_model, O.OracleSched(steps_per_block=16, spec_blocks=2, spec_trigger=-1), prompt, 96)
+    assert np.array_equal(never.generate(), plain)
+
+
+def test_speculation_drafts_never_touch_prefix(tiny_model):
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=22)
+    sched = O.OracleSched(steps_per_block=16, spec_blocks=2, spec_trigger=8, theta_remask=0.5, remask_max=1)
+    sess = O.Session(tiny_model, sched, prompt, 128)
+    sess.prefill()
+    nblk, spec_steps, steps = 0, 0, 0
+    while sess.begin_block():
+        tok, st, kv = sess.state()
+        assert kv == 32 + 32 * nblk
+        c0 = 32 + 32 * nblk
+        assert not (st[c0:c0 + 32] == O.DRAFT).any()  # accepted drafts became COMMITTED
+        while True:
+            out = sess.step()
+            w = sess.window()
+            steps += 1
+            spec_steps += w["spec_on"]
+            assert w["T"] in (32, 64, 96)
+            assert sess.state()[2] == kv  # drafts never extend the prefix
+            tok, st, _ = sess.state()
+            assert not (st[:c0] == O.DRAFT).any()
+            if out["block_done"]:
+                break
+        assert sess.window()["step"] <= 16
+        nblk += 1
+    assert nblk == 4 and spec_steps > 0
+    tok, st, kv = sess.state()
+    assert kv == 160 and not (tok[32:] == TINY.mask_id).any()
+
+
+def test_revision_zero_threshold_equals_no_revision(tiny_model):
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=23)
+    a = O.Session(tiny_model, O.OracleSched(steps_per_block=8), prompt, 64).generate()
+    b = O.Session(tiny_model, O.OracleSched(steps_per_block=8, theta_remask=0.0, theta_stable=0.0), prompt,
+                  64).generate()
+    assert np.array_equal(a, b)
