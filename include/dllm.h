@@ -1,0 +1,189 @@
+/*
+ * dllm.h - C ABI of the GB300 block-wise diffusion-LLM denoising path.
+ *
+ * Implements the decoding loop of "Efficient On-Device Diffusion LLM Inference
+ * with Mobile NPU" (arXiv 2606.13740): block-wise decoding with prefix KV
+ * reuse (Sec. 2.1 "Block-Wise Decoding"), the decoding window with draft
+ * tokens from future blocks (Sec. 3.2 "Multi-Block Speculative Decoding"),
+ * and revisable commits (Sec. 3.3 "Staged Token Stabilization").  Every step
+ * of the path (embedding, RMSNorm, QKV+RoPE, attention, SwiGLU MLP, LM head
+ * with confidence and argmax, commit/re-mask/draft) runs in the library's own
+ * CUDA kernels on one GPU; there is no CPU fallback.
+ *
+ * Conventions for every entry point:
+ *   - Return 0 (DLLM_OK) or a negative DLLM_E* code (DLLM_DONE = 1 is a
+ *     non-error status of dllm_begin_block).  No C++ exception crosses the ABI.
+ *   - After an error the context is poisoned: later calls return
+ *     DLLM_ESTATE until dllm_free.  dllm_last_error gives the message.
+ *   - Host pointers belong to the caller and are only read/written during the
+ *     call.  Device memory belongs to the context (or to the caller's arena,
+ *     which the context never frees).
+ *   - Work is queued on the context's stream.  Calls that return host data
+ *     synchronise that stream; the others are asynchronous.
+ *   - Token ids are int32; token states are uint8 DLLM_FIXED..DLLM_DRAFT.
+ *   - Sequences of a batch are independent and advance in lockstep (same
+ *     prompt length, same block schedule).
+ */
+#ifndef DLLM_H
+#define DLLM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define DLLM_OK 0
+#define DLLM_DONE 1
+#define DLLM_EINVAL (-1)
+#define DLLM_ENOMEM (-2)
+#define DLLM_ECUDA (-3)
+#define DLLM_ETIMEOUT (-4)
+#define DLLM_ESTATE (-5)
+#define DLLM_ECAPACITY (-6)
+
+/* Token states.  COMMITTED is the paper's "visible" state (usable as
+ * context, still revisable); STABLE is long-term (Sec. 3.3); DRAFT marks a
+ * future-block prediction (Sec. 3.2). */
+enum { DLLM_FIXED = 0, DLLM_MASKED = 1, DLLM_COMMITTED = 2, DLLM_STABLE = 3, DLLM_DRAFT = 4 };
+
+typedef struct dllm_ctx dllm_ctx;
+
+/* Model shape and capacities.  The model is the LLaDA architecture the paper
+ * runs (Sec. 5.1 "Models"): pre-norm RMSNorm, multi-head attention without a
+ * causal mask, rotate-half RoPE, SwiGLU MLP, untied LM head.  Weights are
+ * bf16, drawn on the device from weight_seed (N(0, 0.02) by a counter-based
+ * SplitMix64/Irwin-Hall generator); RMSNorm gains are one.
+ * Constraints: head_dim in {64, 128}; d_model, n_heads*head_dim multiples of
+ * 64; vocab, ffn multiples of 8; max_window * max_batch <= 4096. */
+typedef struct {
+    int n_layers, d_model, n_heads, head_dim, ffn, vocab, mask_id;
+    float rope_base, rms_eps;
+    int max_batch;   /* sequences per call */
+    int max_ctx;     /* positions per sequence: prompt + generation (+ window overhang) */
+    int max_window;  /* query tokens per sequence per forward (window or prompt) */
+    int block_len;   /* tokens per block (32) */
+    uint64_t weight_seed;
+} dllm_config;
+
+/* Decoding schedule.  steps_per_block = S; the step-s commit count is
+ * ceil(m / (S - s)) for m masked positions of the current block.
+ * theta_remask > 0 enables the revision pass: committed tokens whose
+ * current-id probability is >= theta_stable become STABLE, and at most
+ * remask_max of those below theta_remask (lowest first) are re-masked; it is
+ * skipped on the block's last step.  spec_blocks > 0 enables lookahead: when
+ * the current block has <= spec_trigger masked positions, the window extends
+ * over the next spec_blocks blocks, each of which drafts its most confident
+ * masked position per step.  use_prefix_cache = 0 gives vanilla decoding:
+ * every step runs the full sequence and nothing is cached. */
+typedef struct {
+    int steps_per_block;
+    float theta_remask;
+    float theta_stable;
+    int remask_max;
+    int spec_trigger;
+    int spec_blocks;
+    int use_prefix_cache;
+} dllm_sched;
+
+/* Result of one denoising step, summed over the batch (block_done: all). */
+typedef struct {
+    int n_committed, n_remasked, n_stable, n_drafts, block_done, masked_after;
+} dllm_step_out;
+
+typedef struct {
+    int steps;        /* denoising steps run */
+    int spec_steps;   /* steps whose window included draft blocks */
+    int blocks;       /* blocks finished */
+} dllm_stats;
+
+/* Device bytes the context needs for cfg (weights, KV cache, activations,
+ * scratch).  Pass an arena of at least this size to dllm_init, or NULL. */
+int dllm_arena_bytes(const dllm_config* cfg, size_t* bytes);
+
+/* Create a context on the current CUDA device.  dev_arena: caller-owned
+ * device memory of arena_bytes (>= dllm_arena_bytes), or NULL to let the
+ * library allocate (and later free) its own.  cuda_stream: a cudaStream_t
+ * (as void*), or NULL for a library-created stream.  Draws all weights.
+ * Errors: DLLM_EINVAL (bad shape), DLLM_ENOMEM, DLLM_ECUDA. */
+int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void* cuda_stream, dllm_ctx** out);
+
+/* Free the context and everything it allocated (not a caller arena). */
+void dllm_free(dllm_ctx* ctx);
+
+/* Last error message of the context (static storage for a NULL ctx). */
+const char* dllm_last_error(const dllm_ctx* ctx);
+
+/* Wait for the context's stream and report device-side errors (a bounded
+ * wait that ran out gives DLLM_ETIMEOUT). */
+int dllm_sync(dllm_ctx* ctx);
+
+/* Start a request (Sec. 2.1): batch sequences, prompt = host int32
+ * [batch][Lp], gen_len masked positions after it.  With the prefix cache on,
+ * runs the prompt through the layers (bidirectional over the prompt) and
+ * stores its K/V as the prefix.  Errors: DLLM_EINVAL, DLLM_ECAPACITY
+ * (Lp + gen_len + window overhang > max_ctx, batch > max_batch). */
+int dllm_prefill(dllm_ctx* ctx, const dllm_sched* sched, int batch, const int32_t* prompt, int Lp, int gen_len);
+
+/* Synthetic prefix instead of a prefill: every sequence gets P cached
+ * positions whose K/V are drawn from seed (N(0,1), same generator), ids 0 and
+ * state FIXED, followed by gen_len masked positions. */
+int dllm_set_prefix_kv_random(dllm_ctx* ctx, const dllm_sched* sched, int batch, int P, int gen_len, uint64_t seed);
+
+/* Advance to the next block.  If a block is current it must be finished (no
+ * MASKED position, else DLLM_EINVAL); with the prefix cache on its K/V are
+ * recomputed from its final ids (attending to prefix + block) and appended.
+ * Drafts of the new block become COMMITTED (re-checked by the revision
+ * pass).  Returns DLLM_DONE when no block is left. */
+int dllm_begin_block(dllm_ctx* ctx);
+
+/* One denoising step on the current window: forward, decisions, commit /
+ * re-mask / drafts.  out (nullable, host): filled after a stream sync; with
+ * NULL the call stays asynchronous unless lookahead needs the masked count. */
+int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out);
+
+/* Restore the request state to what it was at the last dllm_begin_block or
+ * dllm_set_state, and reset the block's step counter (repeats identical
+ * steps). */
+int dllm_rewind_block(dllm_ctx* ctx);
+
+/* Whole request: prefill, then blocks until done.  out_tokens: host int32
+ * [batch][gen_len].  stats nullable. */
+int dllm_generate(dllm_ctx* ctx, const dllm_sched* sched, int batch, const int32_t* prompt, int Lp, int gen_len,
+                  int32_t* out_tokens, dllm_stats* stats);
+
+/* Current window (sequence 0): info[0..6] = w0, T, c0, c1, step, kv_len,
+ * spec_on of the last step (positions absolute within the sequence). */
+int dllm_window(dllm_ctx* ctx, int32_t* info);
+
+/* Copy the whole state out: tokens int32 [batch][n_pos], states uint8
+ * [batch][n_pos], kv_len int32 [batch] (any may be NULL).  Synchronises. */
+int dllm_get_state(dllm_ctx* ctx, int32_t* tokens, uint8_t* status, int32_t* kv_len);
+
+/* Overwrite tokens/states [batch][n_pos] (teacher forcing; either may be
+ * NULL).  Inside a block this also becomes the dllm_rewind_block point. */
+int dllm_set_state(dllm_ctx* ctx, const int32_t* tokens, const uint8_t* status);
+
+/* Debug output of the last step, window-indexed [batch][T]: argmax ids,
+ * max-softmax confidence, probability of the current id; logits fp32
+ * [batch][T][vocab] only when dllm_set_debug enabled them (else pass NULL).
+ * Synchronises. */
+int dllm_get_step_debug(dllm_ctx* ctx, float* logits, int32_t* argmax, float* conf, float* tokconf);
+
+/* flags bit 0: materialise logits; bit 1: disable CUDA graphs. */
+int dllm_set_debug(dllm_ctx* ctx, int flags);
+
+/* Copy one weight back in its logical row-major layout (bf16 bits):
+ * layer -1 with which 1 = embedding, 2 = LM head; otherwise which =
+ * 0 q, 1 k, 2 v, 3 o, 4 gate, 5 up, 6 down.  Synchronises. */
+int dllm_get_weight(dllm_ctx* ctx, int layer, int which, uint16_t* out, size_t n_elems);
+
+/* Copy a slice of the K or V cache (which 0/1) of one layer and sequence:
+ * out fp32 [n][n_heads*head_dim] for positions [p0, p0+n).  Synchronises. */
+int dllm_get_kv(dllm_ctx* ctx, int layer, int which, int seq, int p0, int n, float* out);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

@@ -1,0 +1,57 @@
+/*
+ * dllm_ops.h - single-kernel entry points of the denoising path, for
+ * kernel-level parity tests and micro-benchmarks.  Same conventions as
+ * dllm.h (0 = OK, negative DLLM_E* codes; messages via dllm_last_error(NULL)).
+ * Device pointers are marked "dev"; these calls allocate their own scratch
+ * with cudaMalloc and free it before returning, and synchronise the stream.
+ */
+#ifndef DLLM_OPS_H
+#define DLLM_OPS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Dense projection of the transformer step (Sec. 2.1, the matrix work the
+ * paper offloads to the NPU; here tcgen05 tensor cores):
+ * D[n][m] = sum_k W[m][k] * X[n][k].  W dev bf16 [M][K] row-major, X dev bf16
+ * [N][K] row-major, D dev fp32 [N][M].  K*2 bytes must be a multiple of 16;
+ * W and X 16-byte aligned.  grid = CTAs of the stream-K split (0: one per
+ * SM).  Errors: DLLM_EINVAL, DLLM_ECUDA, DLLM_ETIMEOUT. */
+int dllm_op_gemm(const void* W, const void* X, float* D, int M, int N, int K, int grid, void* stream);
+
+/* Bidirectional attention of the window's queries over cached + window keys
+ * (Sec. 2.1, block-wise decoding with prefix KV reuse; no causal mask).
+ * q dev bf16 [B][H][T][hd]; kc, vc dev bf16 [B][H][cap][hd] (keys of
+ * sequence b: positions [0, kv_len[b] + T)); kv_len dev int32 [B];
+ * out dev bf16 [B*T][H*hd].  hd in {64, 128}. */
+int dllm_op_attention(const void* q, const void* kc, const void* vc, const int32_t* kv_len, void* out, int B, int T,
+                      int H, int hd, int cap, int max_kv_len, void* stream);
+
+/* LM head with decision (Sec. 2.1 confidence-selected commits; Sec. 3.3
+ * selective logits): per token n, z = W X[n]^T over the vocab; x0 = argmax
+ * excluding mask_id (ties: lowest id); conf = softmax(z)[x0] with the mask
+ * excluded; tokconf = softmax(z)[cur[n]] (0 when cur[n] is the mask id).
+ * W dev bf16 [V][d], X dev bf16 [N][d], cur dev int32 [N]; outputs dev [N];
+ * logits dev fp32 [N][V] or NULL. */
+int dllm_op_lmhead(const void* W, const void* X, const int32_t* cur, int32_t* x0, float* conf, float* tokconf,
+                   float* logits, int V, int N, int d, int mask_id, void* stream);
+
+/* One commit / re-mask / draft pass on HOST arrays of one sequence
+ * (Sec. 2.1 commit, Sec. 3.2 drafts, Sec. 3.3 revision): tok int32 and
+ * status uint8 [n_pos] are updated in place; x0, conf, tokconf [T] are
+ * indexed by window offset; window [w0, w0+T), current block [c0, c1),
+ * step index within the block.  sched as in dllm.h; block_len = draft block
+ * size.  out nullable.  Runs the device kernel on copies. */
+int dllm_op_commit(int32_t* tok, uint8_t* status, int n_pos, int w0, int T, int c0, int c1, int step,
+                   const int32_t* x0, const float* conf, const float* tokconf, int steps_per_block,
+                   float theta_remask, float theta_stable, int remask_max, int spec_blocks, int use_prefix_cache,
+                   int block_len, int mask_id, int* out6);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

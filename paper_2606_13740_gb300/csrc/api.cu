@@ -1,0 +1,809 @@
+// C ABI of the denoising path (include/dllm.h): device memory layout,
+// request state, and the host sequencing of the step's kernels.
+//
+// HBM layout (one arena, offsets fixed at init):
+//   weights  per layer: Wqkv [3*qd (pad 128)][d], Wo [d][qd],
+//            Wgu [ceil(F/64)*128][d] (64 gate rows then 64 up rows per
+//            128-row tile), Wd [d][F]; embedding [V][d]; LM head [V pad 128][d]
+//   KV cache [L][K|V][batch][head][position][head_dim] bf16
+//   RoPE     [max_ctx][head_dim/2][cos, sin] fp32
+//   activations for max_batch * max_window tokens (fp32 residual, bf16 GEMM
+//   operands), attention and GEMM split partials, LM-head tile statistics
+//   request state: ids int32 [batch][max_ctx], token states uint8, plan.
+#include "../../include/dllm.h"
+#include "../../include/dllm_ops.h"
+#include "internal.h"
+
+#include <algorithm>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+using namespace dllm;
+
+namespace {
+
+constexpr int kMaxSMs = 256;  // upper bound for scratch sizing
+
+size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
+int rup(int x, int m) { return (x + m - 1) / m * m; }
+
+struct Layout {
+    int qd, qkv_rows, gu_rows, d_rows, o_rows, head_rows, head_tiles, max_tok;
+    size_t off_w, per_layer, off_emb, off_head, off_kv, kv_half, off_rope;
+    size_t off_x, off_xn, off_q, off_attn, off_h;
+    size_t off_apo, apo_floats, off_apml;
+    size_t off_lmp, off_zcur, off_cur, off_x0, off_conf, off_tokconf;
+    size_t off_part, part_floats, off_cnt;
+    int cnt_len;
+    size_t off_tok, off_st, off_stok, off_sst, off_seqkv, off_plan, off_outs, off_status;
+    size_t total;
+    size_t w_qkv, w_o, w_gu, w_d;  // element offsets inside a layer
+};
+
+Layout make_layout(const dllm_config& c) {
+    Layout L{};
+    const int d = c.d_model, H = c.n_heads, hd = c.head_dim, F = c.ffn, V = c.vocab;
+    L.qd = H * hd;
+    L.qkv_rows = rup(3 * L.qd, 128);
+    L.o_rows = rup(d, 128);
+    L.gu_rows = (F + 63) / 64 * 128;
+    L.d_rows = rup(d, 128);
+    L.head_rows = rup(V, 128);
+    L.head_tiles = L.head_rows / 128;
+    L.max_tok = c.max_batch * c.max_window;
+    L.w_qkv = 0;
+    L.w_o = L.w_qkv + static_cast<size_t>(L.qkv_rows) * d;
+    L.w_gu = L.w_o + static_cast<size_t>(L.o_rows) * L.qd;
+    L.w_d = L.w_gu + static_cast<size_t>(L.gu_rows) * d;
+    L.per_layer = L.w_d + static_cast<size_t>(L.d_rows) * F;
+    size_t o = 0;
+    auto take = [&](size_t bytes) {
+        size_t r = o;
+        o = al256(o + bytes);
+        return r;
+    };
+    L.off_w = take(L.per_layer * 2 * c.n_layers);
+    L.off_emb = take(static_cast<size_t>(V) * d * 2);
+    L.off_head = take(static_cast<size_t>(L.head_rows) * d * 2);
+    L.kv_half = static_cast<size_t>(c.max_batch) * H * c.max_ctx * hd;
+    L.off_kv = take(L.kv_half * 2 * 2 * c.n_layers);
+    L.off_rope = take(static_cast<size_t>(c.max_ctx) * hd * 4);
+    const size_t T = L.max_tok;
+    L.off_x = take(T * d * 4);
+    L.off_xn = take(T * std::max(d, L.qd) * 2);
+    L.off_q = take(T * L.qd * 2);
+    L.off_attn = take(T * L.qd * 2);
+    L.off_h = take(T * F * 2);
+    // attention split partials: B*H*nsplit*T rows, nsplit <= 2*SMs/(B*H*qtiles) + 1
+    const size_t rows = static_cast<size_t>(2 * kMaxSMs) * 64 + static_cast<size_t>(c.max_batch) * H * c.max_window;
+    L.apo_floats = rows * hd;
+    L.off_apo = take(L.apo_floats * 4);
+    L.off_apml = take(rows * 2 * 4);
+    L.off_lmp = take(static_cast<size_t>(L.head_tiles) * T * 3 * 4);
+    L.off_zcur = take(T * 4);
+    L.off_cur = take(T * 4);
+    L.off_x0 = take(T * 4);
+    L.off_conf = take(T * 4);
+    L.off_tokconf = take(T * 4);
+    L.part_floats = static_cast<size_t>(kMaxSMs) * 2 * 256 * 128;
+    L.off_part = take(L.part_floats * 4);
+    const int mt_max = std::max(std::max(L.head_tiles, L.gu_rows / 128), std::max(L.qkv_rows, L.d_rows) / 128);
+    L.cnt_len = mt_max * ((L.max_tok + 255) / 256 + 1);
+    L.off_cnt = take(static_cast<size_t>(L.cnt_len) * 4);
+    const size_t S = static_cast<size_t>(c.max_batch) * c.max_ctx;
+    L.off_tok = take(S * 4);
+    L.off_st = take(S);
+    L.off_stok = take(S * 4);
+    L.off_sst = take(S);
+    L.off_seqkv = take(static_cast<size_t>(c.max_batch) * 4);
+    L.off_plan = take(static_cast<size_t>(c.max_batch) * 16);
+    L.off_outs = take(static_cast<size_t>(c.max_batch) * 32);
+    L.off_status = take(16);
+    L.total = o;
+    return L;
+}
+
+const char* check_cfg(const dllm_config& c) {
+    if (c.n_layers < 1 || c.d_model < 64 || c.n_heads < 1 || c.ffn < 8 || c.vocab < 2) return "bad model shape";
+    if (c.head_dim != 64 && c.head_dim != 128) return "head_dim must be 64 or 128";
+    if (c.d_model % 64 || (c.n_heads * c.head_dim) % 64) return "d_model and n_heads*head_dim must be multiples of 64";
+    if (c.ffn % 8 || c.vocab % 8) return "ffn and vocab must be multiples of 8";
+    if (c.mask_id < 0 || c.mask_id >= c.vocab) return "mask_id out of range";
+    if (c.max_batch < 1 || c.max_ctx < 1 || c.max_window < 1 || c.block_len < 1) return "bad capacities";
+    if (c.max_batch * c.max_window > 4096) return "max_batch * max_window must be <= 4096";
+    if (c.block_len > kMaxBlock) return "block_len too large";
+    if (c.rms_eps <= 0.0f || c.rope_base <= 1.0f) return "bad rope_base / rms_eps";
+    return nullptr;
+}
+
+}  // namespace
+
+struct dllm_ctx {
+    dllm_config cfg{};
+    Layout L{};
+    int sms = 0;
+    cudaStream_t stream = nullptr;
+    bool own_stream = false;
+    uint8_t* arena = nullptr;
+    bool own_arena = false;
+    // views
+    __nv_bfloat16* emb = nullptr;
+    __nv_bfloat16* head = nullptr;
+    std::vector<__nv_bfloat16*> wl;
+    std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_d;
+    CUtensorMap tm_head{};
+    __nv_bfloat16* kv = nullptr;
+    float* rope = nullptr;
+    float* x = nullptr;
+    __nv_bfloat16 *xn = nullptr, *q = nullptr, *attn = nullptr, *h = nullptr;
+    float *apo = nullptr, *apml = nullptr, *lmp = nullptr, *zcur = nullptr, *conf = nullptr, *tokconf = nullptr;
+    int *cur = nullptr, *x0 = nullptr;
+    Scratch scr{};
+    int *tok = nullptr, *stok = nullptr, *seq_kv = nullptr, *plan = nullptr, *outs = nullptr, *status = nullptr;
+    uint8_t *st = nullptr, *sst = nullptr;
+    float* logits = nullptr;  // debug, separate allocation
+    size_t logits_cap = 0;
+    // request mirror
+    dllm_sched sched{};
+    bool started = false, have_block = false;
+    int B = 0, Lp = 0, gen_len = 0, n_pos = 0, kv_len = 0;
+    int blk = -1, c0 = 0, c1 = 0, step = 0;
+    int last_w0 = 0, last_T = 0, last_spec = 0;
+    int debug = 0;
+    // graph cache for the step
+    cudaGraphExec_t gexec = nullptr;
+    int g_T = -1, g_B = -1, g_kv = -1, g_dbg = -1;
+    bool poisoned = false;
+    std::string err;
+};
+
+static std::string g_noctx_err;
+
+void dllm_set_noctx_error(const char* msg) { g_noctx_err = msg; }
+
+static int fail(dllm_ctx* c, int code, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    if (c) {
+        c->err = buf;
+        if (code != DLLM_EINVAL && code != DLLM_ECAPACITY) c->poisoned = true;
+    } else {
+        g_noctx_err = buf;
+    }
+    return code;
+}
+
+#define CK(call)                                                                                   \
+    do {                                                                                           \
+        cudaError_t e_ = (call);                                                                   \
+        if (e_ != cudaSuccess) return fail(ctx, DLLM_ECUDA, "%s: %s", #call, cudaGetErrorString(e_)); \
+    } while (0)
+
+#define GUARD(ctx)                                                         \
+    do {                                                                   \
+        if (!(ctx)) return fail(nullptr, DLLM_EINVAL, "null context");     \
+        if ((ctx)->poisoned) return DLLM_ESTATE;                           \
+    } while (0)
+
+static int sync_check(dllm_ctx* ctx) {
+    CK(cudaStreamSynchronize(ctx->stream));
+    int s = 0;
+    CK(cudaMemcpy(&s, ctx->status, 4, cudaMemcpyDeviceToHost));
+    if (s & kStatusTimeout) return fail(ctx, DLLM_ETIMEOUT, "a bounded device wait ran out (status %d)", s);
+    if (s) return fail(ctx, DLLM_ECUDA, "device status %d (index check failed)", s);
+    return DLLM_OK;
+}
+
+// ------------------------------------------------------------------ forward
+// Layers (and optionally the LM head) over T window tokens of each of the B
+// sequences; token ids come from the state at seq_kv[b] + t.
+static int forward(dllm_ctx* ctx, int B, int T, bool head) {
+    const dllm_config& c = ctx->cfg;
+    const Layout& L = ctx->L;
+    const int d = c.d_model, F = c.ffn, qd = L.qd, N = B * T;
+    cudaStream_t s = ctx->stream;
+    CK(launch_embed_norm(ctx->tok, c.max_ctx, ctx->seq_kv, ctx->emb, ctx->x, ctx->xn, B, T, d, c.rms_eps, s));
+    const GemmPlan pq = gemm_plan(L.qkv_rows, N, d, ctx->sms);
+    const GemmPlan po = gemm_plan(L.o_rows, N, qd, ctx->sms);
+    const GemmPlan pg = gemm_plan(L.gu_rows, N, d, ctx->sms);
+    const GemmPlan pd = gemm_plan(L.d_rows, N, F, ctx->sms);
+    CUtensorMap tx_xn, tx_attn, tx_h;
+    if (!make_tmap_bf16(&tx_xn, ctx->xn, N, d, pq.ntile) || !make_tmap_bf16(&tx_attn, ctx->attn, N, qd, po.ntile) ||
+        !make_tmap_bf16(&tx_h, ctx->h, N, F, pd.ntile))
+        return fail(ctx, DLLM_ECUDA, "tensor map encode failed");
+    const AttnPlan ap = attn_plan(B, T, c.n_heads, ctx->kv_len + T, ctx->sms);
+    if (static_cast<size_t>(B) * c.n_heads * ap.nsplit * T * c.head_dim > L.apo_floats)
+        return fail(ctx, DLLM_ECAPACITY, "attention partial buffer too small");
+    EpiArgs ep{};
+    ep.rope = ctx->rope;
+    ep.seq_kv = ctx->seq_kv;
+    ep.T = T;
+    ep.H = c.n_heads;
+    ep.hd = c.head_dim;
+    ep.cap = c.max_ctx;
+    ep.q = ctx->q;
+    ep.h = ctx->h;
+    ep.F = F;
+    for (int l = 0; l < c.n_layers; ++l) {
+        __nv_bfloat16* kc = ctx->kv + static_cast<size_t>(2 * l) * L.kv_half;
+        __nv_bfloat16* vc = ctx->kv + static_cast<size_t>(2 * l + 1) * L.kv_half;
+        ep.kc = kc;
+        ep.vc = vc;
+        CK(gemm_launch(EPI_QKV, pq, ctx->tm_qkv[l], tx_xn, ep, ctx->scr, ctx->status, s));
+        CK(launch_attention(ctx->q, kc, vc, ctx->seq_kv, ctx->apo, ctx->apml, ctx->attn, B, T, c.n_heads, c.head_dim,
+                            c.max_ctx, ap, s));
+        EpiArgs er = ep;
+        er.out = ctx->x;
+        er.ld_out = d;
+        CK(gemm_launch(EPI_RESID, po, ctx->tm_o[l], tx_attn, er, ctx->scr, ctx->status, s));
+        CK(launch_rmsnorm(ctx->x, ctx->xn, N, d, c.rms_eps, s));
+        CK(gemm_launch(EPI_SWIGLU, pg, ctx->tm_gu[l], tx_xn, ep, ctx->scr, ctx->status, s));
+        CK(gemm_launch(EPI_RESID, pd, ctx->tm_d[l], tx_h, er, ctx->scr, ctx->status, s));
+        CK(launch_rmsnorm(ctx->x, ctx->xn, N, d, c.rms_eps, s));
+    }
+    if (head) {
+        const GemmPlan ph = gemm_plan(L.head_rows, N, d, ctx->sms);
+        CK(launch_gather_cur(ctx->tok, c.max_ctx, ctx->seq_kv, ctx->cur, B, T, s));
+        EpiArgs eh{};
+        eh.lm_part = ctx->lmp;
+        eh.zcur = ctx->zcur;
+        eh.cur_tok = ctx->cur;
+        eh.V = c.vocab;
+        eh.mask_id = c.mask_id;
+        eh.logits = (ctx->debug & 1) ? ctx->logits : nullptr;
+        CK(gemm_launch(EPI_LMHEAD, ph, ctx->tm_head, tx_xn, eh, ctx->scr, ctx->status, s));
+        CK(launch_lmhead_reduce(ctx->lmp, ctx->zcur, ctx->cur, L.head_tiles, N, c.mask_id, ctx->x0, ctx->conf,
+                                ctx->tokconf, s));
+    }
+    return DLLM_OK;
+}
+
+static int step_kernels(dllm_ctx* ctx, int T) {
+    int rc = forward(ctx, ctx->B, T, true);
+    if (rc) return rc;
+    CommitArgs a{};
+    a.tok = ctx->tok;
+    a.st = ctx->st;
+    a.ld = ctx->cfg.max_ctx;
+    a.seq_kv = ctx->seq_kv;
+    a.plan = ctx->plan;
+    a.x0 = ctx->x0;
+    a.conf = ctx->conf;
+    a.tokconf = ctx->tokconf;
+    a.outs = ctx->outs;
+    a.B = ctx->B;
+    a.T = T;
+    a.mask_id = ctx->cfg.mask_id;
+    a.use_cache = ctx->sched.use_prefix_cache;
+    a.S = ctx->sched.steps_per_block;
+    a.remask_max = ctx->sched.remask_max;
+    a.spec_blocks = ctx->sched.spec_blocks;
+    a.block_len = ctx->cfg.block_len;
+    a.theta_remask = ctx->sched.theta_remask;
+    a.theta_stable = ctx->sched.theta_stable;
+    CK(launch_commit(a, ctx->stream));
+    return DLLM_OK;
+}
+
+// ------------------------------------------------------------------ ABI
+extern "C" {
+
+int dllm_arena_bytes(const dllm_config* cfg, size_t* bytes) {
+    if (!cfg || !bytes) return fail(nullptr, DLLM_EINVAL, "null argument");
+    if (const char* m = check_cfg(*cfg)) return fail(nullptr, DLLM_EINVAL, "%s", m);
+    *bytes = make_layout(*cfg).total;
+    return DLLM_OK;
+}
+
+const char* dllm_last_error(const dllm_ctx* ctx) { return ctx ? ctx->err.c_str() : g_noctx_err.c_str(); }
+
+void dllm_free(dllm_ctx* ctx) {
+    if (!ctx) return;
+    if (ctx->stream) cudaStreamSynchronize(ctx->stream);
+    if (ctx->gexec) cudaGraphExecDestroy(ctx->gexec);
+    if (ctx->logits) cudaFree(ctx->logits);
+    if (ctx->own_arena && ctx->arena) cudaFree(ctx->arena);
+    if (ctx->own_stream && ctx->stream) cudaStreamDestroy(ctx->stream);
+    delete ctx;
+}
+
+int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void* cuda_stream, dllm_ctx** out) {
+    if (!cfg || !out) return fail(nullptr, DLLM_EINVAL, "null argument");
+    *out = nullptr;
+    if (const char* m = check_cfg(*cfg)) return fail(nullptr, DLLM_EINVAL, "%s", m);
+    dllm_ctx* ctx = new (std::nothrow) dllm_ctx();
+    if (!ctx) return fail(nullptr, DLLM_ENOMEM, "host allocation failed");
+    ctx->cfg = *cfg;
+    ctx->L = make_layout(*cfg);
+    const Layout& L = ctx->L;
+    const dllm_config& c = ctx->cfg;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&ctx->sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) {
+        int rc = fail(nullptr, DLLM_ECUDA, "no CUDA device: %s", cudaGetErrorString(e));
+        delete ctx;
+        return rc;
+    }
+    ctx->sms = std::min(ctx->sms, kMaxSMs);
+    auto bail = [&](int code, const char* msg) {
+        g_noctx_err = msg;
+        dllm_free(ctx);
+        return code;
+    };
+    if (cuda_stream) {
+        ctx->stream = static_cast<cudaStream_t>(cuda_stream);
+    } else {
+        if (cudaStreamCreateWithFlags(&ctx->stream, cudaStreamNonBlocking) != cudaSuccess)
+            return bail(DLLM_ECUDA, "stream creation failed");
+        ctx->own_stream = true;
+    }
+    if (dev_arena) {
+        if (arena_bytes < L.total || (reinterpret_cast<uintptr_t>(dev_arena) & 255))
+            return bail(DLLM_EINVAL, "arena too small or not 256-byte aligned");
+        ctx->arena = static_cast<uint8_t*>(dev_arena);
+    } else {
+        if (cudaMalloc(&ctx->arena, L.total) != cudaSuccess) return bail(DLLM_ENOMEM, "device allocation failed");
+        ctx->own_arena = true;
+    }
+    if (gemm_init_attrs() != cudaSuccess || attn_init_attrs() != cudaSuccess)
+        return bail(DLLM_ECUDA, "kernel attribute setup failed");
+    uint8_t* A = ctx->arena;
+    const int d = c.d_model, F = c.ffn, qd = L.qd;
+    ctx->emb = reinterpret_cast<__nv_bfloat16*>(A + L.off_emb);
+    ctx->head = reinterpret_cast<__nv_bfloat16*>(A + L.off_head);
+    ctx->kv = reinterpret_cast<__nv_bfloat16*>(A + L.off_kv);
+    ctx->rope = reinterpret_cast<float*>(A + L.off_rope);
+    ctx->x = reinterpret_cast<float*>(A + L.off_x);
+    ctx->xn = reinterpret_cast<__nv_bfloat16*>(A + L.off_xn);
+    ctx->q = reinterpret_cast<__nv_bfloat16*>(A + L.off_q);
+    ctx->attn = reinterpret_cast<__nv_bfloat16*>(A + L.off_attn);
+    ctx->h = reinterpret_cast<__nv_bfloat16*>(A + L.off_h);
+    ctx->apo = reinterpret_cast<float*>(A + L.off_apo);
+    ctx->apml = reinterpret_cast<float*>(A + L.off_apml);
+    ctx->lmp = reinterpret_cast<float*>(A + L.off_lmp);
+    ctx->zcur = reinterpret_cast<float*>(A + L.off_zcur);
+    ctx->cur = reinterpret_cast<int*>(A + L.off_cur);
+    ctx->x0 = reinterpret_cast<int*>(A + L.off_x0);
+    ctx->conf = reinterpret_cast<float*>(A + L.off_conf);
+    ctx->tokconf = reinterpret_cast<float*>(A + L.off_tokconf);
+    ctx->scr.partials = reinterpret_cast<float*>(A + L.off_part);
+    ctx->scr.partial_floats = L.part_floats;
+    ctx->scr.counters = reinterpret_cast<int*>(A + L.off_cnt);
+    ctx->scr.counter_len = L.cnt_len;
+    ctx->tok = reinterpret_cast<int*>(A + L.off_tok);
+    ctx->st = A + L.off_st;
+    ctx->stok = reinterpret_cast<int*>(A + L.off_stok);
+    ctx->sst = A + L.off_sst;
+    ctx->seq_kv = reinterpret_cast<int*>(A + L.off_seqkv);
+    ctx->plan = reinterpret_cast<int*>(A + L.off_plan);
+    ctx->outs = reinterpret_cast<int*>(A + L.off_outs);
+    ctx->status = reinterpret_cast<int*>(A + L.off_status);
+    cudaStream_t s = ctx->stream;
+    // zero everything that is read before it is written (counters, state, status)
+    if (cudaMemsetAsync(A + L.off_lmp, 0, L.total - L.off_lmp, s) != cudaSuccess ||
+        cudaMemsetAsync(A + L.off_kv, 0, L.kv_half * 4 * c.n_layers, s) != cudaSuccess)
+        return bail(DLLM_ECUDA, "memset failed");
+    // weights from the seed (tensor ids: embedding 1, head 2, layer l: 16 + 8l + {q,k,v,o,gate,up,down})
+    const uint64_t seed = c.weight_seed;
+    cudaError_t ie = launch_init_weight(ctx->emb, 0, c.vocab, d, c.vocab, seed, 1, qd, s);
+    if (ie == cudaSuccess) ie = launch_init_weight(ctx->head, 0, L.head_rows, d, c.vocab, seed, 2, qd, s);
+    ctx->wl.resize(c.n_layers);
+    ctx->tm_qkv.resize(c.n_layers);
+    ctx->tm_o.resize(c.n_layers);
+    ctx->tm_gu.resize(c.n_layers);
+    ctx->tm_d.resize(c.n_layers);
+    for (int l = 0; l < c.n_layers && ie == cudaSuccess; ++l) {
+        __nv_bfloat16* w = reinterpret_cast<__nv_bfloat16*>(A + L.off_w) + static_cast<size_t>(l) * L.per_layer;
+        ctx->wl[l] = w;
+        const uint64_t t0 = 16 + 8ull * l;
+        ie = launch_init_weight(w + L.w_qkv, 1, L.qkv_rows, d, 3 * qd, seed, t0 + 0, qd, s);
+        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_o, 0, L.o_rows, qd, d, seed, t0 + 3, qd, s);
+        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_gu, 2, L.gu_rows, d, F, seed, t0 + 4, qd, s);
+        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_d, 0, L.d_rows, F, d, seed, t0 + 6, qd, s);
+        bool ok = make_tmap_bf16(&ctx->tm_qkv[l], w + L.w_qkv, L.qkv_rows, d, 128) &&
+                  make_tmap_bf16(&ctx->tm_o[l], w + L.w_o, L.o_rows, qd, 128) &&
+                  make_tmap_bf16(&ctx->tm_gu[l], w + L.w_gu, L.gu_rows, d, 128) &&
+                  make_tmap_bf16(&ctx->tm_d[l], w + L.w_d, L.d_rows, F, 128);
+        if (!ok) return bail(DLLM_ECUDA, "tensor map encode failed");
+    }
+    if (ie == cudaSuccess && !make_tmap_bf16(&ctx->tm_head, ctx->head, L.head_rows, d, 128))
+        return bail(DLLM_ECUDA, "tensor map encode failed");
+    if (ie == cudaSuccess) ie = launch_init_rope(ctx->rope, c.max_ctx, c.head_dim, c.rope_base, s);
+    if (ie != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess) return bail(DLLM_ECUDA, "weight init failed");
+    *out = ctx;
+    return DLLM_OK;
+}
+
+int dllm_sync(dllm_ctx* ctx) {
+    GUARD(ctx);
+    return sync_check(ctx);
+}
+
+static int set_debug_buffers(dllm_ctx* ctx) {
+    if (!(ctx->debug & 1)) return DLLM_OK;
+    size_t need = static_cast<size_t>(ctx->L.max_tok) * ctx->cfg.vocab;
+    if (ctx->logits_cap >= need) return DLLM_OK;
+    if (ctx->logits) cudaFree(ctx->logits);
+    ctx->logits = nullptr;
+    if (cudaMalloc(&ctx->logits, need * 4) != cudaSuccess) return fail(ctx, DLLM_ENOMEM, "logits buffer");
+    ctx->logits_cap = need;
+    return DLLM_OK;
+}
+
+int dllm_set_debug(dllm_ctx* ctx, int flags) {
+    GUARD(ctx);
+    ctx->debug = flags;
+    return set_debug_buffers(ctx);
+}
+
+static int start_request(dllm_ctx* ctx, const dllm_sched* sched, int batch, int Lp, int gen_len,
+                         const int32_t* prompt, int P_random, uint64_t kv_seed) {
+    const dllm_config& c = ctx->cfg;
+    if (!sched || batch < 1 || Lp < 0 || gen_len < 1) return fail(ctx, DLLM_EINVAL, "bad request arguments");
+    if (sched->steps_per_block < 1 || sched->remask_max < 0 || sched->spec_blocks < 0)
+        return fail(ctx, DLLM_EINVAL, "bad schedule");
+    if (batch > c.max_batch) return fail(ctx, DLLM_ECAPACITY, "batch %d > max_batch %d", batch, c.max_batch);
+    const int n_pos = Lp + gen_len;
+    if (n_pos > c.max_ctx) return fail(ctx, DLLM_ECAPACITY, "Lp + gen_len = %d > max_ctx %d", n_pos, c.max_ctx);
+    int maxT = sched->use_prefix_cache ? std::max(P_random ? 0 : Lp, c.block_len * (1 + sched->spec_blocks)) : n_pos;
+    if (maxT > c.max_window) return fail(ctx, DLLM_ECAPACITY, "window of %d tokens > max_window %d", maxT, c.max_window);
+    if (!sched->use_prefix_cache && gen_len > kMaxBlock) return fail(ctx, DLLM_ECAPACITY, "block too long");
+    ctx->sched = *sched;
+    ctx->B = batch;
+    ctx->Lp = Lp;
+    ctx->gen_len = gen_len;
+    ctx->n_pos = n_pos;
+    ctx->blk = -1;
+    ctx->have_block = false;
+    ctx->started = false;
+    ctx->step = 0;
+    ctx->kv_len = 0;
+    // state rows
+    std::vector<int32_t> tok(static_cast<size_t>(batch) * c.max_ctx, c.mask_id);
+    std::vector<uint8_t> st(static_cast<size_t>(batch) * c.max_ctx, DLLM_MASKED);
+    for (int b = 0; b < batch; ++b)
+        for (int p = 0; p < Lp; ++p) {
+            tok[static_cast<size_t>(b) * c.max_ctx + p] = prompt ? prompt[static_cast<size_t>(b) * Lp + p] : 0;
+            st[static_cast<size_t>(b) * c.max_ctx + p] = DLLM_FIXED;
+        }
+    if (prompt)
+        for (int b = 0; b < batch; ++b)
+            for (int p = 0; p < Lp; ++p) {
+                int v = prompt[static_cast<size_t>(b) * Lp + p];
+                if (v < 0 || v >= c.vocab) return fail(ctx, DLLM_EINVAL, "prompt id %d out of range", v);
+            }
+    CK(cudaMemcpyAsync(ctx->tok, tok.data(), tok.size() * 4, cudaMemcpyHostToDevice, ctx->stream));
+    CK(cudaMemcpyAsync(ctx->st, st.data(), st.size(), cudaMemcpyHostToDevice, ctx->stream));
+    CK(launch_set_kv_len(ctx->seq_kv, batch, 0, ctx->stream));
+    CK(cudaStreamSynchronize(ctx->stream));  // host vectors go out of scope
+    if (P_random) {
+        for (int l = 0; l < c.n_layers; ++l)
+            for (int w = 0; w < 2; ++w)
+                CK(launch_init_kv_random(ctx->kv + static_cast<size_t>(2 * l + w) * ctx->L.kv_half, batch, c.n_heads,
+                                         c.head_dim, c.max_ctx, Lp, l, w, c.n_layers, kv_seed, ctx->stream));
+        ctx->kv_len = Lp;
+        CK(launch_set_kv_len(ctx->seq_kv, batch, Lp, ctx->stream));
+    } else if (sched->use_prefix_cache && Lp > 0) {
+        int rc = forward(ctx, batch, Lp, false);
+        if (rc) return rc;
+        ctx->kv_len = Lp;
+        CK(launch_set_kv_len(ctx->seq_kv, batch, Lp, ctx->stream));
+    }
+    ctx->started = true;
+    return sync_check(ctx);
+}
+
+int dllm_prefill(dllm_ctx* ctx, const dllm_sched* sched, int batch, const int32_t* prompt, int Lp, int gen_len) {
+    GUARD(ctx);
+    if (!prompt && Lp > 0) return fail(ctx, DLLM_EINVAL, "null prompt");
+    return start_request(ctx, sched, batch, Lp, gen_len, prompt, 0, 0);
+}
+
+int dllm_set_prefix_kv_random(dllm_ctx* ctx, const dllm_sched* sched, int batch, int P, int gen_len, uint64_t seed) {
+    GUARD(ctx);
+    if (!sched || !sched->use_prefix_cache || P < 1) return fail(ctx, DLLM_EINVAL, "synthetic prefix needs the cache");
+    return start_request(ctx, sched, batch, P, gen_len, nullptr, 1, seed);
+}
+
+static int count_masked_max(dllm_ctx* ctx, int a, int b, int* out) {
+    const int ld = ctx->cfg.max_ctx;
+    std::vector<uint8_t> st(static_cast<size_t>(ctx->B) * ld);
+    CK(cudaMemcpyAsync(st.data(), ctx->st, st.size(), cudaMemcpyDeviceToHost, ctx->stream));
+    int rc = sync_check(ctx);
+    if (rc) return rc;
+    int mx = 0;
+    for (int s = 0; s < ctx->B; ++s) {
+        int m = 0;
+        for (int p = a; p < b; ++p) m += st[static_cast<size_t>(s) * ld + p] == DLLM_MASKED;
+        mx = std::max(mx, m);
+    }
+    *out = mx;
+    return DLLM_OK;
+}
+
+int dllm_begin_block(dllm_ctx* ctx) {
+    GUARD(ctx);
+    if (!ctx->started) return fail(ctx, DLLM_EINVAL, "no request: call dllm_prefill first");
+    const dllm_config& c = ctx->cfg;
+    if (ctx->have_block) {
+        int m = 0;
+        int rc = count_masked_max(ctx, ctx->c0, ctx->c1, &m);
+        if (rc) return rc;
+        if (m) return fail(ctx, DLLM_EINVAL, "current block still has %d masked positions", m);
+        if (ctx->sched.use_prefix_cache) {
+            // recompute the finished block's K/V from its final ids and append them
+            rc = forward(ctx, ctx->B, ctx->c1 - ctx->c0, false);
+            if (rc) return rc;
+            ctx->kv_len += ctx->c1 - ctx->c0;
+            CK(launch_set_kv_len(ctx->seq_kv, ctx->B, ctx->kv_len, ctx->stream));
+        }
+        ctx->have_block = false;
+    }
+    const int bl = ctx->sched.use_prefix_cache ? c.block_len : c.block_len;
+    int nb = ctx->blk + 1;
+    int c0 = ctx->Lp + nb * bl;
+    if (c0 >= ctx->n_pos) {
+        ctx->blk = nb;
+        int rc = sync_check(ctx);
+        return rc ? rc : DLLM_DONE;
+    }
+    ctx->blk = nb;
+    ctx->c0 = c0;
+    ctx->c1 = std::min(c0 + bl, ctx->n_pos);
+    ctx->step = 0;
+    CK(launch_begin_block(ctx->tok, ctx->st, ctx->stok, ctx->sst, c.max_ctx, ctx->n_pos, ctx->plan, ctx->B, ctx->c0,
+                          ctx->c1, ctx->stream));
+    ctx->have_block = true;
+    return DLLM_OK;
+}
+
+int dllm_rewind_block(dllm_ctx* ctx) {
+    GUARD(ctx);
+    if (!ctx->have_block) return fail(ctx, DLLM_EINVAL, "no current block");
+    CK(launch_rewind(ctx->tok, ctx->st, ctx->stok, ctx->sst, ctx->cfg.max_ctx, ctx->n_pos, ctx->plan, ctx->B,
+                     ctx->stream));
+    ctx->step = 0;
+    return DLLM_OK;
+}
+
+int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out) {
+    GUARD(ctx);
+    if (!ctx->have_block) return fail(ctx, DLLM_EINVAL, "no current block: call dllm_begin_block");
+    const dllm_sched& s = ctx->sched;
+    const int bl = ctx->cfg.block_len;
+    int w0, T, spec = 0;
+    if (s.use_prefix_cache) {
+        w0 = ctx->kv_len;
+        int w1 = ctx->c1;
+        if (s.spec_blocks > 0 && ctx->c1 < ctx->n_pos) {
+            int m = 0;
+            int rc = count_masked_max(ctx, ctx->c0, ctx->c1, &m);
+            if (rc) return rc;
+            if (m <= s.spec_trigger) {
+                spec = 1;
+                w1 = std::min(ctx->c1 + s.spec_blocks * bl, ctx->n_pos);
+            }
+        }
+        T = w1 - w0;
+    } else {
+        w0 = 0;
+        T = ctx->n_pos;
+    }
+    ctx->last_w0 = w0;
+    ctx->last_T = T;
+    ctx->last_spec = spec;
+    const bool use_graph = !(ctx->debug & 2);
+    if (use_graph) {
+        if (!ctx->gexec || ctx->g_T != T || ctx->g_B != ctx->B || ctx->g_kv != ctx->kv_len || ctx->g_dbg != ctx->debug) {
+            if (ctx->gexec) {
+                cudaGraphExecDestroy(ctx->gexec);
+                ctx->gexec = nullptr;
+            }
+            cudaGraph_t g = nullptr;
+            CK(cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal));
+            int rc = step_kernels(ctx, T);
+            cudaError_t ee = cudaStreamEndCapture(ctx->stream, &g);
+            if (rc) {
+                if (g) cudaGraphDestroy(g);
+                return rc;
+            }
+            if (ee != cudaSuccess) return fail(ctx, DLLM_ECUDA, "graph capture: %s", cudaGetErrorString(ee));
+            ee = cudaGraphInstantiate(&ctx->gexec, g, 0);
+            cudaGraphDestroy(g);
+            if (ee != cudaSuccess) return fail(ctx, DLLM_ECUDA, "graph instantiate: %s", cudaGetErrorString(ee));
+            ctx->g_T = T;
+            ctx->g_B = ctx->B;
+            ctx->g_kv = ctx->kv_len;
+            ctx->g_dbg = ctx->debug;
+        }
+        CK(cudaGraphLaunch(ctx->gexec, ctx->stream));
+    } else {
+        int rc = step_kernels(ctx, T);
+        if (rc) return rc;
+    }
+    ctx->step++;
+    if (out) {
+        std::vector<int> o(static_cast<size_t>(ctx->B) * 8);
+        CK(cudaMemcpyAsync(o.data(), ctx->outs, o.size() * 4, cudaMemcpyDeviceToHost, ctx->stream));
+        int rc = sync_check(ctx);
+        if (rc) return rc;
+        memset(out, 0, sizeof(*out));
+        out->block_done = 1;
+        for (int b = 0; b < ctx->B; ++b) {
+            const int* r = &o[static_cast<size_t>(b) * 8];
+            out->n_committed += r[0];
+            out->n_remasked += r[1];
+            out->n_stable += r[2];
+            out->n_drafts += r[3];
+            out->block_done &= r[4];
+            out->masked_after += r[5];
+        }
+    }
+    return DLLM_OK;
+}
+
+int dllm_generate(dllm_ctx* ctx, const dllm_sched* sched, int batch, const int32_t* prompt, int Lp, int gen_len,
+                  int32_t* out_tokens, dllm_stats* stats) {
+    GUARD(ctx);
+    int rc = dllm_prefill(ctx, sched, batch, prompt, Lp, gen_len);
+    if (rc) return rc;
+    dllm_stats stt{};
+    while ((rc = dllm_begin_block(ctx)) == DLLM_OK) {
+        dllm_step_out o{};
+        for (int guard = 0; guard < 4 * sched->steps_per_block + 4; ++guard) {
+            rc = dllm_denoise_step(ctx, &o);
+            if (rc) return rc;
+            stt.steps++;
+            stt.spec_steps += ctx->last_spec;
+            if (o.block_done) break;
+        }
+        if (!o.block_done) return fail(ctx, DLLM_ESTATE, "block did not finish");
+        stt.blocks++;
+    }
+    if (rc != DLLM_DONE) return rc;
+    if (stats) *stats = stt;
+    if (out_tokens) {
+        const int ld = ctx->cfg.max_ctx;
+        for (int b = 0; b < batch; ++b)
+            CK(cudaMemcpyAsync(out_tokens + static_cast<size_t>(b) * gen_len, ctx->tok + static_cast<size_t>(b) * ld + Lp,
+                               static_cast<size_t>(gen_len) * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    }
+    return sync_check(ctx);
+}
+
+int dllm_window(dllm_ctx* ctx, int32_t* info) {
+    GUARD(ctx);
+    if (!info) return fail(ctx, DLLM_EINVAL, "null info");
+    info[0] = ctx->last_w0;
+    info[1] = ctx->last_T;
+    info[2] = ctx->c0;
+    info[3] = ctx->c1;
+    info[4] = ctx->step;
+    info[5] = ctx->kv_len;
+    info[6] = ctx->last_spec;
+    return DLLM_OK;
+}
+
+int dllm_get_state(dllm_ctx* ctx, int32_t* tokens, uint8_t* status, int32_t* kv_len) {
+    GUARD(ctx);
+    if (!ctx->started) return fail(ctx, DLLM_EINVAL, "no request");
+    const int ld = ctx->cfg.max_ctx, n = ctx->n_pos;
+    for (int b = 0; b < ctx->B; ++b) {
+        if (tokens)
+            CK(cudaMemcpyAsync(tokens + static_cast<size_t>(b) * n, ctx->tok + static_cast<size_t>(b) * ld,
+                               static_cast<size_t>(n) * 4, cudaMemcpyDeviceToHost, ctx->stream));
+        if (status)
+            CK(cudaMemcpyAsync(status + static_cast<size_t>(b) * n, ctx->st + static_cast<size_t>(b) * ld, n,
+                               cudaMemcpyDeviceToHost, ctx->stream));
+    }
+    if (kv_len)
+        for (int b = 0; b < ctx->B; ++b) kv_len[b] = ctx->kv_len;
+    return sync_check(ctx);
+}
+
+int dllm_set_state(dllm_ctx* ctx, const int32_t* tokens, const uint8_t* status) {
+    GUARD(ctx);
+    if (!ctx->started) return fail(ctx, DLLM_EINVAL, "no request");
+    const int ld = ctx->cfg.max_ctx, n = ctx->n_pos;
+    for (int b = 0; b < ctx->B; ++b) {
+        if (tokens)
+            CK(cudaMemcpyAsync(ctx->tok + static_cast<size_t>(b) * ld, tokens + static_cast<size_t>(b) * n,
+                               static_cast<size_t>(n) * 4, cudaMemcpyHostToDevice, ctx->stream));
+        if (status)
+            CK(cudaMemcpyAsync(ctx->st + static_cast<size_t>(b) * ld, status + static_cast<size_t>(b) * n, n,
+                               cudaMemcpyHostToDevice, ctx->stream));
+    }
+    if (ctx->have_block) {  // the new state is what dllm_rewind_block returns to
+        const size_t rows = static_cast<size_t>(ctx->B) * ld;
+        CK(cudaMemcpyAsync(ctx->stok, ctx->tok, rows * 4, cudaMemcpyDeviceToDevice, ctx->stream));
+        CK(cudaMemcpyAsync(ctx->sst, ctx->st, rows, cudaMemcpyDeviceToDevice, ctx->stream));
+    }
+    return sync_check(ctx);  // the caller's buffers may be reused on return
+}
+
+int dllm_get_step_debug(dllm_ctx* ctx, float* logits, int32_t* argmax, float* conf, float* tokconf) {
+    GUARD(ctx);
+    const size_t n = static_cast<size_t>(ctx->B) * ctx->last_T;
+    if (logits) {
+        if (!(ctx->debug & 1) || !ctx->logits) return fail(ctx, DLLM_EINVAL, "logits need dllm_set_debug(1)");
+        CK(cudaMemcpyAsync(logits, ctx->logits, n * ctx->cfg.vocab * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    }
+    if (argmax) CK(cudaMemcpyAsync(argmax, ctx->x0, n * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    if (conf) CK(cudaMemcpyAsync(conf, ctx->conf, n * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    if (tokconf) CK(cudaMemcpyAsync(tokconf, ctx->tokconf, n * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    return sync_check(ctx);
+}
+
+int dllm_get_weight(dllm_ctx* ctx, int layer, int which, uint16_t* out, size_t n_elems) {
+    GUARD(ctx);
+    const dllm_config& c = ctx->cfg;
+    const Layout& L = ctx->L;
+    const int d = c.d_model, F = c.ffn, qd = L.qd;
+    if (!out) return fail(ctx, DLLM_EINVAL, "null output");
+    auto copy_rows = [&](const __nv_bfloat16* src, int rows, int cols, size_t dst_row0) -> int {
+        CK(cudaMemcpyAsync(out + dst_row0 * cols, src, static_cast<size_t>(rows) * cols * 2, cudaMemcpyDeviceToHost,
+                           ctx->stream));
+        return DLLM_OK;
+    };
+    int rc = DLLM_OK;
+    if (layer < 0) {
+        if (n_elems < static_cast<size_t>(c.vocab) * d) return fail(ctx, DLLM_EINVAL, "buffer too small");
+        if (which == 1) rc = copy_rows(ctx->emb, c.vocab, d, 0);
+        else if (which == 2) rc = copy_rows(ctx->head, c.vocab, d, 0);
+        else return fail(ctx, DLLM_EINVAL, "bad tensor");
+    } else {
+        if (layer >= c.n_layers || which < 0 || which > 6) return fail(ctx, DLLM_EINVAL, "bad tensor");
+        const __nv_bfloat16* w = ctx->wl[layer];
+        int rows = (which <= 2) ? qd : (which == 3 || which == 6) ? d : F;
+        int cols = (which == 3) ? qd : (which == 6) ? F : d;
+        if (n_elems < static_cast<size_t>(rows) * cols) return fail(ctx, DLLM_EINVAL, "buffer too small");
+        if (which <= 2) rc = copy_rows(w + L.w_qkv + static_cast<size_t>(which) * qd * d, qd, d, 0);
+        else if (which == 3) rc = copy_rows(w + L.w_o, d, qd, 0);
+        else if (which == 6) rc = copy_rows(w + L.w_d, d, F, 0);
+        else {
+            const int up = which == 5;
+            for (int t = 0; t * 64 < F && rc == DLLM_OK; ++t) {
+                int nr = std::min(64, F - t * 64);
+                rc = copy_rows(w + L.w_gu + (static_cast<size_t>(t) * 128 + up * 64) * d, nr, d, static_cast<size_t>(t) * 64);
+            }
+        }
+    }
+    if (rc) return rc;
+    return sync_check(ctx);
+}
+
+int dllm_get_kv(dllm_ctx* ctx, int layer, int which, int seq, int p0, int n, float* out) {
+    GUARD(ctx);
+    const dllm_config& c = ctx->cfg;
+    if (!out || layer < 0 || layer >= c.n_layers || which < 0 || which > 1 || seq < 0 || seq >= c.max_batch || p0 < 0 ||
+        n < 0 || p0 + n > c.max_ctx)
+        return fail(ctx, DLLM_EINVAL, "bad KV slice");
+    const int H = c.n_heads, hd = c.head_dim, qd = H * hd;
+    std::vector<uint16_t> buf(static_cast<size_t>(H) * n * hd);
+    const __nv_bfloat16* base = ctx->kv + static_cast<size_t>(2 * layer + which) * ctx->L.kv_half;
+    for (int h = 0; h < H; ++h)
+        CK(cudaMemcpyAsync(buf.data() + static_cast<size_t>(h) * n * hd,
+                           base + ((static_cast<size_t>(seq) * H + h) * c.max_ctx + p0) * hd,
+                           static_cast<size_t>(n) * hd * 2, cudaMemcpyDeviceToHost, ctx->stream));
+    int rc = sync_check(ctx);
+    if (rc) return rc;
+    for (int p = 0; p < n; ++p)
+        for (int h = 0; h < H; ++h)
+            for (int i = 0; i < hd; ++i) {
+                uint32_t bits = static_cast<uint32_t>(buf[(static_cast<size_t>(h) * n + p) * hd + i]) << 16;
+                float f;
+                memcpy(&f, &bits, 4);
+                out[static_cast<size_t>(p) * qd + h * hd + i] = f;
+            }
+    return DLLM_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,487 @@
+// Weight-streaming GEMM on the 5th-generation tensor cores (tcgen05 + TMEM).
+//
+// D[m][n] = sum_k W[m][k] * X[n][k]: W are the layer weights (bf16, K-major,
+// rows padded to 128), X the activations of the window's tokens (bf16,
+// K-major).  The weight rows sit on the UMMA M axis (128 per tile) and the
+// tokens on the N axis, so at batch 1 (32 tokens) one UMMA instruction
+// covers the whole token set and the kernel is a pure stream of weight
+// bytes; at batch 16 (1024 tokens) the same kernel runs 128 x 256 tiles.
+//
+// Work is split "stream-K" style: the flattened (tile, 64-wide k-block)
+// iteration space is cut into one contiguous range per CTA (one CTA per SM),
+// so every SM streams the same number of weight bytes whatever the tile
+// count.  A tile cut between CTAs is finished by whichever CTA arrives last
+// (atomic ticket), which sums the fp32 partials in k order: deterministic,
+// and nobody waits on anybody.
+//
+// Roles (192 threads): warp 0 = TMA producer, warp 1 = TMEM owner and MMA
+// issuer, warps 2..5 = epilogue (one TMEM lane quarter each).  Accumulators
+// are double-buffered in TMEM so the epilogue of one tile overlaps the MMAs
+// of the next.  Epilogues are fused: residual add, RoPE + KV-cache write,
+// SwiGLU, and the LM head's per-tile softmax statistics.
+#include "common.cuh"
+#include "internal.h"
+
+#include <climits>
+#include <cstdio>
+
+namespace dllm {
+
+constexpr int kBK = 64;     // K elements per stage: one 128-byte swizzle row
+constexpr int kBM = 128;    // UMMA M
+constexpr int kThreads = 192;
+constexpr int kStageLd = 33;
+constexpr uint32_t kABytes = kBM * kBK * 2;
+
+__device__ __forceinline__ int owner_of(long long i, long long total, int G) {
+    return static_cast<int>(((i + 1) * G + total - 1) / total) - 1;
+}
+
+__device__ __forceinline__ long long range_begin(int c, long long total, int G) { return total * c / G; }
+
+// ------------------------------------------------------------------ epilogues
+template <int EPI>
+__device__ __forceinline__ void epilogue_chunk(const EpiArgs& ep, const GemmPlan& p, int mt, int nt, int chunk,
+                                               int rt, const float* v, float* stg, int ew, int lane, int* status) {
+    const int row = mt * kBM + rt;
+    const int col0 = nt * p.ntile + chunk * 32;
+    if constexpr (EPI == EPI_F32 || EPI == EPI_RESID) {
+        if (row < p.M) {
+#pragma unroll 8
+            for (int j = 0; j < 32; ++j) {
+                int col = col0 + j;
+                if (col < p.N) {
+                    float* o = ep.out + static_cast<size_t>(col) * ep.ld_out + row;
+                    if constexpr (EPI == EPI_F32) *o = v[j]; else *o += v[j];
+                }
+            }
+        }
+        return;
+    } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) stg[rt * kStageLd + j] = v[j];
+        named_bar(1, 128);
+        if constexpr (EPI == EPI_QKV) {
+            const int qd = ep.H * ep.hd;
+            const int part = row / qd;
+            const int f = row - part * qd;
+            const int hh = f / ep.hd;
+            const int i = f - hh * ep.hd;
+            const int half = ep.hd >> 1;
+            const int partner = rt ^ half;
+            const int ii = i & (half - 1);
+            for (int j = 0; j < 32; ++j) {
+                int col = col0 + j;
+                if (col >= p.N) break;
+                int b = col / ep.T;
+                int t = col - b * ep.T;
+                int pos = ep.seq_kv[b] + t;
+                if (pos < 0 || pos >= ep.cap) {
+                    atomicOr(status, kStatusBadIndex);
+                    continue;
+                }
+                float x = v[j];
+                if (part < 2) {
+                    float xp = stg[partner * kStageLd + j];
+                    const float* cs = ep.rope + (static_cast<size_t>(pos) * half + ii) * 2;
+                    x = (i < half) ? (x * cs[0] - xp * cs[1]) : (x * cs[0] + xp * cs[1]);
+                }
+                __nv_bfloat16 y = __float2bfloat16_rn(x);
+                if (part == 0) {
+                    ep.q[((static_cast<size_t>(b) * ep.H + hh) * ep.T + t) * ep.hd + i] = y;
+                } else {
+                    __nv_bfloat16* c = part == 1 ? ep.kc : ep.vc;
+                    c[((static_cast<size_t>(b) * ep.H + hh) * ep.cap + pos) * ep.hd + i] = y;
+                }
+            }
+        } else if constexpr (EPI == EPI_SWIGLU) {
+            if (rt < 64) {
+                const int f = mt * 64 + rt;
+                if (f < ep.F) {
+                    for (int j = 0; j < 32; ++j) {
+                        int col = col0 + j;
+                        if (col >= p.N) break;
+                        float g = v[j];
+                        float u = stg[(rt + 64) * kStageLd + j];
+                        float s = g / (1.0f + expf(-g));
+                        ep.h[static_cast<size_t>(col) * ep.F + f] = __float2bfloat16_rn(s * u);
+                    }
+                }
+            }
+        } else if constexpr (EPI == EPI_LMHEAD) {
+            if (ep.logits && row < ep.V) {
+                for (int j = 0; j < 32; ++j) {
+                    int col = col0 + j;
+                    if (col < p.N) ep.logits[static_cast<size_t>(col) * ep.V + row] = v[j];
+                }
+            }
+            for (int jj = ew; jj < 32; jj += 4) {
+                int col = col0 + jj;
+                if (col >= p.N) break;
+                float m = -INFINITY;
+                int idx = INT_MAX;
+                float z[4];
+                bool ok[4];
+#pragma unroll
+                for (int r = 0; r < 4; ++r) {
+                    int rr = lane + 32 * r;
+                    int id = mt * kBM + rr;
+                    ok[r] = id < ep.V && id != ep.mask_id;
+                    z[r] = stg[rr * kStageLd + jj];
+                    if (ok[r] && z[r] > m) { m = z[r]; idx = id; }
+                }
+#pragma unroll
+                for (int off = 16; off > 0; off >>= 1) {
+                    float om = __shfl_xor_sync(0xffffffffu, m, off);
+                    int oi = __shfl_xor_sync(0xffffffffu, idx, off);
+                    if (om > m || (om == m && oi < idx)) { m = om; idx = oi; }
+                }
+                float s = 0.0f;
+                if (m != -INFINITY) {
+#pragma unroll
+                    for (int r = 0; r < 4; ++r)
+                        if (ok[r]) s += expf(z[r] - m);
+                }
+#pragma unroll
+                for (int off = 16; off > 0; off >>= 1) s += __shfl_down_sync(0xffffffffu, s, off);
+                if (lane == 0) {
+                    float* o = ep.lm_part + (static_cast<size_t>(mt) * p.N + col) * 3;
+                    o[0] = m;
+                    o[1] = s;
+                    o[2] = __int_as_float(idx);
+                    int cur = ep.cur_tok[col];
+                    if (cur >= mt * kBM && cur < mt * kBM + kBM) ep.zcur[col] = stg[(cur - mt * kBM) * kStageLd + jj];
+                }
+            }
+        }
+        named_bar(1, 128);
+    }
+}
+
+// ------------------------------------------------------------------ kernel
+template <int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_gemm(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX, const GemmPlan p,
+           const EpiArgs ep, float* __restrict__ partials, int* __restrict__ counters, int* status) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int S = p.stages;
+    const uint32_t b_bytes = static_cast<uint32_t>(p.ntile) * kBK * 2;
+    uint8_t* sA = smem;
+    uint8_t* sB = sA + static_cast<size_t>(S) * kABytes;
+    float* stg = reinterpret_cast<float*>(sB + static_cast<size_t>(S) * b_bytes);
+    uint64_t* full = reinterpret_cast<uint64_t*>(stg + kBM * kStageLd);
+    uint64_t* empty = full + S;
+    uint64_t* tfull = empty + S;
+    uint64_t* tempty = tfull + 2;
+    uint64_t* drain = tempty + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    volatile int* s_abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    volatile int* s_last = s_abort + 1;
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int G = p.grid;
+    const long long it0 = range_begin(blockIdx.x, p.total, G);
+    const long long it1 = range_begin(blockIdx.x + 1, p.total, G);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(&tfull[a], 1);
+            mbar_init(&tempty[a], 128);
+        }
+        mbar_init(drain, 1);
+        *s_abort = 0;
+        *s_last = 0;
+        mbar_fence_init();
+    }
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_desc(&tmW);
+        tma_prefetch_desc(&tmX);
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_slot, p.tmem_cols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    if (warp == 0) {
+        // ---------------------------------------------------------- producer
+        if (lane == 0) {
+            const uint64_t pol_w = policy_evict_first();
+            const uint64_t pol_x = policy_evict_last();
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t pending = 0;   // stages with a load in flight
+            uint32_t pend_par = 0;  // parity of that load's phase
+            for (long long it = it0; it < it1; ++it) {
+                const long long tile = it / p.kb;
+                const int k = static_cast<int>(it - tile * p.kb);
+                const int mt = static_cast<int>(tile / p.n_tiles);
+                const int nt = static_cast<int>(tile - static_cast<long long>(mt) * p.n_tiles);
+                if (!mbar_wait(&empty[stage], phase ^ 1u, s_abort, status)) break;
+                mbar_arrive_expect_tx(&full[stage], kABytes + b_bytes);
+                tma_load_2d(sA + static_cast<size_t>(stage) * kABytes, &tmW, k * kBK, mt * kBM, &full[stage], pol_w);
+                tma_load_2d(sB + static_cast<size_t>(stage) * b_bytes, &tmX, k * kBK, nt * p.ntile, &full[stage],
+                            pol_x);
+                pending |= 1u << stage;
+                pend_par = (pend_par & ~(1u << stage)) | (phase << stage);
+                if (++stage == S) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+            if (*s_abort) {
+                // let every copy already issued land before the CTA's shared memory is released
+                for (int s = 0; s < S; ++s) {
+                    if (!(pending >> s & 1u)) continue;
+                    unsigned long long t0 = global_ns();
+                    while (!mbar_try_wait(&full[s], (pend_par >> s) & 1u) && global_ns() - t0 < kWaitLimitNs) {
+                    }
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ---------------------------------------------------------- MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = umma_idesc_bf16(kBM, p.ntile);
+            int stage = 0;
+            uint32_t phase = 0;
+            int acc = 0;
+            uint32_t acc_phase = 0;
+            bool issued = false;
+            for (long long it = it0; it < it1 && !*s_abort;) {
+                const long long tile = it / p.kb;
+                const int k_lo = static_cast<int>(it - tile * p.kb);
+                const long long tend = (tile + 1) * p.kb;
+                const int k_hi = static_cast<int>((it1 < tend ? it1 : tend) - tile * p.kb);
+                if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, s_abort, status)) break;
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * p.acc_cols);
+                bool ok = true;
+                for (int k = k_lo; k < k_hi; ++k) {
+                    if (!mbar_wait(&full[stage], phase, s_abort, status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint64_t adesc = sw128_kmajor_desc(smem_u32(sA + static_cast<size_t>(stage) * kABytes));
+                    const uint64_t bdesc = sw128_kmajor_desc(smem_u32(sB + static_cast<size_t>(stage) * b_bytes));
+#pragma unroll
+                    for (int kk = 0; kk < kBK / 16; ++kk) {
+                        // +32 bytes per 16-element K step inside the 128-byte swizzle row
+                        umma_bf16(d_tmem, adesc + 2ull * kk, bdesc + 2ull * kk, idesc, (k > k_lo || kk > 0) ? 1u : 0u);
+                    }
+                    issued = true;
+                    umma_commit(&empty[stage]);
+                    if (++stage == S) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+                if (!ok) break;
+                umma_commit(&tfull[acc]);
+                if (++acc == 2) {
+                    acc = 0;
+                    acc_phase ^= 1u;
+                }
+                it = tile * p.kb + k_hi;
+            }
+            if (*s_abort && issued) {
+                // wait for the tensor cores before the accumulator memory is released
+                umma_commit(drain);
+                unsigned long long t0 = global_ns();
+                while (!mbar_try_wait(drain, 0) && global_ns() - t0 < kWaitLimitNs) {
+                }
+            }
+        }
+    } else {
+        // ---------------------------------------------------------- epilogue
+        const int ew = warp - 2;                 // 0..3
+        const int quarter = warp & 3;            // TMEM lane quarter this warp may access
+        const int rt = quarter * 32 + lane;      // row within the 128-row tile
+        const int nchunks = p.ntile / 32;
+        const size_t slot_floats = static_cast<size_t>(p.ntile) * kBM;
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        float v[32];
+        for (long long it = it0; it < it1;) {
+            const long long tile = it / p.kb;
+            const int k_lo = static_cast<int>(it - tile * p.kb);
+            const long long tend = (tile + 1) * p.kb;
+            const int k_hi = static_cast<int>((it1 < tend ? it1 : tend) - tile * p.kb);
+            const int mt = static_cast<int>(tile / p.n_tiles);
+            const int nt = static_cast<int>(tile - static_cast<long long>(mt) * p.n_tiles);
+            mbar_wait(&tfull[acc], acc_phase, s_abort, status);
+            named_bar(1, 128);
+            if (*s_abort) break;
+            tc_fence_after();
+            const uint32_t t_acc = tmem_base + static_cast<uint32_t>(acc * p.acc_cols) +
+                                   (static_cast<uint32_t>(quarter * 32) << 16);
+            const bool whole = (k_lo == 0 && k_hi == p.kb);
+            const int slot = (range_begin(blockIdx.x, p.total, G) / p.kb == tile) ? 0 : 1;
+            float* my_part = partials + (static_cast<size_t>(blockIdx.x) * 2 + slot) * slot_floats;
+            for (int c = 0; c < nchunks; ++c) {
+                tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);
+                if (whole) {
+                    epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, stg, ew, lane, status);
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) my_part[static_cast<size_t>(c * 32 + j) * kBM + rt] = v[j];
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(&tempty[acc]);
+            if (++acc == 2) {
+                acc = 0;
+                acc_phase ^= 1u;
+            }
+            if (!whole) {
+                // last-arriver reduction of a tile split between CTAs
+                __threadfence();
+                named_bar(1, 128);
+                if (threadIdx.x == 64) {
+                    const int c_first = owner_of(tile * p.kb, p.total, G);
+                    const int c_last = owner_of(tile * p.kb + p.kb - 1, p.total, G);
+                    const int prev = atomicAdd(&counters[tile], 1);
+                    const int last = prev == c_last - c_first;
+                    if (last) counters[tile] = 0;
+                    *s_last = last;
+                }
+                named_bar(1, 128);
+                if (*s_last) {
+                    __threadfence();
+                    const int c_first = owner_of(tile * p.kb, p.total, G);
+                    const int c_last = owner_of(tile * p.kb + p.kb - 1, p.total, G);
+                    for (int c = 0; c < nchunks; ++c) {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+                        for (int cc = c_first; cc <= c_last; ++cc) {
+                            const int sl = (range_begin(cc, p.total, G) / p.kb == tile) ? 0 : 1;
+                            const float* pp = partials + (static_cast<size_t>(cc) * 2 + sl) * slot_floats +
+                                              static_cast<size_t>(c * 32) * kBM + rt;
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) v[j] += __ldcg(pp + static_cast<size_t>(j) * kBM);
+                        }
+                        epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, stg, ew, lane, status);
+                    }
+                }
+            }
+            it = tile * p.kb + k_hi;
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) {
+        __syncwarp();
+        tmem_dealloc(tmem_base, p.tmem_cols);
+    }
+}
+
+// ------------------------------------------------------------------ host side
+static int pow2ceil(int x) {
+    int p = 32;
+    while (p < x) p <<= 1;
+    return p;
+}
+
+GemmPlan gemm_plan(int M, int N, int K, int grid_max) {
+    GemmPlan p{};
+    p.M = M;
+    p.N = N;
+    p.K = K;
+    p.n_tiles = (N + 255) / 256;
+    int per = (N + p.n_tiles - 1) / p.n_tiles;
+    p.ntile = ((per + 31) / 32) * 32;
+    p.m_tiles = (M + kBM - 1) / kBM;
+    p.kb = (K + kBK - 1) / kBK;
+    p.total = static_cast<long long>(p.m_tiles) * p.n_tiles * p.kb;
+    p.grid = static_cast<int>(p.total < grid_max ? p.total : grid_max);
+    if (p.grid < 1) p.grid = 1;
+    p.acc_cols = pow2ceil(p.ntile);
+    p.tmem_cols = 2 * p.acc_cols;
+    const int fixed = 1024 + kBM * kStageLd * 4 + 64 * 8 + 64;
+    const int stage_bytes = static_cast<int>(kABytes) + p.ntile * kBK * 2;
+    int st = (227 * 1024 - fixed) / stage_bytes;
+    if (st > 16) st = 16;
+    p.stages = st;
+    p.smem = static_cast<size_t>(fixed) + static_cast<size_t>(st) * stage_bytes;
+    return p;
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn get_encode() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void* ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    }
+    return fn;
+}
+
+bool make_tmap_bf16(CUtensorMap* tm, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+    EncodeTiledFn enc = get_encode();
+    if (!enc) return false;
+    if ((reinterpret_cast<uintptr_t>(ptr) & 15) || ((cols * 2) & 15) || box_rows == 0 || box_rows > 256) return false;
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {cols * 2};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+template <int EPI>
+static cudaError_t launch_t(const GemmPlan& p, const CUtensorMap& tmW, const CUtensorMap& tmX, const EpiArgs& ep,
+                            const Scratch& scr, int* status, cudaStream_t st) {
+    k_gemm<EPI><<<p.grid, kThreads, p.smem, st>>>(tmW, tmX, p, ep, scr.partials, scr.counters, status);
+    return cudaGetLastError();
+}
+
+cudaError_t gemm_init_attrs() {
+    cudaError_t e = cudaSuccess;
+    auto set = [&](const void* f) {
+        if (e == cudaSuccess) e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+    };
+    set(reinterpret_cast<const void*>(k_gemm<EPI_F32>));
+    set(reinterpret_cast<const void*>(k_gemm<EPI_RESID>));
+    set(reinterpret_cast<const void*>(k_gemm<EPI_QKV>));
+    set(reinterpret_cast<const void*>(k_gemm<EPI_SWIGLU>));
+    set(reinterpret_cast<const void*>(k_gemm<EPI_LMHEAD>));
+    return e;
+}
+
+cudaError_t gemm_launch(int epi, const GemmPlan& p, const CUtensorMap& tmW, const CUtensorMap& tmX,
+                        const EpiArgs& ep, const Scratch& scr, int* status, cudaStream_t st) {
+    if (static_cast<size_t>(p.grid) * 2 * p.ntile * kBM > scr.partial_floats ||
+        static_cast<long long>(p.m_tiles) * p.n_tiles > scr.counter_len)
+        return cudaErrorInvalidValue;
+    switch (epi) {
+        case EPI_F32: return launch_t<EPI_F32>(p, tmW, tmX, ep, scr, status, st);
+        case EPI_RESID: return launch_t<EPI_RESID>(p, tmW, tmX, ep, scr, status, st);
+        case EPI_QKV: return launch_t<EPI_QKV>(p, tmW, tmX, ep, scr, status, st);
+        case EPI_SWIGLU: return launch_t<EPI_SWIGLU>(p, tmW, tmX, ep, scr, status, st);
+        case EPI_LMHEAD: return launch_t<EPI_LMHEAD>(p, tmW, tmX, ep, scr, status, st);
+    }
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace dllm

@@ -1,0 +1,117 @@
+// Internal declarations shared by the library's translation units.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace dllm {
+
+constexpr int kMaxBlock = 4096;
+constexpr int kStatusTimeout = 1;  // device status word bits
+constexpr int kStatusBadIndex = 2;  // longest current block the commit pass handles
+
+// ---------------------------------------------------------------- GEMM
+// D = W * X^T on tensor cores: W bf16 [M][K] (weights, rows padded to 128),
+// X bf16 [N][K] (tokens).  Row m of D is an output feature, column n a token.
+enum EpiKind { EPI_F32 = 0, EPI_RESID = 1, EPI_QKV = 2, EPI_SWIGLU = 3, EPI_LMHEAD = 4 };
+
+struct EpiArgs {
+    float* out;          // EPI_F32: D[n][m] (ld = ld_out); EPI_RESID: residual x[n][m] += D
+    int ld_out;
+    // EPI_QKV: rows [0,qd) q, [qd,2qd) k, [2qd,3qd) v; rotate-half RoPE on q, k
+    __nv_bfloat16* q;    // [B][H][T][hd]
+    __nv_bfloat16* kc;   // layer's K cache base: [B][H][cap][hd]
+    __nv_bfloat16* vc;
+    const float* rope;   // [cap][hd/2][2] (cos, sin)
+    const int* seq_kv;   // per-sequence first window position (kv_len)
+    int T, H, hd, cap;
+    // EPI_SWIGLU: tile k rows 0..63 gate(64k..), rows 64..127 up(64k..)
+    __nv_bfloat16* h;    // [N][F]
+    int F;
+    // EPI_LMHEAD
+    float* lm_part;      // [m_tiles][N][3]: max, sum exp(z - max), argmax (as float bits)
+    float* zcur;         // [N]: logit of the current token id
+    const int* cur_tok;  // [N]
+    float* logits;       // [N][V] or null
+    int V, mask_id;
+};
+
+struct GemmPlan {
+    int M, N, K;
+    int ntile;           // token tile (UMMA N), multiple of 16, <= 256
+    int m_tiles, n_tiles, kb;
+    long long total;     // m_tiles * n_tiles * kb iterations of 64-wide K blocks
+    int grid;            // CTAs (stream-K partition of the iterations)
+    int stages;
+    int acc_cols;        // TMEM columns per accumulator buffer
+    int tmem_cols;       // allocation (power of two)
+    size_t smem;
+};
+
+struct Scratch {
+    float* partials;     // [grid][2][ntile*128]
+    int* counters;       // [m_tiles*n_tiles], zero between launches
+    size_t partial_floats;
+    int counter_len;
+};
+
+GemmPlan gemm_plan(int M, int N, int K, int grid_max);
+bool make_tmap_bf16(CUtensorMap* tm, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows);
+cudaError_t gemm_launch(int epi, const GemmPlan& p, const CUtensorMap& tmW, const CUtensorMap& tmX,
+                        const EpiArgs& ep, const Scratch& scr, int* status, cudaStream_t st);
+
+// ---------------------------------------------------------------- other kernels
+cudaError_t launch_init_weight(__nv_bfloat16* dst, int mode, int rows_phys, int cols, int logical_rows,
+                               uint64_t seed, uint64_t tid0, int qd, cudaStream_t st);
+cudaError_t launch_init_rope(float* rope, int cap, int hd, double base, cudaStream_t st);
+cudaError_t launch_init_kv_random(__nv_bfloat16* cache, int B, int H, int hd, int cap, int P, int layer,
+                                  int which, int L, uint64_t seed, cudaStream_t st);
+cudaError_t launch_embed_norm(const int* tok, int tok_ld, const int* seq_kv, const __nv_bfloat16* emb,
+                              float* x, __nv_bfloat16* xn, int B, int T, int d, float eps, cudaStream_t st);
+cudaError_t launch_rmsnorm(const float* x, __nv_bfloat16* xn, int ntok, int d, float eps, cudaStream_t st);
+// Attention split plan: CTAs (split, head, sequence x 64-query tile), each
+// over `chunk` keys; nsplit > 1 adds a combine pass over fp32 partials
+// part_o [B][H][nsplit][T][hd] and part_ml [B][H][nsplit][T][2].
+struct AttnPlan {
+    int qtiles, chunk, nsplit;
+};
+AttnPlan attn_plan(int B, int T, int H, int max_keys, int sms);
+cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
+                             const int* seq_kv, float* part_o, float* part_ml, __nv_bfloat16* out, int B, int T,
+                             int H, int hd, int cap, const AttnPlan& a, cudaStream_t st);
+cudaError_t launch_lmhead_reduce(const float* lm_part, const float* zcur, const int* cur_tok, int m_tiles,
+                                 int N, int mask_id, int* x0, float* conf, float* tokconf, cudaStream_t st);
+cudaError_t launch_gather_cur(const int* tok, int tok_ld, const int* seq_kv, int* cur, int B, int T,
+                              cudaStream_t st);
+
+// Commit pass.  Per sequence b: state arrays at tok + b*ld, st + b*ld; the
+// window starts at seq_kv[b] (prefix cache on) or 0 (off); plan[b] holds
+// {c0, c1, step}.
+struct CommitArgs {
+    int* tok;
+    uint8_t* st;
+    int ld;
+    const int* seq_kv;
+    int* plan;           // [B][4]: c0, c1, step, spare
+    const int* x0;       // [B][T] window-indexed
+    const float* conf;
+    const float* tokconf;
+    int* outs;           // [B][8]: committed, remasked, stable, drafts, done, masked_after
+    int B, T, mask_id, use_cache;
+    int S, remask_max, spec_blocks, block_len;
+    float theta_remask, theta_stable;
+};
+cudaError_t launch_commit(const CommitArgs& a, cudaStream_t st);
+
+cudaError_t launch_begin_block(int* tok, uint8_t* st, int* snap_tok, uint8_t* snap_st, int ld, int n_pos, int* plan,
+                               int B, int c0, int c1, cudaStream_t stream);
+cudaError_t launch_rewind(int* tok, uint8_t* st, const int* snap_tok, const uint8_t* snap_st, int ld, int n_pos,
+                          int* plan, int B, cudaStream_t stream);
+cudaError_t launch_set_kv_len(int* seq_kv, int B, int v, cudaStream_t stream);
+cudaError_t gemm_init_attrs();
+cudaError_t attn_init_attrs();
+
+}  // namespace dllm

@@ -1,0 +1,762 @@
+// Element-wise, normalisation, attention and bookkeeping kernels of the
+// denoising step.  The dense projections live in gemm_tc.cu.
+#include "common.cuh"
+#include "internal.h"
+
+#include <climits>
+
+namespace dllm {
+
+// ------------------------------------------------------------------ weight generator
+// SplitMix64 (Steele, Lea & Flood, OOPSLA 2014): the n-th output of a stream
+// whose state starts at `key` is mix(key + (n+1) * golden_gamma).
+__host__ __device__ __forceinline__ uint64_t sm64_at_hd(uint64_t key, uint64_t n) {
+    uint64_t z = key + (n + 1ull) * 0x9E3779B97F4A7C15ull;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+// Element i of a tensor: four 32-bit draws summed (Irwin-Hall of order 4),
+// centred at 2^33, scaled by sqrt(3)/2^32 to unit variance, times sigma;
+// each double operation rounded once (IEEE round-to-nearest).
+__device__ __forceinline__ float gen_value(uint64_t key, uint64_t i, double sigma) {
+    uint64_t s = 0;
+#pragma unroll
+    for (uint64_t j = 0; j < 4; ++j) s += sm64_at_hd(key, 4ull * i + j) >> 32;
+    double centred = __dsub_rn(__ull2double_rn(s), 8589934592.0);
+    double unit = __dmul_rn(centred, 0x1.bb67ae8584caap-32);
+    double scaled = __dmul_rn(unit, sigma);
+    return __double2float_rn(scaled);
+}
+
+// mode 0: plain (physical row = logical row of tensor tid0, zero rows past
+//         logical_rows);
+// mode 1: fused QKV (rows [0,qd) tensor tid0, [qd,2qd) tid0+1, [2qd,3qd) tid0+2);
+// mode 2: fused gate/up: 128-row tile k = gate rows 64k..64k+63 (tensor tid0),
+//         then up rows 64k..64k+63 (tensor tid0+1), zero past logical_rows.
+__global__ void k_init_weight(__nv_bfloat16* dst, int mode, int rows, int cols, int logical_rows, uint64_t seed,
+                              uint64_t tid0, int qd) {
+    const size_t n = static_cast<size_t>(rows) * cols;
+    for (size_t e = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; e < n;
+         e += static_cast<size_t>(gridDim.x) * blockDim.x) {
+        int r = static_cast<int>(e / cols);
+        int c = static_cast<int>(e - static_cast<size_t>(r) * cols);
+        uint64_t tid = tid0;
+        int lr = r;
+        if (mode == 1) {
+            tid = tid0 + r / qd;
+            lr = r % qd;
+        } else if (mode == 2) {
+            int tile = r >> 7, w = r & 127;
+            tid = tid0 + (w >= 64 ? 1 : 0);
+            lr = tile * 64 + (w & 63);
+        }
+        float v = 0.0f;
+        if (lr < logical_rows) {
+            uint64_t key = sm64_at_hd(seed, tid);
+            v = gen_value(key, static_cast<uint64_t>(lr) * cols + c, 0.02);
+        }
+        dst[e] = __float2bfloat16_rn(v);
+    }
+}
+
+cudaError_t launch_init_weight(__nv_bfloat16* dst, int mode, int rows_phys, int cols, int logical_rows,
+                               uint64_t seed, uint64_t tid0, int qd, cudaStream_t st) {
+    size_t n = static_cast<size_t>(rows_phys) * cols;
+    int blocks = static_cast<int>((n + 255) / 256 < 65536 ? (n + 255) / 256 : 65536);
+    k_init_weight<<<blocks, 256, 0, st>>>(dst, mode, rows_phys, cols, logical_rows, seed, tid0, qd);
+    return cudaGetLastError();
+}
+
+// Synthetic prefix KV: cache[b][h][pos][i] for pos < P is element pos*qd + h*hd + i
+// of tensor 2^32 + ((b*L + layer)*2 + which), sigma 1.
+__global__ void k_init_kv(__nv_bfloat16* cache, int B, int H, int hd, int cap, int P, int layer, int which, int L,
+                          uint64_t seed) {
+    const size_t n = static_cast<size_t>(B) * H * P * hd;
+    const int qd = H * hd;
+    for (size_t e = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; e < n;
+         e += static_cast<size_t>(gridDim.x) * blockDim.x) {
+        int i = static_cast<int>(e % hd);
+        size_t r = e / hd;
+        int pos = static_cast<int>(r % P);
+        r /= P;
+        int h = static_cast<int>(r % H);
+        int b = static_cast<int>(r / H);
+        uint64_t tid = 0x100000000ull + (static_cast<uint64_t>(b) * L + layer) * 2ull + which;
+        uint64_t key = sm64_at_hd(seed, tid);
+        float v = gen_value(key, static_cast<uint64_t>(pos) * qd + h * hd + i, 1.0);
+        cache[((static_cast<size_t>(b) * H + h) * cap + pos) * hd + i] = __float2bfloat16_rn(v);
+    }
+}
+
+cudaError_t launch_init_kv_random(__nv_bfloat16* cache, int B, int H, int hd, int cap, int P, int layer, int which,
+                                  int L, uint64_t seed, cudaStream_t st) {
+    size_t n = static_cast<size_t>(B) * H * P * hd;
+    if (n == 0) return cudaSuccess;
+    int blocks = static_cast<int>((n + 255) / 256 < 65536 ? (n + 255) / 256 : 65536);
+    k_init_kv<<<blocks, 256, 0, st>>>(cache, B, H, hd, cap, P, layer, which, L, seed);
+    return cudaGetLastError();
+}
+
+// RoPE table: rope[pos][i] = (cos, sin)(pos * base^(-2i/hd)), computed in double.
+__global__ void k_init_rope(float* rope, int cap, int hd, double base) {
+    const int half = hd / 2;
+    const int n = cap * half;
+    for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < n; e += gridDim.x * blockDim.x) {
+        int pos = e / half, i = e % half;
+        double theta = pow(base, -2.0 * i / hd);
+        double s, c;
+        sincos(static_cast<double>(pos) * theta, &s, &c);
+        rope[2 * e] = static_cast<float>(c);
+        rope[2 * e + 1] = static_cast<float>(s);
+    }
+}
+
+cudaError_t launch_init_rope(float* rope, int cap, int hd, double base, cudaStream_t st) {
+    int n = cap * hd / 2;
+    k_init_rope<<<(n + 255) / 256, 256, 0, st>>>(rope, cap, hd, base);
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ norms
+// Deterministic block sum (fixed shuffle tree, then warp 0 over warp sums).
+__device__ __forceinline__ float block_sum(float v, float* red) {
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    if (l == 0) red[w] = v;
+    __syncthreads();
+    if (w == 0) {
+        v = l < (blockDim.x >> 5) ? red[l] : 0.0f;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
+        if (l == 0) red[32] = v;
+    }
+    __syncthreads();
+    return red[32];
+}
+
+// One CTA per token: x (fp32 residual) = embedding row; xn = bf16(x / rms(x)).
+// The RMSNorm gain is one and is not stored.
+__global__ void __launch_bounds__(256) k_embed_norm(const int* tok, int tok_ld, const int* seq_kv,
+                                                    const __nv_bfloat16* emb, float* x, __nv_bfloat16* xn, int T,
+                                                    int d, float eps) {
+    __shared__ float red[33];
+    const int j = blockIdx.x;
+    const int b = j / T, t = j - b * T;
+    const int id = tok[static_cast<size_t>(b) * tok_ld + seq_kv[b] + t];
+    const __nv_bfloat16* e = emb + static_cast<size_t>(id) * d;
+    float* xr = x + static_cast<size_t>(j) * d;
+    float ss = 0.0f;
+    for (int i = threadIdx.x; i < d; i += blockDim.x) {
+        float v = __bfloat162float(e[i]);
+        xr[i] = v;
+        ss += v * v;
+    }
+    float r = rsqrtf(block_sum(ss, red) / d + eps);
+    for (int i = threadIdx.x; i < d; i += blockDim.x) xn[static_cast<size_t>(j) * d + i] = __float2bfloat16_rn(xr[i] * r);
+}
+
+cudaError_t launch_embed_norm(const int* tok, int tok_ld, const int* seq_kv, const __nv_bfloat16* emb, float* x,
+                              __nv_bfloat16* xn, int B, int T, int d, float eps, cudaStream_t st) {
+    k_embed_norm<<<B * T, 256, 0, st>>>(tok, tok_ld, seq_kv, emb, x, xn, T, d, eps);
+    return cudaGetLastError();
+}
+
+__global__ void __launch_bounds__(256) k_rmsnorm(const float* x, __nv_bfloat16* xn, int d, float eps) {
+    __shared__ float red[33];
+    const float* xr = x + static_cast<size_t>(blockIdx.x) * d;
+    float ss = 0.0f;
+    for (int i = threadIdx.x * 4; i < d; i += blockDim.x * 4) {
+        float4 v = *reinterpret_cast<const float4*>(xr + i);
+        ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+    }
+    float r = rsqrtf(block_sum(ss, red) / d + eps);
+    __nv_bfloat16* o = xn + static_cast<size_t>(blockIdx.x) * d;
+    for (int i = threadIdx.x * 4; i < d; i += blockDim.x * 4) {
+        float4 v = *reinterpret_cast<const float4*>(xr + i);
+        __nv_bfloat162 a = __floats2bfloat162_rn(v.x * r, v.y * r);
+        __nv_bfloat162 c = __floats2bfloat162_rn(v.z * r, v.w * r);
+        *reinterpret_cast<__nv_bfloat162*>(o + i) = a;
+        *reinterpret_cast<__nv_bfloat162*>(o + i + 2) = c;
+    }
+}
+
+cudaError_t launch_rmsnorm(const float* x, __nv_bfloat16* xn, int ntok, int d, float eps, cudaStream_t st) {
+    k_rmsnorm<<<ntok, 256, 0, st>>>(x, xn, d, eps);
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ attention
+// Bidirectional attention of T window queries per sequence over keys
+// [0, kv_len + T) of the KV cache (cached prefix, then the window's own keys
+// written by the QKV epilogue), flash style with split-KV: CTA (split, head,
+// sequence x 64-query tile) covers `chunk` keys in 64-key sub-blocks with an
+// online softmax on bf16 mma.sync tiles, writing unnormalised partials that
+// k_attn_combine merges (or the final output when there is one split).
+constexpr int kAQ = 64;
+constexpr int kAK = 64;
+
+__device__ __forceinline__ int swz(int r, int c, int hd) {
+    return r * hd + ((((c >> 3) ^ (r & 7))) << 3) + (c & 7);
+}
+
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, bool valid) {
+    unsigned s = smem_u32(dst);
+    int n = valid ? 16 : 0;
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(s), "l"(src), "r"(n) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+
+__device__ __forceinline__ void ldm_x4(uint32_t addr, uint32_t& a, uint32_t& b, uint32_t& c, uint32_t& d) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(a), "=r"(b), "=r"(c), "=r"(d)
+                 : "r"(addr));
+}
+__device__ __forceinline__ void ldm_x4_t(uint32_t addr, uint32_t& a, uint32_t& b, uint32_t& c, uint32_t& d) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(a), "=r"(b), "=r"(c), "=r"(d)
+                 : "r"(addr));
+}
+__device__ __forceinline__ void mma16816(float* d, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                                         uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&v);
+}
+
+template <int HD>
+__global__ void __launch_bounds__(128) k_attn(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ kc,
+                                              const __nv_bfloat16* __restrict__ vc, const int* __restrict__ seq_kv,
+                                              float* __restrict__ part_o, float* __restrict__ part_ml,
+                                              __nv_bfloat16* __restrict__ out, int T, int H, int cap, int chunk,
+                                              int nsplit, int qtiles) {
+    extern __shared__ __align__(128) uint8_t smem_attn[];
+    __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem_attn);
+    __nv_bfloat16* sK = sQ + kAQ * HD;       // [2][kAK][HD]
+    __nv_bfloat16* sV = sK + 2 * kAK * HD;   // [2][kAK][HD]
+
+    const int split = blockIdx.x, h = blockIdx.y;
+    const int b = blockIdx.z / qtiles, qt = blockIdx.z - b * qtiles;
+    const int NK = seq_kv[b] + T;
+    const int kbeg = split * chunk;
+    if (kbeg >= NK) return;
+    const int kend = min(NK, kbeg + chunk);
+    const int q0 = qt * kAQ;
+    const int nq = min(kAQ, T - q0);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int g = lane >> 2, c4 = lane & 3;
+    constexpr int CPR = HD / 8;  // 16-byte chunks per row
+
+    const __nv_bfloat16* qbase = q + ((static_cast<size_t>(b) * H + h) * T + q0) * HD;
+    const __nv_bfloat16* kbase = kc + (static_cast<size_t>(b) * H + h) * cap * HD;
+    const __nv_bfloat16* vbase = vc + (static_cast<size_t>(b) * H + h) * cap * HD;
+
+    for (int e = tid; e < kAQ * CPR; e += 128) {
+        int r = e / CPR, cc = (e % CPR) * 8;
+        cp_async16(sQ + swz(r, cc, HD), qbase + static_cast<size_t>(r < nq ? r : 0) * HD + cc, r < nq);
+    }
+    auto load_kv = [&](int buf, int k0) {
+        for (int e = tid; e < kAK * CPR; e += 128) {
+            int r = e / CPR, cc = (e % CPR) * 8;
+            int key = k0 + r;
+            bool ok = key < kend;
+            size_t off = static_cast<size_t>(ok ? key : kbeg) * HD + cc;
+            cp_async16(sK + buf * kAK * HD + swz(r, cc, HD), kbase + off, ok);
+            cp_async16(sV + buf * kAK * HD + swz(r, cc, HD), vbase + off, ok);
+        }
+    };
+    load_kv(0, kbeg);
+    cp_async_commit();
+
+    constexpr int KS = HD / 16;  // k-steps of Q.K
+    constexpr int DN = HD / 8;   // output n-blocks
+    uint32_t qa[KS][4];
+    float o[DN][4];
+#pragma unroll
+    for (int i = 0; i < DN; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.0f;
+    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.0f, l1 = 0.0f;
+    const float sl2 = rsqrtf(static_cast<float>(HD)) * 1.4426950408889634f;
+
+    int buf = 0;
+    bool qloaded = false;
+    for (int k0 = kbeg; k0 < kend; k0 += kAK) {
+        if (k0 + kAK < kend) {
+            load_kv(buf ^ 1, k0 + kAK);
+            cp_async_commit();
+            cp_async_wait_1();
+        } else {
+            cp_async_wait_all();
+        }
+        __syncthreads();
+        if (!qloaded) {
+#pragma unroll
+            for (int ks = 0; ks < KS; ++ks) {
+                int r = warp * 16 + (lane & 15), cc = ks * 16 + (lane >> 4) * 8;
+                ldm_x4(smem_u32(sQ + swz(r, cc, HD)), qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3]);
+            }
+            qloaded = true;
+        }
+        const __nv_bfloat16* K = sK + buf * kAK * HD;
+        const __nv_bfloat16* V = sV + buf * kAK * HD;
+        float s[8][4];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.0f;
+#pragma unroll
+        for (int jp = 0; jp < 4; ++jp) {
+#pragma unroll
+            for (int ks = 0; ks < KS; ++ks) {
+                int mi = lane >> 3, rr = lane & 7;
+                int key = jp * 16 + (mi >> 1) * 8 + rr, cc = ks * 16 + (mi & 1) * 8;
+                uint32_t b0, b1, b2, b3;
+                ldm_x4(smem_u32(K + swz(key, cc, HD)), b0, b1, b2, b3);
+                mma16816(s[2 * jp], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b0, b1);
+                mma16816(s[2 * jp + 1], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b2, b3);
+            }
+        }
+        // scale to log2 units, mask keys past the end, online softmax
+        float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            int key = k0 + j * 8 + 2 * c4;
+            bool v0 = key < kend, v1 = key + 1 < kend;
+            s[j][0] = v0 ? s[j][0] * sl2 : -INFINITY;
+            s[j][1] = v1 ? s[j][1] * sl2 : -INFINITY;
+            s[j][2] = v0 ? s[j][2] * sl2 : -INFINITY;
+            s[j][3] = v1 ? s[j][3] * sl2 : -INFINITY;
+            mx0 = fmaxf(mx0, fmaxf(s[j][0], s[j][1]));
+            mx1 = fmaxf(mx1, fmaxf(s[j][2], s[j][3]));
+        }
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+        const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+        const float ms0 = mn0 == -INFINITY ? 0.0f : mn0, ms1 = mn1 == -INFINITY ? 0.0f : mn1;
+        const float al0 = exp2f(m0 - ms0), al1 = exp2f(m1 - ms1);
+        m0 = mn0;
+        m1 = mn1;
+        l0 *= al0;
+        l1 *= al1;
+#pragma unroll
+        for (int i = 0; i < DN; ++i) {
+            o[i][0] *= al0;
+            o[i][1] *= al0;
+            o[i][2] *= al1;
+            o[i][3] *= al1;
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            s[j][0] = exp2f(s[j][0] - ms0);
+            s[j][1] = exp2f(s[j][1] - ms0);
+            s[j][2] = exp2f(s[j][2] - ms1);
+            s[j][3] = exp2f(s[j][3] - ms1);
+            l0 += s[j][0] + s[j][1];
+            l1 += s[j][2] + s[j][3];
+        }
+        // O += P V
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+            uint32_t a0 = pack_bf16(s[2 * kk][0], s[2 * kk][1]);
+            uint32_t a1 = pack_bf16(s[2 * kk][2], s[2 * kk][3]);
+            uint32_t a2 = pack_bf16(s[2 * kk + 1][0], s[2 * kk + 1][1]);
+            uint32_t a3 = pack_bf16(s[2 * kk + 1][2], s[2 * kk + 1][3]);
+#pragma unroll
+            for (int dn = 0; dn < DN; dn += 2) {
+                int mi = lane >> 3, rr = lane & 7;
+                int key = kk * 16 + (mi & 1) * 8 + rr, cc = (dn + (mi >> 1)) * 8;
+                uint32_t b0, b1, b2, b3;
+                ldm_x4_t(smem_u32(V + swz(key, cc, HD)), b0, b1, b2, b3);
+                mma16816(o[dn], a0, a1, a2, a3, b0, b1);
+                mma16816(o[dn + 1], a0, a1, a2, a3, b2, b3);
+            }
+        }
+        __syncthreads();
+        buf ^= 1;
+    }
+    l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+    l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+
+    const int r0 = warp * 16 + g, r1 = r0 + 8;
+    if (nsplit == 1) {
+        const int qd = H * HD;
+        const float i0 = 1.0f / l0, i1 = 1.0f / l1;
+#pragma unroll
+        for (int dn = 0; dn < DN; ++dn) {
+            int col = h * HD + dn * 8 + 2 * c4;
+            if (r0 < nq)
+                *reinterpret_cast<__nv_bfloat162*>(out + (static_cast<size_t>(b) * T + q0 + r0) * qd + col) =
+                    __floats2bfloat162_rn(o[dn][0] * i0, o[dn][1] * i0);
+            if (r1 < nq)
+                *reinterpret_cast<__nv_bfloat162*>(out + (static_cast<size_t>(b) * T + q0 + r1) * qd + col) =
+                    __floats2bfloat162_rn(o[dn][2] * i1, o[dn][3] * i1);
+        }
+    } else {
+        const size_t base = ((static_cast<size_t>(b) * H + h) * nsplit + split) * T + q0;
+#pragma unroll
+        for (int dn = 0; dn < DN; ++dn) {
+            int col = dn * 8 + 2 * c4;
+            if (r0 < nq) *reinterpret_cast<float2*>(part_o + (base + r0) * HD + col) = make_float2(o[dn][0], o[dn][1]);
+            if (r1 < nq) *reinterpret_cast<float2*>(part_o + (base + r1) * HD + col) = make_float2(o[dn][2], o[dn][3]);
+        }
+        if (c4 == 0) {
+            if (r0 < nq) *reinterpret_cast<float2*>(part_ml + (base + r0) * 2) = make_float2(m0, l0);
+            if (r1 < nq) *reinterpret_cast<float2*>(part_ml + (base + r1) * 2) = make_float2(m1, l1);
+        }
+    }
+}
+
+// One warp per (sequence, head, query): merge the splits in order.
+template <int HD>
+__global__ void __launch_bounds__(128) k_attn_combine(const float* __restrict__ part_o, const float* __restrict__ part_ml,
+                                                      const int* __restrict__ seq_kv, __nv_bfloat16* __restrict__ out,
+                                                      int B, int T, int H, int chunk, int nsplit_alloc) {
+    const int wid = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (wid >= B * H * T) return;
+    const int t = wid % T;
+    const int h = (wid / T) % H;
+    const int b = wid / (T * H);
+    const int NK = seq_kv[b] + T;
+    const int ns = (NK + chunk - 1) / chunk;
+    const size_t base = (static_cast<size_t>(b) * H + h) * nsplit_alloc * T + t;
+    float M = -INFINITY;
+    for (int s = 0; s < ns; ++s) M = fmaxf(M, part_ml[(base + static_cast<size_t>(s) * T) * 2]);
+    constexpr int PER = HD / 32;
+    float acc[PER];
+#pragma unroll
+    for (int i = 0; i < PER; ++i) acc[i] = 0.0f;
+    float L = 0.0f;
+    for (int s = 0; s < ns; ++s) {
+        size_t row = base + static_cast<size_t>(s) * T;
+        float w = exp2f(part_ml[row * 2] - M);
+        L += w * part_ml[row * 2 + 1];
+#pragma unroll
+        for (int i = 0; i < PER; ++i) acc[i] += w * part_o[row * HD + lane + 32 * i];
+    }
+    const float inv = 1.0f / L;
+    const int qd = H * HD;
+#pragma unroll
+    for (int i = 0; i < PER; ++i)
+        out[(static_cast<size_t>(b) * T + t) * qd + h * HD + lane + 32 * i] = __float2bfloat16_rn(acc[i] * inv);
+}
+
+cudaError_t attn_init_attrs() {
+    return cudaFuncSetAttribute(reinterpret_cast<const void*>(k_attn<128>),
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, 100 * 1024);
+}
+
+AttnPlan attn_plan(int B, int T, int H, int max_keys, int sms) {
+    AttnPlan a;
+    a.qtiles = (T + kAQ - 1) / kAQ;
+    int want = (2 * sms + B * H * a.qtiles - 1) / (B * H * a.qtiles);
+    const int blocks64 = (max_keys + kAK - 1) / kAK;
+    if (want > blocks64) want = blocks64;
+    if (want < 1) want = 1;
+    a.chunk = ((blocks64 + want - 1) / want) * kAK;
+    a.nsplit = (max_keys + a.chunk - 1) / a.chunk;
+    return a;
+}
+
+cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
+                             const int* seq_kv, float* part_o, float* part_ml, __nv_bfloat16* out, int B, int T, int H,
+                             int hd, int cap, const AttnPlan& a, cudaStream_t st) {
+    dim3 grid(a.nsplit, H, B * a.qtiles);
+    size_t smem = static_cast<size_t>(kAQ + 4 * kAK) * hd * 2;
+    const int cgrid = (B * H * T * 32 + 127) / 128;
+    if (hd == 128) {
+        k_attn<128><<<grid, 128, smem, st>>>(q, kc, vc, seq_kv, part_o, part_ml, out, T, H, cap, a.chunk, a.nsplit,
+                                              a.qtiles);
+        if (a.nsplit > 1)
+            k_attn_combine<128><<<cgrid, 128, 0, st>>>(part_o, part_ml, seq_kv, out, B, T, H, a.chunk, a.nsplit);
+    } else if (hd == 64) {
+        k_attn<64><<<grid, 128, smem, st>>>(q, kc, vc, seq_kv, part_o, part_ml, out, T, H, cap, a.chunk, a.nsplit,
+                                             a.qtiles);
+        if (a.nsplit > 1)
+            k_attn_combine<64><<<cgrid, 128, 0, st>>>(part_o, part_ml, seq_kv, out, B, T, H, a.chunk, a.nsplit);
+    } else {
+        return cudaErrorInvalidValue;
+    }
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ LM head
+// Merge the per-tile (max, sum exp, argmax) of each token over the vocab
+// tiles in a fixed tree: argmax excludes the mask id, ties go to the lowest
+// id; conf = 1 / sum; tokconf = exp(z_cur - max) / sum.
+__device__ __forceinline__ void lse_merge(float& m, float& s, int& i, float m2, float s2, int i2) {
+    if (m2 == -INFINITY) return;
+    if (m == -INFINITY) {
+        m = m2; s = s2; i = i2;
+        return;
+    }
+    if (m2 > m) {
+        s = s * expf(m - m2) + s2;
+        m = m2;
+        i = i2;
+    } else if (m2 == m) {
+        s += s2;
+        i = min(i, i2);
+    } else {
+        s += s2 * expf(m2 - m);
+    }
+}
+
+__global__ void k_lmhead_reduce(const float* __restrict__ part, const float* __restrict__ zcur,
+                                const int* __restrict__ cur_tok, int m_tiles, int N, int mask_id, int* x0, float* conf,
+                                float* tokconf) {
+    const int col = blockIdx.x;
+    const int lane = threadIdx.x;
+    float m = -INFINITY, s = 0.0f;
+    int idx = INT_MAX;
+    for (int t = lane; t < m_tiles; t += 32) {
+        const float* p = part + (static_cast<size_t>(t) * N + col) * 3;
+        lse_merge(m, s, idx, p[0], p[1], __float_as_int(p[2]));
+    }
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        float m2 = __shfl_down_sync(0xffffffffu, m, off);
+        float s2 = __shfl_down_sync(0xffffffffu, s, off);
+        int i2 = __shfl_down_sync(0xffffffffu, idx, off);
+        if ((lane & (2 * off - 1)) == 0 && lane + off < 32) lse_merge(m, s, idx, m2, s2, i2);
+    }
+    if (lane == 0) {
+        x0[col] = idx;
+        conf[col] = 1.0f / s;
+        int cur = cur_tok[col];
+        tokconf[col] = (cur >= 0 && cur != mask_id) ? expf(zcur[col] - m) / s : 0.0f;
+    }
+}
+
+cudaError_t launch_lmhead_reduce(const float* lm_part, const float* zcur, const int* cur_tok, int m_tiles, int N,
+                                 int mask_id, int* x0, float* conf, float* tokconf, cudaStream_t st) {
+    k_lmhead_reduce<<<N, 32, 0, st>>>(lm_part, zcur, cur_tok, m_tiles, N, mask_id, x0, conf, tokconf);
+    return cudaGetLastError();
+}
+
+__global__ void k_gather_cur(const int* tok, int tok_ld, const int* seq_kv, int* cur, int B, int T) {
+    int j = blockIdx.x * blockDim.x + threadIdx.x;
+    if (j >= B * T) return;
+    int b = j / T, t = j - b * T;
+    cur[j] = tok[static_cast<size_t>(b) * tok_ld + seq_kv[b] + t];
+}
+
+cudaError_t launch_gather_cur(const int* tok, int tok_ld, const int* seq_kv, int* cur, int B, int T,
+                              cudaStream_t st) {
+    k_gather_cur<<<(B * T + 127) / 128, 128, 0, st>>>(tok, tok_ld, seq_kv, cur, B, T);
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ commit pass
+// One CTA per sequence.  Order (all on this step's decisions):
+//  1. revision (theta_remask > 0, not the last step): COMMITTED tokens of the
+//     current block with tokconf >= theta_stable become STABLE; of those below
+//     theta_remask, the remask_max lowest (ties: lower position) are re-masked;
+//  2. k = ceil(m / (S - step)) for the m masked positions of the block;
+//  3. the k masked positions with the highest conf (ties: lower position)
+//     take their argmax and become COMMITTED;
+//  4. with the prefix cache and lookahead on, each future block inside the
+//     window drafts its single most confident masked position.
+__global__ void __launch_bounds__(256) k_commit(CommitArgs a) {
+    const int b = blockIdx.x;
+    int* tok = a.tok + static_cast<size_t>(b) * a.ld;
+    uint8_t* st = a.st + static_cast<size_t>(b) * a.ld;
+    int* plan = a.plan + b * 4;
+    const int c0 = plan[0], c1 = plan[1], step = plan[2];
+    const int n = c1 - c0;  // <= kMaxBlock (checked by the host)
+    const int w0 = a.use_cache ? a.seq_kv[b] : 0;
+    const int* x0 = a.x0 + static_cast<size_t>(b) * a.T;
+    const float* conf = a.conf + static_cast<size_t>(b) * a.T;
+    const float* tc = a.tokconf + static_cast<size_t>(b) * a.T;
+    __shared__ int s_cnt[8];
+    __shared__ uint8_t s_sel[kMaxBlock];
+    if (threadIdx.x < 8) s_cnt[threadIdx.x] = 0;
+    __syncthreads();
+    if (a.theta_remask > 0.0f && step < a.S - 1) {
+        for (int i = threadIdx.x; i < n; i += blockDim.x) {
+            const int p = c0 + i;
+            if (st[p] == 2 && tc[p - w0] >= a.theta_stable) {
+                st[p] = 3;
+                atomicAdd(&s_cnt[2], 1);
+            }
+        }
+        __syncthreads();
+        // candidates ranked by (tokconf ascending, position ascending)
+        for (int i = threadIdx.x; i < n; i += blockDim.x) {
+            const int p = c0 + i;
+            uint8_t sel = 0;
+            if (st[p] == 2 && tc[p - w0] < a.theta_remask) {
+                const float vp = tc[p - w0];
+                int rank = 0;
+                for (int qq = c0; qq < c1; ++qq) {
+                    if (qq == p || st[qq] != 2) continue;
+                    const float vq = tc[qq - w0];
+                    if (!(vq < a.theta_remask)) continue;
+                    if (vq < vp || (vq == vp && qq < p)) ++rank;
+                }
+                sel = rank < a.remask_max;
+            }
+            s_sel[i] = sel;
+        }
+        __syncthreads();
+        for (int i = threadIdx.x; i < n; i += blockDim.x) {
+            if (s_sel[i]) {
+                st[c0 + i] = 1;
+                tok[c0 + i] = a.mask_id;
+                atomicAdd(&s_cnt[1], 1);
+            }
+        }
+        __syncthreads();
+    }
+    int mloc = 0;
+    for (int i = threadIdx.x; i < n; i += blockDim.x) mloc += st[c0 + i] == 1;
+    atomicAdd(&s_cnt[5], mloc);
+    __syncthreads();
+    const int m = s_cnt[5];
+    const int left = a.S - step;
+    const int k = m == 0 ? 0 : (left <= 1 ? m : (m + left - 1) / left);
+    // commit: the k masked positions ranked by (conf descending, position ascending)
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+        const int p = c0 + i;
+        uint8_t sel = 0;
+        if (st[p] == 1) {
+            const float vp = conf[p - w0];
+            int rank = 0;
+            for (int qq = c0; qq < c1; ++qq) {
+                if (qq == p || st[qq] != 1) continue;
+                const float vq = conf[qq - w0];
+                if (vq > vp || (vq == vp && qq < p)) ++rank;
+            }
+            sel = rank < k;
+        }
+        s_sel[i] = sel;
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+        if (s_sel[i]) {
+            const int p = c0 + i;
+            tok[p] = x0[p - w0];
+            st[p] = 2;
+            atomicAdd(&s_cnt[0], 1);
+        }
+    }
+    __syncthreads();
+    // drafts for the future blocks inside the window
+    if (a.use_cache && a.spec_blocks > 0 && threadIdx.x < 32) {
+        const int w1 = w0 + a.T;
+        for (int d0 = c1; d0 < w1; d0 += a.block_len) {
+            const int d1 = min(d0 + a.block_len, w1);
+            float bv = -INFINITY;
+            int bp = INT_MAX;
+            for (int p = d0 + static_cast<int>(threadIdx.x); p < d1; p += 32) {
+                if (st[p] != 1) continue;
+                const float v = conf[p - w0];
+                if (v > bv || (v == bv && p < bp)) {
+                    bv = v;
+                    bp = p;
+                }
+            }
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) {
+                const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+                const int op = __shfl_xor_sync(0xffffffffu, bp, off);
+                if (ov > bv || (ov == bv && op < bp)) {
+                    bv = ov;
+                    bp = op;
+                }
+            }
+            if (threadIdx.x == 0 && bp != INT_MAX) {
+                tok[bp] = x0[bp - w0];
+                st[bp] = 4;
+                s_cnt[3] += 1;
+            }
+            __syncwarp();
+        }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int* o = a.outs + b * 8;
+        o[0] = s_cnt[0];
+        o[1] = s_cnt[1];
+        o[2] = s_cnt[2];
+        o[3] = s_cnt[3];
+        o[5] = m - s_cnt[0];
+        o[4] = o[5] == 0;
+        plan[2] = step + 1;
+    }
+}
+
+cudaError_t launch_commit(const CommitArgs& a, cudaStream_t st) {
+    k_commit<<<a.B, 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace dllm
+
+namespace dllm {
+
+// Start a block on every sequence: plan = {c0, c1, step 0}; drafts inside the
+// block become COMMITTED; snapshot the window region for rewinds.
+__global__ void k_begin_block(int* tok, uint8_t* st, int* snap_tok, uint8_t* snap_st, int ld, int n_pos, int* plan,
+                              int c0, int c1) {
+    const int b = blockIdx.x;
+    int* t = tok + static_cast<size_t>(b) * ld;
+    uint8_t* s = st + static_cast<size_t>(b) * ld;
+    for (int p = c0 + threadIdx.x; p < c1; p += blockDim.x)
+        if (s[p] == 4) s[p] = 2;
+    __syncthreads();
+    for (int p = threadIdx.x; p < n_pos; p += blockDim.x) {
+        snap_tok[static_cast<size_t>(b) * ld + p] = t[p];
+        snap_st[static_cast<size_t>(b) * ld + p] = s[p];
+    }
+    if (threadIdx.x == 0) {
+        plan[b * 4 + 0] = c0;
+        plan[b * 4 + 1] = c1;
+        plan[b * 4 + 2] = 0;
+    }
+}
+
+cudaError_t launch_begin_block(int* tok, uint8_t* st, int* snap_tok, uint8_t* snap_st, int ld, int n_pos, int* plan,
+                               int B, int c0, int c1, cudaStream_t stream) {
+    k_begin_block<<<B, 256, 0, stream>>>(tok, st, snap_tok, snap_st, ld, n_pos, plan, c0, c1);
+    return cudaGetLastError();
+}
+
+__global__ void k_rewind(int* tok, uint8_t* st, const int* snap_tok, const uint8_t* snap_st, int ld, int n_pos,
+                         int* plan) {
+    const int b = blockIdx.x;
+    for (int p = threadIdx.x; p < n_pos; p += blockDim.x) {
+        tok[static_cast<size_t>(b) * ld + p] = snap_tok[static_cast<size_t>(b) * ld + p];
+        st[static_cast<size_t>(b) * ld + p] = snap_st[static_cast<size_t>(b) * ld + p];
+    }
+    if (threadIdx.x == 0) plan[b * 4 + 2] = 0;
+}
+
+cudaError_t launch_rewind(int* tok, uint8_t* st, const int* snap_tok, const uint8_t* snap_st, int ld, int n_pos,
+                          int* plan, int B, cudaStream_t stream) {
+    k_rewind<<<B, 256, 0, stream>>>(tok, st, snap_tok, snap_st, ld, n_pos, plan);
+    return cudaGetLastError();
+}
+
+__global__ void k_set_kv_len(int* seq_kv, int B, int v) {
+    int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b < B) seq_kv[b] = v;
+}
+
+cudaError_t launch_set_kv_len(int* seq_kv, int B, int v, cudaStream_t stream) {
+    k_set_kv_len<<<(B + 127) / 128, 128, 0, stream>>>(seq_kv, B, v);
+    return cudaGetLastError();
+}
+
+}  // namespace dllm

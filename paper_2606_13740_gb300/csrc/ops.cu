@@ -1,0 +1,202 @@
+// Single-kernel entry points (include/dllm_ops.h) for kernel-level tests.
+#include "../../include/dllm.h"
+#include "../../include/dllm_ops.h"
+#include "internal.h"
+
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+using namespace dllm;
+
+extern "C" const char* dllm_last_error(const dllm_ctx* ctx);
+void dllm_set_noctx_error(const char* msg);
+
+namespace {
+
+int op_fail(int code, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    dllm_set_noctx_error(buf);
+    return code;
+}
+
+int sm_count() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    return n;
+}
+
+// Device scratch owned by one op call.
+struct DevBuf {
+    void* p = nullptr;
+    ~DevBuf() {
+        if (p) cudaFree(p);
+    }
+    bool alloc(size_t bytes) { return cudaMalloc(&p, bytes ? bytes : 16) == cudaSuccess; }
+};
+
+int finish(cudaStream_t st, int* status_dev) {
+    cudaError_t e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return op_fail(DLLM_ECUDA, "%s", cudaGetErrorString(e));
+    int s = 0;
+    if (status_dev) {
+        e = cudaMemcpy(&s, status_dev, 4, cudaMemcpyDeviceToHost);
+        if (e != cudaSuccess) return op_fail(DLLM_ECUDA, "%s", cudaGetErrorString(e));
+    }
+    if (s & kStatusTimeout) return op_fail(DLLM_ETIMEOUT, "bounded device wait ran out");
+    if (s) return op_fail(DLLM_ECUDA, "device status %d", s);
+    return DLLM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int dllm_op_gemm(const void* W, const void* X, float* D, int M, int N, int K, int grid, void* stream) {
+    if (!W || !X || !D || M < 1 || N < 1 || K < 1 || (K * 2) % 16) return op_fail(DLLM_EINVAL, "bad gemm arguments");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    int sms = sm_count();
+    if (sms <= 0) return op_fail(DLLM_ECUDA, "no CUDA device");
+    if (gemm_init_attrs() != cudaSuccess) return op_fail(DLLM_ECUDA, "attribute setup failed");
+    GemmPlan p = gemm_plan(M, N, K, grid > 0 ? grid : sms);
+    CUtensorMap tw, tx;
+    if (!make_tmap_bf16(&tw, W, M, K, 128) || !make_tmap_bf16(&tx, X, N, K, p.ntile))
+        return op_fail(DLLM_EINVAL, "tensor map encode failed (alignment?)");
+    DevBuf part, cnt, status;
+    const size_t pf = static_cast<size_t>(p.grid) * 2 * p.ntile * 128;
+    const int cl = p.m_tiles * p.n_tiles;
+    if (!part.alloc(pf * 4) || !cnt.alloc(static_cast<size_t>(cl) * 4) || !status.alloc(16))
+        return op_fail(DLLM_ENOMEM, "scratch allocation failed");
+    if (cudaMemsetAsync(cnt.p, 0, static_cast<size_t>(cl) * 4, st) != cudaSuccess ||
+        cudaMemsetAsync(status.p, 0, 16, st) != cudaSuccess)
+        return op_fail(DLLM_ECUDA, "memset failed");
+    Scratch scr{static_cast<float*>(part.p), static_cast<int*>(cnt.p), pf, cl};
+    EpiArgs ep{};
+    ep.out = D;
+    ep.ld_out = M;
+    cudaError_t e = gemm_launch(EPI_F32, p, tw, tx, ep, scr, static_cast<int*>(status.p), st);
+    if (e != cudaSuccess) return op_fail(DLLM_ECUDA, "gemm launch: %s", cudaGetErrorString(e));
+    return finish(st, static_cast<int*>(status.p));
+}
+
+int dllm_op_attention(const void* q, const void* kc, const void* vc, const int32_t* kv_len, void* out, int B, int T,
+                      int H, int hd, int cap, int max_kv_len, void* stream) {
+    if (!q || !kc || !vc || !kv_len || !out || B < 1 || T < 1 || H < 1 || (hd != 64 && hd != 128) ||
+        max_kv_len < 0 || max_kv_len + T > cap)
+        return op_fail(DLLM_EINVAL, "bad attention arguments");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    int sms = sm_count();
+    if (sms <= 0) return op_fail(DLLM_ECUDA, "no CUDA device");
+    if (attn_init_attrs() != cudaSuccess) return op_fail(DLLM_ECUDA, "attribute setup failed");
+    AttnPlan a = attn_plan(B, T, H, max_kv_len + T, sms);
+    DevBuf po, pml;
+    const size_t rows = static_cast<size_t>(B) * H * a.nsplit * T;
+    if (!po.alloc(rows * hd * 4) || !pml.alloc(rows * 2 * 4)) return op_fail(DLLM_ENOMEM, "scratch allocation failed");
+    cudaError_t e = launch_attention(static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(kc),
+                                     static_cast<const __nv_bfloat16*>(vc), kv_len, static_cast<float*>(po.p),
+                                     static_cast<float*>(pml.p), static_cast<__nv_bfloat16*>(out), B, T, H, hd, cap, a,
+                                     st);
+    if (e != cudaSuccess) return op_fail(DLLM_ECUDA, "attention launch: %s", cudaGetErrorString(e));
+    return finish(st, nullptr);
+}
+
+int dllm_op_lmhead(const void* W, const void* X, const int32_t* cur, int32_t* x0, float* conf, float* tokconf,
+                   float* logits, int V, int N, int d, int mask_id, void* stream) {
+    if (!W || !X || !cur || !x0 || !conf || !tokconf || V < 2 || N < 1 || d < 8 || (d * 2) % 16 || mask_id < 0 ||
+        mask_id >= V)
+        return op_fail(DLLM_EINVAL, "bad lmhead arguments");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    int sms = sm_count();
+    if (sms <= 0) return op_fail(DLLM_ECUDA, "no CUDA device");
+    if (gemm_init_attrs() != cudaSuccess) return op_fail(DLLM_ECUDA, "attribute setup failed");
+    GemmPlan p = gemm_plan(V, N, d, sms);
+    CUtensorMap tw, tx;
+    if (!make_tmap_bf16(&tw, W, V, d, 128) || !make_tmap_bf16(&tx, X, N, d, p.ntile))
+        return op_fail(DLLM_EINVAL, "tensor map encode failed (alignment?)");
+    DevBuf part, cnt, status, lmp, zc;
+    const size_t pf = static_cast<size_t>(p.grid) * 2 * p.ntile * 128;
+    const int cl = p.m_tiles * p.n_tiles;
+    if (!part.alloc(pf * 4) || !cnt.alloc(static_cast<size_t>(cl) * 4) || !status.alloc(16) ||
+        !lmp.alloc(static_cast<size_t>(p.m_tiles) * N * 3 * 4) || !zc.alloc(static_cast<size_t>(N) * 4))
+        return op_fail(DLLM_ENOMEM, "scratch allocation failed");
+    if (cudaMemsetAsync(cnt.p, 0, static_cast<size_t>(cl) * 4, st) != cudaSuccess ||
+        cudaMemsetAsync(status.p, 0, 16, st) != cudaSuccess || cudaMemsetAsync(zc.p, 0, static_cast<size_t>(N) * 4, st))
+        return op_fail(DLLM_ECUDA, "memset failed");
+    Scratch scr{static_cast<float*>(part.p), static_cast<int*>(cnt.p), pf, cl};
+    EpiArgs ep{};
+    ep.lm_part = static_cast<float*>(lmp.p);
+    ep.zcur = static_cast<float*>(zc.p);
+    ep.cur_tok = cur;
+    ep.logits = logits;
+    ep.V = V;
+    ep.mask_id = mask_id;
+    cudaError_t e = gemm_launch(EPI_LMHEAD, p, tw, tx, ep, scr, static_cast<int*>(status.p), st);
+    if (e == cudaSuccess)
+        e = launch_lmhead_reduce(static_cast<float*>(lmp.p), static_cast<float*>(zc.p), cur, p.m_tiles, N, mask_id, x0,
+                                 conf, tokconf, st);
+    if (e != cudaSuccess) return op_fail(DLLM_ECUDA, "lmhead launch: %s", cudaGetErrorString(e));
+    return finish(st, static_cast<int*>(status.p));
+}
+
+int dllm_op_commit(int32_t* tok, uint8_t* status, int n_pos, int w0, int T, int c0, int c1, int step,
+                   const int32_t* x0, const float* conf, const float* tokconf, int steps_per_block,
+                   float theta_remask, float theta_stable, int remask_max, int spec_blocks, int use_prefix_cache,
+                   int block_len, int mask_id, int* out6) {
+    if (!tok || !status || !x0 || !conf || !tokconf || n_pos < 1 || T < 1 || w0 < 0 || w0 + T > n_pos || c0 < w0 ||
+        c1 > w0 + T || c0 > c1 || c1 - c0 > kMaxBlock || steps_per_block < 1 || block_len < 1)
+        return op_fail(DLLM_EINVAL, "bad commit arguments");
+    if (!use_prefix_cache && w0 != 0) return op_fail(DLLM_EINVAL, "without the prefix cache the window starts at 0");
+    DevBuf dtok, dst, dx0, dconf, dtc, dkv, dplan, douts;
+    if (!dtok.alloc(static_cast<size_t>(n_pos) * 4) || !dst.alloc(n_pos) || !dx0.alloc(static_cast<size_t>(T) * 4) ||
+        !dconf.alloc(static_cast<size_t>(T) * 4) || !dtc.alloc(static_cast<size_t>(T) * 4) || !dkv.alloc(4) ||
+        !dplan.alloc(16) || !douts.alloc(32))
+        return op_fail(DLLM_ENOMEM, "allocation failed");
+    int plan[4] = {c0, c1, step, 0};
+    bool ok = cudaMemcpy(dtok.p, tok, static_cast<size_t>(n_pos) * 4, cudaMemcpyHostToDevice) == cudaSuccess &&
+              cudaMemcpy(dst.p, status, n_pos, cudaMemcpyHostToDevice) == cudaSuccess &&
+              cudaMemcpy(dx0.p, x0, static_cast<size_t>(T) * 4, cudaMemcpyHostToDevice) == cudaSuccess &&
+              cudaMemcpy(dconf.p, conf, static_cast<size_t>(T) * 4, cudaMemcpyHostToDevice) == cudaSuccess &&
+              cudaMemcpy(dtc.p, tokconf, static_cast<size_t>(T) * 4, cudaMemcpyHostToDevice) == cudaSuccess &&
+              cudaMemcpy(dkv.p, &w0, 4, cudaMemcpyHostToDevice) == cudaSuccess &&
+              cudaMemcpy(dplan.p, plan, 16, cudaMemcpyHostToDevice) == cudaSuccess;
+    if (!ok) return op_fail(DLLM_ECUDA, "copy in failed");
+    CommitArgs a{};
+    a.tok = static_cast<int*>(dtok.p);
+    a.st = static_cast<uint8_t*>(dst.p);
+    a.ld = n_pos;
+    a.seq_kv = static_cast<int*>(dkv.p);
+    a.plan = static_cast<int*>(dplan.p);
+    a.x0 = static_cast<int*>(dx0.p);
+    a.conf = static_cast<float*>(dconf.p);
+    a.tokconf = static_cast<float*>(dtc.p);
+    a.outs = static_cast<int*>(douts.p);
+    a.B = 1;
+    a.T = T;
+    a.mask_id = mask_id;
+    a.use_cache = use_prefix_cache;
+    a.S = steps_per_block;
+    a.remask_max = remask_max;
+    a.spec_blocks = spec_blocks;
+    a.block_len = block_len;
+    a.theta_remask = theta_remask;
+    a.theta_stable = theta_stable;
+    cudaError_t e = launch_commit(a, nullptr);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return op_fail(DLLM_ECUDA, "commit: %s", cudaGetErrorString(e));
+    int outs[8];
+    ok = cudaMemcpy(tok, dtok.p, static_cast<size_t>(n_pos) * 4, cudaMemcpyDeviceToHost) == cudaSuccess &&
+         cudaMemcpy(status, dst.p, n_pos, cudaMemcpyDeviceToHost) == cudaSuccess &&
+         cudaMemcpy(outs, douts.p, 32, cudaMemcpyDeviceToHost) == cudaSuccess;
+    if (!ok) return op_fail(DLLM_ECUDA, "copy out failed");
+    if (out6) memcpy(out6, outs, 6 * sizeof(int));
+    return DLLM_OK;
+}
+
+}  // extern "C"

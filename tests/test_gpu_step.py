@@ -1,0 +1,195 @@
+"""End-to-end parity of the GPU denoising path with the oracle on the tiny
+LLaDA-shaped config, through the C ABI: seeded weights bit-exact, and every
+step teacher-forced on the oracle's state so the trajectories stay aligned.
+
+Acceptance per step: logits relative L2 <= 1e-2 (bf16 path vs fp32 oracle);
+argmax ids equal wherever the oracle's top-1/top-2 logit margin exceeds 0.05;
+window, commit counts and token states bit-exact; committed positions equal
+wherever the oracle's confidence ranking is unambiguous.
+"""
+import numpy as np
+import pytest
+
+import dllm_inputs as I
+import oracle as O
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+TINY = O.OracleConfig()
+
+
+@pytest.fixture(scope="module")
+def model():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    import paper_2606_13740_gb300 as pkg
+    pkg.lib()
+    return O.Model(TINY)
+
+
+def _gpu_ctx(max_ctx=256, max_window=160, max_batch=1):
+    from paper_2606_13740_gb300 import Config, Context
+    return Context(Config(max_ctx=max_ctx, max_window=max_window, max_batch=max_batch))
+
+
+def test_weights_bit_exact(model):
+    ctx = _gpu_ctx()
+    for which, tid in ((1, O.T_EMBED), (2, O.T_HEAD)):
+        assert np.array_equal(ctx.dllm_get_weight(-1, which), model.weight(-1, tid))
+    for layer in range(TINY.n_layers):
+        for w in range(7):
+            assert np.array_equal(ctx.dllm_get_weight(layer, w), model.weight(layer, w)), (layer, w)
+    ctx.close()
+
+
+def _unambiguous_commits(od, o_tok_before, o_st_before, c0, c1, w0, k):
+    masked = [p for p in range(c0, c1) if o_st_before[p] == O.MASKED]
+    if k == 0 or k >= len(masked):
+        return True
+    c = sorted((float(od["conf"][p - w0]) for p in masked), reverse=True)
+    return (c[k - 1] - c[k]) > 0.02 * c[k - 1]
+
+
+def _run_teacher_forced(model, osched, gsched, prompt, gen_len, ctx):
+    sess = O.Session(model, osched, prompt, gen_len)
+    sess.prefill()
+    ctx.dllm_prefill(gsched, prompt, gen_len)
+    ctx.dllm_set_debug(1)
+    steps = 0
+    worst = 0.0
+    while True:
+        o_more = sess.begin_block()
+        g_more = ctx.dllm_begin_block()
+        assert o_more == g_more
+        if not o_more:
+            break
+        while True:
+            o_tok0, o_st0, _ = sess.state()
+            g_tok0, g_st0, _ = ctx.dllm_get_state()
+            assert np.array_equal(g_tok0[0], o_tok0) and np.array_equal(g_st0[0], o_st0)
+            oo = sess.step(keep_logits=True)
+            go = ctx.dllm_denoise_step()
+            ow, gw = sess.window(), ctx.dllm_window()
+            for key in ("w0", "T", "c0", "c1", "kv_len", "spec_on", "step"):
+                assert ow[key] == gw[key], (key, ow, gw)
+            od = sess.decisions(logits=True)
+            gd = ctx.dllm_get_step_debug(logits=True)
+            lg, ref = gd["logits"][0], od["logits"]
+            rel = float(np.linalg.norm(lg - ref) / np.linalg.norm(ref))
+            worst = max(worst, rel)
+            assert rel <= 1e-2, rel
+            safe = od["margin"] > 0.05
+            assert np.array_equal(gd["x0"][0][safe], od["x0"][safe])
+            assert not (gd["x0"][0] == TINY.mask_id).any()
+            assert np.allclose(gd["conf"][0], od["conf"], rtol=0.05)
+            for key in ("n_committed", "n_drafts", "block_done", "masked_after"):
+                assert go[key] == oo[key], (key, go, oo)
+            g_tok, g_st, _ = ctx.dllm_get_state()
+            o_tok, o_st, _ = sess.state()
+            if _unambiguous_commits(od, o_tok0, o_st0, ow["c0"], ow["c1"], ow["w0"], oo["n_committed"]):
+                newly_o = (o_st == O.COMMITTED) & (o_st0 == O.MASKED)
+                newly_g = (g_st[0] == O.COMMITTED) & (g_st0[0] == O.MASKED)
+                assert np.array_equal(newly_o, newly_g)
+            ctx.dllm_set_state(o_tok[None], o_st[None])  # teacher forcing
+            steps += 1
+            if oo["block_done"]:
+                break
+    o_tok, o_st, o_kv = sess.state()
+    g_tok, g_st, g_kv = ctx.dllm_get_state()
+    assert g_kv[0] == o_kv
+    assert np.array_equal(g_tok[0], o_tok) and np.array_equal(g_st[0], o_st)
+    return sess, steps, worst
+
+
+def test_blockwise_prefix_cache_teacher_forced(model):
+    """Tiny config: 64-token prompt, 2 blocks of 32, 8 steps/block (4 commits/step)."""
+    from paper_2606_13740_gb300 import Sched
+    prompt = I.uniform_prompt(64, TINY.vocab, TINY.mask_id)
+    ctx = _gpu_ctx()
+    sess, steps, worst = _run_teacher_forced(model, O.OracleSched(steps_per_block=8), Sched(steps_per_block=8),
+                                             prompt, 64, ctx)
+    assert steps == 16
+    kv_len = sess.state()[2]
+    for layer in range(TINY.n_layers):
+        for which in (0, 1):
+            ref = sess.prefix_kv(layer, which)
+            got = ctx.dllm_get_kv(layer, which, 0, 0, kv_len)
+            assert np.linalg.norm(got - ref) / np.linalg.norm(ref) <= 1e-2
+    ctx.close()
+
+
+def test_vanilla_full_sequence_teacher_forced(model):
+    from paper_2606_13740_gb300 import Sched
+    prompt = I.uniform_prompt(16, TINY.vocab, TINY.mask_id, seed=11)
+    ctx = _gpu_ctx()
+    _, steps, _ = _run_teacher_forced(model, O.OracleSched(steps_per_block=8, use_prefix_cache=0),
+                                      Sched(steps_per_block=8, use_prefix_cache=0), prompt, 32, ctx)
+    assert steps == 8
+    ctx.close()
+
+
+def test_speculative_revision_teacher_forced(model):
+    """Lookahead of 2 blocks at <= 8 masked, re-mask below 0.5 (config-4 rules)."""
+    from paper_2606_13740_gb300 import Sched
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=22)
+    osched = O.OracleSched(steps_per_block=16, spec_blocks=2, spec_trigger=8, theta_remask=0.5, remask_max=1)
+    gsched = Sched(steps_per_block=16, spec_blocks=2, spec_trigger=8, theta_remask=0.5, remask_max=1)
+    ctx = _gpu_ctx()
+    _, steps, _ = _run_teacher_forced(model, osched, gsched, prompt, 128, ctx)
+    assert steps >= 4 * 1
+    ctx.close()
+
+
+def test_generate_matches_stepwise_and_is_deterministic(model):
+    from paper_2606_13740_gb300 import Sched
+    prompt = I.uniform_prompt(64, TINY.vocab, TINY.mask_id)
+    ctx = _gpu_ctx()
+    a, stats = ctx.dllm_generate(Sched(steps_per_block=8), prompt, 64)
+    b, _ = ctx.dllm_generate(Sched(steps_per_block=8), prompt, 64)
+    assert np.array_equal(a, b)
+    assert stats == {"steps": 16, "spec_steps": 0, "blocks": 2}
+    assert not (a == TINY.mask_id).any()
+    ctx.close()
+
+
+def test_batch_sequences_are_independent(model):
+    from paper_2606_13740_gb300 import Sched
+    prompts = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, batch=3, seed=5)
+    ctx = _gpu_ctx(max_batch=3, max_window=64)
+    batched, _ = ctx.dllm_generate(Sched(steps_per_block=8), prompts, 64)
+    for b in range(3):
+        single, _ = ctx.dllm_generate(Sched(steps_per_block=8), prompts[b:b + 1], 64)
+        assert np.array_equal(single[0], batched[b])
+    ctx.close()
+
+
+def test_rewind_repeats_identical_step(model):
+    from paper_2606_13740_gb300 import Sched
+    prompt = I.uniform_prompt(64, TINY.vocab, TINY.mask_id)
+    ctx = _gpu_ctx()
+    ctx.dllm_prefill(Sched(steps_per_block=8), prompt, 32)
+    ctx.dllm_begin_block()
+    ctx.dllm_denoise_step()
+    s1 = ctx.dllm_get_state()
+    ctx.dllm_rewind_block()
+    ctx.dllm_denoise_step()
+    s2 = ctx.dllm_get_state()
+    assert np.array_equal(s1[0], s2[0]) and np.array_equal(s1[1], s2[1])
+    ctx.close()
+
+
+def test_errors_poison_context(model):
+    from paper_2606_13740_gb300 import DllmError, Sched
+    ctx = _gpu_ctx(max_ctx=96)
+    with pytest.raises(DllmError):  # capacity
+        ctx.dllm_prefill(Sched(), I.uniform_prompt(64, TINY.vocab, TINY.mask_id), 64)
+    with pytest.raises(DllmError):  # no request yet
+        ctx.dllm_begin_block()
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id)
+    ctx.dllm_prefill(Sched(steps_per_block=8), prompt, 32)
+    ctx.dllm_begin_block()
+    ctx.dllm_denoise_step()
+    with pytest.raises(DllmError):  # block unfinished
+        ctx.dllm_begin_block()
+    ctx.close()
