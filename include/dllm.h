@@ -183,6 +183,35 @@ int dllm_get_weight(dllm_ctx* ctx, int layer, int which, uint16_t* out, size_t n
  * out fp32 [n][n_heads*head_dim] for positions [p0, p0+n).  Synchronises. */
 int dllm_get_kv(dllm_ctx* ctx, int layer, int which, int seq, int p0, int n, float* out);
 
+/* Kernel kinds of one denoising step, for dllm_get_profile. */
+enum {
+    DLLM_K_EMBED = 0,       /* embedding gather + first RMSNorm */
+    DLLM_K_NORM = 1,        /* RMSNorm */
+    DLLM_K_QKV = 2,         /* QKV projection + RoPE + window K/V write */
+    DLLM_K_ATTN = 3,        /* attention (+ split combine) */
+    DLLM_K_OPROJ = 4,       /* output projection + residual */
+    DLLM_K_GATEUP = 5,      /* gate/up projection + SwiGLU */
+    DLLM_K_DOWN = 6,        /* down projection + residual */
+    DLLM_K_HEAD = 7,        /* LM head + per-tile softmax statistics */
+    DLLM_K_HEAD_REDUCE = 8, /* current-id gather, vocab-tile merge */
+    DLLM_K_COMMIT = 9,      /* commit / re-mask / drafts */
+    DLLM_NKINDS = 10
+};
+
+/* Per-kernel timing of denoising steps: with enable, every launch of a step
+ * is followed by a CUDA event on the context's stream (captured into the
+ * step's graph) and each step synchronises to accumulate the elapsed time
+ * between consecutive events by kind.  Enabling resets the totals. */
+int dllm_set_profile(dllm_ctx* ctx, int enable);
+
+/* Totals since dllm_set_profile(1): ms_total[DLLM_NKINDS] milliseconds,
+ * launches_per_step[DLLM_NKINDS] launches of each kind in the last step,
+ * steps profiled (any pointer may be NULL). */
+int dllm_get_profile(dllm_ctx* ctx, double* ms_total, int32_t* launches_per_step, int32_t* steps);
+
+/* Kernel launches in the last denoising step (all kinds). */
+int dllm_launches_per_step(dllm_ctx* ctx, int32_t* n);
+
 #ifdef __cplusplus
 }
 #endif

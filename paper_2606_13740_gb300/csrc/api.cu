@@ -157,9 +157,31 @@ struct dllm_ctx {
     // graph cache for the step
     cudaGraphExec_t gexec = nullptr;
     int g_T = -1, g_B = -1, g_kv = -1, g_dbg = -1;
+    // per-kernel timing (events recorded after every launch of the step)
+    bool profiling = false;
+    std::vector<cudaEvent_t> ev;
+    std::vector<int> ev_kind;
+    int n_marks = 0;
+    double prof_ms[DLLM_NKINDS] = {};
+    int prof_launches[DLLM_NKINDS] = {};
+    int prof_steps = 0;
+    int launches_per_step = 0;
+    bool capturing = false;
+    bool in_step = false;
     bool poisoned = false;
     std::string err;
 };
+
+// Record a timing event after a launch of the given kind (or the start mark).
+static void mark(dllm_ctx* ctx, int kind) {
+    if (!ctx->in_step) return;
+    if (kind >= 0) ctx->launches_per_step++;
+    if (!ctx->profiling || ctx->n_marks >= static_cast<int>(ctx->ev.size())) return;
+    cudaEventRecordWithFlags(ctx->ev[ctx->n_marks], ctx->stream,
+                             ctx->capturing ? cudaEventRecordExternal : cudaEventRecordDefault);
+    ctx->ev_kind[ctx->n_marks] = kind;
+    ctx->n_marks++;
+}
 
 static std::string g_noctx_err;
 
@@ -210,6 +232,7 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
     const int d = c.d_model, F = c.ffn, qd = L.qd, N = B * T;
     cudaStream_t s = ctx->stream;
     CK(launch_embed_norm(ctx->tok, c.max_ctx, ctx->seq_kv, ctx->emb, ctx->x, ctx->xn, B, T, d, c.rms_eps, s));
+    mark(ctx, DLLM_K_EMBED);
     const GemmPlan pq = gemm_plan(L.qkv_rows, N, d, ctx->sms);
     const GemmPlan po = gemm_plan(L.o_rows, N, qd, ctx->sms);
     const GemmPlan pg = gemm_plan(L.gu_rows, N, d, ctx->sms);
@@ -237,20 +260,28 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
         ep.kc = kc;
         ep.vc = vc;
         CK(gemm_launch(EPI_QKV, pq, ctx->tm_qkv[l], tx_xn, ep, ctx->scr, ctx->status, s));
+        mark(ctx, DLLM_K_QKV);
         CK(launch_attention(ctx->q, kc, vc, ctx->seq_kv, ctx->apo, ctx->apml, ctx->attn, B, T, c.n_heads, c.head_dim,
                             c.max_ctx, ap, s));
+        mark(ctx, DLLM_K_ATTN);
         EpiArgs er = ep;
         er.out = ctx->x;
         er.ld_out = d;
         CK(gemm_launch(EPI_RESID, po, ctx->tm_o[l], tx_attn, er, ctx->scr, ctx->status, s));
+        mark(ctx, DLLM_K_OPROJ);
         CK(launch_rmsnorm(ctx->x, ctx->xn, N, d, c.rms_eps, s));
+        mark(ctx, DLLM_K_NORM);
         CK(gemm_launch(EPI_SWIGLU, pg, ctx->tm_gu[l], tx_xn, ep, ctx->scr, ctx->status, s));
+        mark(ctx, DLLM_K_GATEUP);
         CK(gemm_launch(EPI_RESID, pd, ctx->tm_d[l], tx_h, er, ctx->scr, ctx->status, s));
+        mark(ctx, DLLM_K_DOWN);
         CK(launch_rmsnorm(ctx->x, ctx->xn, N, d, c.rms_eps, s));
+        mark(ctx, DLLM_K_NORM);
     }
     if (head) {
         const GemmPlan ph = gemm_plan(L.head_rows, N, d, ctx->sms);
         CK(launch_gather_cur(ctx->tok, c.max_ctx, ctx->seq_kv, ctx->cur, B, T, s));
+        mark(ctx, DLLM_K_HEAD_REDUCE);
         EpiArgs eh{};
         eh.lm_part = ctx->lmp;
         eh.zcur = ctx->zcur;
@@ -259,15 +290,24 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
         eh.mask_id = c.mask_id;
         eh.logits = (ctx->debug & 1) ? ctx->logits : nullptr;
         CK(gemm_launch(EPI_LMHEAD, ph, ctx->tm_head, tx_xn, eh, ctx->scr, ctx->status, s));
+        mark(ctx, DLLM_K_HEAD);
         CK(launch_lmhead_reduce(ctx->lmp, ctx->zcur, ctx->cur, L.head_tiles, N, c.mask_id, ctx->x0, ctx->conf,
                                 ctx->tokconf, s));
+        mark(ctx, DLLM_K_HEAD_REDUCE);
     }
     return DLLM_OK;
 }
 
 static int step_kernels(dllm_ctx* ctx, int T) {
+    ctx->n_marks = 0;
+    ctx->launches_per_step = 0;
+    ctx->in_step = true;
+    mark(ctx, -1);
     int rc = forward(ctx, ctx->B, T, true);
-    if (rc) return rc;
+    if (rc) {
+        ctx->in_step = false;
+        return rc;
+    }
     CommitArgs a{};
     a.tok = ctx->tok;
     a.st = ctx->st;
@@ -288,7 +328,28 @@ static int step_kernels(dllm_ctx* ctx, int T) {
     a.block_len = ctx->cfg.block_len;
     a.theta_remask = ctx->sched.theta_remask;
     a.theta_stable = ctx->sched.theta_stable;
-    CK(launch_commit(a, ctx->stream));
+    cudaError_t ce = launch_commit(a, ctx->stream);
+    mark(ctx, DLLM_K_COMMIT);
+    ctx->in_step = false;
+    CK(ce);
+    return DLLM_OK;
+}
+
+static int profile_collect(dllm_ctx* ctx) {
+    if (!ctx->profiling || ctx->n_marks < 2) return DLLM_OK;
+    CK(cudaStreamSynchronize(ctx->stream));
+    int launches[DLLM_NKINDS] = {};
+    for (int i = 1; i < ctx->n_marks; ++i) {
+        float ms = 0.0f;
+        CK(cudaEventElapsedTime(&ms, ctx->ev[i - 1], ctx->ev[i]));
+        int k = ctx->ev_kind[i];
+        if (k >= 0 && k < DLLM_NKINDS) {
+            ctx->prof_ms[k] += ms;
+            launches[k]++;
+        }
+    }
+    for (int k = 0; k < DLLM_NKINDS; ++k) ctx->prof_launches[k] = launches[k];
+    ctx->prof_steps++;
     return DLLM_OK;
 }
 
@@ -308,6 +369,7 @@ void dllm_free(dllm_ctx* ctx) {
     if (!ctx) return;
     if (ctx->stream) cudaStreamSynchronize(ctx->stream);
     if (ctx->gexec) cudaGraphExecDestroy(ctx->gexec);
+    for (cudaEvent_t e : ctx->ev) cudaEventDestroy(e);
     if (ctx->logits) cudaFree(ctx->logits);
     if (ctx->own_arena && ctx->arena) cudaFree(ctx->arena);
     if (ctx->own_stream && ctx->stream) cudaStreamDestroy(ctx->stream);
@@ -602,14 +664,17 @@ int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out) {
     ctx->last_spec = spec;
     const bool use_graph = !(ctx->debug & 2);
     if (use_graph) {
-        if (!ctx->gexec || ctx->g_T != T || ctx->g_B != ctx->B || ctx->g_kv != ctx->kv_len || ctx->g_dbg != ctx->debug) {
+        const int key_dbg = ctx->debug | (ctx->profiling ? 256 : 0);
+        if (!ctx->gexec || ctx->g_T != T || ctx->g_B != ctx->B || ctx->g_kv != ctx->kv_len || ctx->g_dbg != key_dbg) {
             if (ctx->gexec) {
                 cudaGraphExecDestroy(ctx->gexec);
                 ctx->gexec = nullptr;
             }
             cudaGraph_t g = nullptr;
             CK(cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal));
+            ctx->capturing = true;
             int rc = step_kernels(ctx, T);
+            ctx->capturing = false;
             cudaError_t ee = cudaStreamEndCapture(ctx->stream, &g);
             if (rc) {
                 if (g) cudaGraphDestroy(g);
@@ -622,11 +687,15 @@ int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out) {
             ctx->g_T = T;
             ctx->g_B = ctx->B;
             ctx->g_kv = ctx->kv_len;
-            ctx->g_dbg = ctx->debug;
+            ctx->g_dbg = key_dbg;
         }
         CK(cudaGraphLaunch(ctx->gexec, ctx->stream));
     } else {
         int rc = step_kernels(ctx, T);
+        if (rc) return rc;
+    }
+    {
+        int rc = profile_collect(ctx);
         if (rc) return rc;
     }
     ctx->step++;
@@ -677,6 +746,40 @@ int dllm_generate(dllm_ctx* ctx, const dllm_sched* sched, int batch, const int32
                                static_cast<size_t>(gen_len) * 4, cudaMemcpyDeviceToHost, ctx->stream));
     }
     return sync_check(ctx);
+}
+
+int dllm_set_profile(dllm_ctx* ctx, int enable) {
+    GUARD(ctx);
+    if (enable && ctx->ev.empty()) {
+        const int n = 16 * ctx->cfg.n_layers + 32;
+        ctx->ev.resize(n);
+        ctx->ev_kind.assign(n, -1);
+        for (int i = 0; i < n; ++i) CK(cudaEventCreate(&ctx->ev[i]));
+    }
+    ctx->profiling = enable != 0;
+    for (int k = 0; k < DLLM_NKINDS; ++k) {
+        ctx->prof_ms[k] = 0.0;
+        ctx->prof_launches[k] = 0;
+    }
+    ctx->prof_steps = 0;
+    return DLLM_OK;
+}
+
+int dllm_get_profile(dllm_ctx* ctx, double* ms_total, int32_t* launches_per_step, int32_t* steps) {
+    GUARD(ctx);
+    for (int k = 0; k < DLLM_NKINDS; ++k) {
+        if (ms_total) ms_total[k] = ctx->prof_ms[k];
+        if (launches_per_step) launches_per_step[k] = ctx->prof_launches[k];
+    }
+    if (steps) *steps = ctx->prof_steps;
+    return DLLM_OK;
+}
+
+int dllm_launches_per_step(dllm_ctx* ctx, int32_t* n) {
+    GUARD(ctx);
+    if (!n) return fail(ctx, DLLM_EINVAL, "null output");
+    *n = ctx->launches_per_step;
+    return DLLM_OK;
 }
 
 int dllm_window(dllm_ctx* ctx, int32_t* info) {

@@ -73,6 +73,9 @@ SIGNATURES = {
     "dllm_set_debug": (_I, [_P, _I]),
     "dllm_get_weight": (_I, [_P, _I, _I, _P, _SZ]),
     "dllm_get_kv": (_I, [_P, _I, _I, _I, _I, _I, _P]),
+    "dllm_set_profile": (_I, [_P, _I]),
+    "dllm_get_profile": (_I, [_P, _P, _P, _P]),
+    "dllm_launches_per_step": (_I, [_P, _P]),
     "dllm_op_gemm": (_I, [_P, _P, _P, _I, _I, _I, _I, _P]),
     "dllm_op_attention": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P]),
     "dllm_op_lmhead": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _P]),
@@ -268,6 +271,24 @@ class Context:
         out = np.empty((n, qd), np.float32)
         _check(lib().dllm_get_kv(self.h, layer, which, seq, p0, n, _p(out)), self.h)
         return out
+
+    KINDS = ("embed", "norm", "qkv", "attn", "oproj", "gateup", "down", "head", "head_reduce", "commit")
+
+    def dllm_set_profile(self, enable):
+        _check(lib().dllm_set_profile(self.h, int(enable)), self.h)
+
+    def dllm_get_profile(self):
+        ms = np.zeros(len(self.KINDS), np.float64)
+        launches = np.zeros(len(self.KINDS), np.int32)
+        steps = np.zeros(1, np.int32)
+        _check(lib().dllm_get_profile(self.h, _p(ms), _p(launches), _p(steps)), self.h)
+        return {k: {"ms_total": float(ms[i]), "launches_per_step": int(launches[i])} for i, k in
+                enumerate(self.KINDS)}, int(steps[0])
+
+    def dllm_launches_per_step(self):
+        n = np.zeros(1, np.int32)
+        _check(lib().dllm_launches_per_step(self.h, _p(n)), self.h)
+        return int(n[0])
 
     def dllm_sync(self):
         _check(lib().dllm_sync(self.h), self.h)
