@@ -219,7 +219,7 @@ def run_ours(args):
 
     cfg = Config(max_batch=1, max_ctx=LP + T, max_window=LP, **SHAPE)
     ctx = Context(cfg)
-    stream = torch.cuda.current_stream()
+    stream = ctx.stream  # the context's own stream: events and kernels share it
     sched = Sched(steps_per_block=MASKED)
     prompt = I.uniform_prompt(LP, cfg.vocab, cfg.mask_id, seed=I.SEED_PROMPT + rank)
     ctx.dllm_prefill(sched, prompt, T)

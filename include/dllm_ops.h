@@ -23,6 +23,12 @@ extern "C" {
  * SM).  Errors: DLLM_EINVAL, DLLM_ECUDA, DLLM_ETIMEOUT. */
 int dllm_op_gemm(const void* W, const void* X, float* D, int M, int N, int K, int grid, void* stream);
 
+/* dllm_op_gemm launched `reps` times back to back on one scratch
+ * allocation; *ms_per_launch = average kernel time by CUDA events on the
+ * stream (micro-benchmark hook). */
+int dllm_op_gemm_timed(const void* W, const void* X, float* D, int M, int N, int K, int grid, int reps,
+                       float* ms_per_launch, void* stream);
+
 /* Bidirectional attention of the window's queries over cached + window keys
  * (Sec. 2.1, block-wise decoding with prefix KV reuse; no causal mask).
  * q dev bf16 [B][H][T][hd]; kc, vc dev bf16 [B][H][cap][hd] (keys of

@@ -59,8 +59,10 @@ int finish(cudaStream_t st, int* status_dev) {
 
 extern "C" {
 
-int dllm_op_gemm(const void* W, const void* X, float* D, int M, int N, int K, int grid, void* stream) {
-    if (!W || !X || !D || M < 1 || N < 1 || K < 1 || (K * 2) % 16) return op_fail(DLLM_EINVAL, "bad gemm arguments");
+static int gemm_impl(const void* W, const void* X, float* D, int M, int N, int K, int grid, int reps, float* ms,
+                     void* stream) {
+    if (!W || !X || !D || M < 1 || N < 1 || K < 1 || (K * 2) % 16 || reps < 1)
+        return op_fail(DLLM_EINVAL, "bad gemm arguments");
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     int sms = sm_count();
     if (sms <= 0) return op_fail(DLLM_ECUDA, "no CUDA device");
@@ -81,9 +83,39 @@ int dllm_op_gemm(const void* W, const void* X, float* D, int M, int N, int K, in
     EpiArgs ep{};
     ep.out = D;
     ep.ld_out = M;
-    cudaError_t e = gemm_launch(EPI_F32, p, tw, tx, ep, scr, static_cast<int*>(status.p), st);
-    if (e != cudaSuccess) return op_fail(DLLM_ECUDA, "gemm launch: %s", cudaGetErrorString(e));
-    return finish(st, static_cast<int*>(status.p));
+    cudaEvent_t e0 = nullptr, e1 = nullptr;
+    if (ms && (cudaEventCreate(&e0) != cudaSuccess || cudaEventCreate(&e1) != cudaSuccess))
+        return op_fail(DLLM_ECUDA, "event creation failed");
+    cudaError_t e = cudaSuccess;
+    if (ms) {
+        // one untimed launch first (instruction and descriptor caches)
+        e = gemm_launch(EPI_F32, p, tw, tx, ep, scr, static_cast<int*>(status.p), st);
+        if (e == cudaSuccess) e = cudaEventRecord(e0, st);
+    }
+    for (int r = 0; r < reps && e == cudaSuccess; ++r)
+        e = gemm_launch(EPI_F32, p, tw, tx, ep, scr, static_cast<int*>(status.p), st);
+    if (ms && e == cudaSuccess) e = cudaEventRecord(e1, st);
+    int rc = DLLM_OK;
+    if (e != cudaSuccess) rc = op_fail(DLLM_ECUDA, "gemm launch: %s", cudaGetErrorString(e));
+    if (rc == DLLM_OK) rc = finish(st, static_cast<int*>(status.p));
+    if (rc == DLLM_OK && ms) {
+        float t = 0.0f;
+        cudaEventElapsedTime(&t, e0, e1);
+        *ms = t / reps;
+    }
+    if (e0) cudaEventDestroy(e0);
+    if (e1) cudaEventDestroy(e1);
+    return rc;
+}
+
+int dllm_op_gemm(const void* W, const void* X, float* D, int M, int N, int K, int grid, void* stream) {
+    return gemm_impl(W, X, D, M, N, K, grid, 1, nullptr, stream);
+}
+
+int dllm_op_gemm_timed(const void* W, const void* X, float* D, int M, int N, int K, int grid, int reps,
+                       float* ms_per_launch, void* stream) {
+    if (!ms_per_launch) return op_fail(DLLM_EINVAL, "null output");
+    return gemm_impl(W, X, D, M, N, K, grid, reps, ms_per_launch, stream);
 }
 
 int dllm_op_attention(const void* q, const void* kc, const void* vc, const int32_t* kv_len, void* out, int B, int T,

@@ -77,6 +77,7 @@ SIGNATURES = {
     "dllm_get_profile": (_I, [_P, _P, _P, _P]),
     "dllm_launches_per_step": (_I, [_P, _P]),
     "dllm_op_gemm": (_I, [_P, _P, _P, _I, _I, _I, _I, _P]),
+    "dllm_op_gemm_timed": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _P, _P]),
     "dllm_op_attention": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P]),
     "dllm_op_lmhead": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _P]),
     "dllm_op_commit": (_I, [_P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _I, _F, _F, _I, _I, _I, _I, _I, _P]),
@@ -178,7 +179,9 @@ class Context:
             self.arena = torch.empty(nbytes + 256, dtype=torch.uint8, device="cuda")
             arena_ptr = (self.arena.data_ptr() + 255) // 256 * 256
         if stream is None:
-            stream = torch.cuda.current_stream()
+            # a stream of its own: torch's default stream is the legacy stream
+            # (handle 0), which the C ABI would read as "create one"
+            stream = torch.cuda.Stream()
         self.stream = stream
         h = C.c_void_p()
         _check(lib().dllm_init(C.byref(self._c), _p(arena_ptr), nbytes, _p(stream.cuda_stream), C.byref(h)))
@@ -318,6 +321,17 @@ def dllm_op_gemm(W, X, M, N, K, grid=0, stream=None):
     _check(lib().dllm_op_gemm(_p(W.data_ptr()), _p(X.data_ptr()), _p(D.data_ptr()), M, N, K, grid,
                               _p(_stream_ptr(stream))))
     return D
+
+
+def dllm_op_gemm_timed(W, X, M, N, K, reps, grid=0, stream=None):
+    """Average kernel time (ms) of `reps` back-to-back launches, and D."""
+    import torch
+
+    D = torch.empty((N, M), dtype=torch.float32, device=W.device)
+    ms = C.c_float()
+    _check(lib().dllm_op_gemm_timed(_p(W.data_ptr()), _p(X.data_ptr()), _p(D.data_ptr()), M, N, K, grid, reps,
+                                    C.byref(ms), _p(_stream_ptr(stream))))
+    return ms.value, D
 
 
 def dllm_op_attention(q, kc, vc, kv_len, B, T, H, hd, cap, max_kv_len, stream=None):

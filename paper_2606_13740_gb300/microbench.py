@@ -14,12 +14,12 @@ import time
 
 import torch
 
-from .dllm import dllm_op_attention, dllm_op_gemm, lib
+from .dllm import dllm_op_attention, dllm_op_gemm, dllm_op_gemm_timed, lib
 
 
 def main(argv=None):
     ap = argparse.ArgumentParser()
-    ap.add_argument("op", choices=("gemm", "attention"))
+    ap.add_argument("op", choices=("gemm", "attention", "gemm-sweep"))
     ap.add_argument("--M", type=int, default=24576)
     ap.add_argument("--N", type=int, default=32)
     ap.add_argument("--K", type=int, default=4096)
@@ -33,6 +33,20 @@ def main(argv=None):
     dev = torch.device("cuda:0")
     g = torch.Generator(device=dev)
     g.manual_seed(0)
+    if a.op == "gemm-sweep":
+        # kernel time vs weight rows: separates the fixed cost of a launch from the streaming rate
+        rows = []
+        for K in (4096, 12288):
+            for M in (512, 1024, 2048, 4096, 8192, 12288, 24576, 49152, 126464):
+                if M * K > 126464 * 4096:
+                    continue
+                W = (torch.randn(M, K, device=dev, generator=g) * 0.02).to(torch.bfloat16)
+                X = torch.randn(a.N, K, device=dev, generator=g).to(torch.bfloat16)
+                ms, _ = dllm_op_gemm_timed(W, X, M, a.N, K, a.reps)
+                rows.append({"M": M, "N": a.N, "K": K, "us": ms * 1e3, "GBps": M * K * 2 / (ms * 1e-3) / 1e9})
+                del W, X
+        print(json.dumps({"op": "gemm-sweep", "rows": rows}))
+        return
     if a.op == "gemm":
         W = (torch.randn(a.M, a.K, device=dev, generator=g) * 0.02).to(torch.bfloat16)
         X = torch.randn(a.N, a.K, device=dev, generator=g).to(torch.bfloat16)
