@@ -29,6 +29,25 @@ int dllm_op_gemm(const void* W, const void* X, float* D, int M, int N, int K, in
 int dllm_op_gemm_timed(const void* W, const void* X, float* D, int M, int N, int K, int grid, int reps,
                        float* ms_per_launch, void* stream);
 
+/* dllm_op_gemm for callers that cannot allocate device memory, for example
+ * code that runs while a stream is being captured into a CUDA graph (a
+ * cudaMalloc there breaks the capture), or an embedding application whose
+ * memory is owned by its own pool and forbids allocations behind its back.
+ * The paper has no counterpart: this is a property of this library's API.
+ * It computes the same D[n][m] = sum_k W[m][k] * X[n][k] as dllm_op_gemm but
+ * keeps its scratch (split partials, tile tickets, status word) in one
+ * statically sized device array of 8 MiB that every GPU loading the library
+ * holds until the process exits; it calls no cudaMalloc, cudaFree or other
+ * allocating routine.  Limits: at most 16320 output tiles (ceil(M/128) x
+ * token tiles); the grid (0 = one CTA per SM) is shrunk to fit the array when
+ * chosen automatically, and an explicit grid that does not fit is rejected
+ * with DLLM_ECAPACITY.  The first call on a device looks up the array's
+ * device address (cudaGetSymbolAddress) with that device current; make that
+ * first call before any stream capture.  All calls share the one array: two
+ * calls that overlap on the GPU (other streams, other host threads) race and
+ * corrupt each other's results.  Synchronises the stream. */
+int dllm_op_gemm_noalloc(const void* W, const void* X, float* D, int M, int N, int K, int grid, void* stream);
+
 /* Bidirectional attention of the window's queries over cached + window keys
  * (Sec. 2.1, block-wise decoding with prefix KV reuse; no causal mask).
  * q dev bf16 [B][H][T][hd]; kc, vc dev bf16 [B][H][cap][hd] (keys of

@@ -77,6 +77,7 @@ SIGNATURES = {
     "dllm_get_profile": (_I, [_P, _P, _P, _P]),
     "dllm_launches_per_step": (_I, [_P, _P]),
     "dllm_op_gemm": (_I, [_P, _P, _P, _I, _I, _I, _I, _P]),
+    "dllm_op_gemm_noalloc": (_I, [_P, _P, _P, _I, _I, _I, _I, _P]),
     "dllm_op_gemm_timed": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _P, _P]),
     "dllm_op_attention": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P]),
     "dllm_op_lmhead": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _P]),
@@ -320,6 +321,13 @@ def dllm_op_gemm(W, X, M, N, K, grid=0, stream=None):
     D = torch.empty((N, M), dtype=torch.float32, device=W.device)
     _check(lib().dllm_op_gemm(_p(W.data_ptr()), _p(X.data_ptr()), _p(D.data_ptr()), M, N, K, grid,
                               _p(_stream_ptr(stream))))
+    return D
+
+
+def dllm_op_gemm_noalloc(W, X, D, M, N, K, grid=0, stream=None):
+    """dllm_op_gemm into a caller-provided D (fp32 [N][M]); allocates nothing."""
+    _check(lib().dllm_op_gemm_noalloc(_p(W.data_ptr()), _p(X.data_ptr()), _p(D.data_ptr()), M, N, K, grid,
+                                      _p(_stream_ptr(stream))))
     return D
 
 
