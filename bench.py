@@ -219,6 +219,8 @@ def run_ours(args):
 
     cfg = Config(max_batch=1, max_ctx=LP + T, max_window=LP, **SHAPE)
     ctx = Context(cfg)
+    if args.no_pdl:
+        ctx.dllm_set_debug(4)
     stream = ctx.stream  # the context's own stream: events and kernels share it
     sched = Sched(steps_per_block=MASKED)
     prompt = I.uniform_prompt(LP, cfg.vocab, cfg.mask_id, seed=I.SEED_PROMPT + rank)
@@ -364,6 +366,7 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-pdl", action="store_true", help="launch kernels without programmatic dependent launch")
     args = ap.parse_args(argv)
     if args.impl == "reference":
         return run_reference(args)

@@ -56,7 +56,7 @@ typedef struct dllm_ctx dllm_ctx;
  * bf16, drawn on the device from weight_seed (N(0, 0.02) by a counter-based
  * SplitMix64/Irwin-Hall generator); RMSNorm gains are one.
  * Constraints: head_dim in {64, 128}; d_model, n_heads*head_dim multiples of
- * 64; vocab, ffn multiples of 8; max_window * max_batch <= 4096. */
+ * 128; vocab, ffn multiples of 8; max_window * max_batch <= 4096. */
 typedef struct {
     int n_layers, d_model, n_heads, head_dim, ffn, vocab, mask_id;
     float rope_base, rms_eps;

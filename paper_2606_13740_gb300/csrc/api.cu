@@ -34,7 +34,8 @@ int rup(int x, int m) { return (x + m - 1) / m * m; }
 struct Layout {
     int qd, qkv_rows, gu_rows, d_rows, o_rows, head_rows, head_tiles, max_tok;
     size_t off_w, per_layer, off_emb, off_head, off_kv, kv_half, off_rope;
-    size_t off_x, off_xn, off_q, off_attn, off_h;
+    size_t off_x, off_xn, off_q, off_attn, off_h, off_sq, off_actr;
+    int n_sq, actr_len;
     size_t off_apo, apo_floats, off_apml;
     size_t off_lmp, off_zcur, off_cur, off_x0, off_conf, off_tokconf;
     size_t off_part, part_floats, off_cnt;
@@ -78,6 +79,10 @@ Layout make_layout(const dllm_config& c) {
     L.off_q = take(T * L.qd * 2);
     L.off_attn = take(T * L.qd * 2);
     L.off_h = take(T * F * 2);
+    L.n_sq = (d + 127) / 128;
+    L.off_sq = take(static_cast<size_t>(L.n_sq) * T * 4);
+    L.actr_len = c.max_batch * H * ((c.max_window + 63) / 64);
+    L.off_actr = take(static_cast<size_t>(L.actr_len) * 4);
     // attention split partials: B*H*nsplit*T rows, nsplit <= 2*SMs/(B*H*qtiles) + 1
     const size_t rows = static_cast<size_t>(2 * kMaxSMs) * 64 + static_cast<size_t>(c.max_batch) * H * c.max_window;
     L.apo_floats = rows * hd;
@@ -110,7 +115,8 @@ Layout make_layout(const dllm_config& c) {
 const char* check_cfg(const dllm_config& c) {
     if (c.n_layers < 1 || c.d_model < 64 || c.n_heads < 1 || c.ffn < 8 || c.vocab < 2) return "bad model shape";
     if (c.head_dim != 64 && c.head_dim != 128) return "head_dim must be 64 or 128";
-    if (c.d_model % 64 || (c.n_heads * c.head_dim) % 64) return "d_model and n_heads*head_dim must be multiples of 64";
+    if (c.d_model % 128 || (c.n_heads * c.head_dim) % 128)
+        return "d_model and n_heads*head_dim must be multiples of 128";
     if (c.ffn % 8 || c.vocab % 8) return "ffn and vocab must be multiples of 8";
     if (c.mask_id < 0 || c.mask_id >= c.vocab) return "mask_id out of range";
     if (c.max_batch < 1 || c.max_ctx < 1 || c.max_window < 1 || c.block_len < 1) return "bad capacities";
@@ -140,6 +146,8 @@ struct dllm_ctx {
     float* rope = nullptr;
     float* x = nullptr;
     __nv_bfloat16 *xn = nullptr, *q = nullptr, *attn = nullptr, *h = nullptr;
+    float* sq = nullptr;      // RMSNorm statistics [d/128][tokens]
+    int* actr = nullptr;      // attention split tickets
     float *apo = nullptr, *apml = nullptr, *lmp = nullptr, *zcur = nullptr, *conf = nullptr, *tokconf = nullptr;
     int *cur = nullptr, *x0 = nullptr;
     Scratch scr{};
@@ -231,18 +239,20 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
     const Layout& L = ctx->L;
     const int d = c.d_model, F = c.ffn, qd = L.qd, N = B * T;
     cudaStream_t s = ctx->stream;
-    CK(launch_embed_norm(ctx->tok, c.max_ctx, ctx->seq_kv, ctx->emb, ctx->x, ctx->xn, B, T, d, c.rms_eps, s));
+    // x = embedding rows, xb = bf16(x) (the next projection's operand), sq = RMSNorm statistics
+    CK(launch_embed(ctx->tok, c.max_ctx, ctx->seq_kv, ctx->emb, ctx->x, ctx->xn, ctx->sq, ctx->cur, B, T, d, s));
     mark(ctx, DLLM_K_EMBED);
-    const GemmPlan pq = gemm_plan(L.qkv_rows, N, d, ctx->sms);
-    const GemmPlan po = gemm_plan(L.o_rows, N, qd, ctx->sms);
-    const GemmPlan pg = gemm_plan(L.gu_rows, N, d, ctx->sms);
-    const GemmPlan pd = gemm_plan(L.d_rows, N, F, ctx->sms);
+    const GemmPlan pq = gemm_plan(L.qkv_rows, N, d, ctx->sms, EPI_QKV);
+    const GemmPlan po = gemm_plan(L.o_rows, N, qd, ctx->sms, EPI_RESID);
+    const GemmPlan pg = gemm_plan(L.gu_rows, N, d, ctx->sms, EPI_SWIGLU);
+    const GemmPlan pd = gemm_plan(L.d_rows, N, F, ctx->sms, EPI_RESID);
     CUtensorMap tx_xn, tx_attn, tx_h;
     if (!make_tmap_bf16(&tx_xn, ctx->xn, N, d, pq.ntile) || !make_tmap_bf16(&tx_attn, ctx->attn, N, qd, po.ntile) ||
         !make_tmap_bf16(&tx_h, ctx->h, N, F, pd.ntile))
         return fail(ctx, DLLM_ECUDA, "tensor map encode failed");
     const AttnPlan ap = attn_plan(B, T, c.n_heads, ctx->kv_len + T, ctx->sms);
-    if (static_cast<size_t>(B) * c.n_heads * ap.nsplit * T * c.head_dim > L.apo_floats)
+    if (static_cast<size_t>(B) * c.n_heads * ap.nsplit * T * c.head_dim > L.apo_floats ||
+        B * c.n_heads * ap.qtiles > L.actr_len)
         return fail(ctx, DLLM_ECAPACITY, "attention partial buffer too small");
     EpiArgs ep{};
     ep.rope = ctx->rope;
@@ -254,6 +264,15 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
     ep.q = ctx->q;
     ep.h = ctx->h;
     ep.F = F;
+    ep.sq_in = ctx->sq;  // consumers of the residual stream apply RMSNorm as a per-token scale
+    ep.n_sq = L.n_sq;
+    ep.norm_dim = d;
+    ep.eps = c.rms_eps;
+    EpiArgs er{};
+    er.out = ctx->x;
+    er.ld_out = d;
+    er.xb = ctx->xn;
+    er.sq_out = ctx->sq;
     for (int l = 0; l < c.n_layers; ++l) {
         __nv_bfloat16* kc = ctx->kv + static_cast<size_t>(2 * l) * L.kv_half;
         __nv_bfloat16* vc = ctx->kv + static_cast<size_t>(2 * l + 1) * L.kv_half;
@@ -261,28 +280,19 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
         ep.vc = vc;
         CK(gemm_launch(EPI_QKV, pq, ctx->tm_qkv[l], tx_xn, ep, ctx->scr, ctx->status, s));
         mark(ctx, DLLM_K_QKV);
-        CK(launch_attention(ctx->q, kc, vc, ctx->seq_kv, ctx->apo, ctx->apml, ctx->attn, B, T, c.n_heads, c.head_dim,
-                            c.max_ctx, ap, s));
+        CK(launch_attention(ctx->q, kc, vc, ctx->seq_kv, ctx->apo, ctx->apml, ctx->actr, ctx->attn, B, T, c.n_heads,
+                            c.head_dim, c.max_ctx, ap, s));
         mark(ctx, DLLM_K_ATTN);
-        EpiArgs er = ep;
-        er.out = ctx->x;
-        er.ld_out = d;
         CK(gemm_launch(EPI_RESID, po, ctx->tm_o[l], tx_attn, er, ctx->scr, ctx->status, s));
         mark(ctx, DLLM_K_OPROJ);
-        CK(launch_rmsnorm(ctx->x, ctx->xn, N, d, c.rms_eps, s));
-        mark(ctx, DLLM_K_NORM);
         CK(gemm_launch(EPI_SWIGLU, pg, ctx->tm_gu[l], tx_xn, ep, ctx->scr, ctx->status, s));
         mark(ctx, DLLM_K_GATEUP);
         CK(gemm_launch(EPI_RESID, pd, ctx->tm_d[l], tx_h, er, ctx->scr, ctx->status, s));
         mark(ctx, DLLM_K_DOWN);
-        CK(launch_rmsnorm(ctx->x, ctx->xn, N, d, c.rms_eps, s));
-        mark(ctx, DLLM_K_NORM);
     }
     if (head) {
-        const GemmPlan ph = gemm_plan(L.head_rows, N, d, ctx->sms);
-        CK(launch_gather_cur(ctx->tok, c.max_ctx, ctx->seq_kv, ctx->cur, B, T, s));
-        mark(ctx, DLLM_K_HEAD_REDUCE);
-        EpiArgs eh{};
+        const GemmPlan ph = gemm_plan(L.head_rows, N, d, ctx->sms, EPI_LMHEAD);
+        EpiArgs eh = ep;
         eh.lm_part = ctx->lmp;
         eh.zcur = ctx->zcur;
         eh.cur_tok = ctx->cur;
@@ -428,6 +438,8 @@ int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void*
     ctx->q = reinterpret_cast<__nv_bfloat16*>(A + L.off_q);
     ctx->attn = reinterpret_cast<__nv_bfloat16*>(A + L.off_attn);
     ctx->h = reinterpret_cast<__nv_bfloat16*>(A + L.off_h);
+    ctx->sq = reinterpret_cast<float*>(A + L.off_sq);
+    ctx->actr = reinterpret_cast<int*>(A + L.off_actr);
     ctx->apo = reinterpret_cast<float*>(A + L.off_apo);
     ctx->apml = reinterpret_cast<float*>(A + L.off_apml);
     ctx->lmp = reinterpret_cast<float*>(A + L.off_lmp);
@@ -450,13 +462,14 @@ int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void*
     ctx->status = reinterpret_cast<int*>(A + L.off_status);
     cudaStream_t s = ctx->stream;
     // zero everything that is read before it is written (counters, state, status)
-    if (cudaMemsetAsync(A + L.off_lmp, 0, L.total - L.off_lmp, s) != cudaSuccess ||
+    if (cudaMemsetAsync(A + L.off_sq, 0, L.total - L.off_sq, s) != cudaSuccess ||
         cudaMemsetAsync(A + L.off_kv, 0, L.kv_half * 4 * c.n_layers, s) != cudaSuccess)
         return bail(DLLM_ECUDA, "memset failed");
     // weights from the seed (tensor ids: embedding 1, head 2, layer l: 16 + 8l + {q,k,v,o,gate,up,down})
     const uint64_t seed = c.weight_seed;
-    cudaError_t ie = launch_init_weight(ctx->emb, 0, c.vocab, d, c.vocab, seed, 1, qd, s);
-    if (ie == cudaSuccess) ie = launch_init_weight(ctx->head, 0, L.head_rows, d, c.vocab, seed, 2, qd, s);
+    const int hd = c.head_dim;
+    cudaError_t ie = launch_init_weight(ctx->emb, 0, c.vocab, d, c.vocab, seed, 1, qd, hd, s);
+    if (ie == cudaSuccess) ie = launch_init_weight(ctx->head, 0, L.head_rows, d, c.vocab, seed, 2, qd, hd, s);
     ctx->wl.resize(c.n_layers);
     ctx->tm_qkv.resize(c.n_layers);
     ctx->tm_o.resize(c.n_layers);
@@ -466,10 +479,10 @@ int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void*
         __nv_bfloat16* w = reinterpret_cast<__nv_bfloat16*>(A + L.off_w) + static_cast<size_t>(l) * L.per_layer;
         ctx->wl[l] = w;
         const uint64_t t0 = 16 + 8ull * l;
-        ie = launch_init_weight(w + L.w_qkv, 1, L.qkv_rows, d, 3 * qd, seed, t0 + 0, qd, s);
-        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_o, 0, L.o_rows, qd, d, seed, t0 + 3, qd, s);
-        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_gu, 2, L.gu_rows, d, F, seed, t0 + 4, qd, s);
-        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_d, 0, L.d_rows, F, d, seed, t0 + 6, qd, s);
+        ie = launch_init_weight(w + L.w_qkv, 1, L.qkv_rows, d, qd, seed, t0 + 0, qd, hd, s);
+        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_o, 0, L.o_rows, qd, d, seed, t0 + 3, qd, hd, s);
+        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_gu, 2, L.gu_rows, d, F, seed, t0 + 4, qd, hd, s);
+        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_d, 0, L.d_rows, F, d, seed, t0 + 6, qd, hd, s);
         bool ok = make_tmap_bf16(&ctx->tm_qkv[l], w + L.w_qkv, L.qkv_rows, d, 128) &&
                   make_tmap_bf16(&ctx->tm_o[l], w + L.w_o, L.o_rows, qd, 128) &&
                   make_tmap_bf16(&ctx->tm_gu[l], w + L.w_gu, L.gu_rows, d, 128) &&
@@ -503,6 +516,7 @@ static int set_debug_buffers(dllm_ctx* ctx) {
 int dllm_set_debug(dllm_ctx* ctx, int flags) {
     GUARD(ctx);
     ctx->debug = flags;
+    set_pdl(!(flags & 4));
     return set_debug_buffers(ctx);
 }
 
@@ -868,14 +882,26 @@ int dllm_get_weight(dllm_ctx* ctx, int layer, int which, uint16_t* out, size_t n
         int rows = (which <= 2) ? qd : (which == 3 || which == 6) ? d : F;
         int cols = (which == 3) ? qd : (which == 6) ? F : d;
         if (n_elems < static_cast<size_t>(rows) * cols) return fail(ctx, DLLM_EINVAL, "buffer too small");
-        if (which <= 2) rc = copy_rows(w + L.w_qkv + static_cast<size_t>(which) * qd * d, qd, d, 0);
-        else if (which == 3) rc = copy_rows(w + L.w_o, d, qd, 0);
+        if (which == 3) rc = copy_rows(w + L.w_o, d, qd, 0);
         else if (which == 6) rc = copy_rows(w + L.w_d, d, F, 0);
         else {
-            const int up = which == 5;
-            for (int t = 0; t * 64 < F && rc == DLLM_OK; ++t) {
-                int nr = std::min(64, F - t * 64);
-                rc = copy_rows(w + L.w_gu + (static_cast<size_t>(t) * 128 + up * 64) * d, nr, d, static_cast<size_t>(t) * 64);
+            // q/k/v rows are interleaved inside each head; gate/up rows alternate in each tile
+            const size_t phys_rows = which <= 2 ? static_cast<size_t>(qd) : static_cast<size_t>(L.gu_rows);
+            const __nv_bfloat16* src = which <= 2 ? w + L.w_qkv + static_cast<size_t>(which) * qd * d : w + L.w_gu;
+            std::vector<uint16_t> phys(phys_rows * d);
+            CK(cudaMemcpyAsync(phys.data(), src, phys.size() * 2, cudaMemcpyDeviceToHost, ctx->stream));
+            rc = sync_check(ctx);
+            if (rc) return rc;
+            const int hd = c.head_dim, half = hd / 2;
+            for (int r = 0; r < rows; ++r) {
+                size_t pr;
+                if (which <= 2) {
+                    const int hh = r / hd, i = r % hd;
+                    pr = static_cast<size_t>(hh) * hd + 2 * (i % half) + i / half;
+                } else {
+                    pr = static_cast<size_t>(r / 64) * 128 + 2 * (r % 64) + (which == 5 ? 1 : 0);
+                }
+                memcpy(out + static_cast<size_t>(r) * cols, phys.data() + pr * d, static_cast<size_t>(d) * 2);
             }
         }
     }

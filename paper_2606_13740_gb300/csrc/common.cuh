@@ -27,6 +27,13 @@ __device__ __forceinline__ unsigned long long global_ns() {
     return t;
 }
 
+// ------------------------------------------------------------------ PDL
+// Wait until the grids this one depends on have completed and their writes are visible
+// (no-op when launched without programmatic serialisation).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Let the dependent grid start launching (its CTAs still wait before reading our output).
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // ------------------------------------------------------------------ mbarrier
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");

@@ -17,21 +17,29 @@
 // Roles (192 threads): warp 0 = TMA producer, warp 1 = TMEM owner and MMA
 // issuer, warps 2..5 = epilogue (one TMEM lane quarter each).  Accumulators
 // are double-buffered in TMEM so the epilogue of one tile overlaps the MMAs
-// of the next.  Epilogues are fused: residual add, RoPE + KV-cache write,
-// SwiGLU, and the LM head's per-tile softmax statistics.
+// of the next.  Epilogues are fused: residual add with the next RMSNorm's
+// statistics, RoPE + KV-cache write, SwiGLU, and the LM head's per-tile
+// softmax statistics; the consumers of a residual apply RMSNorm as a
+// per-token scale of their fp32 accumulators.
+//
+// Launched with programmatic dependent launch: the producer streams its first
+// pipeline stages of weights (which no earlier kernel writes) before
+// griddepcontrol.wait, so a projection's weight stream starts while the
+// previous kernel is still finishing.
 #include "common.cuh"
 #include "internal.h"
 
 #include <climits>
-#include <cstdio>
 
 namespace dllm {
 
-constexpr int kBK = 64;     // K elements per stage: one 128-byte swizzle row
 constexpr int kBM = 128;    // UMMA M
+constexpr int kBK = 64;     // K elements per stage: one 128-byte swizzle row
 constexpr int kThreads = 192;
-constexpr int kStageLd = 33;
+constexpr int kStageLd = 17;  // LM-head staging: 16 columns + pad
 constexpr uint32_t kABytes = kBM * kBK * 2;
+constexpr int kStreamSmem = 115712;  // two CTAs per SM (228 KB less 1 KB reserved each)
+constexpr int kFullSmem = 227 * 1024;
 
 __device__ __forceinline__ int owner_of(long long i, long long total, int G) {
     return static_cast<int>(((i + 1) * G + total - 1) / total) - 1;
@@ -39,84 +47,142 @@ __device__ __forceinline__ int owner_of(long long i, long long total, int G) {
 
 __device__ __forceinline__ long long range_begin(int c, long long total, int G) { return total * c / G; }
 
+// Sum of v[0..31] over the 32 lanes of a warp, scattered: afterwards lane l
+// holds the total of column l in v[0].  31 shuffles in a fixed order.
+__device__ __forceinline__ void warp_reduce_scatter32(float* v, int lane) {
+#pragma unroll
+    for (int w = 16; w >= 1; w >>= 1) {
+        const bool upper = (lane & w) != 0;
+#pragma unroll
+        for (int i = 0; i < w; ++i) {
+            float send = upper ? v[i] : v[i + w];
+            float keep = upper ? v[i + w] : v[i];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, w);
+        }
+    }
+}
+
+struct EpiSmem {
+    float* stg;   // LM head staging [128][kStageLd]
+    float* rs;    // [32] per-column RMSNorm scale
+    float* red;   // [4][32] cross-warp partial sums
+};
+
 // ------------------------------------------------------------------ epilogues
 template <int EPI>
 __device__ __forceinline__ void epilogue_chunk(const EpiArgs& ep, const GemmPlan& p, int mt, int nt, int chunk,
-                                               int rt, const float* v, float* stg, int ew, int lane, int* status) {
+                                               int rt, float* v, const EpiSmem& sm, int ew, int quarter, int lane,
+                                               int* status) {
     const int row = mt * kBM + rt;
     const int col0 = nt * p.ntile + chunk * 32;
-    if constexpr (EPI == EPI_F32 || EPI == EPI_RESID) {
+    if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
+        if (ep.sq_in) {  // RMSNorm of the operand rows, as a per-token scale
+            if (ew == 0) {
+                const int col = col0 + lane;
+                float s = 0.0f;
+                if (col < p.N)
+                    for (int t = 0; t < ep.n_sq; ++t) s += ep.sq_in[static_cast<size_t>(t) * p.N + col];
+                sm.rs[lane] = rsqrtf(s / static_cast<float>(ep.norm_dim) + ep.eps);
+            }
+            named_bar(1, 128);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] *= sm.rs[j];
+            named_bar(1, 128);
+        }
+    }
+    if constexpr (EPI == EPI_F32) {
         if (row < p.M) {
 #pragma unroll 8
             for (int j = 0; j < 32; ++j) {
-                int col = col0 + j;
-                if (col < p.N) {
-                    float* o = ep.out + static_cast<size_t>(col) * ep.ld_out + row;
-                    if constexpr (EPI == EPI_F32) *o = v[j]; else *o += v[j];
-                }
+                const int col = col0 + j;
+                if (col < p.N) ep.out[static_cast<size_t>(col) * ep.ld_out + row] = v[j];
             }
         }
-        return;
-    } else {
+    } else if constexpr (EPI == EPI_RESID) {
+        const bool rv = row < p.M;
 #pragma unroll
-        for (int j = 0; j < 32; ++j) stg[rt * kStageLd + j] = v[j];
+        for (int j = 0; j < 32; ++j) {
+            const int col = col0 + j;
+            float x = 0.0f;
+            if (rv && col < p.N) {
+                const size_t o = static_cast<size_t>(col) * ep.ld_out + row;
+                x = ep.out[o] + v[j];
+                ep.out[o] = x;
+                ep.xb[o] = __float2bfloat16_rn(x);
+            }
+            v[j] = x * x;
+        }
+        warp_reduce_scatter32(v, lane);
+        sm.red[quarter * 32 + lane] = v[0];
         named_bar(1, 128);
-        if constexpr (EPI == EPI_QKV) {
-            const int qd = ep.H * ep.hd;
-            const int part = row / qd;
-            const int f = row - part * qd;
-            const int hh = f / ep.hd;
-            const int i = f - hh * ep.hd;
-            const int half = ep.hd >> 1;
-            const int partner = rt ^ half;
-            const int ii = i & (half - 1);
+        if (ew == 0) {
+            const int col = col0 + lane;
+            if (col < p.N)
+                ep.sq_out[static_cast<size_t>(mt) * p.N + col] =
+                    ((sm.red[lane] + sm.red[32 + lane]) + sm.red[64 + lane]) + sm.red[96 + lane];
+        }
+        named_bar(1, 128);
+    } else if constexpr (EPI == EPI_QKV) {
+        const int qd = ep.H * ep.hd;
+        const int part = row / qd;
+        const int f = row - part * qd;
+        const int hh = f / ep.hd;
+        const int pp = f - hh * ep.hd;          // physical row inside the head
+        const int half = ep.hd >> 1;
+        const int jr = pp >> 1;                 // rotation pair index
+        const int i = jr + (pp & 1) * half;     // logical feature
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            const float xp = __shfl_xor_sync(0xffffffffu, v[j], 1);
+            const int col = col0 + j;
+            if (col >= p.N) continue;
+            const int b = col / ep.T;
+            const int t = col - b * ep.T;
+            const int pos = ep.seq_kv[b] + t;
+            if (pos < 0 || pos >= ep.cap) {
+                atomicOr(status, kStatusBadIndex);
+                continue;
+            }
+            float x = v[j];
+            if (part < 2) {
+                const float2 cs = *reinterpret_cast<const float2*>(ep.rope + (static_cast<size_t>(pos) * half + jr) * 2);
+                x = (pp & 1) ? (x * cs.x + xp * cs.y) : (x * cs.x - xp * cs.y);
+            }
+            const __nv_bfloat16 y = __float2bfloat16_rn(x);
+            if (part == 0) {
+                ep.q[((static_cast<size_t>(b) * ep.H + hh) * ep.T + t) * ep.hd + i] = y;
+            } else {
+                __nv_bfloat16* c = part == 1 ? ep.kc : ep.vc;
+                c[((static_cast<size_t>(b) * ep.H + hh) * ep.cap + pos) * ep.hd + i] = y;
+            }
+        }
+    } else if constexpr (EPI == EPI_SWIGLU) {
+        const int f = mt * 64 + (rt >> 1);
+        const bool gate = (rt & 1) == 0;
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            const float u = __shfl_xor_sync(0xffffffffu, v[j], 1);
+            const int col = col0 + j;
+            if (gate && f < ep.F && col < p.N) {
+                const float g = v[j];
+                const float s = g / (1.0f + expf(-g));
+                ep.h[static_cast<size_t>(col) * ep.F + f] = __float2bfloat16_rn(s * u);
+            }
+        }
+    } else if constexpr (EPI == EPI_LMHEAD) {
+        if (ep.logits && row < ep.V) {
             for (int j = 0; j < 32; ++j) {
-                int col = col0 + j;
-                if (col >= p.N) break;
-                int b = col / ep.T;
-                int t = col - b * ep.T;
-                int pos = ep.seq_kv[b] + t;
-                if (pos < 0 || pos >= ep.cap) {
-                    atomicOr(status, kStatusBadIndex);
-                    continue;
-                }
-                float x = v[j];
-                if (part < 2) {
-                    float xp = stg[partner * kStageLd + j];
-                    const float* cs = ep.rope + (static_cast<size_t>(pos) * half + ii) * 2;
-                    x = (i < half) ? (x * cs[0] - xp * cs[1]) : (x * cs[0] + xp * cs[1]);
-                }
-                __nv_bfloat16 y = __float2bfloat16_rn(x);
-                if (part == 0) {
-                    ep.q[((static_cast<size_t>(b) * ep.H + hh) * ep.T + t) * ep.hd + i] = y;
-                } else {
-                    __nv_bfloat16* c = part == 1 ? ep.kc : ep.vc;
-                    c[((static_cast<size_t>(b) * ep.H + hh) * ep.cap + pos) * ep.hd + i] = y;
-                }
+                const int col = col0 + j;
+                if (col < p.N) ep.logits[static_cast<size_t>(col) * ep.V + row] = v[j];
             }
-        } else if constexpr (EPI == EPI_SWIGLU) {
-            if (rt < 64) {
-                const int f = mt * 64 + rt;
-                if (f < ep.F) {
-                    for (int j = 0; j < 32; ++j) {
-                        int col = col0 + j;
-                        if (col >= p.N) break;
-                        float g = v[j];
-                        float u = stg[(rt + 64) * kStageLd + j];
-                        float s = g / (1.0f + expf(-g));
-                        ep.h[static_cast<size_t>(col) * ep.F + f] = __float2bfloat16_rn(s * u);
-                    }
-                }
-            }
-        } else if constexpr (EPI == EPI_LMHEAD) {
-            if (ep.logits && row < ep.V) {
-                for (int j = 0; j < 32; ++j) {
-                    int col = col0 + j;
-                    if (col < p.N) ep.logits[static_cast<size_t>(col) * ep.V + row] = v[j];
-                }
-            }
-            for (int jj = ew; jj < 32; jj += 4) {
-                int col = col0 + jj;
+        }
+#pragma unroll
+        for (int hlf = 0; hlf < 2; ++hlf) {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) sm.stg[rt * kStageLd + j] = v[hlf * 16 + j];
+            named_bar(1, 128);
+            for (int jj = ew; jj < 16; jj += 4) {
+                const int col = col0 + hlf * 16 + jj;
                 if (col >= p.N) break;
                 float m = -INFINITY;
                 int idx = INT_MAX;
@@ -124,17 +190,23 @@ __device__ __forceinline__ void epilogue_chunk(const EpiArgs& ep, const GemmPlan
                 bool ok[4];
 #pragma unroll
                 for (int r = 0; r < 4; ++r) {
-                    int rr = lane + 32 * r;
-                    int id = mt * kBM + rr;
+                    const int rr = lane + 32 * r;
+                    const int id = mt * kBM + rr;
                     ok[r] = id < ep.V && id != ep.mask_id;
-                    z[r] = stg[rr * kStageLd + jj];
-                    if (ok[r] && z[r] > m) { m = z[r]; idx = id; }
+                    z[r] = sm.stg[rr * kStageLd + jj];
+                    if (ok[r] && z[r] > m) {
+                        m = z[r];
+                        idx = id;
+                    }
                 }
 #pragma unroll
                 for (int off = 16; off > 0; off >>= 1) {
-                    float om = __shfl_xor_sync(0xffffffffu, m, off);
-                    int oi = __shfl_xor_sync(0xffffffffu, idx, off);
-                    if (om > m || (om == m && oi < idx)) { m = om; idx = oi; }
+                    const float om = __shfl_xor_sync(0xffffffffu, m, off);
+                    const int oi = __shfl_xor_sync(0xffffffffu, idx, off);
+                    if (om > m || (om == m && oi < idx)) {
+                        m = om;
+                        idx = oi;
+                    }
                 }
                 float s = 0.0f;
                 if (m != -INFINITY) {
@@ -145,16 +217,17 @@ __device__ __forceinline__ void epilogue_chunk(const EpiArgs& ep, const GemmPlan
 #pragma unroll
                 for (int off = 16; off > 0; off >>= 1) s += __shfl_down_sync(0xffffffffu, s, off);
                 if (lane == 0) {
-                    float* o = ep.lm_part + (static_cast<size_t>(mt) * p.N + col) * 3;
+                    float* o = ep.lm_part + (static_cast<size_t>(col) * p.m_tiles + mt) * 3;
                     o[0] = m;
                     o[1] = s;
                     o[2] = __int_as_float(idx);
-                    int cur = ep.cur_tok[col];
-                    if (cur >= mt * kBM && cur < mt * kBM + kBM) ep.zcur[col] = stg[(cur - mt * kBM) * kStageLd + jj];
+                    const int cur = ep.cur_tok[col];
+                    if (cur >= mt * kBM && cur < mt * kBM + kBM)
+                        ep.zcur[col] = sm.stg[(cur - mt * kBM) * kStageLd + jj];
                 }
             }
+            named_bar(1, 128);
         }
-        named_bar(1, 128);
     }
 }
 
@@ -169,8 +242,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t b_bytes = static_cast<uint32_t>(p.ntile) * kBK * 2;
     uint8_t* sA = smem;
     uint8_t* sB = sA + static_cast<size_t>(S) * kABytes;
-    float* stg = reinterpret_cast<float*>(sB + static_cast<size_t>(S) * b_bytes);
-    uint64_t* full = reinterpret_cast<uint64_t*>(stg + kBM * kStageLd);
+    float* tail = reinterpret_cast<float*>(sB + static_cast<size_t>(S) * b_bytes);
+    EpiSmem esm;
+    esm.rs = tail;
+    esm.red = tail + 32;
+    esm.stg = tail + 32 + 128;
+    float* after = esm.stg + (EPI == EPI_LMHEAD ? kBM * kStageLd : 0);
+    uint64_t* full = reinterpret_cast<uint64_t*>(after);
     uint64_t* empty = full + S;
     uint64_t* tfull = empty + S;
     uint64_t* tempty = tfull + 2;
@@ -186,6 +264,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const long long it1 = range_begin(blockIdx.x + 1, p.total, G);
 
     if (threadIdx.x == 0) {
+        pdl_launch_dependents();
         for (int s = 0; s < S; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
@@ -221,7 +300,30 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t phase = 0;
             uint32_t pending = 0;   // stages with a load in flight
             uint32_t pend_par = 0;  // parity of that load's phase
-            for (long long it = it0; it < it1; ++it) {
+            // weights of the first stages: no earlier kernel writes them, so they stream
+            // before the dependency wait
+            const long long npre = (it1 - it0) < S ? (it1 - it0) : S;
+            for (long long q = 0; q < npre; ++q) {
+                const long long it = it0 + q;
+                const long long tile = it / p.kb;
+                const int k = static_cast<int>(it - tile * p.kb);
+                const int mt = static_cast<int>(tile / p.n_tiles);
+                mbar_arrive_expect_tx(&full[q], kABytes + b_bytes);
+                tma_load_2d(sA + static_cast<size_t>(q) * kABytes, &tmW, k * kBK, mt * kBM, &full[q], pol_w);
+            }
+            pdl_wait();
+            for (long long q = 0; q < npre; ++q) {
+                const long long it = it0 + q;
+                const long long tile = it / p.kb;
+                const int k = static_cast<int>(it - tile * p.kb);
+                const int mt = static_cast<int>(tile / p.n_tiles);
+                const int nt = static_cast<int>(tile - static_cast<long long>(mt) * p.n_tiles);
+                tma_load_2d(sB + static_cast<size_t>(q) * b_bytes, &tmX, k * kBK, nt * p.ntile, &full[q], pol_x);
+                pending |= 1u << q;
+            }
+            stage = static_cast<int>(npre % S);
+            phase = npre == S ? 1u : 0u;
+            for (long long it = it0 + npre; it < it1; ++it) {
                 const long long tile = it / p.kb;
                 const int k = static_cast<int>(it - tile * p.kb);
                 const int mt = static_cast<int>(tile / p.n_tiles);
@@ -242,7 +344,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // let every copy already issued land before the CTA's shared memory is released
                 for (int s = 0; s < S; ++s) {
                     if (!(pending >> s & 1u)) continue;
-                    unsigned long long t0 = global_ns();
+                    const unsigned long long t0 = global_ns();
                     while (!mbar_try_wait(&full[s], (pend_par >> s) & 1u) && global_ns() - t0 < kWaitLimitNs) {
                     }
                 }
@@ -297,13 +399,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (*s_abort && issued) {
                 // wait for the tensor cores before the accumulator memory is released
                 umma_commit(drain);
-                unsigned long long t0 = global_ns();
+                const unsigned long long t0 = global_ns();
                 while (!mbar_try_wait(drain, 0) && global_ns() - t0 < kWaitLimitNs) {
                 }
             }
         }
     } else {
         // ---------------------------------------------------------- epilogue
+        pdl_wait();
         const int ew = warp - 2;                 // 0..3
         const int quarter = warp & 3;            // TMEM lane quarter this warp may access
         const int rt = quarter * 32 + lane;      // row within the 128-row tile
@@ -331,7 +434,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int c = 0; c < nchunks; ++c) {
                 tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);
                 if (whole) {
-                    epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, stg, ew, lane, status);
+                    epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
                 } else {
 #pragma unroll
                     for (int j = 0; j < 32; ++j) my_part[static_cast<size_t>(c * 32 + j) * kBM + rt] = v[j];
@@ -370,7 +473,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                             for (int j = 0; j < 32; ++j) v[j] += __ldcg(pp + static_cast<size_t>(j) * kBM);
                         }
-                        epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, stg, ew, lane, status);
+                        epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
                     }
                 }
             }
@@ -394,13 +497,13 @@ static int pow2ceil(int x) {
     return p;
 }
 
-GemmPlan gemm_plan(int M, int N, int K, int grid_max) {
+GemmPlan gemm_plan(int M, int N, int K, int grid_max, int epi) {
     GemmPlan p{};
     p.M = M;
     p.N = N;
     p.K = K;
     p.n_tiles = (N + 255) / 256;
-    int per = (N + p.n_tiles - 1) / p.n_tiles;
+    const int per = (N + p.n_tiles - 1) / p.n_tiles;
     p.ntile = ((per + 31) / 32) * 32;
     p.m_tiles = (M + kBM - 1) / kBM;
     p.kb = (K + kBK - 1) / kBK;
@@ -409,12 +512,16 @@ GemmPlan gemm_plan(int M, int N, int K, int grid_max) {
     if (p.grid < 1) p.grid = 1;
     p.acc_cols = pow2ceil(p.ntile);
     p.tmem_cols = 2 * p.acc_cols;
-    const int fixed = 1024 + kBM * kStageLd * 4 + 64 * 8 + 64;
+    const int staging = epi == EPI_LMHEAD ? kBM * kStageLd * 4 : 0;
+    const int fixed = 1024 + (32 + 128) * 4 + staging + 64 * 8 + 64;
     const int stage_bytes = static_cast<int>(kABytes) + p.ntile * kBK * 2;
-    int st = (227 * 1024 - fixed) / stage_bytes;
+    const int budget = p.ntile <= 96 ? kStreamSmem : kFullSmem;
+    int st = (budget - fixed) / stage_bytes;
     if (st > 16) st = 16;
+    if (st < 2) st = 2;
     p.stages = st;
     p.smem = static_cast<size_t>(fixed) + static_cast<size_t>(st) * stage_bytes;
+    p.pdl = true;
     return p;
 }
 
@@ -449,17 +556,10 @@ bool make_tmap_bf16(CUtensorMap* tm, const void* ptr, uint64_t rows, uint64_t co
     return r == CUDA_SUCCESS;
 }
 
-template <int EPI>
-static cudaError_t launch_t(const GemmPlan& p, const CUtensorMap& tmW, const CUtensorMap& tmX, const EpiArgs& ep,
-                            const Scratch& scr, int* status, cudaStream_t st) {
-    k_gemm<EPI><<<p.grid, kThreads, p.smem, st>>>(tmW, tmX, p, ep, scr.partials, scr.counters, status);
-    return cudaGetLastError();
-}
-
 cudaError_t gemm_init_attrs() {
     cudaError_t e = cudaSuccess;
     auto set = [&](const void* f) {
-        if (e == cudaSuccess) e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+        if (e == cudaSuccess) e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, kFullSmem);
     };
     set(reinterpret_cast<const void*>(k_gemm<EPI_F32>));
     set(reinterpret_cast<const void*>(k_gemm<EPI_RESID>));
@@ -467,6 +567,13 @@ cudaError_t gemm_init_attrs() {
     set(reinterpret_cast<const void*>(k_gemm<EPI_SWIGLU>));
     set(reinterpret_cast<const void*>(k_gemm<EPI_LMHEAD>));
     return e;
+}
+
+template <int EPI>
+static cudaError_t launch_t(const GemmPlan& p, const CUtensorMap& tmW, const CUtensorMap& tmX, const EpiArgs& ep,
+                            const Scratch& scr, int* status, cudaStream_t st) {
+    return launch_k(k_gemm<EPI>, dim3(p.grid), dim3(kThreads), p.smem, st, p.pdl, tmW, tmX, p, ep, scr.partials,
+                    scr.counters, status);
 }
 
 cudaError_t gemm_launch(int epi, const GemmPlan& p, const CUtensorMap& tmW, const CUtensorMap& tmX,
@@ -483,5 +590,9 @@ cudaError_t gemm_launch(int epi, const GemmPlan& p, const CUtensorMap& tmW, cons
     }
     return cudaErrorInvalidValue;
 }
+
+static bool g_pdl = true;
+void set_pdl(bool on) { g_pdl = on; }
+bool pdl_enabled() { return g_pdl; }
 
 }  // namespace dllm

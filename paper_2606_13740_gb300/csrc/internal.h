@@ -7,6 +7,8 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include <utility>
+
 namespace dllm {
 
 constexpr int kMaxBlock = 4096;
@@ -21,18 +23,28 @@ enum EpiKind { EPI_F32 = 0, EPI_RESID = 1, EPI_QKV = 2, EPI_SWIGLU = 3, EPI_LMHE
 struct EpiArgs {
     float* out;          // EPI_F32: D[n][m] (ld = ld_out); EPI_RESID: residual x[n][m] += D
     int ld_out;
-    // EPI_QKV: rows [0,qd) q, [qd,2qd) k, [2qd,3qd) v; rotate-half RoPE on q, k
+    // EPI_RESID also writes xb = bf16(x) [n][m] (the next projection's operand) and
+    // sq_out[m_tile][n] = sum over the tile's 128 rows of x^2 (RMSNorm statistics)
+    __nv_bfloat16* xb;
+    float* sq_out;
+    // QKV / SWIGLU / LMHEAD: per-token RMSNorm scale rsqrt(sum_t sq_in[t][n] / norm_dim + eps)
+    // applied to the accumulators (the operand is bf16 of the un-normalised x); null = none
+    const float* sq_in;
+    int n_sq, norm_dim;
+    float eps;
+    // EPI_QKV: rows [0,qd) q, [qd,2qd) k, [2qd,3qd) v; rotate-half RoPE on q, k.  Inside
+    // each head the rows are interleaved: row 2j is feature j, row 2j+1 feature j + hd/2
     __nv_bfloat16* q;    // [B][H][T][hd]
     __nv_bfloat16* kc;   // layer's K cache base: [B][H][cap][hd]
     __nv_bfloat16* vc;
     const float* rope;   // [cap][hd/2][2] (cos, sin)
     const int* seq_kv;   // per-sequence first window position (kv_len)
     int T, H, hd, cap;
-    // EPI_SWIGLU: tile k rows 0..63 gate(64k..), rows 64..127 up(64k..)
+    // EPI_SWIGLU: tile k row 2f is gate feature 64k+f, row 2f+1 the matching up row
     __nv_bfloat16* h;    // [N][F]
     int F;
     // EPI_LMHEAD
-    float* lm_part;      // [m_tiles][N][3]: max, sum exp(z - max), argmax (as float bits)
+    float* lm_part;      // [N][m_tiles][3]: max, sum exp(z - max), argmax (as float bits)
     float* zcur;         // [N]: logit of the current token id
     const int* cur_tok;  // [N]
     float* logits;       // [N][V] or null
@@ -45,6 +57,7 @@ struct GemmPlan {
     int m_tiles, n_tiles, kb;
     long long total;     // m_tiles * n_tiles * kb iterations of 64-wide K blocks
     int grid;            // CTAs (stream-K partition of the iterations)
+    bool pdl;            // launch with programmatic dependent launch (the step's chain)
     int stages;
     int acc_cols;        // TMEM columns per accumulator buffer
     int tmem_cols;       // allocation (power of two)
@@ -58,34 +71,64 @@ struct Scratch {
     int counter_len;
 };
 
-GemmPlan gemm_plan(int M, int N, int K, int grid_max);
+// Shared memory budget: at most 96 tokens per tile the kernel is a weight stream and keeps
+// to 113 KB so that the next projection's CTA fits beside it on the SM (programmatic
+// dependent launch prefetches its weights while this one drains); larger tiles use 227 KB.
+GemmPlan gemm_plan(int M, int N, int K, int grid_max, int epi);
 bool make_tmap_bf16(CUtensorMap* tm, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows);
 cudaError_t gemm_launch(int epi, const GemmPlan& p, const CUtensorMap& tmW, const CUtensorMap& tmX,
                         const EpiArgs& ep, const Scratch& scr, int* status, cudaStream_t st);
 
+// ---------------------------------------------------------------- launches
+// Every kernel is launched with programmatic stream serialisation (PDL): it may start
+// while its predecessor drains, and waits (griddepcontrol.wait) before touching data the
+// predecessor writes.  set_pdl(false) launches them plainly.
+void set_pdl(bool on);
+bool pdl_enabled();
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_k(void (*k)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, bool pdl,
+                            Args&&... args) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = (pdl && pdl_enabled()) ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, k, std::forward<Args>(args)...);
+}
+
 // ---------------------------------------------------------------- other kernels
 cudaError_t launch_init_weight(__nv_bfloat16* dst, int mode, int rows_phys, int cols, int logical_rows,
-                               uint64_t seed, uint64_t tid0, int qd, cudaStream_t st);
+                               uint64_t seed, uint64_t tid0, int qd, int hd, cudaStream_t st);
 cudaError_t launch_init_rope(float* rope, int cap, int hd, double base, cudaStream_t st);
 cudaError_t launch_init_kv_random(__nv_bfloat16* cache, int B, int H, int hd, int cap, int P, int layer,
                                   int which, int L, uint64_t seed, cudaStream_t st);
-cudaError_t launch_embed_norm(const int* tok, int tok_ld, const int* seq_kv, const __nv_bfloat16* emb,
-                              float* x, __nv_bfloat16* xn, int B, int T, int d, float eps, cudaStream_t st);
-cudaError_t launch_rmsnorm(const float* x, __nv_bfloat16* xn, int ntok, int d, float eps, cudaStream_t st);
-// Attention split plan: CTAs (split, head, sequence x 64-query tile), each
-// over `chunk` keys; nsplit > 1 adds a combine pass over fp32 partials
-// part_o [B][H][nsplit][T][hd] and part_ml [B][H][nsplit][T][2].
+// x = embedding rows of the window's ids (fp32), xb = bf16(x), sq[d/128][N] = per-128-feature
+// sums of x^2, cur[N] = the ids (for the LM head's current-token probability).
+cudaError_t launch_embed(const int* tok, int tok_ld, const int* seq_kv, const __nv_bfloat16* emb, float* x,
+                         __nv_bfloat16* xb, float* sq, int* cur, int B, int T, int d, cudaStream_t st);
+// The kernels below are launched with PDL when `pdl` (inside the context's step chain); the
+// single-kernel entry points pass false because their inputs may come from foreign kernels.
+// Attention split plan: CTAs (split, head, sequence x 64-query tile), each over `chunk`
+// keys; with nsplit > 1 the splits leave fp32 partials part_o [B][H][nsplit][T][hd] and
+// part_ml [B][H][nsplit][T][2] and the last CTA of each (sequence, head, query tile) to
+// finish (ticket in counters [B][H][qtiles], zero between launches) merges them in order.
 struct AttnPlan {
     int qtiles, chunk, nsplit;
 };
 AttnPlan attn_plan(int B, int T, int H, int max_keys, int sms);
 cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
-                             const int* seq_kv, float* part_o, float* part_ml, __nv_bfloat16* out, int B, int T,
-                             int H, int hd, int cap, const AttnPlan& a, cudaStream_t st);
+                             const int* seq_kv, float* part_o, float* part_ml, int* counters,
+                             __nv_bfloat16* out, int B, int T, int H, int hd, int cap, const AttnPlan& a,
+                             cudaStream_t st, bool pdl = true);
 cudaError_t launch_lmhead_reduce(const float* lm_part, const float* zcur, const int* cur_tok, int m_tiles,
-                                 int N, int mask_id, int* x0, float* conf, float* tokconf, cudaStream_t st);
-cudaError_t launch_gather_cur(const int* tok, int tok_ld, const int* seq_kv, int* cur, int B, int T,
-                              cudaStream_t st);
+                                 int N, int mask_id, int* x0, float* conf, float* tokconf, cudaStream_t st,
+                                 bool pdl = true);
 
 // Commit pass.  Per sequence b: state arrays at tok + b*ld, st + b*ld; the
 // window starts at seq_kv[b] (prefix cache on) or 0 (off); plan[b] holds
@@ -104,7 +147,7 @@ struct CommitArgs {
     int S, remask_max, spec_blocks, block_len;
     float theta_remask, theta_stable;
 };
-cudaError_t launch_commit(const CommitArgs& a, cudaStream_t st);
+cudaError_t launch_commit(const CommitArgs& a, cudaStream_t st, bool pdl = true);
 
 cudaError_t launch_begin_block(int* tok, uint8_t* st, int* snap_tok, uint8_t* snap_st, int ld, int n_pos, int* plan,
                                int B, int c0, int c1, cudaStream_t stream);

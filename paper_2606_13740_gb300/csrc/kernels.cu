@@ -32,11 +32,13 @@ __device__ __forceinline__ float gen_value(uint64_t key, uint64_t i, double sigm
 
 // mode 0: plain (physical row = logical row of tensor tid0, zero rows past
 //         logical_rows);
-// mode 1: fused QKV (rows [0,qd) tensor tid0, [qd,2qd) tid0+1, [2qd,3qd) tid0+2);
-// mode 2: fused gate/up: 128-row tile k = gate rows 64k..64k+63 (tensor tid0),
-//         then up rows 64k..64k+63 (tensor tid0+1), zero past logical_rows.
+// mode 1: fused QKV: rows [0,qd) tensor tid0 (q), [qd,2qd) tid0+1 (k), [2qd,3qd) tid0+2 (v);
+//         inside each head of hd rows, physical row 2j holds feature j and row 2j+1 feature
+//         j + hd/2 (the rotate-half RoPE pair sits in adjacent TMEM lanes);
+// mode 2: fused gate/up: 128-row tile k, physical row 2f = gate row 64k+f (tensor tid0),
+//         row 2f+1 = up row 64k+f (tensor tid0+1); zero past logical_rows.
 __global__ void k_init_weight(__nv_bfloat16* dst, int mode, int rows, int cols, int logical_rows, uint64_t seed,
-                              uint64_t tid0, int qd) {
+                              uint64_t tid0, int qd, int hd) {
     const size_t n = static_cast<size_t>(rows) * cols;
     for (size_t e = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; e < n;
          e += static_cast<size_t>(gridDim.x) * blockDim.x) {
@@ -45,12 +47,15 @@ __global__ void k_init_weight(__nv_bfloat16* dst, int mode, int rows, int cols, 
         uint64_t tid = tid0;
         int lr = r;
         if (mode == 1) {
-            tid = tid0 + r / qd;
-            lr = r % qd;
+            const int part = r / qd, f = r % qd;
+            const int hh = f / hd, pp = f % hd;
+            tid = tid0 + part;
+            lr = hh * hd + (pp >> 1) + (pp & 1) * (hd >> 1);
+            if (part > 2) lr = logical_rows;  // padding rows
         } else if (mode == 2) {
-            int tile = r >> 7, w = r & 127;
-            tid = tid0 + (w >= 64 ? 1 : 0);
-            lr = tile * 64 + (w & 63);
+            const int tile = r >> 7, w = r & 127;
+            tid = tid0 + (w & 1);
+            lr = tile * 64 + (w >> 1);
         }
         float v = 0.0f;
         if (lr < logical_rows) {
@@ -62,10 +67,10 @@ __global__ void k_init_weight(__nv_bfloat16* dst, int mode, int rows, int cols, 
 }
 
 cudaError_t launch_init_weight(__nv_bfloat16* dst, int mode, int rows_phys, int cols, int logical_rows,
-                               uint64_t seed, uint64_t tid0, int qd, cudaStream_t st) {
+                               uint64_t seed, uint64_t tid0, int qd, int hd, cudaStream_t st) {
     size_t n = static_cast<size_t>(rows_phys) * cols;
     int blocks = static_cast<int>((n + 255) / 256 < 65536 ? (n + 255) / 256 : 65536);
-    k_init_weight<<<blocks, 256, 0, st>>>(dst, mode, rows_phys, cols, logical_rows, seed, tid0, qd);
+    k_init_weight<<<blocks, 256, 0, st>>>(dst, mode, rows_phys, cols, logical_rows, seed, tid0, qd, hd);
     return cudaGetLastError();
 }
 
@@ -119,73 +124,42 @@ cudaError_t launch_init_rope(float* rope, int cap, int hd, double base, cudaStre
     return cudaGetLastError();
 }
 
-// ------------------------------------------------------------------ norms
-// Deterministic block sum (fixed shuffle tree, then warp 0 over warp sums).
-__device__ __forceinline__ float block_sum(float v, float* red) {
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
-    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
-    if (l == 0) red[w] = v;
-    __syncthreads();
-    if (w == 0) {
-        v = l < (blockDim.x >> 5) ? red[l] : 0.0f;
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
-        if (l == 0) red[32] = v;
-    }
-    __syncthreads();
-    return red[32];
-}
-
-// One CTA per token: x (fp32 residual) = embedding row; xn = bf16(x / rms(x)).
-// The RMSNorm gain is one and is not stored.
-__global__ void __launch_bounds__(256) k_embed_norm(const int* tok, int tok_ld, const int* seq_kv,
-                                                    const __nv_bfloat16* emb, float* x, __nv_bfloat16* xn, int T,
-                                                    int d, float eps) {
-    __shared__ float red[33];
+// ------------------------------------------------------------------ embedding
+// One CTA (8 warps) per token: x = embedding row (fp32 residual), xb = bf16(x)
+// (the QKV projection's operand), sq[c][token] = sum of x^2 over features
+// [128c, 128c+128) (the first RMSNorm's statistics, merged in the consumer),
+// cur[token] = the id (for the LM head's current-token probability).
+__global__ void __launch_bounds__(256) k_embed(const int* tok, int tok_ld, const int* seq_kv,
+                                               const __nv_bfloat16* emb, float* x, __nv_bfloat16* xb, float* sq,
+                                               int* cur, int T, int N, int d) {
+    pdl_wait();
+    pdl_launch_dependents();
     const int j = blockIdx.x;
     const int b = j / T, t = j - b * T;
     const int id = tok[static_cast<size_t>(b) * tok_ld + seq_kv[b] + t];
+    if (threadIdx.x == 0) cur[j] = id;
     const __nv_bfloat16* e = emb + static_cast<size_t>(id) * d;
-    float* xr = x + static_cast<size_t>(j) * d;
-    float ss = 0.0f;
-    for (int i = threadIdx.x; i < d; i += blockDim.x) {
-        float v = __bfloat162float(e[i]);
-        xr[i] = v;
-        ss += v * v;
-    }
-    float r = rsqrtf(block_sum(ss, red) / d + eps);
-    for (int i = threadIdx.x; i < d; i += blockDim.x) xn[static_cast<size_t>(j) * d + i] = __float2bfloat16_rn(xr[i] * r);
-}
-
-cudaError_t launch_embed_norm(const int* tok, int tok_ld, const int* seq_kv, const __nv_bfloat16* emb, float* x,
-                              __nv_bfloat16* xn, int B, int T, int d, float eps, cudaStream_t st) {
-    k_embed_norm<<<B * T, 256, 0, st>>>(tok, tok_ld, seq_kv, emb, x, xn, T, d, eps);
-    return cudaGetLastError();
-}
-
-__global__ void __launch_bounds__(256) k_rmsnorm(const float* x, __nv_bfloat16* xn, int d, float eps) {
-    __shared__ float red[33];
-    const float* xr = x + static_cast<size_t>(blockIdx.x) * d;
-    float ss = 0.0f;
-    for (int i = threadIdx.x * 4; i < d; i += blockDim.x * 4) {
-        float4 v = *reinterpret_cast<const float4*>(xr + i);
-        ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
-    }
-    float r = rsqrtf(block_sum(ss, red) / d + eps);
-    __nv_bfloat16* o = xn + static_cast<size_t>(blockIdx.x) * d;
-    for (int i = threadIdx.x * 4; i < d; i += blockDim.x * 4) {
-        float4 v = *reinterpret_cast<const float4*>(xr + i);
-        __nv_bfloat162 a = __floats2bfloat162_rn(v.x * r, v.y * r);
-        __nv_bfloat162 c = __floats2bfloat162_rn(v.z * r, v.w * r);
-        *reinterpret_cast<__nv_bfloat162*>(o + i) = a;
-        *reinterpret_cast<__nv_bfloat162*>(o + i + 2) = c;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int c = warp; c * 128 < d; c += blockDim.x >> 5) {
+        float ss = 0.0f;
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            const int i = c * 128 + r * 32 + lane;
+            const __nv_bfloat16 h = e[i];
+            const float v = __bfloat162float(h);
+            x[static_cast<size_t>(j) * d + i] = v;
+            xb[static_cast<size_t>(j) * d + i] = h;
+            ss += v * v;
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) ss += __shfl_down_sync(0xffffffffu, ss, off);
+        if (lane == 0) sq[static_cast<size_t>(c) * N + j] = ss;
     }
 }
 
-cudaError_t launch_rmsnorm(const float* x, __nv_bfloat16* xn, int ntok, int d, float eps, cudaStream_t st) {
-    k_rmsnorm<<<ntok, 256, 0, st>>>(x, xn, d, eps);
-    return cudaGetLastError();
+cudaError_t launch_embed(const int* tok, int tok_ld, const int* seq_kv, const __nv_bfloat16* emb, float* x,
+                         __nv_bfloat16* xb, float* sq, int* cur, int B, int T, int d, cudaStream_t st) {
+    return launch_k(k_embed, dim3(B * T), dim3(256), 0, st, true, tok, tok_ld, seq_kv, emb, x, xb, sq, cur, T, B * T, d);
 }
 
 // ------------------------------------------------------------------ attention
@@ -193,8 +167,9 @@ cudaError_t launch_rmsnorm(const float* x, __nv_bfloat16* xn, int ntok, int d, f
 // [0, kv_len + T) of the KV cache (cached prefix, then the window's own keys
 // written by the QKV epilogue), flash style with split-KV: CTA (split, head,
 // sequence x 64-query tile) covers `chunk` keys in 64-key sub-blocks with an
-// online softmax on bf16 mma.sync tiles, writing unnormalised partials that
-// k_attn_combine merges (or the final output when there is one split).
+// online softmax on bf16 mma.sync tiles.  With one split it writes the output;
+// otherwise it leaves unnormalised partials and the last CTA of the (sequence,
+// head, query tile) to finish merges all splits in split order.
 constexpr int kAQ = 64;
 constexpr int kAK = 64;
 
@@ -238,9 +213,12 @@ template <int HD>
 __global__ void __launch_bounds__(128) k_attn(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ kc,
                                               const __nv_bfloat16* __restrict__ vc, const int* __restrict__ seq_kv,
                                               float* __restrict__ part_o, float* __restrict__ part_ml,
-                                              __nv_bfloat16* __restrict__ out, int T, int H, int cap, int chunk,
-                                              int nsplit, int qtiles) {
+                                              int* __restrict__ counters, __nv_bfloat16* __restrict__ out, int T,
+                                              int H, int cap, int chunk, int nsplit, int qtiles) {
     extern __shared__ __align__(128) uint8_t smem_attn[];
+    __shared__ int s_last;
+    pdl_wait();
+    pdl_launch_dependents();
     __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem_attn);
     __nv_bfloat16* sK = sQ + kAQ * HD;       // [2][kAK][HD]
     __nv_bfloat16* sV = sK + 2 * kAK * HD;   // [2][kAK][HD]
@@ -414,42 +392,36 @@ __global__ void __launch_bounds__(128) k_attn(const __nv_bfloat16* __restrict__ 
             if (r0 < nq) *reinterpret_cast<float2*>(part_ml + (base + r0) * 2) = make_float2(m0, l0);
             if (r1 < nq) *reinterpret_cast<float2*>(part_ml + (base + r1) * 2) = make_float2(m1, l1);
         }
+        // the last split of this (sequence, head, query tile) to finish merges them all
+        __threadfence();
+        __syncthreads();
+        const int ns = (NK + chunk - 1) / chunk;
+        if (tid == 0) {
+            int* ctr = counters + (static_cast<size_t>(b) * H + h) * qtiles + qt;
+            const int prev = atomicAdd(ctr, 1);
+            s_last = prev == ns - 1;
+            if (s_last) *ctr = 0;
+        }
+        __syncthreads();
+        if (s_last) {
+            __threadfence();
+            const size_t sb = (static_cast<size_t>(b) * H + h) * nsplit * T + q0;
+            const int qd = H * HD;
+            for (int e = tid; e < nq * HD; e += 128) {
+                const int r = e / HD, i = e - r * HD;
+                float M = -INFINITY;
+                for (int sp = 0; sp < ns; ++sp) M = fmaxf(M, __ldcg(part_ml + (sb + static_cast<size_t>(sp) * T + r) * 2));
+                float L = 0.0f, acc = 0.0f;
+                for (int sp = 0; sp < ns; ++sp) {
+                    const size_t row = sb + static_cast<size_t>(sp) * T + r;
+                    const float w = exp2f(__ldcg(part_ml + row * 2) - M);
+                    L += w * __ldcg(part_ml + row * 2 + 1);
+                    acc += w * __ldcg(part_o + row * HD + i);
+                }
+                out[(static_cast<size_t>(b) * T + q0 + r) * qd + h * HD + i] = __float2bfloat16_rn(acc / L);
+            }
+        }
     }
-}
-
-// One warp per (sequence, head, query): merge the splits in order.
-template <int HD>
-__global__ void __launch_bounds__(128) k_attn_combine(const float* __restrict__ part_o, const float* __restrict__ part_ml,
-                                                      const int* __restrict__ seq_kv, __nv_bfloat16* __restrict__ out,
-                                                      int B, int T, int H, int chunk, int nsplit_alloc) {
-    const int wid = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int lane = threadIdx.x & 31;
-    if (wid >= B * H * T) return;
-    const int t = wid % T;
-    const int h = (wid / T) % H;
-    const int b = wid / (T * H);
-    const int NK = seq_kv[b] + T;
-    const int ns = (NK + chunk - 1) / chunk;
-    const size_t base = (static_cast<size_t>(b) * H + h) * nsplit_alloc * T + t;
-    float M = -INFINITY;
-    for (int s = 0; s < ns; ++s) M = fmaxf(M, part_ml[(base + static_cast<size_t>(s) * T) * 2]);
-    constexpr int PER = HD / 32;
-    float acc[PER];
-#pragma unroll
-    for (int i = 0; i < PER; ++i) acc[i] = 0.0f;
-    float L = 0.0f;
-    for (int s = 0; s < ns; ++s) {
-        size_t row = base + static_cast<size_t>(s) * T;
-        float w = exp2f(part_ml[row * 2] - M);
-        L += w * part_ml[row * 2 + 1];
-#pragma unroll
-        for (int i = 0; i < PER; ++i) acc[i] += w * part_o[row * HD + lane + 32 * i];
-    }
-    const float inv = 1.0f / L;
-    const int qd = H * HD;
-#pragma unroll
-    for (int i = 0; i < PER; ++i)
-        out[(static_cast<size_t>(b) * T + t) * qd + h * HD + lane + 32 * i] = __float2bfloat16_rn(acc[i] * inv);
 }
 
 cudaError_t attn_init_attrs() {
@@ -470,25 +442,17 @@ AttnPlan attn_plan(int B, int T, int H, int max_keys, int sms) {
 }
 
 cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
-                             const int* seq_kv, float* part_o, float* part_ml, __nv_bfloat16* out, int B, int T, int H,
-                             int hd, int cap, const AttnPlan& a, cudaStream_t st) {
-    dim3 grid(a.nsplit, H, B * a.qtiles);
-    size_t smem = static_cast<size_t>(kAQ + 4 * kAK) * hd * 2;
-    const int cgrid = (B * H * T * 32 + 127) / 128;
-    if (hd == 128) {
-        k_attn<128><<<grid, 128, smem, st>>>(q, kc, vc, seq_kv, part_o, part_ml, out, T, H, cap, a.chunk, a.nsplit,
-                                              a.qtiles);
-        if (a.nsplit > 1)
-            k_attn_combine<128><<<cgrid, 128, 0, st>>>(part_o, part_ml, seq_kv, out, B, T, H, a.chunk, a.nsplit);
-    } else if (hd == 64) {
-        k_attn<64><<<grid, 128, smem, st>>>(q, kc, vc, seq_kv, part_o, part_ml, out, T, H, cap, a.chunk, a.nsplit,
-                                             a.qtiles);
-        if (a.nsplit > 1)
-            k_attn_combine<64><<<cgrid, 128, 0, st>>>(part_o, part_ml, seq_kv, out, B, T, H, a.chunk, a.nsplit);
-    } else {
-        return cudaErrorInvalidValue;
-    }
-    return cudaGetLastError();
+                             const int* seq_kv, float* part_o, float* part_ml, int* counters, __nv_bfloat16* out, int B,
+                             int T, int H, int hd, int cap, const AttnPlan& a, cudaStream_t st, bool pdl) {
+    const dim3 grid(a.nsplit, H, B * a.qtiles);
+    const size_t smem = static_cast<size_t>(kAQ + 4 * kAK) * hd * 2;
+    if (hd == 128)
+        return launch_k(k_attn<128>, grid, dim3(128), smem, st, pdl, q, kc, vc, seq_kv, part_o, part_ml, counters, out, T,
+                        H, cap, a.chunk, a.nsplit, a.qtiles);
+    if (hd == 64)
+        return launch_k(k_attn<64>, grid, dim3(128), smem, st, pdl, q, kc, vc, seq_kv, part_o, part_ml, counters, out, T,
+                        H, cap, a.chunk, a.nsplit, a.qtiles);
+    return cudaErrorInvalidValue;
 }
 
 // ------------------------------------------------------------------ LM head
@@ -513,49 +477,49 @@ __device__ __forceinline__ void lse_merge(float& m, float& s, int& i, float m2, 
     }
 }
 
-__global__ void k_lmhead_reduce(const float* __restrict__ part, const float* __restrict__ zcur,
-                                const int* __restrict__ cur_tok, int m_tiles, int N, int mask_id, int* x0, float* conf,
-                                float* tokconf) {
+__global__ void __launch_bounds__(256) k_lmhead_reduce(const float* __restrict__ part, const float* __restrict__ zcur,
+                                                        const int* __restrict__ cur_tok, int m_tiles, int mask_id,
+                                                        int* x0, float* conf, float* tokconf) {
+    pdl_wait();
+    pdl_launch_dependents();
+    __shared__ float sm_m[8], sm_s[8];
+    __shared__ int sm_i[8];
     const int col = blockIdx.x;
-    const int lane = threadIdx.x;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     float m = -INFINITY, s = 0.0f;
     int idx = INT_MAX;
-    for (int t = lane; t < m_tiles; t += 32) {
-        const float* p = part + (static_cast<size_t>(t) * N + col) * 3;
-        lse_merge(m, s, idx, p[0], p[1], __float_as_int(p[2]));
-    }
+    const float* pc = part + static_cast<size_t>(col) * m_tiles * 3;
+    for (int t = threadIdx.x; t < m_tiles; t += blockDim.x)
+        lse_merge(m, s, idx, pc[t * 3], pc[t * 3 + 1], __float_as_int(pc[t * 3 + 2]));
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
-        float m2 = __shfl_down_sync(0xffffffffu, m, off);
-        float s2 = __shfl_down_sync(0xffffffffu, s, off);
-        int i2 = __shfl_down_sync(0xffffffffu, idx, off);
+        const float m2 = __shfl_down_sync(0xffffffffu, m, off);
+        const float s2 = __shfl_down_sync(0xffffffffu, s, off);
+        const int i2 = __shfl_down_sync(0xffffffffu, idx, off);
         if ((lane & (2 * off - 1)) == 0 && lane + off < 32) lse_merge(m, s, idx, m2, s2, i2);
     }
     if (lane == 0) {
+        sm_m[warp] = m;
+        sm_s[warp] = s;
+        sm_i[warp] = idx;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        m = sm_m[0];
+        s = sm_s[0];
+        idx = sm_i[0];
+        for (int w = 1; w < static_cast<int>(blockDim.x >> 5); ++w) lse_merge(m, s, idx, sm_m[w], sm_s[w], sm_i[w]);
         x0[col] = idx;
         conf[col] = 1.0f / s;
-        int cur = cur_tok[col];
+        const int cur = cur_tok[col];
         tokconf[col] = (cur >= 0 && cur != mask_id) ? expf(zcur[col] - m) / s : 0.0f;
     }
 }
 
 cudaError_t launch_lmhead_reduce(const float* lm_part, const float* zcur, const int* cur_tok, int m_tiles, int N,
-                                 int mask_id, int* x0, float* conf, float* tokconf, cudaStream_t st) {
-    k_lmhead_reduce<<<N, 32, 0, st>>>(lm_part, zcur, cur_tok, m_tiles, N, mask_id, x0, conf, tokconf);
-    return cudaGetLastError();
-}
-
-__global__ void k_gather_cur(const int* tok, int tok_ld, const int* seq_kv, int* cur, int B, int T) {
-    int j = blockIdx.x * blockDim.x + threadIdx.x;
-    if (j >= B * T) return;
-    int b = j / T, t = j - b * T;
-    cur[j] = tok[static_cast<size_t>(b) * tok_ld + seq_kv[b] + t];
-}
-
-cudaError_t launch_gather_cur(const int* tok, int tok_ld, const int* seq_kv, int* cur, int B, int T,
-                              cudaStream_t st) {
-    k_gather_cur<<<(B * T + 127) / 128, 128, 0, st>>>(tok, tok_ld, seq_kv, cur, B, T);
-    return cudaGetLastError();
+                                 int mask_id, int* x0, float* conf, float* tokconf, cudaStream_t st, bool pdl) {
+    return launch_k(k_lmhead_reduce, dim3(N), dim3(256), 0, st, pdl, lm_part, zcur, cur_tok, m_tiles, mask_id, x0, conf,
+                    tokconf);
 }
 
 // ------------------------------------------------------------------ commit pass
@@ -569,6 +533,8 @@ cudaError_t launch_gather_cur(const int* tok, int tok_ld, const int* seq_kv, int
 //  4. with the prefix cache and lookahead on, each future block inside the
 //     window drafts its single most confident masked position.
 __global__ void __launch_bounds__(256) k_commit(CommitArgs a) {
+    pdl_wait();
+    pdl_launch_dependents();
     const int b = blockIdx.x;
     int* tok = a.tok + static_cast<size_t>(b) * a.ld;
     uint8_t* st = a.st + static_cast<size_t>(b) * a.ld;
@@ -697,9 +663,8 @@ __global__ void __launch_bounds__(256) k_commit(CommitArgs a) {
     }
 }
 
-cudaError_t launch_commit(const CommitArgs& a, cudaStream_t st) {
-    k_commit<<<a.B, 256, 0, st>>>(a);
-    return cudaGetLastError();
+cudaError_t launch_commit(const CommitArgs& a, cudaStream_t st, bool pdl) {
+    return launch_k(k_commit, dim3(a.B), dim3(256), 0, st, pdl, a);
 }
 
 }  // namespace dllm
@@ -710,6 +675,8 @@ namespace dllm {
 // block become COMMITTED; snapshot the window region for rewinds.
 __global__ void k_begin_block(int* tok, uint8_t* st, int* snap_tok, uint8_t* snap_st, int ld, int n_pos, int* plan,
                               int c0, int c1) {
+    pdl_wait();
+    pdl_launch_dependents();
     const int b = blockIdx.x;
     int* t = tok + static_cast<size_t>(b) * ld;
     uint8_t* s = st + static_cast<size_t>(b) * ld;
@@ -729,12 +696,13 @@ __global__ void k_begin_block(int* tok, uint8_t* st, int* snap_tok, uint8_t* sna
 
 cudaError_t launch_begin_block(int* tok, uint8_t* st, int* snap_tok, uint8_t* snap_st, int ld, int n_pos, int* plan,
                                int B, int c0, int c1, cudaStream_t stream) {
-    k_begin_block<<<B, 256, 0, stream>>>(tok, st, snap_tok, snap_st, ld, n_pos, plan, c0, c1);
-    return cudaGetLastError();
+    return launch_k(k_begin_block, dim3(B), dim3(256), 0, stream, true, tok, st, snap_tok, snap_st, ld, n_pos, plan, c0, c1);
 }
 
 __global__ void k_rewind(int* tok, uint8_t* st, const int* snap_tok, const uint8_t* snap_st, int ld, int n_pos,
                          int* plan) {
+    pdl_wait();
+    pdl_launch_dependents();
     const int b = blockIdx.x;
     for (int p = threadIdx.x; p < n_pos; p += blockDim.x) {
         tok[static_cast<size_t>(b) * ld + p] = snap_tok[static_cast<size_t>(b) * ld + p];
@@ -745,18 +713,18 @@ __global__ void k_rewind(int* tok, uint8_t* st, const int* snap_tok, const uint8
 
 cudaError_t launch_rewind(int* tok, uint8_t* st, const int* snap_tok, const uint8_t* snap_st, int ld, int n_pos,
                           int* plan, int B, cudaStream_t stream) {
-    k_rewind<<<B, 256, 0, stream>>>(tok, st, snap_tok, snap_st, ld, n_pos, plan);
-    return cudaGetLastError();
+    return launch_k(k_rewind, dim3(B), dim3(256), 0, stream, true, tok, st, snap_tok, snap_st, ld, n_pos, plan);
 }
 
 __global__ void k_set_kv_len(int* seq_kv, int B, int v) {
+    pdl_wait();
+    pdl_launch_dependents();
     int b = blockIdx.x * blockDim.x + threadIdx.x;
     if (b < B) seq_kv[b] = v;
 }
 
 cudaError_t launch_set_kv_len(int* seq_kv, int B, int v, cudaStream_t stream) {
-    k_set_kv_len<<<(B + 127) / 128, 128, 0, stream>>>(seq_kv, B, v);
-    return cudaGetLastError();
+    return launch_k(k_set_kv_len, dim3((B + 127) / 128), dim3(128), 0, stream, true, seq_kv, B, v);
 }
 
 }  // namespace dllm

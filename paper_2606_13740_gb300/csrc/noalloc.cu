@@ -63,7 +63,8 @@ extern "C" int dllm_op_gemm_noalloc(const void* W, const void* X, float* D, int 
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0)
         return noalloc_fail(DLLM_ECUDA, "device query failed");
-    GemmPlan p = gemm_plan(M, N, K, grid > 0 ? grid : sms);
+    GemmPlan p = gemm_plan(M, N, K, grid > 0 ? grid : sms, EPI_F32);
+    p.pdl = false;
     // the split partials take [grid][2][ntile x 128] floats behind the tickets
     const size_t per_cta = static_cast<size_t>(2) * p.ntile * 128 * sizeof(float);
     const size_t cap_ctas = (kNoAllocScratchBytes - kTicketBytes) / per_cta;
@@ -71,7 +72,8 @@ extern "C" int dllm_op_gemm_noalloc(const void* W, const void* X, float* D, int 
         return noalloc_fail(DLLM_ECAPACITY, "too many output tiles for the static scratch (M x N too large)");
     if (static_cast<size_t>(p.grid) > cap_ctas) {
         if (grid > 0) return noalloc_fail(DLLM_ECAPACITY, "grid too large for the static scratch");
-        p = gemm_plan(M, N, K, static_cast<int>(cap_ctas));  // auto grid: shrink to fit
+        p = gemm_plan(M, N, K, static_cast<int>(cap_ctas), EPI_F32);  // auto grid: shrink to fit
+        p.pdl = false;
     }
     if (gemm_init_attrs() != cudaSuccess) return noalloc_fail(DLLM_ECUDA, "attribute setup failed");
     CUtensorMap tw, tx;

@@ -67,7 +67,8 @@ static int gemm_impl(const void* W, const void* X, float* D, int M, int N, int K
     int sms = sm_count();
     if (sms <= 0) return op_fail(DLLM_ECUDA, "no CUDA device");
     if (gemm_init_attrs() != cudaSuccess) return op_fail(DLLM_ECUDA, "attribute setup failed");
-    GemmPlan p = gemm_plan(M, N, K, grid > 0 ? grid : sms);
+    GemmPlan p = gemm_plan(M, N, K, grid > 0 ? grid : sms, EPI_F32);
+    p.pdl = false;  // the operands come from the caller's kernels
     CUtensorMap tw, tx;
     if (!make_tmap_bf16(&tw, W, M, K, 128) || !make_tmap_bf16(&tx, X, N, K, p.ntile))
         return op_fail(DLLM_EINVAL, "tensor map encode failed (alignment?)");
@@ -128,13 +129,16 @@ int dllm_op_attention(const void* q, const void* kc, const void* vc, const int32
     if (sms <= 0) return op_fail(DLLM_ECUDA, "no CUDA device");
     if (attn_init_attrs() != cudaSuccess) return op_fail(DLLM_ECUDA, "attribute setup failed");
     AttnPlan a = attn_plan(B, T, H, max_kv_len + T, sms);
-    DevBuf po, pml;
+    DevBuf po, pml, ctr;
     const size_t rows = static_cast<size_t>(B) * H * a.nsplit * T;
-    if (!po.alloc(rows * hd * 4) || !pml.alloc(rows * 2 * 4)) return op_fail(DLLM_ENOMEM, "scratch allocation failed");
+    const size_t nctr = static_cast<size_t>(B) * H * a.qtiles;
+    if (!po.alloc(rows * hd * 4) || !pml.alloc(rows * 2 * 4) || !ctr.alloc(nctr * 4))
+        return op_fail(DLLM_ENOMEM, "scratch allocation failed");
+    if (cudaMemsetAsync(ctr.p, 0, nctr * 4, st) != cudaSuccess) return op_fail(DLLM_ECUDA, "memset failed");
     cudaError_t e = launch_attention(static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(kc),
                                      static_cast<const __nv_bfloat16*>(vc), kv_len, static_cast<float*>(po.p),
-                                     static_cast<float*>(pml.p), static_cast<__nv_bfloat16*>(out), B, T, H, hd, cap, a,
-                                     st);
+                                     static_cast<float*>(pml.p), static_cast<int*>(ctr.p),
+                                     static_cast<__nv_bfloat16*>(out), B, T, H, hd, cap, a, st, false);
     if (e != cudaSuccess) return op_fail(DLLM_ECUDA, "attention launch: %s", cudaGetErrorString(e));
     return finish(st, nullptr);
 }
@@ -148,7 +152,8 @@ int dllm_op_lmhead(const void* W, const void* X, const int32_t* cur, int32_t* x0
     int sms = sm_count();
     if (sms <= 0) return op_fail(DLLM_ECUDA, "no CUDA device");
     if (gemm_init_attrs() != cudaSuccess) return op_fail(DLLM_ECUDA, "attribute setup failed");
-    GemmPlan p = gemm_plan(V, N, d, sms);
+    GemmPlan p = gemm_plan(V, N, d, sms, EPI_LMHEAD);
+    p.pdl = false;
     CUtensorMap tw, tx;
     if (!make_tmap_bf16(&tw, W, V, d, 128) || !make_tmap_bf16(&tx, X, N, d, p.ntile))
         return op_fail(DLLM_EINVAL, "tensor map encode failed (alignment?)");
@@ -172,7 +177,7 @@ int dllm_op_lmhead(const void* W, const void* X, const int32_t* cur, int32_t* x0
     cudaError_t e = gemm_launch(EPI_LMHEAD, p, tw, tx, ep, scr, static_cast<int*>(status.p), st);
     if (e == cudaSuccess)
         e = launch_lmhead_reduce(static_cast<float*>(lmp.p), static_cast<float*>(zc.p), cur, p.m_tiles, N, mask_id, x0,
-                                 conf, tokconf, st);
+                                 conf, tokconf, st, false);
     if (e != cudaSuccess) return op_fail(DLLM_ECUDA, "lmhead launch: %s", cudaGetErrorString(e));
     return finish(st, static_cast<int*>(status.p));
 }
@@ -219,7 +224,7 @@ int dllm_op_commit(int32_t* tok, uint8_t* status, int n_pos, int w0, int T, int 
     a.block_len = block_len;
     a.theta_remask = theta_remask;
     a.theta_stable = theta_stable;
-    cudaError_t e = launch_commit(a, nullptr);
+    cudaError_t e = launch_commit(a, nullptr, false);
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) return op_fail(DLLM_ECUDA, "commit: %s", cudaGetErrorString(e));
     int outs[8];
