@@ -219,8 +219,8 @@ def run_ours(args):
 
     cfg = Config(max_batch=1, max_ctx=LP + T, max_window=LP, **SHAPE)
     ctx = Context(cfg)
-    if args.no_pdl:
-        ctx.dllm_set_debug(4)
+    if args.no_pdl or args.full_smem:
+        ctx.dllm_set_debug((4 if args.no_pdl else 0) | (8 if args.full_smem else 0))
     stream = ctx.stream  # the context's own stream: events and kernels share it
     sched = Sched(steps_per_block=MASKED)
     prompt = I.uniform_prompt(LP, cfg.vocab, cfg.mask_id, seed=I.SEED_PROMPT + rank)
@@ -367,6 +367,7 @@ def main(argv=None):
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-pdl", action="store_true", help="launch kernels without programmatic dependent launch")
+    ap.add_argument("--full-smem", action="store_true", help="one 227 KB projection CTA per SM (no co-residency)")
     args = ap.parse_args(argv)
     if args.impl == "reference":
         return run_reference(args)

@@ -171,7 +171,11 @@ int dllm_set_state(dllm_ctx* ctx, const int32_t* tokens, const uint8_t* status);
  * Synchronises. */
 int dllm_get_step_debug(dllm_ctx* ctx, float* logits, int32_t* argmax, float* conf, float* tokconf);
 
-/* flags bit 0: materialise logits; bit 1: disable CUDA graphs. */
+/* flags bit 0: materialise logits; bit 1: disable CUDA graphs; bit 2: launch
+ * without programmatic dependent launch; bit 3: give the weight-streaming
+ * projections 227 KB of shared memory (one CTA per SM) instead of 113 KB;
+ * bit 4: record GEMM timelines (dllm_get_trace).  Bits 2 and 3 apply
+ * process-wide (for A/B measurements). */
 int dllm_set_debug(dllm_ctx* ctx, int flags);
 
 /* Copy one weight back in its logical row-major layout (bf16 bits):
@@ -208,6 +212,11 @@ int dllm_set_profile(dllm_ctx* ctx, int enable);
  * launches_per_step[DLLM_NKINDS] launches of each kind in the last step,
  * steps profiled (any pointer may be NULL). */
 int dllm_get_profile(dllm_ctx* ctx, double* ms_total, int32_t* launches_per_step, int32_t* steps);
+
+/* With dllm_set_debug(16): per-CTA timelines (%globaltimer stamps, see
+ * dllm_op_gemm_trace) of the GEMM launches of the last step, in launch order:
+ * out [n_launches][256][16].  Synchronises. */
+int dllm_get_trace(dllm_ctx* ctx, unsigned long long* out, int max_launches, int32_t* n_launches);
 
 /* Kernel launches in the last denoising step (all kinds). */
 int dllm_launches_per_step(dllm_ctx* ctx, int32_t* n);

@@ -25,9 +25,21 @@ int dllm_op_gemm(const void* W, const void* X, float* D, int M, int N, int K, in
 
 /* dllm_op_gemm launched `reps` times back to back on one scratch
  * allocation; *ms_per_launch = average kernel time by CUDA events on the
- * stream (micro-benchmark hook). */
-int dllm_op_gemm_timed(const void* W, const void* X, float* D, int M, int N, int K, int grid, int reps,
+ * stream (micro-benchmark hook).  flags bit 0: chain the timed launches with
+ * programmatic dependent launch; bit 1: plan 227 KB of shared memory instead
+ * of 113 KB (one CTA per SM) for <= 96 tokens. */
+int dllm_op_gemm_timed(const void* W, const void* X, float* D, int M, int N, int K, int grid, int reps, int flags,
                        float* ms_per_launch, void* stream);
+
+/* dllm_op_gemm_timed that also returns a timeline of the last launch:
+ * trace [grid_used][16] holds, per CTA, %globaltimer stamps (ns) at entry,
+ * after the prologue, first operand stage arrived, last stage consumed,
+ * epilogue done, exit; the SM id; the stamp when the dependency wait
+ * returned; for the CTA's last output tile: accumulator ready, split partial
+ * stored, ticket taken, partials reduced (0 when not the last arriver), the
+ * last-arriver flag and the tile index.  trace must hold 16 values per SM. */
+int dllm_op_gemm_trace(const void* W, const void* X, float* D, int M, int N, int K, int grid, int reps,
+                       float* ms_per_launch, unsigned long long* trace, int* grid_used, void* stream);
 
 /* dllm_op_gemm for callers that cannot allocate device memory, for example
  * code that runs while a stream is being captured into a CUDA graph (a
@@ -38,7 +50,7 @@ int dllm_op_gemm_timed(const void* W, const void* X, float* D, int M, int N, int
  * keeps its scratch (split partials, tile tickets, status word) in one
  * statically sized device array of 8 MiB that every GPU loading the library
  * holds until the process exits; it calls no cudaMalloc, cudaFree or other
- * allocating routine.  Limits: at most 16320 output tiles (ceil(M/128) x
+ * allocating routine.  Limits: at most 2046 output tiles (ceil(M/128) x
  * token tiles); the grid (0 = one CTA per SM) is shrunk to fit the array when
  * chosen automatically, and an explicit grid that does not fit is rejected
  * with DLLM_ECAPACITY.  The first call on a device looks up the array's

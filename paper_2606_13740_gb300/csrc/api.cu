@@ -6,7 +6,6 @@
 //            Wgu [ceil(F/64)*128][d] (64 gate rows then 64 up rows per
 //            128-row tile), Wd [d][F]; embedding [V][d]; LM head [V pad 128][d]
 //   KV cache [L][K|V][batch][head][position][head_dim] bf16
-//   RoPE     [max_ctx][head_dim/2][cos, sin] fp32
 //   activations for max_batch * max_window tokens (fp32 residual, bf16 GEMM
 //   operands), attention and GEMM split partials, LM-head tile statistics
 //   request state: ids int32 [batch][max_ctx], token states uint8, plan.
@@ -15,6 +14,7 @@
 #include "internal.h"
 
 #include <algorithm>
+#include <cmath>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -33,8 +33,8 @@ int rup(int x, int m) { return (x + m - 1) / m * m; }
 
 struct Layout {
     int qd, qkv_rows, gu_rows, d_rows, o_rows, head_rows, head_tiles, max_tok;
-    size_t off_w, per_layer, off_emb, off_head, off_kv, kv_half, off_rope;
-    size_t off_x, off_xn, off_q, off_attn, off_h, off_sq, off_actr;
+    size_t off_w, per_layer, off_emb, off_head, off_kv, kv_half;
+    size_t off_x, off_xn, off_q, off_attn, off_h, off_sq, off_actr, off_theta;
     int n_sq, actr_len;
     size_t off_apo, apo_floats, off_apml;
     size_t off_lmp, off_zcur, off_cur, off_x0, off_conf, off_tokconf;
@@ -72,7 +72,6 @@ Layout make_layout(const dllm_config& c) {
     L.off_head = take(static_cast<size_t>(L.head_rows) * d * 2);
     L.kv_half = static_cast<size_t>(c.max_batch) * H * c.max_ctx * hd;
     L.off_kv = take(L.kv_half * 2 * 2 * c.n_layers);
-    L.off_rope = take(static_cast<size_t>(c.max_ctx) * hd * 4);
     const size_t T = L.max_tok;
     L.off_x = take(T * d * 4);
     L.off_xn = take(T * std::max(d, L.qd) * 2);
@@ -83,6 +82,7 @@ Layout make_layout(const dllm_config& c) {
     L.off_sq = take(static_cast<size_t>(L.n_sq) * T * 4);
     L.actr_len = c.max_batch * H * ((c.max_window + 63) / 64);
     L.off_actr = take(static_cast<size_t>(L.actr_len) * 4);
+    L.off_theta = take(static_cast<size_t>(hd / 2) * 4);
     // attention split partials: B*H*nsplit*T rows, nsplit <= 2*SMs/(B*H*qtiles) + 1
     const size_t rows = static_cast<size_t>(2 * kMaxSMs) * 64 + static_cast<size_t>(c.max_batch) * H * c.max_window;
     L.apo_floats = rows * hd;
@@ -97,7 +97,7 @@ Layout make_layout(const dllm_config& c) {
     L.part_floats = static_cast<size_t>(kMaxSMs) * 2 * 256 * 128;
     L.off_part = take(L.part_floats * 4);
     const int mt_max = std::max(std::max(L.head_tiles, L.gu_rows / 128), std::max(L.qkv_rows, L.d_rows) / 128);
-    L.cnt_len = mt_max * ((L.max_tok + 255) / 256 + 1);
+    L.cnt_len = mt_max * ((L.max_tok + 255) / 256 + 1) * 32;  // one ticket per 128-byte line
     L.off_cnt = take(static_cast<size_t>(L.cnt_len) * 4);
     const size_t S = static_cast<size_t>(c.max_batch) * c.max_ctx;
     L.off_tok = take(S * 4);
@@ -121,6 +121,7 @@ const char* check_cfg(const dllm_config& c) {
     if (c.mask_id < 0 || c.mask_id >= c.vocab) return "mask_id out of range";
     if (c.max_batch < 1 || c.max_ctx < 1 || c.max_window < 1 || c.block_len < 1) return "bad capacities";
     if (c.max_batch * c.max_window > 4096) return "max_batch * max_window must be <= 4096";
+    if (c.max_batch > 256) return "max_batch must be <= 256";
     if (c.block_len > kMaxBlock) return "block_len too large";
     if (c.rms_eps <= 0.0f || c.rope_base <= 1.0f) return "bad rope_base / rms_eps";
     return nullptr;
@@ -143,10 +144,10 @@ struct dllm_ctx {
     std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_d;
     CUtensorMap tm_head{};
     __nv_bfloat16* kv = nullptr;
-    float* rope = nullptr;
     float* x = nullptr;
     __nv_bfloat16 *xn = nullptr, *q = nullptr, *attn = nullptr, *h = nullptr;
     float* sq = nullptr;      // RMSNorm statistics [d/128][tokens]
+    float* theta = nullptr;   // RoPE frequencies [hd/2]
     int* actr = nullptr;      // attention split tickets
     float *apo = nullptr, *apml = nullptr, *lmp = nullptr, *zcur = nullptr, *conf = nullptr, *tokconf = nullptr;
     int *cur = nullptr, *x0 = nullptr;
@@ -176,6 +177,9 @@ struct dllm_ctx {
     int launches_per_step = 0;
     bool capturing = false;
     bool in_step = false;
+    // GEMM timelines of one step (debug flag 16): [launch][256 CTAs][16] stamps
+    unsigned long long* trace = nullptr;
+    int trace_launch = 0;
     bool poisoned = false;
     std::string err;
 };
@@ -189,6 +193,15 @@ static void mark(dllm_ctx* ctx, int kind) {
                              ctx->capturing ? cudaEventRecordExternal : cudaEventRecordDefault);
     ctx->ev_kind[ctx->n_marks] = kind;
     ctx->n_marks++;
+}
+
+constexpr int kTraceLaunches = 512;
+constexpr size_t kTraceStride = 256 * 16;  // per launch: 256 CTAs x 16 slots
+
+// Trace buffer for the GEMM launch about to be made in a step (null when off).
+static unsigned long long* next_trace(dllm_ctx* ctx) {
+    if (!ctx->trace || !ctx->in_step || ctx->trace_launch >= kTraceLaunches) return nullptr;
+    return ctx->trace + static_cast<size_t>(ctx->trace_launch++) * kTraceStride;
 }
 
 static std::string g_noctx_err;
@@ -255,8 +268,9 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
         B * c.n_heads * ap.qtiles > L.actr_len)
         return fail(ctx, DLLM_ECAPACITY, "attention partial buffer too small");
     EpiArgs ep{};
-    ep.rope = ctx->rope;
     ep.seq_kv = ctx->seq_kv;
+    ep.n_seq = B;
+    ep.theta = ctx->theta;
     ep.T = T;
     ep.H = c.n_heads;
     ep.hd = c.head_dim;
@@ -278,15 +292,19 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
         __nv_bfloat16* vc = ctx->kv + static_cast<size_t>(2 * l + 1) * L.kv_half;
         ep.kc = kc;
         ep.vc = vc;
+        ep.trace = next_trace(ctx);
         CK(gemm_launch(EPI_QKV, pq, ctx->tm_qkv[l], tx_xn, ep, ctx->scr, ctx->status, s));
         mark(ctx, DLLM_K_QKV);
         CK(launch_attention(ctx->q, kc, vc, ctx->seq_kv, ctx->apo, ctx->apml, ctx->actr, ctx->attn, B, T, c.n_heads,
                             c.head_dim, c.max_ctx, ap, s));
         mark(ctx, DLLM_K_ATTN);
+        er.trace = next_trace(ctx);
         CK(gemm_launch(EPI_RESID, po, ctx->tm_o[l], tx_attn, er, ctx->scr, ctx->status, s));
         mark(ctx, DLLM_K_OPROJ);
+        ep.trace = next_trace(ctx);
         CK(gemm_launch(EPI_SWIGLU, pg, ctx->tm_gu[l], tx_xn, ep, ctx->scr, ctx->status, s));
         mark(ctx, DLLM_K_GATEUP);
+        er.trace = next_trace(ctx);
         CK(gemm_launch(EPI_RESID, pd, ctx->tm_d[l], tx_h, er, ctx->scr, ctx->status, s));
         mark(ctx, DLLM_K_DOWN);
     }
@@ -299,6 +317,7 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
         eh.V = c.vocab;
         eh.mask_id = c.mask_id;
         eh.logits = (ctx->debug & 1) ? ctx->logits : nullptr;
+        eh.trace = next_trace(ctx);
         CK(gemm_launch(EPI_LMHEAD, ph, ctx->tm_head, tx_xn, eh, ctx->scr, ctx->status, s));
         mark(ctx, DLLM_K_HEAD);
         CK(launch_lmhead_reduce(ctx->lmp, ctx->zcur, ctx->cur, L.head_tiles, N, c.mask_id, ctx->x0, ctx->conf,
@@ -311,6 +330,7 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
 static int step_kernels(dllm_ctx* ctx, int T) {
     ctx->n_marks = 0;
     ctx->launches_per_step = 0;
+    ctx->trace_launch = 0;
     ctx->in_step = true;
     mark(ctx, -1);
     int rc = forward(ctx, ctx->B, T, true);
@@ -381,6 +401,7 @@ void dllm_free(dllm_ctx* ctx) {
     if (ctx->gexec) cudaGraphExecDestroy(ctx->gexec);
     for (cudaEvent_t e : ctx->ev) cudaEventDestroy(e);
     if (ctx->logits) cudaFree(ctx->logits);
+    if (ctx->trace) cudaFree(ctx->trace);
     if (ctx->own_arena && ctx->arena) cudaFree(ctx->arena);
     if (ctx->own_stream && ctx->stream) cudaStreamDestroy(ctx->stream);
     delete ctx;
@@ -432,7 +453,6 @@ int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void*
     ctx->emb = reinterpret_cast<__nv_bfloat16*>(A + L.off_emb);
     ctx->head = reinterpret_cast<__nv_bfloat16*>(A + L.off_head);
     ctx->kv = reinterpret_cast<__nv_bfloat16*>(A + L.off_kv);
-    ctx->rope = reinterpret_cast<float*>(A + L.off_rope);
     ctx->x = reinterpret_cast<float*>(A + L.off_x);
     ctx->xn = reinterpret_cast<__nv_bfloat16*>(A + L.off_xn);
     ctx->q = reinterpret_cast<__nv_bfloat16*>(A + L.off_q);
@@ -440,6 +460,7 @@ int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void*
     ctx->h = reinterpret_cast<__nv_bfloat16*>(A + L.off_h);
     ctx->sq = reinterpret_cast<float*>(A + L.off_sq);
     ctx->actr = reinterpret_cast<int*>(A + L.off_actr);
+    ctx->theta = reinterpret_cast<float*>(A + L.off_theta);
     ctx->apo = reinterpret_cast<float*>(A + L.off_apo);
     ctx->apml = reinterpret_cast<float*>(A + L.off_apml);
     ctx->lmp = reinterpret_cast<float*>(A + L.off_lmp);
@@ -491,7 +512,11 @@ int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void*
     }
     if (ie == cudaSuccess && !make_tmap_bf16(&ctx->tm_head, ctx->head, L.head_rows, d, 128))
         return bail(DLLM_ECUDA, "tensor map encode failed");
-    if (ie == cudaSuccess) ie = launch_init_rope(ctx->rope, c.max_ctx, c.head_dim, c.rope_base, s);
+    // RoPE frequencies base^(-2j/hd), in double on the host
+    std::vector<float> th(c.head_dim / 2);
+    for (int j = 0; j < c.head_dim / 2; ++j)
+        th[j] = static_cast<float>(std::pow(static_cast<double>(c.rope_base), -2.0 * j / c.head_dim));
+    if (ie == cudaSuccess) ie = cudaMemcpyAsync(ctx->theta, th.data(), th.size() * 4, cudaMemcpyHostToDevice, s);
     if (ie != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess) return bail(DLLM_ECUDA, "weight init failed");
     *out = ctx;
     return DLLM_OK;
@@ -503,10 +528,16 @@ int dllm_sync(dllm_ctx* ctx) {
 }
 
 static int set_debug_buffers(dllm_ctx* ctx) {
+    if ((ctx->debug & 16) && !ctx->trace) {
+        if (cudaMalloc(&ctx->trace, kTraceLaunches * kTraceStride * 8) != cudaSuccess)
+            return fail(ctx, DLLM_ENOMEM, "trace buffer");
+        cudaMemset(ctx->trace, 0, kTraceLaunches * kTraceStride * 8);
+    }
     if (!(ctx->debug & 1)) return DLLM_OK;
     size_t need = static_cast<size_t>(ctx->L.max_tok) * ctx->cfg.vocab;
     if (ctx->logits_cap >= need) return DLLM_OK;
     if (ctx->logits) cudaFree(ctx->logits);
+    if (ctx->trace) cudaFree(ctx->trace);
     ctx->logits = nullptr;
     if (cudaMalloc(&ctx->logits, need * 4) != cudaSuccess) return fail(ctx, DLLM_ENOMEM, "logits buffer");
     ctx->logits_cap = need;
@@ -517,6 +548,7 @@ int dllm_set_debug(dllm_ctx* ctx, int flags) {
     GUARD(ctx);
     ctx->debug = flags;
     set_pdl(!(flags & 4));
+    set_stream_smem(!(flags & 8));
     return set_debug_buffers(ctx);
 }
 
@@ -678,7 +710,7 @@ int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out) {
     ctx->last_spec = spec;
     const bool use_graph = !(ctx->debug & 2);
     if (use_graph) {
-        const int key_dbg = ctx->debug | (ctx->profiling ? 256 : 0);
+        const int key_dbg = ctx->debug | (ctx->profiling ? 256 : 0);  // trace pointers are baked in too
         if (!ctx->gexec || ctx->g_T != T || ctx->g_B != ctx->B || ctx->g_kv != ctx->kv_len || ctx->g_dbg != key_dbg) {
             if (ctx->gexec) {
                 cudaGraphExecDestroy(ctx->gexec);
@@ -787,6 +819,16 @@ int dllm_get_profile(dllm_ctx* ctx, double* ms_total, int32_t* launches_per_step
     }
     if (steps) *steps = ctx->prof_steps;
     return DLLM_OK;
+}
+
+int dllm_get_trace(dllm_ctx* ctx, unsigned long long* out, int max_launches, int32_t* n_launches) {
+    GUARD(ctx);
+    if (!ctx->trace || !out || !n_launches) return fail(ctx, DLLM_EINVAL, "tracing needs dllm_set_debug(16)");
+    const int n = ctx->trace_launch < max_launches ? ctx->trace_launch : max_launches;
+    CK(cudaMemcpyAsync(out, ctx->trace, static_cast<size_t>(n) * kTraceStride * 8, cudaMemcpyDeviceToHost,
+                       ctx->stream));
+    *n_launches = n;
+    return sync_check(ctx);
 }
 
 int dllm_launches_per_step(dllm_ctx* ctx, int32_t* n) {

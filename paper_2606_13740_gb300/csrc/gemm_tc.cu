@@ -12,7 +12,9 @@
 // so every SM streams the same number of weight bytes whatever the tile
 // count.  A tile cut between CTAs is finished by whichever CTA arrives last
 // (atomic ticket), which sums the fp32 partials in k order: deterministic,
-// and nobody waits on anybody.
+// and nobody waits on anybody.  When that tile is the CTA's final one, its
+// drained pipeline memory receives every partial through one round of bulk
+// copies.
 //
 // Roles (192 threads): warp 0 = TMA producer, warp 1 = TMEM owner and MMA
 // issuer, warps 2..5 = epilogue (one TMEM lane quarter each).  Accumulators
@@ -26,6 +28,10 @@
 // pipeline stages of weights (which no earlier kernel writes) before
 // griddepcontrol.wait, so a projection's weight stream starts while the
 // previous kernel is still finishing.
+//
+// The epilogue runs once per tile on the step's critical path, so it avoids
+// dependent chains of global loads (everything it reads is loaded before it
+// stores, or staged in shared memory early) and keeps its code compact.
 #include "common.cuh"
 #include "internal.h"
 
@@ -40,6 +46,19 @@ constexpr int kStageLd = 17;  // LM-head staging: 16 columns + pad
 constexpr uint32_t kABytes = kBM * kBK * 2;
 constexpr int kStreamSmem = 115712;  // two CTAs per SM (228 KB less 1 KB reserved each)
 constexpr int kFullSmem = 227 * 1024;
+static int g_stream_budget = kStreamSmem;
+constexpr int kTicketStride = 32;  // one tile ticket per 128-byte line
+
+// Timeline trace slots per CTA (when EpiArgs::trace is set).
+enum { kTrStart = 0, kTrPrologue = 1, kTrFirstData = 2, kTrLastData = 3, kTrEpiDone = 4, kTrExit = 5, kTrSm = 6,
+       kTrDepWait = 7, kTrAccReady = 8, kTrPartStored = 9, kTrTicket = 10, kTrReduced = 11, kTrIsLast = 12,
+       kTrTile = 13, kTrSlots = 16 };
+
+__device__ __forceinline__ unsigned smid() {
+    unsigned id;
+    asm volatile("mov.u32 %0, %%smid;" : "=r"(id));
+    return id;
+}
 
 __device__ __forceinline__ int owner_of(long long i, long long total, int G) {
     return static_cast<int>(((i + 1) * G + total - 1) / total) - 1;
@@ -64,9 +83,48 @@ __device__ __forceinline__ void warp_reduce_scatter32(float* v, int lane) {
 
 struct EpiSmem {
     float* stg;   // LM head staging [128][kStageLd]
-    float* rs;    // [32] per-column RMSNorm scale
-    float* red;   // [4][32] cross-warp partial sums
+    float* rs;    // [256] per-column RMSNorm scale of the current token tile
+    float* red;   // [4][256] cross-warp / quarter partial sums
+    int* kvs;     // [256] per-sequence first window position (QKV)
+    float* theta; // [128] rotation frequency of each tile row's feature pair (QKV)
 };
+
+// RMSNorm scale of every column of token tile nt: rs[c] = rsqrt(sum_t sq[t][col] / dim + eps).
+// 128 threads, 4 per column (each over a quarter of the statistics, loads independent), summed
+// in a fixed order: deterministic.
+__device__ __forceinline__ void compute_norm_scale(const EpiArgs& ep, const GemmPlan& p, int nt, const EpiSmem& sm,
+                                                   int e) {
+    for (int item = e; item < 4 * p.ntile; item += 128) {
+        const int c = item % p.ntile, q = item / p.ntile;
+        const int col = nt * p.ntile + c;
+        float s = 0.0f;
+        if (col < p.N) {
+            float a[8];
+            int t = q;
+            for (; t + 28 < ep.n_sq; t += 32) {
+#pragma unroll
+                for (int u = 0; u < 8; ++u) a[u] = ep.sq_in[static_cast<size_t>(t + 4 * u) * p.N + col];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) s += a[u];
+            }
+            for (; t < ep.n_sq; t += 4) s += ep.sq_in[static_cast<size_t>(t) * p.N + col];
+        }
+        sm.red[q * 256 + c] = s;
+    }
+    named_bar(1, 128);
+    for (int c = e; c < p.ntile; c += 128) {
+        const float s = ((sm.red[c] + sm.red[256 + c]) + sm.red[512 + c]) + sm.red[768 + c];
+        sm.rs[c] = rsqrtf(s / static_cast<float>(ep.norm_dim) + ep.eps);
+    }
+    named_bar(1, 128);
+}
+
+// (cos, sin) of an angle: one out-of-line copy, called twice per chunk on the common path.
+__device__ __noinline__ float2 rot_cs(float angle) {
+    float sn, cn;
+    sincosf(angle, &sn, &cn);
+    return make_float2(cn, sn);
+}
 
 // ------------------------------------------------------------------ epilogues
 template <int EPI>
@@ -76,18 +134,9 @@ __device__ __forceinline__ void epilogue_chunk(const EpiArgs& ep, const GemmPlan
     const int row = mt * kBM + rt;
     const int col0 = nt * p.ntile + chunk * 32;
     if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
-        if (ep.sq_in) {  // RMSNorm of the operand rows, as a per-token scale
-            if (ew == 0) {
-                const int col = col0 + lane;
-                float s = 0.0f;
-                if (col < p.N)
-                    for (int t = 0; t < ep.n_sq; ++t) s += ep.sq_in[static_cast<size_t>(t) * p.N + col];
-                sm.rs[lane] = rsqrtf(s / static_cast<float>(ep.norm_dim) + ep.eps);
-            }
-            named_bar(1, 128);
+        if (ep.sq_in) {  // RMSNorm of the operand rows, as a per-token scale (computed per token tile)
 #pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] *= sm.rs[j];
-            named_bar(1, 128);
+            for (int j = 0; j < 32; ++j) v[j] *= sm.rs[chunk * 32 + j];
         }
     }
     if constexpr (EPI == EPI_F32) {
@@ -101,16 +150,25 @@ __device__ __forceinline__ void epilogue_chunk(const EpiArgs& ep, const GemmPlan
     } else if constexpr (EPI == EPI_RESID) {
         const bool rv = row < p.M;
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-            const int col = col0 + j;
-            float x = 0.0f;
-            if (rv && col < p.N) {
-                const size_t o = static_cast<size_t>(col) * ep.ld_out + row;
-                x = ep.out[o] + v[j];
-                ep.out[o] = x;
-                ep.xb[o] = __float2bfloat16_rn(x);
+        for (int h0 = 0; h0 < 32; h0 += 16) {
+            float xo[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {  // the residual loads issued before any store
+                const int col = col0 + h0 + j;
+                xo[j] = (rv && col < p.N) ? ep.out[static_cast<size_t>(col) * ep.ld_out + row] : 0.0f;
             }
-            v[j] = x * x;
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                const int col = col0 + h0 + j;
+                float x = 0.0f;
+                if (rv && col < p.N) {
+                    const size_t o = static_cast<size_t>(col) * ep.ld_out + row;
+                    x = xo[j] + v[h0 + j];
+                    ep.out[o] = x;
+                    ep.xb[o] = __float2bfloat16_rn(x);
+                }
+                v[h0 + j] = x * x;
+            }
         }
         warp_reduce_scatter32(v, lane);
         sm.red[quarter * 32 + lane] = v[0];
@@ -129,31 +187,56 @@ __device__ __forceinline__ void epilogue_chunk(const EpiArgs& ep, const GemmPlan
         const int hh = f / ep.hd;
         const int pp = f - hh * ep.hd;          // physical row inside the head
         const int half = ep.hd >> 1;
-        const int jr = pp >> 1;                 // rotation pair index
-        const int i = jr + (pp & 1) * half;     // logical feature
+        const int i = (pp >> 1) + (pp & 1) * half;  // logical feature
+        const float theta = sm.theta[rt];
+        // The chunk's 32 columns are consecutive positions of one sequence when the window
+        // length is a multiple of 32: rotate by the angle-addition recurrence (two sincosf
+        // per chunk; the table of cos/sin would be DRAM-cold behind the weight stream).
+        const int bl = col0 / ep.T;
+        const int last = min(col0 + 31, p.N - 1);
+        const bool run = last / ep.T == bl;  // uniform across the CTA
+        float cn = 1.0f, sn = 0.0f, cd = 1.0f, sd = 0.0f;
+        if (part < 2 && run) {
+            const float2 a = rot_cs(static_cast<float>(sm.kvs[bl] + (col0 - bl * ep.T)) * theta);
+            const float2 d = rot_cs(theta);
+            cn = a.x;
+            sn = a.y;
+            cd = d.x;
+            sd = d.y;
+        }
 #pragma unroll
         for (int j = 0; j < 32; ++j) {
             const float xp = __shfl_xor_sync(0xffffffffu, v[j], 1);
             const int col = col0 + j;
-            if (col >= p.N) continue;
-            const int b = col / ep.T;
-            const int t = col - b * ep.T;
-            const int pos = ep.seq_kv[b] + t;
-            if (pos < 0 || pos >= ep.cap) {
-                atomicOr(status, kStatusBadIndex);
-                continue;
+            if (col < p.N) {
+                const int b = run ? bl : col / ep.T;
+                const int t = col - b * ep.T;
+                const int pos = sm.kvs[b] + t;
+                if (pos < 0 || pos >= ep.cap) {
+                    atomicOr(status, kStatusBadIndex);
+                } else {
+                    float x = v[j];
+                    if (part < 2) {
+                        if (!run) {
+                            const float2 a = rot_cs(static_cast<float>(pos) * theta);
+                            cn = a.x;
+                            sn = a.y;
+                        }
+                        x = (pp & 1) ? (x * cn + xp * sn) : (x * cn - xp * sn);
+                    }
+                    const __nv_bfloat16 y = __float2bfloat16_rn(x);
+                    if (part == 0) {
+                        ep.q[((static_cast<size_t>(b) * ep.H + hh) * ep.T + t) * ep.hd + i] = y;
+                    } else {
+                        __nv_bfloat16* c = part == 1 ? ep.kc : ep.vc;
+                        c[((static_cast<size_t>(b) * ep.H + hh) * ep.cap + pos) * ep.hd + i] = y;
+                    }
+                }
             }
-            float x = v[j];
-            if (part < 2) {
-                const float2 cs = *reinterpret_cast<const float2*>(ep.rope + (static_cast<size_t>(pos) * half + jr) * 2);
-                x = (pp & 1) ? (x * cs.x + xp * cs.y) : (x * cs.x - xp * cs.y);
-            }
-            const __nv_bfloat16 y = __float2bfloat16_rn(x);
-            if (part == 0) {
-                ep.q[((static_cast<size_t>(b) * ep.H + hh) * ep.T + t) * ep.hd + i] = y;
-            } else {
-                __nv_bfloat16* c = part == 1 ? ep.kc : ep.vc;
-                c[((static_cast<size_t>(b) * ep.H + hh) * ep.cap + pos) * ep.hd + i] = y;
+            if (run) {  // advance the rotation by one position
+                const float c2 = cn * cd - sn * sd;
+                sn = sn * cd + cn * sd;
+                cn = c2;
             }
         }
     } else if constexpr (EPI == EPI_SWIGLU) {
@@ -165,7 +248,7 @@ __device__ __forceinline__ void epilogue_chunk(const EpiArgs& ep, const GemmPlan
             const int col = col0 + j;
             if (gate && f < ep.F && col < p.N) {
                 const float g = v[j];
-                const float s = g / (1.0f + expf(-g));
+                const float s = g / (1.0f + __expf(-g));
                 ep.h[static_cast<size_t>(col) * ep.F + f] = __float2bfloat16_rn(s * u);
             }
         }
@@ -233,7 +316,7 @@ __device__ __forceinline__ void epilogue_chunk(const EpiArgs& ep, const GemmPlan
 
 // ------------------------------------------------------------------ kernel
 template <int EPI>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, 2)
     k_gemm(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX, const GemmPlan p,
            const EpiArgs ep, float* __restrict__ partials, int* __restrict__ counters, int* status) {
     extern __shared__ uint8_t smem_raw[];
@@ -245,15 +328,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     float* tail = reinterpret_cast<float*>(sB + static_cast<size_t>(S) * b_bytes);
     EpiSmem esm;
     esm.rs = tail;
-    esm.red = tail + 32;
-    esm.stg = tail + 32 + 128;
+    esm.red = tail + 256;
+    esm.kvs = reinterpret_cast<int*>(tail + 256 + 1024);
+    esm.theta = tail + 256 + 1024 + 256;
+    esm.stg = tail + 256 + 1024 + 256 + 128;
     float* after = esm.stg + (EPI == EPI_LMHEAD ? kBM * kStageLd : 0);
     uint64_t* full = reinterpret_cast<uint64_t*>(after);
     uint64_t* empty = full + S;
     uint64_t* tfull = empty + S;
     uint64_t* tempty = tfull + 2;
     uint64_t* drain = tempty + 2;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    uint64_t* redbar = drain + 1;  // split-partial bulk loads of the last arriver
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(redbar + 1);
     volatile int* s_abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
     volatile int* s_last = s_abort + 1;
 
@@ -263,6 +349,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     const long long it0 = range_begin(blockIdx.x, p.total, G);
     const long long it1 = range_begin(blockIdx.x + 1, p.total, G);
 
+    unsigned long long* tr = ep.trace ? ep.trace + static_cast<size_t>(blockIdx.x) * kTrSlots : nullptr;
+    if (tr && threadIdx.x == 0) {
+        tr[kTrStart] = global_ns();
+        tr[kTrSm] = smid();
+        for (int i = kTrAccReady; i < kTrSlots; ++i) tr[i] = 0;
+    }
     if (threadIdx.x == 0) {
         pdl_launch_dependents();
         for (int s = 0; s < S; ++s) {
@@ -274,6 +366,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&tempty[a], 128);
         }
         mbar_init(drain, 1);
+        mbar_init(redbar, 1);
         *s_abort = 0;
         *s_last = 0;
         mbar_fence_init();
@@ -290,6 +383,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    if (tr && threadIdx.x == 0) tr[kTrPrologue] = global_ns();
 
     if (warp == 0) {
         // ---------------------------------------------------------- producer
@@ -312,6 +406,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tma_load_2d(sA + static_cast<size_t>(q) * kABytes, &tmW, k * kBK, mt * kBM, &full[q], pol_w);
             }
             pdl_wait();
+            if (tr) tr[kTrDepWait] = global_ns();
             for (long long q = 0; q < npre; ++q) {
                 const long long it = it0 + q;
                 const long long tile = it / p.kb;
@@ -353,6 +448,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp == 1) {
         // ---------------------------------------------------------- MMA issuer
         if (lane == 0) {
+            pdl_wait();  // operands arrive only after the producer's own wait: block here, do not spin
             const uint32_t idesc = umma_idesc_bf16(kBM, p.ntile);
             int stage = 0;
             uint32_t phase = 0;
@@ -373,6 +469,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         ok = false;
                         break;
                     }
+                    if (tr && !issued) tr[kTrFirstData] = global_ns();
                     tc_fence_after();
                     const uint64_t adesc = sw128_kmajor_desc(smem_u32(sA + static_cast<size_t>(stage) * kABytes));
                     const uint64_t bdesc = sw128_kmajor_desc(smem_u32(sB + static_cast<size_t>(stage) * b_bytes));
@@ -396,6 +493,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 it = tile * p.kb + k_hi;
             }
+            if (tr) tr[kTrLastData] = global_ns();
             if (*s_abort && issued) {
                 // wait for the tensor cores before the accumulator memory is released
                 umma_commit(drain);
@@ -410,10 +508,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int ew = warp - 2;                 // 0..3
         const int quarter = warp & 3;            // TMEM lane quarter this warp may access
         const int rt = quarter * 32 + lane;      // row within the 128-row tile
+        if constexpr (EPI == EPI_QKV) {
+            for (int b = ew * 32 + lane; b < ep.n_seq; b += 128) esm.kvs[b] = ep.seq_kv[b];
+            // frequency of this tile row's rotation pair (rows interleave the pairs inside a head,
+            // and tiles start at head boundaries)
+            esm.theta[rt] = ep.theta[(rt % ep.hd) >> 1];
+            named_bar(1, 128);
+        }
         const int nchunks = p.ntile / 32;
         const size_t slot_floats = static_cast<size_t>(p.ntile) * kBM;
         int acc = 0;
         uint32_t acc_phase = 0;
+        uint32_t red_phase = 0;
+        int rs_nt = -1;
         float v[32];
         for (long long it = it0; it < it1;) {
             const long long tile = it / p.kb;
@@ -422,9 +529,21 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int k_hi = static_cast<int>((it1 < tend ? it1 : tend) - tile * p.kb);
             const int mt = static_cast<int>(tile / p.n_tiles);
             const int nt = static_cast<int>(tile - static_cast<long long>(mt) * p.n_tiles);
+            if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
+                // the operand's RMSNorm scale only needs the previous kernel: computed while the
+                // accumulator is still being produced
+                if (ep.sq_in && nt != rs_nt) {
+                    compute_norm_scale(ep, p, nt, esm, ew * 32 + lane);
+                    rs_nt = nt;
+                }
+            }
             mbar_wait(&tfull[acc], acc_phase, s_abort, status);
             named_bar(1, 128);
             if (*s_abort) break;
+            if (tr && threadIdx.x == 64) {
+                tr[kTrAccReady] = global_ns();
+                tr[kTrTile] = static_cast<unsigned long long>(tile);
+            }
             tc_fence_after();
             const uint32_t t_acc = tmem_base + static_cast<uint32_t>(acc * p.acc_cols) +
                                    (static_cast<uint32_t>(quarter * 32) << 16);
@@ -436,8 +555,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (whole) {
                     epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
                 } else {
+                    // float4 (c*8 + j, row): coalesced here, conflict-free when the reducer stages it
+                    float4* dst = reinterpret_cast<float4*>(my_part);
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) my_part[static_cast<size_t>(c * 32 + j) * kBM + rt] = v[j];
+                    for (int j = 0; j < 8; ++j)
+                        dst[static_cast<size_t>(c * 8 + j) * kBM + rt] =
+                            make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
                 }
             }
             tc_fence_before();
@@ -451,39 +574,99 @@ __global__ void __launch_bounds__(kThreads, 1)
                 __threadfence();
                 named_bar(1, 128);
                 if (threadIdx.x == 64) {
+                    if (tr) tr[kTrPartStored] = global_ns();
                     const int c_first = owner_of(tile * p.kb, p.total, G);
                     const int c_last = owner_of(tile * p.kb + p.kb - 1, p.total, G);
-                    const int prev = atomicAdd(&counters[tile], 1);
+                    int* ticket = &counters[tile * kTicketStride];
+                    const int prev = atomicAdd(ticket, 1);
                     const int last = prev == c_last - c_first;
-                    if (last) counters[tile] = 0;
+                    if (last) *ticket = 0;
                     *s_last = last;
+                    if (tr) {
+                        tr[kTrTicket] = global_ns();
+                        tr[kTrIsLast] = last;
+                    }
                 }
                 named_bar(1, 128);
                 if (*s_last) {
                     __threadfence();
                     const int c_first = owner_of(tile * p.kb, p.total, G);
                     const int c_last = owner_of(tile * p.kb + p.kb - 1, p.total, G);
-                    for (int c = 0; c < nchunks; ++c) {
+                    const int nparts = c_last - c_first + 1;
+                    const uint32_t part_bytes = static_cast<uint32_t>(slot_floats * 4);
+                    const uint32_t stage_room = static_cast<uint32_t>(S) * (kABytes + b_bytes);
+                    const bool final_seg = tile * p.kb + k_hi == it1;  // pipeline drained: stage memory free
+                    if (final_seg && nchunks == 1 && part_bytes <= stage_room) {
+                        // one round trip: bulk-copy every partial into the stage memory at once
+                        const int per_batch = static_cast<int>(stage_room / part_bytes);
 #pragma unroll
                         for (int j = 0; j < 32; ++j) v[j] = 0.0f;
-                        for (int cc = c_first; cc <= c_last; ++cc) {
-                            const int sl = (range_begin(cc, p.total, G) / p.kb == tile) ? 0 : 1;
-                            const float* pp = partials + (static_cast<size_t>(cc) * 2 + sl) * slot_floats +
-                                              static_cast<size_t>(c * 32) * kBM + rt;
+                        for (int b0 = 0; b0 < nparts; b0 += per_batch) {
+                            const int nb = nparts - b0 < per_batch ? nparts - b0 : per_batch;
+                            if (threadIdx.x == 64) {
+                                fence_proxy_async_global();
+                                mbar_arrive_expect_tx(redbar, part_bytes * static_cast<uint32_t>(nb));
+                                for (int q = 0; q < nb; ++q) {
+                                    const int cc = c_first + b0 + q;
+                                    const int sl = (range_begin(cc, p.total, G) / p.kb == tile) ? 0 : 1;
+                                    bulk_load(smem + static_cast<size_t>(q) * part_bytes,
+                                              partials + (static_cast<size_t>(cc) * 2 + sl) * slot_floats, part_bytes,
+                                              redbar);
+                                }
+                            }
+                            mbar_wait(redbar, red_phase, s_abort, status);
+                            red_phase ^= 1u;
+                            for (int q = 0; q < nb; ++q) {
+                                const float4* src =
+                                    reinterpret_cast<const float4*>(smem + static_cast<size_t>(q) * part_bytes);
 #pragma unroll
-                            for (int j = 0; j < 32; ++j) v[j] += __ldcg(pp + static_cast<size_t>(j) * kBM);
+                                for (int j = 0; j < 8; ++j) {
+                                    const float4 a = src[j * kBM + rt];
+                                    v[4 * j] += a.x;
+                                    v[4 * j + 1] += a.y;
+                                    v[4 * j + 2] += a.z;
+                                    v[4 * j + 3] += a.w;
+                                }
+                            }
+                            named_bar(1, 128);  // the next batch overwrites the staging memory
                         }
-                        epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
+                        if (tr && threadIdx.x == 64) tr[kTrReduced] = global_ns();
+                        epilogue_chunk<EPI>(ep, p, mt, nt, 0, rt, v, esm, ew, quarter, lane, status);
+                    } else {
+                        for (int c = 0; c < nchunks; ++c) {
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+                            // partials in k order (each one's 8 loads in flight together)
+                            for (int cc = c_first; cc <= c_last; ++cc) {
+                                const int sl0 = (range_begin(cc, p.total, G) / p.kb == tile) ? 0 : 1;
+                                const float4* p0 = reinterpret_cast<const float4*>(
+                                    partials + (static_cast<size_t>(cc) * 2 + sl0) * slot_floats);
+                                float4 a[8];
+#pragma unroll
+                                for (int j = 0; j < 8; ++j) a[j] = __ldcg(p0 + static_cast<size_t>(c * 8 + j) * kBM + rt);
+#pragma unroll
+                                for (int j = 0; j < 8; ++j) {
+                                    v[4 * j] += a[j].x;
+                                    v[4 * j + 1] += a[j].y;
+                                    v[4 * j + 2] += a[j].z;
+                                    v[4 * j + 3] += a[j].w;
+                                }
+                            }
+                            if (tr && threadIdx.x == 64 && c == 0) tr[kTrReduced] = global_ns();
+                            epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
+                        }
                     }
                 }
             }
             it = tile * p.kb + k_hi;
         }
+        if (tr && threadIdx.x == 64) tr[kTrEpiDone] = global_ns();
     }
 
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    if (tr && threadIdx.x == 0) tr[kTrExit] = global_ns();
     if (warp == 1) {
         __syncwarp();
         tmem_dealloc(tmem_base, p.tmem_cols);
@@ -513,9 +696,9 @@ GemmPlan gemm_plan(int M, int N, int K, int grid_max, int epi) {
     p.acc_cols = pow2ceil(p.ntile);
     p.tmem_cols = 2 * p.acc_cols;
     const int staging = epi == EPI_LMHEAD ? kBM * kStageLd * 4 : 0;
-    const int fixed = 1024 + (32 + 128) * 4 + staging + 64 * 8 + 64;
+    const int fixed = 1024 + (256 + 1024 + 256 + 128) * 4 + staging + 64 * 8 + 64;
     const int stage_bytes = static_cast<int>(kABytes) + p.ntile * kBK * 2;
-    const int budget = p.ntile <= 96 ? kStreamSmem : kFullSmem;
+    const int budget = p.ntile <= 96 ? g_stream_budget : kFullSmem;
     int st = (budget - fixed) / stage_bytes;
     if (st > 16) st = 16;
     if (st < 2) st = 2;
@@ -579,7 +762,7 @@ static cudaError_t launch_t(const GemmPlan& p, const CUtensorMap& tmW, const CUt
 cudaError_t gemm_launch(int epi, const GemmPlan& p, const CUtensorMap& tmW, const CUtensorMap& tmX,
                         const EpiArgs& ep, const Scratch& scr, int* status, cudaStream_t st) {
     if (static_cast<size_t>(p.grid) * 2 * p.ntile * kBM > scr.partial_floats ||
-        static_cast<long long>(p.m_tiles) * p.n_tiles > scr.counter_len)
+        static_cast<long long>(p.m_tiles) * p.n_tiles * kTicketStride > scr.counter_len)
         return cudaErrorInvalidValue;
     switch (epi) {
         case EPI_F32: return launch_t<EPI_F32>(p, tmW, tmX, ep, scr, status, st);
@@ -590,6 +773,8 @@ cudaError_t gemm_launch(int epi, const GemmPlan& p, const CUtensorMap& tmW, cons
     }
     return cudaErrorInvalidValue;
 }
+
+void set_stream_smem(bool coresident) { g_stream_budget = coresident ? kStreamSmem : kFullSmem; }
 
 static bool g_pdl = true;
 void set_pdl(bool on) { g_pdl = on; }

@@ -37,9 +37,10 @@ struct EpiArgs {
     __nv_bfloat16* q;    // [B][H][T][hd]
     __nv_bfloat16* kc;   // layer's K cache base: [B][H][cap][hd]
     __nv_bfloat16* vc;
-    const float* rope;   // [cap][hd/2][2] (cos, sin)
     const int* seq_kv;   // per-sequence first window position (kv_len)
     int T, H, hd, cap;
+    int n_seq;           // sequences (B), <= 256
+    const float* theta;  // [hd/2]: rotation of feature pair j at position p is p * theta[j]
     // EPI_SWIGLU: tile k row 2f is gate feature 64k+f, row 2f+1 the matching up row
     __nv_bfloat16* h;    // [N][F]
     int F;
@@ -49,6 +50,8 @@ struct EpiArgs {
     const int* cur_tok;  // [N]
     float* logits;       // [N][V] or null
     int V, mask_id;
+    // timeline trace (null = off): per CTA 16 %globaltimer stamps / ids, see kTr* in gemm_tc.cu
+    unsigned long long* trace;
 };
 
 struct GemmPlan {
@@ -66,7 +69,7 @@ struct GemmPlan {
 
 struct Scratch {
     float* partials;     // [grid][2][ntile*128]
-    int* counters;       // [m_tiles*n_tiles], zero between launches
+    int* counters;       // tile tickets, one per 128-byte line ([m_tiles*n_tiles][32]), zero between launches
     size_t partial_floats;
     int counter_len;
 };
@@ -84,6 +87,8 @@ cudaError_t gemm_launch(int epi, const GemmPlan& p, const CUtensorMap& tmW, cons
 // while its predecessor drains, and waits (griddepcontrol.wait) before touching data the
 // predecessor writes.  set_pdl(false) launches them plainly.
 void set_pdl(bool on);
+// GEMM shared-memory plan for <= 96 tokens: true = 113 KB (two CTAs per SM), false = 227 KB.
+void set_stream_smem(bool coresident);
 bool pdl_enabled();
 
 template <typename... KArgs, typename... Args>
@@ -105,7 +110,6 @@ inline cudaError_t launch_k(void (*k)(KArgs...), dim3 grid, dim3 block, size_t s
 // ---------------------------------------------------------------- other kernels
 cudaError_t launch_init_weight(__nv_bfloat16* dst, int mode, int rows_phys, int cols, int logical_rows,
                                uint64_t seed, uint64_t tid0, int qd, int hd, cudaStream_t st);
-cudaError_t launch_init_rope(float* rope, int cap, int hd, double base, cudaStream_t st);
 cudaError_t launch_init_kv_random(__nv_bfloat16* cache, int B, int H, int hd, int cap, int P, int layer,
                                   int which, int L, uint64_t seed, cudaStream_t st);
 // x = embedding rows of the window's ids (fp32), xb = bf16(x), sq[d/128][N] = per-128-feature

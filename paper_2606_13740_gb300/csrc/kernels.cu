@@ -104,26 +104,6 @@ cudaError_t launch_init_kv_random(__nv_bfloat16* cache, int B, int H, int hd, in
     return cudaGetLastError();
 }
 
-// RoPE table: rope[pos][i] = (cos, sin)(pos * base^(-2i/hd)), computed in double.
-__global__ void k_init_rope(float* rope, int cap, int hd, double base) {
-    const int half = hd / 2;
-    const int n = cap * half;
-    for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < n; e += gridDim.x * blockDim.x) {
-        int pos = e / half, i = e % half;
-        double theta = pow(base, -2.0 * i / hd);
-        double s, c;
-        sincos(static_cast<double>(pos) * theta, &s, &c);
-        rope[2 * e] = static_cast<float>(c);
-        rope[2 * e + 1] = static_cast<float>(s);
-    }
-}
-
-cudaError_t launch_init_rope(float* rope, int cap, int hd, double base, cudaStream_t st) {
-    int n = cap * hd / 2;
-    k_init_rope<<<(n + 255) / 256, 256, 0, st>>>(rope, cap, hd, base);
-    return cudaGetLastError();
-}
-
 // ------------------------------------------------------------------ embedding
 // One CTA (8 warps) per token: x = embedding row (fp32 residual), xb = bf16(x)
 // (the QKV projection's operand), sq[c][token] = sum of x^2 over features
@@ -172,6 +152,7 @@ cudaError_t launch_embed(const int* tok, int tok_ld, const int* seq_kv, const __
 // head, query tile) to finish merges all splits in split order.
 constexpr int kAQ = 64;
 constexpr int kAK = 64;
+constexpr int kMaxSplit = 64;  // key splits per (sequence, head, query tile)
 
 __device__ __forceinline__ int swz(int r, int c, int hd) {
     return r * hd + ((((c >> 3) ^ (r & 7))) << 3) + (c & 7);
@@ -217,7 +198,9 @@ __global__ void __launch_bounds__(128) k_attn(const __nv_bfloat16* __restrict__ 
                                               int H, int cap, int chunk, int nsplit, int qtiles) {
     extern __shared__ __align__(128) uint8_t smem_attn[];
     __shared__ int s_last;
-    pdl_wait();
+    // seq_kv and the cached prefix rows are not written by the preceding kernel (the QKV
+    // projection writes the window rows [kv_len, kv_len + T)), so they may be read before
+    // the dependency wait
     pdl_launch_dependents();
     __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem_attn);
     __nv_bfloat16* sK = sQ + kAQ * HD;       // [2][kAK][HD]
@@ -239,10 +222,6 @@ __global__ void __launch_bounds__(128) k_attn(const __nv_bfloat16* __restrict__ 
     const __nv_bfloat16* kbase = kc + (static_cast<size_t>(b) * H + h) * cap * HD;
     const __nv_bfloat16* vbase = vc + (static_cast<size_t>(b) * H + h) * cap * HD;
 
-    for (int e = tid; e < kAQ * CPR; e += 128) {
-        int r = e / CPR, cc = (e % CPR) * 8;
-        cp_async16(sQ + swz(r, cc, HD), qbase + static_cast<size_t>(r < nq ? r : 0) * HD + cc, r < nq);
-    }
     auto load_kv = [&](int buf, int k0) {
         for (int e = tid; e < kAK * CPR; e += 128) {
             int r = e / CPR, cc = (e % CPR) * 8;
@@ -253,7 +232,17 @@ __global__ void __launch_bounds__(128) k_attn(const __nv_bfloat16* __restrict__ 
             cp_async16(sV + buf * kAK * HD + swz(r, cc, HD), vbase + off, ok);
         }
     };
-    load_kv(0, kbeg);
+    const bool prefix_first = kbeg + kAK <= seq_kv[b];
+    if (prefix_first) {  // the first sub-block lies in the cached prefix: fetch it early
+        load_kv(0, kbeg);
+        cp_async_commit();
+    }
+    pdl_wait();
+    for (int e = tid; e < kAQ * CPR; e += 128) {
+        int r = e / CPR, cc = (e % CPR) * 8;
+        cp_async16(sQ + swz(r, cc, HD), qbase + static_cast<size_t>(r < nq ? r : 0) * HD + cc, r < nq);
+    }
+    if (!prefix_first) load_kv(0, kbeg);
     cp_async_commit();
 
     constexpr int KS = HD / 16;  // k-steps of Q.K
@@ -405,20 +394,42 @@ __global__ void __launch_bounds__(128) k_attn(const __nv_bfloat16* __restrict__ 
         __syncthreads();
         if (s_last) {
             __threadfence();
+            // per-row split weights once (exp2(m_s - M) / L), then the weighted sum of
+            // the split outputs with independent float4 loads
+            float* wts = reinterpret_cast<float*>(smem_attn);  // [kAQ][kMaxSplit]: Q/K tiles are done
             const size_t sb = (static_cast<size_t>(b) * H + h) * nsplit * T + q0;
-            const int qd = H * HD;
-            for (int e = tid; e < nq * HD; e += 128) {
-                const int r = e / HD, i = e - r * HD;
+            for (int r = tid; r < nq; r += 128) {
                 float M = -INFINITY;
-                for (int sp = 0; sp < ns; ++sp) M = fmaxf(M, __ldcg(part_ml + (sb + static_cast<size_t>(sp) * T + r) * 2));
-                float L = 0.0f, acc = 0.0f;
+                for (int sp = 0; sp < ns; ++sp)
+                    M = fmaxf(M, __ldcg(part_ml + (sb + static_cast<size_t>(sp) * T + r) * 2));
+                float L = 0.0f;
                 for (int sp = 0; sp < ns; ++sp) {
                     const size_t row = sb + static_cast<size_t>(sp) * T + r;
                     const float w = exp2f(__ldcg(part_ml + row * 2) - M);
+                    wts[r * kMaxSplit + sp] = w;
                     L += w * __ldcg(part_ml + row * 2 + 1);
-                    acc += w * __ldcg(part_o + row * HD + i);
                 }
-                out[(static_cast<size_t>(b) * T + q0 + r) * qd + h * HD + i] = __float2bfloat16_rn(acc / L);
+                const float inv = 1.0f / L;
+                for (int sp = 0; sp < ns; ++sp) wts[r * kMaxSplit + sp] *= inv;
+            }
+            __syncthreads();
+            const int qd = H * HD;
+            constexpr int V4 = HD / 4;
+            for (int e = tid; e < nq * V4; e += 128) {
+                const int r = e / V4, i4 = e - r * V4;
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int sp = 0; sp < ns; ++sp) {
+                    const float w = wts[r * kMaxSplit + sp];
+                    const float4 o4 = __ldcg(reinterpret_cast<const float4*>(
+                        part_o + (sb + static_cast<size_t>(sp) * T + r) * HD) + i4);
+                    acc.x += w * o4.x;
+                    acc.y += w * o4.y;
+                    acc.z += w * o4.z;
+                    acc.w += w * o4.w;
+                }
+                __nv_bfloat16* op = out + (static_cast<size_t>(b) * T + q0 + r) * qd + h * HD + i4 * 4;
+                *reinterpret_cast<__nv_bfloat162*>(op) = __floats2bfloat162_rn(acc.x, acc.y);
+                *reinterpret_cast<__nv_bfloat162*>(op + 2) = __floats2bfloat162_rn(acc.z, acc.w);
             }
         }
     }
@@ -430,11 +441,15 @@ cudaError_t attn_init_attrs() {
 }
 
 AttnPlan attn_plan(int B, int T, int H, int max_keys, int sms) {
+    // about one CTA per SM: splitting further only adds merge work (each split's
+    // 64-key sub-blocks already run back to back with a double-buffered prefetch)
     AttnPlan a;
     a.qtiles = (T + kAQ - 1) / kAQ;
-    int want = (2 * sms + B * H * a.qtiles - 1) / (B * H * a.qtiles);
+    const int units = B * H * a.qtiles;
+    int want = sms / units;
     const int blocks64 = (max_keys + kAK - 1) / kAK;
     if (want > blocks64) want = blocks64;
+    if (want > kMaxSplit) want = kMaxSplit;
     if (want < 1) want = 1;
     a.chunk = ((blocks64 + want - 1) / want) * kAK;
     a.nsplit = (max_keys + a.chunk - 1) / a.chunk;

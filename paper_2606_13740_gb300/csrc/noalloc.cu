@@ -20,8 +20,8 @@ void dllm_set_noctx_error(const char* msg);
 namespace {
 
 constexpr size_t kNoAllocScratchBytes = size_t(8) << 20;   // 8 MiB per GPU
-constexpr size_t kTicketBytes = 64 << 10;                  // tickets + status word at the front
-constexpr int kMaxTickets = (kTicketBytes - 256) / 4;      // tiles x token tiles
+constexpr size_t kTicketBytes = 256 << 10;                 // tickets + status word at the front
+constexpr int kMaxTickets = (kTicketBytes - 256) / 128;    // tiles x token tiles, one per 128-byte line
 constexpr int kMaxDevices = 64;
 
 __device__ __align__(256) unsigned char g_gemm_scratch[kNoAllocScratchBytes];
@@ -86,7 +86,7 @@ extern "C" int dllm_op_gemm_noalloc(const void* W, const void* X, float* D, int 
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     // the array keeps the previous call's contents: start tickets and status at zero
     if (cudaMemsetAsync(s, 0, kTicketBytes, st) != cudaSuccess) return noalloc_fail(DLLM_ECUDA, "memset failed");
-    Scratch scr{partials, tickets, (kNoAllocScratchBytes - kTicketBytes) / sizeof(float), kMaxTickets};
+    Scratch scr{partials, tickets, (kNoAllocScratchBytes - kTicketBytes) / sizeof(float), kMaxTickets * 32};
     EpiArgs ep{};
     ep.out = D;
     ep.ld_out = M;

@@ -60,7 +60,7 @@ int finish(cudaStream_t st, int* status_dev) {
 extern "C" {
 
 static int gemm_impl(const void* W, const void* X, float* D, int M, int N, int K, int grid, int reps, float* ms,
-                     void* stream) {
+                     void* stream, unsigned long long* trace_host = nullptr, int* grid_out = nullptr, int flags = 0) {
     if (!W || !X || !D || M < 1 || N < 1 || K < 1 || (K * 2) % 16 || reps < 1)
         return op_fail(DLLM_EINVAL, "bad gemm arguments");
     cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -74,7 +74,7 @@ static int gemm_impl(const void* W, const void* X, float* D, int M, int N, int K
         return op_fail(DLLM_EINVAL, "tensor map encode failed (alignment?)");
     DevBuf part, cnt, status;
     const size_t pf = static_cast<size_t>(p.grid) * 2 * p.ntile * 128;
-    const int cl = p.m_tiles * p.n_tiles;
+    const int cl = p.m_tiles * p.n_tiles * 32;
     if (!part.alloc(pf * 4) || !cnt.alloc(static_cast<size_t>(cl) * 4) || !status.alloc(16))
         return op_fail(DLLM_ENOMEM, "scratch allocation failed");
     if (cudaMemsetAsync(cnt.p, 0, static_cast<size_t>(cl) * 4, st) != cudaSuccess ||
@@ -84,6 +84,12 @@ static int gemm_impl(const void* W, const void* X, float* D, int M, int N, int K
     EpiArgs ep{};
     ep.out = D;
     ep.ld_out = M;
+    DevBuf tr;
+    if (trace_host) {
+        if (!tr.alloc(static_cast<size_t>(p.grid) * 16 * 8)) return op_fail(DLLM_ENOMEM, "trace allocation failed");
+        ep.trace = static_cast<unsigned long long*>(tr.p);
+    }
+    if (grid_out) *grid_out = p.grid;
     cudaEvent_t e0 = nullptr, e1 = nullptr;
     if (ms && (cudaEventCreate(&e0) != cudaSuccess || cudaEventCreate(&e1) != cudaSuccess))
         return op_fail(DLLM_ECUDA, "event creation failed");
@@ -92,6 +98,9 @@ static int gemm_impl(const void* W, const void* X, float* D, int M, int N, int K
         // one untimed launch first (instruction and descriptor caches)
         e = gemm_launch(EPI_F32, p, tw, tx, ep, scr, static_cast<int*>(status.p), st);
         if (e == cudaSuccess) e = cudaEventRecord(e0, st);
+        // flags bit 0: the timed launches form a programmatic-dependent-launch chain (each one
+        // only follows this library's own GEMM, which writes neither operand)
+        p.pdl = (flags & 1) != 0;
     }
     for (int r = 0; r < reps && e == cudaSuccess; ++r)
         e = gemm_launch(EPI_F32, p, tw, tx, ep, scr, static_cast<int*>(status.p), st);
@@ -104,6 +113,9 @@ static int gemm_impl(const void* W, const void* X, float* D, int M, int N, int K
         cudaEventElapsedTime(&t, e0, e1);
         *ms = t / reps;
     }
+    if (rc == DLLM_OK && trace_host &&
+        cudaMemcpy(trace_host, tr.p, static_cast<size_t>(p.grid) * 16 * 8, cudaMemcpyDeviceToHost) != cudaSuccess)
+        rc = op_fail(DLLM_ECUDA, "trace copy failed");
     if (e0) cudaEventDestroy(e0);
     if (e1) cudaEventDestroy(e1);
     return rc;
@@ -113,10 +125,19 @@ int dllm_op_gemm(const void* W, const void* X, float* D, int M, int N, int K, in
     return gemm_impl(W, X, D, M, N, K, grid, 1, nullptr, stream);
 }
 
-int dllm_op_gemm_timed(const void* W, const void* X, float* D, int M, int N, int K, int grid, int reps,
+int dllm_op_gemm_timed(const void* W, const void* X, float* D, int M, int N, int K, int grid, int reps, int flags,
                        float* ms_per_launch, void* stream) {
     if (!ms_per_launch) return op_fail(DLLM_EINVAL, "null output");
-    return gemm_impl(W, X, D, M, N, K, grid, reps, ms_per_launch, stream);
+    set_stream_smem(!(flags & 2));
+    int rc = gemm_impl(W, X, D, M, N, K, grid, reps, ms_per_launch, stream, nullptr, nullptr, flags);
+    set_stream_smem(true);
+    return rc;
+}
+
+int dllm_op_gemm_trace(const void* W, const void* X, float* D, int M, int N, int K, int grid, int reps,
+                       float* ms_per_launch, unsigned long long* trace, int* grid_used, void* stream) {
+    if (!ms_per_launch || !trace || !grid_used) return op_fail(DLLM_EINVAL, "null output");
+    return gemm_impl(W, X, D, M, N, K, grid, reps, ms_per_launch, stream, trace, grid_used);
 }
 
 int dllm_op_attention(const void* q, const void* kc, const void* vc, const int32_t* kv_len, void* out, int B, int T,
@@ -159,7 +180,7 @@ int dllm_op_lmhead(const void* W, const void* X, const int32_t* cur, int32_t* x0
         return op_fail(DLLM_EINVAL, "tensor map encode failed (alignment?)");
     DevBuf part, cnt, status, lmp, zc;
     const size_t pf = static_cast<size_t>(p.grid) * 2 * p.ntile * 128;
-    const int cl = p.m_tiles * p.n_tiles;
+    const int cl = p.m_tiles * p.n_tiles * 32;
     if (!part.alloc(pf * 4) || !cnt.alloc(static_cast<size_t>(cl) * 4) || !status.alloc(16) ||
         !lmp.alloc(static_cast<size_t>(p.m_tiles) * N * 3 * 4) || !zc.alloc(static_cast<size_t>(N) * 4))
         return op_fail(DLLM_ENOMEM, "scratch allocation failed");

@@ -76,9 +76,11 @@ SIGNATURES = {
     "dllm_set_profile": (_I, [_P, _I]),
     "dllm_get_profile": (_I, [_P, _P, _P, _P]),
     "dllm_launches_per_step": (_I, [_P, _P]),
+    "dllm_get_trace": (_I, [_P, _P, _I, _P]),
     "dllm_op_gemm": (_I, [_P, _P, _P, _I, _I, _I, _I, _P]),
     "dllm_op_gemm_noalloc": (_I, [_P, _P, _P, _I, _I, _I, _I, _P]),
-    "dllm_op_gemm_timed": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _P, _P]),
+    "dllm_op_gemm_trace": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P]),
+    "dllm_op_gemm_timed": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P]),
     "dllm_op_attention": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P]),
     "dllm_op_lmhead": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _P]),
     "dllm_op_commit": (_I, [_P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _I, _F, _F, _I, _I, _I, _I, _I, _P]),
@@ -289,6 +291,12 @@ class Context:
         return {k: {"ms_total": float(ms[i]), "launches_per_step": int(launches[i])} for i, k in
                 enumerate(self.KINDS)}, int(steps[0])
 
+    def dllm_get_trace(self, max_launches=512):
+        out = np.zeros((max_launches, 256, 16), np.uint64)
+        n = np.zeros(1, np.int32)
+        _check(lib().dllm_get_trace(self.h, _p(out), max_launches, _p(n)), self.h)
+        return out[: int(n[0])]
+
     def dllm_launches_per_step(self):
         n = np.zeros(1, np.int32)
         _check(lib().dllm_launches_per_step(self.h, _p(n)), self.h)
@@ -331,15 +339,28 @@ def dllm_op_gemm_noalloc(W, X, D, M, N, K, grid=0, stream=None):
     return D
 
 
-def dllm_op_gemm_timed(W, X, M, N, K, reps, grid=0, stream=None):
-    """Average kernel time (ms) of `reps` back-to-back launches, and D."""
+def dllm_op_gemm_timed(W, X, M, N, K, reps, grid=0, flags=0, stream=None):
+    """Average kernel time (ms) of `reps` back-to-back launches, and D (flags: see dllm_ops.h)."""
     import torch
 
     D = torch.empty((N, M), dtype=torch.float32, device=W.device)
     ms = C.c_float()
     _check(lib().dllm_op_gemm_timed(_p(W.data_ptr()), _p(X.data_ptr()), _p(D.data_ptr()), M, N, K, grid, reps,
-                                    C.byref(ms), _p(_stream_ptr(stream))))
+                                    flags, C.byref(ms), _p(_stream_ptr(stream))))
     return ms.value, D
+
+
+def dllm_op_gemm_trace(W, X, M, N, K, reps, grid=0, stream=None):
+    """(ms per launch, per-CTA timeline [grid][8] of the last launch)."""
+    import torch
+
+    D = torch.empty((N, M), dtype=torch.float32, device=W.device)
+    ms = C.c_float()
+    used = C.c_int()
+    tr = np.zeros((1024, 16), np.uint64)
+    _check(lib().dllm_op_gemm_trace(_p(W.data_ptr()), _p(X.data_ptr()), _p(D.data_ptr()), M, N, K, grid, reps,
+                                    C.byref(ms), _p(tr), C.byref(used), _p(_stream_ptr(stream))))
+    return ms.value, tr[:used.value]
 
 
 def dllm_op_attention(q, kc, vc, kv_len, B, T, H, hd, cap, max_kv_len, stream=None):
