@@ -314,6 +314,198 @@ __device__ __forceinline__ void epilogue_chunk(const EpiArgs& ep, const GemmPlan
     }
 }
 
+// Epilogue of a 32-token tile (the batch-1 weight stream), compact: one rolled loop over 8
+// groups of 4 columns read from TMEM (t_src; for the residual, the old x of the tile was
+// staged at t_x before the accumulator was ready), so its code stays small and no global load
+// waits on a store.
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
+    return v;
+}
+
+template <int EPI>
+__device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& p, int mt, int nt, int rt,
+                                             uint32_t t_src, uint32_t t_x, const EpiSmem& sm, int ew, int quarter,
+                                             int lane, int* status) {
+    const int row = mt * kBM + rt;
+    const int col0 = nt * 32;
+    const bool scale = (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) && ep.sq_in != nullptr;
+    // QKV state: feature, head, rotation (angle-addition recurrence along the positions)
+    int part = 0, hh = 0, pp = 0, fi = 0, bl = 0;
+    bool run = true;
+    float cn = 1.0f, sn = 0.0f, cd = 1.0f, sd = 0.0f, theta = 0.0f;
+    if constexpr (EPI == EPI_QKV) {
+        const int qd = ep.H * ep.hd;
+        part = row / qd;
+        const int f = row - part * qd;
+        hh = f / ep.hd;
+        pp = f - hh * ep.hd;
+        fi = (pp >> 1) + (pp & 1) * (ep.hd >> 1);
+        theta = sm.theta[rt];
+        bl = col0 / ep.T;
+        run = min(col0 + 31, p.N - 1) / ep.T == bl;
+        if (part < 2 && run) {
+            const float2 a = rot_cs(static_cast<float>(sm.kvs[bl] + (col0 - bl * ep.T)) * theta);
+            const float2 d = rot_cs(theta);
+            cn = a.x;
+            sn = a.y;
+            cd = d.x;
+            sd = d.y;
+        }
+    }
+#pragma unroll 1
+    for (int g = 0; g < 8; ++g) {
+        float a[4];
+        tmem_ld_32x4(t_src + static_cast<uint32_t>(4 * g), a);
+        if (scale) {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) a[u] *= sm.rs[4 * g + u];
+        }
+        if constexpr (EPI == EPI_F32) {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int col = col0 + 4 * g + u;
+                if (row < p.M && col < p.N) ep.out[static_cast<size_t>(col) * ep.ld_out + row] = a[u];
+            }
+        } else if constexpr (EPI == EPI_RESID) {
+            float xo[4];
+            tmem_ld_32x4(t_x + static_cast<uint32_t>(4 * g), xo);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int col = col0 + 4 * g + u;
+                float x = 0.0f;
+                if (row < p.M && col < p.N) {
+                    const size_t o = static_cast<size_t>(col) * ep.ld_out + row;
+                    x = xo[u] + a[u];
+                    ep.out[o] = x;
+                    ep.xb[o] = __float2bfloat16_rn(x);
+                }
+                const float s = warp_sum(x * x);
+                if (lane == 0) sm.red[quarter * 32 + 4 * g + u] = s;
+            }
+        } else if constexpr (EPI == EPI_QKV) {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const float xp = __shfl_xor_sync(0xffffffffu, a[u], 1);
+                const int col = col0 + 4 * g + u;
+                if (col < p.N) {
+                    const int b = run ? bl : col / ep.T;
+                    const int t = col - b * ep.T;
+                    const int pos = sm.kvs[b] + t;
+                    if (pos < 0 || pos >= ep.cap) {
+                        atomicOr(status, kStatusBadIndex);
+                    } else {
+                        float x = a[u];
+                        if (part < 2) {
+                            if (!run) {
+                                const float2 r = rot_cs(static_cast<float>(pos) * theta);
+                                cn = r.x;
+                                sn = r.y;
+                            }
+                            x = (pp & 1) ? (x * cn + xp * sn) : (x * cn - xp * sn);
+                        }
+                        const __nv_bfloat16 y = __float2bfloat16_rn(x);
+                        if (part == 0) {
+                            ep.q[((static_cast<size_t>(b) * ep.H + hh) * ep.T + t) * ep.hd + fi] = y;
+                        } else {
+                            __nv_bfloat16* c = part == 1 ? ep.kc : ep.vc;
+                            c[((static_cast<size_t>(b) * ep.H + hh) * ep.cap + pos) * ep.hd + fi] = y;
+                        }
+                    }
+                }
+                if (run) {
+                    const float c2 = cn * cd - sn * sd;
+                    sn = sn * cd + cn * sd;
+                    cn = c2;
+                }
+            }
+        } else if constexpr (EPI == EPI_SWIGLU) {
+            const int f = mt * 64 + (rt >> 1);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const float up = __shfl_xor_sync(0xffffffffu, a[u], 1);
+                const int col = col0 + 4 * g + u;
+                if ((rt & 1) == 0 && f < ep.F && col < p.N) {
+                    const float gv = a[u];
+                    ep.h[static_cast<size_t>(col) * ep.F + f] = __float2bfloat16_rn(gv / (1.0f + __expf(-gv)) * up);
+                }
+            }
+        } else if constexpr (EPI == EPI_LMHEAD) {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int col = col0 + 4 * g + u;
+                const bool ok = row < ep.V && row != ep.mask_id;
+                if (ep.logits && row < ep.V && col < p.N) ep.logits[static_cast<size_t>(col) * ep.V + row] = a[u];
+                // this warp's (max, argmax, sum exp) over its 32 rows
+                float m = ok ? a[u] : -INFINITY;
+                int idx = ok ? row : INT_MAX;
+#pragma unroll
+                for (int off = 16; off > 0; off >>= 1) {
+                    const float om = __shfl_xor_sync(0xffffffffu, m, off);
+                    const int oi = __shfl_xor_sync(0xffffffffu, idx, off);
+                    if (om > m || (om == m && oi < idx)) {
+                        m = om;
+                        idx = oi;
+                    }
+                }
+                const float s = warp_sum((ok && m != -INFINITY) ? __expf(a[u] - m) : 0.0f);
+                if (lane == 0) {
+                    sm.red[(quarter * 32 + 4 * g + u) * 3] = m;
+                    sm.red[(quarter * 32 + 4 * g + u) * 3 + 1] = s;
+                    sm.red[(quarter * 32 + 4 * g + u) * 3 + 2] = __int_as_float(idx);
+                }
+                if (col < p.N && row == sm.kvs[col]) ep.zcur[col] = a[u];  // current ids staged in kvs
+            }
+        }
+    }
+    if constexpr (EPI == EPI_RESID) {
+        named_bar(1, 128);
+        if (ew == 0) {
+            const int col = col0 + lane;
+            if (col < p.N)
+                ep.sq_out[static_cast<size_t>(mt) * p.N + col] =
+                    ((sm.red[lane] + sm.red[32 + lane]) + sm.red[64 + lane]) + sm.red[96 + lane];
+        }
+        named_bar(1, 128);
+    } else if constexpr (EPI == EPI_LMHEAD) {
+        named_bar(1, 128);
+        if (ew == 0) {  // merge the four row quarters in a fixed order
+            const int col = col0 + lane;
+            float m = -INFINITY, s = 0.0f;
+            int idx = INT_MAX;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const float* r = sm.red + (q * 32 + lane) * 3;
+                const float m2 = r[0], s2 = r[1];
+                const int i2 = __float_as_int(r[2]);
+                if (m2 == -INFINITY) continue;
+                if (m == -INFINITY) {
+                    m = m2;
+                    s = s2;
+                    idx = i2;
+                } else if (m2 > m) {
+                    s = s * __expf(m - m2) + s2;
+                    m = m2;
+                    idx = i2;
+                } else if (m2 == m) {
+                    s += s2;
+                    idx = min(idx, i2);
+                } else {
+                    s += s2 * __expf(m2 - m);
+                }
+            }
+            if (col < p.N) {
+                float* o = ep.lm_part + (static_cast<size_t>(col) * p.m_tiles + mt) * 3;
+                o[0] = m;
+                o[1] = s;
+                o[2] = __int_as_float(idx);
+            }
+        }
+        named_bar(1, 128);
+    }
+}
+
 // ------------------------------------------------------------------ kernel
 template <int EPI>
 __global__ void __launch_bounds__(kThreads, 2)
@@ -515,8 +707,16 @@ __global__ void __launch_bounds__(kThreads, 2)
             esm.theta[rt] = ep.theta[(rt % ep.hd) >> 1];
             named_bar(1, 128);
         }
+        if constexpr (EPI == EPI_LMHEAD) {
+            if (p.ntile == 32) {  // the window's current ids, for the compact epilogue
+                for (int c = ew * 32 + lane; c < p.N && c < 256; c += 128) esm.kvs[c] = ep.cur_tok[c];
+                named_bar(1, 128);
+            }
+        }
         const int nchunks = p.ntile / 32;
         const size_t slot_floats = static_cast<size_t>(p.ntile) * kBM;
+        const bool c32 = p.ntile == 32;  // batch-1 weight stream: compact TMEM-sourced epilogue
+        const uint32_t t_x = tmem_base + static_cast<uint32_t>(2 * p.acc_cols) + (static_cast<uint32_t>(quarter * 32) << 16);
         int acc = 0;
         uint32_t acc_phase = 0;
         uint32_t red_phase = 0;
@@ -529,12 +729,24 @@ __global__ void __launch_bounds__(kThreads, 2)
             const int k_hi = static_cast<int>((it1 < tend ? it1 : tend) - tile * p.kb);
             const int mt = static_cast<int>(tile / p.n_tiles);
             const int nt = static_cast<int>(tile - static_cast<long long>(mt) * p.n_tiles);
+            const bool whole = (k_lo == 0 && k_hi == p.kb);
             if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
                 // the operand's RMSNorm scale only needs the previous kernel: computed while the
                 // accumulator is still being produced
                 if (ep.sq_in && nt != rs_nt) {
                     compute_norm_scale(ep, p, nt, esm, ew * 32 + lane);
                     rs_nt = nt;
+                }
+            }
+            if constexpr (EPI == EPI_RESID) {
+                if (c32) {  // stage the tile's old residual in TMEM while the accumulator is produced
+                    const int row = mt * kBM + rt;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const int col = nt * 32 + j;
+                        v[j] = (row < p.M && col < p.N) ? ep.out[static_cast<size_t>(col) * ep.ld_out + row] : 0.0f;
+                    }
+                    tmem_st_32x32(t_x, v);
                 }
             }
             mbar_wait(&tfull[acc], acc_phase, s_abort, status);
@@ -547,27 +759,28 @@ __global__ void __launch_bounds__(kThreads, 2)
             tc_fence_after();
             const uint32_t t_acc = tmem_base + static_cast<uint32_t>(acc * p.acc_cols) +
                                    (static_cast<uint32_t>(quarter * 32) << 16);
-            const bool whole = (k_lo == 0 && k_hi == p.kb);
             const int slot = (range_begin(blockIdx.x, p.total, G) / p.kb == tile) ? 0 : 1;
             float* my_part = partials + (static_cast<size_t>(blockIdx.x) * 2 + slot) * slot_floats;
-            for (int c = 0; c < nchunks; ++c) {
-                tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);
-                if (whole) {
-                    epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
-                } else {
-                    // float4 (c*8 + j, row): coalesced here, conflict-free when the reducer stages it
-                    float4* dst = reinterpret_cast<float4*>(my_part);
+            if (whole && c32) {
+                epilogue_c32<EPI>(ep, p, mt, nt, rt, t_acc, t_x, esm, ew, quarter, lane, status);
+            } else {
+                for (int c = 0; c < nchunks; ++c) {
+                    tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);
+                    if (whole) {
+                        epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
+                    } else {
+                        // float4 (c*8 + j, row): coalesced here, conflict-free when the reducer stages it
+                        float4* dst = reinterpret_cast<float4*>(my_part);
 #pragma unroll
-                    for (int j = 0; j < 8; ++j)
-                        dst[static_cast<size_t>(c * 8 + j) * kBM + rt] =
-                            make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+                        for (int j = 0; j < 8; ++j)
+                            dst[static_cast<size_t>(c * 8 + j) * kBM + rt] =
+                                make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+                    }
                 }
             }
-            tc_fence_before();
-            mbar_arrive(&tempty[acc]);
-            if (++acc == 2) {
-                acc = 0;
-                acc_phase ^= 1u;
+            if (!c32) {  // wide tiles release the accumulator as soon as it is read
+                tc_fence_before();
+                mbar_arrive(&tempty[acc]);
             }
             if (!whole) {
                 // last-arriver reduction of a tile split between CTAs
@@ -596,46 +809,42 @@ __global__ void __launch_bounds__(kThreads, 2)
                     const uint32_t part_bytes = static_cast<uint32_t>(slot_floats * 4);
                     const uint32_t stage_room = static_cast<uint32_t>(S) * (kABytes + b_bytes);
                     const bool final_seg = tile * p.kb + k_hi == it1;  // pipeline drained: stage memory free
-                    if (final_seg && nchunks == 1 && part_bytes <= stage_room) {
-                        // one round trip: bulk-copy every partial into the stage memory at once
-                        const int per_batch = static_cast<int>(stage_room / part_bytes);
+                    for (int c = 0; c < nchunks; ++c) {
 #pragma unroll
                         for (int j = 0; j < 32; ++j) v[j] = 0.0f;
-                        for (int b0 = 0; b0 < nparts; b0 += per_batch) {
-                            const int nb = nparts - b0 < per_batch ? nparts - b0 : per_batch;
-                            if (threadIdx.x == 64) {
-                                fence_proxy_async_global();
-                                mbar_arrive_expect_tx(redbar, part_bytes * static_cast<uint32_t>(nb));
+                        if (final_seg && c32 && part_bytes <= stage_room) {
+                            // one round trip: bulk-copy every partial into the stage memory at once
+                            const int per_batch = static_cast<int>(stage_room / part_bytes);
+                            for (int b0 = 0; b0 < nparts; b0 += per_batch) {
+                                const int nb = nparts - b0 < per_batch ? nparts - b0 : per_batch;
+                                if (threadIdx.x == 64) {
+                                    fence_proxy_async_global();
+                                    mbar_arrive_expect_tx(redbar, part_bytes * static_cast<uint32_t>(nb));
+                                    for (int q = 0; q < nb; ++q) {
+                                        const int cc = c_first + b0 + q;
+                                        const int sl = (range_begin(cc, p.total, G) / p.kb == tile) ? 0 : 1;
+                                        bulk_load(smem + static_cast<size_t>(q) * part_bytes,
+                                                  partials + (static_cast<size_t>(cc) * 2 + sl) * slot_floats,
+                                                  part_bytes, redbar);
+                                    }
+                                }
+                                mbar_wait(redbar, red_phase, s_abort, status);
+                                red_phase ^= 1u;
                                 for (int q = 0; q < nb; ++q) {
-                                    const int cc = c_first + b0 + q;
-                                    const int sl = (range_begin(cc, p.total, G) / p.kb == tile) ? 0 : 1;
-                                    bulk_load(smem + static_cast<size_t>(q) * part_bytes,
-                                              partials + (static_cast<size_t>(cc) * 2 + sl) * slot_floats, part_bytes,
-                                              redbar);
-                                }
-                            }
-                            mbar_wait(redbar, red_phase, s_abort, status);
-                            red_phase ^= 1u;
-                            for (int q = 0; q < nb; ++q) {
-                                const float4* src =
-                                    reinterpret_cast<const float4*>(smem + static_cast<size_t>(q) * part_bytes);
+                                    const float4* src =
+                                        reinterpret_cast<const float4*>(smem + static_cast<size_t>(q) * part_bytes);
 #pragma unroll
-                                for (int j = 0; j < 8; ++j) {
-                                    const float4 a = src[j * kBM + rt];
-                                    v[4 * j] += a.x;
-                                    v[4 * j + 1] += a.y;
-                                    v[4 * j + 2] += a.z;
-                                    v[4 * j + 3] += a.w;
+                                    for (int j = 0; j < 8; ++j) {
+                                        const float4 a = src[j * kBM + rt];
+                                        v[4 * j] += a.x;
+                                        v[4 * j + 1] += a.y;
+                                        v[4 * j + 2] += a.z;
+                                        v[4 * j + 3] += a.w;
+                                    }
                                 }
+                                named_bar(1, 128);  // the next batch overwrites the staging memory
                             }
-                            named_bar(1, 128);  // the next batch overwrites the staging memory
-                        }
-                        if (tr && threadIdx.x == 64) tr[kTrReduced] = global_ns();
-                        epilogue_chunk<EPI>(ep, p, mt, nt, 0, rt, v, esm, ew, quarter, lane, status);
-                    } else {
-                        for (int c = 0; c < nchunks; ++c) {
-#pragma unroll
-                            for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+                        } else {
                             // partials in k order (each one's 8 loads in flight together)
                             for (int cc = c_first; cc <= c_last; ++cc) {
                                 const int sl0 = (range_begin(cc, p.total, G) / p.kb == tile) ? 0 : 1;
@@ -652,11 +861,24 @@ __global__ void __launch_bounds__(kThreads, 2)
                                     v[4 * j + 3] += a[j].w;
                                 }
                             }
-                            if (tr && threadIdx.x == 64 && c == 0) tr[kTrReduced] = global_ns();
+                        }
+                        if (tr && threadIdx.x == 64 && c == 0) tr[kTrReduced] = global_ns();
+                        if (c32) {
+                            tmem_st_32x32(t_acc, v);  // the sum goes back into the (still owned) accumulator
+                            epilogue_c32<EPI>(ep, p, mt, nt, rt, t_acc, t_x, esm, ew, quarter, lane, status);
+                        } else {
                             epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
                         }
                     }
                 }
+            }
+            if (c32) {
+                tc_fence_before();
+                mbar_arrive(&tempty[acc]);
+            }
+            if (++acc == 2) {
+                acc = 0;
+                acc_phase ^= 1u;
             }
             it = tile * p.kb + k_hi;
         }
@@ -694,7 +916,8 @@ GemmPlan gemm_plan(int M, int N, int K, int grid_max, int epi) {
     p.grid = static_cast<int>(p.total < grid_max ? p.total : grid_max);
     if (p.grid < 1) p.grid = 1;
     p.acc_cols = pow2ceil(p.ntile);
-    p.tmem_cols = 2 * p.acc_cols;
+    // 32-token tiles also keep the residual's old values in 32 extra columns
+    p.tmem_cols = pow2ceil(2 * p.acc_cols + (p.ntile == 32 ? 32 : 0));
     const int staging = epi == EPI_LMHEAD ? kBM * kStageLd * 4 : 0;
     const int fixed = 1024 + (256 + 1024 + 256 + 128) * 4 + staging + 64 * 8 + 64;
     const int stage_bytes = static_cast<int>(kABytes) + p.ntile * kBK * 2;
