@@ -213,9 +213,12 @@ int dllm_set_profile(dllm_ctx* ctx, int enable);
  * steps profiled (any pointer may be NULL). */
 int dllm_get_profile(dllm_ctx* ctx, double* ms_total, int32_t* launches_per_step, int32_t* steps);
 
-/* With dllm_set_debug(16): per-CTA timelines (%globaltimer stamps, see
- * dllm_op_gemm_trace) of the GEMM launches of the last step, in launch order:
- * out [n_launches][256][16].  Synchronises. */
+/* With dllm_set_debug(16): per-CTA timelines (%globaltimer stamps) of the
+ * GEMM and attention launches of the last step, in launch order: out
+ * [n_launches][256][16].  GEMM slots as in dllm_op_gemm_trace; attention
+ * slots 0 start, 1 dependency wait passed, 2 key loop done, 3 split ticket
+ * taken, 4 merge done (last split only), 5 SM id, 6 last split.
+ * Synchronises. */
 int dllm_get_trace(dllm_ctx* ctx, unsigned long long* out, int max_launches, int32_t* n_launches);
 
 /* Kernel launches in the last denoising step (all kinds). */

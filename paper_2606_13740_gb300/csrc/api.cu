@@ -34,9 +34,8 @@ int rup(int x, int m) { return (x + m - 1) / m * m; }
 struct Layout {
     int qd, qkv_rows, gu_rows, d_rows, o_rows, head_rows, head_tiles, max_tok;
     size_t off_w, per_layer, off_emb, off_head, off_kv, kv_half;
-    size_t off_x, off_xn, off_q, off_attn, off_h, off_sq, off_actr, off_theta;
-    int n_sq, actr_len;
-    size_t off_apo, apo_floats, off_apml;
+    size_t off_x, off_xn, off_q, off_attn, off_h, off_sq, off_theta;
+    int n_sq;
     size_t off_lmp, off_zcur, off_cur, off_x0, off_conf, off_tokconf;
     size_t off_part, part_floats, off_cnt;
     int cnt_len;
@@ -80,14 +79,7 @@ Layout make_layout(const dllm_config& c) {
     L.off_h = take(T * F * 2);
     L.n_sq = (d + 127) / 128;
     L.off_sq = take(static_cast<size_t>(L.n_sq) * T * 4);
-    L.actr_len = c.max_batch * H * ((c.max_window + 63) / 64);
-    L.off_actr = take(static_cast<size_t>(L.actr_len) * 4);
     L.off_theta = take(static_cast<size_t>(hd / 2) * 4);
-    // attention split partials: B*H*nsplit*T rows, nsplit <= 2*SMs/(B*H*qtiles) + 1
-    const size_t rows = static_cast<size_t>(2 * kMaxSMs) * 64 + static_cast<size_t>(c.max_batch) * H * c.max_window;
-    L.apo_floats = rows * hd;
-    L.off_apo = take(L.apo_floats * 4);
-    L.off_apml = take(rows * 2 * 4);
     L.off_lmp = take(static_cast<size_t>(L.head_tiles) * T * 3 * 4);
     L.off_zcur = take(T * 4);
     L.off_cur = take(T * 4);
@@ -148,8 +140,7 @@ struct dllm_ctx {
     __nv_bfloat16 *xn = nullptr, *q = nullptr, *attn = nullptr, *h = nullptr;
     float* sq = nullptr;      // RMSNorm statistics [d/128][tokens]
     float* theta = nullptr;   // RoPE frequencies [hd/2]
-    int* actr = nullptr;      // attention split tickets
-    float *apo = nullptr, *apml = nullptr, *lmp = nullptr, *zcur = nullptr, *conf = nullptr, *tokconf = nullptr;
+    float *lmp = nullptr, *zcur = nullptr, *conf = nullptr, *tokconf = nullptr;
     int *cur = nullptr, *x0 = nullptr;
     Scratch scr{};
     int *tok = nullptr, *stok = nullptr, *seq_kv = nullptr, *plan = nullptr, *outs = nullptr, *status = nullptr;
@@ -264,9 +255,6 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
         !make_tmap_bf16(&tx_h, ctx->h, N, F, pd.ntile))
         return fail(ctx, DLLM_ECUDA, "tensor map encode failed");
     const AttnPlan ap = attn_plan(B, T, c.n_heads, ctx->kv_len + T, ctx->sms);
-    if (static_cast<size_t>(B) * c.n_heads * ap.nsplit * T * c.head_dim > L.apo_floats ||
-        B * c.n_heads * ap.qtiles > L.actr_len)
-        return fail(ctx, DLLM_ECAPACITY, "attention partial buffer too small");
     EpiArgs ep{};
     ep.seq_kv = ctx->seq_kv;
     ep.n_seq = B;
@@ -295,8 +283,8 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
         ep.trace = next_trace(ctx);
         CK(gemm_launch(EPI_QKV, pq, ctx->tm_qkv[l], tx_xn, ep, ctx->scr, ctx->status, s));
         mark(ctx, DLLM_K_QKV);
-        CK(launch_attention(ctx->q, kc, vc, ctx->seq_kv, ctx->apo, ctx->apml, ctx->actr, ctx->attn, B, T, c.n_heads,
-                            c.head_dim, c.max_ctx, ap, s));
+        CK(launch_attention(ctx->q, kc, vc, ctx->seq_kv, ctx->attn, B, T, c.n_heads, c.head_dim, c.max_ctx, ap, s,
+                            true, next_trace(ctx)));
         mark(ctx, DLLM_K_ATTN);
         er.trace = next_trace(ctx);
         CK(gemm_launch(EPI_RESID, po, ctx->tm_o[l], tx_attn, er, ctx->scr, ctx->status, s));
@@ -459,10 +447,7 @@ int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void*
     ctx->attn = reinterpret_cast<__nv_bfloat16*>(A + L.off_attn);
     ctx->h = reinterpret_cast<__nv_bfloat16*>(A + L.off_h);
     ctx->sq = reinterpret_cast<float*>(A + L.off_sq);
-    ctx->actr = reinterpret_cast<int*>(A + L.off_actr);
     ctx->theta = reinterpret_cast<float*>(A + L.off_theta);
-    ctx->apo = reinterpret_cast<float*>(A + L.off_apo);
-    ctx->apml = reinterpret_cast<float*>(A + L.off_apml);
     ctx->lmp = reinterpret_cast<float*>(A + L.off_lmp);
     ctx->zcur = reinterpret_cast<float*>(A + L.off_zcur);
     ctx->cur = reinterpret_cast<int*>(A + L.off_cur);

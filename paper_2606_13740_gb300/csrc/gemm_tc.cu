@@ -52,7 +52,7 @@ constexpr int kTicketStride = 32;  // one tile ticket per 128-byte line
 // Timeline trace slots per CTA (when EpiArgs::trace is set).
 enum { kTrStart = 0, kTrPrologue = 1, kTrFirstData = 2, kTrLastData = 3, kTrEpiDone = 4, kTrExit = 5, kTrSm = 6,
        kTrDepWait = 7, kTrAccReady = 8, kTrPartStored = 9, kTrTicket = 10, kTrReduced = 11, kTrIsLast = 12,
-       kTrTile = 13, kTrSlots = 16 };
+       kTrTile = 13, kTrEpiG0 = 14, kTrEpiLoop = 15, kTrSlots = 16 };
 
 __device__ __forceinline__ unsigned smid() {
     unsigned id;
@@ -354,8 +354,10 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
             sd = d.y;
         }
     }
+    unsigned long long* tr = (ep.trace && ew == 0 && lane == 0) ? ep.trace + static_cast<size_t>(blockIdx.x) * kTrSlots : nullptr;
 #pragma unroll 1
     for (int g = 0; g < 8; ++g) {
+        if (tr && g == 1) tr[kTrEpiG0] = global_ns();
         float a[4];
         tmem_ld_32x4(t_src + static_cast<uint32_t>(4 * g), a);
         if (scale) {
@@ -459,6 +461,7 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
             }
         }
     }
+    if (tr) tr[kTrEpiLoop] = global_ns();
     if constexpr (EPI == EPI_RESID) {
         named_bar(1, 128);
         if (ew == 0) {

@@ -118,18 +118,17 @@ cudaError_t launch_embed(const int* tok, int tok_ld, const int* seq_kv, const __
                          __nv_bfloat16* xb, float* sq, int* cur, int B, int T, int d, cudaStream_t st);
 // The kernels below are launched with PDL when `pdl` (inside the context's step chain); the
 // single-kernel entry points pass false because their inputs may come from foreign kernels.
-// Attention split plan: CTAs (split, head, sequence x 64-query tile), each over `chunk`
-// keys; with nsplit > 1 the splits leave fp32 partials part_o [B][H][nsplit][T][hd] and
-// part_ml [B][H][nsplit][T][2] and the last CTA of each (sequence, head, query tile) to
-// finish (ticket in counters [B][H][qtiles], zero between launches) merges them in order.
+// Attention plan: CTAs (split, head, sequence x query tile of 16*nw rows); the csize
+// splits of one (sequence, head, query tile) form a thread-block cluster and merge
+// their partials through distributed shared memory.
 struct AttnPlan {
-    int qtiles, chunk, nsplit;
+    int qtiles, nw, csize;
 };
 AttnPlan attn_plan(int B, int T, int H, int max_keys, int sms);
 cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
-                             const int* seq_kv, float* part_o, float* part_ml, int* counters,
-                             __nv_bfloat16* out, int B, int T, int H, int hd, int cap, const AttnPlan& a,
-                             cudaStream_t st, bool pdl = true);
+                             const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int hd, int cap,
+                             const AttnPlan& a, cudaStream_t st, bool pdl = true,
+                             unsigned long long* trace = nullptr);
 cudaError_t launch_lmhead_reduce(const float* lm_part, const float* zcur, const int* cur_tok, int m_tiles,
                                  int N, int mask_id, int* x0, float* conf, float* tokconf, cudaStream_t st,
                                  bool pdl = true);

@@ -145,14 +145,25 @@ cudaError_t launch_embed(const int* tok, int tok_ld, const int* seq_kv, const __
 // ------------------------------------------------------------------ attention
 // Bidirectional attention of T window queries per sequence over keys
 // [0, kv_len + T) of the KV cache (cached prefix, then the window's own keys
-// written by the QKV epilogue), flash style with split-KV: CTA (split, head,
-// sequence x 64-query tile) covers `chunk` keys in 64-key sub-blocks with an
-// online softmax on bf16 mma.sync tiles.  With one split it writes the output;
-// otherwise it leaves unnormalised partials and the last CTA of the (sequence,
-// head, query tile) to finish merges all splits in split order.
-constexpr int kAQ = 64;
-constexpr int kAK = 64;
-constexpr int kMaxSplit = 64;  // key splits per (sequence, head, query tile)
+// written by the QKV epilogue), flash style: online softmax over 64-key
+// sub-blocks on bf16 mma.sync tiles, NW warps of 16 query rows per CTA.
+//
+// Split-KV over a thread-block cluster: the csize CTAs of a cluster share one
+// (sequence, head, query tile) and take consecutive, balanced shares of its
+// key sub-blocks.  Each leaves its unnormalised output and (max, sum) per row
+// in its own shared memory; after a cluster barrier every CTA merges a slice
+// of the rows by reading all csize partials through distributed shared memory,
+// so the merge needs no global scratch, no fences and no atomics.
+constexpr int kAK = 64;      // keys per sub-block
+constexpr int kMaxCluster = 8;
+// attention timeline slots (%globaltimer ns)
+enum { kAtStart = 0, kAtDepWait = 1, kAtLoop = 2, kAtTicket = 3, kAtMerged = 4, kAtSm = 5, kAtLast = 6 };
+
+__device__ __forceinline__ unsigned smid_attn() {
+    unsigned r;
+    asm volatile("mov.u32 %0, %%smid;" : "=r"(r));
+    return r;
+}
 
 __device__ __forceinline__ int swz(int r, int c, int hd) {
     return r * hd + ((((c >> 3) ^ (r & 7))) << 3) + (c & 7);
@@ -190,30 +201,69 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
-template <int HD>
-__global__ void __launch_bounds__(128) k_attn(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ kc,
-                                              const __nv_bfloat16* __restrict__ vc, const int* __restrict__ seq_kv,
-                                              float* __restrict__ part_o, float* __restrict__ part_ml,
-                                              int* __restrict__ counters, __nv_bfloat16* __restrict__ out, int T,
-                                              int H, int cap, int chunk, int nsplit, int qtiles) {
+// ---- thread-block cluster helpers
+__device__ __forceinline__ void cluster_sync_all() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Address of the same shared-memory location in CTA `rank` of this cluster.
+__device__ __forceinline__ uint32_t dsmem_map(uint32_t saddr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ float2 dsmem_ld2(uint32_t addr) {
+    float2 v;
+    asm volatile("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(addr) : "memory");
+    return v;
+}
+__device__ __forceinline__ float4 dsmem_ld4(uint32_t addr) {
+    float4 v;
+    asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(addr)
+                 : "memory");
+    return v;
+}
+
+// Shared memory: Q tile [16*NW][HD], one K and one V sub-block [64][HD] (bf16,
+// XOR-swizzled 16-byte chunks).  The next sub-block's K streams in while this
+// one's softmax and P.V run, its V while the next Q.K^T runs.  After the key
+// loop the same memory holds the CTA's partial: O [16*NW][HD] fp32 and
+// (max, sum) [16*NW][2].
+template <int HD, int NW>
+__global__ void __launch_bounds__(NW * 32) k_attn(const __nv_bfloat16* __restrict__ q,
+                                                  const __nv_bfloat16* __restrict__ kc,
+                                                  const __nv_bfloat16* __restrict__ vc, const int* __restrict__ seq_kv,
+                                                  __nv_bfloat16* __restrict__ out, int T, int H, int cap, int qtiles,
+                                                  int csize, unsigned long long* trace) {
+    constexpr int AQ = NW * 16;  // query rows per CTA
+    constexpr int NT = NW * 32;
     extern __shared__ __align__(128) uint8_t smem_attn[];
-    __shared__ int s_last;
+    const int cta = (blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
+    unsigned long long* tr = (trace && cta < 256 && threadIdx.x == 0) ? trace + static_cast<size_t>(cta) * 16 : nullptr;
+    if (tr) {
+        tr[kAtStart] = global_ns();
+        tr[kAtSm] = smid_attn();
+        tr[kAtLast] = blockIdx.x == 0;
+        tr[kAtMerged] = 0;
+    }
     // seq_kv and the cached prefix rows are not written by the preceding kernel (the QKV
     // projection writes the window rows [kv_len, kv_len + T)), so they may be read before
     // the dependency wait
     pdl_launch_dependents();
     __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem_attn);
-    __nv_bfloat16* sK = sQ + kAQ * HD;       // [2][kAK][HD]
-    __nv_bfloat16* sV = sK + 2 * kAK * HD;   // [2][kAK][HD]
+    __nv_bfloat16* sK = sQ + AQ * HD;
+    __nv_bfloat16* sV = sK + kAK * HD;
 
-    const int split = blockIdx.x, h = blockIdx.y;
+    const int split = blockIdx.x, h = blockIdx.y;  // split = rank in the cluster
     const int b = blockIdx.z / qtiles, qt = blockIdx.z - b * qtiles;
-    const int NK = seq_kv[b] + T;
-    const int kbeg = split * chunk;
-    if (kbeg >= NK) return;
-    const int kend = min(NK, kbeg + chunk);
-    const int q0 = qt * kAQ;
-    const int nq = min(kAQ, T - q0);
+    const int kv = seq_kv[b];
+    const int NK = kv + T;
+    const int nblk = (NK + kAK - 1) / kAK;
+    const int kbeg = (split * nblk / csize) * kAK;
+    const int kend = min(NK, ((split + 1) * nblk / csize) * kAK);  // empty when kbeg >= kend
+    const int q0 = qt * AQ;
+    const int nq = min(AQ, T - q0);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int g = lane >> 2, c4 = lane & 3;
     constexpr int CPR = HD / 8;  // 16-byte chunks per row
@@ -222,28 +272,34 @@ __global__ void __launch_bounds__(128) k_attn(const __nv_bfloat16* __restrict__ 
     const __nv_bfloat16* kbase = kc + (static_cast<size_t>(b) * H + h) * cap * HD;
     const __nv_bfloat16* vbase = vc + (static_cast<size_t>(b) * H + h) * cap * HD;
 
-    auto load_kv = [&](int buf, int k0) {
-        for (int e = tid; e < kAK * CPR; e += 128) {
-            int r = e / CPR, cc = (e % CPR) * 8;
-            int key = k0 + r;
-            bool ok = key < kend;
-            size_t off = static_cast<size_t>(ok ? key : kbeg) * HD + cc;
-            cp_async16(sK + buf * kAK * HD + swz(r, cc, HD), kbase + off, ok);
-            cp_async16(sV + buf * kAK * HD + swz(r, cc, HD), vbase + off, ok);
+    auto load_rows = [&](__nv_bfloat16* dst, const __nv_bfloat16* base, int k0) {
+        for (int e = tid; e < kAK * CPR; e += NT) {
+            const int r = e / CPR, cc = (e % CPR) * 8;
+            const int key = k0 + r;
+            const bool ok = key < kend;
+            cp_async16(dst + swz(r, cc, HD), base + static_cast<size_t>(ok ? key : kbeg) * HD + cc, ok);
         }
     };
-    const bool prefix_first = kbeg + kAK <= seq_kv[b];
-    if (prefix_first) {  // the first sub-block lies in the cached prefix: fetch it early
-        load_kv(0, kbeg);
+    const bool has = kbeg < kend;
+    const bool prefix_first = has && kbeg + kAK <= kv;  // first sub-block entirely in the cached prefix
+    if (prefix_first) {  // groups: K0, V0 (then Q)
+        load_rows(sK, kbase, kbeg);
+        cp_async_commit();
+        load_rows(sV, vbase, kbeg);
         cp_async_commit();
     }
     pdl_wait();
-    for (int e = tid; e < kAQ * CPR; e += 128) {
-        int r = e / CPR, cc = (e % CPR) * 8;
+    if (tr) tr[kAtDepWait] = global_ns();
+    for (int e = tid; e < AQ * CPR; e += NT) {
+        const int r = e / CPR, cc = (e % CPR) * 8;
         cp_async16(sQ + swz(r, cc, HD), qbase + static_cast<size_t>(r < nq ? r : 0) * HD + cc, r < nq);
     }
-    if (!prefix_first) load_kv(0, kbeg);
-    cp_async_commit();
+    if (has && !prefix_first) load_rows(sK, kbase, kbeg);
+    cp_async_commit();  // group: Q (+ K0)
+    if (has && !prefix_first) {
+        load_rows(sV, vbase, kbeg);
+        cp_async_commit();  // group: V0
+    }
 
     constexpr int KS = HD / 16;  // k-steps of Q.K
     constexpr int DN = HD / 8;   // output n-blocks
@@ -254,27 +310,20 @@ __global__ void __launch_bounds__(128) k_attn(const __nv_bfloat16* __restrict__ 
     float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.0f, l1 = 0.0f;
     const float sl2 = rsqrtf(static_cast<float>(HD)) * 1.4426950408889634f;
 
-    int buf = 0;
-    bool qloaded = false;
     for (int k0 = kbeg; k0 < kend; k0 += kAK) {
-        if (k0 + kAK < kend) {
-            load_kv(buf ^ 1, k0 + kAK);
-            cp_async_commit();
-            cp_async_wait_1();
-        } else {
-            cp_async_wait_all();
-        }
+        const bool first = k0 == kbeg;
+        const bool more = k0 + kAK < kend;
+        // pending groups, oldest first: K_i, V_i (first: K0, V0, Q or Q+K0, V0)
+        if (first && prefix_first) cp_async_wait_all();
+        else cp_async_wait_1();
         __syncthreads();
-        if (!qloaded) {
+        if (first) {
 #pragma unroll
             for (int ks = 0; ks < KS; ++ks) {
-                int r = warp * 16 + (lane & 15), cc = ks * 16 + (lane >> 4) * 8;
+                const int r = warp * 16 + (lane & 15), cc = ks * 16 + (lane >> 4) * 8;
                 ldm_x4(smem_u32(sQ + swz(r, cc, HD)), qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3]);
             }
-            qloaded = true;
         }
-        const __nv_bfloat16* K = sK + buf * kAK * HD;
-        const __nv_bfloat16* V = sV + buf * kAK * HD;
         float s[8][4];
 #pragma unroll
         for (int j = 0; j < 8; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.0f;
@@ -282,20 +331,25 @@ __global__ void __launch_bounds__(128) k_attn(const __nv_bfloat16* __restrict__ 
         for (int jp = 0; jp < 4; ++jp) {
 #pragma unroll
             for (int ks = 0; ks < KS; ++ks) {
-                int mi = lane >> 3, rr = lane & 7;
-                int key = jp * 16 + (mi >> 1) * 8 + rr, cc = ks * 16 + (mi & 1) * 8;
+                const int mi = lane >> 3, rr = lane & 7;
+                const int key = jp * 16 + (mi >> 1) * 8 + rr, cc = ks * 16 + (mi & 1) * 8;
                 uint32_t b0, b1, b2, b3;
-                ldm_x4(smem_u32(K + swz(key, cc, HD)), b0, b1, b2, b3);
+                ldm_x4(smem_u32(sK + swz(key, cc, HD)), b0, b1, b2, b3);
                 mma16816(s[2 * jp], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b0, b1);
                 mma16816(s[2 * jp + 1], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b2, b3);
             }
+        }
+        __syncthreads();  // K consumed: the next sub-block's K streams in behind the softmax and P.V
+        if (more) {
+            load_rows(sK, kbase, k0 + kAK);
+            cp_async_commit();
         }
         // scale to log2 units, mask keys past the end, online softmax
         float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-            int key = k0 + j * 8 + 2 * c4;
-            bool v0 = key < kend, v1 = key + 1 < kend;
+            const int key = k0 + j * 8 + 2 * c4;
+            const bool v0 = key < kend, v1 = key + 1 < kend;
             s[j][0] = v0 ? s[j][0] * sl2 : -INFINITY;
             s[j][1] = v1 ? s[j][1] * sl2 : -INFINITY;
             s[j][2] = v0 ? s[j][2] * sl2 : -INFINITY;
@@ -330,38 +384,48 @@ __global__ void __launch_bounds__(128) k_attn(const __nv_bfloat16* __restrict__ 
             l0 += s[j][0] + s[j][1];
             l1 += s[j][2] + s[j][3];
         }
+        // pending: V_i (+ K_{i+1})
+        if (more) cp_async_wait_1();
+        else cp_async_wait_all();
+        __syncthreads();
         // O += P V
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk) {
-            uint32_t a0 = pack_bf16(s[2 * kk][0], s[2 * kk][1]);
-            uint32_t a1 = pack_bf16(s[2 * kk][2], s[2 * kk][3]);
-            uint32_t a2 = pack_bf16(s[2 * kk + 1][0], s[2 * kk + 1][1]);
-            uint32_t a3 = pack_bf16(s[2 * kk + 1][2], s[2 * kk + 1][3]);
+            const uint32_t a0 = pack_bf16(s[2 * kk][0], s[2 * kk][1]);
+            const uint32_t a1 = pack_bf16(s[2 * kk][2], s[2 * kk][3]);
+            const uint32_t a2 = pack_bf16(s[2 * kk + 1][0], s[2 * kk + 1][1]);
+            const uint32_t a3 = pack_bf16(s[2 * kk + 1][2], s[2 * kk + 1][3]);
 #pragma unroll
             for (int dn = 0; dn < DN; dn += 2) {
-                int mi = lane >> 3, rr = lane & 7;
-                int key = kk * 16 + (mi & 1) * 8 + rr, cc = (dn + (mi >> 1)) * 8;
+                const int mi = lane >> 3, rr = lane & 7;
+                const int key = kk * 16 + (mi & 1) * 8 + rr, cc = (dn + (mi >> 1)) * 8;
                 uint32_t b0, b1, b2, b3;
-                ldm_x4_t(smem_u32(V + swz(key, cc, HD)), b0, b1, b2, b3);
+                ldm_x4_t(smem_u32(sV + swz(key, cc, HD)), b0, b1, b2, b3);
                 mma16816(o[dn], a0, a1, a2, a3, b0, b1);
                 mma16816(o[dn + 1], a0, a1, a2, a3, b2, b3);
             }
         }
-        __syncthreads();
-        buf ^= 1;
+        __syncthreads();  // V consumed
+        if (more) {
+            load_rows(sV, vbase, k0 + kAK);
+            cp_async_commit();
+        }
     }
+    cp_async_wait_all();  // a CTA without keys still has its Q copy in flight
+    __syncthreads();
     l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
     l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
     l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
     l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+    if (tr) tr[kAtLoop] = global_ns();
 
     const int r0 = warp * 16 + g, r1 = r0 + 8;
-    if (nsplit == 1) {
-        const int qd = H * HD;
+    const int qd = H * HD;
+    if (csize == 1) {
         const float i0 = 1.0f / l0, i1 = 1.0f / l1;
 #pragma unroll
         for (int dn = 0; dn < DN; ++dn) {
-            int col = h * HD + dn * 8 + 2 * c4;
+            const int col = h * HD + dn * 8 + 2 * c4;
             if (r0 < nq)
                 *reinterpret_cast<__nv_bfloat162*>(out + (static_cast<size_t>(b) * T + q0 + r0) * qd + col) =
                     __floats2bfloat162_rn(o[dn][0] * i0, o[dn][1] * i0);
@@ -369,105 +433,128 @@ __global__ void __launch_bounds__(128) k_attn(const __nv_bfloat16* __restrict__ 
                 *reinterpret_cast<__nv_bfloat162*>(out + (static_cast<size_t>(b) * T + q0 + r1) * qd + col) =
                     __floats2bfloat162_rn(o[dn][2] * i1, o[dn][3] * i1);
         }
-    } else {
-        const size_t base = ((static_cast<size_t>(b) * H + h) * nsplit + split) * T + q0;
-#pragma unroll
-        for (int dn = 0; dn < DN; ++dn) {
-            int col = dn * 8 + 2 * c4;
-            if (r0 < nq) *reinterpret_cast<float2*>(part_o + (base + r0) * HD + col) = make_float2(o[dn][0], o[dn][1]);
-            if (r1 < nq) *reinterpret_cast<float2*>(part_o + (base + r1) * HD + col) = make_float2(o[dn][2], o[dn][3]);
-        }
-        if (c4 == 0) {
-            if (r0 < nq) *reinterpret_cast<float2*>(part_ml + (base + r0) * 2) = make_float2(m0, l0);
-            if (r1 < nq) *reinterpret_cast<float2*>(part_ml + (base + r1) * 2) = make_float2(m1, l1);
-        }
-        // the last split of this (sequence, head, query tile) to finish merges them all
-        __threadfence();
-        __syncthreads();
-        const int ns = (NK + chunk - 1) / chunk;
-        if (tid == 0) {
-            int* ctr = counters + (static_cast<size_t>(b) * H + h) * qtiles + qt;
-            const int prev = atomicAdd(ctr, 1);
-            s_last = prev == ns - 1;
-            if (s_last) *ctr = 0;
-        }
-        __syncthreads();
-        if (s_last) {
-            __threadfence();
-            // per-row split weights once (exp2(m_s - M) / L), then the weighted sum of
-            // the split outputs with independent float4 loads
-            float* wts = reinterpret_cast<float*>(smem_attn);  // [kAQ][kMaxSplit]: Q/K tiles are done
-            const size_t sb = (static_cast<size_t>(b) * H + h) * nsplit * T + q0;
-            for (int r = tid; r < nq; r += 128) {
-                float M = -INFINITY;
-                for (int sp = 0; sp < ns; ++sp)
-                    M = fmaxf(M, __ldcg(part_ml + (sb + static_cast<size_t>(sp) * T + r) * 2));
-                float L = 0.0f;
-                for (int sp = 0; sp < ns; ++sp) {
-                    const size_t row = sb + static_cast<size_t>(sp) * T + r;
-                    const float w = exp2f(__ldcg(part_ml + row * 2) - M);
-                    wts[r * kMaxSplit + sp] = w;
-                    L += w * __ldcg(part_ml + row * 2 + 1);
-                }
-                const float inv = 1.0f / L;
-                for (int sp = 0; sp < ns; ++sp) wts[r * kMaxSplit + sp] *= inv;
-            }
-            __syncthreads();
-            const int qd = H * HD;
-            constexpr int V4 = HD / 4;
-            for (int e = tid; e < nq * V4; e += 128) {
-                const int r = e / V4, i4 = e - r * V4;
-                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-                for (int sp = 0; sp < ns; ++sp) {
-                    const float w = wts[r * kMaxSplit + sp];
-                    const float4 o4 = __ldcg(reinterpret_cast<const float4*>(
-                        part_o + (sb + static_cast<size_t>(sp) * T + r) * HD) + i4);
-                    acc.x += w * o4.x;
-                    acc.y += w * o4.y;
-                    acc.z += w * o4.z;
-                    acc.w += w * o4.w;
-                }
-                __nv_bfloat16* op = out + (static_cast<size_t>(b) * T + q0 + r) * qd + h * HD + i4 * 4;
-                *reinterpret_cast<__nv_bfloat162*>(op) = __floats2bfloat162_rn(acc.x, acc.y);
-                *reinterpret_cast<__nv_bfloat162*>(op + 2) = __floats2bfloat162_rn(acc.z, acc.w);
-            }
-        }
+        return;
     }
+    // partial of this split into shared memory (the Q/K/V tiles are no longer needed)
+    float* sO = reinterpret_cast<float*>(smem_attn);  // [AQ][HD]
+    float* sML = sO + AQ * HD;                        // [AQ][2]
+#pragma unroll
+    for (int dn = 0; dn < DN; ++dn) {
+        const int col = dn * 8 + 2 * c4;
+        *reinterpret_cast<float2*>(sO + r0 * HD + col) = make_float2(o[dn][0], o[dn][1]);
+        *reinterpret_cast<float2*>(sO + r1 * HD + col) = make_float2(o[dn][2], o[dn][3]);
+    }
+    if (c4 == 0) {
+        *reinterpret_cast<float2*>(sML + r0 * 2) = make_float2(m0, l0);
+        *reinterpret_cast<float2*>(sML + r1 * 2) = make_float2(m1, l1);
+    }
+    cluster_sync_all();  // every split's partial is in place
+    if (tr) tr[kAtTicket] = global_ns();
+    // this CTA merges output elements split*NT + tid (+ k * csize * NT): row r, 4 features
+    constexpr int V4 = HD / 4;
+    for (int e = split * NT + tid; e < nq * V4; e += csize * NT) {
+        const int r = e / V4, i4 = e - r * V4;
+        const uint32_t a_ml = smem_u32(sML + r * 2);
+        const uint32_t a_o = smem_u32(sO + r * HD + i4 * 4);
+        float2 ml[kMaxCluster];
+        float4 ov[kMaxCluster];
+#pragma unroll
+        for (int c = 0; c < kMaxCluster; ++c) {
+            if (c < csize) {
+                ml[c] = dsmem_ld2(dsmem_map(a_ml, c));
+                ov[c] = dsmem_ld4(dsmem_map(a_o, c));
+            }
+        }
+        float M = -INFINITY;
+#pragma unroll
+        for (int c = 0; c < kMaxCluster; ++c)
+            if (c < csize) M = fmaxf(M, ml[c].x);
+        float L = 0.0f;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int c = 0; c < kMaxCluster; ++c) {
+            if (c < csize) {
+                const float w = ml[c].x == -INFINITY ? 0.0f : exp2f(ml[c].x - M);  // split without keys: 0
+                L += w * ml[c].y;
+                acc.x += w * ov[c].x;
+                acc.y += w * ov[c].y;
+                acc.z += w * ov[c].z;
+                acc.w += w * ov[c].w;
+            }
+        }
+        const float inv = 1.0f / L;
+        __nv_bfloat16* op = out + (static_cast<size_t>(b) * T + q0 + r) * qd + h * HD + i4 * 4;
+        *reinterpret_cast<__nv_bfloat162*>(op) = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
+        *reinterpret_cast<__nv_bfloat162*>(op + 2) = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
+    }
+    cluster_sync_all();  // no CTA leaves while its partial may still be read
+    if (tr) tr[kAtMerged] = global_ns();
 }
 
+static size_t attn_smem(int nw, int hd) { return static_cast<size_t>(nw * 16 + 2 * kAK) * hd * 2; }
+
 cudaError_t attn_init_attrs() {
-    return cudaFuncSetAttribute(reinterpret_cast<const void*>(k_attn<128>),
-                                cudaFuncAttributeMaxDynamicSharedMemorySize, 100 * 1024);
+    cudaError_t e = cudaSuccess;
+    auto set = [&](const void* f, size_t bytes) {
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
+    };
+    set(reinterpret_cast<const void*>(k_attn<128, 2>), attn_smem(2, 128));
+    set(reinterpret_cast<const void*>(k_attn<128, 4>), attn_smem(4, 128));
+    set(reinterpret_cast<const void*>(k_attn<64, 2>), attn_smem(2, 64));
+    set(reinterpret_cast<const void*>(k_attn<64, 4>), attn_smem(4, 64));
+    return e;
 }
 
 AttnPlan attn_plan(int B, int T, int H, int max_keys, int sms) {
-    // about one CTA per SM: splitting further only adds merge work (each split's
-    // 64-key sub-blocks already run back to back with a double-buffered prefetch)
     AttnPlan a;
-    a.qtiles = (T + kAQ - 1) / kAQ;
+    // two warps (32 query rows) for the short windows of cached decoding, four otherwise
+    a.nw = T <= 64 ? 2 : 4;
+    a.qtiles = (T + a.nw * 16 - 1) / (a.nw * 16);
+    // key splits (cluster size): about two CTAs per SM, at most one split per sub-block
     const int units = B * H * a.qtiles;
-    int want = sms / units;
-    const int blocks64 = (max_keys + kAK - 1) / kAK;
-    if (want > blocks64) want = blocks64;
-    if (want > kMaxSplit) want = kMaxSplit;
-    if (want < 1) want = 1;
-    a.chunk = ((blocks64 + want - 1) / want) * kAK;
-    a.nsplit = (max_keys + a.chunk - 1) / a.chunk;
+    const int blocks = (max_keys + kAK - 1) / kAK;
+    int c = (2 * sms) / units;
+    if (c > kMaxCluster) c = kMaxCluster;
+    if (c > blocks) c = blocks;
+    if (c < 1) c = 1;
+    a.csize = c;
     return a;
 }
 
 cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
-                             const int* seq_kv, float* part_o, float* part_ml, int* counters, __nv_bfloat16* out, int B,
-                             int T, int H, int hd, int cap, const AttnPlan& a, cudaStream_t st, bool pdl) {
-    const dim3 grid(a.nsplit, H, B * a.qtiles);
-    const size_t smem = static_cast<size_t>(kAQ + 4 * kAK) * hd * 2;
+                             const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int hd, int cap,
+                             const AttnPlan& a, cudaStream_t st, bool pdl, unsigned long long* trace) {
+    if (a.csize < 1 || a.csize > kMaxCluster || (a.nw != 2 && a.nw != 4) || (hd != 64 && hd != 128))
+        return cudaErrorInvalidValue;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(a.csize, H, B * a.qtiles);
+    cfg.blockDim = dim3(a.nw * 32);
+    cfg.dynamicSmemBytes = attn_smem(a.nw, hd);
+    cfg.stream = st;
+    cudaLaunchAttribute at[2];
+    int n = 0;
+    at[n].id = cudaLaunchAttributeClusterDimension;
+    at[n].val.clusterDim.x = static_cast<unsigned>(a.csize);
+    at[n].val.clusterDim.y = 1;
+    at[n].val.clusterDim.z = 1;
+    ++n;
+    if (pdl && pdl_enabled()) {
+        at[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        at[n].val.programmaticStreamSerializationAllowed = 1;
+        ++n;
+    }
+    cfg.attrs = at;
+    cfg.numAttrs = n;
     if (hd == 128)
-        return launch_k(k_attn<128>, grid, dim3(128), smem, st, pdl, q, kc, vc, seq_kv, part_o, part_ml, counters, out, T,
-                        H, cap, a.chunk, a.nsplit, a.qtiles);
-    if (hd == 64)
-        return launch_k(k_attn<64>, grid, dim3(128), smem, st, pdl, q, kc, vc, seq_kv, part_o, part_ml, counters, out, T,
-                        H, cap, a.chunk, a.nsplit, a.qtiles);
-    return cudaErrorInvalidValue;
+        return a.nw == 2 ? cudaLaunchKernelEx(&cfg, k_attn<128, 2>, q, kc, vc, seq_kv, out, T, H, cap, a.qtiles,
+                                              a.csize, trace)
+                         : cudaLaunchKernelEx(&cfg, k_attn<128, 4>, q, kc, vc, seq_kv, out, T, H, cap, a.qtiles,
+                                              a.csize, trace);
+    return a.nw == 2 ? cudaLaunchKernelEx(&cfg, k_attn<64, 2>, q, kc, vc, seq_kv, out, T, H, cap, a.qtiles, a.csize,
+                                          trace)
+                     : cudaLaunchKernelEx(&cfg, k_attn<64, 4>, q, kc, vc, seq_kv, out, T, H, cap, a.qtiles, a.csize,
+                                          trace);
 }
 
 // ------------------------------------------------------------------ LM head

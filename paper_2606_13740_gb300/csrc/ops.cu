@@ -150,16 +150,9 @@ int dllm_op_attention(const void* q, const void* kc, const void* vc, const int32
     if (sms <= 0) return op_fail(DLLM_ECUDA, "no CUDA device");
     if (attn_init_attrs() != cudaSuccess) return op_fail(DLLM_ECUDA, "attribute setup failed");
     AttnPlan a = attn_plan(B, T, H, max_kv_len + T, sms);
-    DevBuf po, pml, ctr;
-    const size_t rows = static_cast<size_t>(B) * H * a.nsplit * T;
-    const size_t nctr = static_cast<size_t>(B) * H * a.qtiles;
-    if (!po.alloc(rows * hd * 4) || !pml.alloc(rows * 2 * 4) || !ctr.alloc(nctr * 4))
-        return op_fail(DLLM_ENOMEM, "scratch allocation failed");
-    if (cudaMemsetAsync(ctr.p, 0, nctr * 4, st) != cudaSuccess) return op_fail(DLLM_ECUDA, "memset failed");
     cudaError_t e = launch_attention(static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(kc),
-                                     static_cast<const __nv_bfloat16*>(vc), kv_len, static_cast<float*>(po.p),
-                                     static_cast<float*>(pml.p), static_cast<int*>(ctr.p),
-                                     static_cast<__nv_bfloat16*>(out), B, T, H, hd, cap, a, st, false);
+                                     static_cast<const __nv_bfloat16*>(vc), kv_len, static_cast<__nv_bfloat16*>(out),
+                                     B, T, H, hd, cap, a, st, false);
     if (e != cudaSuccess) return op_fail(DLLM_ECUDA, "attention launch: %s", cudaGetErrorString(e));
     return finish(st, nullptr);
 }

@@ -149,12 +149,22 @@ def step_trace(a):
     tr = ctx.dllm_get_trace().astype(np.int64)
     if a.dump:
         np.save(a.dump, tr)
-    names = ["qkv", "oproj", "gateup", "down"] * 32 + ["head"]
+    names = ["qkv", "attn", "oproj", "gateup", "down"] * 32 + ["head"]
     t0 = min(int(x[:, 0][x[:, 0] > 0].min()) for x in tr)
     rows = []
     prev_exit = None
     for i, x in enumerate(tr):
         v = x[x[:, 0] > 0]
+        if i < len(names) and names[i] == "attn":  # slots: start, dep wait, loop end, ticket, merged
+            rel = lambda c: (v[:, c][v[:, c] > 0] - t0) / 1e3  # noqa: E731
+            r = {"k": "attn", "start_min": float(rel(0).min()), "depwait_med": float(np.median(rel(1))),
+                 "loop_max": float(rel(2).max()), "ticket_max": float(rel(3).max()),
+                 "merged_max": float(rel(4).max()) if (v[:, 4] > 0).any() else None}
+            if prev_exit is not None:
+                r["gap_prev_exit_to_depwait"] = r["depwait_med"] - prev_exit
+            prev_exit = r["merged_max"] if r["merged_max"] is not None else r["loop_max"]
+            rows.append({k: (round(v, 2) if isinstance(v, float) else v) for k, v in r.items()})
+            continue
         rel = lambda c: (v[:, c][v[:, c] > 0] - t0) / 1e3  # noqa: E731
         r = {"k": names[i] if i < len(names) else str(i), "start_min": float(rel(0).min()),
              "start_max": float(rel(0).max()), "depwait_med": float(np.median(rel(7))),
@@ -170,7 +180,7 @@ def step_trace(a):
         rows.append({k: (round(v, 2) if isinstance(v, float) else v) for k, v in r.items()})
     span = rows[-1]["exit_max"] - rows[0]["start_min"]
     print(json.dumps({"op": "step-trace", "pdl": not a.no_pdl, "gemm_span_us": round(span, 1),
-                      "first_layer": rows[:4], "layer_16": rows[64:68], "head": rows[-1]}))
+                      "first_layer": rows[:5], "layer_16": rows[80:85], "head": rows[-1]}))
     ctx.close()
 
 
