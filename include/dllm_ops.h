@@ -19,8 +19,10 @@ extern "C" {
  * paper offloads to the NPU; here tcgen05 tensor cores):
  * D[n][m] = sum_k W[m][k] * X[n][k].  W dev bf16 [M][K] row-major, X dev bf16
  * [N][K] row-major, D dev fp32 [N][M].  K*2 bytes must be a multiple of 16;
- * W and X 16-byte aligned.  grid = CTAs of the stream-K split (0: one per
- * SM).  Errors: DLLM_EINVAL, DLLM_ECUDA, DLLM_ETIMEOUT. */
+ * W and X 16-byte aligned.  grid = CTAs of the stream-K split (0 or more
+ * than the SM count: one per SM; the CTAs that finish a split tile wait for
+ * its other contributors, so all of them must be resident at once).
+ * Errors: DLLM_EINVAL, DLLM_ECUDA, DLLM_ETIMEOUT. */
 int dllm_op_gemm(const void* W, const void* X, float* D, int M, int N, int K, int grid, void* stream);
 
 /* dllm_op_gemm launched `reps` times back to back on one scratch
@@ -36,8 +38,10 @@ int dllm_op_gemm_timed(const void* W, const void* X, float* D, int M, int N, int
  * after the prologue, first operand stage arrived, last stage consumed,
  * epilogue done, exit; the SM id; the stamp when the dependency wait
  * returned; for the CTA's last output tile: accumulator ready, split partial
- * stored, ticket taken, partials reduced (0 when not the last arriver), the
- * last-arriver flag and the tile index.  trace must hold 16 values per SM. */
+ * stored (or, for the CTA that finishes the tile, its wait started), all
+ * contributors arrived and partials reduced (0 unless this CTA finishes the
+ * tile), the finishing flag and the tile index.  trace must hold 16 values
+ * per SM. */
 int dllm_op_gemm_trace(const void* W, const void* X, float* D, int M, int N, int K, int grid, int reps,
                        float* ms_per_launch, unsigned long long* trace, int* grid_used, void* stream);
 
@@ -51,9 +55,9 @@ int dllm_op_gemm_trace(const void* W, const void* X, float* D, int M, int N, int
  * statically sized device array of 8 MiB that every GPU loading the library
  * holds until the process exits; it calls no cudaMalloc, cudaFree or other
  * allocating routine.  Limits: at most 2046 output tiles (ceil(M/128) x
- * token tiles); the grid (0 = one CTA per SM) is shrunk to fit the array when
- * chosen automatically, and an explicit grid that does not fit is rejected
- * with DLLM_ECAPACITY.  The first call on a device looks up the array's
+ * token tiles); the grid (0 = one CTA per SM, at most the SM count) is
+ * shrunk to fit the array when chosen automatically, and an explicit grid
+ * that does not fit is rejected with DLLM_ECAPACITY.  The first call on a device looks up the array's
  * device address (cudaGetSymbolAddress) with that device current; make that
  * first call before any stream capture.  All calls share the one array: two
  * calls that overlap on the GPU (other streams, other host threads) race and

@@ -10,11 +10,14 @@
 // Work is split "stream-K" style: the flattened (tile, 64-wide k-block)
 // iteration space is cut into one contiguous range per CTA (one CTA per SM),
 // so every SM streams the same number of weight bytes whatever the tile
-// count.  A tile cut between CTAs is finished by whichever CTA arrives last
-// (atomic ticket), which sums the fp32 partials in k order: deterministic,
-// and nobody waits on anybody.  When that tile is the CTA's final one, its
-// drained pipeline memory receives every partial through one round of bulk
-// copies.
+// count.  A tile cut between CTAs is finished by the CTA holding its first
+// k-blocks, which are the end of that CTA's range: the other contributors
+// store fp32 partials and publish them with one release increment each, and
+// the finishing CTA waits (bounded) for the count, bulk-copies the partials
+// into its drained pipeline memory and adds them to its own accumulator in k
+// order (deterministic).  Every CTA waits at most once, at its end, on CTAs
+// that wait on nothing, and the grid never exceeds the SM count, so all of
+// them are resident.
 //
 // Roles (192 threads): warp 0 = TMA producer, warp 1 = TMEM owner and MMA
 // issuer, warps 2..5 = epilogue (one TMEM lane quarter each).  Accumulators
@@ -536,7 +539,6 @@ __global__ void __launch_bounds__(kThreads, 2)
     uint64_t* redbar = drain + 1;  // split-partial bulk loads of the last arriver
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(redbar + 1);
     volatile int* s_abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
-    volatile int* s_last = s_abort + 1;
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -563,7 +565,6 @@ __global__ void __launch_bounds__(kThreads, 2)
         mbar_init(drain, 1);
         mbar_init(redbar, 1);
         *s_abort = 0;
-        *s_last = 0;
         mbar_fence_init();
     }
     if (warp == 0 && lane == 0) {
@@ -762,11 +763,20 @@ __global__ void __launch_bounds__(kThreads, 2)
             tc_fence_after();
             const uint32_t t_acc = tmem_base + static_cast<uint32_t>(acc * p.acc_cols) +
                                    (static_cast<uint32_t>(quarter * 32) << 16);
-            const int slot = (range_begin(blockIdx.x, p.total, G) / p.kb == tile) ? 0 : 1;
-            float* my_part = partials + (static_cast<size_t>(blockIdx.x) * 2 + slot) * slot_floats;
+            // A tile cut between CTAs is finished by the CTA that holds its first k-blocks (for
+            // that CTA they are the end of its range); the others store fp32 partials for it.
+            int c_first = 0, c_last = 0;
+            bool reducer = false;
+            if (!whole) {
+                c_first = owner_of(tile * p.kb, p.total, G);
+                c_last = owner_of(tile * p.kb + p.kb - 1, p.total, G);
+                reducer = static_cast<int>(blockIdx.x) == c_first;
+            }
             if (whole && c32) {
                 epilogue_c32<EPI>(ep, p, mt, nt, rt, t_acc, t_x, esm, ew, quarter, lane, status);
-            } else {
+            } else if (!reducer) {
+                // a contributor's partial is the first segment of its range: slot 0
+                float* my_part = partials + static_cast<size_t>(blockIdx.x) * 2 * slot_floats;
                 for (int c = 0; c < nchunks; ++c) {
                     tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);
                     if (whole) {
@@ -781,98 +791,101 @@ __global__ void __launch_bounds__(kThreads, 2)
                     }
                 }
             }
-            if (!c32) {  // wide tiles release the accumulator as soon as it is read
+            if (!c32 && !reducer) {  // wide tiles release the accumulator as soon as it is read
                 tc_fence_before();
                 mbar_arrive(&tempty[acc]);
             }
-            if (!whole) {
-                // last-arriver reduction of a tile split between CTAs
-                __threadfence();
+            if (!whole && !reducer) {
+                // publish: the barrier orders the quarter-warps' stores before one release increment
                 named_bar(1, 128);
                 if (threadIdx.x == 64) {
                     if (tr) tr[kTrPartStored] = global_ns();
-                    const int c_first = owner_of(tile * p.kb, p.total, G);
-                    const int c_last = owner_of(tile * p.kb + p.kb - 1, p.total, G);
-                    int* ticket = &counters[tile * kTicketStride];
-                    const int prev = atomicAdd(ticket, 1);
-                    const int last = prev == c_last - c_first;
-                    if (last) *ticket = 0;
-                    *s_last = last;
+                    red_release_add(&counters[tile * kTicketStride], 1);
+                }
+            } else if (reducer) {
+                const int nparts = c_last - c_first + 1;
+                int* ticket = &counters[tile * kTicketStride];
+                if (threadIdx.x == 64) {
+                    if (tr) tr[kTrPartStored] = global_ns();
+                    const unsigned long long t0 = global_ns();
+                    while (ld_acquire(ticket) != nparts - 1) {
+                        if (*s_abort) break;
+                        if (global_ns() - t0 > kWaitLimitNs) {
+                            *s_abort = 1;
+                            atomicOr(status, kStatusTimeout);
+                            break;
+                        }
+                    }
+                    *ticket = 0;  // every contributor has arrived: ready for the next launch
                     if (tr) {
                         tr[kTrTicket] = global_ns();
-                        tr[kTrIsLast] = last;
+                        tr[kTrIsLast] = 1;
                     }
                 }
                 named_bar(1, 128);
-                if (*s_last) {
-                    __threadfence();
-                    const int c_first = owner_of(tile * p.kb, p.total, G);
-                    const int c_last = owner_of(tile * p.kb + p.kb - 1, p.total, G);
-                    const int nparts = c_last - c_first + 1;
-                    const uint32_t part_bytes = static_cast<uint32_t>(slot_floats * 4);
-                    const uint32_t stage_room = static_cast<uint32_t>(S) * (kABytes + b_bytes);
-                    const bool final_seg = tile * p.kb + k_hi == it1;  // pipeline drained: stage memory free
-                    for (int c = 0; c < nchunks; ++c) {
-#pragma unroll
-                        for (int j = 0; j < 32; ++j) v[j] = 0.0f;
-                        if (final_seg && c32 && part_bytes <= stage_room) {
-                            // one round trip: bulk-copy every partial into the stage memory at once
-                            const int per_batch = static_cast<int>(stage_room / part_bytes);
-                            for (int b0 = 0; b0 < nparts; b0 += per_batch) {
-                                const int nb = nparts - b0 < per_batch ? nparts - b0 : per_batch;
-                                if (threadIdx.x == 64) {
-                                    fence_proxy_async_global();
-                                    mbar_arrive_expect_tx(redbar, part_bytes * static_cast<uint32_t>(nb));
-                                    for (int q = 0; q < nb; ++q) {
-                                        const int cc = c_first + b0 + q;
-                                        const int sl = (range_begin(cc, p.total, G) / p.kb == tile) ? 0 : 1;
-                                        bulk_load(smem + static_cast<size_t>(q) * part_bytes,
-                                                  partials + (static_cast<size_t>(cc) * 2 + sl) * slot_floats,
-                                                  part_bytes, redbar);
-                                    }
-                                }
-                                mbar_wait(redbar, red_phase, s_abort, status);
-                                red_phase ^= 1u;
-                                for (int q = 0; q < nb; ++q) {
-                                    const float4* src =
-                                        reinterpret_cast<const float4*>(smem + static_cast<size_t>(q) * part_bytes);
-#pragma unroll
-                                    for (int j = 0; j < 8; ++j) {
-                                        const float4 a = src[j * kBM + rt];
-                                        v[4 * j] += a.x;
-                                        v[4 * j + 1] += a.y;
-                                        v[4 * j + 2] += a.z;
-                                        v[4 * j + 3] += a.w;
-                                    }
-                                }
-                                named_bar(1, 128);  // the next batch overwrites the staging memory
+                if (*s_abort) break;
+                const uint32_t part_bytes = static_cast<uint32_t>(slot_floats * 4);
+                const uint32_t stage_room = static_cast<uint32_t>(S) * (kABytes + b_bytes);
+                const bool final_seg = tile * p.kb + k_hi == it1;  // pipeline drained: stage memory free
+                for (int c = 0; c < nchunks; ++c) {
+                    tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);  // own (first) k-range
+                    if (final_seg && c32 && part_bytes <= stage_room) {
+                        // one round trip: bulk-copy the contributors' partials into the stage memory
+                        const int per_batch = static_cast<int>(stage_room / part_bytes);
+                        for (int b0 = 1; b0 < nparts; b0 += per_batch) {
+                            const int nb = nparts - b0 < per_batch ? nparts - b0 : per_batch;
+                            if (threadIdx.x == 64) {
+                                fence_proxy_async_global();
+                                mbar_arrive_expect_tx(redbar, part_bytes * static_cast<uint32_t>(nb));
+                                for (int q = 0; q < nb; ++q)
+                                    bulk_load(smem + static_cast<size_t>(q) * part_bytes,
+                                              partials + static_cast<size_t>(c_first + b0 + q) * 2 * slot_floats,
+                                              part_bytes, redbar);
                             }
-                        } else {
-                            // partials in k order (each one's 8 loads in flight together)
-                            for (int cc = c_first; cc <= c_last; ++cc) {
-                                const int sl0 = (range_begin(cc, p.total, G) / p.kb == tile) ? 0 : 1;
-                                const float4* p0 = reinterpret_cast<const float4*>(
-                                    partials + (static_cast<size_t>(cc) * 2 + sl0) * slot_floats);
-                                float4 a[8];
-#pragma unroll
-                                for (int j = 0; j < 8; ++j) a[j] = __ldcg(p0 + static_cast<size_t>(c * 8 + j) * kBM + rt);
+                            mbar_wait(redbar, red_phase, s_abort, status);
+                            red_phase ^= 1u;
+                            for (int q = 0; q < nb; ++q) {
+                                const float4* src =
+                                    reinterpret_cast<const float4*>(smem + static_cast<size_t>(q) * part_bytes);
 #pragma unroll
                                 for (int j = 0; j < 8; ++j) {
-                                    v[4 * j] += a[j].x;
-                                    v[4 * j + 1] += a[j].y;
-                                    v[4 * j + 2] += a[j].z;
-                                    v[4 * j + 3] += a[j].w;
+                                    const float4 a = src[j * kBM + rt];
+                                    v[4 * j] += a.x;
+                                    v[4 * j + 1] += a.y;
+                                    v[4 * j + 2] += a.z;
+                                    v[4 * j + 3] += a.w;
                                 }
                             }
+                            named_bar(1, 128);  // the next batch overwrites the staging memory
                         }
-                        if (tr && threadIdx.x == 64 && c == 0) tr[kTrReduced] = global_ns();
-                        if (c32) {
-                            tmem_st_32x32(t_acc, v);  // the sum goes back into the (still owned) accumulator
-                            epilogue_c32<EPI>(ep, p, mt, nt, rt, t_acc, t_x, esm, ew, quarter, lane, status);
-                        } else {
-                            epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
+                    } else {
+                        // contributors in k order (each one's 8 loads in flight together)
+                        for (int cc = c_first + 1; cc <= c_last; ++cc) {
+                            const float4* p0 =
+                                reinterpret_cast<const float4*>(partials + static_cast<size_t>(cc) * 2 * slot_floats);
+                            float4 a[8];
+#pragma unroll
+                            for (int j = 0; j < 8; ++j) a[j] = __ldcg(p0 + static_cast<size_t>(c * 8 + j) * kBM + rt);
+#pragma unroll
+                            for (int j = 0; j < 8; ++j) {
+                                v[4 * j] += a[j].x;
+                                v[4 * j + 1] += a[j].y;
+                                v[4 * j + 2] += a[j].z;
+                                v[4 * j + 3] += a[j].w;
+                            }
                         }
                     }
+                    if (tr && threadIdx.x == 64 && c == 0) tr[kTrReduced] = global_ns();
+                    if (c32) {
+                        tmem_st_32x32(t_acc, v);  // the sum goes back into the (still owned) accumulator
+                        epilogue_c32<EPI>(ep, p, mt, nt, rt, t_acc, t_x, esm, ew, quarter, lane, status);
+                    } else {
+                        epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
+                    }
+                }
+                if (!c32) {
+                    tc_fence_before();
+                    mbar_arrive(&tempty[acc]);
                 }
             }
             if (c32) {

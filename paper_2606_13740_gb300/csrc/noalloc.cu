@@ -63,7 +63,7 @@ extern "C" int dllm_op_gemm_noalloc(const void* W, const void* X, float* D, int 
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0)
         return noalloc_fail(DLLM_ECUDA, "device query failed");
-    GemmPlan p = gemm_plan(M, N, K, grid > 0 ? grid : sms, EPI_F32);
+    GemmPlan p = gemm_plan(M, N, K, (grid > 0 && grid < sms) ? grid : sms, EPI_F32);
     p.pdl = false;
     // the split partials take [grid][2][ntile x 128] floats behind the tickets
     const size_t per_cta = static_cast<size_t>(2) * p.ntile * 128 * sizeof(float);

@@ -67,7 +67,7 @@ static int gemm_impl(const void* W, const void* X, float* D, int M, int N, int K
     int sms = sm_count();
     if (sms <= 0) return op_fail(DLLM_ECUDA, "no CUDA device");
     if (gemm_init_attrs() != cudaSuccess) return op_fail(DLLM_ECUDA, "attribute setup failed");
-    GemmPlan p = gemm_plan(M, N, K, grid > 0 ? grid : sms, EPI_F32);
+    GemmPlan p = gemm_plan(M, N, K, (grid > 0 && grid < sms) ? grid : sms, EPI_F32);
     p.pdl = false;  // the operands come from the caller's kernels
     CUtensorMap tw, tx;
     if (!make_tmap_bf16(&tw, W, M, K, 128) || !make_tmap_bf16(&tx, X, N, K, p.ntile))
