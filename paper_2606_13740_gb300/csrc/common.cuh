@@ -225,6 +225,16 @@ __device__ __forceinline__ void tmem_ld_32x4(uint32_t taddr, float* v) {
     v[3] = __uint_as_float(r3);
 }
 
+__device__ __forceinline__ void tmem_ld_32x8(uint32_t taddr, float* v) {
+    uint32_t r[8];
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                 : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
+}
+
 // 32 registers per thread -> its TMEM lane, 32 consecutive columns.
 __device__ __forceinline__ void tmem_st_32x32(uint32_t taddr, const float* v) {
     asm volatile(

@@ -317,20 +317,34 @@ __device__ __forceinline__ void epilogue_chunk(const EpiArgs& ep, const GemmPlan
     }
 }
 
-// Epilogue of a 32-token tile (the batch-1 weight stream), compact: one rolled loop over 8
-// groups of 4 columns read from TMEM (t_src; for the residual, the old x of the tile was
-// staged at t_x before the accumulator was ready), so its code stays small and no global load
-// waits on a store.
-__device__ __forceinline__ float warp_sum(float v) {
+// Sum of v[0..7] over the 32 lanes of a warp, scattered: afterwards the four lanes
+// 4c..4c+3 hold the total of column c in v[0].  9 shuffles in a fixed order.
+__device__ __forceinline__ void warp_reduce_scatter8(float* v, int lane) {
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
-    return v;
+    for (int w = 16, h = 4; w >= 4; w >>= 1, h >>= 1) {
+        const bool upper = (lane & w) != 0;
+#pragma unroll
+        for (int i = 0; i < h; ++i) {
+            const float send = upper ? v[i] : v[i + h];
+            const float keep = upper ? v[i + h] : v[i];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, w);
+        }
+    }
+    v[0] += __shfl_xor_sync(0xffffffffu, v[0], 2);
+    v[0] += __shfl_xor_sync(0xffffffffu, v[0], 1);
 }
 
+// Epilogue of a 32-token tile (the batch-1 weight stream), compact: one rolled loop over 4
+// groups of 8 columns read from TMEM (t_src; for the residual, the old x of the tile was
+// staged at t_x before the accumulator was ready), so its code stays small and no global load
+// waits on a store.  Inside a group every step runs over the 8 columns side by side with no
+// branch between them (stores are predicated), so their dependent chains (shuffles, special
+// functions) overlap.
 template <int EPI>
 __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& p, int mt, int nt, int rt,
                                              uint32_t t_src, uint32_t t_x, const EpiSmem& sm, int ew, int quarter,
                                              int lane, int* status) {
+    constexpr int GW = 8;  // columns per group
     const int row = mt * kBM + rt;
     const int col0 = nt * 32;
     const bool scale = (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) && ep.sq_in != nullptr;
@@ -338,16 +352,18 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
     int part = 0, hh = 0, pp = 0, fi = 0, bl = 0;
     bool run = true;
     float cn = 1.0f, sn = 0.0f, cd = 1.0f, sd = 0.0f, theta = 0.0f;
+    __nv_bfloat16* qkv_dst = nullptr;
     if constexpr (EPI == EPI_QKV) {
         const int qd = ep.H * ep.hd;
-        part = row / qd;
+        part = row / qd;  // the same for the whole warp (qd is a multiple of 128)
         const int f = row - part * qd;
         hh = f / ep.hd;
         pp = f - hh * ep.hd;
         fi = (pp >> 1) + (pp & 1) * (ep.hd >> 1);
         theta = sm.theta[rt];
         bl = col0 / ep.T;
-        run = min(col0 + 31, p.N - 1) / ep.T == bl;
+        run = min(col0 + 31, p.N - 1) / ep.T == bl;  // all 32 columns in one sequence
+        qkv_dst = part == 0 ? ep.q : (part == 1 ? ep.kc : ep.vc);
         if (part < 2 && run) {
             const float2 a = rot_cs(static_cast<float>(sm.kvs[bl] + (col0 - bl * ep.T)) * theta);
             const float2 d = rot_cs(theta);
@@ -357,109 +373,121 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
             sd = d.y;
         }
     }
+    bool lm_ok = false;
+    if constexpr (EPI == EPI_LMHEAD) lm_ok = row < ep.V && row != ep.mask_id;
     unsigned long long* tr = (ep.trace && ew == 0 && lane == 0) ? ep.trace + static_cast<size_t>(blockIdx.x) * kTrSlots : nullptr;
 #pragma unroll 1
-    for (int g = 0; g < 8; ++g) {
+    for (int g = 0; g < 32 / GW; ++g) {
         if (tr && g == 1) tr[kTrEpiG0] = global_ns();
-        float a[4];
-        tmem_ld_32x4(t_src + static_cast<uint32_t>(4 * g), a);
+        const int cg = col0 + GW * g;  // first column of the group
+        float a[GW];
+        tmem_ld_32x8(t_src + static_cast<uint32_t>(GW * g), a);
         if (scale) {
 #pragma unroll
-            for (int u = 0; u < 4; ++u) a[u] *= sm.rs[4 * g + u];
+            for (int u = 0; u < GW; ++u) a[u] *= sm.rs[GW * g + u];
         }
         if constexpr (EPI == EPI_F32) {
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int col = col0 + 4 * g + u;
-                if (row < p.M && col < p.N) ep.out[static_cast<size_t>(col) * ep.ld_out + row] = a[u];
-            }
+            for (int u = 0; u < GW; ++u)
+                if (row < p.M && cg + u < p.N) ep.out[static_cast<size_t>(cg + u) * ep.ld_out + row] = a[u];
         } else if constexpr (EPI == EPI_RESID) {
-            float xo[4];
-            tmem_ld_32x4(t_x + static_cast<uint32_t>(4 * g), xo);
+            float xo[GW], ss[GW];
+            tmem_ld_32x8(t_x + static_cast<uint32_t>(GW * g), xo);
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int col = col0 + 4 * g + u;
-                float x = 0.0f;
-                if (row < p.M && col < p.N) {
-                    const size_t o = static_cast<size_t>(col) * ep.ld_out + row;
-                    x = xo[u] + a[u];
-                    ep.out[o] = x;
-                    ep.xb[o] = __float2bfloat16_rn(x);
+            for (int u = 0; u < GW; ++u) {
+                const bool ok = row < p.M && cg + u < p.N;
+                xo[u] += a[u];
+                ss[u] = ok ? xo[u] * xo[u] : 0.0f;
+                if (ok) {
+                    const size_t o = static_cast<size_t>(cg + u) * ep.ld_out + row;
+                    ep.out[o] = xo[u];
+                    ep.xb[o] = __float2bfloat16_rn(xo[u]);
                 }
-                const float s = warp_sum(x * x);
-                if (lane == 0) sm.red[quarter * 32 + 4 * g + u] = s;
             }
+            warp_reduce_scatter8(ss, lane);
+            if ((lane & 3) == 0) sm.red[quarter * 32 + GW * g + (lane >> 2)] = ss[0];
         } else if constexpr (EPI == EPI_QKV) {
+            float xp[GW];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const float xp = __shfl_xor_sync(0xffffffffu, a[u], 1);
-                const int col = col0 + 4 * g + u;
-                if (col < p.N) {
-                    const int b = run ? bl : col / ep.T;
-                    const int t = col - b * ep.T;
-                    const int pos = sm.kvs[b] + t;
-                    if (pos < 0 || pos >= ep.cap) {
-                        atomicOr(status, kStatusBadIndex);
-                    } else {
-                        float x = a[u];
-                        if (part < 2) {
-                            if (!run) {
-                                const float2 r = rot_cs(static_cast<float>(pos) * theta);
-                                cn = r.x;
-                                sn = r.y;
-                            }
-                            x = (pp & 1) ? (x * cn + xp * sn) : (x * cn - xp * sn);
-                        }
-                        const __nv_bfloat16 y = __float2bfloat16_rn(x);
-                        if (part == 0) {
-                            ep.q[((static_cast<size_t>(b) * ep.H + hh) * ep.T + t) * ep.hd + fi] = y;
-                        } else {
-                            __nv_bfloat16* c = part == 1 ? ep.kc : ep.vc;
-                            c[((static_cast<size_t>(b) * ep.H + hh) * ep.cap + pos) * ep.hd + fi] = y;
-                        }
+            for (int u = 0; u < GW; ++u) xp[u] = __shfl_xor_sync(0xffffffffu, a[u], 1);
+            bool bad = false;
+#pragma unroll
+            for (int u = 0; u < GW; ++u) {
+                const int col = cg + u;
+                int b = bl, t = col - bl * ep.T;
+                if (!run) {  // the tile spans sequences (uniform over the warp)
+                    b = min(col / ep.T, ep.n_seq - 1);
+                    t = col - b * ep.T;
+                }
+                const int pos = sm.kvs[b] + t;
+                const bool inb = pos >= 0 && pos < ep.cap;
+                bad |= col < p.N && !inb;
+                float x = a[u];
+                if (part < 2) {
+                    if (!run) {
+                        const float2 r = rot_cs(static_cast<float>(pos) * theta);
+                        cn = r.x;
+                        sn = r.y;
+                    }
+                    x = (pp & 1) ? (x * cn + xp[u] * sn) : (x * cn - xp[u] * sn);
+                    if (run) {
+                        const float c2 = cn * cd - sn * sd;
+                        sn = sn * cd + cn * sd;
+                        cn = c2;
                     }
                 }
-                if (run) {
-                    const float c2 = cn * cd - sn * sd;
-                    sn = sn * cd + cn * sd;
-                    cn = c2;
-                }
+                const size_t o = part == 0 ? ((static_cast<size_t>(b) * ep.H + hh) * ep.T + t) * ep.hd + fi
+                                           : ((static_cast<size_t>(b) * ep.H + hh) * ep.cap + pos) * ep.hd + fi;
+                if (col < p.N && inb) qkv_dst[o] = __float2bfloat16_rn(x);
             }
+            if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(status, kStatusBadIndex);
         } else if constexpr (EPI == EPI_SWIGLU) {
+            // tile row 2f is gate feature f, row 2f+1 the matching up row
             const int f = mt * 64 + (rt >> 1);
+            const bool gate_lane = (rt & 1) == 0 && f < ep.F;
+            float up[GW];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const float up = __shfl_xor_sync(0xffffffffu, a[u], 1);
-                const int col = col0 + 4 * g + u;
-                if ((rt & 1) == 0 && f < ep.F && col < p.N) {
-                    const float gv = a[u];
-                    ep.h[static_cast<size_t>(col) * ep.F + f] = __float2bfloat16_rn(gv / (1.0f + __expf(-gv)) * up);
-                }
+            for (int u = 0; u < GW; ++u) up[u] = __shfl_xor_sync(0xffffffffu, a[u], 1);
+#pragma unroll
+            for (int u = 0; u < GW; ++u) {
+                const __nv_bfloat16 hv = __float2bfloat16_rn(__fdividef(a[u], 1.0f + __expf(-a[u])) * up[u]);
+                if (gate_lane && cg + u < p.N) ep.h[static_cast<size_t>(cg + u) * ep.F + f] = hv;
             }
         } else if constexpr (EPI == EPI_LMHEAD) {
+            // this warp's (max, argmax, sum exp) over its 32 rows, for the 8 columns side by side
+            float m[GW], e[GW];
+            int idx[GW];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int col = col0 + 4 * g + u;
-                const bool ok = row < ep.V && row != ep.mask_id;
+            for (int u = 0; u < GW; ++u) {
+                m[u] = lm_ok ? a[u] : -INFINITY;
+                idx[u] = lm_ok ? row : INT_MAX;
+            }
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) {
+#pragma unroll
+                for (int u = 0; u < GW; ++u) {
+                    const float om = __shfl_xor_sync(0xffffffffu, m[u], off);
+                    const int oi = __shfl_xor_sync(0xffffffffu, idx[u], off);
+                    const bool take = om > m[u] || (om == m[u] && oi < idx[u]);
+                    m[u] = take ? om : m[u];
+                    idx[u] = take ? oi : idx[u];
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < GW; ++u) e[u] = (lm_ok && m[u] != -INFINITY) ? __expf(a[u] - m[u]) : 0.0f;
+            if (lane == 0) {
+#pragma unroll
+                for (int u = 0; u < GW; ++u) {
+                    sm.red[(quarter * 32 + GW * g + u) * 3] = m[u];
+                    sm.red[(quarter * 32 + GW * g + u) * 3 + 2] = __int_as_float(idx[u]);
+                }
+            }
+            warp_reduce_scatter8(e, lane);
+            if ((lane & 3) == 0) sm.red[(quarter * 32 + GW * g + (lane >> 2)) * 3 + 1] = e[0];
+#pragma unroll
+            for (int u = 0; u < GW; ++u) {
+                const int col = cg + u;
                 if (ep.logits && row < ep.V && col < p.N) ep.logits[static_cast<size_t>(col) * ep.V + row] = a[u];
-                // this warp's (max, argmax, sum exp) over its 32 rows
-                float m = ok ? a[u] : -INFINITY;
-                int idx = ok ? row : INT_MAX;
-#pragma unroll
-                for (int off = 16; off > 0; off >>= 1) {
-                    const float om = __shfl_xor_sync(0xffffffffu, m, off);
-                    const int oi = __shfl_xor_sync(0xffffffffu, idx, off);
-                    if (om > m || (om == m && oi < idx)) {
-                        m = om;
-                        idx = oi;
-                    }
-                }
-                const float s = warp_sum((ok && m != -INFINITY) ? __expf(a[u] - m) : 0.0f);
-                if (lane == 0) {
-                    sm.red[(quarter * 32 + 4 * g + u) * 3] = m;
-                    sm.red[(quarter * 32 + 4 * g + u) * 3 + 1] = s;
-                    sm.red[(quarter * 32 + 4 * g + u) * 3 + 2] = __int_as_float(idx);
-                }
                 if (col < p.N && row == sm.kvs[col]) ep.zcur[col] = a[u];  // current ids staged in kvs
             }
         }
