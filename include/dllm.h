@@ -199,7 +199,10 @@ enum {
     DLLM_K_HEAD = 7,        /* LM head + per-tile softmax statistics */
     DLLM_K_HEAD_REDUCE = 8, /* current-id gather, vocab-tile merge */
     DLLM_K_COMMIT = 9,      /* commit / re-mask / drafts */
-    DLLM_NKINDS = 10
+    DLLM_K_LAYER = 10,      /* chained projections of one layer: output (+ residual),
+                               gate/up (+ SwiGLU), down (+ residual), then the next
+                               layer's QKV or the LM head */
+    DLLM_NKINDS = 11
 };
 
 /* Per-kernel timing of denoising steps: with enable, every launch of a step

@@ -37,8 +37,8 @@ struct Layout {
     size_t off_x, off_xn, off_q, off_attn, off_h, off_sq, off_theta;
     int n_sq;
     size_t off_lmp, off_zcur, off_cur, off_x0, off_conf, off_tokconf;
-    size_t off_part, part_floats, off_cnt;
-    int cnt_len;
+    size_t off_part, part_floats, off_cnt, off_done, off_epoch;
+    int cnt_len, done_len;  // per phase slot
     size_t off_tok, off_st, off_stok, off_sst, off_seqkv, off_plan, off_outs, off_status;
     size_t total;
     size_t w_qkv, w_o, w_gu, w_d;  // element offsets inside a layer
@@ -86,11 +86,16 @@ Layout make_layout(const dllm_config& c) {
     L.off_x0 = take(T * 4);
     L.off_conf = take(T * 4);
     L.off_tokconf = take(T * 4);
-    L.part_floats = static_cast<size_t>(kMaxSMs) * 2 * 256 * 128;
-    L.off_part = take(L.part_floats * 4);
+    // chained projections: per phase slot, split partials (one per CTA), tile tickets (one per
+    // 128-byte line) and tile completion flags
+    L.part_floats = static_cast<size_t>(kMaxSMs) * 256 * 128;
+    L.off_part = take(L.part_floats * 4 * kMaxPhases);
     const int mt_max = std::max(std::max(L.head_tiles, L.gu_rows / 128), std::max(L.qkv_rows, L.d_rows) / 128);
-    L.cnt_len = mt_max * ((L.max_tok + 255) / 256 + 1) * 32;  // one ticket per 128-byte line
-    L.off_cnt = take(static_cast<size_t>(L.cnt_len) * 4);
+    L.done_len = mt_max * ((L.max_tok + 255) / 256 + 1);
+    L.cnt_len = L.done_len * 32;
+    L.off_cnt = take(static_cast<size_t>(L.cnt_len) * 4 * kMaxPhases);
+    L.off_done = take(static_cast<size_t>(L.done_len) * 4 * kMaxPhases);
+    L.off_epoch = take(256);
     const size_t S = static_cast<size_t>(c.max_batch) * c.max_ctx;
     L.off_tok = take(S * 4);
     L.off_st = take(S);
@@ -142,7 +147,8 @@ struct dllm_ctx {
     float* theta = nullptr;   // RoPE frequencies [hd/2]
     float *lmp = nullptr, *zcur = nullptr, *conf = nullptr, *tokconf = nullptr;
     int *cur = nullptr, *x0 = nullptr;
-    Scratch scr{};
+    float* chain_part = nullptr;
+    int *chain_cnt = nullptr, *chain_done = nullptr, *epoch = nullptr;
     int *tok = nullptr, *stok = nullptr, *seq_kv = nullptr, *plan = nullptr, *outs = nullptr, *status = nullptr;
     uint8_t *st = nullptr, *sst = nullptr;
     float* logits = nullptr;  // debug, separate allocation
@@ -243,13 +249,16 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
     const Layout& L = ctx->L;
     const int d = c.d_model, F = c.ffn, qd = L.qd, N = B * T;
     cudaStream_t s = ctx->stream;
-    // x = embedding rows, xb = bf16(x) (the next projection's operand), sq = RMSNorm statistics
-    CK(launch_embed(ctx->tok, c.max_ctx, ctx->seq_kv, ctx->emb, ctx->x, ctx->xn, ctx->sq, ctx->cur, B, T, d, s));
+    // x = embedding rows, xb = bf16(x) (the next projection's operand), sq = RMSNorm statistics;
+    // the step counter advances (it tags the chained projections' completion flags)
+    CK(launch_embed(ctx->tok, c.max_ctx, ctx->seq_kv, ctx->emb, ctx->x, ctx->xn, ctx->sq, ctx->cur, ctx->epoch, B, T,
+                    d, s));
     mark(ctx, DLLM_K_EMBED);
     const GemmPlan pq = gemm_plan(L.qkv_rows, N, d, ctx->sms, EPI_QKV);
     const GemmPlan po = gemm_plan(L.o_rows, N, qd, ctx->sms, EPI_RESID);
     const GemmPlan pg = gemm_plan(L.gu_rows, N, d, ctx->sms, EPI_SWIGLU);
     const GemmPlan pd = gemm_plan(L.d_rows, N, F, ctx->sms, EPI_RESID);
+    const GemmPlan ph = gemm_plan(L.head_rows, N, d, ctx->sms, EPI_LMHEAD);
     CUtensorMap tx_xn, tx_attn, tx_h;
     if (!make_tmap_bf16(&tx_xn, ctx->xn, N, d, pq.ntile) || !make_tmap_bf16(&tx_attn, ctx->attn, N, qd, po.ntile) ||
         !make_tmap_bf16(&tx_h, ctx->h, N, F, pd.ntile))
@@ -275,39 +284,68 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
     er.ld_out = d;
     er.xb = ctx->xn;
     er.sq_out = ctx->sq;
+    EpiArgs eh = ep;
+    eh.lm_part = ctx->lmp;
+    eh.zcur = ctx->zcur;
+    eh.cur_tok = ctx->cur;
+    eh.V = c.vocab;
+    eh.mask_id = c.mask_id;
+    eh.logits = (ctx->debug & 1) ? ctx->logits : nullptr;
+    auto qkv_args = [&](int l) {
+        EpiArgs e = ep;
+        e.kc = ctx->kv + static_cast<size_t>(2 * l) * L.kv_half;
+        e.vc = ctx->kv + static_cast<size_t>(2 * l + 1) * L.kv_half;
+        return e;
+    };
+    // phase slot i of a chain uses scratch slot i; consecutive chains are ordered by the stream
+    auto add_phase = [&](ChainArgs& ca, ChainMaps& m, const GemmPlan& p, int epi, EpiArgs e, int dep_rows,
+                         const CUtensorMap& w, const CUtensorMap& x) {
+        const int i = ca.n_phases++;
+        ChainPhase& P = ca.ph[i];
+        P.p = p;
+        P.epi = epi;
+        e.trace = next_trace(ctx);
+        P.ep = e;
+        P.dep_rows = dep_rows;
+        P.partials = ctx->chain_part + static_cast<size_t>(i) * L.part_floats;
+        P.tickets = ctx->chain_cnt + static_cast<size_t>(i) * L.cnt_len;
+        P.done = ctx->chain_done + static_cast<size_t>(i) * L.done_len;
+        m.w[i] = w;
+        m.x[i] = x;
+    };
+    const int smem_budget = (ctx->debug & 8) ? kChainSmemShared : kChainSmemFull;
+    auto run_chain = [&](ChainArgs& ca, const ChainMaps& m, int tag_add, int kind) -> int {
+        ca.epoch = ctx->epoch;
+        ca.tag_mul = c.n_layers + 2;
+        ca.tag_add = tag_add;
+        ca.status = ctx->status;
+        if (!chain_plan(ca, smem_budget)) return fail(ctx, DLLM_ECAPACITY, "projection chain does not fit");
+        CK(chain_launch(m, ca, s, true));
+        mark(ctx, kind);
+        return DLLM_OK;
+    };
+    {
+        ChainArgs ca{};
+        ChainMaps m;
+        add_phase(ca, m, pq, EPI_QKV, qkv_args(0), 0, ctx->tm_qkv[0], tx_xn);
+        if (int rc = run_chain(ca, m, 1, DLLM_K_QKV)) return rc;
+    }
     for (int l = 0; l < c.n_layers; ++l) {
-        __nv_bfloat16* kc = ctx->kv + static_cast<size_t>(2 * l) * L.kv_half;
-        __nv_bfloat16* vc = ctx->kv + static_cast<size_t>(2 * l + 1) * L.kv_half;
-        ep.kc = kc;
-        ep.vc = vc;
-        ep.trace = next_trace(ctx);
-        CK(gemm_launch(EPI_QKV, pq, ctx->tm_qkv[l], tx_xn, ep, ctx->scr, ctx->status, s));
-        mark(ctx, DLLM_K_QKV);
-        CK(launch_attention(ctx->q, kc, vc, ctx->seq_kv, ctx->attn, B, T, c.n_heads, c.head_dim, c.max_ctx, ap, s,
+        const EpiArgs el = qkv_args(l);
+        CK(launch_attention(ctx->q, el.kc, el.vc, ctx->seq_kv, ctx->attn, B, T, c.n_heads, c.head_dim, c.max_ctx, ap, s,
                             true, next_trace(ctx)));
         mark(ctx, DLLM_K_ATTN);
-        er.trace = next_trace(ctx);
-        CK(gemm_launch(EPI_RESID, po, ctx->tm_o[l], tx_attn, er, ctx->scr, ctx->status, s));
-        mark(ctx, DLLM_K_OPROJ);
-        ep.trace = next_trace(ctx);
-        CK(gemm_launch(EPI_SWIGLU, pg, ctx->tm_gu[l], tx_xn, ep, ctx->scr, ctx->status, s));
-        mark(ctx, DLLM_K_GATEUP);
-        er.trace = next_trace(ctx);
-        CK(gemm_launch(EPI_RESID, pd, ctx->tm_d[l], tx_h, er, ctx->scr, ctx->status, s));
-        mark(ctx, DLLM_K_DOWN);
+        // output projection (+ residual) -> gate/up (+ SwiGLU) -> down (+ residual) -> next QKV or LM head
+        ChainArgs ca{};
+        ChainMaps m;
+        add_phase(ca, m, po, EPI_RESID, er, 0, ctx->tm_o[l], tx_attn);
+        add_phase(ca, m, pg, EPI_SWIGLU, ep, 128, ctx->tm_gu[l], tx_xn);
+        add_phase(ca, m, pd, EPI_RESID, er, 64, ctx->tm_d[l], tx_h);
+        if (l + 1 < c.n_layers) add_phase(ca, m, pq, EPI_QKV, qkv_args(l + 1), 128, ctx->tm_qkv[l + 1], tx_xn);
+        else if (head) add_phase(ca, m, ph, EPI_LMHEAD, eh, 128, ctx->tm_head, tx_xn);
+        if (int rc = run_chain(ca, m, l + 2, DLLM_K_LAYER)) return rc;
     }
     if (head) {
-        const GemmPlan ph = gemm_plan(L.head_rows, N, d, ctx->sms, EPI_LMHEAD);
-        EpiArgs eh = ep;
-        eh.lm_part = ctx->lmp;
-        eh.zcur = ctx->zcur;
-        eh.cur_tok = ctx->cur;
-        eh.V = c.vocab;
-        eh.mask_id = c.mask_id;
-        eh.logits = (ctx->debug & 1) ? ctx->logits : nullptr;
-        eh.trace = next_trace(ctx);
-        CK(gemm_launch(EPI_LMHEAD, ph, ctx->tm_head, tx_xn, eh, ctx->scr, ctx->status, s));
-        mark(ctx, DLLM_K_HEAD);
         CK(launch_lmhead_reduce(ctx->lmp, ctx->zcur, ctx->cur, L.head_tiles, N, c.mask_id, ctx->x0, ctx->conf,
                                 ctx->tokconf, s));
         mark(ctx, DLLM_K_HEAD_REDUCE);
@@ -434,7 +472,7 @@ int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void*
         if (cudaMalloc(&ctx->arena, L.total) != cudaSuccess) return bail(DLLM_ENOMEM, "device allocation failed");
         ctx->own_arena = true;
     }
-    if (gemm_init_attrs() != cudaSuccess || attn_init_attrs() != cudaSuccess)
+    if (gemm_init_attrs() != cudaSuccess || attn_init_attrs() != cudaSuccess || chain_init_attrs() != cudaSuccess)
         return bail(DLLM_ECUDA, "kernel attribute setup failed");
     uint8_t* A = ctx->arena;
     const int d = c.d_model, F = c.ffn, qd = L.qd;
@@ -454,10 +492,10 @@ int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void*
     ctx->x0 = reinterpret_cast<int*>(A + L.off_x0);
     ctx->conf = reinterpret_cast<float*>(A + L.off_conf);
     ctx->tokconf = reinterpret_cast<float*>(A + L.off_tokconf);
-    ctx->scr.partials = reinterpret_cast<float*>(A + L.off_part);
-    ctx->scr.partial_floats = L.part_floats;
-    ctx->scr.counters = reinterpret_cast<int*>(A + L.off_cnt);
-    ctx->scr.counter_len = L.cnt_len;
+    ctx->chain_part = reinterpret_cast<float*>(A + L.off_part);
+    ctx->chain_cnt = reinterpret_cast<int*>(A + L.off_cnt);
+    ctx->chain_done = reinterpret_cast<int*>(A + L.off_done);
+    ctx->epoch = reinterpret_cast<int*>(A + L.off_epoch);
     ctx->tok = reinterpret_cast<int*>(A + L.off_tok);
     ctx->st = A + L.off_st;
     ctx->stok = reinterpret_cast<int*>(A + L.off_stok);

@@ -144,7 +144,7 @@ __device__ __forceinline__ void epilogue_chunk(const EpiArgs& ep, const GemmPlan
     }
     if constexpr (EPI == EPI_F32) {
         if (row < p.M) {
-#pragma unroll 8
+#pragma unroll
             for (int j = 0; j < 32; ++j) {
                 const int col = col0 + j;
                 if (col < p.N) ep.out[static_cast<size_t>(col) * ep.ld_out + row] = v[j];
@@ -407,38 +407,48 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
             warp_reduce_scatter8(ss, lane);
             if ((lane & 3) == 0) sm.red[quarter * 32 + GW * g + (lane >> 2)] = ss[0];
         } else if constexpr (EPI == EPI_QKV) {
+            // positions and rotations of the group's 8 columns first (the rare tile that spans
+            // sequences takes the out-of-line sincos per column), then the branch-free column pass
+            int bs[GW], ts[GW];
+            float cs[GW], ss[GW];
+            if (run) {
+#pragma unroll
+                for (int u = 0; u < GW; ++u) {
+                    bs[u] = bl;
+                    ts[u] = cg + u - bl * ep.T;
+                    cs[u] = cn;
+                    ss[u] = sn;
+                    const float c2 = cn * cd - sn * sd;  // angle-addition step to the next position
+                    sn = sn * cd + cn * sd;
+                    cn = c2;
+                }
+            } else {
+#pragma unroll
+                for (int u = 0; u < GW; ++u) {
+                    const int b = min((cg + u) / ep.T, ep.n_seq - 1);
+                    bs[u] = b;
+                    ts[u] = cg + u - b * ep.T;
+                    const float2 r = rot_cs(static_cast<float>(sm.kvs[b] + ts[u]) * theta);
+                    cs[u] = r.x;
+                    ss[u] = r.y;
+                }
+            }
             float xp[GW];
 #pragma unroll
             for (int u = 0; u < GW; ++u) xp[u] = __shfl_xor_sync(0xffffffffu, a[u], 1);
             bool bad = false;
+            const size_t head_base = static_cast<size_t>(hh) * (part == 0 ? ep.T : ep.cap);
+            const size_t seq_stride = static_cast<size_t>(ep.H) * (part == 0 ? ep.T : ep.cap);
 #pragma unroll
             for (int u = 0; u < GW; ++u) {
                 const int col = cg + u;
-                int b = bl, t = col - bl * ep.T;
-                if (!run) {  // the tile spans sequences (uniform over the warp)
-                    b = min(col / ep.T, ep.n_seq - 1);
-                    t = col - b * ep.T;
-                }
-                const int pos = sm.kvs[b] + t;
+                const int pos = sm.kvs[bs[u]] + ts[u];
                 const bool inb = pos >= 0 && pos < ep.cap;
                 bad |= col < p.N && !inb;
                 float x = a[u];
-                if (part < 2) {
-                    if (!run) {
-                        const float2 r = rot_cs(static_cast<float>(pos) * theta);
-                        cn = r.x;
-                        sn = r.y;
-                    }
-                    x = (pp & 1) ? (x * cn + xp[u] * sn) : (x * cn - xp[u] * sn);
-                    if (run) {
-                        const float c2 = cn * cd - sn * sd;
-                        sn = sn * cd + cn * sd;
-                        cn = c2;
-                    }
-                }
-                const size_t o = part == 0 ? ((static_cast<size_t>(b) * ep.H + hh) * ep.T + t) * ep.hd + fi
-                                           : ((static_cast<size_t>(b) * ep.H + hh) * ep.cap + pos) * ep.hd + fi;
-                if (col < p.N && inb) qkv_dst[o] = __float2bfloat16_rn(x);
+                if (part < 2) x = (pp & 1) ? (x * cs[u] + xp[u] * ss[u]) : (x * cs[u] - xp[u] * ss[u]);
+                const size_t r = static_cast<size_t>(bs[u]) * seq_stride + head_base + (part == 0 ? ts[u] : pos);
+                if (col < p.N && inb) qkv_dst[r * ep.hd + fi] = __float2bfloat16_rn(x);
             }
             if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(status, kStatusBadIndex);
         } else if constexpr (EPI == EPI_SWIGLU) {
@@ -782,8 +792,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 }
             }
             mbar_wait(&tfull[acc], acc_phase, s_abort, status);
-            named_bar(1, 128);
-            if (*s_abort) break;
+            if (named_bar_any(1, 128, *s_abort != 0)) break;
             if (tr && threadIdx.x == 64) {
                 tr[kTrAccReady] = global_ns();
                 tr[kTrTile] = static_cast<unsigned long long>(tile);
@@ -850,8 +859,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                         tr[kTrIsLast] = 1;
                     }
                 }
-                named_bar(1, 128);
-                if (*s_abort) break;
+                if (named_bar_any(1, 128, *s_abort != 0)) break;
                 const uint32_t part_bytes = static_cast<uint32_t>(slot_floats * 4);
                 const uint32_t stage_room = static_cast<uint32_t>(S) * (kABytes + b_bytes);
                 const bool final_seg = tile * p.kb + k_hi == it1;  // pipeline drained: stage memory free
@@ -936,6 +944,533 @@ __global__ void __launch_bounds__(kThreads, 2)
     if (warp == 1) {
         __syncwarp();
         tmem_dealloc(tmem_base, p.tmem_cols);
+    }
+}
+
+// ================================================================== chained projections
+// k_chain runs the phases of a ChainArgs in one launch, one CTA per SM.  Roles (224
+// threads): warp 0 = weight producer (never waits on data: weights are constant, so it runs
+// ahead by the whole ring, across phase boundaries), warp 6 = operand producer (waits for
+// the completion flag of the tile that writes each X k-block), warp 1 = TMEM owner and MMA
+// issuer, warps 2..5 = epilogue.  Ring stages, TMEM accumulators and their barriers are
+// shared by all phases; a running iteration counter gives every stage its use parity.
+constexpr int kChainThreads = 224;
+
+struct ChainEpiState {
+    int acc;
+    uint32_t acc_phase;
+    uint32_t red_phase;
+};
+
+__device__ __forceinline__ int chain_tag(const ChainArgs& ca) {
+    return ca.epoch ? *reinterpret_cast<const volatile int*>(ca.epoch) * ca.tag_mul + ca.tag_add : ca.tag_add;
+}
+
+// Wait (bounded) until flag == tag.  Returns false after raising *abort on a timeout.
+__device__ __forceinline__ bool wait_flag(const int* flag, int tag, volatile int* abort, int* status) {
+    if (ld_acquire(flag) == tag) return true;
+    const unsigned long long t0 = global_ns();
+    while (ld_acquire(flag) != tag) {
+        if (*abort) return false;
+        if (global_ns() - t0 > kWaitLimitNs) {
+            *abort = 1;
+            atomicOr(status, kStatusTimeout);
+            return false;
+        }
+    }
+    return true;
+}
+
+// The epilogue warps' share of one phase: every tile of this CTA's range.
+template <int EPI>
+__device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph, int tag, uint8_t* red_stage,
+                                                  uint64_t* tfull, uint64_t* tempty, uint64_t* redbar,
+                                                  volatile int* s_abort, uint32_t tmem_base, const EpiSmem& esm,
+                                                  ChainEpiState& es) {
+    const ChainPhase& P = ca.ph[ph];
+    const GemmPlan& p = P.p;
+    const EpiArgs& ep = P.ep;
+    int* status = ca.status;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int ew = warp - 2;
+    const int quarter = warp & 3;
+    const int rt = quarter * 32 + lane;
+    const int G = p.grid;
+    if (static_cast<int>(blockIdx.x) >= G) return;
+    const long long it0 = range_begin(blockIdx.x, p.total, G);
+    const long long it1 = range_begin(blockIdx.x + 1, p.total, G);
+    if (it0 >= it1) return;
+    unsigned long long* tr = ep.trace ? ep.trace + static_cast<size_t>(blockIdx.x) * kTrSlots : nullptr;
+    if (tr && threadIdx.x == 64) {
+        tr[kTrSm] = smid();
+        for (int i = kTrAccReady; i < kTrSlots; ++i) tr[i] = 0;
+    }
+    // every tile of the previous phase: its RMSNorm statistics and residual rows are read here
+    if (ph > 0 && ca.ph[ph - 1].done) {
+        const ChainPhase& Q = ca.ph[ph - 1];
+        if (ew == 0) {
+            const int n = Q.p.m_tiles * Q.p.n_tiles;
+            for (int i = lane; i < n; i += 32)
+                if (!wait_flag(Q.done + i, tag, s_abort, status)) break;
+        }
+        if (named_bar_any(1, 128, *s_abort != 0)) return;
+    }
+    if (tr && threadIdx.x == 64) tr[kTrDepWait] = global_ns();
+    if constexpr (EPI == EPI_QKV) {
+        for (int b = ew * 32 + lane; b < ep.n_seq; b += 128) esm.kvs[b] = ep.seq_kv[b];
+        esm.theta[rt] = ep.theta[(rt % ep.hd) >> 1];
+        named_bar(1, 128);
+    }
+    if constexpr (EPI == EPI_LMHEAD) {
+        if (p.ntile == 32) {
+            for (int c = ew * 32 + lane; c < p.N && c < 256; c += 128) esm.kvs[c] = ep.cur_tok[c];
+            named_bar(1, 128);
+        }
+    }
+    const int nchunks = p.ntile / 32;
+    const size_t slot_floats = static_cast<size_t>(p.ntile) * kBM;
+    const bool c32 = p.ntile == 32;
+    // TMEM: two accumulators of acc_cols columns, then (32-token tiles) the staged residual
+    const uint32_t t_x = tmem_base + static_cast<uint32_t>(2 * ca.acc_cols) + (static_cast<uint32_t>(quarter * 32) << 16);
+    int rs_nt = -1;
+    float v[32];
+    for (long long it = it0; it < it1;) {
+        const long long tile = it / p.kb;
+        const int k_lo = static_cast<int>(it - tile * p.kb);
+        const long long tend = (tile + 1) * p.kb;
+        const int k_hi = static_cast<int>((it1 < tend ? it1 : tend) - tile * p.kb);
+        const int mt = static_cast<int>(tile / p.n_tiles);
+        const int nt = static_cast<int>(tile - static_cast<long long>(mt) * p.n_tiles);
+        const bool whole = (k_lo == 0 && k_hi == p.kb);
+        int c_first = 0, c_last = 0;
+        bool reducer = false;
+        if (!whole) {
+            c_first = owner_of(tile * p.kb, p.total, G);
+            c_last = owner_of(tile * p.kb + p.kb - 1, p.total, G);
+            reducer = static_cast<int>(blockIdx.x) == c_first;
+        }
+        const bool finisher = whole || reducer;
+        if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
+            if (finisher && ep.sq_in && nt != rs_nt) {
+                compute_norm_scale(ep, p, nt, esm, ew * 32 + lane);
+                rs_nt = nt;
+            }
+        }
+        if constexpr (EPI == EPI_RESID) {
+            if (c32 && finisher) {  // stage the tile's old residual in TMEM while the accumulator is produced
+                const int row = mt * kBM + rt;
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                    const int col = nt * 32 + j;
+                    v[j] = (row < p.M && col < p.N) ? ep.out[static_cast<size_t>(col) * ep.ld_out + row] : 0.0f;
+                }
+                tmem_st_32x32(t_x, v);
+            }
+        }
+        mbar_wait(&tfull[es.acc], es.acc_phase, s_abort, status);
+        if (named_bar_any(1, 128, *s_abort != 0)) return;
+        if (tr && threadIdx.x == 64) {
+            tr[kTrAccReady] = global_ns();
+            tr[kTrTile] = static_cast<unsigned long long>(tile);
+        }
+        tc_fence_after();
+        const uint32_t t_acc = tmem_base + static_cast<uint32_t>(es.acc * ca.acc_cols) +
+                               (static_cast<uint32_t>(quarter * 32) << 16);
+        if (whole && c32) {
+            epilogue_c32<EPI>(ep, p, mt, nt, rt, t_acc, t_x, esm, ew, quarter, lane, status);
+        } else if (!reducer) {
+            float* my_part = P.partials + static_cast<size_t>(blockIdx.x) * slot_floats;
+            for (int c = 0; c < nchunks; ++c) {
+                tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);
+                if (whole) {
+                    epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
+                } else {
+                    float4* dst = reinterpret_cast<float4*>(my_part);
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        dst[static_cast<size_t>(c * 8 + j) * kBM + rt] =
+                            make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+                }
+            }
+        }
+        if (!c32 && !reducer) {
+            tc_fence_before();
+            mbar_arrive(&tempty[es.acc]);
+        }
+        if (!whole && !reducer) {
+            named_bar(1, 128);
+            if (threadIdx.x == 64) {
+                if (tr) tr[kTrPartStored] = global_ns();
+                red_release_add(&P.tickets[tile * kTicketStride], 1);
+            }
+        } else if (reducer) {
+            const int nparts = c_last - c_first + 1;
+            int* ticket = &P.tickets[tile * kTicketStride];
+            if (threadIdx.x == 64) {
+                if (tr) tr[kTrPartStored] = global_ns();
+                wait_flag(ticket, nparts - 1, s_abort, status);
+                *ticket = 0;
+                if (tr) {
+                    tr[kTrTicket] = global_ns();
+                    tr[kTrIsLast] = 1;
+                }
+            }
+            if (named_bar_any(1, 128, *s_abort != 0)) return;
+            const uint32_t part_bytes = static_cast<uint32_t>(slot_floats * 4);
+            for (int c = 0; c < nchunks; ++c) {
+                tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);  // own (first) k-range
+                if (c32 && ca.red_bytes >= static_cast<int>(part_bytes)) {
+                    const int per_batch = ca.red_bytes / static_cast<int>(part_bytes);
+                    for (int b0 = 1; b0 < nparts; b0 += per_batch) {
+                        const int nb = nparts - b0 < per_batch ? nparts - b0 : per_batch;
+                        if (threadIdx.x == 64) {
+                            fence_proxy_async_global();
+                            mbar_arrive_expect_tx(redbar, part_bytes * static_cast<uint32_t>(nb));
+                            for (int q = 0; q < nb; ++q)
+                                bulk_load(red_stage + static_cast<size_t>(q) * part_bytes,
+                                          P.partials + static_cast<size_t>(c_first + b0 + q) * slot_floats, part_bytes,
+                                          redbar);
+                        }
+                        mbar_wait(redbar, es.red_phase, s_abort, status);
+                        es.red_phase ^= 1u;
+                        for (int q = 0; q < nb; ++q) {
+                            const float4* src =
+                                reinterpret_cast<const float4*>(red_stage + static_cast<size_t>(q) * part_bytes);
+#pragma unroll
+                            for (int j = 0; j < 8; ++j) {
+                                const float4 a = src[j * kBM + rt];
+                                v[4 * j] += a.x;
+                                v[4 * j + 1] += a.y;
+                                v[4 * j + 2] += a.z;
+                                v[4 * j + 3] += a.w;
+                            }
+                        }
+                        named_bar(1, 128);  // the next batch overwrites the staging memory
+                    }
+                } else {
+                    for (int cc = c_first + 1; cc <= c_last; ++cc) {
+                        const float4* p0 =
+                            reinterpret_cast<const float4*>(P.partials + static_cast<size_t>(cc) * slot_floats);
+                        float4 a[8];
+#pragma unroll
+                        for (int j = 0; j < 8; ++j) a[j] = __ldcg(p0 + static_cast<size_t>(c * 8 + j) * kBM + rt);
+#pragma unroll
+                        for (int j = 0; j < 8; ++j) {
+                            v[4 * j] += a[j].x;
+                            v[4 * j + 1] += a[j].y;
+                            v[4 * j + 2] += a[j].z;
+                            v[4 * j + 3] += a[j].w;
+                        }
+                    }
+                }
+                if (tr && threadIdx.x == 64 && c == 0) tr[kTrReduced] = global_ns();
+                if (c32) {
+                    tmem_st_32x32(t_acc, v);
+                    epilogue_c32<EPI>(ep, p, mt, nt, rt, t_acc, t_x, esm, ew, quarter, lane, status);
+                } else {
+                    epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
+                }
+            }
+            if (!c32) {
+                tc_fence_before();
+                mbar_arrive(&tempty[es.acc]);
+            }
+        }
+        if (c32) {
+            tc_fence_before();
+            mbar_arrive(&tempty[es.acc]);
+        }
+        if (finisher && P.done) {  // publish the finished tile to the next phase's operand producer
+            named_bar(1, 128);
+            if (threadIdx.x == 64) st_release(&P.done[mt * p.n_tiles + nt], tag);
+        }
+        if (++es.acc == 2) {
+            es.acc = 0;
+            es.acc_phase ^= 1u;
+        }
+        it = tile * p.kb + k_hi;
+    }
+    if (tr && threadIdx.x == 64) tr[kTrEpiDone] = global_ns();
+}
+
+__global__ void __launch_bounds__(kChainThreads, 1)
+    k_chain(const __grid_constant__ ChainMaps maps, const __grid_constant__ ChainArgs ca) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int S = ca.stages;
+    const uint32_t b_bytes = static_cast<uint32_t>(ca.ntile) * kBK * 2;
+    uint8_t* sA = smem;
+    uint8_t* sB = sA + static_cast<size_t>(S) * kABytes;
+    uint8_t* red_stage = sB + static_cast<size_t>(S) * b_bytes;
+    float* tail = reinterpret_cast<float*>(red_stage + ca.red_bytes);
+    EpiSmem esm;
+    esm.rs = tail;
+    esm.red = tail + 256;
+    esm.kvs = reinterpret_cast<int*>(tail + 256 + 1024);
+    esm.theta = tail + 256 + 1024 + 256;
+    esm.stg = tail + 256 + 1024 + 256 + 128;
+    float* after = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(esm.stg) + ca.stg_bytes);
+    uint64_t* full = reinterpret_cast<uint64_t*>(after);
+    uint64_t* empty = full + S;
+    uint64_t* tfull = empty + S;
+    uint64_t* tempty = tfull + 2;
+    uint64_t* drain = tempty + 2;
+    uint64_t* redbar = drain + 1;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(redbar + 1);
+    volatile int* s_abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    int* status = ca.status;
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        pdl_launch_dependents();
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(&tfull[a], 1);
+            mbar_init(&tempty[a], 128);
+        }
+        mbar_init(drain, 1);
+        mbar_init(redbar, 1);
+        *s_abort = 0;
+        mbar_fence_init();
+    }
+    if (warp == 0 && lane == 0) {
+        for (int ph = 0; ph < ca.n_phases; ++ph) tma_prefetch_desc(&maps.w[ph]);
+    }
+    if (warp == 6 && lane == 0) {
+        for (int ph = 0; ph < ca.n_phases; ++ph) tma_prefetch_desc(&maps.x[ph]);
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_slot, ca.tmem_cols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+    const int acc_cols = ca.acc_cols;
+
+    if (warp == 0) {
+        // ---------------------------------------------------------- weight producer
+        if (lane == 0) {
+            const uint64_t pol_w = policy_evict_first();
+            int stage = 0;
+            uint32_t par = 0;
+            uint32_t pending = 0, pend_par = 0;
+            for (int ph = 0; ph < ca.n_phases && !*s_abort; ++ph) {
+                const GemmPlan& p = ca.ph[ph].p;
+                if (static_cast<int>(blockIdx.x) >= p.grid) continue;
+                const int it0 = static_cast<int>(range_begin(blockIdx.x, p.total, p.grid));
+                const int it1 = static_cast<int>(range_begin(blockIdx.x + 1, p.total, p.grid));
+                unsigned long long* tr = ca.ph[ph].ep.trace ? ca.ph[ph].ep.trace + static_cast<size_t>(blockIdx.x) * kTrSlots : nullptr;
+                if (tr) tr[kTrStart] = global_ns();
+                // (m-tile, k-block) walked incrementally: no division in the loop
+                int tile = it0 / p.kb, k = it0 - tile * p.kb;
+                int mt = tile / p.n_tiles, nt = tile - mt * p.n_tiles;
+                for (int it = it0; it < it1; ++it) {
+                    if (!mbar_wait(&empty[stage], par ^ 1u, s_abort, status)) break;
+                    mbar_arrive_expect_tx(&full[stage], kABytes + b_bytes);
+                    tma_load_2d(sA + static_cast<size_t>(stage) * kABytes, &maps.w[ph], k * kBK, mt * kBM, &full[stage],
+                                pol_w);
+                    pending |= 1u << stage;
+                    pend_par = (pend_par & ~(1u << stage)) | (par << stage);
+                    if (++stage == S) {
+                        stage = 0;
+                        par ^= 1u;
+                    }
+                    if (++k == p.kb) {
+                        k = 0;
+                        if (++nt == p.n_tiles) {
+                            nt = 0;
+                            ++mt;
+                        }
+                    }
+                }
+            }
+            if (*s_abort) {
+                // let the copies in flight land before the CTA's shared memory is released (a
+                // stage whose operand was never issued does not complete: one deadline for all)
+                const unsigned long long t0 = global_ns();
+                for (int s = 0; s < S; ++s) {
+                    if (!(pending >> s & 1u)) continue;
+                    while (!mbar_try_wait(&full[s], (pend_par >> s) & 1u) && global_ns() - t0 < kWaitLimitNs) {
+                    }
+                }
+            }
+        }
+    } else if (warp == 6) {
+        // ---------------------------------------------------------- operand producer
+        // The whole warp runs the loop: lane 0 issues the copies, and the completion flags of
+        // the producing tiles are polled 32 at a time (one round trip covers the next 32).
+        const uint64_t pol_x = policy_evict_last();
+        pdl_wait();
+        const int tag = chain_tag(ca);
+        int stage = 0;
+        uint32_t par = 0;
+        bool stop = false;
+        for (int ph = 0; ph < ca.n_phases && !stop; ++ph) {
+            const ChainPhase& P = ca.ph[ph];
+            const GemmPlan& p = P.p;
+            if (static_cast<int>(blockIdx.x) >= p.grid) continue;
+            const int it0 = static_cast<int>(range_begin(blockIdx.x, p.total, p.grid));
+            const int it1 = static_cast<int>(range_begin(blockIdx.x + 1, p.total, p.grid));
+            const int* dep = (ph > 0 && P.dep_rows > 0) ? ca.ph[ph - 1].done : nullptr;
+            const int dep_tiles = dep ? ca.ph[ph - 1].p.m_tiles : 0;
+            int win_base = -1, win_nt = -1;  // the 32 producing tiles last polled
+            uint32_t win_ready = 0;
+            int tile = it0 / p.kb, k = it0 - tile * p.kb;
+            int mt = tile / p.n_tiles, nt = tile - mt * p.n_tiles;
+            for (int it = it0; it < it1; ++it) {
+                int free_stage = 1;
+                if (lane == 0) free_stage = mbar_wait(&empty[stage], par ^ 1u, s_abort, status) ? 1 : 0;
+                if (!__shfl_sync(0xffffffffu, free_stage, 0)) {  // warp-uniform decision
+                    stop = true;
+                    break;
+                }
+                if (dep) {
+                    const int pmt = (k * kBK) / P.dep_rows;
+                    if (nt != win_nt || pmt < win_base || pmt >= win_base + 32) {
+                        win_base = pmt;
+                        win_nt = nt;
+                        win_ready = 0;
+                    }
+                    const unsigned long long t0 = global_ns();
+                    while (!(win_ready >> (pmt - win_base) & 1u)) {
+                        const int i = win_base + lane;
+                        const bool ok = i >= dep_tiles || ld_acquire(dep + i * p.n_tiles + nt) == tag;
+                        win_ready = __ballot_sync(0xffffffffu, ok);
+                        if (win_ready >> (pmt - win_base) & 1u) {
+                            fence_proxy_async_global();  // generic-proxy writes of other CTAs -> these TMA reads
+                            break;
+                        }
+                        int give_up = 0;
+                        if (lane == 0) give_up = (*s_abort || global_ns() - t0 > kWaitLimitNs) ? 1 : 0;
+                        if (__shfl_sync(0xffffffffu, give_up, 0)) {  // warp-uniform decision
+                            if (lane == 0 && !*s_abort) {
+                                *s_abort = 1;
+                                atomicOr(status, kStatusTimeout);
+                            }
+                            stop = true;
+                            break;
+                        }
+                    }
+                    if (stop) break;
+                }
+                if (lane == 0)
+                    tma_load_2d(sB + static_cast<size_t>(stage) * b_bytes, &maps.x[ph], k * kBK, nt * ca.ntile,
+                                &full[stage], pol_x);
+                __syncwarp();
+                if (++stage == S) {
+                    stage = 0;
+                    par ^= 1u;
+                }
+                if (++k == p.kb) {
+                    k = 0;
+                    if (++nt == p.n_tiles) {
+                        nt = 0;
+                        ++mt;
+                    }
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ---------------------------------------------------------- MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = umma_idesc_bf16(kBM, ca.ntile);
+            int stage = 0;
+            uint32_t par = 0;
+            int acc = 0;
+            uint32_t acc_phase = 0;
+            bool issued = false;
+            for (int ph = 0; ph < ca.n_phases && !*s_abort; ++ph) {
+                const GemmPlan& p = ca.ph[ph].p;
+                if (static_cast<int>(blockIdx.x) >= p.grid) continue;
+                const long long it0 = range_begin(blockIdx.x, p.total, p.grid);
+                const long long it1 = range_begin(blockIdx.x + 1, p.total, p.grid);
+                unsigned long long* tr = ca.ph[ph].ep.trace ? ca.ph[ph].ep.trace + static_cast<size_t>(blockIdx.x) * kTrSlots : nullptr;
+                bool first = true;
+                for (long long it = it0; it < it1 && !*s_abort;) {
+                    const long long tile = it / p.kb;
+                    const int k_lo = static_cast<int>(it - tile * p.kb);
+                    const long long tend = (tile + 1) * p.kb;
+                    const int k_hi = static_cast<int>((it1 < tend ? it1 : tend) - tile * p.kb);
+                    if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, s_abort, status)) break;
+                    tc_fence_after();
+                    const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * acc_cols);
+                    bool ok = true;
+                    for (int k = k_lo; k < k_hi; ++k) {
+                        if (!mbar_wait(&full[stage], par, s_abort, status)) {
+                            ok = false;
+                            break;
+                        }
+                        if (tr && first) tr[kTrFirstData] = global_ns();
+                        first = false;
+                        tc_fence_after();
+                        const uint64_t adesc = sw128_kmajor_desc(smem_u32(sA + static_cast<size_t>(stage) * kABytes));
+                        const uint64_t bdesc = sw128_kmajor_desc(smem_u32(sB + static_cast<size_t>(stage) * b_bytes));
+#pragma unroll
+                        for (int kk = 0; kk < kBK / 16; ++kk)
+                            umma_bf16(d_tmem, adesc + 2ull * kk, bdesc + 2ull * kk, idesc,
+                                      (k > k_lo || kk > 0) ? 1u : 0u);
+                        issued = true;
+                        umma_commit(&empty[stage]);
+                        if (++stage == S) {
+                            stage = 0;
+                            par ^= 1u;
+                        }
+                    }
+                    if (!ok) break;
+                    umma_commit(&tfull[acc]);
+                    if (++acc == 2) {
+                        acc = 0;
+                        acc_phase ^= 1u;
+                    }
+                    it = tile * p.kb + k_hi;
+                }
+                if (tr) tr[kTrLastData] = global_ns();
+            }
+            if (*s_abort && issued) {
+                umma_commit(drain);
+                const unsigned long long t0 = global_ns();
+                while (!mbar_try_wait(drain, 0) && global_ns() - t0 < kWaitLimitNs) {
+                }
+            }
+        }
+    } else {
+        // ---------------------------------------------------------- epilogue
+        pdl_wait();
+        const int tag = chain_tag(ca);
+        ChainEpiState es{0, 0u, 0u};
+        for (int ph = 0; ph < ca.n_phases; ++ph) {  // on abort every phase returns at its first barrier
+            switch (ca.ph[ph].epi) {
+                case EPI_F32:
+                    chain_phase_epilogue<EPI_F32>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    break;
+                case EPI_RESID:
+                    chain_phase_epilogue<EPI_RESID>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    break;
+                case EPI_QKV:
+                    chain_phase_epilogue<EPI_QKV>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    break;
+                case EPI_SWIGLU:
+                    chain_phase_epilogue<EPI_SWIGLU>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    break;
+                default:
+                    chain_phase_epilogue<EPI_LMHEAD>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    break;
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) {
+        __syncwarp();
+        tmem_dealloc(tmem_base, ca.tmem_cols);
     }
 }
 
@@ -1046,5 +1581,48 @@ void set_stream_smem(bool coresident) { g_stream_budget = coresident ? kStreamSm
 static bool g_pdl = true;
 void set_pdl(bool on) { g_pdl = on; }
 bool pdl_enabled() { return g_pdl; }
+
+
+bool chain_plan(ChainArgs& ca, int smem_budget) {
+    if (ca.n_phases < 1 || ca.n_phases > kMaxPhases) return false;
+    const int ntile = ca.ph[0].p.ntile;
+    int grid = 0;
+    bool lm_wide = false;
+    for (int i = 0; i < ca.n_phases; ++i) {
+        const GemmPlan& p = ca.ph[i].p;
+        if (p.ntile != ntile || p.N != ca.ph[0].p.N) return false;
+        grid = grid > p.grid ? grid : p.grid;
+        if (ca.ph[i].epi == EPI_LMHEAD && ntile != 32) lm_wide = true;
+    }
+    const bool c32 = ntile == 32;
+    ca.grid = grid;
+    ca.ntile = ntile;
+    ca.acc_cols = c32 ? 32 : pow2ceil(ntile);
+    ca.tmem_cols = pow2ceil(2 * ca.acc_cols + (c32 ? 32 : 0));
+    ca.red_bytes = c32 ? 2 * 32 * kBM * 4 : 0;  // two split partials per bulk-copy round
+    ca.stg_bytes = lm_wide ? kBM * kStageLd * 4 : 0;
+    const int fixed = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.stg_bytes + ca.red_bytes + 6 * 8 + 16;
+    const int stage_bytes = static_cast<int>(kABytes) + ntile * kBK * 2;
+    int st = (smem_budget - fixed) / (stage_bytes + 16);
+    if (st > 32) st = 32;
+    if (st < 2) return false;
+    ca.stages = st;
+    ca.smem = static_cast<size_t>(fixed) + static_cast<size_t>(st) * (stage_bytes + 16);
+    return ca.smem <= static_cast<size_t>(kFullSmem);
+}
+
+cudaError_t chain_init_attrs() {
+    return cudaFuncSetAttribute(reinterpret_cast<const void*>(k_chain), cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                kFullSmem);
+}
+
+cudaError_t chain_launch(const ChainMaps& maps, const ChainArgs& ca, cudaStream_t st, bool pdl) {
+    for (int i = 0; i < ca.n_phases; ++i) {
+        const GemmPlan& p = ca.ph[i].p;
+        if (p.grid > ca.grid || !ca.ph[i].partials || !ca.ph[i].tickets || (i > 0 && ca.ph[i].dep_rows < 0))
+            return cudaErrorInvalidValue;
+    }
+    return launch_k(k_chain, dim3(ca.grid), dim3(kChainThreads), ca.smem, st, pdl, maps, ca);
+}
 
 }  // namespace dllm

@@ -74,6 +74,45 @@ struct Scratch {
     int counter_len;
 };
 
+// ---------------------------------------------------------------- chained projections
+// One persistent launch (one CTA per SM) runs up to kMaxPhases projections back to back,
+// e.g. output projection -> gate/up -> down -> the next layer's QKV.  The weight ring
+// streams on from one phase into the next while the previous phase's split tiles are
+// reduced and its epilogues run; the operand (X) of phase i, k-block k, is loaded once the
+// tile of phase i-1 that produces it has published its completion flag.
+constexpr int kMaxPhases = 4;
+struct ChainPhase {
+    GemmPlan p;          // from gemm_plan (grid <= the chain's grid)
+    EpiArgs ep;
+    int epi;             // EpiKind
+    int dep_rows;        // X k-block k comes from tile (64k)/dep_rows of the previous phase; 0: ready at launch
+    int* done;           // [m_tiles][n_tiles] completion flags (value: the launch's tag); may be null
+    float* partials;     // [grid][ntile*128] split partials (a CTA contributes to at most one tile per phase)
+    int* tickets;        // [m_tiles*n_tiles][32], zero between launches
+};
+struct ChainArgs {
+    int n_phases;
+    int grid, stages, ntile, acc_cols, tmem_cols;
+    int red_bytes;       // shared staging for split partials (32-token tiles)
+    int stg_bytes;       // LM-head staging (wide token tiles)
+    size_t smem;
+    const int* epoch;    // device step counter; tag = *epoch * tag_mul + tag_add (null: tag = tag_add)
+    int tag_mul, tag_add;
+    int* status;
+    ChainPhase ph[kMaxPhases];
+};
+struct ChainMaps {
+    CUtensorMap w[kMaxPhases];
+    CUtensorMap x[kMaxPhases];
+};
+// Fills grid, stages, ntile, acc_cols, tmem_cols, red_bytes, stg_bytes and smem from the phases' plans for a
+// shared-memory budget (bytes, <= 227 KB).  False if the phases do not share one token tiling.
+bool chain_plan(ChainArgs& ca, int smem_budget);
+constexpr int kChainSmemFull = 227 * 1024;    // one CTA per SM, deepest ring
+constexpr int kChainSmemShared = 146 * 1024;  // leaves room for two attention CTAs beside it
+cudaError_t chain_launch(const ChainMaps& maps, const ChainArgs& ca, cudaStream_t st, bool pdl);
+cudaError_t chain_init_attrs();
+
 // Shared memory budget: at most 96 tokens per tile the kernel is a weight stream and keeps
 // to 113 KB so that the next projection's CTA fits beside it on the SM (programmatic
 // dependent launch prefetches its weights while this one drains); larger tiles use 227 KB.
@@ -115,7 +154,7 @@ cudaError_t launch_init_kv_random(__nv_bfloat16* cache, int B, int H, int hd, in
 // x = embedding rows of the window's ids (fp32), xb = bf16(x), sq[d/128][N] = per-128-feature
 // sums of x^2, cur[N] = the ids (for the LM head's current-token probability).
 cudaError_t launch_embed(const int* tok, int tok_ld, const int* seq_kv, const __nv_bfloat16* emb, float* x,
-                         __nv_bfloat16* xb, float* sq, int* cur, int B, int T, int d, cudaStream_t st);
+                         __nv_bfloat16* xb, float* sq, int* cur, int* epoch, int B, int T, int d, cudaStream_t st);
 // The kernels below are launched with PDL when `pdl` (inside the context's step chain); the
 // single-kernel entry points pass false because their inputs may come from foreign kernels.
 // Attention plan: CTAs (split, head, sequence x query tile of 16*nw rows); the csize

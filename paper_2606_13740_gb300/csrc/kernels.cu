@@ -111,10 +111,11 @@ cudaError_t launch_init_kv_random(__nv_bfloat16* cache, int B, int H, int hd, in
 // cur[token] = the id (for the LM head's current-token probability).
 __global__ void __launch_bounds__(256) k_embed(const int* tok, int tok_ld, const int* seq_kv,
                                                const __nv_bfloat16* emb, float* x, __nv_bfloat16* xb, float* sq,
-                                               int* cur, int T, int N, int d) {
+                                               int* cur, int* epoch, int T, int N, int d) {
     pdl_wait();
     pdl_launch_dependents();
     const int j = blockIdx.x;
+    if (j == 0 && threadIdx.x == 0) *epoch += 1;  // one forward pass: a new tag for the chained projections
     const int b = j / T, t = j - b * T;
     const int id = tok[static_cast<size_t>(b) * tok_ld + seq_kv[b] + t];
     if (threadIdx.x == 0) cur[j] = id;
@@ -138,8 +139,9 @@ __global__ void __launch_bounds__(256) k_embed(const int* tok, int tok_ld, const
 }
 
 cudaError_t launch_embed(const int* tok, int tok_ld, const int* seq_kv, const __nv_bfloat16* emb, float* x,
-                         __nv_bfloat16* xb, float* sq, int* cur, int B, int T, int d, cudaStream_t st) {
-    return launch_k(k_embed, dim3(B * T), dim3(256), 0, st, true, tok, tok_ld, seq_kv, emb, x, xb, sq, cur, T, B * T, d);
+                         __nv_bfloat16* xb, float* sq, int* cur, int* epoch, int B, int T, int d, cudaStream_t st) {
+    return launch_k(k_embed, dim3(B * T), dim3(256), 0, st, true, tok, tok_ld, seq_kv, emb, x, xb, sq, cur, epoch, T,
+                    B * T, d);
 }
 
 // ------------------------------------------------------------------ attention

@@ -278,7 +278,7 @@ class Context:
         _check(lib().dllm_get_kv(self.h, layer, which, seq, p0, n, _p(out)), self.h)
         return out
 
-    KINDS = ("embed", "norm", "qkv", "attn", "oproj", "gateup", "down", "head", "head_reduce", "commit")
+    KINDS = ("embed", "norm", "qkv", "attn", "oproj", "gateup", "down", "head", "head_reduce", "commit", "layer")
 
     def dllm_set_profile(self, enable):
         _check(lib().dllm_set_profile(self.h, int(enable)), self.h)

@@ -169,7 +169,8 @@ def step_trace(a):
         r = {"k": names[i] if i < len(names) else str(i), "start_min": float(rel(0).min()),
              "start_max": float(rel(0).max()), "depwait_med": float(np.median(rel(7))),
              "first_data_med": float(np.median(rel(2))), "last_data_max": float(rel(3).max()),
-             "epi_done_max": float(rel(4).max()), "exit_max": float(rel(5).max())}
+             "epi_done_max": float(rel(4).max()),
+             "exit_max": float(rel(5).max()) if (v[:, 5] > 0).any() else float(rel(4).max())}
         if prev_exit is not None:
             r["gap_prev_exit_to_depwait"] = r["depwait_med"] - prev_exit
         prev_exit = r["exit_max"]
