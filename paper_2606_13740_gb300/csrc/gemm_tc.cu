@@ -1033,7 +1033,34 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
     // TMEM: two accumulators of acc_cols columns, then (32-token tiles) the staged residual
     const uint32_t t_x = tmem_base + static_cast<uint32_t>(2 * ca.acc_cols) + (static_cast<uint32_t>(quarter * 32) << 16);
     int rs_nt = -1;
+    long long prepared = -1;
     float v[32];
+    // Work a finisher needs before its accumulator: the RMSNorm scale of its token tile and
+    // (residual, 32-token tiles) the old x staged in TMEM.  Done as early as possible: for a
+    // contributor tile, ahead of it for the finisher tile that follows in the range.
+    auto prepare = [&](long long ptile) {
+        if (ptile == prepared) return;
+        prepared = ptile;
+        const int pmt = static_cast<int>(ptile / p.n_tiles);
+        const int pnt = static_cast<int>(ptile - static_cast<long long>(pmt) * p.n_tiles);
+        if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
+            if (ep.sq_in && pnt != rs_nt) {
+                compute_norm_scale(ep, p, pnt, esm, ew * 32 + lane);
+                rs_nt = pnt;
+            }
+        }
+        if constexpr (EPI == EPI_RESID) {
+            if (c32) {
+                const int row = pmt * kBM + rt;
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                    const int col = pnt * 32 + j;
+                    v[j] = (row < p.M && col < p.N) ? ep.out[static_cast<size_t>(col) * ep.ld_out + row] : 0.0f;
+                }
+                tmem_st_32x32(t_x, v);
+            }
+        }
+    };
     for (long long it = it0; it < it1;) {
         const long long tile = it / p.kb;
         const int k_lo = static_cast<int>(it - tile * p.kb);
@@ -1050,23 +1077,9 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             reducer = static_cast<int>(blockIdx.x) == c_first;
         }
         const bool finisher = whole || reducer;
-        if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
-            if (finisher && ep.sq_in && nt != rs_nt) {
-                compute_norm_scale(ep, p, nt, esm, ew * 32 + lane);
-                rs_nt = nt;
-            }
-        }
-        if constexpr (EPI == EPI_RESID) {
-            if (c32 && finisher) {  // stage the tile's old residual in TMEM while the accumulator is produced
-                const int row = mt * kBM + rt;
-#pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    const int col = nt * 32 + j;
-                    v[j] = (row < p.M && col < p.N) ? ep.out[static_cast<size_t>(col) * ep.ld_out + row] : 0.0f;
-                }
-                tmem_st_32x32(t_x, v);
-            }
-        }
+        // a contributor's range goes on into a tile whose first k-blocks it holds: a finisher
+        if (finisher) prepare(tile);
+        else if (tend < it1) prepare(tile + 1);
         mbar_wait(&tfull[es.acc], es.acc_phase, s_abort, status);
         if (named_bar_any(1, 128, *s_abort != 0)) return;
         if (tr && threadIdx.x == 64) {
