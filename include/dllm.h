@@ -173,8 +173,10 @@ int dllm_get_step_debug(dllm_ctx* ctx, float* logits, int32_t* argmax, float* co
 
 /* flags bit 0: materialise logits; bit 1: disable CUDA graphs; bit 2: launch
  * without programmatic dependent launch; bit 3: give the weight-streaming
- * projections 227 KB of shared memory (one CTA per SM) instead of 113 KB;
- * bit 4: record GEMM timelines (dllm_get_trace).  Bits 2 and 3 apply
+ * projections 227 KB of shared memory (one CTA per SM, the deepest weight
+ * ring) instead of leaving room beside them for the attention kernel's CTAs
+ * (146 KB for the chained projections, 113 KB for dllm_op_gemm_*); bit 4:
+ * record GEMM and attention timelines (dllm_get_trace).  Bits 2 and 3 apply
  * process-wide (for A/B measurements). */
 int dllm_set_debug(dllm_ctx* ctx, int flags);
 

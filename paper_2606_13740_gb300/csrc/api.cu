@@ -313,7 +313,7 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
         m.w[i] = w;
         m.x[i] = x;
     };
-    const int smem_budget = (ctx->debug & 8) ? kChainSmemShared : kChainSmemFull;
+    const int smem_budget = (ctx->debug & 8) ? kChainSmemFull : kChainSmemShared;
     auto run_chain = [&](ChainArgs& ca, const ChainMaps& m, int tag_add, int kind) -> int {
         ca.epoch = ctx->epoch;
         ca.tag_mul = c.n_layers + 2;
