@@ -1,4 +1,4 @@
-// Weight-streaming GEMM on the 5th-generation tensor cores (tcgen05 + TMEM).
+// Weight-streaming projections on the 5th-generation tensor cores (tcgen05 + TMEM).
 //
 // D[m][n] = sum_k W[m][k] * X[n][k]: W are the layer weights (bf16, K-major,
 // rows padded to 128), X the activations of the window's tokens (bf16,
@@ -7,34 +7,31 @@
 // covers the whole token set and the kernel is a pure stream of weight
 // bytes; at batch 16 (1024 tokens) the same kernel runs 128 x 256 tiles.
 //
-// Work is split "stream-K" style: the flattened (tile, 64-wide k-block)
-// iteration space is cut into one contiguous range per CTA (one CTA per SM),
-// so every SM streams the same number of weight bytes whatever the tile
-// count.  A tile cut between CTAs is finished by the CTA holding its first
-// k-blocks, which are the end of that CTA's range: the other contributors
-// store fp32 partials and publish them with one release increment each, and
-// the finishing CTA waits (bounded) for the count, bulk-copies the partials
-// into its drained pipeline memory and adds them to its own accumulator in k
-// order (deterministic).  Every CTA waits at most once, at its end, on CTAs
-// that wait on nothing, and the grid never exceeds the SM count, so all of
-// them are resident.
+// One kernel, k_chain, runs one or several projections ("phases") in one
+// persistent launch with one CTA per SM: a layer's output projection,
+// gate/up, down and the next layer's QKV stream their weights through one
+// shared-memory ring, the operand of each phase being loaded once the tiles
+// of the previous phase that write it have published completion flags.  A
+// single projection (dllm_op_gemm, the first layer's QKV) is a chain of one.
 //
-// Roles (192 threads): warp 0 = TMA producer, warp 1 = TMEM owner and MMA
-// issuer, warps 2..5 = epilogue (one TMEM lane quarter each).  Accumulators
-// are double-buffered in TMEM so the epilogue of one tile overlaps the MMAs
-// of the next.  Epilogues are fused: residual add with the next RMSNorm's
-// statistics, RoPE + KV-cache write, SwiGLU, and the LM head's per-tile
-// softmax statistics; the consumers of a residual apply RMSNorm as a
-// per-token scale of their fp32 accumulators.
+// Work in a phase is split "stream-K" style: the flattened (tile, 64-wide
+// k-block) iteration space is cut into one contiguous range per CTA, so
+// every SM streams the same number of weight bytes whatever the tile count.
+// A tile cut between CTAs is finished by the CTA holding its first k-blocks,
+// which are the end of that CTA's range: the other contributors store fp32
+// partials and publish them with one release increment each, and the
+// finishing CTA waits (bounded) for the count, bulk-copies the partials into
+// shared memory and adds them to its own accumulator in k order
+// (deterministic).  Every CTA waits only on CTAs that wait on nothing later
+// than it, and the grid never exceeds the SM count, so all are resident.
 //
-// Launched with programmatic dependent launch: the producer streams its first
-// pipeline stages of weights (which no earlier kernel writes) before
-// griddepcontrol.wait, so a projection's weight stream starts while the
-// previous kernel is still finishing.
-//
-// The epilogue runs once per tile on the step's critical path, so it avoids
-// dependent chains of global loads (everything it reads is loaded before it
-// stores, or staged in shared memory early) and keeps its code compact.
+// Epilogues are fused: residual add with the next RMSNorm's statistics,
+// RoPE + KV-cache write, SwiGLU, and the LM head's per-tile softmax
+// statistics; the consumers of a residual apply RMSNorm as a per-token scale
+// of their fp32 accumulators.  The epilogue runs once per tile on the step's
+// critical path, so it avoids dependent chains of global loads (everything
+// it reads is loaded before it stores, or staged early) and keeps its code
+// compact.
 #include "common.cuh"
 #include "internal.h"
 
@@ -44,12 +41,10 @@ namespace dllm {
 
 constexpr int kBM = 128;    // UMMA M
 constexpr int kBK = 64;     // K elements per stage: one 128-byte swizzle row
-constexpr int kThreads = 192;
 constexpr int kStageLd = 17;  // LM-head staging: 16 columns + pad
 constexpr uint32_t kABytes = kBM * kBK * 2;
-constexpr int kStreamSmem = 115712;  // two CTAs per SM (228 KB less 1 KB reserved each)
 constexpr int kFullSmem = 227 * 1024;
-static int g_stream_budget = kStreamSmem;
+static int g_stream_budget = kChainSmemShared;  // single projections: shared-memory plan
 constexpr int kTicketStride = 32;  // one tile ticket per 128-byte line
 
 // Timeline trace slots per CTA (when EpiArgs::trace is set).
@@ -547,403 +542,6 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
             }
         }
         named_bar(1, 128);
-    }
-}
-
-// ------------------------------------------------------------------ kernel
-template <int EPI>
-__global__ void __launch_bounds__(kThreads, 2)
-    k_gemm(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX, const GemmPlan p,
-           const EpiArgs ep, float* __restrict__ partials, int* __restrict__ counters, int* status) {
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    const int S = p.stages;
-    const uint32_t b_bytes = static_cast<uint32_t>(p.ntile) * kBK * 2;
-    uint8_t* sA = smem;
-    uint8_t* sB = sA + static_cast<size_t>(S) * kABytes;
-    float* tail = reinterpret_cast<float*>(sB + static_cast<size_t>(S) * b_bytes);
-    EpiSmem esm;
-    esm.rs = tail;
-    esm.red = tail + 256;
-    esm.kvs = reinterpret_cast<int*>(tail + 256 + 1024);
-    esm.theta = tail + 256 + 1024 + 256;
-    esm.stg = tail + 256 + 1024 + 256 + 128;
-    float* after = esm.stg + (EPI == EPI_LMHEAD ? kBM * kStageLd : 0);
-    uint64_t* full = reinterpret_cast<uint64_t*>(after);
-    uint64_t* empty = full + S;
-    uint64_t* tfull = empty + S;
-    uint64_t* tempty = tfull + 2;
-    uint64_t* drain = tempty + 2;
-    uint64_t* redbar = drain + 1;  // split-partial bulk loads of the last arriver
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(redbar + 1);
-    volatile int* s_abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
-
-    const int warp = threadIdx.x >> 5;
-    const int lane = threadIdx.x & 31;
-    const int G = p.grid;
-    const long long it0 = range_begin(blockIdx.x, p.total, G);
-    const long long it1 = range_begin(blockIdx.x + 1, p.total, G);
-
-    unsigned long long* tr = ep.trace ? ep.trace + static_cast<size_t>(blockIdx.x) * kTrSlots : nullptr;
-    if (tr && threadIdx.x == 0) {
-        tr[kTrStart] = global_ns();
-        tr[kTrSm] = smid();
-        for (int i = kTrAccReady; i < kTrSlots; ++i) tr[i] = 0;
-    }
-    if (threadIdx.x == 0) {
-        pdl_launch_dependents();
-        for (int s = 0; s < S; ++s) {
-            mbar_init(&full[s], 1);
-            mbar_init(&empty[s], 1);
-        }
-        for (int a = 0; a < 2; ++a) {
-            mbar_init(&tfull[a], 1);
-            mbar_init(&tempty[a], 128);
-        }
-        mbar_init(drain, 1);
-        mbar_init(redbar, 1);
-        *s_abort = 0;
-        mbar_fence_init();
-    }
-    if (warp == 0 && lane == 0) {
-        tma_prefetch_desc(&tmW);
-        tma_prefetch_desc(&tmX);
-    }
-    if (warp == 1) {
-        tmem_alloc(tmem_slot, p.tmem_cols);
-        tmem_relinquish();
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem_base = *tmem_slot;
-    if (tr && threadIdx.x == 0) tr[kTrPrologue] = global_ns();
-
-    if (warp == 0) {
-        // ---------------------------------------------------------- producer
-        if (lane == 0) {
-            const uint64_t pol_w = policy_evict_first();
-            const uint64_t pol_x = policy_evict_last();
-            int stage = 0;
-            uint32_t phase = 0;
-            uint32_t pending = 0;   // stages with a load in flight
-            uint32_t pend_par = 0;  // parity of that load's phase
-            // weights of the first stages: no earlier kernel writes them, so they stream
-            // before the dependency wait
-            const long long npre = (it1 - it0) < S ? (it1 - it0) : S;
-            for (long long q = 0; q < npre; ++q) {
-                const long long it = it0 + q;
-                const long long tile = it / p.kb;
-                const int k = static_cast<int>(it - tile * p.kb);
-                const int mt = static_cast<int>(tile / p.n_tiles);
-                mbar_arrive_expect_tx(&full[q], kABytes + b_bytes);
-                tma_load_2d(sA + static_cast<size_t>(q) * kABytes, &tmW, k * kBK, mt * kBM, &full[q], pol_w);
-            }
-            pdl_wait();
-            if (tr) tr[kTrDepWait] = global_ns();
-            for (long long q = 0; q < npre; ++q) {
-                const long long it = it0 + q;
-                const long long tile = it / p.kb;
-                const int k = static_cast<int>(it - tile * p.kb);
-                const int mt = static_cast<int>(tile / p.n_tiles);
-                const int nt = static_cast<int>(tile - static_cast<long long>(mt) * p.n_tiles);
-                tma_load_2d(sB + static_cast<size_t>(q) * b_bytes, &tmX, k * kBK, nt * p.ntile, &full[q], pol_x);
-                pending |= 1u << q;
-            }
-            stage = static_cast<int>(npre % S);
-            phase = npre == S ? 1u : 0u;
-            for (long long it = it0 + npre; it < it1; ++it) {
-                const long long tile = it / p.kb;
-                const int k = static_cast<int>(it - tile * p.kb);
-                const int mt = static_cast<int>(tile / p.n_tiles);
-                const int nt = static_cast<int>(tile - static_cast<long long>(mt) * p.n_tiles);
-                if (!mbar_wait(&empty[stage], phase ^ 1u, s_abort, status)) break;
-                mbar_arrive_expect_tx(&full[stage], kABytes + b_bytes);
-                tma_load_2d(sA + static_cast<size_t>(stage) * kABytes, &tmW, k * kBK, mt * kBM, &full[stage], pol_w);
-                tma_load_2d(sB + static_cast<size_t>(stage) * b_bytes, &tmX, k * kBK, nt * p.ntile, &full[stage],
-                            pol_x);
-                pending |= 1u << stage;
-                pend_par = (pend_par & ~(1u << stage)) | (phase << stage);
-                if (++stage == S) {
-                    stage = 0;
-                    phase ^= 1u;
-                }
-            }
-            if (*s_abort) {
-                // let every copy already issued land before the CTA's shared memory is released
-                for (int s = 0; s < S; ++s) {
-                    if (!(pending >> s & 1u)) continue;
-                    const unsigned long long t0 = global_ns();
-                    while (!mbar_try_wait(&full[s], (pend_par >> s) & 1u) && global_ns() - t0 < kWaitLimitNs) {
-                    }
-                }
-            }
-        }
-    } else if (warp == 1) {
-        // ---------------------------------------------------------- MMA issuer
-        if (lane == 0) {
-            pdl_wait();  // operands arrive only after the producer's own wait: block here, do not spin
-            const uint32_t idesc = umma_idesc_bf16(kBM, p.ntile);
-            int stage = 0;
-            uint32_t phase = 0;
-            int acc = 0;
-            uint32_t acc_phase = 0;
-            bool issued = false;
-            for (long long it = it0; it < it1 && !*s_abort;) {
-                const long long tile = it / p.kb;
-                const int k_lo = static_cast<int>(it - tile * p.kb);
-                const long long tend = (tile + 1) * p.kb;
-                const int k_hi = static_cast<int>((it1 < tend ? it1 : tend) - tile * p.kb);
-                if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, s_abort, status)) break;
-                tc_fence_after();
-                const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * p.acc_cols);
-                bool ok = true;
-                for (int k = k_lo; k < k_hi; ++k) {
-                    if (!mbar_wait(&full[stage], phase, s_abort, status)) {
-                        ok = false;
-                        break;
-                    }
-                    if (tr && !issued) tr[kTrFirstData] = global_ns();
-                    tc_fence_after();
-                    const uint64_t adesc = sw128_kmajor_desc(smem_u32(sA + static_cast<size_t>(stage) * kABytes));
-                    const uint64_t bdesc = sw128_kmajor_desc(smem_u32(sB + static_cast<size_t>(stage) * b_bytes));
-#pragma unroll
-                    for (int kk = 0; kk < kBK / 16; ++kk) {
-                        // +32 bytes per 16-element K step inside the 128-byte swizzle row
-                        umma_bf16(d_tmem, adesc + 2ull * kk, bdesc + 2ull * kk, idesc, (k > k_lo || kk > 0) ? 1u : 0u);
-                    }
-                    issued = true;
-                    umma_commit(&empty[stage]);
-                    if (++stage == S) {
-                        stage = 0;
-                        phase ^= 1u;
-                    }
-                }
-                if (!ok) break;
-                umma_commit(&tfull[acc]);
-                if (++acc == 2) {
-                    acc = 0;
-                    acc_phase ^= 1u;
-                }
-                it = tile * p.kb + k_hi;
-            }
-            if (tr) tr[kTrLastData] = global_ns();
-            if (*s_abort && issued) {
-                // wait for the tensor cores before the accumulator memory is released
-                umma_commit(drain);
-                const unsigned long long t0 = global_ns();
-                while (!mbar_try_wait(drain, 0) && global_ns() - t0 < kWaitLimitNs) {
-                }
-            }
-        }
-    } else {
-        // ---------------------------------------------------------- epilogue
-        pdl_wait();
-        const int ew = warp - 2;                 // 0..3
-        const int quarter = warp & 3;            // TMEM lane quarter this warp may access
-        const int rt = quarter * 32 + lane;      // row within the 128-row tile
-        if constexpr (EPI == EPI_QKV) {
-            for (int b = ew * 32 + lane; b < ep.n_seq; b += 128) esm.kvs[b] = ep.seq_kv[b];
-            // frequency of this tile row's rotation pair (rows interleave the pairs inside a head,
-            // and tiles start at head boundaries)
-            esm.theta[rt] = ep.theta[(rt % ep.hd) >> 1];
-            named_bar(1, 128);
-        }
-        if constexpr (EPI == EPI_LMHEAD) {
-            if (p.ntile == 32) {  // the window's current ids, for the compact epilogue
-                for (int c = ew * 32 + lane; c < p.N && c < 256; c += 128) esm.kvs[c] = ep.cur_tok[c];
-                named_bar(1, 128);
-            }
-        }
-        const int nchunks = p.ntile / 32;
-        const size_t slot_floats = static_cast<size_t>(p.ntile) * kBM;
-        const bool c32 = p.ntile == 32;  // batch-1 weight stream: compact TMEM-sourced epilogue
-        const uint32_t t_x = tmem_base + static_cast<uint32_t>(2 * p.acc_cols) + (static_cast<uint32_t>(quarter * 32) << 16);
-        int acc = 0;
-        uint32_t acc_phase = 0;
-        uint32_t red_phase = 0;
-        int rs_nt = -1;
-        float v[32];
-        for (long long it = it0; it < it1;) {
-            const long long tile = it / p.kb;
-            const int k_lo = static_cast<int>(it - tile * p.kb);
-            const long long tend = (tile + 1) * p.kb;
-            const int k_hi = static_cast<int>((it1 < tend ? it1 : tend) - tile * p.kb);
-            const int mt = static_cast<int>(tile / p.n_tiles);
-            const int nt = static_cast<int>(tile - static_cast<long long>(mt) * p.n_tiles);
-            const bool whole = (k_lo == 0 && k_hi == p.kb);
-            if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
-                // the operand's RMSNorm scale only needs the previous kernel: computed while the
-                // accumulator is still being produced
-                if (ep.sq_in && nt != rs_nt) {
-                    compute_norm_scale(ep, p, nt, esm, ew * 32 + lane);
-                    rs_nt = nt;
-                }
-            }
-            if constexpr (EPI == EPI_RESID) {
-                if (c32) {  // stage the tile's old residual in TMEM while the accumulator is produced
-                    const int row = mt * kBM + rt;
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        const int col = nt * 32 + j;
-                        v[j] = (row < p.M && col < p.N) ? ep.out[static_cast<size_t>(col) * ep.ld_out + row] : 0.0f;
-                    }
-                    tmem_st_32x32(t_x, v);
-                }
-            }
-            mbar_wait(&tfull[acc], acc_phase, s_abort, status);
-            if (named_bar_any(1, 128, *s_abort != 0)) break;
-            if (tr && threadIdx.x == 64) {
-                tr[kTrAccReady] = global_ns();
-                tr[kTrTile] = static_cast<unsigned long long>(tile);
-            }
-            tc_fence_after();
-            const uint32_t t_acc = tmem_base + static_cast<uint32_t>(acc * p.acc_cols) +
-                                   (static_cast<uint32_t>(quarter * 32) << 16);
-            // A tile cut between CTAs is finished by the CTA that holds its first k-blocks (for
-            // that CTA they are the end of its range); the others store fp32 partials for it.
-            int c_first = 0, c_last = 0;
-            bool reducer = false;
-            if (!whole) {
-                c_first = owner_of(tile * p.kb, p.total, G);
-                c_last = owner_of(tile * p.kb + p.kb - 1, p.total, G);
-                reducer = static_cast<int>(blockIdx.x) == c_first;
-            }
-            if (whole && c32) {
-                epilogue_c32<EPI>(ep, p, mt, nt, rt, t_acc, t_x, esm, ew, quarter, lane, status);
-            } else if (!reducer) {
-                // a contributor's partial is the first segment of its range: slot 0
-                float* my_part = partials + static_cast<size_t>(blockIdx.x) * 2 * slot_floats;
-                for (int c = 0; c < nchunks; ++c) {
-                    tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);
-                    if (whole) {
-                        epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
-                    } else {
-                        // float4 (c*8 + j, row): coalesced here, conflict-free when the reducer stages it
-                        float4* dst = reinterpret_cast<float4*>(my_part);
-#pragma unroll
-                        for (int j = 0; j < 8; ++j)
-                            dst[static_cast<size_t>(c * 8 + j) * kBM + rt] =
-                                make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
-                    }
-                }
-            }
-            if (!c32 && !reducer) {  // wide tiles release the accumulator as soon as it is read
-                tc_fence_before();
-                mbar_arrive(&tempty[acc]);
-            }
-            if (!whole && !reducer) {
-                // publish: the barrier orders the quarter-warps' stores before one release increment
-                named_bar(1, 128);
-                if (threadIdx.x == 64) {
-                    if (tr) tr[kTrPartStored] = global_ns();
-                    red_release_add(&counters[tile * kTicketStride], 1);
-                }
-            } else if (reducer) {
-                const int nparts = c_last - c_first + 1;
-                int* ticket = &counters[tile * kTicketStride];
-                if (threadIdx.x == 64) {
-                    if (tr) tr[kTrPartStored] = global_ns();
-                    const unsigned long long t0 = global_ns();
-                    while (ld_acquire(ticket) != nparts - 1) {
-                        if (*s_abort) break;
-                        if (global_ns() - t0 > kWaitLimitNs) {
-                            *s_abort = 1;
-                            atomicOr(status, kStatusTimeout);
-                            break;
-                        }
-                    }
-                    *ticket = 0;  // every contributor has arrived: ready for the next launch
-                    if (tr) {
-                        tr[kTrTicket] = global_ns();
-                        tr[kTrIsLast] = 1;
-                    }
-                }
-                if (named_bar_any(1, 128, *s_abort != 0)) break;
-                const uint32_t part_bytes = static_cast<uint32_t>(slot_floats * 4);
-                const uint32_t stage_room = static_cast<uint32_t>(S) * (kABytes + b_bytes);
-                const bool final_seg = tile * p.kb + k_hi == it1;  // pipeline drained: stage memory free
-                for (int c = 0; c < nchunks; ++c) {
-                    tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);  // own (first) k-range
-                    if (final_seg && c32 && part_bytes <= stage_room) {
-                        // one round trip: bulk-copy the contributors' partials into the stage memory
-                        const int per_batch = static_cast<int>(stage_room / part_bytes);
-                        for (int b0 = 1; b0 < nparts; b0 += per_batch) {
-                            const int nb = nparts - b0 < per_batch ? nparts - b0 : per_batch;
-                            if (threadIdx.x == 64) {
-                                fence_proxy_async_global();
-                                mbar_arrive_expect_tx(redbar, part_bytes * static_cast<uint32_t>(nb));
-                                for (int q = 0; q < nb; ++q)
-                                    bulk_load(smem + static_cast<size_t>(q) * part_bytes,
-                                              partials + static_cast<size_t>(c_first + b0 + q) * 2 * slot_floats,
-                                              part_bytes, redbar);
-                            }
-                            mbar_wait(redbar, red_phase, s_abort, status);
-                            red_phase ^= 1u;
-                            for (int q = 0; q < nb; ++q) {
-                                const float4* src =
-                                    reinterpret_cast<const float4*>(smem + static_cast<size_t>(q) * part_bytes);
-#pragma unroll
-                                for (int j = 0; j < 8; ++j) {
-                                    const float4 a = src[j * kBM + rt];
-                                    v[4 * j] += a.x;
-                                    v[4 * j + 1] += a.y;
-                                    v[4 * j + 2] += a.z;
-                                    v[4 * j + 3] += a.w;
-                                }
-                            }
-                            named_bar(1, 128);  // the next batch overwrites the staging memory
-                        }
-                    } else {
-                        // contributors in k order (each one's 8 loads in flight together)
-                        for (int cc = c_first + 1; cc <= c_last; ++cc) {
-                            const float4* p0 =
-                                reinterpret_cast<const float4*>(partials + static_cast<size_t>(cc) * 2 * slot_floats);
-                            float4 a[8];
-#pragma unroll
-                            for (int j = 0; j < 8; ++j) a[j] = __ldcg(p0 + static_cast<size_t>(c * 8 + j) * kBM + rt);
-#pragma unroll
-                            for (int j = 0; j < 8; ++j) {
-                                v[4 * j] += a[j].x;
-                                v[4 * j + 1] += a[j].y;
-                                v[4 * j + 2] += a[j].z;
-                                v[4 * j + 3] += a[j].w;
-                            }
-                        }
-                    }
-                    if (tr && threadIdx.x == 64 && c == 0) tr[kTrReduced] = global_ns();
-                    if (c32) {
-                        tmem_st_32x32(t_acc, v);  // the sum goes back into the (still owned) accumulator
-                        epilogue_c32<EPI>(ep, p, mt, nt, rt, t_acc, t_x, esm, ew, quarter, lane, status);
-                    } else {
-                        epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
-                    }
-                }
-                if (!c32) {
-                    tc_fence_before();
-                    mbar_arrive(&tempty[acc]);
-                }
-            }
-            if (c32) {
-                tc_fence_before();
-                mbar_arrive(&tempty[acc]);
-            }
-            if (++acc == 2) {
-                acc = 0;
-                acc_phase ^= 1u;
-            }
-            it = tile * p.kb + k_hi;
-        }
-        if (tr && threadIdx.x == 64) tr[kTrEpiDone] = global_ns();
-    }
-
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    if (tr && threadIdx.x == 0) tr[kTrExit] = global_ns();
-    if (warp == 1) {
-        __syncwarp();
-        tmem_dealloc(tmem_base, p.tmem_cols);
     }
 }
 
@@ -1507,18 +1105,6 @@ GemmPlan gemm_plan(int M, int N, int K, int grid_max, int epi) {
     p.total = static_cast<long long>(p.m_tiles) * p.n_tiles * p.kb;
     p.grid = static_cast<int>(p.total < grid_max ? p.total : grid_max);
     if (p.grid < 1) p.grid = 1;
-    p.acc_cols = pow2ceil(p.ntile);
-    // 32-token tiles also keep the residual's old values in 32 extra columns
-    p.tmem_cols = pow2ceil(2 * p.acc_cols + (p.ntile == 32 ? 32 : 0));
-    const int staging = epi == EPI_LMHEAD ? kBM * kStageLd * 4 : 0;
-    const int fixed = 1024 + (256 + 1024 + 256 + 128) * 4 + staging + 64 * 8 + 64;
-    const int stage_bytes = static_cast<int>(kABytes) + p.ntile * kBK * 2;
-    const int budget = p.ntile <= 96 ? g_stream_budget : kFullSmem;
-    int st = (budget - fixed) / stage_bytes;
-    if (st > 16) st = 16;
-    if (st < 2) st = 2;
-    p.stages = st;
-    p.smem = static_cast<size_t>(fixed) + static_cast<size_t>(st) * stage_bytes;
     p.pdl = true;
     return p;
 }
@@ -1554,42 +1140,32 @@ bool make_tmap_bf16(CUtensorMap* tm, const void* ptr, uint64_t rows, uint64_t co
     return r == CUDA_SUCCESS;
 }
 
-cudaError_t gemm_init_attrs() {
-    cudaError_t e = cudaSuccess;
-    auto set = [&](const void* f) {
-        if (e == cudaSuccess) e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, kFullSmem);
-    };
-    set(reinterpret_cast<const void*>(k_gemm<EPI_F32>));
-    set(reinterpret_cast<const void*>(k_gemm<EPI_RESID>));
-    set(reinterpret_cast<const void*>(k_gemm<EPI_QKV>));
-    set(reinterpret_cast<const void*>(k_gemm<EPI_SWIGLU>));
-    set(reinterpret_cast<const void*>(k_gemm<EPI_LMHEAD>));
-    return e;
-}
+cudaError_t gemm_init_attrs() { return chain_init_attrs(); }
 
-template <int EPI>
-static cudaError_t launch_t(const GemmPlan& p, const CUtensorMap& tmW, const CUtensorMap& tmX, const EpiArgs& ep,
-                            const Scratch& scr, int* status, cudaStream_t st) {
-    return launch_k(k_gemm<EPI>, dim3(p.grid), dim3(kThreads), p.smem, st, p.pdl, tmW, tmX, p, ep, scr.partials,
-                    scr.counters, status);
-}
-
+// One projection = a chain of one phase.
 cudaError_t gemm_launch(int epi, const GemmPlan& p, const CUtensorMap& tmW, const CUtensorMap& tmX,
                         const EpiArgs& ep, const Scratch& scr, int* status, cudaStream_t st) {
-    if (static_cast<size_t>(p.grid) * 2 * p.ntile * kBM > scr.partial_floats ||
+    if (static_cast<size_t>(p.grid) * p.ntile * kBM > scr.partial_floats ||
         static_cast<long long>(p.m_tiles) * p.n_tiles * kTicketStride > scr.counter_len)
         return cudaErrorInvalidValue;
-    switch (epi) {
-        case EPI_F32: return launch_t<EPI_F32>(p, tmW, tmX, ep, scr, status, st);
-        case EPI_RESID: return launch_t<EPI_RESID>(p, tmW, tmX, ep, scr, status, st);
-        case EPI_QKV: return launch_t<EPI_QKV>(p, tmW, tmX, ep, scr, status, st);
-        case EPI_SWIGLU: return launch_t<EPI_SWIGLU>(p, tmW, tmX, ep, scr, status, st);
-        case EPI_LMHEAD: return launch_t<EPI_LMHEAD>(p, tmW, tmX, ep, scr, status, st);
-    }
-    return cudaErrorInvalidValue;
+    ChainArgs ca{};
+    ca.n_phases = 1;
+    ca.status = status;
+    ca.tag_add = 1;
+    ChainPhase& P = ca.ph[0];
+    P.p = p;
+    P.ep = ep;
+    P.epi = epi;
+    P.partials = scr.partials;
+    P.tickets = scr.counters;
+    if (!chain_plan(ca, g_stream_budget)) return cudaErrorInvalidValue;
+    ChainMaps m;
+    m.w[0] = tmW;
+    m.x[0] = tmX;
+    return chain_launch(m, ca, st, p.pdl);
 }
 
-void set_stream_smem(bool coresident) { g_stream_budget = coresident ? kStreamSmem : kFullSmem; }
+void set_stream_smem(bool coresident) { g_stream_budget = coresident ? kChainSmemShared : kChainSmemFull; }
 
 static bool g_pdl = true;
 void set_pdl(bool on) { g_pdl = on; }

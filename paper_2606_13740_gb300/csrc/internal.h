@@ -61,10 +61,6 @@ struct GemmPlan {
     long long total;     // m_tiles * n_tiles * kb iterations of 64-wide K blocks
     int grid;            // CTAs (stream-K partition of the iterations)
     bool pdl;            // launch with programmatic dependent launch (the step's chain)
-    int stages;
-    int acc_cols;        // TMEM columns per accumulator buffer
-    int tmem_cols;       // allocation (power of two)
-    size_t smem;
 };
 
 struct Scratch {
@@ -113,9 +109,8 @@ constexpr int kChainSmemShared = 146 * 1024;  // leaves room for two attention C
 cudaError_t chain_launch(const ChainMaps& maps, const ChainArgs& ca, cudaStream_t st, bool pdl);
 cudaError_t chain_init_attrs();
 
-// Shared memory budget: at most 96 tokens per tile the kernel is a weight stream and keeps
-// to 113 KB so that the next projection's CTA fits beside it on the SM (programmatic
-// dependent launch prefetches its weights while this one drains); larger tiles use 227 KB.
+// Tiling of one projection: token tiles of at most 256 (multiples of 32), 128 weight rows
+// per tile, 64-wide k-blocks, grid = min(iterations, grid_max).
 GemmPlan gemm_plan(int M, int N, int K, int grid_max, int epi);
 bool make_tmap_bf16(CUtensorMap* tm, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows);
 cudaError_t gemm_launch(int epi, const GemmPlan& p, const CUtensorMap& tmW, const CUtensorMap& tmX,
@@ -126,7 +121,7 @@ cudaError_t gemm_launch(int epi, const GemmPlan& p, const CUtensorMap& tmW, cons
 // while its predecessor drains, and waits (griddepcontrol.wait) before touching data the
 // predecessor writes.  set_pdl(false) launches them plainly.
 void set_pdl(bool on);
-// GEMM shared-memory plan for <= 96 tokens: true = 113 KB (two CTAs per SM), false = 227 KB.
+// Single projections (dllm_op_gemm_*): true = the chain's 146 KB plan, false = 227 KB.
 void set_stream_smem(bool coresident);
 bool pdl_enabled();
 

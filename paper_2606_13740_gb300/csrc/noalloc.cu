@@ -65,8 +65,8 @@ extern "C" int dllm_op_gemm_noalloc(const void* W, const void* X, float* D, int 
         return noalloc_fail(DLLM_ECUDA, "device query failed");
     GemmPlan p = gemm_plan(M, N, K, (grid > 0 && grid < sms) ? grid : sms, EPI_F32);
     p.pdl = false;
-    // the split partials take [grid][2][ntile x 128] floats behind the tickets
-    const size_t per_cta = static_cast<size_t>(2) * p.ntile * 128 * sizeof(float);
+    // the split partials take [grid][ntile x 128] floats behind the tickets
+    const size_t per_cta = static_cast<size_t>(p.ntile) * 128 * sizeof(float);
     const size_t cap_ctas = (kNoAllocScratchBytes - kTicketBytes) / per_cta;
     if (static_cast<long long>(p.m_tiles) * p.n_tiles > kMaxTickets)
         return noalloc_fail(DLLM_ECAPACITY, "too many output tiles for the static scratch (M x N too large)");
