@@ -30,6 +30,7 @@ def main(argv=None):
     ap.add_argument("--reps", type=int, default=3)
     ap.add_argument("--dump", default="", help="gemm-trace: write every CTA's timeline to this JSON file")
     ap.add_argument("--no-pdl", action="store_true")
+    ap.add_argument("--debug", type=int, default=0, help="step-trace: extra dllm_set_debug flags")
     a = ap.parse_args(argv)
     lib()
     dev = torch.device("cuda:0")
@@ -137,7 +138,7 @@ def step_trace(a):
                  rope_base=500000.0)
     cfg = Config(max_batch=1, max_ctx=544, max_window=512, **shape)
     ctx = Context(cfg)
-    flags = 16 | (4 if a.no_pdl else 0)
+    flags = 16 | (4 if a.no_pdl else 0) | a.debug
     ctx.dllm_set_debug(flags)
     rng = np.random.default_rng(1)
     prompt = rng.integers(0, cfg.vocab - 1, 512).astype(np.int32)
