@@ -580,7 +580,7 @@ __device__ __forceinline__ bool wait_flag(const int* flag, int tag, volatile int
 }
 
 // The epilogue warps' share of one phase: every tile of this CTA's range.
-template <int EPI>
+template <int EPI, bool C32>
 __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph, int tag, uint8_t* red_stage,
                                                   uint64_t* tfull, uint64_t* tempty, uint64_t* redbar,
                                                   volatile int* s_abort, uint32_t tmem_base, const EpiSmem& esm,
@@ -627,7 +627,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
     }
     const int nchunks = p.ntile / 32;
     const size_t slot_floats = static_cast<size_t>(p.ntile) * kBM;
-    const bool c32 = p.ntile == 32;
+    constexpr bool c32 = C32;  // the launch's token tile is 32 (compact epilogue, bulk-copy reduction)
     // TMEM: two accumulators of acc_cols columns, then (32-token tiles) the staged residual
     const uint32_t t_x = tmem_base + static_cast<uint32_t>(2 * ca.acc_cols) + (static_cast<uint32_t>(quarter * 32) << 16);
     int rs_nt = -1;
@@ -648,7 +648,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             }
         }
         if constexpr (EPI == EPI_RESID) {
-            if (c32) {
+            if constexpr (c32) {
                 const int row = pmt * kBM + rt;
 #pragma unroll
                 for (int j = 0; j < 32; ++j) {
@@ -687,14 +687,14 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         tc_fence_after();
         const uint32_t t_acc = tmem_base + static_cast<uint32_t>(es.acc * ca.acc_cols) +
                                (static_cast<uint32_t>(quarter * 32) << 16);
-        if (whole && c32) {
-            epilogue_c32<EPI>(ep, p, mt, nt, rt, t_acc, t_x, esm, ew, quarter, lane, status);
+        if (c32 && whole) {
+            if constexpr (c32) epilogue_c32<EPI>(ep, p, mt, nt, rt, t_acc, t_x, esm, ew, quarter, lane, status);
         } else if (!reducer) {
             float* my_part = P.partials + static_cast<size_t>(blockIdx.x) * slot_floats;
             for (int c = 0; c < nchunks; ++c) {
                 tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);
                 if (whole) {
-                    epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
+                    if constexpr (!c32) epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
                 } else {
                     float4* dst = reinterpret_cast<float4*>(my_part);
 #pragma unroll
@@ -730,7 +730,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             const uint32_t part_bytes = static_cast<uint32_t>(slot_floats * 4);
             for (int c = 0; c < nchunks; ++c) {
                 tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);  // own (first) k-range
-                if (c32 && ca.red_bytes >= static_cast<int>(part_bytes)) {
+                if (c32) {
                     const int per_batch = ca.red_bytes / static_cast<int>(part_bytes);
                     for (int b0 = 1; b0 < nparts; b0 += per_batch) {
                         const int nb = nparts - b0 < per_batch ? nparts - b0 : per_batch;
@@ -775,7 +775,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                     }
                 }
                 if (tr && threadIdx.x == 64 && c == 0) tr[kTrReduced] = global_ns();
-                if (c32) {
+                if constexpr (c32) {
                     tmem_st_32x32(t_acc, v);
                     epilogue_c32<EPI>(ep, p, mt, nt, rt, t_acc, t_x, esm, ew, quarter, lane, status);
                 } else {
@@ -804,6 +804,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
     if (tr && threadIdx.x == 64) tr[kTrEpiDone] = global_ns();
 }
 
+template <bool C32>
 __global__ void __launch_bounds__(kChainThreads, 1)
     k_chain(const __grid_constant__ ChainMaps maps, const __grid_constant__ ChainArgs ca) {
     extern __shared__ uint8_t smem_raw[];
@@ -1058,19 +1059,19 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         for (int ph = 0; ph < ca.n_phases; ++ph) {  // on abort every phase returns at its first barrier
             switch (ca.ph[ph].epi) {
                 case EPI_F32:
-                    chain_phase_epilogue<EPI_F32>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    chain_phase_epilogue<EPI_F32, C32>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
                     break;
                 case EPI_RESID:
-                    chain_phase_epilogue<EPI_RESID>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    chain_phase_epilogue<EPI_RESID, C32>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
                     break;
                 case EPI_QKV:
-                    chain_phase_epilogue<EPI_QKV>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    chain_phase_epilogue<EPI_QKV, C32>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
                     break;
                 case EPI_SWIGLU:
-                    chain_phase_epilogue<EPI_SWIGLU>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    chain_phase_epilogue<EPI_SWIGLU, C32>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
                     break;
                 default:
-                    chain_phase_epilogue<EPI_LMHEAD>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    chain_phase_epilogue<EPI_LMHEAD, C32>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
                     break;
             }
         }
@@ -1201,8 +1202,12 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
 }
 
 cudaError_t chain_init_attrs() {
-    return cudaFuncSetAttribute(reinterpret_cast<const void*>(k_chain), cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                kFullSmem);
+    cudaError_t e = cudaFuncSetAttribute(reinterpret_cast<const void*>(k_chain<true>),
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kFullSmem);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(reinterpret_cast<const void*>(k_chain<false>),
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, kFullSmem);
+    return e;
 }
 
 cudaError_t chain_launch(const ChainMaps& maps, const ChainArgs& ca, cudaStream_t st, bool pdl) {
@@ -1211,7 +1216,10 @@ cudaError_t chain_launch(const ChainMaps& maps, const ChainArgs& ca, cudaStream_
         if (p.grid > ca.grid || !ca.ph[i].partials || !ca.ph[i].tickets || (i > 0 && ca.ph[i].dep_rows < 0))
             return cudaErrorInvalidValue;
     }
-    return launch_k(k_chain, dim3(ca.grid), dim3(kChainThreads), ca.smem, st, pdl, maps, ca);
+    // 32-token chains (the batch-1 weight stream) and wider token tiles are separate kernels, so
+    // each carries only its own epilogue code
+    if (ca.ntile == 32) return launch_k(k_chain<true>, dim3(ca.grid), dim3(kChainThreads), ca.smem, st, pdl, maps, ca);
+    return launch_k(k_chain<false>, dim3(ca.grid), dim3(kChainThreads), ca.smem, st, pdl, maps, ca);
 }
 
 }  // namespace dllm
