@@ -41,7 +41,6 @@ namespace dllm {
 
 constexpr int kBM = 128;    // UMMA M
 constexpr int kBK = 64;     // K elements per stage: one 128-byte swizzle row
-constexpr int kStageLd = 17;  // LM-head staging: 16 columns + pad
 constexpr uint32_t kABytes = kBM * kBK * 2;
 constexpr int kFullSmem = 227 * 1024;
 static int g_stream_budget = kChainSmemShared;  // single projections: shared-memory plan
@@ -64,26 +63,11 @@ __device__ __forceinline__ int owner_of(long long i, long long total, int G) {
 
 __device__ __forceinline__ long long range_begin(int c, long long total, int G) { return total * c / G; }
 
-// Sum of v[0..31] over the 32 lanes of a warp, scattered: afterwards lane l
-// holds the total of column l in v[0].  31 shuffles in a fixed order.
-__device__ __forceinline__ void warp_reduce_scatter32(float* v, int lane) {
-#pragma unroll
-    for (int w = 16; w >= 1; w >>= 1) {
-        const bool upper = (lane & w) != 0;
-#pragma unroll
-        for (int i = 0; i < w; ++i) {
-            float send = upper ? v[i] : v[i + w];
-            float keep = upper ? v[i + w] : v[i];
-            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, w);
-        }
-    }
-}
 
 struct EpiSmem {
-    float* stg;   // LM head staging [128][kStageLd]
     float* rs;    // [256] per-column RMSNorm scale of the current token tile
     float* red;   // [4][256] cross-warp / quarter partial sums
-    int* kvs;     // [256] per-sequence first window position (QKV)
+    int* kvs;     // [256] per-sequence first window position (QKV); current ids of the token tile (LM head)
     float* theta; // [128] rotation frequency of each tile row's feature pair (QKV)
 };
 
@@ -125,193 +109,6 @@ __device__ __noinline__ float2 rot_cs(float angle) {
 }
 
 // ------------------------------------------------------------------ epilogues
-template <int EPI>
-__device__ __forceinline__ void epilogue_chunk(const EpiArgs& ep, const GemmPlan& p, int mt, int nt, int chunk,
-                                               int rt, float* v, const EpiSmem& sm, int ew, int quarter, int lane,
-                                               int* status) {
-    const int row = mt * kBM + rt;
-    const int col0 = nt * p.ntile + chunk * 32;
-    if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
-        if (ep.sq_in) {  // RMSNorm of the operand rows, as a per-token scale (computed per token tile)
-#pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] *= sm.rs[chunk * 32 + j];
-        }
-    }
-    if constexpr (EPI == EPI_F32) {
-        if (row < p.M) {
-#pragma unroll
-            for (int j = 0; j < 32; ++j) {
-                const int col = col0 + j;
-                if (col < p.N) ep.out[static_cast<size_t>(col) * ep.ld_out + row] = v[j];
-            }
-        }
-    } else if constexpr (EPI == EPI_RESID) {
-        const bool rv = row < p.M;
-#pragma unroll
-        for (int h0 = 0; h0 < 32; h0 += 16) {
-            float xo[16];
-#pragma unroll
-            for (int j = 0; j < 16; ++j) {  // the residual loads issued before any store
-                const int col = col0 + h0 + j;
-                xo[j] = (rv && col < p.N) ? ep.out[static_cast<size_t>(col) * ep.ld_out + row] : 0.0f;
-            }
-#pragma unroll
-            for (int j = 0; j < 16; ++j) {
-                const int col = col0 + h0 + j;
-                float x = 0.0f;
-                if (rv && col < p.N) {
-                    const size_t o = static_cast<size_t>(col) * ep.ld_out + row;
-                    x = xo[j] + v[h0 + j];
-                    ep.out[o] = x;
-                    ep.xb[o] = __float2bfloat16_rn(x);
-                }
-                v[h0 + j] = x * x;
-            }
-        }
-        warp_reduce_scatter32(v, lane);
-        sm.red[quarter * 32 + lane] = v[0];
-        named_bar(1, 128);
-        if (ew == 0) {
-            const int col = col0 + lane;
-            if (col < p.N)
-                ep.sq_out[static_cast<size_t>(mt) * p.N + col] =
-                    ((sm.red[lane] + sm.red[32 + lane]) + sm.red[64 + lane]) + sm.red[96 + lane];
-        }
-        named_bar(1, 128);
-    } else if constexpr (EPI == EPI_QKV) {
-        const int qd = ep.H * ep.hd;
-        const int part = row / qd;
-        const int f = row - part * qd;
-        const int hh = f / ep.hd;
-        const int pp = f - hh * ep.hd;          // physical row inside the head
-        const int half = ep.hd >> 1;
-        const int i = (pp >> 1) + (pp & 1) * half;  // logical feature
-        const float theta = sm.theta[rt];
-        // The chunk's 32 columns are consecutive positions of one sequence when the window
-        // length is a multiple of 32: rotate by the angle-addition recurrence (two sincosf
-        // per chunk; the table of cos/sin would be DRAM-cold behind the weight stream).
-        const int bl = col0 / ep.T;
-        const int last = min(col0 + 31, p.N - 1);
-        const bool run = last / ep.T == bl;  // uniform across the CTA
-        float cn = 1.0f, sn = 0.0f, cd = 1.0f, sd = 0.0f;
-        if (part < 2 && run) {
-            const float2 a = rot_cs(static_cast<float>(sm.kvs[bl] + (col0 - bl * ep.T)) * theta);
-            const float2 d = rot_cs(theta);
-            cn = a.x;
-            sn = a.y;
-            cd = d.x;
-            sd = d.y;
-        }
-#pragma unroll
-        for (int j = 0; j < 32; ++j) {
-            const float xp = __shfl_xor_sync(0xffffffffu, v[j], 1);
-            const int col = col0 + j;
-            if (col < p.N) {
-                const int b = run ? bl : col / ep.T;
-                const int t = col - b * ep.T;
-                const int pos = sm.kvs[b] + t;
-                if (pos < 0 || pos >= ep.cap) {
-                    atomicOr(status, kStatusBadIndex);
-                } else {
-                    float x = v[j];
-                    if (part < 2) {
-                        if (!run) {
-                            const float2 a = rot_cs(static_cast<float>(pos) * theta);
-                            cn = a.x;
-                            sn = a.y;
-                        }
-                        x = (pp & 1) ? (x * cn + xp * sn) : (x * cn - xp * sn);
-                    }
-                    const __nv_bfloat16 y = __float2bfloat16_rn(x);
-                    if (part == 0) {
-                        ep.q[((static_cast<size_t>(b) * ep.H + hh) * ep.T + t) * ep.hd + i] = y;
-                    } else {
-                        __nv_bfloat16* c = part == 1 ? ep.kc : ep.vc;
-                        c[((static_cast<size_t>(b) * ep.H + hh) * ep.cap + pos) * ep.hd + i] = y;
-                    }
-                }
-            }
-            if (run) {  // advance the rotation by one position
-                const float c2 = cn * cd - sn * sd;
-                sn = sn * cd + cn * sd;
-                cn = c2;
-            }
-        }
-    } else if constexpr (EPI == EPI_SWIGLU) {
-        const int f = mt * 64 + (rt >> 1);
-        const bool gate = (rt & 1) == 0;
-#pragma unroll
-        for (int j = 0; j < 32; ++j) {
-            const float u = __shfl_xor_sync(0xffffffffu, v[j], 1);
-            const int col = col0 + j;
-            if (gate && f < ep.F && col < p.N) {
-                const float g = v[j];
-                const float s = g / (1.0f + __expf(-g));
-                ep.h[static_cast<size_t>(col) * ep.F + f] = __float2bfloat16_rn(s * u);
-            }
-        }
-    } else if constexpr (EPI == EPI_LMHEAD) {
-        if (ep.logits && row < ep.V) {
-            for (int j = 0; j < 32; ++j) {
-                const int col = col0 + j;
-                if (col < p.N) ep.logits[static_cast<size_t>(col) * ep.V + row] = v[j];
-            }
-        }
-#pragma unroll
-        for (int hlf = 0; hlf < 2; ++hlf) {
-#pragma unroll
-            for (int j = 0; j < 16; ++j) sm.stg[rt * kStageLd + j] = v[hlf * 16 + j];
-            named_bar(1, 128);
-            for (int jj = ew; jj < 16; jj += 4) {
-                const int col = col0 + hlf * 16 + jj;
-                if (col >= p.N) break;
-                float m = -INFINITY;
-                int idx = INT_MAX;
-                float z[4];
-                bool ok[4];
-#pragma unroll
-                for (int r = 0; r < 4; ++r) {
-                    const int rr = lane + 32 * r;
-                    const int id = mt * kBM + rr;
-                    ok[r] = id < ep.V && id != ep.mask_id;
-                    z[r] = sm.stg[rr * kStageLd + jj];
-                    if (ok[r] && z[r] > m) {
-                        m = z[r];
-                        idx = id;
-                    }
-                }
-#pragma unroll
-                for (int off = 16; off > 0; off >>= 1) {
-                    const float om = __shfl_xor_sync(0xffffffffu, m, off);
-                    const int oi = __shfl_xor_sync(0xffffffffu, idx, off);
-                    if (om > m || (om == m && oi < idx)) {
-                        m = om;
-                        idx = oi;
-                    }
-                }
-                float s = 0.0f;
-                if (m != -INFINITY) {
-#pragma unroll
-                    for (int r = 0; r < 4; ++r)
-                        if (ok[r]) s += expf(z[r] - m);
-                }
-#pragma unroll
-                for (int off = 16; off > 0; off >>= 1) s += __shfl_down_sync(0xffffffffu, s, off);
-                if (lane == 0) {
-                    float* o = ep.lm_part + (static_cast<size_t>(col) * p.m_tiles + mt) * 3;
-                    o[0] = m;
-                    o[1] = s;
-                    o[2] = __int_as_float(idx);
-                    const int cur = ep.cur_tok[col];
-                    if (cur >= mt * kBM && cur < mt * kBM + kBM)
-                        ep.zcur[col] = sm.stg[(cur - mt * kBM) * kStageLd + jj];
-                }
-            }
-            named_bar(1, 128);
-        }
-    }
-}
-
 // Sum of v[0..7] over the 32 lanes of a warp, scattered: afterwards the four lanes
 // 4c..4c+3 hold the total of column c in v[0].  9 shuffles in a fixed order.
 __device__ __forceinline__ void warp_reduce_scatter8(float* v, int lane) {
@@ -336,12 +133,13 @@ __device__ __forceinline__ void warp_reduce_scatter8(float* v, int lane) {
 // branch between them (stores are predicated), so their dependent chains (shuffles, special
 // functions) overlap.
 template <int EPI>
-__device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& p, int mt, int nt, int rt,
-                                             uint32_t t_src, uint32_t t_x, const EpiSmem& sm, int ew, int quarter,
-                                             int lane, int* status) {
+__device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& p, int mt, int col0, int c_in,
+                                             int rt, uint32_t t_src, uint32_t t_x, const EpiSmem& sm, int ew,
+                                             int quarter, int lane, int* status) {
+    // col0: the chunk's first token column; c_in: its offset inside the token tile (index into
+    // the tile's RMSNorm scales and staged ids); t_x == 0: the old residual is read from global
     constexpr int GW = 8;  // columns per group
     const int row = mt * kBM + rt;
-    const int col0 = nt * 32;
     const bool scale = (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) && ep.sq_in != nullptr;
     // QKV state: feature, head, rotation (angle-addition recurrence along the positions)
     int part = 0, hh = 0, pp = 0, fi = 0, bl = 0;
@@ -379,7 +177,7 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
         tmem_ld_32x8(t_src + static_cast<uint32_t>(GW * g), a);
         if (scale) {
 #pragma unroll
-            for (int u = 0; u < GW; ++u) a[u] *= sm.rs[GW * g + u];
+            for (int u = 0; u < GW; ++u) a[u] *= sm.rs[c_in + GW * g + u];
         }
         if constexpr (EPI == EPI_F32) {
 #pragma unroll
@@ -387,7 +185,13 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                 if (row < p.M && cg + u < p.N) ep.out[static_cast<size_t>(cg + u) * ep.ld_out + row] = a[u];
         } else if constexpr (EPI == EPI_RESID) {
             float xo[GW], ss[GW];
-            tmem_ld_32x8(t_x + static_cast<uint32_t>(GW * g), xo);
+            if (t_x) {
+                tmem_ld_32x8(t_x + static_cast<uint32_t>(GW * g), xo);
+            } else {
+#pragma unroll
+                for (int u = 0; u < GW; ++u)
+                    xo[u] = (row < p.M && cg + u < p.N) ? ep.out[static_cast<size_t>(cg + u) * ep.ld_out + row] : 0.0f;
+            }
 #pragma unroll
             for (int u = 0; u < GW; ++u) {
                 const bool ok = row < p.M && cg + u < p.N;
@@ -493,7 +297,7 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
             for (int u = 0; u < GW; ++u) {
                 const int col = cg + u;
                 if (ep.logits && row < ep.V && col < p.N) ep.logits[static_cast<size_t>(col) * ep.V + row] = a[u];
-                if (col < p.N && row == sm.kvs[col]) ep.zcur[col] = a[u];  // current ids staged in kvs
+                if (col < p.N && row == sm.kvs[c_in + GW * g + u]) ep.zcur[col] = a[u];  // current ids staged
             }
         }
     }
@@ -619,23 +423,19 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         esm.theta[rt] = ep.theta[(rt % ep.hd) >> 1];
         named_bar(1, 128);
     }
-    if constexpr (EPI == EPI_LMHEAD) {
-        if (p.ntile == 32) {
-            for (int c = ew * 32 + lane; c < p.N && c < 256; c += 128) esm.kvs[c] = ep.cur_tok[c];
-            named_bar(1, 128);
-        }
-    }
     const int nchunks = p.ntile / 32;
     const size_t slot_floats = static_cast<size_t>(p.ntile) * kBM;
-    constexpr bool c32 = C32;  // the launch's token tile is 32 (compact epilogue, bulk-copy reduction)
+    constexpr bool c32 = C32;  // the launch's token tile is 32 (residual staged in TMEM, bulk-copy reduction)
     // TMEM: two accumulators of acc_cols columns, then (32-token tiles) the staged residual
-    const uint32_t t_x = tmem_base + static_cast<uint32_t>(2 * ca.acc_cols) + (static_cast<uint32_t>(quarter * 32) << 16);
-    int rs_nt = -1;
+    const uint32_t t_x =
+        c32 ? tmem_base + static_cast<uint32_t>(2 * ca.acc_cols) + (static_cast<uint32_t>(quarter * 32) << 16) : 0u;
+    int rs_nt = -1, ids_nt = -1;
     long long prepared = -1;
     float v[32];
-    // Work a finisher needs before its accumulator: the RMSNorm scale of its token tile and
-    // (residual, 32-token tiles) the old x staged in TMEM.  Done as early as possible: for a
-    // contributor tile, ahead of it for the finisher tile that follows in the range.
+    // Work a finisher needs before its accumulator: the RMSNorm scale of its token tile, the
+    // LM head's current ids of the token tile, and (residual, 32-token tiles) the old x staged
+    // in TMEM.  Done as early as possible: for a contributor tile, ahead of it for the finisher
+    // tile that follows in the range.
     auto prepare = [&](long long ptile) {
         if (ptile == prepared) return;
         prepared = ptile;
@@ -647,16 +447,24 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                 rs_nt = pnt;
             }
         }
-        if constexpr (EPI == EPI_RESID) {
-            if constexpr (c32) {
-                const int row = pmt * kBM + rt;
-#pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    const int col = pnt * 32 + j;
-                    v[j] = (row < p.M && col < p.N) ? ep.out[static_cast<size_t>(col) * ep.ld_out + row] : 0.0f;
+        if constexpr (EPI == EPI_LMHEAD) {
+            if (pnt != ids_nt) {
+                for (int c = ew * 32 + lane; c < p.ntile; c += 128) {
+                    const int col = pnt * p.ntile + c;
+                    esm.kvs[c] = col < p.N ? ep.cur_tok[col] : -1;
                 }
-                tmem_st_32x32(t_x, v);
+                named_bar(1, 128);
+                ids_nt = pnt;
             }
+        }
+        if constexpr (EPI == EPI_RESID && c32) {
+            const int row = pmt * kBM + rt;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                const int col = pnt * 32 + j;
+                v[j] = (row < p.M && col < p.N) ? ep.out[static_cast<size_t>(col) * ep.ld_out + row] : 0.0f;
+            }
+            tmem_st_32x32(t_x, v);
         }
     };
     for (long long it = it0; it < it1;) {
@@ -687,34 +495,31 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         tc_fence_after();
         const uint32_t t_acc = tmem_base + static_cast<uint32_t>(es.acc * ca.acc_cols) +
                                (static_cast<uint32_t>(quarter * 32) << 16);
-        if (c32 && whole) {
-            if constexpr (c32) epilogue_c32<EPI>(ep, p, mt, nt, rt, t_acc, t_x, esm, ew, quarter, lane, status);
+        if (whole) {
+            // the compact epilogue per 32-column chunk, straight from the accumulator in TMEM
+            for (int c = 0; c < nchunks; ++c)
+                epilogue_c32<EPI>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt, t_acc + static_cast<uint32_t>(c * 32),
+                                  t_x, esm, ew, quarter, lane, status);
         } else if (!reducer) {
             float* my_part = P.partials + static_cast<size_t>(blockIdx.x) * slot_floats;
             for (int c = 0; c < nchunks; ++c) {
                 tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);
-                if (whole) {
-                    if constexpr (!c32) epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
-                } else {
-                    float4* dst = reinterpret_cast<float4*>(my_part);
+                float4* dst = reinterpret_cast<float4*>(my_part);
 #pragma unroll
-                    for (int j = 0; j < 8; ++j)
-                        dst[static_cast<size_t>(c * 8 + j) * kBM + rt] =
-                            make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
-                }
+                for (int j = 0; j < 8; ++j)
+                    dst[static_cast<size_t>(c * 8 + j) * kBM + rt] =
+                        make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
             }
-        }
-        if (!c32 && !reducer) {
+            // the partial is in registers' way out: the accumulator is free again
             tc_fence_before();
             mbar_arrive(&tempty[es.acc]);
-        }
-        if (!whole && !reducer) {
             named_bar(1, 128);
             if (threadIdx.x == 64) {
                 if (tr) tr[kTrPartStored] = global_ns();
                 red_release_add(&P.tickets[tile * kTicketStride], 1);
             }
-        } else if (reducer) {
+        }
+        if (reducer) {
             const int nparts = c_last - c_first + 1;
             int* ticket = &P.tickets[tile * kTicketStride];
             if (threadIdx.x == 64) {
@@ -730,7 +535,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             const uint32_t part_bytes = static_cast<uint32_t>(slot_floats * 4);
             for (int c = 0; c < nchunks; ++c) {
                 tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);  // own (first) k-range
-                if (c32) {
+                if constexpr (c32) {
                     const int per_batch = ca.red_bytes / static_cast<int>(part_bytes);
                     for (int b0 = 1; b0 < nparts; b0 += per_batch) {
                         const int nb = nparts - b0 < per_batch ? nparts - b0 : per_batch;
@@ -775,19 +580,13 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                     }
                 }
                 if (tr && threadIdx.x == 64 && c == 0) tr[kTrReduced] = global_ns();
-                if constexpr (c32) {
-                    tmem_st_32x32(t_acc, v);
-                    epilogue_c32<EPI>(ep, p, mt, nt, rt, t_acc, t_x, esm, ew, quarter, lane, status);
-                } else {
-                    epilogue_chunk<EPI>(ep, p, mt, nt, c, rt, v, esm, ew, quarter, lane, status);
-                }
-            }
-            if (!c32) {
-                tc_fence_before();
-                mbar_arrive(&tempty[es.acc]);
+                // the sum goes back into the (still owned) accumulator, then the compact epilogue
+                tmem_st_32x32(t_acc + static_cast<uint32_t>(c * 32), v);
+                epilogue_c32<EPI>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt, t_acc + static_cast<uint32_t>(c * 32),
+                                  t_x, esm, ew, quarter, lane, status);
             }
         }
-        if (c32) {
+        if (finisher) {
             tc_fence_before();
             mbar_arrive(&tempty[es.acc]);
         }
@@ -820,8 +619,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     esm.red = tail + 256;
     esm.kvs = reinterpret_cast<int*>(tail + 256 + 1024);
     esm.theta = tail + 256 + 1024 + 256;
-    esm.stg = tail + 256 + 1024 + 256 + 128;
-    float* after = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(esm.stg) + ca.stg_bytes);
+    float* after = tail + 256 + 1024 + 256 + 128;
     uint64_t* full = reinterpret_cast<uint64_t*>(after);
     uint64_t* empty = full + S;
     uint64_t* tfull = empty + S;
@@ -1177,21 +975,21 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
     if (ca.n_phases < 1 || ca.n_phases > kMaxPhases) return false;
     const int ntile = ca.ph[0].p.ntile;
     int grid = 0;
-    bool lm_wide = false;
     for (int i = 0; i < ca.n_phases; ++i) {
         const GemmPlan& p = ca.ph[i].p;
         if (p.ntile != ntile || p.N != ca.ph[0].p.N) return false;
         grid = grid > p.grid ? grid : p.grid;
-        if (ca.ph[i].epi == EPI_LMHEAD && ntile != 32) lm_wide = true;
     }
     const bool c32 = ntile == 32;
+    // wider token tiles are tensor-bound: the deepest ring (the attention CTAs' room matters
+    // only to the batch-1 weight stream)
+    if (!c32) smem_budget = kFullSmem;
     ca.grid = grid;
     ca.ntile = ntile;
     ca.acc_cols = c32 ? 32 : pow2ceil(ntile);
     ca.tmem_cols = pow2ceil(2 * ca.acc_cols + (c32 ? 32 : 0));
     ca.red_bytes = c32 ? 2 * 32 * kBM * 4 : 0;  // two split partials per bulk-copy round
-    ca.stg_bytes = lm_wide ? kBM * kStageLd * 4 : 0;
-    const int fixed = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.stg_bytes + ca.red_bytes + 6 * 8 + 16;
+    const int fixed = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + 6 * 8 + 16;
     const int stage_bytes = static_cast<int>(kABytes) + ntile * kBK * 2;
     int st = (smem_budget - fixed) / (stage_bytes + 16);
     if (st > 32) st = 32;

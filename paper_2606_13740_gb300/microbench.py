@@ -19,7 +19,9 @@ from .dllm import dllm_op_attention, dllm_op_gemm, dllm_op_gemm_timed, dllm_op_g
 
 def main(argv=None):
     ap = argparse.ArgumentParser()
-    ap.add_argument("op", choices=("gemm", "attention", "gemm-sweep", "gemm-trace", "step-trace", "step-small"))
+    ap.add_argument("op", choices=("gemm", "attention", "gemm-sweep", "gemm-trace", "step-trace", "step-small",
+                                   "step-b16", "window-sweep", "generate"))
+    ap.add_argument("--layers", type=int, default=32)
     ap.add_argument("--M", type=int, default=24576)
     ap.add_argument("--N", type=int, default=32)
     ap.add_argument("--K", type=int, default=4096)
@@ -57,6 +59,15 @@ def main(argv=None):
         return
     if a.op == "step-small":
         step_small(a)
+        return
+    if a.op == "step-b16":
+        step_b16(a)
+        return
+    if a.op == "window-sweep":
+        window_sweep(a)
+        return
+    if a.op == "generate":
+        generate(a)
         return
     if a.op == "step-trace":
         step_trace(a)
@@ -105,6 +116,135 @@ def main(argv=None):
         torch.cuda.synchronize()
         times.append(time.perf_counter() - t0)
     print(json.dumps({"op": a.op, "wall_ms_per_call": [t * 1e3 for t in times], "bytes": nbytes}))
+
+
+
+SHAPE_8B = dict(d_model=4096, n_heads=32, head_dim=128, ffn=12288, vocab=126464, mask_id=126463, rope_base=500000.0)
+
+
+def _timed_steps(ctx, step, n, warm=3):
+    import torch
+    for _ in range(warm):
+        step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(ctx.stream)
+    for _ in range(n):
+        step()
+    e1.record(ctx.stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / n
+
+
+def step_b16(a):
+    """Batch-16 denoising step: synthetic prefix KV of 4096 positions per sequence, a 64-token
+    window (current block + one speculative block) with 32 masked, Zipf(1.1) ids.  Prints
+    ms/step and the projections' achieved bf16 TFLOP/s (events around each launch)."""
+    import numpy as np
+
+    import dllm_inputs as I
+
+    from .dllm import COMMITTED, MASKED, Config, Context, Sched
+
+    B, P, T, L = 16, 4096, 64, a.layers
+    cfg = Config(max_batch=B, max_ctx=P + T, max_window=T, n_layers=L, **SHAPE_8B)
+    ctx = Context(cfg)
+    sched = Sched(steps_per_block=32, spec_trigger=32, spec_blocks=1)
+    ctx.dllm_set_prefix_kv_random(sched, B, P, T, I.SEED_KV)
+    ctx.dllm_begin_block()
+    tok, st, _ = ctx.dllm_get_state()
+    win = np.arange(P, P + T)
+    tok[:, win] = I.zipf_ids((B, T), cfg.vocab, cfg.mask_id)
+    st[:, win] = COMMITTED
+    for b in range(B):
+        m = win[I.masked_positions(T, 32, seed=I.SEED_PROMPT + 100 + b)]
+        tok[b, m], st[b, m] = cfg.mask_id, MASKED
+    ctx.dllm_set_state(tok, st)
+    w = ctx.dllm_window()
+
+    def step():
+        ctx.dllm_rewind_block()
+        ctx.dllm_denoise_step(want_out=False)
+
+    ms = _timed_steps(ctx, step, a.reps)
+    ctx.dllm_set_profile(1)
+    for _ in range(8):
+        step()
+    prof, psteps = ctx.dllm_get_profile()
+    ctx.dllm_set_profile(0)
+    N = B * T
+    d, F, V = cfg.d_model, cfg.ffn, cfg.vocab
+    layer_flops = 2 * N * (4 * d * d + 3 * d * F)
+    head_flops = 2 * N * V * d
+    attn_flops = B * L * 4 * T * (P + T) * d
+    chain_ms = (prof["qkv"]["ms_total"] + prof["layer"]["ms_total"]) / psteps
+    gemm_flops = L * layer_flops + head_flops
+    print(json.dumps({"op": "step-b16", "window": w, "ms_per_step": ms, "steps_per_s": 1e3 / ms,
+                      "kernel_ms_per_step": {k: v["ms_total"] / psteps for k, v in prof.items()},
+                      "gemm_tflops": gemm_flops / (chain_ms * 1e-3) / 1e12,
+                      "attn_kv_GBps": B * L * 2 * (P + T) * d * 2 / (prof["attn"]["ms_total"] / psteps * 1e-3) / 1e9,
+                      "step_tflops": (gemm_flops + L * 0 + attn_flops) / (ms * 1e-3) / 1e12}))
+    ctx.close()
+
+
+def window_sweep(a):
+    """LLaDA-8B step time against the window length (512-token prefix, batch 1): flat while the
+    projections stream weights, rising once the token tile makes them tensor-bound."""
+    import numpy as np
+
+    from .dllm import COMMITTED, MASKED, Config, Context, Sched
+
+    rows = []
+    for T in (32, 64, 96, 128, 192, 256):
+        cfg = Config(max_batch=1, max_ctx=512 + T, max_window=max(T, 512), block_len=T, n_layers=a.layers,
+                     **SHAPE_8B)
+        ctx = Context(cfg)
+        rng = np.random.default_rng(1)
+        ctx.dllm_prefill(Sched(steps_per_block=T), rng.integers(0, 126463, 512).astype(np.int32), T)
+        # one block of length T: the window is the whole block, every position masked
+        ctx.dllm_begin_block()
+        ctx.dllm_set_state(*ctx.dllm_get_state()[:2])  # rewind point
+        w = ctx.dllm_window()
+
+        def step():
+            ctx.dllm_rewind_block()
+            ctx.dllm_denoise_step(want_out=False)
+
+        ms = _timed_steps(ctx, step, a.reps)
+        rows.append({"T": T, "window": w["T"], "ms_per_step": round(ms, 4)})
+        ctx.close()
+    print(json.dumps({"op": "window-sweep", "rows": rows}))
+
+
+def generate(a):
+    """Whole generations through dllm_generate at LLaDA-8B shape: 256-token prompt, 4 blocks of
+    32 with 32 steps per block (one commit per step); and a 1024-token prompt, 8 blocks, with
+    speculation (window 96 when <= 8 masked) and revision (theta 0.5, at most 1 per step)."""
+    import time
+
+    import numpy as np
+
+    import dllm_inputs as I
+
+    from .dllm import Config, Context, Sched
+
+    out = []
+    for name, Lp, gen, sched in (
+            ("blocks_p256_g128", 256, 128, Sched(steps_per_block=32)),
+            ("spec_revision_p1024_g256", 1024, 256,
+             Sched(steps_per_block=32, spec_trigger=8, spec_blocks=2, theta_remask=0.5, remask_max=1))):
+        cfg = Config(max_batch=1, max_ctx=Lp + gen, max_window=max(Lp, 96), n_layers=a.layers, **SHAPE_8B)
+        ctx = Context(cfg)
+        prompt = I.uniform_prompt(Lp, cfg.vocab, cfg.mask_id)
+        ctx.dllm_generate(sched, prompt, gen)  # warm-up: graphs for every window shape
+        ctx.dllm_sync()
+        t0 = time.perf_counter()
+        toks, stats = ctx.dllm_generate(sched, prompt, gen)
+        dt = time.perf_counter() - t0
+        out.append({"workload": name, "seconds": round(dt, 4), "gen_tokens_per_s": gen / dt,
+                    "steps_per_s": stats["steps"] / dt, **stats})
+        ctx.close()
+    print(json.dumps({"op": "generate", "runs": out}))
 
 
 def step_small(a):
