@@ -228,6 +228,19 @@ __device__ __forceinline__ void tmem_ld_32x4(uint32_t taddr, float* v) {
     v[3] = __uint_as_float(r3);
 }
 
+__device__ __forceinline__ void tmem_ld_32x16(uint32_t taddr, float* v) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+        "%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
 __device__ __forceinline__ void tmem_ld_32x8(uint32_t taddr, float* v) {
     uint32_t r[8];
     asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
@@ -236,6 +249,13 @@ __device__ __forceinline__ void tmem_ld_32x8(uint32_t taddr, float* v) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
     for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// N consecutive columns (8 or 16) of the warp's 32 TMEM lanes.
+template <int N>
+__device__ __forceinline__ void tmem_ld_32xn(uint32_t taddr, float* v) {
+    if constexpr (N == 16) tmem_ld_32x16(taddr, v);
+    else tmem_ld_32x8(taddr, v);
 }
 
 // 32 registers per thread -> its TMEM lane, 32 consecutive columns.

@@ -15,7 +15,10 @@
 // single projection (dllm_op_gemm, the first layer's QKV) is a chain of one.
 //
 // Work in a phase is split "stream-K" style: the flattened (tile, 64-wide
-// k-block) iteration space is cut into one contiguous range per CTA, so
+// k-block) iteration space (tiles token-tile-major: the m-tiles of token tile
+// 0, then of token tile 1, ..., so that with several token tiles the CTAs
+// that read the same weight tile for different token tiles run about in step
+// and share it through L2) is cut into one contiguous range per CTA, so
 // every SM streams the same number of weight bytes whatever the tile count.
 // A tile cut between CTAs is finished by the CTA holding its first k-blocks,
 // which are the end of that CTA's range: the other contributors store fp32
@@ -45,6 +48,7 @@ constexpr uint32_t kABytes = kBM * kBK * 2;
 constexpr int kFullSmem = 227 * 1024;
 static int g_stream_budget = kChainSmemShared;  // single projections: shared-memory plan
 constexpr int kTicketStride = 32;  // one tile ticket per 128-byte line
+constexpr int kEpiGroup = 16;      // epilogue columns processed side by side
 
 // Timeline trace slots per CTA (when EpiArgs::trace is set).
 enum { kTrStart = 0, kTrPrologue = 1, kTrFirstData = 2, kTrLastData = 3, kTrEpiDone = 4, kTrExit = 5, kTrSm = 6,
@@ -109,11 +113,13 @@ __device__ __noinline__ float2 rot_cs(float angle) {
 }
 
 // ------------------------------------------------------------------ epilogues
-// Sum of v[0..7] over the 32 lanes of a warp, scattered: afterwards the four lanes
-// 4c..4c+3 hold the total of column c in v[0].  9 shuffles in a fixed order.
-__device__ __forceinline__ void warp_reduce_scatter8(float* v, int lane) {
+// Sum of v[0..N-1] (N a power of two <= 32) over the 32 lanes of a warp, scattered:
+// afterwards the 32/N lanes c*(32/N) .. c*(32/N)+32/N-1 hold the total of column c in v[0].
+// N-1 + log2(32/N) shuffles in a fixed order.
+template <int N>
+__device__ __forceinline__ void warp_reduce_scatter(float* v, int lane) {
 #pragma unroll
-    for (int w = 16, h = 4; w >= 4; w >>= 1, h >>= 1) {
+    for (int w = 16, h = N / 2; h >= 1; w >>= 1, h >>= 1) {
         const bool upper = (lane & w) != 0;
 #pragma unroll
         for (int i = 0; i < h; ++i) {
@@ -122,8 +128,8 @@ __device__ __forceinline__ void warp_reduce_scatter8(float* v, int lane) {
             v[i] = keep + __shfl_xor_sync(0xffffffffu, send, w);
         }
     }
-    v[0] += __shfl_xor_sync(0xffffffffu, v[0], 2);
-    v[0] += __shfl_xor_sync(0xffffffffu, v[0], 1);
+#pragma unroll
+    for (int w = 16 / N; w >= 1; w >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], w);
 }
 
 // Epilogue of a 32-token tile (the batch-1 weight stream), compact: one rolled loop over 4
@@ -138,7 +144,8 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                                              int quarter, int lane, int* status) {
     // col0: the chunk's first token column; c_in: its offset inside the token tile (index into
     // the tile's RMSNorm scales and staged ids); t_x == 0: the old residual is read from global
-    constexpr int GW = 8;  // columns per group
+    constexpr int GW = kEpiGroup;  // columns per group
+    constexpr int LS = 32 / GW;    // lanes sharing one column's sum after the scatter
     const int row = mt * kBM + rt;
     const bool scale = (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) && ep.sq_in != nullptr;
     // QKV state: feature, head, rotation (angle-addition recurrence along the positions)
@@ -174,7 +181,7 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
         if (tr && g == 1) tr[kTrEpiG0] = global_ns();
         const int cg = col0 + GW * g;  // first column of the group
         float a[GW];
-        tmem_ld_32x8(t_src + static_cast<uint32_t>(GW * g), a);
+        tmem_ld_32xn<GW>(t_src + static_cast<uint32_t>(GW * g), a);
         if (scale) {
 #pragma unroll
             for (int u = 0; u < GW; ++u) a[u] *= sm.rs[c_in + GW * g + u];
@@ -186,7 +193,7 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
         } else if constexpr (EPI == EPI_RESID) {
             float xo[GW], ss[GW];
             if (t_x) {
-                tmem_ld_32x8(t_x + static_cast<uint32_t>(GW * g), xo);
+                tmem_ld_32xn<GW>(t_x + static_cast<uint32_t>(GW * g), xo);
             } else {
 #pragma unroll
                 for (int u = 0; u < GW; ++u)
@@ -203,8 +210,8 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                     ep.xb[o] = __float2bfloat16_rn(xo[u]);
                 }
             }
-            warp_reduce_scatter8(ss, lane);
-            if ((lane & 3) == 0) sm.red[quarter * 32 + GW * g + (lane >> 2)] = ss[0];
+            warp_reduce_scatter<GW>(ss, lane);
+            if (lane % LS == 0) sm.red[quarter * 32 + GW * g + lane / LS] = ss[0];
         } else if constexpr (EPI == EPI_QKV) {
             // positions and rotations of the group's 8 columns first (the rare tile that spans
             // sequences takes the out-of-line sincos per column), then the branch-free column pass
@@ -291,8 +298,8 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                     sm.red[(quarter * 32 + GW * g + u) * 3 + 2] = __int_as_float(idx[u]);
                 }
             }
-            warp_reduce_scatter8(e, lane);
-            if ((lane & 3) == 0) sm.red[(quarter * 32 + GW * g + (lane >> 2)) * 3 + 1] = e[0];
+            warp_reduce_scatter<GW>(e, lane);
+            if (lane % LS == 0) sm.red[(quarter * 32 + GW * g + lane / LS) * 3 + 1] = e[0];
 #pragma unroll
             for (int u = 0; u < GW; ++u) {
                 const int col = cg + u;
@@ -384,7 +391,7 @@ __device__ __forceinline__ bool wait_flag(const int* flag, int tag, volatile int
 }
 
 // The epilogue warps' share of one phase: every tile of this CTA's range.
-template <int EPI, bool C32>
+template <int EPI>
 __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph, int tag, uint8_t* red_stage,
                                                   uint64_t* tfull, uint64_t* tempty, uint64_t* redbar,
                                                   volatile int* s_abort, uint32_t tmem_base, const EpiSmem& esm,
@@ -425,10 +432,11 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
     }
     const int nchunks = p.ntile / 32;
     const size_t slot_floats = static_cast<size_t>(p.ntile) * kBM;
-    constexpr bool c32 = C32;  // the launch's token tile is 32 (residual staged in TMEM, bulk-copy reduction)
-    // TMEM: two accumulators of acc_cols columns, then (32-token tiles) the staged residual
+    // TMEM: two accumulators of acc_cols columns, then (token tiles up to 128) the staged old
+    // residual of the finisher's tile, x_cols columns
     const uint32_t t_x =
-        c32 ? tmem_base + static_cast<uint32_t>(2 * ca.acc_cols) + (static_cast<uint32_t>(quarter * 32) << 16) : 0u;
+        ca.x_cols ? tmem_base + static_cast<uint32_t>(2 * ca.acc_cols) + (static_cast<uint32_t>(quarter * 32) << 16)
+                  : 0u;
     int rs_nt = -1, ids_nt = -1;
     long long prepared = -1;
     float v[32];
@@ -439,8 +447,8 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
     auto prepare = [&](long long ptile) {
         if (ptile == prepared) return;
         prepared = ptile;
-        const int pmt = static_cast<int>(ptile / p.n_tiles);
-        const int pnt = static_cast<int>(ptile - static_cast<long long>(pmt) * p.n_tiles);
+        const int pnt = static_cast<int>(ptile / p.m_tiles);
+        const int pmt = static_cast<int>(ptile - static_cast<long long>(pnt) * p.m_tiles);
         if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
             if (ep.sq_in && pnt != rs_nt) {
                 compute_norm_scale(ep, p, pnt, esm, ew * 32 + lane);
@@ -457,14 +465,18 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                 ids_nt = pnt;
             }
         }
-        if constexpr (EPI == EPI_RESID && c32) {
-            const int row = pmt * kBM + rt;
+        if constexpr (EPI == EPI_RESID) {
+            if (t_x) {
+                const int row = pmt * kBM + rt;
+                for (int c = 0; c < nchunks; ++c) {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-                const int col = pnt * 32 + j;
-                v[j] = (row < p.M && col < p.N) ? ep.out[static_cast<size_t>(col) * ep.ld_out + row] : 0.0f;
+                    for (int j = 0; j < 32; ++j) {
+                        const int col = pnt * p.ntile + c * 32 + j;
+                        v[j] = (row < p.M && col < p.N) ? ep.out[static_cast<size_t>(col) * ep.ld_out + row] : 0.0f;
+                    }
+                    tmem_st_32x32(t_x + static_cast<uint32_t>(c * 32), v);
+                }
             }
-            tmem_st_32x32(t_x, v);
         }
     };
     for (long long it = it0; it < it1;) {
@@ -472,8 +484,8 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         const int k_lo = static_cast<int>(it - tile * p.kb);
         const long long tend = (tile + 1) * p.kb;
         const int k_hi = static_cast<int>((it1 < tend ? it1 : tend) - tile * p.kb);
-        const int mt = static_cast<int>(tile / p.n_tiles);
-        const int nt = static_cast<int>(tile - static_cast<long long>(mt) * p.n_tiles);
+        const int nt = static_cast<int>(tile / p.m_tiles);
+        const int mt = static_cast<int>(tile - static_cast<long long>(nt) * p.m_tiles);
         const bool whole = (k_lo == 0 && k_hi == p.kb);
         int c_first = 0, c_last = 0;
         bool reducer = false;
@@ -499,7 +511,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             // the compact epilogue per 32-column chunk, straight from the accumulator in TMEM
             for (int c = 0; c < nchunks; ++c)
                 epilogue_c32<EPI>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt, t_acc + static_cast<uint32_t>(c * 32),
-                                  t_x, esm, ew, quarter, lane, status);
+                                  t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, esm, ew, quarter, lane, status);
         } else if (!reducer) {
             float* my_part = P.partials + static_cast<size_t>(blockIdx.x) * slot_floats;
             for (int c = 0; c < nchunks; ++c) {
@@ -532,58 +544,44 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                 }
             }
             if (named_bar_any(1, 128, *s_abort != 0)) return;
-            const uint32_t part_bytes = static_cast<uint32_t>(slot_floats * 4);
+            // a contributor's partial: chunk c (32 columns) is the contiguous slice
+            // [c*8 + j][row] float4, 16 KB; the slices are bulk-copied, red_bytes at a time
+            constexpr uint32_t slice_bytes = 32 * kBM * 4;
+            const int per_batch = ca.red_bytes / static_cast<int>(slice_bytes);
             for (int c = 0; c < nchunks; ++c) {
                 tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);  // own (first) k-range
-                if constexpr (c32) {
-                    const int per_batch = ca.red_bytes / static_cast<int>(part_bytes);
-                    for (int b0 = 1; b0 < nparts; b0 += per_batch) {
-                        const int nb = nparts - b0 < per_batch ? nparts - b0 : per_batch;
-                        if (threadIdx.x == 64) {
-                            fence_proxy_async_global();
-                            mbar_arrive_expect_tx(redbar, part_bytes * static_cast<uint32_t>(nb));
-                            for (int q = 0; q < nb; ++q)
-                                bulk_load(red_stage + static_cast<size_t>(q) * part_bytes,
-                                          P.partials + static_cast<size_t>(c_first + b0 + q) * slot_floats, part_bytes,
-                                          redbar);
-                        }
-                        mbar_wait(redbar, es.red_phase, s_abort, status);
-                        es.red_phase ^= 1u;
-                        for (int q = 0; q < nb; ++q) {
-                            const float4* src =
-                                reinterpret_cast<const float4*>(red_stage + static_cast<size_t>(q) * part_bytes);
-#pragma unroll
-                            for (int j = 0; j < 8; ++j) {
-                                const float4 a = src[j * kBM + rt];
-                                v[4 * j] += a.x;
-                                v[4 * j + 1] += a.y;
-                                v[4 * j + 2] += a.z;
-                                v[4 * j + 3] += a.w;
-                            }
-                        }
-                        named_bar(1, 128);  // the next batch overwrites the staging memory
+                for (int b0 = 1; b0 < nparts; b0 += per_batch) {
+                    const int nb = nparts - b0 < per_batch ? nparts - b0 : per_batch;
+                    if (threadIdx.x == 64) {
+                        fence_proxy_async_global();
+                        mbar_arrive_expect_tx(redbar, slice_bytes * static_cast<uint32_t>(nb));
+                        for (int q = 0; q < nb; ++q)
+                            bulk_load(red_stage + static_cast<size_t>(q) * slice_bytes,
+                                      P.partials + static_cast<size_t>(c_first + b0 + q) * slot_floats +
+                                          static_cast<size_t>(c) * 32 * kBM,
+                                      slice_bytes, redbar);
                     }
-                } else {
-                    for (int cc = c_first + 1; cc <= c_last; ++cc) {
-                        const float4* p0 =
-                            reinterpret_cast<const float4*>(P.partials + static_cast<size_t>(cc) * slot_floats);
-                        float4 a[8];
-#pragma unroll
-                        for (int j = 0; j < 8; ++j) a[j] = __ldcg(p0 + static_cast<size_t>(c * 8 + j) * kBM + rt);
+                    mbar_wait(redbar, es.red_phase, s_abort, status);
+                    es.red_phase ^= 1u;
+                    for (int q = 0; q < nb; ++q) {
+                        const float4* src =
+                            reinterpret_cast<const float4*>(red_stage + static_cast<size_t>(q) * slice_bytes);
 #pragma unroll
                         for (int j = 0; j < 8; ++j) {
-                            v[4 * j] += a[j].x;
-                            v[4 * j + 1] += a[j].y;
-                            v[4 * j + 2] += a[j].z;
-                            v[4 * j + 3] += a[j].w;
+                            const float4 a = src[j * kBM + rt];
+                            v[4 * j] += a.x;
+                            v[4 * j + 1] += a.y;
+                            v[4 * j + 2] += a.z;
+                            v[4 * j + 3] += a.w;
                         }
                     }
+                    named_bar(1, 128);  // the next batch overwrites the staging memory
                 }
                 if (tr && threadIdx.x == 64 && c == 0) tr[kTrReduced] = global_ns();
                 // the sum goes back into the (still owned) accumulator, then the compact epilogue
                 tmem_st_32x32(t_acc + static_cast<uint32_t>(c * 32), v);
                 epilogue_c32<EPI>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt, t_acc + static_cast<uint32_t>(c * 32),
-                                  t_x, esm, ew, quarter, lane, status);
+                                  t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, esm, ew, quarter, lane, status);
             }
         }
         if (finisher) {
@@ -603,7 +601,6 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
     if (tr && threadIdx.x == 64) tr[kTrEpiDone] = global_ns();
 }
 
-template <bool C32>
 __global__ void __launch_bounds__(kChainThreads, 1)
     k_chain(const __grid_constant__ ChainMaps maps, const __grid_constant__ ChainArgs ca) {
     extern __shared__ uint8_t smem_raw[];
@@ -679,7 +676,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
                 if (tr) tr[kTrStart] = global_ns();
                 // (m-tile, k-block) walked incrementally: no division in the loop
                 int tile = it0 / p.kb, k = it0 - tile * p.kb;
-                int mt = tile / p.n_tiles, nt = tile - mt * p.n_tiles;
+                int nt = tile / p.m_tiles, mt = tile - nt * p.m_tiles;
                 for (int it = it0; it < it1; ++it) {
                     if (!mbar_wait(&empty[stage], par ^ 1u, s_abort, status)) break;
                     mbar_arrive_expect_tx(&full[stage], kABytes + b_bytes);
@@ -693,9 +690,9 @@ __global__ void __launch_bounds__(kChainThreads, 1)
                     }
                     if (++k == p.kb) {
                         k = 0;
-                        if (++nt == p.n_tiles) {
-                            nt = 0;
-                            ++mt;
+                        if (++mt == p.m_tiles) {
+                            mt = 0;
+                            ++nt;
                         }
                     }
                 }
@@ -732,7 +729,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             int win_base = -1, win_nt = -1;  // the 32 producing tiles last polled
             uint32_t win_ready = 0;
             int tile = it0 / p.kb, k = it0 - tile * p.kb;
-            int mt = tile / p.n_tiles, nt = tile - mt * p.n_tiles;
+            int nt = tile / p.m_tiles, mt = tile - nt * p.m_tiles;
             for (int it = it0; it < it1; ++it) {
                 int free_stage = 1;
                 if (lane == 0) free_stage = mbar_wait(&empty[stage], par ^ 1u, s_abort, status) ? 1 : 0;
@@ -779,9 +776,9 @@ __global__ void __launch_bounds__(kChainThreads, 1)
                 }
                 if (++k == p.kb) {
                     k = 0;
-                    if (++nt == p.n_tiles) {
-                        nt = 0;
-                        ++mt;
+                    if (++mt == p.m_tiles) {
+                        mt = 0;
+                        ++nt;
                     }
                 }
             }
@@ -857,19 +854,19 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         for (int ph = 0; ph < ca.n_phases; ++ph) {  // on abort every phase returns at its first barrier
             switch (ca.ph[ph].epi) {
                 case EPI_F32:
-                    chain_phase_epilogue<EPI_F32, C32>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    chain_phase_epilogue<EPI_F32>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
                     break;
                 case EPI_RESID:
-                    chain_phase_epilogue<EPI_RESID, C32>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    chain_phase_epilogue<EPI_RESID>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
                     break;
                 case EPI_QKV:
-                    chain_phase_epilogue<EPI_QKV, C32>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    chain_phase_epilogue<EPI_QKV>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
                     break;
                 case EPI_SWIGLU:
-                    chain_phase_epilogue<EPI_SWIGLU, C32>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    chain_phase_epilogue<EPI_SWIGLU>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
                     break;
                 default:
-                    chain_phase_epilogue<EPI_LMHEAD, C32>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    chain_phase_epilogue<EPI_LMHEAD>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
                     break;
             }
         }
@@ -987,8 +984,9 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
     ca.grid = grid;
     ca.ntile = ntile;
     ca.acc_cols = c32 ? 32 : pow2ceil(ntile);
-    ca.tmem_cols = pow2ceil(2 * ca.acc_cols + (c32 ? 32 : 0));
-    ca.red_bytes = c32 ? 2 * 32 * kBM * 4 : 0;  // two split partials per bulk-copy round
+    ca.x_cols = ntile <= 128 ? ntile : 0;  // staged residual (none for 256-token tiles: TMEM is full)
+    ca.tmem_cols = pow2ceil(2 * ca.acc_cols + ca.x_cols);
+    ca.red_bytes = 2 * 32 * kBM * 4;  // two 32-column partial slices per bulk-copy round
     const int fixed = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + 6 * 8 + 16;
     const int stage_bytes = static_cast<int>(kABytes) + ntile * kBK * 2;
     int st = (smem_budget - fixed) / (stage_bytes + 16);
@@ -1000,12 +998,8 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
 }
 
 cudaError_t chain_init_attrs() {
-    cudaError_t e = cudaFuncSetAttribute(reinterpret_cast<const void*>(k_chain<true>),
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kFullSmem);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(reinterpret_cast<const void*>(k_chain<false>),
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, kFullSmem);
-    return e;
+    return cudaFuncSetAttribute(reinterpret_cast<const void*>(k_chain), cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                kFullSmem);
 }
 
 cudaError_t chain_launch(const ChainMaps& maps, const ChainArgs& ca, cudaStream_t st, bool pdl) {
@@ -1014,10 +1008,7 @@ cudaError_t chain_launch(const ChainMaps& maps, const ChainArgs& ca, cudaStream_
         if (p.grid > ca.grid || !ca.ph[i].partials || !ca.ph[i].tickets || (i > 0 && ca.ph[i].dep_rows < 0))
             return cudaErrorInvalidValue;
     }
-    // 32-token chains (the batch-1 weight stream) and wider token tiles are separate kernels, so
-    // each carries only its own epilogue code
-    if (ca.ntile == 32) return launch_k(k_chain<true>, dim3(ca.grid), dim3(kChainThreads), ca.smem, st, pdl, maps, ca);
-    return launch_k(k_chain<false>, dim3(ca.grid), dim3(kChainThreads), ca.smem, st, pdl, maps, ca);
+    return launch_k(k_chain, dim3(ca.grid), dim3(kChainThreads), ca.smem, st, pdl, maps, ca);
 }
 
 }  // namespace dllm

@@ -89,7 +89,8 @@ struct ChainPhase {
 struct ChainArgs {
     int n_phases;
     int grid, stages, ntile, acc_cols, tmem_cols;
-    int red_bytes;       // shared staging for split partials (32-token tiles)
+    int red_bytes;       // shared staging for split partials
+    int x_cols;          // TMEM columns for the staged old residual (0: read from global)
     size_t smem;
     const int* epoch;    // device step counter; tag = *epoch * tag_mul + tag_add (null: tag = tag_add)
     int tag_mul, tag_add;
@@ -100,7 +101,7 @@ struct ChainMaps {
     CUtensorMap w[kMaxPhases];
     CUtensorMap x[kMaxPhases];
 };
-// Fills grid, stages, ntile, acc_cols, tmem_cols, red_bytes and smem from the phases' plans for a
+// Fills grid, stages, ntile, acc_cols, x_cols, tmem_cols, red_bytes and smem from the phases' plans for a
 // shared-memory budget (bytes, <= 227 KB).  False if the phases do not share one token tiling.
 bool chain_plan(ChainArgs& ca, int smem_budget);
 constexpr int kChainSmemFull = 227 * 1024;    // one CTA per SM, deepest ring
