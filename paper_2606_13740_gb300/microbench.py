@@ -26,7 +26,7 @@ def main(argv=None):
     ap.add_argument("--N", type=int, default=32)
     ap.add_argument("--K", type=int, default=4096)
     ap.add_argument("--B", type=int, default=16)
-    ap.add_argument("--T", type=int, default=64)
+    ap.add_argument("--T", type=int, default=64, help="attention / step-trace: window tokens")
     ap.add_argument("--H", type=int, default=32)
     ap.add_argument("--P", type=int, default=4096)
     ap.add_argument("--reps", type=int, default=3)
@@ -276,13 +276,14 @@ def step_trace(a):
 
     shape = dict(n_layers=32, d_model=4096, n_heads=32, head_dim=128, ffn=12288, vocab=126464, mask_id=126463,
                  rope_base=500000.0)
-    cfg = Config(max_batch=1, max_ctx=544, max_window=512, **shape)
+    T = a.T if a.T in (32, 64, 96, 128, 192, 256) else 32
+    cfg = Config(max_batch=1, max_ctx=512 + T, max_window=512, block_len=T, **shape)
     ctx = Context(cfg)
     flags = 16 | (4 if a.no_pdl else 0) | a.debug
     ctx.dllm_set_debug(flags)
     rng = np.random.default_rng(1)
     prompt = rng.integers(0, cfg.vocab - 1, 512).astype(np.int32)
-    ctx.dllm_prefill(Sched(steps_per_block=24), prompt, 32)
+    ctx.dllm_prefill(Sched(steps_per_block=24), prompt, T)
     ctx.dllm_begin_block()
     for _ in range(4):
         ctx.dllm_denoise_step(want_out=False)
