@@ -1,5 +1,6 @@
 // Element-wise, normalisation, attention and bookkeeping kernels of the
 // denoising step.  The dense projections live in gemm_tc.cu.
+#include "attn.cuh"
 #include "common.cuh"
 #include "internal.h"
 
@@ -156,7 +157,6 @@ cudaError_t launch_embed(const int* tok, int tok_ld, const int* seq_kv, const __
 // in its own shared memory; after a cluster barrier every CTA merges a slice
 // of the rows by reading all csize partials through distributed shared memory,
 // so the merge needs no global scratch, no fences and no atomics.
-constexpr int kAK = 64;      // keys per sub-block
 constexpr int kMaxCluster = 8;
 // attention timeline slots (%globaltimer ns)
 enum { kAtStart = 0, kAtDepWait = 1, kAtLoop = 2, kAtTicket = 3, kAtMerged = 4, kAtSm = 5, kAtLast = 6 };
@@ -165,42 +165,6 @@ __device__ __forceinline__ unsigned smid_attn() {
     unsigned r;
     asm volatile("mov.u32 %0, %%smid;" : "=r"(r));
     return r;
-}
-
-__device__ __forceinline__ int swz(int r, int c, int hd) {
-    return r * hd + ((((c >> 3) ^ (r & 7))) << 3) + (c & 7);
-}
-
-__device__ __forceinline__ void cp_async16(void* dst, const void* src, bool valid) {
-    unsigned s = smem_u32(dst);
-    int n = valid ? 16 : 0;
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(s), "l"(src), "r"(n) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
-
-__device__ __forceinline__ void ldm_x4(uint32_t addr, uint32_t& a, uint32_t& b, uint32_t& c, uint32_t& d) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(a), "=r"(b), "=r"(c), "=r"(d)
-                 : "r"(addr));
-}
-__device__ __forceinline__ void ldm_x4_t(uint32_t addr, uint32_t& a, uint32_t& b, uint32_t& c, uint32_t& d) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(a), "=r"(b), "=r"(c), "=r"(d)
-                 : "r"(addr));
-}
-__device__ __forceinline__ void mma16816(float* d, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
-                                         uint32_t b1) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-        "{%0,%1,%2,%3};"
-        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
-}
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<uint32_t*>(&v);
 }
 
 // ---- thread-block cluster helpers
@@ -268,157 +232,19 @@ __global__ void __launch_bounds__(NW * 32) k_attn(const __nv_bfloat16* __restric
     const int nq = min(AQ, T - q0);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int g = lane >> 2, c4 = lane & 3;
-    constexpr int CPR = HD / 8;  // 16-byte chunks per row
 
     const __nv_bfloat16* qbase = q + ((static_cast<size_t>(b) * H + h) * T + q0) * HD;
     const __nv_bfloat16* kbase = kc + (static_cast<size_t>(b) * H + h) * cap * HD;
     const __nv_bfloat16* vbase = vc + (static_cast<size_t>(b) * H + h) * cap * HD;
 
-    auto load_rows = [&](__nv_bfloat16* dst, const __nv_bfloat16* base, int k0) {
-        for (int e = tid; e < kAK * CPR; e += NT) {
-            const int r = e / CPR, cc = (e % CPR) * 8;
-            const int key = k0 + r;
-            const bool ok = key < kend;
-            cp_async16(dst + swz(r, cc, HD), base + static_cast<size_t>(ok ? key : kbeg) * HD + cc, ok);
-        }
-    };
-    const bool has = kbeg < kend;
-    const bool prefix_first = has && kbeg + kAK <= kv;  // first sub-block entirely in the cached prefix
-    if (prefix_first) {  // groups: K0, V0 (then Q)
-        load_rows(sK, kbase, kbeg);
-        cp_async_commit();
-        load_rows(sV, vbase, kbeg);
-        cp_async_commit();
-    }
+    auto sync = []() { __syncthreads(); };
+    const bool prefix_first = attn_prefetch_prefix<HD, NT>(kbase, vbase, kv, kbeg, kend, sK, sV, tid);
     pdl_wait();
     if (tr) tr[kAtDepWait] = global_ns();
-    for (int e = tid; e < AQ * CPR; e += NT) {
-        const int r = e / CPR, cc = (e % CPR) * 8;
-        cp_async16(sQ + swz(r, cc, HD), qbase + static_cast<size_t>(r < nq ? r : 0) * HD + cc, r < nq);
-    }
-    if (has && !prefix_first) load_rows(sK, kbase, kbeg);
-    cp_async_commit();  // group: Q (+ K0)
-    if (has && !prefix_first) {
-        load_rows(sV, vbase, kbeg);
-        cp_async_commit();  // group: V0
-    }
-
-    constexpr int KS = HD / 16;  // k-steps of Q.K
     constexpr int DN = HD / 8;   // output n-blocks
-    uint32_t qa[KS][4];
     float o[DN][4];
-#pragma unroll
-    for (int i = 0; i < DN; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.0f;
-    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.0f, l1 = 0.0f;
-    const float sl2 = rsqrtf(static_cast<float>(HD)) * 1.4426950408889634f;
-
-    for (int k0 = kbeg; k0 < kend; k0 += kAK) {
-        const bool first = k0 == kbeg;
-        const bool more = k0 + kAK < kend;
-        // pending groups, oldest first: K_i, V_i (first: K0, V0, Q or Q+K0, V0)
-        if (first && prefix_first) cp_async_wait_all();
-        else cp_async_wait_1();
-        __syncthreads();
-        if (first) {
-#pragma unroll
-            for (int ks = 0; ks < KS; ++ks) {
-                const int r = warp * 16 + (lane & 15), cc = ks * 16 + (lane >> 4) * 8;
-                ldm_x4(smem_u32(sQ + swz(r, cc, HD)), qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3]);
-            }
-        }
-        float s[8][4];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.0f;
-#pragma unroll
-        for (int jp = 0; jp < 4; ++jp) {
-#pragma unroll
-            for (int ks = 0; ks < KS; ++ks) {
-                const int mi = lane >> 3, rr = lane & 7;
-                const int key = jp * 16 + (mi >> 1) * 8 + rr, cc = ks * 16 + (mi & 1) * 8;
-                uint32_t b0, b1, b2, b3;
-                ldm_x4(smem_u32(sK + swz(key, cc, HD)), b0, b1, b2, b3);
-                mma16816(s[2 * jp], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b0, b1);
-                mma16816(s[2 * jp + 1], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b2, b3);
-            }
-        }
-        __syncthreads();  // K consumed: the next sub-block's K streams in behind the softmax and P.V
-        if (more) {
-            load_rows(sK, kbase, k0 + kAK);
-            cp_async_commit();
-        }
-        // scale to log2 units, mask keys past the end, online softmax
-        float mx0 = -INFINITY, mx1 = -INFINITY;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            const int key = k0 + j * 8 + 2 * c4;
-            const bool v0 = key < kend, v1 = key + 1 < kend;
-            s[j][0] = v0 ? s[j][0] * sl2 : -INFINITY;
-            s[j][1] = v1 ? s[j][1] * sl2 : -INFINITY;
-            s[j][2] = v0 ? s[j][2] * sl2 : -INFINITY;
-            s[j][3] = v1 ? s[j][3] * sl2 : -INFINITY;
-            mx0 = fmaxf(mx0, fmaxf(s[j][0], s[j][1]));
-            mx1 = fmaxf(mx1, fmaxf(s[j][2], s[j][3]));
-        }
-        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-        const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-        const float ms0 = mn0 == -INFINITY ? 0.0f : mn0, ms1 = mn1 == -INFINITY ? 0.0f : mn1;
-        const float al0 = exp2f(m0 - ms0), al1 = exp2f(m1 - ms1);
-        m0 = mn0;
-        m1 = mn1;
-        l0 *= al0;
-        l1 *= al1;
-#pragma unroll
-        for (int i = 0; i < DN; ++i) {
-            o[i][0] *= al0;
-            o[i][1] *= al0;
-            o[i][2] *= al1;
-            o[i][3] *= al1;
-        }
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            s[j][0] = exp2f(s[j][0] - ms0);
-            s[j][1] = exp2f(s[j][1] - ms0);
-            s[j][2] = exp2f(s[j][2] - ms1);
-            s[j][3] = exp2f(s[j][3] - ms1);
-            l0 += s[j][0] + s[j][1];
-            l1 += s[j][2] + s[j][3];
-        }
-        // pending: V_i (+ K_{i+1})
-        if (more) cp_async_wait_1();
-        else cp_async_wait_all();
-        __syncthreads();
-        // O += P V
-#pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
-            const uint32_t a0 = pack_bf16(s[2 * kk][0], s[2 * kk][1]);
-            const uint32_t a1 = pack_bf16(s[2 * kk][2], s[2 * kk][3]);
-            const uint32_t a2 = pack_bf16(s[2 * kk + 1][0], s[2 * kk + 1][1]);
-            const uint32_t a3 = pack_bf16(s[2 * kk + 1][2], s[2 * kk + 1][3]);
-#pragma unroll
-            for (int dn = 0; dn < DN; dn += 2) {
-                const int mi = lane >> 3, rr = lane & 7;
-                const int key = kk * 16 + (mi & 1) * 8 + rr, cc = (dn + (mi >> 1)) * 8;
-                uint32_t b0, b1, b2, b3;
-                ldm_x4_t(smem_u32(sV + swz(key, cc, HD)), b0, b1, b2, b3);
-                mma16816(o[dn], a0, a1, a2, a3, b0, b1);
-                mma16816(o[dn + 1], a0, a1, a2, a3, b2, b3);
-            }
-        }
-        __syncthreads();  // V consumed
-        if (more) {
-            load_rows(sV, vbase, k0 + kAK);
-            cp_async_commit();
-        }
-    }
-    cp_async_wait_all();  // a CTA without keys still has its Q copy in flight
-    __syncthreads();
-    l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
-    l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
-    l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
-    l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+    float m0, m1, l0, l1;
+    attn_split<HD, NW>(qbase, kbase, vbase, kbeg, kend, nq, prefix_first, sQ, sK, sV, tid, sync, o, m0, m1, l0, l1);
     if (tr) tr[kAtLoop] = global_ns();
 
     const int r0 = warp * 16 + g, r1 = r0 + 8;
