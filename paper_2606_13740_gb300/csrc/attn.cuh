@@ -21,6 +21,10 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src, bool vali
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
 
 __device__ __forceinline__ void ldm_x4(uint32_t addr, uint32_t& a, uint32_t& b, uint32_t& c, uint32_t& d) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
@@ -71,11 +75,12 @@ __device__ __forceinline__ bool attn_prefetch_prefix(const __nv_bfloat16* kbase,
 }
 
 // The split proper (after the dependency wait): NW warps, tid in [0, 32 NW), nq valid query
-// rows of the tile at qbase; shared Q [16 NW][HD], K and V [kAK][HD]; sync() synchronises
-// the NW warps.  Out: unnormalised o for rows r0 = 16 warp + lane/4 and r1 = r0 + 8
+// rows of the tile at qbase; shared Q [16 NW][HD], K and V [NB][kAK][HD]; sync() synchronises
+// the NW warps.  NB = 1: the next sub-block's K streams in behind this one's softmax and P.V,
+// its V behind the next Q.K^T; NB = 2 (long key ranges): two sub-blocks ahead.  Out: unnormalised o for rows r0 = 16 warp + lane/4 and r1 = r0 + 8
 // (columns dn*8 + 2 (lane%4) + {0,1}), their running max (log2 units) and sum.  A split
 // without keys leaves o = 0, m = -inf, l = 0.
-template <int HD, int NW, typename Sync>
+template <int HD, int NW, int NB, typename Sync>
 __device__ __forceinline__ void attn_split(const __nv_bfloat16* qbase, const __nv_bfloat16* kbase,
                                            const __nv_bfloat16* vbase, int kbeg, int kend, int nq, bool prefix_first,
                                            __nv_bfloat16* sQ, __nv_bfloat16* sK, __nv_bfloat16* sV, int tid, Sync sync,
@@ -104,6 +109,13 @@ __device__ __forceinline__ void attn_split(const __nv_bfloat16* qbase, const __n
         load_rows(sV, vbase, kbeg);
         cp_async_commit();  // group: V0
     }
+    if constexpr (NB == 2) {
+        // groups so far: K0, V0, Q (prefix first) or Q+K0, V0; then K1, V1 (empty past the end)
+        if (kbeg + kAK < kend) load_rows(sK + kAK * HD, kbase, kbeg + kAK);
+        cp_async_commit();
+        if (kbeg + kAK < kend) load_rows(sV + kAK * HD, vbase, kbeg + kAK);
+        cp_async_commit();
+    }
 
     constexpr int KS = HD / 16;  // k-steps of Q.K
     constexpr int DN = HD / 8;   // output n-blocks
@@ -116,12 +128,22 @@ __device__ __forceinline__ void attn_split(const __nv_bfloat16* qbase, const __n
     l1 = 0.0f;
     const float sl2 = rsqrtf(static_cast<float>(HD)) * 1.4426950408889634f;
 
-    for (int k0 = kbeg; k0 < kend; k0 += kAK) {
+    int it = 0;
+    for (int k0 = kbeg; k0 < kend; k0 += kAK, ++it) {
         const bool first = k0 == kbeg;
         const bool more = k0 + kAK < kend;
-        // pending groups, oldest first: K_i, V_i (first: K0, V0, Q or Q+K0, V0)
-        if (first && prefix_first) cp_async_wait_all();
-        else cp_async_wait_1();
+        __nv_bfloat16* K = sK + (NB == 2 ? (it & 1) * kAK * HD : 0);
+        __nv_bfloat16* V = sV + (NB == 2 ? (it & 1) * kAK * HD : 0);
+        if constexpr (NB == 1) {
+            // pending groups, oldest first: K_i, V_i (first: K0, V0, Q or Q+K0, V0)
+            if (first && prefix_first) cp_async_wait_all();
+            else cp_async_wait_1();
+        } else {
+            // the three most recent groups may stay pending (V_i, K_i+1, V_i+1; first sub-block
+            // with the prefix fetched early: K1, V1 after Q)
+            if (first && prefix_first) cp_async_wait<2>();
+            else cp_async_wait<3>();
+        }
         sync();
         if (first) {
 #pragma unroll
@@ -140,14 +162,19 @@ __device__ __forceinline__ void attn_split(const __nv_bfloat16* qbase, const __n
                 const int mi = lane >> 3, rr = lane & 7;
                 const int key = jp * 16 + (mi >> 1) * 8 + rr, cc = ks * 16 + (mi & 1) * 8;
                 uint32_t b0, b1, b2, b3;
-                ldm_x4(smem_u32(sK + swz(key, cc, HD)), b0, b1, b2, b3);
+                ldm_x4(smem_u32(K + swz(key, cc, HD)), b0, b1, b2, b3);
                 mma16816(s[2 * jp], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b0, b1);
                 mma16816(s[2 * jp + 1], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b2, b3);
             }
         }
         sync();  // K consumed: the next sub-block's K streams in behind the softmax and P.V
-        if (more) {
-            load_rows(sK, kbase, k0 + kAK);
+        if constexpr (NB == 1) {
+            if (more) {
+                load_rows(sK, kbase, k0 + kAK);
+                cp_async_commit();
+            }
+        } else {  // K two sub-blocks ahead into the buffer just read (an empty group past the end)
+            if (k0 + 2 * kAK < kend) load_rows(K, kbase, k0 + 2 * kAK);
             cp_async_commit();
         }
         // scale to log2 units, mask keys past the end, online softmax
@@ -190,9 +217,13 @@ __device__ __forceinline__ void attn_split(const __nv_bfloat16* qbase, const __n
             l0 += s[j][0] + s[j][1];
             l1 += s[j][2] + s[j][3];
         }
-        // pending: V_i (+ K_{i+1})
-        if (more) cp_async_wait_1();
-        else cp_async_wait_all();
+        if constexpr (NB == 1) {
+            // pending: V_i (+ K_{i+1})
+            if (more) cp_async_wait_1();
+            else cp_async_wait_all();
+        } else {
+            cp_async_wait<3>();  // V_i done; K_i+1, V_i+1, K_i+2 may stay pending
+        }
         sync();
         // O += P V
 #pragma unroll
@@ -206,14 +237,19 @@ __device__ __forceinline__ void attn_split(const __nv_bfloat16* qbase, const __n
                 const int mi = lane >> 3, rr = lane & 7;
                 const int key = kk * 16 + (mi & 1) * 8 + rr, cc = (dn + (mi >> 1)) * 8;
                 uint32_t b0, b1, b2, b3;
-                ldm_x4_t(smem_u32(sV + swz(key, cc, HD)), b0, b1, b2, b3);
+                ldm_x4_t(smem_u32(V + swz(key, cc, HD)), b0, b1, b2, b3);
                 mma16816(o[dn], a0, a1, a2, a3, b0, b1);
                 mma16816(o[dn + 1], a0, a1, a2, a3, b2, b3);
             }
         }
         sync();  // V consumed
-        if (more) {
-            load_rows(sV, vbase, k0 + kAK);
+        if constexpr (NB == 1) {
+            if (more) {
+                load_rows(sV, vbase, k0 + kAK);
+                cp_async_commit();
+            }
+        } else {
+            if (k0 + 2 * kAK < kend) load_rows(V, vbase, k0 + 2 * kAK);
             cp_async_commit();
         }
     }

@@ -196,7 +196,7 @@ __device__ __forceinline__ float4 dsmem_ld4(uint32_t addr) {
 // one's softmax and P.V run, its V while the next Q.K^T runs.  After the key
 // loop the same memory holds the CTA's partial: O [16*NW][HD] fp32 and
 // (max, sum) [16*NW][2].
-template <int HD, int NW>
+template <int HD, int NW, int NB>
 __global__ void __launch_bounds__(NW * 32) k_attn(const __nv_bfloat16* __restrict__ q,
                                                   const __nv_bfloat16* __restrict__ kc,
                                                   const __nv_bfloat16* __restrict__ vc, const int* __restrict__ seq_kv,
@@ -219,7 +219,7 @@ __global__ void __launch_bounds__(NW * 32) k_attn(const __nv_bfloat16* __restric
     pdl_launch_dependents();
     __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem_attn);
     __nv_bfloat16* sK = sQ + AQ * HD;
-    __nv_bfloat16* sV = sK + kAK * HD;
+    __nv_bfloat16* sV = sK + NB * kAK * HD;
 
     const int split = blockIdx.x, h = blockIdx.y;  // split = rank in the cluster
     const int b = blockIdx.z / qtiles, qt = blockIdx.z - b * qtiles;
@@ -244,7 +244,8 @@ __global__ void __launch_bounds__(NW * 32) k_attn(const __nv_bfloat16* __restric
     constexpr int DN = HD / 8;   // output n-blocks
     float o[DN][4];
     float m0, m1, l0, l1;
-    attn_split<HD, NW>(qbase, kbase, vbase, kbeg, kend, nq, prefix_first, sQ, sK, sV, tid, sync, o, m0, m1, l0, l1);
+    attn_split<HD, NW, NB>(qbase, kbase, vbase, kbeg, kend, nq, prefix_first, sQ, sK, sV, tid, sync, o, m0, m1, l0,
+                           l1);
     if (tr) tr[kAtLoop] = global_ns();
 
     const int r0 = warp * 16 + g, r1 = r0 + 8;
@@ -319,25 +320,31 @@ __global__ void __launch_bounds__(NW * 32) k_attn(const __nv_bfloat16* __restric
     if (tr) tr[kAtMerged] = global_ns();
 }
 
-static size_t attn_smem(int nw, int hd) { return static_cast<size_t>(nw * 16 + 2 * kAK) * hd * 2; }
+static size_t attn_smem(int nw, int nb, int hd) { return static_cast<size_t>(nw * 16 + 2 * nb * kAK) * hd * 2; }
+
+template <int HD, int NW, int NB>
+static cudaError_t attn_attr() {
+    return cudaFuncSetAttribute(reinterpret_cast<const void*>(k_attn<HD, NW, NB>),
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(attn_smem(NW, NB, HD)));
+}
 
 cudaError_t attn_init_attrs() {
-    cudaError_t e = cudaSuccess;
-    auto set = [&](const void* f, size_t bytes) {
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
-    };
-    set(reinterpret_cast<const void*>(k_attn<128, 2>), attn_smem(2, 128));
-    set(reinterpret_cast<const void*>(k_attn<128, 4>), attn_smem(4, 128));
-    set(reinterpret_cast<const void*>(k_attn<64, 2>), attn_smem(2, 64));
-    set(reinterpret_cast<const void*>(k_attn<64, 4>), attn_smem(4, 64));
+    cudaError_t e = attn_attr<128, 2, 1>();
+    if (e == cudaSuccess) e = attn_attr<128, 2, 2>();
+    if (e == cudaSuccess) e = attn_attr<128, 4, 1>();
+    if (e == cudaSuccess) e = attn_attr<128, 4, 2>();
+    if (e == cudaSuccess) e = attn_attr<64, 2, 1>();
+    if (e == cudaSuccess) e = attn_attr<64, 2, 2>();
+    if (e == cudaSuccess) e = attn_attr<64, 4, 1>();
+    if (e == cudaSuccess) e = attn_attr<64, 4, 2>();
     return e;
 }
 
 AttnPlan attn_plan(int B, int T, int H, int max_keys, int sms) {
     AttnPlan a;
-    // two warps (32 query rows) for the short windows of cached decoding, four otherwise
-    a.nw = T <= 64 ? 2 : 4;
+    // two warps (32 query rows) for the short windows of cached decoding, four otherwise: a
+    // 64-token window is one query tile, so its keys and values are read once
+    a.nw = T <= 32 ? 2 : 4;
     a.qtiles = (T + a.nw * 16 - 1) / (a.nw * 16);
     // key splits (cluster size): about two CTAs per SM, at most one split per sub-block
     const int units = B * H * a.qtiles;
@@ -347,18 +354,28 @@ AttnPlan attn_plan(int B, int T, int H, int max_keys, int sms) {
     if (c > blocks) c = blocks;
     if (c < 1) c = 1;
     a.csize = c;
+    // long key ranges per CTA keep two sub-blocks of K and V in flight
+    a.nb = (blocks + c - 1) / c >= 3 ? 2 : 1;
     return a;
+}
+
+template <int HD, int NW, int NB>
+static cudaError_t attn_go(cudaLaunchConfig_t& cfg, const __nv_bfloat16* q, const __nv_bfloat16* kc,
+                           const __nv_bfloat16* vc, const int* seq_kv, __nv_bfloat16* out, int T, int H, int cap,
+                           const AttnPlan& a, unsigned long long* trace) {
+    cfg.dynamicSmemBytes = attn_smem(NW, NB, HD);
+    return cudaLaunchKernelEx(&cfg, k_attn<HD, NW, NB>, q, kc, vc, seq_kv, out, T, H, cap, a.qtiles, a.csize, trace);
 }
 
 cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
                              const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int hd, int cap,
                              const AttnPlan& a, cudaStream_t st, bool pdl, unsigned long long* trace) {
-    if (a.csize < 1 || a.csize > kMaxCluster || (a.nw != 2 && a.nw != 4) || (hd != 64 && hd != 128))
+    if (a.csize < 1 || a.csize > kMaxCluster || (a.nw != 2 && a.nw != 4) || (a.nb != 1 && a.nb != 2) ||
+        (hd != 64 && hd != 128))
         return cudaErrorInvalidValue;
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3(a.csize, H, B * a.qtiles);
     cfg.blockDim = dim3(a.nw * 32);
-    cfg.dynamicSmemBytes = attn_smem(a.nw, hd);
     cfg.stream = st;
     cudaLaunchAttribute at[2];
     int n = 0;
@@ -374,15 +391,17 @@ cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, co
     }
     cfg.attrs = at;
     cfg.numAttrs = n;
-    if (hd == 128)
-        return a.nw == 2 ? cudaLaunchKernelEx(&cfg, k_attn<128, 2>, q, kc, vc, seq_kv, out, T, H, cap, a.qtiles,
-                                              a.csize, trace)
-                         : cudaLaunchKernelEx(&cfg, k_attn<128, 4>, q, kc, vc, seq_kv, out, T, H, cap, a.qtiles,
-                                              a.csize, trace);
-    return a.nw == 2 ? cudaLaunchKernelEx(&cfg, k_attn<64, 2>, q, kc, vc, seq_kv, out, T, H, cap, a.qtiles, a.csize,
-                                          trace)
-                     : cudaLaunchKernelEx(&cfg, k_attn<64, 4>, q, kc, vc, seq_kv, out, T, H, cap, a.qtiles, a.csize,
-                                          trace);
+    const int key = (hd == 128 ? 4 : 0) + (a.nw == 4 ? 2 : 0) + (a.nb == 2 ? 1 : 0);
+    switch (key) {
+        case 0: return attn_go<64, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        case 1: return attn_go<64, 2, 2>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        case 2: return attn_go<64, 4, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        case 3: return attn_go<64, 4, 2>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        case 4: return attn_go<128, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        case 5: return attn_go<128, 2, 2>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        case 6: return attn_go<128, 4, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        default: return attn_go<128, 4, 2>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+    }
 }
 
 // ------------------------------------------------------------------ LM head
