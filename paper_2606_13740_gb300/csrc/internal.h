@@ -157,7 +157,8 @@ cudaError_t launch_embed(const int* tok, int tok_ld, const int* seq_kv, const __
 // their partials through distributed shared memory.
 struct AttnPlan {
     int qtiles, nw, csize;
-    int nb;  // K/V sub-blocks in flight per CTA (1 or 2)
+    int nb;     // K/V sub-blocks in flight per CTA (1 or 2)
+    int pairs;  // warp groups per CTA, each on its own share of the CTA's sub-blocks (1 or 2)
 };
 AttnPlan attn_plan(int B, int T, int H, int max_keys, int sms);
 cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,

@@ -196,14 +196,16 @@ __device__ __forceinline__ float4 dsmem_ld4(uint32_t addr) {
 // one's softmax and P.V run, its V while the next Q.K^T runs.  After the key
 // loop the same memory holds the CTA's partial: O [16*NW][HD] fp32 and
 // (max, sum) [16*NW][2].
-template <int HD, int NW, int NB>
-__global__ void __launch_bounds__(NW * 32) k_attn(const __nv_bfloat16* __restrict__ q,
-                                                  const __nv_bfloat16* __restrict__ kc,
-                                                  const __nv_bfloat16* __restrict__ vc, const int* __restrict__ seq_kv,
-                                                  __nv_bfloat16* __restrict__ out, int T, int H, int cap, int qtiles,
-                                                  int csize, unsigned long long* trace) {
+template <int HD, int NW, int NB, int PR>
+__global__ void __launch_bounds__(PR * NW * 32) k_attn(const __nv_bfloat16* __restrict__ q,
+                                                       const __nv_bfloat16* __restrict__ kc,
+                                                       const __nv_bfloat16* __restrict__ vc,
+                                                       const int* __restrict__ seq_kv, __nv_bfloat16* __restrict__ out,
+                                                       int T, int H, int cap, int qtiles, int csize,
+                                                       unsigned long long* trace) {
     constexpr int AQ = NW * 16;  // query rows per CTA
-    constexpr int NT = NW * 32;
+    constexpr int NT = NW * 32;  // threads of one warp group
+    constexpr int PART = (AQ + 2 * NB * kAK) * HD * 2;  // one group's Q, K, V tiles
     extern __shared__ __align__(128) uint8_t smem_attn[];
     const int cta = (blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
     unsigned long long* tr = (trace && cta < 256 && threadIdx.x == 0) ? trace + static_cast<size_t>(cta) * 16 : nullptr;
@@ -217,7 +219,9 @@ __global__ void __launch_bounds__(NW * 32) k_attn(const __nv_bfloat16* __restric
     // projection writes the window rows [kv_len, kv_len + T)), so they may be read before
     // the dependency wait
     pdl_launch_dependents();
-    __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem_attn);
+    // PR groups of NW warps per CTA, each on its own share of the CTA's key sub-blocks
+    const int grp = threadIdx.x / NT;
+    __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem_attn + grp * PART);
     __nv_bfloat16* sK = sQ + AQ * HD;
     __nv_bfloat16* sV = sK + NB * kAK * HD;
 
@@ -226,22 +230,26 @@ __global__ void __launch_bounds__(NW * 32) k_attn(const __nv_bfloat16* __restric
     const int kv = seq_kv[b];
     const int NK = kv + T;
     const int nblk = (NK + kAK - 1) / kAK;
-    const int kbeg = (split * nblk / csize) * kAK;
-    const int kend = min(NK, ((split + 1) * nblk / csize) * kAK);  // empty when kbeg >= kend
+    const int blk0 = split * nblk / csize, blk1 = (split + 1) * nblk / csize;  // the CTA's sub-blocks
+    const int kbeg = (blk0 + grp * (blk1 - blk0) / PR) * kAK;
+    const int kend = min(NK, (blk0 + (grp + 1) * (blk1 - blk0) / PR) * kAK);  // empty when kbeg >= kend
     const int q0 = qt * AQ;
     const int nq = min(AQ, T - q0);
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int tid = threadIdx.x - grp * NT, warp = tid >> 5, lane = tid & 31;
     const int g = lane >> 2, c4 = lane & 3;
 
     const __nv_bfloat16* qbase = q + ((static_cast<size_t>(b) * H + h) * T + q0) * HD;
     const __nv_bfloat16* kbase = kc + (static_cast<size_t>(b) * H + h) * cap * HD;
     const __nv_bfloat16* vbase = vc + (static_cast<size_t>(b) * H + h) * cap * HD;
 
-    auto sync = []() { __syncthreads(); };
+    auto sync = [grp]() {
+        if constexpr (PR == 1) __syncthreads();
+        else named_bar(1 + grp, NT);
+    };
     const bool prefix_first = attn_prefetch_prefix<HD, NT>(kbase, vbase, kv, kbeg, kend, sK, sV, tid);
     pdl_wait();
     if (tr) tr[kAtDepWait] = global_ns();
-    constexpr int DN = HD / 8;   // output n-blocks
+    constexpr int DN = HD / 8;  // output n-blocks
     float o[DN][4];
     float m0, m1, l0, l1;
     attn_split<HD, NW, NB>(qbase, kbase, vbase, kbeg, kend, nq, prefix_first, sQ, sK, sV, tid, sync, o, m0, m1, l0,
@@ -250,7 +258,7 @@ __global__ void __launch_bounds__(NW * 32) k_attn(const __nv_bfloat16* __restric
 
     const int r0 = warp * 16 + g, r1 = r0 + 8;
     const int qd = H * HD;
-    if (csize == 1) {
+    if (csize == 1 && PR == 1) {
         const float i0 = 1.0f / l0, i1 = 1.0f / l1;
 #pragma unroll
         for (int dn = 0; dn < DN; ++dn) {
@@ -264,9 +272,9 @@ __global__ void __launch_bounds__(NW * 32) k_attn(const __nv_bfloat16* __restric
         }
         return;
     }
-    // partial of this split into shared memory (the Q/K/V tiles are no longer needed)
-    float* sO = reinterpret_cast<float*>(smem_attn);  // [AQ][HD]
-    float* sML = sO + AQ * HD;                        // [AQ][2]
+    // each group's partial into its own shared memory (its Q/K/V tiles are no longer needed)
+    float* sO = reinterpret_cast<float*>(smem_attn + grp * PART);  // [AQ][HD]
+    float* sML = sO + AQ * HD;                                      // [AQ][2]
 #pragma unroll
     for (int dn = 0; dn < DN; ++dn) {
         const int col = dn * 8 + 2 * c4;
@@ -277,38 +285,43 @@ __global__ void __launch_bounds__(NW * 32) k_attn(const __nv_bfloat16* __restric
         *reinterpret_cast<float2*>(sML + r0 * 2) = make_float2(m0, l0);
         *reinterpret_cast<float2*>(sML + r1 * 2) = make_float2(m1, l1);
     }
-    cluster_sync_all();  // every split's partial is in place
+    cluster_sync_all();  // every split's partials are in place
     if (tr) tr[kAtTicket] = global_ns();
-    // this CTA merges output elements split*NT + tid (+ k * csize * NT): row r, 4 features
+    // this CTA merges output elements split*PR*NT + tid (+ k * csize * PR * NT): row r, 4
+    // features, over the csize * PR partials (CTA c, group p) in that order
     constexpr int V4 = HD / 4;
-    for (int e = split * NT + tid; e < nq * V4; e += csize * NT) {
+    constexpr int MP = kMaxCluster * PR;
+    const int all = threadIdx.x;
+    for (int e = split * PR * NT + all; e < nq * V4; e += csize * PR * NT) {
         const int r = e / V4, i4 = e - r * V4;
-        const uint32_t a_ml = smem_u32(sML + r * 2);
-        const uint32_t a_o = smem_u32(sO + r * HD + i4 * 4);
-        float2 ml[kMaxCluster];
-        float4 ov[kMaxCluster];
+        float2 ml[MP];
+        float4 ov[MP];
 #pragma unroll
         for (int c = 0; c < kMaxCluster; ++c) {
-            if (c < csize) {
-                ml[c] = dsmem_ld2(dsmem_map(a_ml, c));
-                ov[c] = dsmem_ld4(dsmem_map(a_o, c));
+#pragma unroll
+            for (int p = 0; p < PR; ++p) {
+                if (c < csize) {
+                    const float* po = reinterpret_cast<const float*>(smem_attn + p * PART);
+                    ml[c * PR + p] = dsmem_ld2(dsmem_map(smem_u32(po + AQ * HD + r * 2), c));
+                    ov[c * PR + p] = dsmem_ld4(dsmem_map(smem_u32(po + r * HD + i4 * 4), c));
+                }
             }
         }
         float M = -INFINITY;
 #pragma unroll
-        for (int c = 0; c < kMaxCluster; ++c)
-            if (c < csize) M = fmaxf(M, ml[c].x);
+        for (int k = 0; k < MP; ++k)
+            if (k < csize * PR) M = fmaxf(M, ml[k].x);
         float L = 0.0f;
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-        for (int c = 0; c < kMaxCluster; ++c) {
-            if (c < csize) {
-                const float w = ml[c].x == -INFINITY ? 0.0f : exp2f(ml[c].x - M);  // split without keys: 0
-                L += w * ml[c].y;
-                acc.x += w * ov[c].x;
-                acc.y += w * ov[c].y;
-                acc.z += w * ov[c].z;
-                acc.w += w * ov[c].w;
+        for (int k = 0; k < MP; ++k) {
+            if (k < csize * PR) {
+                const float w = ml[k].x == -INFINITY ? 0.0f : exp2f(ml[k].x - M);  // a share without keys: 0
+                L += w * ml[k].y;
+                acc.x += w * ov[k].x;
+                acc.y += w * ov[k].y;
+                acc.z += w * ov[k].z;
+                acc.w += w * ov[k].w;
             }
         }
         const float inv = 1.0f / L;
@@ -316,27 +329,32 @@ __global__ void __launch_bounds__(NW * 32) k_attn(const __nv_bfloat16* __restric
         *reinterpret_cast<__nv_bfloat162*>(op) = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
         *reinterpret_cast<__nv_bfloat162*>(op + 2) = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
     }
-    cluster_sync_all();  // no CTA leaves while its partial may still be read
+    cluster_sync_all();  // no CTA leaves while its partials may still be read
     if (tr) tr[kAtMerged] = global_ns();
 }
 
-static size_t attn_smem(int nw, int nb, int hd) { return static_cast<size_t>(nw * 16 + 2 * nb * kAK) * hd * 2; }
+static size_t attn_smem(int nw, int nb, int pr, int hd) {
+    return static_cast<size_t>(pr) * (nw * 16 + 2 * nb * kAK) * hd * 2;
+}
 
-template <int HD, int NW, int NB>
+template <int HD, int NW, int NB, int PR>
 static cudaError_t attn_attr() {
-    return cudaFuncSetAttribute(reinterpret_cast<const void*>(k_attn<HD, NW, NB>),
-                                cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(attn_smem(NW, NB, HD)));
+    return cudaFuncSetAttribute(reinterpret_cast<const void*>(k_attn<HD, NW, NB, PR>),
+                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>(attn_smem(NW, NB, PR, HD)));
 }
 
 cudaError_t attn_init_attrs() {
-    cudaError_t e = attn_attr<128, 2, 1>();
-    if (e == cudaSuccess) e = attn_attr<128, 2, 2>();
-    if (e == cudaSuccess) e = attn_attr<128, 4, 1>();
-    if (e == cudaSuccess) e = attn_attr<128, 4, 2>();
-    if (e == cudaSuccess) e = attn_attr<64, 2, 1>();
-    if (e == cudaSuccess) e = attn_attr<64, 2, 2>();
-    if (e == cudaSuccess) e = attn_attr<64, 4, 1>();
-    if (e == cudaSuccess) e = attn_attr<64, 4, 2>();
+    cudaError_t e = attn_attr<128, 2, 1, 1>();
+    if (e == cudaSuccess) e = attn_attr<128, 2, 1, 2>();
+    if (e == cudaSuccess) e = attn_attr<128, 2, 2, 1>();
+    if (e == cudaSuccess) e = attn_attr<128, 4, 1, 1>();
+    if (e == cudaSuccess) e = attn_attr<128, 4, 2, 1>();
+    if (e == cudaSuccess) e = attn_attr<64, 2, 1, 1>();
+    if (e == cudaSuccess) e = attn_attr<64, 2, 1, 2>();
+    if (e == cudaSuccess) e = attn_attr<64, 2, 2, 1>();
+    if (e == cudaSuccess) e = attn_attr<64, 4, 1, 1>();
+    if (e == cudaSuccess) e = attn_attr<64, 4, 2, 1>();
     return e;
 }
 
@@ -346,9 +364,18 @@ AttnPlan attn_plan(int B, int T, int H, int max_keys, int sms) {
     // 64-token window is one query tile, so its keys and values are read once
     a.nw = T <= 32 ? 2 : 4;
     a.qtiles = (T + a.nw * 16 - 1) / (a.nw * 16);
-    // key splits (cluster size): about two CTAs per SM, at most one split per sub-block
     const int units = B * H * a.qtiles;
     const int blocks = (max_keys + kAK - 1) / kAK;
+    a.pairs = 1;
+    a.nb = 1;
+    if (a.nw == 2 && blocks >= 2 && units * ((blocks + 1) / 2) <= sms + sms / 4 && (blocks + 1) / 2 <= kMaxCluster) {
+        // few (sequence, head) units and a short prefix: one CTA per about two sub-blocks, its
+        // two warp pairs taking one sub-block each (about one CTA per SM)
+        a.pairs = 2;
+        a.csize = (blocks + 1) / 2;
+        return a;
+    }
+    // key splits (cluster size): about two CTAs per SM, at most one split per sub-block
     int c = (2 * sms) / units;
     if (c > kMaxCluster) c = kMaxCluster;
     if (c > blocks) c = blocks;
@@ -359,23 +386,24 @@ AttnPlan attn_plan(int B, int T, int H, int max_keys, int sms) {
     return a;
 }
 
-template <int HD, int NW, int NB>
+template <int HD, int NW, int NB, int PR>
 static cudaError_t attn_go(cudaLaunchConfig_t& cfg, const __nv_bfloat16* q, const __nv_bfloat16* kc,
                            const __nv_bfloat16* vc, const int* seq_kv, __nv_bfloat16* out, int T, int H, int cap,
                            const AttnPlan& a, unsigned long long* trace) {
-    cfg.dynamicSmemBytes = attn_smem(NW, NB, HD);
-    return cudaLaunchKernelEx(&cfg, k_attn<HD, NW, NB>, q, kc, vc, seq_kv, out, T, H, cap, a.qtiles, a.csize, trace);
+    cfg.blockDim = dim3(PR * NW * 32);
+    cfg.dynamicSmemBytes = attn_smem(NW, NB, PR, HD);
+    return cudaLaunchKernelEx(&cfg, k_attn<HD, NW, NB, PR>, q, kc, vc, seq_kv, out, T, H, cap, a.qtiles, a.csize,
+                              trace);
 }
 
 cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
                              const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int hd, int cap,
                              const AttnPlan& a, cudaStream_t st, bool pdl, unsigned long long* trace) {
     if (a.csize < 1 || a.csize > kMaxCluster || (a.nw != 2 && a.nw != 4) || (a.nb != 1 && a.nb != 2) ||
-        (hd != 64 && hd != 128))
+        (a.pairs != 1 && a.pairs != 2) || (a.pairs == 2 && (a.nw != 2 || a.nb != 1)) || (hd != 64 && hd != 128))
         return cudaErrorInvalidValue;
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3(a.csize, H, B * a.qtiles);
-    cfg.blockDim = dim3(a.nw * 32);
     cfg.stream = st;
     cudaLaunchAttribute at[2];
     int n = 0;
@@ -391,16 +419,19 @@ cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, co
     }
     cfg.attrs = at;
     cfg.numAttrs = n;
+    if (a.pairs == 2)
+        return hd == 128 ? attn_go<128, 2, 1, 2>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace)
+                         : attn_go<64, 2, 1, 2>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
     const int key = (hd == 128 ? 4 : 0) + (a.nw == 4 ? 2 : 0) + (a.nb == 2 ? 1 : 0);
     switch (key) {
-        case 0: return attn_go<64, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
-        case 1: return attn_go<64, 2, 2>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
-        case 2: return attn_go<64, 4, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
-        case 3: return attn_go<64, 4, 2>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
-        case 4: return attn_go<128, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
-        case 5: return attn_go<128, 2, 2>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
-        case 6: return attn_go<128, 4, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
-        default: return attn_go<128, 4, 2>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        case 0: return attn_go<64, 2, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        case 1: return attn_go<64, 2, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        case 2: return attn_go<64, 4, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        case 3: return attn_go<64, 4, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        case 4: return attn_go<128, 2, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        case 5: return attn_go<128, 2, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        case 6: return attn_go<128, 4, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        default: return attn_go<128, 4, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
     }
 }
 
