@@ -59,7 +59,7 @@ Layout make_layout(const dllm_config& c) {
     L.w_o = L.w_qkv + static_cast<size_t>(L.qkv_rows) * d;
     L.w_gu = L.w_o + static_cast<size_t>(L.o_rows) * L.qd;
     L.w_d = L.w_gu + static_cast<size_t>(L.gu_rows) * d;
-    L.per_layer = L.w_d + static_cast<size_t>(L.d_rows) * F;
+    L.per_layer = L.w_d + static_cast<size_t>(L.d_rows) * rup(F, 64);  // tile-major: K padded to 64
     size_t o = 0;
     auto take = [&](size_t bytes) {
         size_t r = o;
@@ -138,8 +138,7 @@ struct dllm_ctx {
     __nv_bfloat16* emb = nullptr;
     __nv_bfloat16* head = nullptr;
     std::vector<__nv_bfloat16*> wl;
-    std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_d;
-    CUtensorMap tm_head{};
+
     __nv_bfloat16* kv = nullptr;
     float* x = nullptr;
     __nv_bfloat16 *xn = nullptr, *q = nullptr, *attn = nullptr, *h = nullptr;
@@ -299,7 +298,7 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
     };
     // phase slot i of a chain uses scratch slot i; consecutive chains are ordered by the stream
     auto add_phase = [&](ChainArgs& ca, ChainMaps& m, const GemmPlan& p, int epi, EpiArgs e, int dep_rows,
-                         const CUtensorMap& w, const CUtensorMap& x) {
+                         const __nv_bfloat16* w_tiles, const CUtensorMap& x) {
         const int i = ca.n_phases++;
         ChainPhase& P = ca.ph[i];
         P.p = p;
@@ -310,7 +309,7 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
         P.partials = ctx->chain_part + static_cast<size_t>(i) * L.part_floats;
         P.tickets = ctx->chain_cnt + static_cast<size_t>(i) * L.cnt_len;
         P.done = ctx->chain_done + static_cast<size_t>(i) * L.done_len;
-        m.w[i] = w;
+        P.w_tiles = w_tiles;
         m.x[i] = x;
     };
     const int smem_budget = (ctx->debug & 8) ? kChainSmemFull : kChainSmemShared;
@@ -326,8 +325,8 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
     };
     {
         ChainArgs ca{};
-        ChainMaps m;
-        add_phase(ca, m, pq, EPI_QKV, qkv_args(0), 0, ctx->tm_qkv[0], tx_xn);
+        ChainMaps m{};
+        add_phase(ca, m, pq, EPI_QKV, qkv_args(0), 0, ctx->wl[0] + L.w_qkv, tx_xn);
         if (int rc = run_chain(ca, m, 1, DLLM_K_QKV)) return rc;
     }
     for (int l = 0; l < c.n_layers; ++l) {
@@ -337,12 +336,13 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
         mark(ctx, DLLM_K_ATTN);
         // output projection (+ residual) -> gate/up (+ SwiGLU) -> down (+ residual) -> next QKV or LM head
         ChainArgs ca{};
-        ChainMaps m;
-        add_phase(ca, m, po, EPI_RESID, er, 0, ctx->tm_o[l], tx_attn);
-        add_phase(ca, m, pg, EPI_SWIGLU, ep, 128, ctx->tm_gu[l], tx_xn);
-        add_phase(ca, m, pd, EPI_RESID, er, 64, ctx->tm_d[l], tx_h);
-        if (l + 1 < c.n_layers) add_phase(ca, m, pq, EPI_QKV, qkv_args(l + 1), 128, ctx->tm_qkv[l + 1], tx_xn);
-        else if (head) add_phase(ca, m, ph, EPI_LMHEAD, eh, 128, ctx->tm_head, tx_xn);
+        ChainMaps m{};
+        const __nv_bfloat16* w = ctx->wl[l];
+        add_phase(ca, m, po, EPI_RESID, er, 0, w + L.w_o, tx_attn);
+        add_phase(ca, m, pg, EPI_SWIGLU, ep, 128, w + L.w_gu, tx_xn);
+        add_phase(ca, m, pd, EPI_RESID, er, 64, w + L.w_d, tx_h);
+        if (l + 1 < c.n_layers) add_phase(ca, m, pq, EPI_QKV, qkv_args(l + 1), 128, ctx->wl[l + 1] + L.w_qkv, tx_xn);
+        else if (head) add_phase(ca, m, ph, EPI_LMHEAD, eh, 128, ctx->head, tx_xn);
         if (int rc = run_chain(ca, m, l + 2, DLLM_K_LAYER)) return rc;
     }
     if (head) {
@@ -512,29 +512,19 @@ int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void*
     // weights from the seed (tensor ids: embedding 1, head 2, layer l: 16 + 8l + {q,k,v,o,gate,up,down})
     const uint64_t seed = c.weight_seed;
     const int hd = c.head_dim;
-    cudaError_t ie = launch_init_weight(ctx->emb, 0, c.vocab, d, c.vocab, seed, 1, qd, hd, s);
-    if (ie == cudaSuccess) ie = launch_init_weight(ctx->head, 0, L.head_rows, d, c.vocab, seed, 2, qd, hd, s);
+    // (the embedding is gathered by rows: row-major; the projections are streamed: tile-major)
+    cudaError_t ie = launch_init_weight(ctx->emb, 0, c.vocab, d, c.vocab, seed, 1, qd, hd, false, s);
+    if (ie == cudaSuccess) ie = launch_init_weight(ctx->head, 0, L.head_rows, d, c.vocab, seed, 2, qd, hd, true, s);
     ctx->wl.resize(c.n_layers);
-    ctx->tm_qkv.resize(c.n_layers);
-    ctx->tm_o.resize(c.n_layers);
-    ctx->tm_gu.resize(c.n_layers);
-    ctx->tm_d.resize(c.n_layers);
     for (int l = 0; l < c.n_layers && ie == cudaSuccess; ++l) {
         __nv_bfloat16* w = reinterpret_cast<__nv_bfloat16*>(A + L.off_w) + static_cast<size_t>(l) * L.per_layer;
         ctx->wl[l] = w;
         const uint64_t t0 = 16 + 8ull * l;
-        ie = launch_init_weight(w + L.w_qkv, 1, L.qkv_rows, d, qd, seed, t0 + 0, qd, hd, s);
-        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_o, 0, L.o_rows, qd, d, seed, t0 + 3, qd, hd, s);
-        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_gu, 2, L.gu_rows, d, F, seed, t0 + 4, qd, hd, s);
-        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_d, 0, L.d_rows, F, d, seed, t0 + 6, qd, hd, s);
-        bool ok = make_tmap_bf16(&ctx->tm_qkv[l], w + L.w_qkv, L.qkv_rows, d, 128) &&
-                  make_tmap_bf16(&ctx->tm_o[l], w + L.w_o, L.o_rows, qd, 128) &&
-                  make_tmap_bf16(&ctx->tm_gu[l], w + L.w_gu, L.gu_rows, d, 128) &&
-                  make_tmap_bf16(&ctx->tm_d[l], w + L.w_d, L.d_rows, F, 128);
-        if (!ok) return bail(DLLM_ECUDA, "tensor map encode failed");
+        ie = launch_init_weight(w + L.w_qkv, 1, L.qkv_rows, d, qd, seed, t0 + 0, qd, hd, true, s);
+        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_o, 0, L.o_rows, qd, d, seed, t0 + 3, qd, hd, true, s);
+        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_gu, 2, L.gu_rows, d, F, seed, t0 + 4, qd, hd, true, s);
+        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_d, 0, L.d_rows, F, d, seed, t0 + 6, qd, hd, true, s);
     }
-    if (ie == cudaSuccess && !make_tmap_bf16(&ctx->tm_head, ctx->head, L.head_rows, d, 128))
-        return bail(DLLM_ECUDA, "tensor map encode failed");
     // RoPE frequencies base^(-2j/hd), in double on the host
     std::vector<float> th(c.head_dim / 2);
     for (int j = 0; j < c.head_dim / 2; ++j)
@@ -930,48 +920,50 @@ int dllm_get_weight(dllm_ctx* ctx, int layer, int which, uint16_t* out, size_t n
     const Layout& L = ctx->L;
     const int d = c.d_model, F = c.ffn, qd = L.qd;
     if (!out) return fail(ctx, DLLM_EINVAL, "null output");
-    auto copy_rows = [&](const __nv_bfloat16* src, int rows, int cols, size_t dst_row0) -> int {
-        CK(cudaMemcpyAsync(out + dst_row0 * cols, src, static_cast<size_t>(rows) * cols * 2, cudaMemcpyDeviceToHost,
-                           ctx->stream));
-        return DLLM_OK;
-    };
     int rc = DLLM_OK;
     if (layer < 0) {
         if (n_elems < static_cast<size_t>(c.vocab) * d) return fail(ctx, DLLM_EINVAL, "buffer too small");
-        if (which == 1) rc = copy_rows(ctx->emb, c.vocab, d, 0);
-        else if (which == 2) rc = copy_rows(ctx->head, c.vocab, d, 0);
-        else return fail(ctx, DLLM_EINVAL, "bad tensor");
-    } else {
-        if (layer >= c.n_layers || which < 0 || which > 6) return fail(ctx, DLLM_EINVAL, "bad tensor");
-        const __nv_bfloat16* w = ctx->wl[layer];
-        int rows = (which <= 2) ? qd : (which == 3 || which == 6) ? d : F;
-        int cols = (which == 3) ? qd : (which == 6) ? F : d;
-        if (n_elems < static_cast<size_t>(rows) * cols) return fail(ctx, DLLM_EINVAL, "buffer too small");
-        if (which == 3) rc = copy_rows(w + L.w_o, d, qd, 0);
-        else if (which == 6) rc = copy_rows(w + L.w_d, d, F, 0);
-        else {
-            // q/k/v rows are interleaved inside each head; gate/up rows alternate in each tile
-            const size_t phys_rows = which <= 2 ? static_cast<size_t>(qd) : static_cast<size_t>(L.gu_rows);
-            const __nv_bfloat16* src = which <= 2 ? w + L.w_qkv + static_cast<size_t>(which) * qd * d : w + L.w_gu;
-            std::vector<uint16_t> phys(phys_rows * d);
-            CK(cudaMemcpyAsync(phys.data(), src, phys.size() * 2, cudaMemcpyDeviceToHost, ctx->stream));
-            rc = sync_check(ctx);
-            if (rc) return rc;
-            const int hd = c.head_dim, half = hd / 2;
-            for (int r = 0; r < rows; ++r) {
-                size_t pr;
-                if (which <= 2) {
-                    const int hh = r / hd, i = r % hd;
-                    pr = static_cast<size_t>(hh) * hd + 2 * (i % half) + i / half;
-                } else {
-                    pr = static_cast<size_t>(r / 64) * 128 + 2 * (r % 64) + (which == 5 ? 1 : 0);
-                }
-                memcpy(out + static_cast<size_t>(r) * cols, phys.data() + pr * d, static_cast<size_t>(d) * 2);
-            }
+        if (which == 1) {  // the embedding is row-major
+            CK(cudaMemcpyAsync(out, ctx->emb, static_cast<size_t>(c.vocab) * d * 2, cudaMemcpyDeviceToHost,
+                               ctx->stream));
+            return sync_check(ctx);
         }
+        if (which != 2) return fail(ctx, DLLM_EINVAL, "bad tensor");
+    } else if (layer >= c.n_layers || which < 0 || which > 6) {
+        return fail(ctx, DLLM_EINVAL, "bad tensor");
     }
+    // a projection: copy its tile-major matrix, then gather the logical rows
+    const int rows = layer < 0 ? c.vocab : (which <= 2) ? qd : (which == 3 || which == 6) ? d : F;
+    const int cols = layer < 0 ? d : (which == 3) ? qd : (which == 6) ? F : d;
+    if (n_elems < static_cast<size_t>(rows) * cols) return fail(ctx, DLLM_EINVAL, "buffer too small");
+    const __nv_bfloat16* src;
+    int phys_rows;
+    if (layer < 0) {
+        src = ctx->head;
+        phys_rows = L.head_rows;
+    } else {
+        const __nv_bfloat16* w = ctx->wl[layer];
+        src = w + (which <= 2 ? L.w_qkv : which == 3 ? L.w_o : which == 6 ? L.w_d : L.w_gu);
+        phys_rows = which <= 2 ? L.qkv_rows : which == 3 ? L.o_rows : which == 6 ? L.d_rows : L.gu_rows;
+    }
+    const int kb = (cols + 63) / 64;
+    std::vector<uint16_t> phys(static_cast<size_t>(phys_rows) * kb * 64);
+    CK(cudaMemcpyAsync(phys.data(), src, phys.size() * 2, cudaMemcpyDeviceToHost, ctx->stream));
+    rc = sync_check(ctx);
     if (rc) return rc;
-    return sync_check(ctx);
+    const int hd = c.head_dim, half = hd / 2;
+    for (int r = 0; r < rows; ++r) {
+        int pr = r;
+        if (layer >= 0 && which <= 2) {  // q/k/v rows are interleaved inside each head
+            const int hh = r / hd, i = r % hd;
+            pr = which * qd + hh * hd + 2 * (i % half) + i / half;
+        } else if (layer >= 0 && (which == 4 || which == 5)) {  // gate/up rows alternate in each tile
+            pr = (r / 64) * 128 + 2 * (r % 64) + (which == 5 ? 1 : 0);
+        }
+        uint16_t* o = out + static_cast<size_t>(r) * cols;
+        for (int col = 0; col < cols; ++col) o[col] = phys[tiled_index(pr, col, kb)];
+    }
+    return DLLM_OK;
 }
 
 int dllm_get_kv(dllm_ctx* ctx, int layer, int which, int seq, int p0, int n, float* out) {

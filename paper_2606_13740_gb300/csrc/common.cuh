@@ -1,8 +1,8 @@
 // Shared device helpers for the sm_103a kernels: inline PTX for mbarrier,
 // TMA (cp.async.bulk.tensor), tcgen05 (UMMA into TMEM), and bounded waits.
 //
-// Every spin in this library is bounded by a wall-clock limit read from
-// %globaltimer; when it runs out the waiter records DLLM_ETIMEOUT in the
+// Every spin in this library is bounded by a limit on the SM's cycle counter
+// (kWaitLimitCycles); when it runs out the waiter records DLLM_ETIMEOUT in the
 // context's device status word and the kernel unwinds instead of hanging.
 #pragma once
 
@@ -15,7 +15,11 @@
 
 namespace dllm {
 
-constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s
+// Spin deadlines count SM cycles: clock64 is a register read that never leaves the SM (the
+// spinning loops of the producers and the MMA issuer re-check it often).  4e9 cycles is 2 s
+// at the maximum SM clock, longer at lower clocks.
+constexpr long long kWaitLimitCycles = 4000000000ll;
+__device__ __forceinline__ long long spin_clock() { return clock64(); }
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -78,16 +82,16 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Wait for the phase with the given parity to complete.  Gives up (returns
-// false) when *abort becomes non-zero or after kWaitLimitNs; on a timeout it
+// false) when *abort becomes non-zero or after kWaitLimitCycles; on a timeout it
 // raises *abort and ORs kStatusTimeout into *status.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort, int* status) {
     if (mbar_try_wait(bar, parity)) return true;
-    unsigned long long t0 = global_ns();
+    const long long t0 = spin_clock();
     for (uint32_t it = 1;; ++it) {
         if (mbar_try_wait(bar, parity)) return true;
         if ((it & 63u) == 0) {
             if (*abort) return false;
-            if (global_ns() - t0 > kWaitLimitNs) {
+            if (spin_clock() - t0 > kWaitLimitCycles) {
                 *abort = 1;
                 if (status) atomicOr(status, kStatusTimeout);
                 return false;
@@ -119,6 +123,16 @@ __device__ __forceinline__ void bulk_load(void* smem_dst, const void* gsrc, uint
                      smem_u32(smem_dst)),
                  "l"(reinterpret_cast<uint64_t>(gsrc)), "r"(bytes), "r"(smem_u32(bar))
                  : "memory");
+}
+
+// The same with an L2 eviction policy (createpolicy) for the source lines.
+__device__ __forceinline__ void bulk_load_hint(void* smem_dst, const void* gsrc, uint32_t bytes, uint64_t* bar,
+                                               uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::
+            "r"(smem_u32(smem_dst)),
+        "l"(reinterpret_cast<uint64_t>(gsrc)), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
+        : "memory");
 }
 
 // Order this thread's earlier generic-proxy view of global memory before its later

@@ -179,6 +179,7 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
 #pragma unroll 1
     for (int g = 0; g < 32 / GW; ++g) {
         if (tr && g == 1) tr[kTrEpiG0] = global_ns();
+
         const int cg = col0 + GW * g;  // first column of the group
         float a[GW];
         tmem_ld_32xn<GW>(t_src + static_cast<uint32_t>(GW * g), a);
@@ -364,6 +365,7 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
 // issuer, warps 2..5 = epilogue.  Ring stages, TMEM accumulators and their barriers are
 // shared by all phases; a running iteration counter gives every stage its use parity.
 constexpr int kChainThreads = 224;
+constexpr int kMaxDepTiles = 256;  // the operand producer keeps a readiness bit per producing tile: 8 per lane
 
 struct ChainEpiState {
     int acc;
@@ -378,10 +380,10 @@ __device__ __forceinline__ int chain_tag(const ChainArgs& ca) {
 // Wait (bounded) until flag == tag.  Returns false after raising *abort on a timeout.
 __device__ __forceinline__ bool wait_flag(const int* flag, int tag, volatile int* abort, int* status) {
     if (ld_acquire(flag) == tag) return true;
-    const unsigned long long t0 = global_ns();
+    const long long t0 = spin_clock();
     while (ld_acquire(flag) != tag) {
         if (*abort) return false;
-        if (global_ns() - t0 > kWaitLimitNs) {
+        if (spin_clock() - t0 > kWaitLimitCycles) {
             *abort = 1;
             atomicOr(status, kStatusTimeout);
             return false;
@@ -645,7 +647,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         mbar_fence_init();
     }
     if (warp == 0 && lane == 0) {
-        for (int ph = 0; ph < ca.n_phases; ++ph) tma_prefetch_desc(&maps.w[ph]);
+        for (int ph = 0; ph < ca.n_phases; ++ph)
+            if (!ca.ph[ph].w_tiles) tma_prefetch_desc(&maps.w[ph]);
     }
     if (warp == 6 && lane == 0) {
         for (int ph = 0; ph < ca.n_phases; ++ph) tma_prefetch_desc(&maps.x[ph]);
@@ -677,21 +680,29 @@ __global__ void __launch_bounds__(kChainThreads, 1)
                 // (m-tile, k-block) walked incrementally: no division in the loop
                 int tile = it0 / p.kb, k = it0 - tile * p.kb;
                 int nt = tile / p.m_tiles, mt = tile - nt * p.m_tiles;
+                const char* wt = reinterpret_cast<const char*>(ca.ph[ph].w_tiles);
+                size_t woff = (static_cast<size_t>(mt) * p.kb + k) * kABytes;  // tile-major: (mt*kb + k) tiles
                 for (int it = it0; it < it1; ++it) {
                     if (!mbar_wait(&empty[stage], par ^ 1u, s_abort, status)) break;
                     mbar_arrive_expect_tx(&full[stage], kABytes + b_bytes);
-                    tma_load_2d(sA + static_cast<size_t>(stage) * kABytes, &maps.w[ph], k * kBK, mt * kBM, &full[stage],
-                                pol_w);
+                    if (wt)
+                        bulk_load_hint(sA + static_cast<size_t>(stage) * kABytes, wt + woff, kABytes, &full[stage],
+                                       pol_w);
+                    else
+                        tma_load_2d(sA + static_cast<size_t>(stage) * kABytes, &maps.w[ph], k * kBK, mt * kBM,
+                                    &full[stage], pol_w);
                     pending |= 1u << stage;
                     pend_par = (pend_par & ~(1u << stage)) | (par << stage);
                     if (++stage == S) {
                         stage = 0;
                         par ^= 1u;
                     }
+                    woff += kABytes;
                     if (++k == p.kb) {
                         k = 0;
                         if (++mt == p.m_tiles) {
                             mt = 0;
+                            woff = 0;
                             ++nt;
                         }
                     }
@@ -700,10 +711,10 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             if (*s_abort) {
                 // let the copies in flight land before the CTA's shared memory is released (a
                 // stage whose operand was never issued does not complete: one deadline for all)
-                const unsigned long long t0 = global_ns();
+                const long long t0 = spin_clock();
                 for (int s = 0; s < S; ++s) {
                     if (!(pending >> s & 1u)) continue;
-                    while (!mbar_try_wait(&full[s], (pend_par >> s) & 1u) && global_ns() - t0 < kWaitLimitNs) {
+                    while (!mbar_try_wait(&full[s], (pend_par >> s) & 1u) && spin_clock() - t0 < kWaitLimitCycles) {
                     }
                 }
             }
@@ -726,8 +737,10 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             const int it1 = static_cast<int>(range_begin(blockIdx.x + 1, p.total, p.grid));
             const int* dep = (ph > 0 && P.dep_rows > 0) ? ca.ph[ph - 1].done : nullptr;
             const int dep_tiles = dep ? ca.ph[ph - 1].p.m_tiles : 0;
-            int win_base = -1, win_nt = -1;  // the 32 producing tiles last polled
-            uint32_t win_ready = 0;
+            // completion of the previous phase's tiles for token tile mine_nt, as far as seen:
+            // lane l, bit w = tile 32w + l (a flag, once complete, stays so for the launch)
+            uint32_t mine = 0;
+            int mine_nt = -1;
             int tile = it0 / p.kb, k = it0 - tile * p.kb;
             int nt = tile / p.m_tiles, mt = tile - nt * p.m_tiles;
             for (int it = it0; it < it1; ++it) {
@@ -739,32 +752,38 @@ __global__ void __launch_bounds__(kChainThreads, 1)
                 }
                 if (dep) {
                     const int pmt = (k * kBK) / P.dep_rows;
-                    if (nt != win_nt || pmt < win_base || pmt >= win_base + 32) {
-                        win_base = pmt;
-                        win_nt = nt;
-                        win_ready = 0;
+                    if (nt != mine_nt) {
+                        mine = 0;
+                        mine_nt = nt;
                     }
-                    const unsigned long long t0 = global_ns();
-                    while (!(win_ready >> (pmt - win_base) & 1u)) {
-                        const int i = win_base + lane;
-                        const bool ok = i >= dep_tiles || ld_acquire(dep + i * p.n_tiles + nt) == tag;
-                        win_ready = __ballot_sync(0xffffffffu, ok);
-                        if (win_ready >> (pmt - win_base) & 1u) {
-                            fence_proxy_async_global();  // generic-proxy writes of other CTAs -> these TMA reads
-                            break;
-                        }
-                        int give_up = 0;
-                        if (lane == 0) give_up = (*s_abort || global_ns() - t0 > kWaitLimitNs) ? 1 : 0;
-                        if (__shfl_sync(0xffffffffu, give_up, 0)) {  // warp-uniform decision
-                            if (lane == 0 && !*s_abort) {
-                                *s_abort = 1;
-                                atomicOr(status, kStatusTimeout);
+                    if (!(__shfl_sync(0xffffffffu, mine, pmt & 31) >> (pmt >> 5) & 1u)) {
+                        // poll the 32 producing tiles around pmt (one acquire load per lane) until
+                        // pmt is complete; what is seen complete is kept for the later k-blocks
+                        const int w = pmt >> 5;
+                        const long long t0 = spin_clock();
+                        for (;;) {
+                            const int i = w * 32 + lane;
+                            const bool ok = i >= dep_tiles || ld_acquire(dep + i * p.n_tiles + nt) == tag;
+                            const uint32_t seen = __ballot_sync(0xffffffffu, ok);
+                            mine |= ((seen >> lane) & 1u) << w;
+                            if (seen >> (pmt & 31) & 1u) {
+                                fence_proxy_async_global();  // generic-proxy writes of other CTAs -> these TMA reads
+                                break;
                             }
-                            stop = true;
-                            break;
+                            int give_up = 0;
+                            if (lane == 0) give_up = (*s_abort || spin_clock() - t0 > kWaitLimitCycles) ? 1 : 0;
+                            if (__shfl_sync(0xffffffffu, give_up, 0)) {  // warp-uniform decision
+                                if (lane == 0 && !*s_abort) {
+                                    *s_abort = 1;
+                                    atomicOr(status, kStatusTimeout);
+                                }
+                                stop = true;
+                                break;
+                            }
+                            __nanosleep(32);
                         }
+                        if (stop) break;
                     }
-                    if (stop) break;
                 }
                 if (lane == 0)
                     tma_load_2d(sB + static_cast<size_t>(stage) * b_bytes, &maps.x[ph], k * kBK, nt * ca.ntile,
@@ -841,8 +860,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             }
             if (*s_abort && issued) {
                 umma_commit(drain);
-                const unsigned long long t0 = global_ns();
-                while (!mbar_try_wait(drain, 0) && global_ns() - t0 < kWaitLimitNs) {
+                const long long t0 = spin_clock();
+                while (!mbar_try_wait(drain, 0) && spin_clock() - t0 < kWaitLimitCycles) {
                 }
             }
         }
@@ -977,6 +996,8 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
         if (p.ntile != ntile || p.N != ca.ph[0].p.N) return false;
         grid = grid > p.grid ? grid : p.grid;
     }
+    for (int i = 1; i < ca.n_phases; ++i)
+        if (ca.ph[i].dep_rows > 0 && ca.ph[i - 1].p.m_tiles > kMaxDepTiles) return false;
     const bool c32 = ntile == 32;
     // wider token tiles are tensor-bound: the deepest ring (the attention CTAs' room matters
     // only to the batch-1 weight stream)

@@ -15,6 +15,19 @@ constexpr int kMaxBlock = 4096;
 constexpr int kStatusTimeout = 1;  // device status word bits
 constexpr int kStatusBadIndex = 2;  // longest current block the commit pass handles
 
+// ---------------------------------------------------------------- weight storage
+// The context's projection weights are stored tile-major: the 128-row x 64-column tile
+// (m-tile r/128, k-block c/64) of a [rows][K] matrix is 16 KB at ((r/128)*kb + c/64)*8192
+// elements (kb = ceil(K/64), columns past K zero), row r%128 of the tile 64 elements long,
+// and the 16-byte chunk (c%64)/8 of that row placed at chunk ((c%64)/8) ^ (r%8).  That is the
+// 128-byte-swizzled K-major image the UMMA shared-memory descriptor reads, so a tile moves
+// from HBM to shared memory as one contiguous copy (long DRAM bursts instead of 128 rows of
+// 128 bytes).
+__host__ __device__ inline size_t tiled_index(int r, int c, int kb) {
+    return (static_cast<size_t>(r >> 7) * kb + (c >> 6)) * 8192 + static_cast<size_t>(r & 127) * 64 +
+           ((((c & 63) >> 3) ^ (r & 7)) << 3) + (c & 7);
+}
+
 // ---------------------------------------------------------------- GEMM
 // D = W * X^T on tensor cores: W bf16 [M][K] (weights, rows padded to 128),
 // X bf16 [N][K] (tokens).  Row m of D is an output feature, column n a token.
@@ -85,6 +98,9 @@ struct ChainPhase {
     int* done;           // [m_tiles][n_tiles] completion flags (value: the launch's tag); may be null
     float* partials;     // [grid][ntile*128] split partials (a CTA contributes to at most one tile per phase)
     int* tickets;        // [m_tiles*n_tiles][32], zero between launches
+    // non-null: the weights are stored tile-major (tiled_index) and each 16 KB tile arrives with
+    // one contiguous bulk copy; null: row-major [M][K] through the chain's tensor map
+    const __nv_bfloat16* w_tiles;
 };
 struct ChainArgs {
     int n_phases;
@@ -142,8 +158,10 @@ inline cudaError_t launch_k(void (*k)(KArgs...), dim3 grid, dim3 block, size_t s
 }
 
 // ---------------------------------------------------------------- other kernels
+// Seeded weights (rows_phys x cols, see k_init_weight for the row orders), stored tile-major
+// (tiled_index; rows_phys a multiple of 128) when `tiled`, else row-major.
 cudaError_t launch_init_weight(__nv_bfloat16* dst, int mode, int rows_phys, int cols, int logical_rows,
-                               uint64_t seed, uint64_t tid0, int qd, int hd, cudaStream_t st);
+                               uint64_t seed, uint64_t tid0, int qd, int hd, bool tiled, cudaStream_t st);
 cudaError_t launch_init_kv_random(__nv_bfloat16* cache, int B, int H, int hd, int cap, int P, int layer,
                                   int which, int L, uint64_t seed, cudaStream_t st);
 // x = embedding rows of the window's ids (fp32), xb = bf16(x), sq[d/128][N] = per-128-feature

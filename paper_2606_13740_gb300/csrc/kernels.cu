@@ -38,13 +38,29 @@ __device__ __forceinline__ float gen_value(uint64_t key, uint64_t i, double sigm
 //         j + hd/2 (the rotate-half RoPE pair sits in adjacent TMEM lanes);
 // mode 2: fused gate/up: 128-row tile k, physical row 2f = gate row 64k+f (tensor tid0),
 //         row 2f+1 = up row 64k+f (tensor tid0+1); zero past logical_rows.
+// Storage: row-major, or tile-major (tiled_index) when tiled; the loop walks the destination in
+// storage order.
 __global__ void k_init_weight(__nv_bfloat16* dst, int mode, int rows, int cols, int logical_rows, uint64_t seed,
-                              uint64_t tid0, int qd, int hd) {
-    const size_t n = static_cast<size_t>(rows) * cols;
+                              uint64_t tid0, int qd, int hd, int tiled) {
+    const int kb = (cols + 63) / 64;
+    const size_t n = tiled ? static_cast<size_t>(rows) * kb * 64 : static_cast<size_t>(rows) * cols;
     for (size_t e = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; e < n;
          e += static_cast<size_t>(gridDim.x) * blockDim.x) {
-        int r = static_cast<int>(e / cols);
-        int c = static_cast<int>(e - static_cast<size_t>(r) * cols);
+        int r, c;
+        if (tiled) {
+            const size_t tile = e >> 13;
+            const int w = static_cast<int>(e & 8191), rr = w >> 6;
+            const int mt = static_cast<int>(tile / kb), kt = static_cast<int>(tile - static_cast<size_t>(mt) * kb);
+            r = mt * 128 + rr;
+            c = kt * 64 + ((((w & 63) >> 3) ^ (rr & 7)) << 3) + (w & 7);
+            if (c >= cols) {
+                dst[e] = __float2bfloat16_rn(0.0f);
+                continue;
+            }
+        } else {
+            r = static_cast<int>(e / cols);
+            c = static_cast<int>(e - static_cast<size_t>(r) * cols);
+        }
         uint64_t tid = tid0;
         int lr = r;
         if (mode == 1) {
@@ -68,10 +84,12 @@ __global__ void k_init_weight(__nv_bfloat16* dst, int mode, int rows, int cols, 
 }
 
 cudaError_t launch_init_weight(__nv_bfloat16* dst, int mode, int rows_phys, int cols, int logical_rows,
-                               uint64_t seed, uint64_t tid0, int qd, int hd, cudaStream_t st) {
-    size_t n = static_cast<size_t>(rows_phys) * cols;
+                               uint64_t seed, uint64_t tid0, int qd, int hd, bool tiled, cudaStream_t st) {
+    if (tiled && (rows_phys & 127)) return cudaErrorInvalidValue;
+    size_t n = static_cast<size_t>(rows_phys) * (tiled ? (cols + 63) / 64 * 64 : cols);
     int blocks = static_cast<int>((n + 255) / 256 < 65536 ? (n + 255) / 256 : 65536);
-    k_init_weight<<<blocks, 256, 0, st>>>(dst, mode, rows_phys, cols, logical_rows, seed, tid0, qd, hd);
+    k_init_weight<<<blocks, 256, 0, st>>>(dst, mode, rows_phys, cols, logical_rows, seed, tid0, qd, hd,
+                                          tiled ? 1 : 0);
     return cudaGetLastError();
 }
 
