@@ -177,7 +177,8 @@ cudaError_t launch_embed(const int* tok, int tok_ld, const int* seq_kv, const __
 // so the merge needs no global scratch, no fences and no atomics.
 constexpr int kMaxCluster = 8;
 // attention timeline slots (%globaltimer ns)
-enum { kAtStart = 0, kAtDepWait = 1, kAtLoop = 2, kAtTicket = 3, kAtMerged = 4, kAtSm = 5, kAtLast = 6 };
+enum { kAtStart = 0, kAtDepWait = 1, kAtLoop = 2, kAtTicket = 3, kAtMerged = 4, kAtSm = 5, kAtLast = 6,
+       kAtMergeLoop = 7 };
 
 __device__ __forceinline__ unsigned smid_attn() {
     unsigned r;
@@ -195,17 +196,18 @@ __device__ __forceinline__ uint32_t dsmem_map(uint32_t saddr, uint32_t rank) {
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
     return r;
 }
+// (no memory clobber: used only between cluster barriers, so the loads may be scheduled
+// together)
 __device__ __forceinline__ float2 dsmem_ld2(uint32_t addr) {
     float2 v;
-    asm volatile("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(addr) : "memory");
+    asm volatile("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(addr));
     return v;
 }
 __device__ __forceinline__ float4 dsmem_ld4(uint32_t addr) {
     float4 v;
     asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
                  : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-                 : "r"(addr)
-                 : "memory");
+                 : "r"(addr));
     return v;
 }
 
@@ -276,77 +278,131 @@ __global__ void __launch_bounds__(PR * NW * 32) k_attn(const __nv_bfloat16* __re
 
     const int r0 = warp * 16 + g, r1 = r0 + 8;
     const int qd = H * HD;
-    if (csize == 1 && PR == 1) {
-        const float i0 = 1.0f / l0, i1 = 1.0f / l1;
+    if constexpr (PR == 2) {
+        // the two groups hold the same rows and columns of the tile (same warp, same lane):
+        // group 1 hands its partial over through its own, finished, shared memory and group 0
+        // merges it in registers, so the cluster sees one partial per CTA
+        float* x = reinterpret_cast<float*>(smem_attn + PART);  // [DN*4 + 4][NT], conflict-free
+        if (grp == 1) {
 #pragma unroll
-        for (int dn = 0; dn < DN; ++dn) {
-            const int col = h * HD + dn * 8 + 2 * c4;
-            if (r0 < nq)
-                *reinterpret_cast<__nv_bfloat162*>(out + (static_cast<size_t>(b) * T + q0 + r0) * qd + col) =
-                    __floats2bfloat162_rn(o[dn][0] * i0, o[dn][1] * i0);
-            if (r1 < nq)
-                *reinterpret_cast<__nv_bfloat162*>(out + (static_cast<size_t>(b) * T + q0 + r1) * qd + col) =
-                    __floats2bfloat162_rn(o[dn][2] * i1, o[dn][3] * i1);
+            for (int dn = 0; dn < DN; ++dn)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) x[(dn * 4 + j) * NT + tid] = o[dn][j];
+            x[(DN * 4 + 0) * NT + tid] = m0;
+            x[(DN * 4 + 1) * NT + tid] = m1;
+            x[(DN * 4 + 2) * NT + tid] = l0;
+            x[(DN * 4 + 3) * NT + tid] = l1;
+        }
+        __syncthreads();
+        if (grp == 0) {
+            const float n0 = x[(DN * 4 + 0) * NT + tid], n1 = x[(DN * 4 + 1) * NT + tid];
+            const float k0 = x[(DN * 4 + 2) * NT + tid], k1 = x[(DN * 4 + 3) * NT + tid];
+            const float M0 = fmaxf(m0, n0), M1 = fmaxf(m1, n1);
+            const float s0 = M0 == -INFINITY ? 0.0f : M0, s1 = M1 == -INFINITY ? 0.0f : M1;
+            const float a0 = exp2f(m0 - s0), b0 = exp2f(n0 - s0), a1 = exp2f(m1 - s1), b1 = exp2f(n1 - s1);
+#pragma unroll
+            for (int dn = 0; dn < DN; ++dn) {
+                o[dn][0] = a0 * o[dn][0] + b0 * x[(dn * 4 + 0) * NT + tid];
+                o[dn][1] = a0 * o[dn][1] + b0 * x[(dn * 4 + 1) * NT + tid];
+                o[dn][2] = a1 * o[dn][2] + b1 * x[(dn * 4 + 2) * NT + tid];
+                o[dn][3] = a1 * o[dn][3] + b1 * x[(dn * 4 + 3) * NT + tid];
+            }
+            l0 = a0 * l0 + b0 * k0;
+            l1 = a1 * l1 + b1 * k1;
+            m0 = M0;
+            m1 = M1;
+        }
+    }
+    if (csize == 1) {
+        if (grp == 0) {
+            const float i0 = 1.0f / l0, i1 = 1.0f / l1;
+#pragma unroll
+            for (int dn = 0; dn < DN; ++dn) {
+                const int col = h * HD + dn * 8 + 2 * c4;
+                if (r0 < nq)
+                    *reinterpret_cast<__nv_bfloat162*>(out + (static_cast<size_t>(b) * T + q0 + r0) * qd + col) =
+                        __floats2bfloat162_rn(o[dn][0] * i0, o[dn][1] * i0);
+                if (r1 < nq)
+                    *reinterpret_cast<__nv_bfloat162*>(out + (static_cast<size_t>(b) * T + q0 + r1) * qd + col) =
+                        __floats2bfloat162_rn(o[dn][2] * i1, o[dn][3] * i1);
+            }
         }
         return;
     }
-    // each group's partial into its own shared memory (its Q/K/V tiles are no longer needed)
-    float* sO = reinterpret_cast<float*>(smem_attn + grp * PART);  // [AQ][HD]
-    float* sML = sO + AQ * HD;                                      // [AQ][2]
+    // the CTA's partial into the first group's shared memory (its Q/K/V tiles are done)
+    float* sO = reinterpret_cast<float*>(smem_attn);  // [AQ][HD]
+    float* sML = sO + AQ * HD;                        // [AQ][2]
+    if (grp == 0) {
 #pragma unroll
-    for (int dn = 0; dn < DN; ++dn) {
-        const int col = dn * 8 + 2 * c4;
-        *reinterpret_cast<float2*>(sO + r0 * HD + col) = make_float2(o[dn][0], o[dn][1]);
-        *reinterpret_cast<float2*>(sO + r1 * HD + col) = make_float2(o[dn][2], o[dn][3]);
-    }
-    if (c4 == 0) {
-        *reinterpret_cast<float2*>(sML + r0 * 2) = make_float2(m0, l0);
-        *reinterpret_cast<float2*>(sML + r1 * 2) = make_float2(m1, l1);
-    }
-    cluster_sync_all();  // every split's partials are in place
-    if (tr) tr[kAtTicket] = global_ns();
-    // this CTA merges output elements split*PR*NT + tid (+ k * csize * PR * NT): row r, 4
-    // features, over the csize * PR partials (CTA c, group p) in that order
-    constexpr int V4 = HD / 4;
-    constexpr int MP = kMaxCluster * PR;
-    const int all = threadIdx.x;
-    for (int e = split * PR * NT + all; e < nq * V4; e += csize * PR * NT) {
-        const int r = e / V4, i4 = e - r * V4;
-        float2 ml[MP];
-        float4 ov[MP];
-#pragma unroll
-        for (int c = 0; c < kMaxCluster; ++c) {
-#pragma unroll
-            for (int p = 0; p < PR; ++p) {
-                if (c < csize) {
-                    const float* po = reinterpret_cast<const float*>(smem_attn + p * PART);
-                    ml[c * PR + p] = dsmem_ld2(dsmem_map(smem_u32(po + AQ * HD + r * 2), c));
-                    ov[c * PR + p] = dsmem_ld4(dsmem_map(smem_u32(po + r * HD + i4 * 4), c));
-                }
-            }
+        for (int dn = 0; dn < DN; ++dn) {
+            const int col = dn * 8 + 2 * c4;
+            *reinterpret_cast<float2*>(sO + r0 * HD + col) = make_float2(o[dn][0], o[dn][1]);
+            *reinterpret_cast<float2*>(sO + r1 * HD + col) = make_float2(o[dn][2], o[dn][3]);
         }
-        float M = -INFINITY;
+        if (c4 == 0) {
+            *reinterpret_cast<float2*>(sML + r0 * 2) = make_float2(m0, l0);
+            *reinterpret_cast<float2*>(sML + r1 * 2) = make_float2(m1, l1);
+        }
+    }
+    cluster_sync_all();  // every split's partial is in place
+    if (tr) tr[kAtTicket] = global_ns();
+    // This CTA merges output elements e = split * NTT + threadIdx.x (+ k * csize * NTT): row
+    // e / V4, features 4 (e % V4) .. +3, over the csize partials in CTA order.  A row is one
+    // aligned segment of V4 lanes; lane k of the segment reads partial k's (max, sum) and the
+    // merge weights are shared by shuffles, so each partial's statistics cross the cluster once.
+    constexpr int V4 = HD / 4;
+    constexpr int NTT = PR * NT;
+    const int ln = threadIdx.x & 31;
+    const int seg0 = ln & ~(V4 - 1);
+    uint32_t pb[kMaxCluster];
 #pragma unroll
-        for (int k = 0; k < MP; ++k)
-            if (k < csize * PR) M = fmaxf(M, ml[k].x);
-        float L = 0.0f;
+    for (int c = 0; c < kMaxCluster; ++c) pb[c] = c < csize ? dsmem_map(smem_u32(sO), c) : 0u;
+    const int nel = nq * V4;
+    // all lanes of a warp take the same passes (the shuffles); lanes past the end work on a
+    // clamped row and store nothing
+    for (int ew0 = split * NTT + (threadIdx.x & ~31); ew0 < nel; ew0 += csize * NTT) {
+        const int e = ew0 + ln;
+        const int r = min(e / V4, AQ - 1), i4 = e % V4;
+        float mk = -INFINITY, lk = 0.0f;
+        if (i4 < csize) {
+            const float2 v = dsmem_ld2(dsmem_map(smem_u32(sML + r * 2), static_cast<uint32_t>(i4)));
+            mk = v.x;
+            lk = v.y;
+        }
+        float4 ov[kMaxCluster];
+#pragma unroll
+        for (int c = 0; c < kMaxCluster; ++c)
+            if (c < csize) ov[c] = dsmem_ld4(pb[c] + static_cast<uint32_t>((r * HD + i4 * 4) * 4));
+        float M = mk;  // over the first 8 lanes of the segment (csize <= 8)
+        M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 1));
+        M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 2));
+        M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 4));
+        M = __shfl_sync(0xffffffffu, M, seg0);
+        const float wk = mk == -INFINITY ? 0.0f : exp2f(mk - M);  // a share without keys: 0
+        float L = wk * lk;
+        L += __shfl_xor_sync(0xffffffffu, L, 1);
+        L += __shfl_xor_sync(0xffffffffu, L, 2);
+        L += __shfl_xor_sync(0xffffffffu, L, 4);
+        L = __shfl_sync(0xffffffffu, L, seg0);
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-        for (int k = 0; k < MP; ++k) {
-            if (k < csize * PR) {
-                const float w = ml[k].x == -INFINITY ? 0.0f : exp2f(ml[k].x - M);  // a share without keys: 0
-                L += w * ml[k].y;
-                acc.x += w * ov[k].x;
-                acc.y += w * ov[k].y;
-                acc.z += w * ov[k].z;
-                acc.w += w * ov[k].w;
+        for (int c = 0; c < kMaxCluster; ++c) {
+            if (c < csize) {
+                const float w = __shfl_sync(0xffffffffu, wk, seg0 + c);
+                acc.x += w * ov[c].x;
+                acc.y += w * ov[c].y;
+                acc.z += w * ov[c].z;
+                acc.w += w * ov[c].w;
             }
         }
-        const float inv = 1.0f / L;
-        __nv_bfloat16* op = out + (static_cast<size_t>(b) * T + q0 + r) * qd + h * HD + i4 * 4;
-        *reinterpret_cast<__nv_bfloat162*>(op) = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
-        *reinterpret_cast<__nv_bfloat162*>(op + 2) = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
+        if (e < nel) {
+            const float inv = 1.0f / L;
+            __nv_bfloat16* op = out + (static_cast<size_t>(b) * T + q0 + r) * qd + h * HD + i4 * 4;
+            *reinterpret_cast<__nv_bfloat162*>(op) = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
+            *reinterpret_cast<__nv_bfloat162*>(op + 2) = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
+        }
     }
+    if (tr) tr[kAtMergeLoop] = global_ns();
     cluster_sync_all();  // no CTA leaves while its partials may still be read
     if (tr) tr[kAtMerged] = global_ns();
 }
