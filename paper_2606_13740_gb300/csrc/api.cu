@@ -94,7 +94,7 @@ Layout make_layout(const dllm_config& c) {
     L.done_len = mt_max * ((L.max_tok + 255) / 256 + 1);
     L.cnt_len = L.done_len * 32;
     L.off_cnt = take(static_cast<size_t>(L.cnt_len) * 4 * kMaxPhases);
-    L.off_done = take(static_cast<size_t>(L.done_len) * 4 * kMaxPhases);
+    L.off_done = take(static_cast<size_t>(L.done_len) * 4 * kMaxPhases * 2);  // done, then done2 slots
     L.off_epoch = take(256);
     const size_t S = static_cast<size_t>(c.max_batch) * c.max_ctx;
     L.off_tok = take(S * 4);
@@ -309,6 +309,7 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
         P.partials = ctx->chain_part + static_cast<size_t>(i) * L.part_floats;
         P.tickets = ctx->chain_cnt + static_cast<size_t>(i) * L.cnt_len;
         P.done = ctx->chain_done + static_cast<size_t>(i) * L.done_len;
+        P.done2 = epi == EPI_RESID ? ctx->chain_done + static_cast<size_t>(kMaxPhases + i) * L.done_len : nullptr;
         P.w_tiles = w_tiles;
         m.x[i] = x;
     };

@@ -138,7 +138,10 @@ __device__ __forceinline__ void warp_reduce_scatter(float* v, int lane) {
 // waits on a store.  Inside a group every step runs over the 8 columns side by side with no
 // branch between them (stores are predicated), so their dependent chains (shuffles, special
 // functions) overlap.
-template <int EPI>
+// Residual epilogue in two passes (PASS 1: the bf16 copy, the next projection's operand, and
+// the RMSNorm partial sums; PASS 2: the fp32 residual and the sums' store), so the tile can be
+// published to the next phase's operand producer between them; PASS 0: both at once.
+template <int EPI, int PASS = 0>
 __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& p, int mt, int col0, int c_in,
                                              int rt, uint32_t t_src, uint32_t t_x, const EpiSmem& sm, int ew,
                                              int quarter, int lane, int* status) {
@@ -207,12 +210,14 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                 ss[u] = ok ? xo[u] * xo[u] : 0.0f;
                 if (ok) {
                     const size_t o = static_cast<size_t>(cg + u) * ep.ld_out + row;
-                    ep.out[o] = xo[u];
-                    ep.xb[o] = __float2bfloat16_rn(xo[u]);
+                    if constexpr (PASS != 1) ep.out[o] = xo[u];
+                    if constexpr (PASS != 2) ep.xb[o] = __float2bfloat16_rn(xo[u]);
                 }
             }
-            warp_reduce_scatter<GW>(ss, lane);
-            if (lane % LS == 0) sm.red[quarter * 32 + GW * g + lane / LS] = ss[0];
+            if constexpr (PASS != 2) {
+                warp_reduce_scatter<GW>(ss, lane);
+                if (lane % LS == 0) sm.red[(c_in / 32) * 128 + quarter * 32 + GW * g + lane / LS] = ss[0];
+            }
         } else if constexpr (EPI == EPI_QKV) {
             // positions and rotations of the group's 8 columns first (the rare tile that spans
             // sequences takes the out-of-line sincos per column), then the branch-free column pass
@@ -310,13 +315,13 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
         }
     }
     if (tr) tr[kTrEpiLoop] = global_ns();
-    if constexpr (EPI == EPI_RESID) {
+    if constexpr (EPI == EPI_RESID && PASS != 1) {
         named_bar(1, 128);
         if (ew == 0) {
             const int col = col0 + lane;
+            const float* rd = sm.red + (c_in / 32) * 128;
             if (col < p.N)
-                ep.sq_out[static_cast<size_t>(mt) * p.N + col] =
-                    ((sm.red[lane] + sm.red[32 + lane]) + sm.red[64 + lane]) + sm.red[96 + lane];
+                ep.sq_out[static_cast<size_t>(mt) * p.N + col] = ((rd[lane] + rd[32 + lane]) + rd[64 + lane]) + rd[96 + lane];
         }
         named_bar(1, 128);
     } else if constexpr (EPI == EPI_LMHEAD) {
@@ -419,10 +424,11 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
     // every tile of the previous phase: its RMSNorm statistics and residual rows are read here
     if (ph > 0 && ca.ph[ph - 1].done) {
         const ChainPhase& Q = ca.ph[ph - 1];
+        const int* qdone = Q.done2 ? Q.done2 : Q.done;  // the residual phases finish their tiles in two steps
         if (ew == 0) {
             const int n = Q.p.m_tiles * Q.p.n_tiles;
             for (int i = lane; i < n; i += 32)
-                if (!wait_flag(Q.done + i, tag, s_abort, status)) break;
+                if (!wait_flag(qdone + i, tag, s_abort, status)) break;
         }
         if (named_bar_any(1, 128, *s_abort != 0)) return;
     }
@@ -433,6 +439,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         named_bar(1, 128);
     }
     const int nchunks = p.ntile / 32;
+    constexpr int kPass1 = EPI == EPI_RESID ? 1 : 0;  // the residual epilogue runs in two passes
     const size_t slot_floats = static_cast<size_t>(p.ntile) * kBM;
     // TMEM: two accumulators of acc_cols columns, then (token tiles up to 128) the staged old
     // residual of the finisher's tile, x_cols columns
@@ -512,8 +519,9 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         if (whole) {
             // the compact epilogue per 32-column chunk, straight from the accumulator in TMEM
             for (int c = 0; c < nchunks; ++c)
-                epilogue_c32<EPI>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt, t_acc + static_cast<uint32_t>(c * 32),
-                                  t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, esm, ew, quarter, lane, status);
+                epilogue_c32<EPI, kPass1>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt,
+                                          t_acc + static_cast<uint32_t>(c * 32),
+                                          t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, esm, ew, quarter, lane, status);
         } else if (!reducer) {
             float* my_part = P.partials + static_cast<size_t>(blockIdx.x) * slot_floats;
             for (int c = 0; c < nchunks; ++c) {
@@ -582,17 +590,30 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                 if (tr && threadIdx.x == 64 && c == 0) tr[kTrReduced] = global_ns();
                 // the sum goes back into the (still owned) accumulator, then the compact epilogue
                 tmem_st_32x32(t_acc + static_cast<uint32_t>(c * 32), v);
-                epilogue_c32<EPI>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt, t_acc + static_cast<uint32_t>(c * 32),
-                                  t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, esm, ew, quarter, lane, status);
+                epilogue_c32<EPI, kPass1>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt,
+                                          t_acc + static_cast<uint32_t>(c * 32),
+                                          t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, esm, ew, quarter, lane, status);
+            }
+        }
+        if (finisher && P.done) {  // publish the finished tile to the next phase's operand producer
+            named_bar(1, 128);
+            if (threadIdx.x == 64) st_release(&P.done[mt * p.n_tiles + nt], tag);
+        }
+        if constexpr (EPI == EPI_RESID) {
+            if (finisher) {  // then the fp32 residual and the RMSNorm sums, for the later phases' epilogues
+                for (int c = 0; c < nchunks; ++c)
+                    epilogue_c32<EPI, 2>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt,
+                                         t_acc + static_cast<uint32_t>(c * 32),
+                                         t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, esm, ew, quarter, lane, status);
+                if (P.done2) {
+                    named_bar(1, 128);
+                    if (threadIdx.x == 64) st_release(&P.done2[mt * p.n_tiles + nt], tag);
+                }
             }
         }
         if (finisher) {
             tc_fence_before();
             mbar_arrive(&tempty[es.acc]);
-        }
-        if (finisher && P.done) {  // publish the finished tile to the next phase's operand producer
-            named_bar(1, 128);
-            if (threadIdx.x == 64) st_release(&P.done[mt * p.n_tiles + nt], tag);
         }
         if (++es.acc == 2) {
             es.acc = 0;

@@ -96,6 +96,9 @@ struct ChainPhase {
     int epi;             // EpiKind
     int dep_rows;        // X k-block k comes from tile (64k)/dep_rows of the previous phase; 0: ready at launch
     int* done;           // [m_tiles][n_tiles] completion flags (value: the launch's tag); may be null
+    // residual phases: done = the bf16 operand is written, done2 = also the fp32 residual and
+    // the RMSNorm sums (what the later phases' epilogues read); null: done covers both
+    int* done2;
     float* partials;     // [grid][ntile*128] split partials (a CTA contributes to at most one tile per phase)
     int* tickets;        // [m_tiles*n_tiles][32], zero between launches
     // non-null: the weights are stored tile-major (tiled_index) and each 16 KB tile arrives with
