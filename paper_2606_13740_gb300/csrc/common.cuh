@@ -140,6 +140,10 @@ __device__ __forceinline__ void bulk_load_hint(void* smem_dst, const void* gsrc,
 __device__ __forceinline__ void fence_proxy_async_global() {
     asm volatile("fence.proxy.async.global;" ::: "memory");
 }
+// The same for this CTA's shared memory (generic accesses -> later bulk copies into it).
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
 
 __device__ __forceinline__ uint64_t policy_evict_first() {
     uint64_t p;

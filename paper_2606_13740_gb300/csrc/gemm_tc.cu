@@ -73,6 +73,7 @@ struct EpiSmem {
     float* red;   // [4][256] cross-warp / quarter partial sums
     int* kvs;     // [256] per-sequence first window position (QKV); current ids of the token tile (LM head)
     float* theta; // [128] rotation frequency of each tile row's feature pair (QKV)
+    uint8_t* stg; // staging of a 32-token chunk's residual outputs (the partial staging memory, free by then)
 };
 
 // RMSNorm scale of every column of token tile nt: rs[c] = rsqrt(sum_t sq[t][col] / dim + eps).
@@ -208,10 +209,16 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                 const bool ok = row < p.M && cg + u < p.N;
                 xo[u] += a[u];
                 ss[u] = ok ? xo[u] * xo[u] : 0.0f;
-                if (ok) {
-                    const size_t o = static_cast<size_t>(cg + u) * ep.ld_out + row;
-                    if constexpr (PASS != 1) ep.out[o] = xo[u];
-                    if constexpr (PASS != 2) ep.xb[o] = __float2bfloat16_rn(xo[u]);
+                if constexpr (PASS == 0) {
+                    if (ok) {
+                        const size_t o = static_cast<size_t>(cg + u) * ep.ld_out + row;
+                        ep.out[o] = xo[u];
+                        ep.xb[o] = __float2bfloat16_rn(xo[u]);
+                    }
+                } else if constexpr (PASS == 1) {  // token-major staging, stored below in 16-byte pieces
+                    reinterpret_cast<__nv_bfloat16*>(sm.stg)[(GW * g + u) * kBM + rt] = __float2bfloat16_rn(xo[u]);
+                } else {
+                    reinterpret_cast<float*>(sm.stg)[(GW * g + u) * kBM + rt] = xo[u];
                 }
             }
             if constexpr (PASS != 2) {
@@ -315,6 +322,27 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
         }
     }
     if (tr) tr[kTrEpiLoop] = global_ns();
+    if constexpr (EPI == EPI_RESID && PASS != 0) {
+        // the staged chunk: thread t stores token t/4, features 32 (t%4) .. +31 of the tile
+        named_bar(1, 128);
+        const int t = ew * 32 + lane, tok = t >> 2, f0 = (t & 3) * 32;
+        const int col = col0 + tok;
+        if (col < p.N) {
+            if constexpr (PASS == 1) {
+                const uint4* src =
+                    reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(sm.stg) + tok * kBM + f0);
+                uint4* dst = reinterpret_cast<uint4*>(ep.xb + static_cast<size_t>(col) * ep.ld_out + mt * kBM + f0);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) dst[i] = src[i];
+            } else {
+                const float4* src = reinterpret_cast<const float4*>(reinterpret_cast<const float*>(sm.stg) + tok * kBM + f0);
+                float4* dst = reinterpret_cast<float4*>(ep.out + static_cast<size_t>(col) * ep.ld_out + mt * kBM + f0);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) dst[i] = src[i];
+            }
+        }
+        named_bar(1, 128);  // the staging memory is free again
+    }
     if constexpr (EPI == EPI_RESID && PASS != 1) {
         named_bar(1, 128);
         if (ew == 0) {
@@ -564,6 +592,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                     const int nb = nparts - b0 < per_batch ? nparts - b0 : per_batch;
                     if (threadIdx.x == 64) {
                         fence_proxy_async_global();
+                        fence_proxy_async_smem();  // the staging memory was last touched by generic accesses
                         mbar_arrive_expect_tx(redbar, slice_bytes * static_cast<uint32_t>(nb));
                         for (int q = 0; q < nb; ++q)
                             bulk_load(red_stage + static_cast<size_t>(q) * slice_bytes,
@@ -639,6 +668,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     esm.red = tail + 256;
     esm.kvs = reinterpret_cast<int*>(tail + 256 + 1024);
     esm.theta = tail + 256 + 1024 + 256;
+    esm.stg = red_stage;
     float* after = tail + 256 + 1024 + 256 + 128;
     uint64_t* full = reinterpret_cast<uint64_t*>(after);
     uint64_t* empty = full + S;
