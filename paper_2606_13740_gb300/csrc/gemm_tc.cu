@@ -255,21 +255,15 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
             float xp[GW];
 #pragma unroll
             for (int u = 0; u < GW; ++u) xp[u] = __shfl_xor_sync(0xffffffffu, a[u], 1);
-            bool bad = false;
-            const size_t head_base = static_cast<size_t>(hh) * (part == 0 ? ep.T : ep.cap);
-            const size_t seq_stride = static_cast<size_t>(ep.H) * (part == 0 ? ep.T : ep.cap);
+            // staged token-major in feature order ([32][128]: the tile's head(s) side by side),
+            // stored below in 16-byte pieces
+            __nv_bfloat16* st = reinterpret_cast<__nv_bfloat16*>(sm.stg) + (rt / ep.hd) * ep.hd + fi;
 #pragma unroll
             for (int u = 0; u < GW; ++u) {
-                const int col = cg + u;
-                const int pos = sm.kvs[bs[u]] + ts[u];
-                const bool inb = pos >= 0 && pos < ep.cap;
-                bad |= col < p.N && !inb;
                 float x = a[u];
                 if (part < 2) x = (pp & 1) ? (x * cs[u] + xp[u] * ss[u]) : (x * cs[u] - xp[u] * ss[u]);
-                const size_t r = static_cast<size_t>(bs[u]) * seq_stride + head_base + (part == 0 ? ts[u] : pos);
-                if (col < p.N && inb) qkv_dst[r * ep.hd + fi] = __float2bfloat16_rn(x);
+                st[(GW * g + u) * kBM] = __float2bfloat16_rn(x);
             }
-            if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(status, kStatusBadIndex);
         } else if constexpr (EPI == EPI_SWIGLU) {
             // tile row 2f is gate feature f, row 2f+1 the matching up row
             const int f = mt * 64 + (rt >> 1);
@@ -277,10 +271,12 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
             float up[GW];
 #pragma unroll
             for (int u = 0; u < GW; ++u) up[u] = __shfl_xor_sync(0xffffffffu, a[u], 1);
+            // staged token-major ([32][64] features), stored below in 16-byte pieces
+            __nv_bfloat16* st = reinterpret_cast<__nv_bfloat16*>(sm.stg) + (rt >> 1);
 #pragma unroll
             for (int u = 0; u < GW; ++u) {
                 const __nv_bfloat16 hv = __float2bfloat16_rn(__fdividef(a[u], 1.0f + __expf(-a[u])) * up[u]);
-                if (gate_lane && cg + u < p.N) ep.h[static_cast<size_t>(cg + u) * ep.F + f] = hv;
+                if (gate_lane) st[(GW * g + u) * 64] = hv;
             }
         } else if constexpr (EPI == EPI_LMHEAD) {
             // this warp's (max, argmax, sum exp) over its 32 rows, for the 8 columns side by side
@@ -322,6 +318,49 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
         }
     }
     if (tr) tr[kTrEpiLoop] = global_ns();
+    if constexpr (EPI == EPI_QKV) {
+        // thread t stores token t/4, tile features 32 (t%4) .. +31: one head's contiguous run
+        // at the token's row of the q tensor or of the K/V cache
+        named_bar(1, 128);
+        const int t = ew * 32 + lane, tok = t >> 2, f0 = (t & 3) * 32;
+        const int col = col0 + tok;
+        bool bad = false;
+        if (col < p.N) {
+            const int b = min(col / ep.T, ep.n_seq - 1);
+            const int ts = col - b * ep.T;
+            const int pos = sm.kvs[b] + ts;
+            const int head = (mt * kBM - part * ep.H * ep.hd + f0) / ep.hd;
+            const int fi0 = f0 % ep.hd;
+            if (pos >= 0 && pos < ep.cap) {
+                const size_t plane = part == 0 ? static_cast<size_t>(ep.T) : static_cast<size_t>(ep.cap);
+                const size_t r = (static_cast<size_t>(b) * ep.H + head) * plane + (part == 0 ? ts : pos);
+                const uint4* src = reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(sm.stg) +
+                                                                  tok * kBM + f0);
+                uint4* dst = reinterpret_cast<uint4*>(qkv_dst + r * ep.hd + fi0);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) dst[i] = src[i];
+            } else {
+                bad = true;
+            }
+        }
+        if (bad) atomicOr(status, kStatusBadIndex);
+        named_bar(1, 128);  // the staging memory is free again
+    } else if constexpr (EPI == EPI_SWIGLU) {
+        // thread t stores token t/4, features 16 (t%4) .. +15 of the tile's 64
+        named_bar(1, 128);
+        const int t = ew * 32 + lane, tok = t >> 2, f0 = (t & 3) * 16;
+        const int col = col0 + tok;
+        if (col < p.N) {
+            const uint4* src =
+                reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(sm.stg) + tok * 64 + f0);
+            const int fg = mt * 64 + f0;  // F is a multiple of 8: each 8-feature piece is all in or all out
+            uint4* dst = reinterpret_cast<uint4*>(ep.h + static_cast<size_t>(col) * ep.F + fg);
+#pragma unroll
+            for (int i = 0; i < 2; ++i)
+                if (fg + 8 * i < ep.F) dst[i] = src[i];
+        }
+        named_bar(1, 128);
+    }
     if constexpr (EPI == EPI_RESID && PASS != 0) {
         // the staged chunk: thread t stores token t/4, features 32 (t%4) .. +31 of the tile
         named_bar(1, 128);
