@@ -47,7 +47,7 @@ constexpr int kBK = 64;     // K elements per stage: one 128-byte swizzle row
 constexpr uint32_t kABytes = kBM * kBK * 2;
 constexpr int kFullSmem = 227 * 1024;
 static int g_stream_budget = kChainSmemShared;  // single projections: shared-memory plan
-constexpr int kTicketStride = 32;  // one tile ticket per 128-byte line
+constexpr int kTicketStride = 32;  // a tile's part flags: one 128-byte line (parts 1..31)
 constexpr int kEpiGroup = 16;      // epilogue columns processed side by side
 
 // Timeline trace slots per CTA (when EpiArgs::trace is set).
@@ -603,65 +603,84 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             tc_fence_before();
             mbar_arrive(&tempty[es.acc]);
             named_bar(1, 128);
-            if (threadIdx.x == 64) {
+            if (threadIdx.x == 64) {  // part q of the tile publishes its partial on flag q
                 if (tr) tr[kTrPartStored] = global_ns();
-                red_release_add(&P.tickets[tile * kTicketStride], 1);
+                st_release(&P.tickets[tile * kTicketStride + (static_cast<int>(blockIdx.x) - c_first)], tag);
             }
         }
         if (reducer) {
+            // Part q's partial, chunk c (32 columns), is the contiguous 16 KB slice [c*8 + j][row]
+            // float4.  Its slices go through staging slot (q-1) % 2, each bulk copy issued as
+            // soon as part q has published (flag q == tag) and the slot's previous slice is added:
+            // the early parts' slices arrive while the late ones still compute.  The sum runs over
+            // q in order, so it does not depend on the arrival order.
             const int nparts = c_last - c_first + 1;
-            int* ticket = &P.tickets[tile * kTicketStride];
-            if (threadIdx.x == 64) {
-                if (tr) tr[kTrPartStored] = global_ns();
-                wait_flag(ticket, nparts - 1, s_abort, status);
-                *ticket = 0;
-                if (tr) {
+            int* flags = &P.tickets[tile * kTicketStride];
+            constexpr uint32_t slice_bytes = 32 * kBM * 4;
+            uint32_t inflight = 0;  // thread 64: slots with a copy not yet waited for
+            auto issue = [&](int q, int c) {  // thread 64
+                if (c == 0 && !wait_flag(flags + q, tag, s_abort, status)) return;
+                const int sl = (q - 1) & 1;
+                fence_proxy_async_global();
+                fence_proxy_async_smem();  // the slot was last touched by generic accesses
+                mbar_arrive_expect_tx(redbar + sl, slice_bytes);
+                bulk_load(red_stage + static_cast<size_t>(sl) * slice_bytes,
+                          P.partials + static_cast<size_t>(c_first + q) * slot_floats + static_cast<size_t>(c) * 32 * kBM,
+                          slice_bytes, redbar + sl);
+                inflight |= 1u << sl;
+            };
+            if (tr && threadIdx.x == 64) tr[kTrPartStored] = global_ns();
+            bool stop = false;
+            for (int c = 0; c < nchunks && !stop; ++c) {
+                if (threadIdx.x == 64) {
+                    if (nparts > 1) issue(1, c);
+                    if (nparts > 2) issue(2, c);
+                }
+                tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);  // own (first) k-range
+                for (int q = 1; q < nparts; ++q) {
+                    const int sl = (q - 1) & 1;
+                    mbar_wait(redbar + sl, (es.red_phase >> sl) & 1u, s_abort, status);
+                    es.red_phase ^= 1u << sl;
+                    if (threadIdx.x == 64) inflight &= ~(1u << sl);
+                    const float4* src = reinterpret_cast<const float4*>(red_stage + static_cast<size_t>(sl) * slice_bytes);
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        const float4 a = src[j * kBM + rt];
+                        v[4 * j] += a.x;
+                        v[4 * j + 1] += a.y;
+                        v[4 * j + 2] += a.z;
+                        v[4 * j + 3] += a.w;
+                    }
+                    if (named_bar_any(1, 128, *s_abort != 0)) {  // the slot is free again (or the launch failed)
+                        stop = true;
+                        break;
+                    }
+                    if (threadIdx.x == 64 && q + 2 < nparts) issue(q + 2, c);
+                }
+                if (stop) break;
+                if (tr && threadIdx.x == 64 && c == 0) {
                     tr[kTrTicket] = global_ns();
+                    tr[kTrReduced] = global_ns();
                     tr[kTrIsLast] = 1;
                 }
-            }
-            if (named_bar_any(1, 128, *s_abort != 0)) return;
-            // a contributor's partial: chunk c (32 columns) is the contiguous slice
-            // [c*8 + j][row] float4, 16 KB; the slices are bulk-copied, red_bytes at a time
-            constexpr uint32_t slice_bytes = 32 * kBM * 4;
-            const int per_batch = ca.red_bytes / static_cast<int>(slice_bytes);
-            for (int c = 0; c < nchunks; ++c) {
-                tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);  // own (first) k-range
-                for (int b0 = 1; b0 < nparts; b0 += per_batch) {
-                    const int nb = nparts - b0 < per_batch ? nparts - b0 : per_batch;
-                    if (threadIdx.x == 64) {
-                        fence_proxy_async_global();
-                        fence_proxy_async_smem();  // the staging memory was last touched by generic accesses
-                        mbar_arrive_expect_tx(redbar, slice_bytes * static_cast<uint32_t>(nb));
-                        for (int q = 0; q < nb; ++q)
-                            bulk_load(red_stage + static_cast<size_t>(q) * slice_bytes,
-                                      P.partials + static_cast<size_t>(c_first + b0 + q) * slot_floats +
-                                          static_cast<size_t>(c) * 32 * kBM,
-                                      slice_bytes, redbar);
-                    }
-                    mbar_wait(redbar, es.red_phase, s_abort, status);
-                    es.red_phase ^= 1u;
-                    for (int q = 0; q < nb; ++q) {
-                        const float4* src =
-                            reinterpret_cast<const float4*>(red_stage + static_cast<size_t>(q) * slice_bytes);
-#pragma unroll
-                        for (int j = 0; j < 8; ++j) {
-                            const float4 a = src[j * kBM + rt];
-                            v[4 * j] += a.x;
-                            v[4 * j + 1] += a.y;
-                            v[4 * j + 2] += a.z;
-                            v[4 * j + 3] += a.w;
-                        }
-                    }
-                    named_bar(1, 128);  // the next batch overwrites the staging memory
-                }
-                if (tr && threadIdx.x == 64 && c == 0) tr[kTrReduced] = global_ns();
                 // the sum goes back into the (still owned) accumulator, then the compact epilogue
                 tmem_st_32x32(t_acc + static_cast<uint32_t>(c * 32), v);
                 epilogue_c32<EPI, kPass1>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt,
                                           t_acc + static_cast<uint32_t>(c * 32),
                                           t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, esm, ew, quarter, lane, status);
             }
+            if (threadIdx.x == 64) {
+                if (stop) {  // let copies in flight land before the shared memory is released
+                    const long long t0 = spin_clock();
+                    for (int sl = 0; sl < 2; ++sl)
+                        while ((inflight >> sl & 1u) && !mbar_try_wait(redbar + sl, (es.red_phase >> sl) & 1u) &&
+                               spin_clock() - t0 < kWaitLimitCycles) {
+                        }
+                } else {
+                    for (int q = 1; q < nparts; ++q) flags[q] = 0;  // ready for the next launch
+                }
+            }
+            if (stop) return;
         }
         if (finisher && P.done) {  // publish the finished tile to the next phase's operand producer
             named_bar(1, 128);
@@ -714,8 +733,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     uint64_t* tfull = empty + S;
     uint64_t* tempty = tfull + 2;
     uint64_t* drain = tempty + 2;
-    uint64_t* redbar = drain + 1;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(redbar + 1);
+    uint64_t* redbar = drain + 1;  // two partial staging slots
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(redbar + 2);
     volatile int* s_abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
     int* status = ca.status;
 
@@ -732,7 +751,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             mbar_init(&tempty[a], 128);
         }
         mbar_init(drain, 1);
-        mbar_init(redbar, 1);
+        mbar_init(&redbar[0], 1);
+        mbar_init(&redbar[1], 1);
         *s_abort = 0;
         mbar_fence_init();
     }
@@ -1009,6 +1029,10 @@ GemmPlan gemm_plan(int M, int N, int K, int grid_max, int epi) {
     p.kb = (K + kBK - 1) / kBK;
     p.total = static_cast<long long>(p.m_tiles) * p.n_tiles * p.kb;
     p.grid = static_cast<int>(p.total < grid_max ? p.total : grid_max);
+    // at least ceil(kb/30) iterations per CTA, so a tile has at most 31 parts (one completion
+    // flag each in its 32-int line)
+    const long long min_iters = (p.kb + 29) / 30;
+    if (p.grid > p.total / min_iters) p.grid = static_cast<int>(p.total / min_iters);
     if (p.grid < 1) p.grid = 1;
     p.pdl = true;
     return p;
@@ -1098,7 +1122,7 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
     ca.x_cols = ntile <= 128 ? ntile : 0;  // staged residual (none for 256-token tiles: TMEM is full)
     ca.tmem_cols = pow2ceil(2 * ca.acc_cols + ca.x_cols);
     ca.red_bytes = 2 * 32 * kBM * 4;  // two 32-column partial slices per bulk-copy round
-    const int fixed = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + 6 * 8 + 16;
+    const int fixed = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + 7 * 8 + 16;
     const int stage_bytes = static_cast<int>(kABytes) + ntile * kBK * 2;
     int st = (smem_budget - fixed) / (stage_bytes + 16);
     if (st > 32) st = 32;
