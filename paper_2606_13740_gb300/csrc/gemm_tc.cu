@@ -53,7 +53,7 @@ constexpr int kEpiGroup = 16;      // epilogue columns processed side by side
 // Timeline trace slots per CTA (when EpiArgs::trace is set).
 enum { kTrStart = 0, kTrPrologue = 1, kTrFirstData = 2, kTrLastData = 3, kTrEpiDone = 4, kTrExit = 5, kTrSm = 6,
        kTrDepWait = 7, kTrAccReady = 8, kTrPartStored = 9, kTrTicket = 10, kTrReduced = 11, kTrIsLast = 12,
-       kTrTile = 13, kTrEpiG0 = 14, kTrEpiLoop = 15, kTrSlots = 16 };
+       kTrTile = 13, kTrEpiPass1 = 14, kTrPublished = 15, kTrSlots = 16 };
 
 __device__ __forceinline__ unsigned smid() {
     unsigned id;
@@ -179,10 +179,8 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
     }
     bool lm_ok = false;
     if constexpr (EPI == EPI_LMHEAD) lm_ok = row < ep.V && row != ep.mask_id;
-    unsigned long long* tr = (ep.trace && ew == 0 && lane == 0) ? ep.trace + static_cast<size_t>(blockIdx.x) * kTrSlots : nullptr;
 #pragma unroll 1
     for (int g = 0; g < 32 / GW; ++g) {
-        if (tr && g == 1) tr[kTrEpiG0] = global_ns();
 
         const int cg = col0 + GW * g;  // first column of the group
         float a[GW];
@@ -317,7 +315,6 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
             }
         }
     }
-    if (tr) tr[kTrEpiLoop] = global_ns();
     if constexpr (EPI == EPI_QKV) {
         // thread t stores token t/4, tile features 32 (t%4) .. +31: one head's contiguous run
         // at the token's row of the q tensor or of the K/V cache
@@ -682,9 +679,13 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             }
             if (stop) return;
         }
+        if (tr && threadIdx.x == 64) tr[kTrEpiPass1] = global_ns();
         if (finisher && P.done) {  // publish the finished tile to the next phase's operand producer
             named_bar(1, 128);
-            if (threadIdx.x == 64) st_release(&P.done[mt * p.n_tiles + nt], tag);
+            if (threadIdx.x == 64) {
+                st_release(&P.done[mt * p.n_tiles + nt], tag);
+                if (tr) tr[kTrPublished] = global_ns();
+            }
         }
         if constexpr (EPI == EPI_RESID) {
             if (finisher) {  // then the fp32 residual and the RMSNorm sums, for the later phases' epilogues
