@@ -614,22 +614,46 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             const int nparts = c_last - c_first + 1;
             int* flags = &P.tickets[tile * kTicketStride];
             constexpr uint32_t slice_bytes = 32 * kBM * 4;
+            uint32_t ready = 0;     // warp 2: parts seen published (bit q)
             uint32_t inflight = 0;  // thread 64: slots with a copy not yet waited for
-            auto issue = [&](int q, int c) {  // thread 64
-                if (c == 0 && !wait_flag(flags + q, tag, s_abort, status)) return;
-                const int sl = (q - 1) & 1;
-                fence_proxy_async_global();
-                fence_proxy_async_smem();  // the slot was last touched by generic accesses
-                mbar_arrive_expect_tx(redbar + sl, slice_bytes);
-                bulk_load(red_stage + static_cast<size_t>(sl) * slice_bytes,
-                          P.partials + static_cast<size_t>(c_first + q) * slot_floats + static_cast<size_t>(c) * 32 * kBM,
-                          slice_bytes, redbar + sl);
-                inflight |= 1u << sl;
+            // warp 2, warp-uniform: make sure part q has published, polling every part's flag at
+            // once (lane i reads flag i, so one round trip covers them all), then thread 64
+            // issues the copy of q's chunk-c slice into slot (q-1) % 2
+            auto issue = [&](int q, int c) {
+                if (c == 0) {
+                    const long long t0 = spin_clock();
+                    while (!(ready >> q & 1u)) {
+                        const bool ok = lane >= 1 && lane < nparts && ld_acquire(flags + lane) == tag;
+                        ready |= __ballot_sync(0xffffffffu, ok);
+                        if (ready >> q & 1u) break;
+                        int give_up = 0;
+                        if (lane == 0) give_up = (*s_abort || spin_clock() - t0 > kWaitLimitCycles) ? 1 : 0;
+                        if (__shfl_sync(0xffffffffu, give_up, 0)) {  // warp-uniform decision
+                            if (lane == 0 && !*s_abort) {
+                                *s_abort = 1;
+                                atomicOr(status, kStatusTimeout);
+                            }
+                            return;
+                        }
+                        __nanosleep(32);
+                    }
+                }
+                if (lane == 0) {
+                    const int sl = (q - 1) & 1;
+                    fence_proxy_async_global();
+                    fence_proxy_async_smem();  // the slot was last touched by generic accesses
+                    mbar_arrive_expect_tx(redbar + sl, slice_bytes);
+                    bulk_load(red_stage + static_cast<size_t>(sl) * slice_bytes,
+                              P.partials + static_cast<size_t>(c_first + q) * slot_floats +
+                                  static_cast<size_t>(c) * 32 * kBM,
+                              slice_bytes, redbar + sl);
+                    inflight |= 1u << sl;
+                }
             };
             if (tr && threadIdx.x == 64) tr[kTrPartStored] = global_ns();
             bool stop = false;
             for (int c = 0; c < nchunks && !stop; ++c) {
-                if (threadIdx.x == 64) {
+                if (ew == 0) {
                     if (nparts > 1) issue(1, c);
                     if (nparts > 2) issue(2, c);
                 }
@@ -652,7 +676,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                         stop = true;
                         break;
                     }
-                    if (threadIdx.x == 64 && q + 2 < nparts) issue(q + 2, c);
+                    if (ew == 0 && q + 2 < nparts) issue(q + 2, c);
                 }
                 if (stop) break;
                 if (tr && threadIdx.x == 64 && c == 0) {
