@@ -16,7 +16,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(os.path.dirname(PKG), "include")
 OUT = os.path.join(PKG, "libdllm.so")
 BUILD = os.path.join(PKG, "_build")
-SOURCES = ["gemm_tc.cu", "kernels.cu", "api.cu", "ops.cu", "noalloc.cu"]
+SOURCES = ["gemm_tc.cu", "attn_tc.cu", "kernels.cu", "api.cu", "ops.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE]
 

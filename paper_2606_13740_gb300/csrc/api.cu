@@ -262,7 +262,7 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
     if (!make_tmap_bf16(&tx_xn, ctx->xn, N, d, pq.ntile) || !make_tmap_bf16(&tx_attn, ctx->attn, N, qd, po.ntile) ||
         !make_tmap_bf16(&tx_h, ctx->h, N, F, pd.ntile))
         return fail(ctx, DLLM_ECUDA, "tensor map encode failed");
-    const AttnPlan ap = attn_plan(B, T, c.n_heads, ctx->kv_len + T, ctx->sms);
+    const AttnPlan ap = attn_plan(B, T, c.n_heads, c.head_dim, ctx->kv_len + T, ctx->sms);
     EpiArgs ep{};
     ep.seq_kv = ctx->seq_kv;
     ep.n_seq = B;
@@ -333,7 +333,7 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
     for (int l = 0; l < c.n_layers; ++l) {
         const EpiArgs el = qkv_args(l);
         CK(launch_attention(ctx->q, el.kc, el.vc, ctx->seq_kv, ctx->attn, B, T, c.n_heads, c.head_dim, c.max_ctx, ap, s,
-                            true, next_trace(ctx)));
+                            true, next_trace(ctx), ctx->status));
         mark(ctx, DLLM_K_ATTN);
         // output projection (+ residual) -> gate/up (+ SwiGLU) -> down (+ residual) -> next QKV or LM head
         ChainArgs ca{};

@@ -180,12 +180,22 @@ struct AttnPlan {
     int qtiles, nw, csize;
     int nb;     // K/V sub-blocks in flight per CTA (1 or 2)
     int pairs;  // warp groups per CTA, each on its own share of the CTA's sub-blocks (1 or 2)
+    bool tc;    // head dim 128: the tcgen05 kernel (128-row query tiles, 64-key sub-blocks)
 };
-AttnPlan attn_plan(int B, int T, int H, int max_keys, int sms);
+// head dim 128 and at least kTcMinKeys keys: the tcgen05 kernel's plan; otherwise the
+// mma.sync kernel's
+constexpr int kTcMinKeys = 1024;
+AttnPlan attn_plan(int B, int T, int H, int hd, int max_keys, int sms);
+AttnPlan attn_plan_tc(int B, int T, int H, int max_keys, int sms);
+cudaError_t attn_tc_init_attrs();
+cudaError_t launch_attention_tc(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
+                                const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int cap,
+                                const AttnPlan& a, cudaStream_t st, bool pdl, unsigned long long* trace,
+                                int* status);
 cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
                              const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int hd, int cap,
                              const AttnPlan& a, cudaStream_t st, bool pdl = true,
-                             unsigned long long* trace = nullptr);
+                             unsigned long long* trace = nullptr, int* status = nullptr);
 cudaError_t launch_lmhead_reduce(const float* lm_part, const float* zcur, const int* cur_tok, int m_tiles,
                                  int N, int mask_id, int* x0, float* conf, float* tokconf, cudaStream_t st,
                                  bool pdl = true);

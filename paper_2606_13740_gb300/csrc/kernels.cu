@@ -419,7 +419,8 @@ static cudaError_t attn_attr() {
 }
 
 cudaError_t attn_init_attrs() {
-    cudaError_t e = attn_attr<128, 2, 1, 1>();
+    cudaError_t e = attn_tc_init_attrs();
+    if (e == cudaSuccess) e = attn_attr<128, 2, 1, 1>();
     if (e == cudaSuccess) e = attn_attr<128, 2, 1, 2>();
     if (e == cudaSuccess) e = attn_attr<128, 2, 2, 1>();
     if (e == cudaSuccess) e = attn_attr<128, 4, 1, 1>();
@@ -432,8 +433,11 @@ cudaError_t attn_init_attrs() {
     return e;
 }
 
-AttnPlan attn_plan(int B, int T, int H, int max_keys, int sms) {
-    AttnPlan a;
+AttnPlan attn_plan(int B, int T, int H, int hd, int max_keys, int sms) {
+    // long key ranges (head dim 128) go to the tensor-core kernel; on short ones, a few
+    // sub-blocks per CTA, the mma.sync kernel has less latency per sub-block
+    if (hd == 128 && max_keys >= kTcMinKeys) return attn_plan_tc(B, T, H, max_keys, sms);
+    AttnPlan a{};
     // two warps (32 query rows) for the short windows of cached decoding, four otherwise: a
     // 64-token window is one query tile, so its keys and values are read once
     a.nw = T <= 32 ? 2 : 4;
@@ -472,7 +476,11 @@ static cudaError_t attn_go(cudaLaunchConfig_t& cfg, const __nv_bfloat16* q, cons
 
 cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
                              const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int hd, int cap,
-                             const AttnPlan& a, cudaStream_t st, bool pdl, unsigned long long* trace) {
+                             const AttnPlan& a, cudaStream_t st, bool pdl, unsigned long long* trace, int* status) {
+    if (a.tc) {
+        if (hd != 128) return cudaErrorInvalidValue;
+        return launch_attention_tc(q, kc, vc, seq_kv, out, B, T, H, cap, a, st, pdl, trace, status);
+    }
     if (a.csize < 1 || a.csize > kMaxCluster || (a.nw != 2 && a.nw != 4) || (a.nb != 1 && a.nb != 2) ||
         (a.pairs != 1 && a.pairs != 2) || (a.pairs == 2 && (a.nw != 2 || a.nb != 1)) || (hd != 64 && hd != 128))
         return cudaErrorInvalidValue;

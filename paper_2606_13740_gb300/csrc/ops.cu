@@ -149,7 +149,7 @@ int dllm_op_attention(const void* q, const void* kc, const void* vc, const int32
     int sms = sm_count();
     if (sms <= 0) return op_fail(DLLM_ECUDA, "no CUDA device");
     if (attn_init_attrs() != cudaSuccess) return op_fail(DLLM_ECUDA, "attribute setup failed");
-    AttnPlan a = attn_plan(B, T, H, max_kv_len + T, sms);
+    AttnPlan a = attn_plan(B, T, H, hd, max_kv_len + T, sms);
     cudaError_t e = launch_attention(static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(kc),
                                      static_cast<const __nv_bfloat16*>(vc), kv_len, static_cast<__nv_bfloat16*>(out),
                                      B, T, H, hd, cap, a, st, false);

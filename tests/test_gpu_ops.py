@@ -81,6 +81,9 @@ def _attn_ref(q, k, v, kv_len, T):
 @pytest.mark.parametrize("B,T,H,hd,kv,cap", [
     (1, 32, 4, 128, [512], 600), (2, 96, 2, 64, [0, 37], 160), (1, 512, 2, 128, [0], 512),
     (3, 32, 2, 128, [5, 300, 1000], 1100), (2, 64, 4, 128, [4096, 4096], 4160), (1, 1, 1, 64, [3], 8),
+    # the tensor-core kernel (head dim 128, >= 1024 keys): two 128-row query tiles (the second
+    # ragged), eight key splits per cluster, a sequence whose keys fill no split but the first
+    (1, 192, 2, 128, [1100], 1300), (1, 32, 1, 128, [2000], 2048), (2, 40, 3, 128, [1, 1500], 1600),
 ])
 def test_attention_matches_numpy(dev, B, T, H, hd, kv, cap):
     from paper_2606_13740_gb300 import dllm_op_attention
