@@ -21,12 +21,15 @@
 // and share it through L2) is cut into one contiguous range per CTA, so
 // every SM streams the same number of weight bytes whatever the tile count.
 // A tile cut between CTAs is finished by the CTA holding its first k-blocks,
-// which are the end of that CTA's range: the other contributors store fp32
-// partials and publish them with one release increment each, and the
-// finishing CTA waits (bounded) for the count, bulk-copies the partials into
-// shared memory and adds them to its own accumulator in k order
+// which are the end of that CTA's range: the other parts store fp32 partials
+// and publish each on its own flag, and the finishing CTA polls every part's
+// flag at once (bounded), bulk-copies each part's slice into shared memory as
+// soon as it is published and adds them to its own accumulator in part order
 // (deterministic).  Every CTA waits only on CTAs that wait on nothing later
 // than it, and the grid never exceeds the SM count, so all are resident.
+// The weights (the context's, stored tile-major) arrive as one contiguous
+// bulk copy per 16 KB tile; row-major weights of the single-projection entry
+// points arrive through a 2-D tensor map.
 //
 // Epilogues are fused: residual add with the next RMSNorm's statistics,
 // RoPE + KV-cache write, SwiGLU, and the LM head's per-tile softmax
