@@ -77,7 +77,17 @@ struct EpiSmem {
     int* kvs;     // [256] per-sequence first window position (QKV); current ids of the token tile (LM head)
     float* theta; // [128] rotation frequency of each tile row's feature pair (QKV)
     uint8_t* stg; // staging of a 32-token chunk's residual outputs (the partial staging memory, free by then)
+    float* xs;    // [2][32][128] the old fp32 residual of a wide tile's chunks (nullptr: none), see xs_offset
 };
+
+// Word offset of (token j, tile row f) in a 32-token chunk of staged residual: [token][128 rows],
+// the 16-byte pieces of a token's row rotated so that neither the copies (thread = token, 8
+// pieces) nor the epilogue's reads (lane = row) meet bank conflicts.
+__device__ __forceinline__ int xs_offset(int j, int f) {
+    const int c16 = f >> 2;
+    const int key = (j + 2 * (c16 >> 3)) & 7;
+    return j * kBM + (((c16 & ~7) | ((c16 & 7) ^ key)) << 2) + (f & 3);
+}
 
 // RMSNorm scale of every column of token tile nt: rs[c] = rsqrt(sum_t sq[t][col] / dim + eps).
 // 128 threads, 4 per column (each over a quarter of the statistics, loads independent), summed
@@ -147,10 +157,12 @@ __device__ __forceinline__ void warp_reduce_scatter(float* v, int lane) {
 // published to the next phase's operand producer between them; PASS 0: both at once.
 template <int EPI, int PASS = 0>
 __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& p, int mt, int col0, int c_in,
-                                             int rt, uint32_t t_src, uint32_t t_x, const EpiSmem& sm, int ew,
-                                             int quarter, int lane, int* status) {
+                                             int rt, uint32_t t_src, uint32_t t_x, const float* xs, const EpiSmem& sm,
+                                             int ew, int quarter, int lane, int* status) {
     // col0: the chunk's first token column; c_in: its offset inside the token tile (index into
-    // the tile's RMSNorm scales and staged ids); t_x == 0: the old residual is read from global
+    // the tile's RMSNorm scales and staged ids).  The old residual (pass 1) comes from TMEM
+    // (t_x), else from shared memory (xs, the chunk's staged copy), else from global; pass 1
+    // leaves the new residual in the accumulator, where pass 2 reads it.
     constexpr int GW = kEpiGroup;  // columns per group
     constexpr int LS = 32 / GW;    // lanes sharing one column's sum after the scatter
     const int row = mt * kBM + rt;
@@ -198,17 +210,28 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                 if (row < p.M && cg + u < p.N) ep.out[static_cast<size_t>(cg + u) * ep.ld_out + row] = a[u];
         } else if constexpr (EPI == EPI_RESID) {
             float xo[GW], ss[GW];
-            if (t_x) {
-                tmem_ld_32xn<GW>(t_x + static_cast<uint32_t>(GW * g), xo);
-            } else {
+            if constexpr (PASS == 2) {
 #pragma unroll
-                for (int u = 0; u < GW; ++u)
-                    xo[u] = (row < p.M && cg + u < p.N) ? ep.out[static_cast<size_t>(cg + u) * ep.ld_out + row] : 0.0f;
+                for (int u = 0; u < GW; ++u) xo[u] = a[u];
+            } else {
+                if (t_x) {
+                    tmem_ld_32xn<GW>(t_x + static_cast<uint32_t>(GW * g), xo);
+                } else if (xs) {
+#pragma unroll
+                    for (int u = 0; u < GW; ++u) xo[u] = xs[xs_offset(GW * g + u, rt)];
+                } else {
+#pragma unroll
+                    for (int u = 0; u < GW; ++u)
+                        xo[u] = (row < p.M && cg + u < p.N) ? ep.out[static_cast<size_t>(cg + u) * ep.ld_out + row]
+                                                            : 0.0f;
+                }
+#pragma unroll
+                for (int u = 0; u < GW; ++u) xo[u] += a[u];
             }
+            if constexpr (PASS == 1) tmem_st_32xn<GW>(t_src + static_cast<uint32_t>(GW * g), xo);
 #pragma unroll
             for (int u = 0; u < GW; ++u) {
                 const bool ok = row < p.M && cg + u < p.N;
-                xo[u] += a[u];
                 ss[u] = ok ? xo[u] * xo[u] : 0.0f;
                 if constexpr (PASS == 0) {
                     if (ok) {
@@ -513,6 +536,33 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
     const uint32_t t_x =
         ca.x_cols ? tmem_base + static_cast<uint32_t>(2 * ca.acc_cols) + (static_cast<uint32_t>(quarter * 32) << 16)
                   : 0u;
+    // Wide residual tiles (no TMEM room for the old x): each 32-token chunk of the old fp32
+    // residual is copied into shared memory (two buffers, chunk c in buffer c % 2) by cp.async,
+    // 16 bytes a copy, thread t taking token t/4's rows 32 (t%4) .. +31, one chunk ahead of
+    // its use; x_chunk starts the next chunk's copies, then waits for this chunk's.
+    const bool use_xs = EPI == EPI_RESID && esm.xs != nullptr && (ep.ld_out & 3) == 0 &&
+                        (reinterpret_cast<uintptr_t>(ep.out) & 15) == 0;
+    auto x_fetch = [&](int fmt, int fnt, int c) {
+        const int t = ew * 32 + lane, tok = t >> 2, q = t & 3;
+        const int col = fnt * p.ntile + c * 32 + tok;
+        float* buf = esm.xs + (c & 1) * (32 * kBM);
+        if (col < p.N) {
+            const int f0 = fmt * kBM + q * 32;
+            const float* src = ep.out + static_cast<size_t>(col) * ep.ld_out + f0;
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+                if (f0 + 4 * i < p.M) cp_async16(buf + xs_offset(tok, q * 32 + 4 * i), src + 4 * i);
+        }
+        cp_async_commit();
+    };
+    auto x_chunk = [&](int cmt, int cnt, int c) -> const float* {
+        if (!use_xs) return nullptr;
+        if (c + 1 < nchunks) x_fetch(cmt, cnt, c + 1);
+        else cp_async_commit();
+        cp_async_wait<1>();
+        named_bar(1, 128);
+        return esm.xs + (c & 1) * (32 * kBM);
+    };
     int rs_nt = -1, ids_nt = -1;
     long long prepared = -1;
     float v[32];
@@ -542,6 +592,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             }
         }
         if constexpr (EPI == EPI_RESID) {
+            if (use_xs) x_fetch(pmt, pnt, 0);
             if (t_x) {
                 const int row = pmt * kBM + rt;
                 for (int c = 0; c < nchunks; ++c) {
@@ -575,7 +626,10 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         if (finisher) prepare(tile);
         else if (tend < it1) prepare(tile + 1);
         mbar_wait(&tfull[es.acc], es.acc_phase, s_abort, status);
-        if (named_bar_any(1, 128, *s_abort != 0)) return;
+        if (named_bar_any(1, 128, *s_abort != 0)) {
+            cp_async_wait<0>();  // no copy lands in shared memory after the launch has ended
+            return;
+        }
         if (tr && threadIdx.x == 64) {
             tr[kTrAccReady] = global_ns();
             tr[kTrTile] = static_cast<unsigned long long>(tile);
@@ -585,10 +639,13 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                                (static_cast<uint32_t>(quarter * 32) << 16);
         if (whole) {
             // the compact epilogue per 32-column chunk, straight from the accumulator in TMEM
-            for (int c = 0; c < nchunks; ++c)
+            for (int c = 0; c < nchunks; ++c) {
+                const float* xs = x_chunk(mt, nt, c);
                 epilogue_c32<EPI, kPass1>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt,
                                           t_acc + static_cast<uint32_t>(c * 32),
-                                          t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, esm, ew, quarter, lane, status);
+                                          t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, xs, esm, ew, quarter, lane,
+                                          status);
+            }
         } else if (!reducer) {
             float* my_part = P.partials + static_cast<size_t>(blockIdx.x) * slot_floats;
             for (int c = 0; c < nchunks; ++c) {
@@ -689,9 +746,11 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                 }
                 // the sum goes back into the (still owned) accumulator, then the compact epilogue
                 tmem_st_32x32(t_acc + static_cast<uint32_t>(c * 32), v);
+                const float* xs = x_chunk(mt, nt, c);
                 epilogue_c32<EPI, kPass1>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt,
                                           t_acc + static_cast<uint32_t>(c * 32),
-                                          t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, esm, ew, quarter, lane, status);
+                                          t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, xs, esm, ew, quarter, lane,
+                                          status);
             }
             if (threadIdx.x == 64) {
                 if (stop) {  // let copies in flight land before the shared memory is released
@@ -704,7 +763,10 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                     for (int q = 1; q < nparts; ++q) flags[q] = 0;  // ready for the next launch
                 }
             }
-            if (stop) return;
+            if (stop) {
+                cp_async_wait<0>();
+                return;
+            }
         }
         if (tr && threadIdx.x == 64) tr[kTrEpiPass1] = global_ns();
         if (finisher && P.done) {  // publish the finished tile to the next phase's operand producer
@@ -718,8 +780,8 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             if (finisher) {  // then the fp32 residual and the RMSNorm sums, for the later phases' epilogues
                 for (int c = 0; c < nchunks; ++c)
                     epilogue_c32<EPI, 2>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt,
-                                         t_acc + static_cast<uint32_t>(c * 32),
-                                         t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, esm, ew, quarter, lane, status);
+                                         t_acc + static_cast<uint32_t>(c * 32), 0u, nullptr, esm, ew, quarter, lane,
+                                         status);
                 if (P.done2) {
                     named_bar(1, 128);
                     if (threadIdx.x == 64) st_release(&P.done2[mt * p.n_tiles + nt], tag);
@@ -736,6 +798,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         }
         it = tile * p.kb + k_hi;
     }
+    cp_async_wait<0>();
     if (tr && threadIdx.x == 64) tr[kTrEpiDone] = global_ns();
 }
 
@@ -748,8 +811,9 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     uint8_t* sA = smem;
     uint8_t* sB = sA + static_cast<size_t>(S) * kABytes;
     uint8_t* red_stage = sB + static_cast<size_t>(S) * b_bytes;
-    float* tail = reinterpret_cast<float*>(red_stage + ca.red_bytes);
+    float* tail = reinterpret_cast<float*>(red_stage + ca.red_bytes + ca.xs_bytes);
     EpiSmem esm;
+    esm.xs = ca.xs_bytes ? reinterpret_cast<float*>(red_stage + ca.red_bytes) : nullptr;
     esm.rs = tail;
     esm.red = tail + 256;
     esm.kvs = reinterpret_cast<int*>(tail + 256 + 1024);
@@ -1150,8 +1214,15 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
     ca.x_cols = ntile <= 128 ? ntile : 0;  // staged residual (none for 256-token tiles: TMEM is full)
     ca.tmem_cols = pow2ceil(2 * ca.acc_cols + ca.x_cols);
     ca.red_bytes = 2 * 32 * kBM * 4;  // two 32-column partial slices per bulk-copy round
-    const int fixed = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + 7 * 8 + 16;
     const int stage_bytes = static_cast<int>(kABytes) + ntile * kBK * 2;
+    // the old residual of wide tiles, staged in shared memory two 32-token chunks at a time,
+    // where that leaves the ring at least 3 stages
+    ca.xs_bytes = 0;
+    if (ca.x_cols == 0) {
+        const int fixed_xs = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + 2 * 32 * kBM * 4 + 7 * 8 + 16;
+        if ((smem_budget - fixed_xs) / (stage_bytes + 16) >= 3) ca.xs_bytes = 2 * 32 * kBM * 4;
+    }
+    const int fixed = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + ca.xs_bytes + 7 * 8 + 16;
     int st = (smem_budget - fixed) / (stage_bytes + 16);
     if (st > 32) st = 32;
     if (st < 2) return false;

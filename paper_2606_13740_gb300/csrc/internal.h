@@ -109,7 +109,8 @@ struct ChainArgs {
     int n_phases;
     int grid, stages, ntile, acc_cols, tmem_cols;
     int red_bytes;       // shared staging for split partials
-    int x_cols;          // TMEM columns for the staged old residual (0: read from global)
+    int x_cols;          // TMEM columns for the staged old residual (0: none)
+    int xs_bytes;        // shared staging of the old residual when x_cols == 0 (0: read from global)
     size_t smem;
     const int* epoch;    // device step counter; tag = *epoch * tag_mul + tag_add (null: tag = tag_add)
     int tag_mul, tag_add;
@@ -120,7 +121,7 @@ struct ChainMaps {
     CUtensorMap w[kMaxPhases];
     CUtensorMap x[kMaxPhases];
 };
-// Fills grid, stages, ntile, acc_cols, x_cols, tmem_cols, red_bytes and smem from the phases' plans for a
+// Fills grid, stages, ntile, acc_cols, x_cols, xs_bytes, tmem_cols, red_bytes and smem from the phases' plans for a
 // shared-memory budget (bytes, <= 227 KB).  False if the phases do not share one token tiling.
 bool chain_plan(ChainArgs& ca, int smem_budget);
 constexpr int kChainSmemFull = 227 * 1024;    // one CTA per SM, deepest ring
