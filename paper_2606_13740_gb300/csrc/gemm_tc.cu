@@ -51,7 +51,9 @@ constexpr uint32_t kABytes = kBM * kBK * 2;
 constexpr int kFullSmem = 227 * 1024;
 static int g_stream_budget = kChainSmemShared;  // single projections: shared-memory plan
 constexpr int kTicketStride = 32;  // a tile's part flags: one 128-byte line (parts 1..31)
-constexpr int kEpiGroup = 16;      // epilogue columns processed side by side
+constexpr int kEpiGroup = 16;      // epilogue columns processed side by side: half a 32-token chunk
+constexpr int kEpiWarps = 8;       // two per TMEM lane quarter, one per half chunk
+constexpr int kEpiThreads = kEpiWarps * 32;
 
 // Timeline trace slots per CTA (when EpiArgs::trace is set).
 enum { kTrStart = 0, kTrPrologue = 1, kTrFirstData = 2, kTrLastData = 3, kTrEpiDone = 4, kTrExit = 5, kTrSm = 6,
@@ -76,7 +78,9 @@ struct EpiSmem {
     float* red;   // [4][256] cross-warp / quarter partial sums
     int* kvs;     // [256] per-sequence first window position (QKV); current ids of the token tile (LM head)
     float* theta; // [128] rotation frequency of each tile row's feature pair (QKV)
-    uint8_t* stg; // staging of a 32-token chunk's residual outputs (the partial staging memory, free by then)
+    uint8_t* stg;  // staging of a 32-token chunk's bf16 outputs, 8 KB (for tiles of more than one chunk its
+                   // own memory: the next chunk's partial slices arrive meanwhile)
+    uint8_t* stg2; // staging of a chunk's fp32 residual (second pass), 16 KB: the partial staging memory
     float* xs;    // [2][32][128] the old fp32 residual of a wide tile's chunks (nullptr: none), see xs_offset
 };
 
@@ -90,11 +94,11 @@ __device__ __forceinline__ int xs_offset(int j, int f) {
 }
 
 // RMSNorm scale of every column of token tile nt: rs[c] = rsqrt(sum_t sq[t][col] / dim + eps).
-// 128 threads, 4 per column (each over a quarter of the statistics, loads independent), summed
-// in a fixed order: deterministic.
+// The epilogue threads, 4 per column (each over a quarter of the statistics, loads
+// independent), summed in a fixed order: deterministic.
 __device__ __forceinline__ void compute_norm_scale(const EpiArgs& ep, const GemmPlan& p, int nt, const EpiSmem& sm,
                                                    int e) {
-    for (int item = e; item < 4 * p.ntile; item += 128) {
+    for (int item = e; item < 4 * p.ntile; item += kEpiThreads) {
         const int c = item % p.ntile, q = item / p.ntile;
         const int col = nt * p.ntile + c;
         float s = 0.0f;
@@ -111,12 +115,12 @@ __device__ __forceinline__ void compute_norm_scale(const EpiArgs& ep, const Gemm
         }
         sm.red[q * 256 + c] = s;
     }
-    named_bar(1, 128);
-    for (int c = e; c < p.ntile; c += 128) {
+    named_bar(1, kEpiThreads);
+    for (int c = e; c < p.ntile; c += kEpiThreads) {
         const float s = ((sm.red[c] + sm.red[256 + c]) + sm.red[512 + c]) + sm.red[768 + c];
         sm.rs[c] = rsqrtf(s / static_cast<float>(ep.norm_dim) + ep.eps);
     }
-    named_bar(1, 128);
+    named_bar(1, kEpiThreads);
 }
 
 // (cos, sin) of an angle: one out-of-line copy, called twice per chunk on the common path.
@@ -146,23 +150,24 @@ __device__ __forceinline__ void warp_reduce_scatter(float* v, int lane) {
     for (int w = 16 / N; w >= 1; w >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], w);
 }
 
-// Epilogue of a 32-token tile (the batch-1 weight stream), compact: one rolled loop over 4
-// groups of 8 columns read from TMEM (t_src; for the residual, the old x of the tile was
-// staged at t_x before the accumulator was ready), so its code stays small and no global load
-// waits on a store.  Inside a group every step runs over the 8 columns side by side with no
-// branch between them (stores are predicated), so their dependent chains (shuffles, special
-// functions) overlap.
+// Epilogue of a 32-token chunk, compact: each epilogue thread takes its TMEM lane (tile row)
+// and one half of the chunk, 16 columns read from TMEM (t_src; for the residual, the old x of
+// a narrow tile was staged at t_x before the accumulator was ready), so its code stays small
+// and no global load waits on a store.  The 16 columns run side by side with no branch between
+// them (stores are predicated), so their dependent chains (shuffles, special functions)
+// overlap; the chunk's outputs are staged in shared memory and stored in 16-byte pieces.
 // Residual epilogue in two passes (PASS 1: the bf16 copy, the next projection's operand, and
 // the RMSNorm partial sums; PASS 2: the fp32 residual and the sums' store), so the tile can be
 // published to the next phase's operand producer between them; PASS 0: both at once.
 template <int EPI, int PASS = 0>
 __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& p, int mt, int col0, int c_in,
                                              int rt, uint32_t t_src, uint32_t t_x, const float* xs, const EpiSmem& sm,
-                                             int ew, int quarter, int lane, int* status) {
+                                             int e, int half, int quarter, int lane, int* status) {
     // col0: the chunk's first token column; c_in: its offset inside the token tile (index into
     // the tile's RMSNorm scales and staged ids).  The old residual (pass 1) comes from TMEM
     // (t_x), else from shared memory (xs, the chunk's staged copy), else from global; pass 1
-    // leaves the new residual in the accumulator, where pass 2 reads it.
+    // leaves the new residual in the accumulator, where pass 2 reads it.  e: the epilogue
+    // thread (0 .. kEpiThreads-1), half: which 16 columns of the chunk.
     constexpr int GW = kEpiGroup;  // columns per group
     constexpr int LS = 32 / GW;    // lanes sharing one column's sum after the scatter
     const int row = mt * kBM + rt;
@@ -184,7 +189,7 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
         run = min(col0 + 31, p.N - 1) / ep.T == bl;  // all 32 columns in one sequence
         qkv_dst = part == 0 ? ep.q : (part == 1 ? ep.kc : ep.vc);
         if (part < 2 && run) {
-            const float2 a = rot_cs(static_cast<float>(sm.kvs[bl] + (col0 - bl * ep.T)) * theta);
+            const float2 a = rot_cs(static_cast<float>(sm.kvs[bl] + (col0 + GW * half - bl * ep.T)) * theta);
             const float2 d = rot_cs(theta);
             cn = a.x;
             sn = a.y;
@@ -194,8 +199,9 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
     }
     bool lm_ok = false;
     if constexpr (EPI == EPI_LMHEAD) lm_ok = row < ep.V && row != ep.mask_id;
-#pragma unroll 1
-    for (int g = 0; g < 32 / GW; ++g) {
+    static_assert(32 / GW == 2, "one column group per half chunk");
+    {
+        const int g = half;
 
         const int cg = col0 + GW * g;  // first column of the group
         float a[GW];
@@ -242,7 +248,7 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                 } else if constexpr (PASS == 1) {  // token-major staging, stored below in 16-byte pieces
                     reinterpret_cast<__nv_bfloat16*>(sm.stg)[(GW * g + u) * kBM + rt] = __float2bfloat16_rn(xo[u]);
                 } else {
-                    reinterpret_cast<float*>(sm.stg)[(GW * g + u) * kBM + rt] = xo[u];
+                    reinterpret_cast<float*>(sm.stg2)[(GW * g + u) * kBM + rt] = xo[u];
                 }
             }
             if constexpr (PASS != 2) {
@@ -342,10 +348,10 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
         }
     }
     if constexpr (EPI == EPI_QKV) {
-        // thread t stores token t/4, tile features 32 (t%4) .. +31: one head's contiguous run
-        // at the token's row of the q tensor or of the K/V cache
-        named_bar(1, 128);
-        const int t = ew * 32 + lane, tok = t >> 2, f0 = (t & 3) * 32;
+        // thread t stores token t/8, tile features 16 (t%8) .. +15: part of one head's
+        // contiguous run at the token's row of the q tensor or of the K/V cache
+        named_bar(1, kEpiThreads);
+        const int t = e, tok = t >> 3, f0 = (t & 7) * 16;
         const int col = col0 + tok;
         bool bad = false;
         if (col < p.N) {
@@ -361,33 +367,30 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                                                                   tok * kBM + f0);
                 uint4* dst = reinterpret_cast<uint4*>(qkv_dst + r * ep.hd + fi0);
 #pragma unroll
-                for (int i = 0; i < 4; ++i) dst[i] = src[i];
+                for (int i = 0; i < 2; ++i) dst[i] = src[i];
             } else {
                 bad = true;
             }
         }
         if (bad) atomicOr(status, kStatusBadIndex);
-        named_bar(1, 128);  // the staging memory is free again
+        named_bar(1, kEpiThreads);  // the staging memory is free again
     } else if constexpr (EPI == EPI_SWIGLU) {
-        // thread t stores token t/4, features 16 (t%4) .. +15 of the tile's 64
-        named_bar(1, 128);
-        const int t = ew * 32 + lane, tok = t >> 2, f0 = (t & 3) * 16;
+        // thread t stores token t/8, features 8 (t%8) .. +7 of the tile's 64
+        named_bar(1, kEpiThreads);
+        const int t = e, tok = t >> 3, f0 = (t & 7) * 8;
         const int col = col0 + tok;
         if (col < p.N) {
             const uint4* src =
                 reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(sm.stg) + tok * 64 + f0);
             const int fg = mt * 64 + f0;  // F is a multiple of 8: each 8-feature piece is all in or all out
-            uint4* dst = reinterpret_cast<uint4*>(ep.h + static_cast<size_t>(col) * ep.F + fg);
-#pragma unroll
-            for (int i = 0; i < 2; ++i)
-                if (fg + 8 * i < ep.F) dst[i] = src[i];
+            if (fg < ep.F) *reinterpret_cast<uint4*>(ep.h + static_cast<size_t>(col) * ep.F + fg) = *src;
         }
-        named_bar(1, 128);
+        named_bar(1, kEpiThreads);
     }
     if constexpr (EPI == EPI_RESID && PASS != 0) {
-        // the staged chunk: thread t stores token t/4, features 32 (t%4) .. +31 of the tile
-        named_bar(1, 128);
-        const int t = ew * 32 + lane, tok = t >> 2, f0 = (t & 3) * 32;
+        // the staged chunk: thread t stores token t/8, features 16 (t%8) .. +15 of the tile
+        named_bar(1, kEpiThreads);
+        const int t = e, tok = t >> 3, f0 = (t & 7) * 16;
         const int col = col0 + tok;
         if (col < p.N) {
             if constexpr (PASS == 1) {
@@ -395,28 +398,29 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                     reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(sm.stg) + tok * kBM + f0);
                 uint4* dst = reinterpret_cast<uint4*>(ep.xb + static_cast<size_t>(col) * ep.ld_out + mt * kBM + f0);
 #pragma unroll
-                for (int i = 0; i < 4; ++i) dst[i] = src[i];
+                for (int i = 0; i < 2; ++i) dst[i] = src[i];
             } else {
-                const float4* src = reinterpret_cast<const float4*>(reinterpret_cast<const float*>(sm.stg) + tok * kBM + f0);
+                const float4* src =
+                    reinterpret_cast<const float4*>(reinterpret_cast<const float*>(sm.stg2) + tok * kBM + f0);
                 float4* dst = reinterpret_cast<float4*>(ep.out + static_cast<size_t>(col) * ep.ld_out + mt * kBM + f0);
 #pragma unroll
-                for (int i = 0; i < 8; ++i) dst[i] = src[i];
+                for (int i = 0; i < 4; ++i) dst[i] = src[i];
             }
         }
-        named_bar(1, 128);  // the staging memory is free again
+        named_bar(1, kEpiThreads);  // the staging memory is free again
     }
     if constexpr (EPI == EPI_RESID && PASS != 1) {
-        named_bar(1, 128);
-        if (ew == 0) {
+        named_bar(1, kEpiThreads);
+        if (e < 32) {
             const int col = col0 + lane;
             const float* rd = sm.red + (c_in / 32) * 128;
             if (col < p.N)
                 ep.sq_out[static_cast<size_t>(mt) * p.N + col] = ((rd[lane] + rd[32 + lane]) + rd[64 + lane]) + rd[96 + lane];
         }
-        named_bar(1, 128);
+        named_bar(1, kEpiThreads);
     } else if constexpr (EPI == EPI_LMHEAD) {
-        named_bar(1, 128);
-        if (ew == 0) {  // merge the four row quarters in a fixed order
+        named_bar(1, kEpiThreads);
+        if (e < 32) {  // merge the four row quarters in a fixed order
             const int col = col0 + lane;
             float m = -INFINITY, s = 0.0f;
             int idx = INT_MAX;
@@ -448,18 +452,19 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                 o[2] = __int_as_float(idx);
             }
         }
-        named_bar(1, 128);
+        named_bar(1, kEpiThreads);
     }
 }
 
 // ================================================================== chained projections
-// k_chain runs the phases of a ChainArgs in one launch, one CTA per SM.  Roles (224
+// k_chain runs the phases of a ChainArgs in one launch, one CTA per SM.  Roles (352
 // threads): warp 0 = weight producer (never waits on data: weights are constant, so it runs
 // ahead by the whole ring, across phase boundaries), warp 6 = operand producer (waits for
 // the completion flag of the tile that writes each X k-block), warp 1 = TMEM owner and MMA
-// issuer, warps 2..5 = epilogue.  Ring stages, TMEM accumulators and their barriers are
-// shared by all phases; a running iteration counter gives every stage its use parity.
-constexpr int kChainThreads = 224;
+// issuer, warps 2..5 and 7..10 = epilogue (two warps per TMEM lane quarter).  Ring stages,
+// TMEM accumulators and their barriers are shared by all phases; a running iteration counter
+// gives every stage its use parity.
+constexpr int kChainThreads = 64 + 32 + 32 * kEpiWarps;
 constexpr int kMaxDepTiles = 256;  // the operand producer keeps a readiness bit per producing tile: 8 per lane
 
 struct ChainEpiState {
@@ -498,8 +503,10 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
     const EpiArgs& ep = P.ep;
     int* status = ca.status;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int ew = warp - 2;
-    const int quarter = warp & 3;
+    const int ew = warp < 6 ? warp - 2 : warp - 3;  // epilogue warps 2..5 and 7..10
+    const int e = ew * 32 + lane;                     // epilogue thread
+    const int half = ew >> 2;                         // columns 16 half .. +15 of every chunk
+    const int quarter = warp & 3;                     // TMEM lane quarter = tile rows 32 quarter ..
     const int rt = quarter * 32 + lane;
     const int G = p.grid;
     if (static_cast<int>(blockIdx.x) >= G) return;
@@ -520,13 +527,13 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             for (int i = lane; i < n; i += 32)
                 if (!wait_flag(qdone + i, tag, s_abort, status)) break;
         }
-        if (named_bar_any(1, 128, *s_abort != 0)) return;
+        if (named_bar_any(1, kEpiThreads, *s_abort != 0)) return;
     }
     if (tr && threadIdx.x == 64) tr[kTrDepWait] = global_ns();
     if constexpr (EPI == EPI_QKV) {
-        for (int b = ew * 32 + lane; b < ep.n_seq; b += 128) esm.kvs[b] = ep.seq_kv[b];
-        esm.theta[rt] = ep.theta[(rt % ep.hd) >> 1];
-        named_bar(1, 128);
+        for (int b = e; b < ep.n_seq; b += kEpiThreads) esm.kvs[b] = ep.seq_kv[b];
+        if (half == 0) esm.theta[rt] = ep.theta[(rt % ep.hd) >> 1];
+        named_bar(1, kEpiThreads);
     }
     const int nchunks = p.ntile / 32;
     constexpr int kPass1 = EPI == EPI_RESID ? 1 : 0;  // the residual epilogue runs in two passes
@@ -538,15 +545,15 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                   : 0u;
     // Wide residual tiles (no TMEM room for the old x): each 32-token chunk of the old fp32
     // residual is copied into shared memory (two buffers, chunk c in buffer c % 2) by cp.async,
-    // 16 bytes a copy, thread t taking token t/4's rows 32 (t%4) .. +31, one chunk ahead of
-    // its use; x_chunk starts the next chunk's copies, then waits for this chunk's.
+    // 16 bytes a copy, epilogue thread t < 128 taking token t/4's rows 32 (t%4) .. +31, one
+    // chunk ahead of its use; x_chunk starts the next chunk's copies, then waits for this chunk's.
     const bool use_xs = EPI == EPI_RESID && esm.xs != nullptr && (ep.ld_out & 3) == 0 &&
                         (reinterpret_cast<uintptr_t>(ep.out) & 15) == 0;
     auto x_fetch = [&](int fmt, int fnt, int c) {
-        const int t = ew * 32 + lane, tok = t >> 2, q = t & 3;
+        const int t = e, tok = t >> 2, q = t & 3;
         const int col = fnt * p.ntile + c * 32 + tok;
         float* buf = esm.xs + (c & 1) * (32 * kBM);
-        if (col < p.N) {
+        if (t < 128 && col < p.N) {
             const int f0 = fmt * kBM + q * 32;
             const float* src = ep.out + static_cast<size_t>(col) * ep.ld_out + f0;
 #pragma unroll
@@ -560,12 +567,12 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         if (c + 1 < nchunks) x_fetch(cmt, cnt, c + 1);
         else cp_async_commit();
         cp_async_wait<1>();
-        named_bar(1, 128);
+        named_bar(1, kEpiThreads);
         return esm.xs + (c & 1) * (32 * kBM);
     };
     int rs_nt = -1, ids_nt = -1;
     long long prepared = -1;
-    float v[32];
+    float v[16];
     // Work a finisher needs before its accumulator: the RMSNorm scale of its token tile, the
     // LM head's current ids of the token tile, and (residual, 32-token tiles) the old x staged
     // in TMEM.  Done as early as possible: for a contributor tile, ahead of it for the finisher
@@ -577,17 +584,17 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         const int pmt = static_cast<int>(ptile - static_cast<long long>(pnt) * p.m_tiles);
         if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
             if (ep.sq_in && pnt != rs_nt) {
-                compute_norm_scale(ep, p, pnt, esm, ew * 32 + lane);
+                compute_norm_scale(ep, p, pnt, esm, e);
                 rs_nt = pnt;
             }
         }
         if constexpr (EPI == EPI_LMHEAD) {
             if (pnt != ids_nt) {
-                for (int c = ew * 32 + lane; c < p.ntile; c += 128) {
+                for (int c = e; c < p.ntile; c += kEpiThreads) {
                     const int col = pnt * p.ntile + c;
                     esm.kvs[c] = col < p.N ? ep.cur_tok[col] : -1;
                 }
-                named_bar(1, 128);
+                named_bar(1, kEpiThreads);
                 ids_nt = pnt;
             }
         }
@@ -597,11 +604,11 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                 const int row = pmt * kBM + rt;
                 for (int c = 0; c < nchunks; ++c) {
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        const int col = pnt * p.ntile + c * 32 + j;
+                    for (int j = 0; j < 16; ++j) {
+                        const int col = pnt * p.ntile + c * 32 + half * 16 + j;
                         v[j] = (row < p.M && col < p.N) ? ep.out[static_cast<size_t>(col) * ep.ld_out + row] : 0.0f;
                     }
-                    tmem_st_32x32(t_x + static_cast<uint32_t>(c * 32), v);
+                    tmem_st_32x16(t_x + static_cast<uint32_t>(c * 32 + half * 16), v);
                 }
             }
         }
@@ -626,7 +633,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         if (finisher) prepare(tile);
         else if (tend < it1) prepare(tile + 1);
         mbar_wait(&tfull[es.acc], es.acc_phase, s_abort, status);
-        if (named_bar_any(1, 128, *s_abort != 0)) {
+        if (named_bar_any(1, kEpiThreads, *s_abort != 0)) {
             cp_async_wait<0>();  // no copy lands in shared memory after the launch has ended
             return;
         }
@@ -643,23 +650,23 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                 const float* xs = x_chunk(mt, nt, c);
                 epilogue_c32<EPI, kPass1>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt,
                                           t_acc + static_cast<uint32_t>(c * 32),
-                                          t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, xs, esm, ew, quarter, lane,
-                                          status);
+                                          t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, xs, esm, e, half, quarter,
+                                          lane, status);
             }
         } else if (!reducer) {
             float* my_part = P.partials + static_cast<size_t>(blockIdx.x) * slot_floats;
             for (int c = 0; c < nchunks; ++c) {
-                tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);
+                tmem_ld_32x16(t_acc + static_cast<uint32_t>(c * 32 + half * 16), v);
                 float4* dst = reinterpret_cast<float4*>(my_part);
 #pragma unroll
-                for (int j = 0; j < 8; ++j)
-                    dst[static_cast<size_t>(c * 8 + j) * kBM + rt] =
+                for (int j = 0; j < 4; ++j)
+                    dst[static_cast<size_t>(c * 8 + half * 4 + j) * kBM + rt] =
                         make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
             }
             // the partial is in registers' way out: the accumulator is free again
             tc_fence_before();
             mbar_arrive(&tempty[es.acc]);
-            named_bar(1, 128);
+            named_bar(1, kEpiThreads);
             if (threadIdx.x == 64) {  // part q of the tile publishes its partial on flag q
                 if (tr) tr[kTrPartStored] = global_ns();
                 st_release(&P.tickets[tile * kTicketStride + (static_cast<int>(blockIdx.x) - c_first)], tag);
@@ -667,19 +674,24 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         }
         if (reducer) {
             // Part q's partial, chunk c (32 columns), is the contiguous 16 KB slice [c*8 + j][row]
-            // float4.  Its slices go through staging slot (q-1) % 2, each bulk copy issued as
-            // soon as part q has published (flag q == tag) and the slot's previous slice is added:
-            // the early parts' slices arrive while the late ones still compute.  The sum runs over
+            // float4.  The slices go through the two staging slots in one stream, chunk-major
+            // (slice s = chunk s / (nparts-1), part s % (nparts-1) + 1, slot s % 2), two in flight:
+            // each copy is issued as soon as its part has published (flag q == tag) and its slot's
+            // previous slice is added, so the next chunk's slices arrive during this chunk's
+            // epilogue and the early parts' while the late ones still compute.  The sum runs over
             // q in order, so it does not depend on the arrival order.
             const int nparts = c_last - c_first + 1;
+            const int np1 = nparts - 1;
+            const int nslices = nchunks * np1;
             int* flags = &P.tickets[tile * kTicketStride];
             constexpr uint32_t slice_bytes = 32 * kBM * 4;
             uint32_t ready = 0;     // warp 2: parts seen published (bit q)
             uint32_t inflight = 0;  // thread 64: slots with a copy not yet waited for
-            // warp 2, warp-uniform: make sure part q has published, polling every part's flag at
-            // once (lane i reads flag i, so one round trip covers them all), then thread 64
-            // issues the copy of q's chunk-c slice into slot (q-1) % 2
-            auto issue = [&](int q, int c) {
+            // warp 2, warp-uniform: make sure slice s's part has published, polling every part's
+            // flag at once (lane i reads flag i, so one round trip covers them all), then thread
+            // 64 issues the copy
+            auto issue = [&](int si) {
+                const int c = si / np1, q = si - c * np1 + 1;
                 if (c == 0) {
                     const long long t0 = spin_clock();
                     while (!(ready >> q & 1u)) {
@@ -699,7 +711,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                     }
                 }
                 if (lane == 0) {
-                    const int sl = (q - 1) & 1;
+                    const int sl = si & 1;
                     fence_proxy_async_global();
                     fence_proxy_async_smem();  // the slot was last touched by generic accesses
                     mbar_arrive_expect_tx(redbar + sl, slice_bytes);
@@ -711,32 +723,33 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                 }
             };
             if (tr && threadIdx.x == 64) tr[kTrPartStored] = global_ns();
+            if (ew == 0) {
+                if (nslices > 0) issue(0);
+                if (nslices > 1) issue(1);
+            }
             bool stop = false;
+            int si = 0;
             for (int c = 0; c < nchunks && !stop; ++c) {
-                if (ew == 0) {
-                    if (nparts > 1) issue(1, c);
-                    if (nparts > 2) issue(2, c);
-                }
-                tmem_ld_32x32(t_acc + static_cast<uint32_t>(c * 32), v);  // own (first) k-range
-                for (int q = 1; q < nparts; ++q) {
-                    const int sl = (q - 1) & 1;
+                tmem_ld_32x16(t_acc + static_cast<uint32_t>(c * 32 + half * 16), v);  // own (first) k-range
+                for (int q = 1; q < nparts; ++q, ++si) {
+                    const int sl = si & 1;
                     mbar_wait(redbar + sl, (es.red_phase >> sl) & 1u, s_abort, status);
                     es.red_phase ^= 1u << sl;
                     if (threadIdx.x == 64) inflight &= ~(1u << sl);
                     const float4* src = reinterpret_cast<const float4*>(red_stage + static_cast<size_t>(sl) * slice_bytes);
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) {
-                        const float4 a = src[j * kBM + rt];
+                    for (int j = 0; j < 4; ++j) {
+                        const float4 a = src[(half * 4 + j) * kBM + rt];
                         v[4 * j] += a.x;
                         v[4 * j + 1] += a.y;
                         v[4 * j + 2] += a.z;
                         v[4 * j + 3] += a.w;
                     }
-                    if (named_bar_any(1, 128, *s_abort != 0)) {  // the slot is free again (or the launch failed)
+                    if (named_bar_any(1, kEpiThreads, *s_abort != 0)) {  // the slot is free again (or the launch failed)
                         stop = true;
                         break;
                     }
-                    if (ew == 0 && q + 2 < nparts) issue(q + 2, c);
+                    if (ew == 0 && si + 2 < nslices) issue(si + 2);
                 }
                 if (stop) break;
                 if (tr && threadIdx.x == 64 && c == 0) {
@@ -745,12 +758,12 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                     tr[kTrIsLast] = 1;
                 }
                 // the sum goes back into the (still owned) accumulator, then the compact epilogue
-                tmem_st_32x32(t_acc + static_cast<uint32_t>(c * 32), v);
+                tmem_st_32x16(t_acc + static_cast<uint32_t>(c * 32 + half * 16), v);
                 const float* xs = x_chunk(mt, nt, c);
                 epilogue_c32<EPI, kPass1>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt,
                                           t_acc + static_cast<uint32_t>(c * 32),
-                                          t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, xs, esm, ew, quarter, lane,
-                                          status);
+                                          t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, xs, esm, e, half, quarter,
+                                          lane, status);
             }
             if (threadIdx.x == 64) {
                 if (stop) {  // let copies in flight land before the shared memory is released
@@ -770,7 +783,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         }
         if (tr && threadIdx.x == 64) tr[kTrEpiPass1] = global_ns();
         if (finisher && P.done) {  // publish the finished tile to the next phase's operand producer
-            named_bar(1, 128);
+            named_bar(1, kEpiThreads);
             if (threadIdx.x == 64) {
                 st_release(&P.done[mt * p.n_tiles + nt], tag);
                 if (tr) tr[kTrPublished] = global_ns();
@@ -780,10 +793,10 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             if (finisher) {  // then the fp32 residual and the RMSNorm sums, for the later phases' epilogues
                 for (int c = 0; c < nchunks; ++c)
                     epilogue_c32<EPI, 2>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt,
-                                         t_acc + static_cast<uint32_t>(c * 32), 0u, nullptr, esm, ew, quarter, lane,
-                                         status);
+                                         t_acc + static_cast<uint32_t>(c * 32), 0u, nullptr, esm, e, half, quarter,
+                                         lane, status);
                 if (P.done2) {
-                    named_bar(1, 128);
+                    named_bar(1, kEpiThreads);
                     if (threadIdx.x == 64) st_release(&P.done2[mt * p.n_tiles + nt], tag);
                 }
             }
@@ -811,14 +824,15 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     uint8_t* sA = smem;
     uint8_t* sB = sA + static_cast<size_t>(S) * kABytes;
     uint8_t* red_stage = sB + static_cast<size_t>(S) * b_bytes;
-    float* tail = reinterpret_cast<float*>(red_stage + ca.red_bytes + ca.xs_bytes);
+    float* tail = reinterpret_cast<float*>(red_stage + ca.red_bytes + ca.xs_bytes + ca.stg_bytes);
     EpiSmem esm;
     esm.xs = ca.xs_bytes ? reinterpret_cast<float*>(red_stage + ca.red_bytes) : nullptr;
     esm.rs = tail;
     esm.red = tail + 256;
     esm.kvs = reinterpret_cast<int*>(tail + 256 + 1024);
     esm.theta = tail + 256 + 1024 + 256;
-    esm.stg = red_stage;
+    esm.stg = ca.stg_bytes ? red_stage + ca.red_bytes + ca.xs_bytes : red_stage;
+    esm.stg2 = red_stage;
     float* after = tail + 256 + 1024 + 256 + 128;
     uint64_t* full = reinterpret_cast<uint64_t*>(after);
     uint64_t* empty = full + S;
@@ -840,7 +854,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&tfull[a], 1);
-            mbar_init(&tempty[a], 128);
+            mbar_init(&tempty[a], kEpiThreads);
         }
         mbar_init(drain, 1);
         mbar_init(&redbar[0], 1);
@@ -1215,14 +1229,15 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
     ca.tmem_cols = pow2ceil(2 * ca.acc_cols + ca.x_cols);
     ca.red_bytes = 2 * 32 * kBM * 4;  // two 32-column partial slices per bulk-copy round
     const int stage_bytes = static_cast<int>(kABytes) + ntile * kBK * 2;
-    // the old residual of wide tiles, staged in shared memory two 32-token chunks at a time,
-    // where that leaves the ring at least 3 stages
+    // tiles of more than one 32-token chunk: their own 8 KB for the bf16 output staging; wide
+    // tiles: the old residual staged in shared memory two chunks at a time, where that leaves
+    // the ring at least 3 stages
+    ca.stg_bytes = c32 ? 0 : 32 * kBM * 2;
     ca.xs_bytes = 0;
-    if (ca.x_cols == 0) {
-        const int fixed_xs = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + 2 * 32 * kBM * 4 + 7 * 8 + 16;
-        if ((smem_budget - fixed_xs) / (stage_bytes + 16) >= 3) ca.xs_bytes = 2 * 32 * kBM * 4;
-    }
-    const int fixed = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + ca.xs_bytes + 7 * 8 + 16;
+    const int fixed0 = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + ca.stg_bytes + 7 * 8 + 16;
+    if (ca.x_cols == 0 && (smem_budget - fixed0 - 2 * 32 * kBM * 4) / (stage_bytes + 16) >= 3)
+        ca.xs_bytes = 2 * 32 * kBM * 4;
+    const int fixed = fixed0 + ca.xs_bytes;
     int st = (smem_budget - fixed) / (stage_bytes + 16);
     if (st > 32) st = 32;
     if (st < 2) return false;
