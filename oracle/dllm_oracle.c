@@ -434,27 +434,52 @@ int orc_commit(const orc_sched* s, int mask_id, int n_pos, int32_t* tok, uint8_t
     }
     int m = 0;
     for (int p = c0; p < c1; ++p) m += st[p] == ORC_MASKED;
-    int left = S - step;
-    int k = m == 0 ? 0 : (left <= 1 ? m : (m + left - 1) / left);
-    int* committed = (int*)malloc(sizeof(int) * (size_t)(c1 - c0 + 1));
     int nc = 0;
-    for (int p = c0; p < c1; ++p) {
-        if (st[p] != ORC_MASKED) continue;
-        int rank = 0;
-        for (int q = c0; q < c1; ++q) {
-            if (q == p || st[q] != ORC_MASKED) continue;
-            float a = conf[q - w0], b = conf[p - w0];
-            if (a > b || (a == b && q < p)) rank++;
+    if (s->commit_mode == ORC_COMMIT_THRESHOLD) {
+        /* Sec. 3.3: masked positions at or above theta_visible take their prediction and become
+         * visible, or stable when they also reach theta_stable */
+        for (int p = c0; p < c1; ++p) {
+            if (st[p] != ORC_MASKED || !(conf[p - w0] >= s->theta_visible)) continue;
+            tok[p] = x0[p - w0];
+            if (conf[p - w0] >= s->theta_stable) {
+                st[p] = ORC_STABLE;
+                r.n_stable++;
+            } else {
+                st[p] = ORC_COMMITTED;
+            }
+            nc++;
         }
-        if (rank < k) committed[nc++] = p;
-    }
-    for (int i = 0; i < nc; ++i) {
-        int p = committed[i];
-        tok[p] = x0[p - w0];
-        st[p] = ORC_COMMITTED;
+        /* none did: the most confident masked position (the first of equals) becomes visible */
+        if (nc == 0 && m > 0) {
+            int best = -1;
+            for (int p = c0; p < c1; ++p)
+                if (st[p] == ORC_MASKED && (best < 0 || conf[p - w0] > conf[best - w0])) best = p;
+            tok[best] = x0[best - w0];
+            st[best] = ORC_COMMITTED;
+            nc = 1;
+        }
+    } else {
+        int left = S - step;
+        int k = m == 0 ? 0 : (left <= 1 ? m : (m + left - 1) / left);
+        int* committed = (int*)malloc(sizeof(int) * (size_t)(c1 - c0 + 1));
+        for (int p = c0; p < c1; ++p) {
+            if (st[p] != ORC_MASKED) continue;
+            int rank = 0;
+            for (int q = c0; q < c1; ++q) {
+                if (q == p || st[q] != ORC_MASKED) continue;
+                float a = conf[q - w0], b = conf[p - w0];
+                if (a > b || (a == b && q < p)) rank++;
+            }
+            if (rank < k) committed[nc++] = p;
+        }
+        for (int i = 0; i < nc; ++i) {
+            int p = committed[i];
+            tok[p] = x0[p - w0];
+            st[p] = ORC_COMMITTED;
+        }
+        free(committed);
     }
     r.n_committed = nc;
-    free(committed);
     if (s->use_prefix_cache && s->spec_blocks > 0) {
         int w1 = w0 + T;
         for (int b0 = c1; b0 < w1; b0 += s->block_len) {

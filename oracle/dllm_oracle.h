@@ -46,7 +46,16 @@ typedef struct {
     int spec_trigger;      /* lookahead when masked count <= trigger */
     int spec_blocks;       /* future blocks added to the window; 0 = off */
     int use_prefix_cache;  /* 0 = vanilla full-sequence decoding */
+    int commit_mode;       /* ORC_COMMIT_SCHEDULE or ORC_COMMIT_THRESHOLD */
+    float theta_visible;   /* threshold mode: promotion of a masked position to visible */
 } orc_sched;
+
+/* Commit rules.  SCHEDULE: LLaDA's fixed schedule, ceil(m / (S - step)) of the m masked
+ * positions per step, the most confident first.  THRESHOLD: staged token stabilization
+ * (Sec. 3.3): every masked position whose confidence reaches theta_visible becomes visible
+ * (COMMITTED), STABLE if it also reaches theta_stable; when none reaches theta_visible, the
+ * single most confident one becomes visible, so every step makes progress. */
+enum { ORC_COMMIT_SCHEDULE = 0, ORC_COMMIT_THRESHOLD = 1 };
 
 typedef struct {
     int n_committed, n_remasked, n_stable, n_drafts, block_done, masked_after;

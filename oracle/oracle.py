@@ -46,7 +46,8 @@ class _Cfg(C.Structure):
 class _Sched(C.Structure):
     _fields_ = [("steps_per_block", C.c_int), ("block_len", C.c_int), ("theta_remask", C.c_float),
                 ("theta_stable", C.c_float), ("remask_max", C.c_int), ("spec_trigger", C.c_int),
-                ("spec_blocks", C.c_int), ("use_prefix_cache", C.c_int)]
+                ("spec_blocks", C.c_int), ("use_prefix_cache", C.c_int), ("commit_mode", C.c_int),
+                ("theta_visible", C.c_float)]
 
 
 class _StepOut(C.Structure):
@@ -141,10 +142,13 @@ class OracleSched:
     spec_trigger: int = 8
     spec_blocks: int = 0
     use_prefix_cache: int = 1
+    commit_mode: int = 0          # 0: LLaDA's fixed schedule; 1: threshold (staged stabilization)
+    theta_visible: float = 0.7
 
     def c(self):
         return _Sched(self.steps_per_block, self.block_len, self.theta_remask, self.theta_stable,
-                      self.remask_max, self.spec_trigger, self.spec_blocks, self.use_prefix_cache)
+                      self.remask_max, self.spec_trigger, self.spec_blocks, self.use_prefix_cache,
+                      self.commit_mode, self.theta_visible)
 
 
 def gen_f32(seed, tensor_id, first, n, sigma):

@@ -256,3 +256,82 @@ def test_revision_zero_threshold_equals_no_revision(tiny_model):
     b = O.Session(tiny_model, O.OracleSched(steps_per_block=8, theta_remask=0.0, theta_stable=0.0), prompt,
                   64).generate()
     assert np.array_equal(a, b)
+
+
+# ------------------------------------------------------------ threshold commit (Sec. 3.3)
+def _threshold(theta_visible=0.7, theta_stable=0.9, **kw):
+    return O.OracleSched(commit_mode=1, theta_visible=theta_visible, theta_stable=theta_stable, **kw)
+
+
+def test_threshold_commit_worked_case(oracle_lib):
+    # a block of eight masked positions, the paper's default thresholds (0.7 visible, 0.9 stable)
+    n, c0, c1 = 12, 2, 10
+    st = np.full(n, O.MASKED, np.uint8)
+    st[:c0] = O.FIXED
+    st[c1:] = O.FIXED
+    tok = np.where(st == O.MASKED, TINY.mask_id, 3).astype(np.int32)
+    conf = np.array([0, 0, 0.95, 0.8, 0.6, 0.2, 0.9, 0.6999, 0.7, 0.5, 0, 0], np.float32)
+    x0 = np.arange(100, 100 + n, dtype=np.int32)
+    tok2, st2, out = O.commit(_threshold(), TINY.mask_id, tok, st, 0, n, c0, c1, 0, x0, conf, np.zeros(n, np.float32))
+    want = [O.FIXED, O.FIXED, O.STABLE, O.COMMITTED, O.MASKED, O.MASKED, O.STABLE, O.MASKED, O.COMMITTED, O.MASKED,
+            O.FIXED, O.FIXED]
+    assert st2.tolist() == want
+    assert tok2.tolist() == [3, 3, 102, 103, TINY.mask_id, TINY.mask_id, 106, TINY.mask_id, 108, TINY.mask_id, 3, 3]
+    assert out["n_committed"] == 4 and out["n_stable"] == 2 and out["masked_after"] == 4 and not out["block_done"]
+
+
+def test_threshold_fallback_promotes_the_most_confident(oracle_lib):
+    # nothing reaches theta_visible: exactly one position, the first of the most confident, becomes visible
+    n, c0, c1 = 10, 0, 10
+    st = np.full(n, O.MASKED, np.uint8)
+    tok = np.full(n, TINY.mask_id, np.int32)
+    conf = np.array([0.1, 0.5, 0.3, 0.5, 0.2, 0.0, 0.5, 0.4, 0.1, 0.1], np.float32)
+    x0 = np.arange(n, dtype=np.int32) + 7
+    tok2, st2, out = O.commit(_threshold(), TINY.mask_id, tok, st, 0, n, c0, c1, 5, x0, conf, np.zeros(n, np.float32))
+    assert out["n_committed"] == 1 and out["n_stable"] == 0 and out["masked_after"] == 9
+    assert st2[1] == O.COMMITTED and tok2[1] == 8
+    assert int((st2 == O.MASKED).sum()) == 9
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_threshold_reduces_to_the_schedule_rule(oracle_lib, seed):
+    # theta_visible = 0: every masked position is taken, as the schedule does on a block's last step;
+    # theta_visible unreachable: one per step, the schedule's top-1 (k = 1 when m steps are left)
+    n, c0, c1 = 48, 8, 40
+    rng = np.random.default_rng(seed)
+    st = np.where(rng.random(n) < 0.6, O.MASKED, O.COMMITTED).astype(np.uint8)
+    tok = np.where(st == O.MASKED, TINY.mask_id, 1).astype(np.int32)
+    conf = I.scripted_confidences(n, seed=seed, ties=True)
+    x0 = rng.integers(0, 1000, n).astype(np.int32)
+    tc = np.zeros(n, np.float32)
+    m = int((st[c0:c1] == O.MASKED).sum())
+    S = 64
+    all_t = O.commit(_threshold(0.0, 2.0, steps_per_block=S), TINY.mask_id, tok, st, 0, n, c0, c1, 0, x0, conf, tc)
+    all_s = O.commit(O.OracleSched(steps_per_block=S), TINY.mask_id, tok, st, 0, n, c0, c1, S - 1, x0, conf, tc)
+    assert np.array_equal(all_t[0], all_s[0]) and np.array_equal(all_t[1], all_s[1])
+    assert all_t[2]["n_committed"] == m and all_t[2]["block_done"]
+    one_t = O.commit(_threshold(2.0, 2.0, steps_per_block=S), TINY.mask_id, tok, st, 0, n, c0, c1, 0, x0, conf, tc)
+    one_s = O.commit(O.OracleSched(steps_per_block=S), TINY.mask_id, tok, st, 0, n, c0, c1, S - m, x0, conf, tc)
+    assert np.array_equal(one_t[0], one_s[0]) and np.array_equal(one_t[1], one_s[1])
+    assert one_t[2]["n_committed"] == 1
+
+
+def test_threshold_session_blocks_progress_and_finish(tiny_model):
+    # unreachable visibility: one commit per step, block_len steps per block; theta_visible = 0: one step
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=31)
+    for tv, steps_per_block in ((2.0, 32), (0.0, 1)):
+        sess = O.Session(tiny_model, _threshold(tv, 2.0, steps_per_block=8), prompt, 64)
+        sess.prefill()
+        blocks = 0
+        while sess.begin_block():
+            counts = []
+            while True:
+                out = sess.step()
+                counts.append(out["n_committed"])
+                assert out["n_committed"] >= 1
+                if out["block_done"]:
+                    break
+            assert len(counts) == steps_per_block and sum(counts) == 32
+            blocks += 1
+        tok, st, kv = sess.state()
+        assert blocks == 2 and kv == 96 and not (tok[32:] == TINY.mask_id).any()
