@@ -67,8 +67,17 @@ typedef struct {
     uint64_t weight_seed;
 } dllm_config;
 
-/* Decoding schedule.  steps_per_block = S; the step-s commit count is
- * ceil(m / (S - s)) for m masked positions of the current block.
+/* Commit rules (dllm_sched.commit_mode). */
+enum { DLLM_COMMIT_SCHEDULE = 0, DLLM_COMMIT_THRESHOLD = 1 };
+
+/* Decoding schedule.  steps_per_block = S.  commit_mode DLLM_COMMIT_SCHEDULE
+ * (LLaDA's fixed schedule): the step-s commit count is ceil(m / (S - s)) for
+ * m masked positions of the current block, the most confident first.
+ * DLLM_COMMIT_THRESHOLD (staged token stabilization, Sec. 3.3): every masked
+ * position whose confidence reaches theta_visible becomes COMMITTED (visible),
+ * STABLE if it also reaches theta_stable; when none reaches theta_visible the
+ * single most confident one becomes COMMITTED, so a block takes between 1 and
+ * block_len steps (plus re-masks); S is then only the revision horizon.
  * theta_remask > 0 enables the revision pass: committed tokens whose
  * current-id probability is >= theta_stable become STABLE, and at most
  * remask_max of those below theta_remask (lowest first) are re-masked; it is
@@ -85,6 +94,8 @@ typedef struct {
     int spec_trigger;
     int spec_blocks;
     int use_prefix_cache;
+    int commit_mode;      /* DLLM_COMMIT_SCHEDULE or DLLM_COMMIT_THRESHOLD */
+    float theta_visible;  /* threshold mode only */
 } dllm_sched;
 
 /* Result of one denoising step, summed over the batch (block_done: all). */

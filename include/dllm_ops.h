@@ -82,7 +82,8 @@ int dllm_op_lmhead(const void* W, const void* X, const int32_t* cur, int32_t* x0
                    float* logits, int V, int N, int d, int mask_id, void* stream);
 
 /* One commit / re-mask / draft pass on HOST arrays of one sequence
- * (Sec. 2.1 commit, Sec. 3.2 drafts, Sec. 3.3 revision): tok int32 and
+ * (Sec. 2.1 commit, Sec. 3.2 drafts, Sec. 3.3 revision and staged token
+ * stabilization; commit_mode / theta_visible as in dllm_sched): tok int32 and
  * status uint8 [n_pos] are updated in place; x0, conf, tokconf [T] are
  * indexed by window offset; window [w0, w0+T), current block [c0, c1),
  * step index within the block.  sched as in dllm.h; block_len = draft block
@@ -90,7 +91,7 @@ int dllm_op_lmhead(const void* W, const void* X, const int32_t* cur, int32_t* x0
 int dllm_op_commit(int32_t* tok, uint8_t* status, int n_pos, int w0, int T, int c0, int c1, int step,
                    const int32_t* x0, const float* conf, const float* tokconf, int steps_per_block,
                    float theta_remask, float theta_stable, int remask_max, int spec_blocks, int use_prefix_cache,
-                   int block_len, int mask_id, int* out6);
+                   int block_len, int mask_id, int commit_mode, float theta_visible, int* out6);
 
 #ifdef __cplusplus
 }

@@ -9,6 +9,7 @@ ctypes binding.
 """
 from .build import build  # noqa: F401
 from .dllm import (  # noqa: F401
-    COMMITTED, DRAFT, FIXED, MASKED, STABLE, Config, Context, DllmError, Sched, dllm_arena_bytes, dllm_op_attention,
+    COMMIT_SCHEDULE, COMMIT_THRESHOLD, COMMITTED, DRAFT, FIXED, MASKED, STABLE, Config, Context, DllmError, Sched,
+    dllm_arena_bytes, dllm_op_attention,
     dllm_op_commit, dllm_op_gemm, dllm_op_lmhead, lib,
 )

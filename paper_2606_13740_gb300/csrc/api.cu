@@ -385,6 +385,8 @@ static int step_kernels(dllm_ctx* ctx, int T) {
     a.block_len = ctx->cfg.block_len;
     a.theta_remask = ctx->sched.theta_remask;
     a.theta_stable = ctx->sched.theta_stable;
+    a.commit_mode = ctx->sched.commit_mode;
+    a.theta_visible = ctx->sched.theta_visible;
     cudaError_t ce = launch_commit(a, ctx->stream);
     mark(ctx, DLLM_K_COMMIT);
     ctx->in_step = false;
@@ -570,7 +572,9 @@ static int start_request(dllm_ctx* ctx, const dllm_sched* sched, int batch, int 
                          const int32_t* prompt, int P_random, uint64_t kv_seed) {
     const dllm_config& c = ctx->cfg;
     if (!sched || batch < 1 || Lp < 0 || gen_len < 1) return fail(ctx, DLLM_EINVAL, "bad request arguments");
-    if (sched->steps_per_block < 1 || sched->remask_max < 0 || sched->spec_blocks < 0)
+    if (sched->steps_per_block < 1 || sched->remask_max < 0 || sched->spec_blocks < 0 ||
+        (sched->commit_mode != DLLM_COMMIT_SCHEDULE && sched->commit_mode != DLLM_COMMIT_THRESHOLD) ||
+        !(sched->theta_visible == sched->theta_visible))
         return fail(ctx, DLLM_EINVAL, "bad schedule");
     if (batch > c.max_batch) return fail(ctx, DLLM_ECAPACITY, "batch %d > max_batch %d", batch, c.max_batch);
     const int n_pos = Lp + gen_len;
@@ -787,7 +791,9 @@ int dllm_generate(dllm_ctx* ctx, const dllm_sched* sched, int batch, const int32
     dllm_stats stt{};
     while ((rc = dllm_begin_block(ctx)) == DLLM_OK) {
         dllm_step_out o{};
-        for (int guard = 0; guard < 4 * sched->steps_per_block + 4; ++guard) {
+        // a block finishes within S steps (schedule), or within the revision horizon S plus one
+        // step per position (threshold: every step commits at least one)
+        for (int guard = 0; guard < 4 * sched->steps_per_block + 4 + ctx->cfg.block_len; ++guard) {
             rc = dllm_denoise_step(ctx, &o);
             if (rc) return rc;
             stt.steps++;

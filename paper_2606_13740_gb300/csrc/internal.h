@@ -219,6 +219,8 @@ struct CommitArgs {
     int B, T, mask_id, use_cache;
     int S, remask_max, spec_blocks, block_len;
     float theta_remask, theta_stable;
+    int commit_mode;     // DLLM_COMMIT_SCHEDULE / DLLM_COMMIT_THRESHOLD (dllm.h)
+    float theta_visible;
 };
 cudaError_t launch_commit(const CommitArgs& a, cudaStream_t st, bool pdl = true);
 

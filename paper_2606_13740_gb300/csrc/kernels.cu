@@ -589,9 +589,13 @@ cudaError_t launch_lmhead_reduce(const float* lm_part, const float* zcur, const 
 //  1. revision (theta_remask > 0, not the last step): COMMITTED tokens of the
 //     current block with tokconf >= theta_stable become STABLE; of those below
 //     theta_remask, the remask_max lowest (ties: lower position) are re-masked;
-//  2. k = ceil(m / (S - step)) for the m masked positions of the block;
-//  3. the k masked positions with the highest conf (ties: lower position)
-//     take their argmax and become COMMITTED;
+//  2. schedule mode: k = ceil(m / (S - step)) for the m masked positions of
+//     the block, and the k masked positions with the highest conf (ties: lower
+//     position) take their argmax and become COMMITTED;
+//  3. threshold mode (staged token stabilization): the masked positions with
+//     conf >= theta_visible take their argmax and become COMMITTED (STABLE at
+//     conf >= theta_stable); when there is none, the single most confident one
+//     (ties: lower position) becomes COMMITTED;
 //  4. with the prefix cache and lookahead on, each future block inside the
 //     window drafts its single most confident masked position.
 __global__ void __launch_bounds__(256) k_commit(CommitArgs a) {
@@ -652,9 +656,50 @@ __global__ void __launch_bounds__(256) k_commit(CommitArgs a) {
     atomicAdd(&s_cnt[5], mloc);
     __syncthreads();
     const int m = s_cnt[5];
+    if (a.commit_mode == 1) {
+        for (int i = threadIdx.x; i < n; i += blockDim.x) {
+            const int p = c0 + i;
+            const float v = conf[p - w0];
+            if (st[p] == 1 && v >= a.theta_visible) {
+                tok[p] = x0[p - w0];
+                const bool stable = v >= a.theta_stable;
+                st[p] = stable ? 3 : 2;
+                atomicAdd(&s_cnt[0], 1);
+                if (stable) atomicAdd(&s_cnt[2], 1);
+            }
+        }
+        __syncthreads();
+        if (s_cnt[0] == 0 && m > 0 && threadIdx.x < 32) {  // the most confident masked position
+            float bv = -INFINITY;
+            int bp = INT_MAX;
+            for (int p = c0 + static_cast<int>(threadIdx.x); p < c1; p += 32) {
+                if (st[p] != 1) continue;
+                const float v = conf[p - w0];
+                if (v > bv || (v == bv && p < bp)) {
+                    bv = v;
+                    bp = p;
+                }
+            }
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) {
+                const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+                const int op = __shfl_xor_sync(0xffffffffu, bp, off);
+                if (ov > bv || (ov == bv && op < bp)) {
+                    bv = ov;
+                    bp = op;
+                }
+            }
+            if (threadIdx.x == 0 && bp != INT_MAX) {
+                tok[bp] = x0[bp - w0];
+                st[bp] = 2;
+                s_cnt[0] = 1;
+            }
+        }
+        __syncthreads();
+    }
     const int left = a.S - step;
-    const int k = m == 0 ? 0 : (left <= 1 ? m : (m + left - 1) / left);
-    // commit: the k masked positions ranked by (conf descending, position ascending)
+    const int k = a.commit_mode == 1 || m == 0 ? 0 : (left <= 1 ? m : (m + left - 1) / left);
+    // schedule mode: the k masked positions ranked by (conf descending, position ascending)
     for (int i = threadIdx.x; i < n; i += blockDim.x) {
         const int p = c0 + i;
         uint8_t sel = 0;

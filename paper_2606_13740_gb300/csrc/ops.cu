@@ -199,9 +199,10 @@ int dllm_op_lmhead(const void* W, const void* X, const int32_t* cur, int32_t* x0
 int dllm_op_commit(int32_t* tok, uint8_t* status, int n_pos, int w0, int T, int c0, int c1, int step,
                    const int32_t* x0, const float* conf, const float* tokconf, int steps_per_block,
                    float theta_remask, float theta_stable, int remask_max, int spec_blocks, int use_prefix_cache,
-                   int block_len, int mask_id, int* out6) {
+                   int block_len, int mask_id, int commit_mode, float theta_visible, int* out6) {
     if (!tok || !status || !x0 || !conf || !tokconf || n_pos < 1 || T < 1 || w0 < 0 || w0 + T > n_pos || c0 < w0 ||
-        c1 > w0 + T || c0 > c1 || c1 - c0 > kMaxBlock || steps_per_block < 1 || block_len < 1)
+        c1 > w0 + T || c0 > c1 || c1 - c0 > kMaxBlock || steps_per_block < 1 || block_len < 1 ||
+        (commit_mode != DLLM_COMMIT_SCHEDULE && commit_mode != DLLM_COMMIT_THRESHOLD))
         return op_fail(DLLM_EINVAL, "bad commit arguments");
     if (!use_prefix_cache && w0 != 0) return op_fail(DLLM_EINVAL, "without the prefix cache the window starts at 0");
     DevBuf dtok, dst, dx0, dconf, dtc, dkv, dplan, douts;
@@ -238,6 +239,8 @@ int dllm_op_commit(int32_t* tok, uint8_t* status, int n_pos, int w0, int T, int 
     a.block_len = block_len;
     a.theta_remask = theta_remask;
     a.theta_stable = theta_stable;
+    a.commit_mode = commit_mode;
+    a.theta_visible = theta_visible;
     cudaError_t e = launch_commit(a, nullptr, false);
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) return op_fail(DLLM_ECUDA, "commit: %s", cudaGetErrorString(e));

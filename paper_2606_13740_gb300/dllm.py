@@ -19,6 +19,7 @@ from .build import build as _build_lib
 DLLM_OK, DLLM_DONE = 0, 1
 ERRORS = {-1: "EINVAL", -2: "ENOMEM", -3: "ECUDA", -4: "ETIMEOUT", -5: "ESTATE", -6: "ECAPACITY"}
 FIXED, MASKED, COMMITTED, STABLE, DRAFT = 0, 1, 2, 3, 4
+COMMIT_SCHEDULE, COMMIT_THRESHOLD = 0, 1  # dllm_sched.commit_mode
 
 
 class DllmError(RuntimeError):
@@ -37,7 +38,7 @@ class dllm_config(C.Structure):
 class dllm_sched(C.Structure):
     _fields_ = [("steps_per_block", C.c_int), ("theta_remask", C.c_float), ("theta_stable", C.c_float),
                 ("remask_max", C.c_int), ("spec_trigger", C.c_int), ("spec_blocks", C.c_int),
-                ("use_prefix_cache", C.c_int)]
+                ("use_prefix_cache", C.c_int), ("commit_mode", C.c_int), ("theta_visible", C.c_float)]
 
 
 class dllm_step_out(C.Structure):
@@ -83,7 +84,7 @@ SIGNATURES = {
     "dllm_op_gemm_timed": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P]),
     "dllm_op_attention": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P]),
     "dllm_op_lmhead": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _P]),
-    "dllm_op_commit": (_I, [_P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _I, _F, _F, _I, _I, _I, _I, _I, _P]),
+    "dllm_op_commit": (_I, [_P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _I, _F, _F, _I, _I, _I, _I, _I, _I, _F, _P]),
 }
 
 _lib = None
@@ -154,10 +155,13 @@ class Sched:
     spec_trigger: int = 8
     spec_blocks: int = 0
     use_prefix_cache: int = 1
+    commit_mode: int = COMMIT_SCHEDULE
+    theta_visible: float = 0.7
 
     def c(self):
         return dllm_sched(self.steps_per_block, self.theta_remask, self.theta_stable, self.remask_max,
-                          self.spec_trigger, self.spec_blocks, self.use_prefix_cache)
+                          self.spec_trigger, self.spec_blocks, self.use_prefix_cache, self.commit_mode,
+                          self.theta_visible)
 
 
 def dllm_arena_bytes(cfg: Config) -> int:
@@ -395,6 +399,7 @@ def dllm_op_commit(sched: Sched, mask_id, tok, st, w0, T, c0, c1, step, x0, conf
     out = np.zeros(6, np.int32)
     _check(lib().dllm_op_commit(_p(tok), _p(st), tok.size, w0, T, c0, c1, step, _p(x0), _p(conf), _p(tokconf),
                                 sched.steps_per_block, sched.theta_remask, sched.theta_stable, sched.remask_max,
-                                sched.spec_blocks, sched.use_prefix_cache, block_len, mask_id, _p(out)))
+                                sched.spec_blocks, sched.use_prefix_cache, block_len, mask_id, sched.commit_mode,
+                                sched.theta_visible, _p(out)))
     keys = ("n_committed", "n_remasked", "n_stable", "n_drafts", "block_done", "masked_after")
     return tok, st, dict(zip(keys, (int(v) for v in out)))

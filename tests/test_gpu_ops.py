@@ -167,3 +167,32 @@ def test_commit_bit_exact_vs_oracle(dev, seed):
     assert np.array_equal(gst, ost)
     assert np.array_equal(gt, ot)
     assert gout == {k: oout[k] for k in gout}
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_commit_threshold_bit_exact_vs_oracle(dev, seed):
+    """Staged token stabilization (Sec. 3.3) on random states, ties included: the same
+    positions become visible / stable, the same fallback position, the same counts."""
+    from paper_2606_13740_gb300 import COMMIT_THRESHOLD, Sched, dllm_op_commit
+    rng = np.random.default_rng(1000 + seed)
+    use_cache = int(seed % 4 != 3)
+    spec = int(rng.integers(0, 3)) if use_cache else 0
+    S = int(rng.choice([4, 8, 32]))
+    step = int(rng.integers(0, S))
+    theta = float(rng.choice([0.0, 0.5]))
+    rmax = int(rng.integers(1, 4))
+    tv = float(rng.choice([0.0, 0.3, 0.5, 0.75, 2.0]))
+    ts = float(rng.choice([0.5, 0.9, 2.0]))
+    tok, st, w0, T, c0, c1, x0, conf, tokconf = _random_case(rng, use_cache, spec)
+    gs = Sched(steps_per_block=S, theta_remask=theta, theta_stable=ts, remask_max=rmax, spec_blocks=spec,
+               use_prefix_cache=use_cache, commit_mode=COMMIT_THRESHOLD, theta_visible=tv)
+    os_ = O.OracleSched(steps_per_block=S, block_len=32, theta_remask=theta, theta_stable=ts, remask_max=rmax,
+                        spec_blocks=spec, use_prefix_cache=use_cache, commit_mode=1, theta_visible=tv)
+    gt, gst, gout = dllm_op_commit(gs, 1023, tok, st, w0, T, c0, c1, step, x0, conf, tokconf)
+    ot, ost, oout = O.commit(os_, 1023, tok, st, w0, T, c0, c1, step, x0, conf, tokconf)
+    assert np.array_equal(gst, ost)
+    assert np.array_equal(gt, ot)
+    assert gout == {k: oout[k] for k in gout}
+    m = int((st[c0:c1] == 1).sum())
+    if m:
+        assert gout["n_committed"] >= 1  # every step makes progress

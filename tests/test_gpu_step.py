@@ -141,6 +141,50 @@ def test_speculative_revision_teacher_forced(model):
     ctx.close()
 
 
+@pytest.mark.parametrize("theta_visible,steps_per_block", [(2.0, 32), (0.0, 1)])
+def test_threshold_commit_teacher_forced(model, theta_visible, steps_per_block):
+    """Staged token stabilization at its two exact ends: theta_visible out of reach (the
+    fallback, one position per step, 32 steps per block) and 0 (the whole block at once)."""
+    from paper_2606_13740_gb300 import COMMIT_THRESHOLD, Sched
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=41)
+    osched = O.OracleSched(steps_per_block=8, commit_mode=1, theta_visible=theta_visible, theta_stable=2.0)
+    gsched = Sched(steps_per_block=8, commit_mode=COMMIT_THRESHOLD, theta_visible=theta_visible, theta_stable=2.0)
+    ctx = _gpu_ctx()
+    _, steps, _ = _run_teacher_forced(model, osched, gsched, prompt, 64, ctx)
+    assert steps == 2 * steps_per_block
+    ctx.close()
+
+
+def test_threshold_commit_generation_mid_thresholds(model):
+    """Thresholds inside the tiny model's confidence range: every step commits at least one
+    position, positions reaching theta_stable go straight to STABLE, every block finishes in
+    at most 32 steps, and a rerun gives the same tokens."""
+    from paper_2606_13740_gb300 import COMMIT_THRESHOLD, STABLE, Sched
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=42)
+    sched = Sched(steps_per_block=8, commit_mode=COMMIT_THRESHOLD, theta_visible=0.00256, theta_stable=0.0026)
+    ctx = _gpu_ctx()
+    ctx.dllm_prefill(sched, prompt, 64)
+    blocks, steps, stable_direct = 0, 0, 0
+    while ctx.dllm_begin_block():
+        n = 0
+        while True:
+            out = ctx.dllm_denoise_step()
+            n += 1
+            assert out["n_committed"] >= 1
+            stable_direct += out["n_stable"]
+            if out["block_done"]:
+                break
+        assert 1 <= n <= 32
+        blocks += 1
+        steps += n
+    tok, st, kv = ctx.dllm_get_state()
+    assert blocks == 2 and kv[0] == 96 and not (tok[0, 32:96] == TINY.mask_id).any()
+    assert stable_direct == int((st[0, 32:96] == STABLE).sum())
+    again, _ = ctx.dllm_generate(sched, prompt, 64)
+    assert np.array_equal(again[0], tok[0, 32:96])
+    ctx.close()
+
+
 def test_generate_matches_stepwise_and_is_deterministic(model):
     from paper_2606_13740_gb300 import Sched
     prompt = I.uniform_prompt(64, TINY.vocab, TINY.mask_id)
