@@ -218,21 +218,29 @@ def window_sweep(a):
 
 def generate(a):
     """Whole generations through dllm_generate at LLaDA-8B shape: 256-token prompt, 4 blocks of
-    32 with 32 steps per block (one commit per step); and a 1024-token prompt, 8 blocks, with
-    speculation (window 96 when <= 8 masked) and revision (theta 0.5, at most 1 per step)."""
+    32 with 32 steps per block (one commit per step); a 1024-token prompt, 8 blocks, with
+    speculation (window 96 when <= 8 masked) and revision (theta 0.5, at most 1 per step); and
+    the threshold commit rule (staged token stabilization) on the 256-token prompt with the
+    paper's thresholds (0.7 visible, 0.9 stable; a random-weight model's confidences stay near
+    1/V, so every step takes the single-position fallback) and with theta_visible 0 (a whole
+    block per step: the rule's fastest case)."""
     import time
 
     import numpy as np
 
     import dllm_inputs as I
 
-    from .dllm import Config, Context, Sched
+    from .dllm import COMMIT_THRESHOLD, Config, Context, Sched
 
     out = []
     for name, Lp, gen, sched in (
             ("blocks_p256_g128", 256, 128, Sched(steps_per_block=32)),
             ("spec_revision_p1024_g256", 1024, 256,
-             Sched(steps_per_block=32, spec_trigger=8, spec_blocks=2, theta_remask=0.5, remask_max=1))):
+             Sched(steps_per_block=32, spec_trigger=8, spec_blocks=2, theta_remask=0.5, remask_max=1)),
+            ("threshold_0.7_0.9_p256_g128", 256, 128,
+             Sched(steps_per_block=32, commit_mode=COMMIT_THRESHOLD, theta_visible=0.7, theta_stable=0.9)),
+            ("threshold_0_p256_g128", 256, 128,
+             Sched(steps_per_block=32, commit_mode=COMMIT_THRESHOLD, theta_visible=0.0, theta_stable=0.9))):
         cfg = Config(max_batch=1, max_ctx=Lp + gen, max_window=max(Lp, 96), n_layers=a.layers, **SHAPE_8B)
         ctx = Context(cfg)
         prompt = I.uniform_prompt(Lp, cfg.vocab, cfg.mask_id)
