@@ -282,12 +282,19 @@ static void embed_row(const orc_model* m, int32_t tok, float* out) {
 int orc_forward(const orc_model* m, int T, const int32_t* tok, const int32_t* pos, int P, const float* pk,
                 const float* pv, const int32_t* group, float* out_k, float* out_v, float* logits,
                 int n_layers_run) {
+    return orc_forward_ex(m, T, T, tok, pos, P, pk, pv, group, out_k, out_v, logits, n_layers_run);
+}
+
+int orc_forward_ex(const orc_model* m, int T, int Tk, const int32_t* tok, const int32_t* pos, int P, const float* pk,
+                   const float* pv, const int32_t* group, float* out_k, float* out_v, float* logits,
+                   int n_layers_run) {
     const orc_config* c = &m->c;
     int d = c->d_model, H = c->n_heads, hd = c->head_dim, F = c->ffn, V = c->vocab;
     int qd = H * hd;
     int L = n_layers_run < 0 || n_layers_run > c->n_layers ? c->n_layers : n_layers_run;
     if (L > m->n_gen_layers) return -1;
     if (T <= 0) return 0;
+    if (Tk < 0 || Tk > T) return -1;
     size_t Td = (size_t)T * d;
     float* x = (float*)malloc(sizeof(float) * Td);
     float* h = (float*)malloc(sizeof(float) * Td);
@@ -319,7 +326,7 @@ int orc_forward(const orc_model* m, int T, const int32_t* tok, const int32_t* po
         if (out_v) memcpy(out_v + (size_t)l * T * qd, v, sizeof(float) * (size_t)T * qd);
         const float* lk = P > 0 ? pk + (size_t)l * P * qd : NULL;
         const float* lv = P > 0 ? pv + (size_t)l * P * qd : NULL;
-        int NK = P + T;
+        int NK = P + Tk; /* rows from Tk on are queries only */
 #pragma omp parallel
         {
             double* sc = (double*)malloc(sizeof(double) * (size_t)NK);
@@ -519,6 +526,10 @@ struct orc_session {
     int w0, T, spec_on;
     int32_t* x0;
     float *conf, *tokconf, *margin, *logits;
+    /* sparse cache refresh of the last step: tracked positions and their decisions */
+    int scr_n;
+    int32_t *scr_pos, *scr_x0;
+    float *scr_conf, *scr_tokconf, *scr_margin;
 };
 
 orc_session* orc_session_new(const orc_model* m, const orc_sched* s, int Lp, const int32_t* prompt, int G) {
@@ -548,7 +559,19 @@ void orc_session_free(orc_session* x) {
     if (!x) return;
     free(x->tok); free(x->st); free(x->pk); free(x->pv);
     free(x->x0); free(x->conf); free(x->tokconf); free(x->margin); free(x->logits);
+    free(x->scr_pos); free(x->scr_x0); free(x->scr_conf); free(x->scr_tokconf); free(x->scr_margin);
     free(x);
+}
+
+int orc_scr_decisions(const orc_session* x, int32_t* pos, int32_t* x0, float* conf, float* tokconf, float* margin) {
+    int n = x->scr_n;
+    if (n <= 0) return 0;
+    if (pos) memcpy(pos, x->scr_pos, sizeof(int32_t) * (size_t)n);
+    if (x0) memcpy(x0, x->scr_x0, sizeof(int32_t) * (size_t)n);
+    if (conf) memcpy(conf, x->scr_conf, sizeof(float) * (size_t)n);
+    if (tokconf) memcpy(tokconf, x->scr_tokconf, sizeof(float) * (size_t)n);
+    if (margin) memcpy(margin, x->scr_margin, sizeof(float) * (size_t)n);
+    return n;
 }
 
 int orc_n_pos(const orc_session* x) { return x->n_pos; }
@@ -636,8 +659,24 @@ int orc_denoise_step(orc_session* x, orc_step_out* out, int keep_logits) {
     }
     int T = w1 - w0, P = x->s.use_prefix_cache ? x->kv_len : 0;
     x->w0 = w0; x->T = T; x->spec_on = spec;
-    int32_t* pos = (int32_t*)malloc(sizeof(int32_t) * (size_t)T);
-    for (int t = 0; t < T; ++t) pos[t] = w0 + t;
+    /* sparse cache refresh: the first scr_rows visible (COMMITTED) prefix positions ride along
+     * as query-only rows */
+    int R = x->s.use_prefix_cache ? x->s.scr_rows : 0, nt = 0;
+    if (R > 0 && !x->scr_pos) {
+        x->scr_pos = (int32_t*)calloc((size_t)R, sizeof(int32_t));
+        x->scr_x0 = (int32_t*)calloc((size_t)R, sizeof(int32_t));
+        x->scr_conf = (float*)calloc((size_t)R, sizeof(float));
+        x->scr_tokconf = (float*)calloc((size_t)R, sizeof(float));
+        x->scr_margin = (float*)calloc((size_t)R, sizeof(float));
+    }
+    for (int p = 0; p < x->kv_len && nt < R; ++p)
+        if (x->st[p] == ORC_COMMITTED) x->scr_pos[nt++] = p;
+    x->scr_n = nt;
+    int Tq = T + nt;
+    int32_t* pos = (int32_t*)malloc(sizeof(int32_t) * (size_t)Tq);
+    int32_t* rows = (int32_t*)malloc(sizeof(int32_t) * (size_t)Tq);
+    for (int t = 0; t < T; ++t) { pos[t] = w0 + t; rows[t] = x->tok[w0 + t]; }
+    for (int r = 0; r < nt; ++r) { pos[T + r] = x->scr_pos[r]; rows[T + r] = x->tok[x->scr_pos[r]]; }
     float* pk = NULL;
     float* pv = NULL;
     if (P > 0) {
@@ -649,16 +688,42 @@ int orc_denoise_step(orc_session* x, orc_step_out* out, int keep_logits) {
         }
     }
     free(x->logits);
-    x->logits = (float*)malloc(sizeof(float) * (size_t)T * V);
-    int rc = orc_forward(x->m, T, x->tok + w0, pos, P, pk, pv, NULL, NULL, NULL, x->logits, -1);
-    free(pos); free(pk); free(pv);
-    if (rc) return rc;
+    x->logits = (float*)malloc(sizeof(float) * (size_t)Tq * V);
+    float* nk = nt ? (float*)malloc(sizeof(float) * (size_t)L * Tq * qd) : NULL;
+    float* nv = nt ? (float*)malloc(sizeof(float) * (size_t)L * Tq * qd) : NULL;
+    int rc = orc_forward_ex(x->m, Tq, T, rows, pos, P, pk, pv, NULL, nk, nv, x->logits, -1);
+    free(pos); free(rows); free(pk); free(pv);
+    if (rc) { free(nk); free(nv); return rc; }
     for (int t = 0; t < T; ++t)
         orc_decide(V, c->mask_id, x->logits + (size_t)t * V, x->tok[w0 + t], x->x0 + t, x->conf + t, x->tokconf + t,
                    x->margin + t);
+    for (int r = 0; r < nt; ++r)
+        orc_decide(V, c->mask_id, x->logits + (size_t)(T + r) * V, x->tok[x->scr_pos[r]], x->scr_x0 + r,
+                   x->scr_conf + r, x->scr_tokconf + r, x->scr_margin + r);
     if (!keep_logits) { free(x->logits); x->logits = NULL; }
+    orc_step_out so;
     rc = orc_commit(&x->s, c->mask_id, x->n_pos, x->tok, x->st, w0, T, x->c0, x->c1, x->step, x->x0, x->conf,
-                    x->tokconf, out);
+                    x->tokconf, &so);
+    /* the tracked positions: re-scored, then their refreshed K/V merged at the step boundary */
+    for (int r = 0; r < nt && !rc; ++r) {
+        int p = x->scr_pos[r];
+        float tc = x->scr_tokconf[r];
+        if (tc >= x->s.theta_stable) {
+            x->st[p] = ORC_STABLE;
+            so.n_stable++;
+        } else if (x->s.theta_remask > 0.0f && tc < x->s.theta_remask && x->scr_x0[r] != x->tok[p]) {
+            x->tok[p] = x->scr_x0[r];
+            so.n_revised++;
+            continue;
+        }
+        for (int l = 0; l < L; ++l) {
+            memcpy(x->pk + ((size_t)l * x->n_pos + p) * qd, nk + ((size_t)l * Tq + T + r) * qd, sizeof(float) * qd);
+            memcpy(x->pv + ((size_t)l * x->n_pos + p) * qd, nv + ((size_t)l * Tq + T + r) * qd, sizeof(float) * qd);
+        }
+        so.n_refreshed++;
+    }
+    free(nk); free(nv);
+    if (out) *out = so;
     x->step++;
     return rc;
 }

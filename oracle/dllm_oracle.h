@@ -48,6 +48,7 @@ typedef struct {
     int use_prefix_cache;  /* 0 = vanilla full-sequence decoding */
     int commit_mode;       /* ORC_COMMIT_SCHEDULE or ORC_COMMIT_THRESHOLD */
     float theta_visible;   /* threshold mode: promotion of a masked position to visible */
+    int scr_rows;          /* sparse cache refresh: prefix positions re-scored per step (0 = off) */
 } orc_sched;
 
 /* Commit rules.  SCHEDULE: LLaDA's fixed schedule, ceil(m / (S - step)) of the m masked
@@ -59,7 +60,17 @@ enum { ORC_COMMIT_SCHEDULE = 0, ORC_COMMIT_THRESHOLD = 1 };
 
 typedef struct {
     int n_committed, n_remasked, n_stable, n_drafts, block_done, masked_after;
+    int n_refreshed, n_revised;  /* sparse cache refresh: prefix K/V rows merged, prefix ids revised */
 } orc_step_out;
+
+/* Sparse cache refresh (Sec. 3.3, with the prefix cache on): each step the first scr_rows
+ * prefix positions (ascending) in the visible state (COMMITTED) ride along with the window as
+ * extra query rows at their own positions; they attend to the cached prefix as it stands and
+ * to the window, and add no keys.  After the window's commit pass each of them is re-scored:
+ * at tokconf >= theta_stable it becomes STABLE; below theta_remask (when > 0) with an argmax
+ * other than its id it takes that argmax; otherwise it keeps its id.  Every one that keeps its
+ * id has the K/V computed for it this step written into the cache at its position (the merge
+ * happens at the step boundary: nothing of it is visible inside the step). */
 
 /* ---- counter-based generator (SplitMix64, Steele/Lea/Flood 2014) ---- */
 uint64_t orc_splitmix_at(uint64_t key, uint64_t n);
@@ -94,6 +105,10 @@ void orc_decide(int V, int mask_id, const float* logits, int32_t cur_tok,
 int orc_forward(const orc_model* m, int T, const int32_t* tok, const int32_t* pos,
                 int P, const float* prefix_k, const float* prefix_v, const int32_t* group,
                 float* out_k, float* out_v, float* logits, int n_layers_run);
+/* The same with only the first Tk of the T rows as keys (the rest are queries only). */
+int orc_forward_ex(const orc_model* m, int T, int Tk, const int32_t* tok, const int32_t* pos,
+                   int P, const float* prefix_k, const float* prefix_v, const int32_t* group,
+                   float* out_k, float* out_v, float* logits, int n_layers_run);
 
 /* One commit / re-mask / draft pass (C5-C9 of the scope table) over a
  * single sequence's state arrays (length n_pos).  Pure function. */
@@ -105,6 +120,9 @@ int orc_commit(const orc_sched* s, int mask_id, int n_pos, int32_t* tok, uint8_t
 typedef struct orc_session orc_session;
 orc_session* orc_session_new(const orc_model* m, const orc_sched* s, int Lp, const int32_t* prompt, int gen_len);
 void orc_session_free(orc_session* x);
+/* The last step's tracked prefix positions (sparse cache refresh) and their decisions (arrays
+ * of scr_rows entries, nullable); returns how many there were. */
+int orc_scr_decisions(const orc_session* x, int32_t* pos, int32_t* x0, float* conf, float* tokconf, float* margin);
 int orc_prefill(orc_session* x);
 /* 0: started a block; 1: generation finished (last block appended). */
 int orc_begin_block(orc_session* x);

@@ -47,12 +47,13 @@ class _Sched(C.Structure):
     _fields_ = [("steps_per_block", C.c_int), ("block_len", C.c_int), ("theta_remask", C.c_float),
                 ("theta_stable", C.c_float), ("remask_max", C.c_int), ("spec_trigger", C.c_int),
                 ("spec_blocks", C.c_int), ("use_prefix_cache", C.c_int), ("commit_mode", C.c_int),
-                ("theta_visible", C.c_float)]
+                ("theta_visible", C.c_float), ("scr_rows", C.c_int)]
 
 
 class _StepOut(C.Structure):
     _fields_ = [("n_committed", C.c_int), ("n_remasked", C.c_int), ("n_stable", C.c_int),
-                ("n_drafts", C.c_int), ("block_done", C.c_int), ("masked_after", C.c_int)]
+                ("n_drafts", C.c_int), ("block_done", C.c_int), ("masked_after", C.c_int),
+                ("n_refreshed", C.c_int), ("n_revised", C.c_int)]
 
     def as_dict(self):
         return {k: getattr(self, k) for k, _ in self._fields_}
@@ -100,6 +101,8 @@ def lib():
         L.orc_window.argtypes = [P, P]
         L.orc_step_decisions.restype = I
         L.orc_step_decisions.argtypes = [P, P, P, P, P, P]
+        L.orc_scr_decisions.restype = I
+        L.orc_scr_decisions.argtypes = [P, P, P, P, P, P]
         L.orc_get_state.argtypes = [P, P, P, P]
         L.orc_set_state.argtypes = [P, P, P]
         L.orc_prefix_kv.restype = P
@@ -144,11 +147,12 @@ class OracleSched:
     use_prefix_cache: int = 1
     commit_mode: int = 0          # 0: LLaDA's fixed schedule; 1: threshold (staged stabilization)
     theta_visible: float = 0.7
+    scr_rows: int = 0             # sparse cache refresh: visible prefix positions re-scored per step
 
     def c(self):
         return _Sched(self.steps_per_block, self.block_len, self.theta_remask, self.theta_stable,
                       self.remask_max, self.spec_trigger, self.spec_blocks, self.use_prefix_cache,
-                      self.commit_mode, self.theta_visible)
+                      self.commit_mode, self.theta_visible, self.scr_rows)
 
 
 def gen_f32(seed, tensor_id, first, n, sigma):
@@ -317,6 +321,17 @@ class Session:
         if rc:
             raise RuntimeError(rc)
         return {"x0": x0, "conf": conf, "tokconf": tokconf, "margin": margin, "logits": lg}
+
+    def scr_decisions(self):
+        """The last step's tracked prefix positions (sparse cache refresh) and their decisions."""
+        R = max(1, self.sched.scr_rows)
+        pos = np.empty(R, np.int32)
+        x0 = np.empty(R, np.int32)
+        conf = np.empty(R, np.float32)
+        tokconf = np.empty(R, np.float32)
+        margin = np.empty(R, np.float32)
+        n = lib().orc_scr_decisions(self.h, _p(pos), _p(x0), _p(conf), _p(tokconf), _p(margin))
+        return {"pos": pos[:n], "x0": x0[:n], "conf": conf[:n], "tokconf": tokconf[:n], "margin": margin[:n]}
 
     def state(self):
         tok = np.empty(self.n_pos, np.int32)

@@ -335,3 +335,80 @@ def test_threshold_session_blocks_progress_and_finish(tiny_model):
             blocks += 1
         tok, st, kv = sess.state()
         assert blocks == 2 and kv == 96 and not (tok[32:] == TINY.mask_id).any()
+
+
+# ------------------------------------------------------------ sparse cache refresh (Sec. 3.3)
+def _scr_session(model, scr_rows, seed=51, **kw):
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=seed)
+    sess = O.Session(model, O.OracleSched(steps_per_block=4, scr_rows=scr_rows, **kw), prompt, 96)
+    sess.prefill()
+    assert sess.begin_block()
+    while not sess.step()["block_done"]:
+        pass
+    assert sess.begin_block()  # the first block is prefix now: its tokens are visible, not stable
+    return sess
+
+
+def test_scr_merge_is_not_visible_within_the_step(tiny_model):
+    # the tracked rows are queries only: the window's logits are those of a session without them
+    a = _scr_session(tiny_model, 8, theta_stable=2.0)
+    b = _scr_session(tiny_model, 0, theta_stable=2.0)
+    ka, kb = a.prefix_kv(1, 0).copy(), b.prefix_kv(1, 0).copy()
+    assert np.array_equal(ka, kb)
+    k0 = a.prefix_kv(0, 0).copy()
+    oa, ob = a.step(keep_logits=True), b.step(keep_logits=True)
+    da, db = a.decisions(logits=True), b.decisions(logits=True)
+    assert np.array_equal(da["logits"], db["logits"])
+    assert {k: oa[k] for k in ("n_committed", "block_done", "masked_after")} == \
+        {k: ob[k] for k in ("n_committed", "block_done", "masked_after")}
+    assert oa["n_refreshed"] == 8 and ob["n_refreshed"] == 0
+    # after the step the refreshed rows of layer 1 differ from the appended ones, the others do
+    # not; layer 0's K/V depend on the token and its position only, so its refresh changes nothing
+    ka2 = a.prefix_kv(1, 0)
+    pos = a.scr_decisions()["pos"]
+    changed = np.flatnonzero(np.abs(ka2 - ka).max(axis=1) > 0)
+    assert set(changed.tolist()) == set(pos.tolist())
+    assert np.array_equal(a.prefix_kv(0, 0), k0)
+
+
+def test_scr_tracks_the_first_visible_prefix_positions(tiny_model):
+    sess = _scr_session(tiny_model, 5, theta_stable=2.0)
+    tok, st, kv = sess.state()
+    sess.step()
+    pos = sess.scr_decisions()["pos"]
+    want = [p for p in range(kv) if st[p] == O.COMMITTED][:5]
+    assert pos.tolist() == want and len(want) == 5
+
+
+def test_scr_stable_threshold_zero_stabilizes_every_tracked_row(tiny_model):
+    sess = _scr_session(tiny_model, 6, theta_stable=0.0)
+    _, st0, kv = sess.state()
+    visible = [p for p in range(kv) if st0[p] == O.COMMITTED]
+    seen = []
+    for _ in range(3):
+        out = sess.step()
+        pos = sess.scr_decisions()["pos"].tolist()
+        assert out["n_refreshed"] == len(pos) and out["n_revised"] == 0
+        seen += pos
+        _, st, _ = sess.state()
+        assert all(st[p] == O.STABLE for p in pos)
+    assert seen == visible[:len(seen)] and len(seen) == min(18, len(visible))
+
+
+def test_scr_revision_replaces_ids_and_skips_their_merge(tiny_model):
+    # theta_remask above 1: every tracked row whose argmax differs from its id takes the argmax,
+    # and only the rows that keep their id have their K/V merged
+    sess = _scr_session(tiny_model, 8, theta_stable=2.0, theta_remask=1.5, remask_max=0)
+    tok0, st0, _ = sess.state()
+    k0 = sess.prefix_kv(1, 1).copy()
+    out = sess.step()
+    d = sess.scr_decisions()
+    tok1, st1, _ = sess.state()
+    k1 = sess.prefix_kv(1, 1)
+    revised = [int(p) for p, x in zip(d["pos"], d["x0"]) if x != tok0[p]]
+    kept = [int(p) for p, x in zip(d["pos"], d["x0"]) if x == tok0[p]]
+    assert out["n_revised"] == len(revised) and out["n_refreshed"] == len(kept) and len(revised) > 0
+    for p, x in zip(d["pos"], d["x0"]):
+        assert tok1[p] == x and st1[p] == O.COMMITTED
+    moved = set(np.flatnonzero(np.abs(k1 - k0).max(axis=1) > 0).tolist())
+    assert moved == set(kept)
