@@ -96,11 +96,23 @@ typedef struct {
     int use_prefix_cache;
     int commit_mode;      /* DLLM_COMMIT_SCHEDULE or DLLM_COMMIT_THRESHOLD */
     float theta_visible;  /* threshold mode only */
+    /* Sparse cache refresh (Sec. 3.3; one sequence with the prefix cache on; 0 = off, at most
+     * DLLM_MAX_SCR_ROWS): each step the first scr_rows prefix positions that are COMMITTED
+     * (visible, not stable) run with the window as extra query rows at their own positions,
+     * attending to the prefix as cached and to the window and adding no keys.  After the
+     * commit pass each is re-scored: STABLE at tokconf >= theta_stable; below theta_remask
+     * (when > 0) with another argmax it takes that argmax; otherwise it keeps its id.  The K/V
+     * computed for the rows that keep their id replace theirs in the prefix cache after the
+     * step (the merge is not visible inside the step).  The window then counts scr_rows more
+     * rows against max_window. */
+    int scr_rows;
 } dllm_sched;
+#define DLLM_MAX_SCR_ROWS 32
 
 /* Result of one denoising step, summed over the batch (block_done: all). */
 typedef struct {
     int n_committed, n_remasked, n_stable, n_drafts, block_done, masked_after;
+    int n_refreshed, n_revised;  /* sparse cache refresh: prefix K/V rows merged, prefix ids revised */
 } dllm_step_out;
 
 typedef struct {
@@ -181,6 +193,10 @@ int dllm_set_state(dllm_ctx* ctx, const int32_t* tokens, const uint8_t* status);
  * [batch][T][vocab] only when dllm_set_debug enabled them (else pass NULL).
  * Synchronises. */
 int dllm_get_step_debug(dllm_ctx* ctx, float* logits, int32_t* argmax, float* conf, float* tokconf);
+
+/* The last step's sparse-cache-refresh rows: pos, argmax, conf, tokconf (host arrays of
+ * scr_rows entries, nullable; pos -1 = an unused row); *n = scr_rows.  Synchronises. */
+int dllm_get_scr_debug(dllm_ctx* ctx, int32_t* pos, int32_t* argmax, float* conf, float* tokconf, int* n);
 
 /* flags bit 0: materialise logits; bit 1: disable CUDA graphs; bit 2: launch
  * without programmatic dependent launch; bit 3: give the weight-streaming

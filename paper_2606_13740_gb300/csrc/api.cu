@@ -37,7 +37,7 @@ struct Layout {
     size_t off_x, off_xn, off_q, off_attn, off_h, off_sq, off_theta;
     int n_sq;
     size_t off_lmp, off_zcur, off_cur, off_x0, off_conf, off_tokconf;
-    size_t off_part, part_floats, off_cnt, off_done, off_epoch;
+    size_t off_part, part_floats, off_cnt, off_done, off_epoch, off_trk, off_smerge, off_side;
     int cnt_len, done_len;  // per phase slot
     size_t off_tok, off_st, off_stok, off_sst, off_seqkv, off_plan, off_outs, off_status;
     size_t total;
@@ -105,6 +105,11 @@ Layout make_layout(const dllm_config& c) {
     L.off_plan = take(static_cast<size_t>(c.max_batch) * 16);
     L.off_outs = take(static_cast<size_t>(c.max_batch) * 32);
     L.off_status = take(16);
+    // sparse cache refresh (one sequence): tracked positions, merge flags, side K/V
+    // [L][2][H][DLLM_MAX_SCR_ROWS][hd]
+    L.off_trk = take(DLLM_MAX_SCR_ROWS * 4);
+    L.off_smerge = take(DLLM_MAX_SCR_ROWS * 4);
+    L.off_side = take(static_cast<size_t>(c.n_layers) * 2 * L.qd * DLLM_MAX_SCR_ROWS * 2);
     L.total = o;
     return L;
 }
@@ -147,6 +152,9 @@ struct dllm_ctx {
     float *lmp = nullptr, *zcur = nullptr, *conf = nullptr, *tokconf = nullptr;
     int *cur = nullptr, *x0 = nullptr;
     float* chain_part = nullptr;
+    int* trk = nullptr;
+    int* scr_merge = nullptr;
+    __nv_bfloat16* scr_side = nullptr;
     int *chain_cnt = nullptr, *chain_done = nullptr, *epoch = nullptr;
     int *tok = nullptr, *stok = nullptr, *seq_kv = nullptr, *plan = nullptr, *outs = nullptr, *status = nullptr;
     uint8_t *st = nullptr, *sst = nullptr;
@@ -243,7 +251,11 @@ static int sync_check(dllm_ctx* ctx) {
 // ------------------------------------------------------------------ forward
 // Layers (and optionally the LM head) over T window tokens of each of the B
 // sequences; token ids come from the state at seq_kv[b] + t.
-static int forward(dllm_ctx* ctx, int B, int T, bool head) {
+// T window rows per sequence, then (sparse cache refresh, one sequence) R tracked prefix rows:
+// they run through every projection and the head, attend as queries only, and their K/V go to
+// the side buffers.
+static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0) {
+    const int T = Tw + R;  // rows per sequence
     const dllm_config& c = ctx->cfg;
     const Layout& L = ctx->L;
     const int d = c.d_model, F = c.ffn, qd = L.qd, N = B * T;
@@ -251,7 +263,7 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
     // x = embedding rows, xb = bf16(x) (the next projection's operand), sq = RMSNorm statistics;
     // the step counter advances (it tags the chained projections' completion flags)
     CK(launch_embed(ctx->tok, c.max_ctx, ctx->seq_kv, ctx->emb, ctx->x, ctx->xn, ctx->sq, ctx->cur, ctx->epoch, B, T,
-                    d, s));
+                    d, s, Tw, ctx->trk));
     mark(ctx, DLLM_K_EMBED);
     const GemmPlan pq = gemm_plan(L.qkv_rows, N, d, ctx->sms, EPI_QKV);
     const GemmPlan po = gemm_plan(L.o_rows, N, qd, ctx->sms, EPI_RESID);
@@ -262,12 +274,16 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
     if (!make_tmap_bf16(&tx_xn, ctx->xn, N, d, pq.ntile) || !make_tmap_bf16(&tx_attn, ctx->attn, N, qd, po.ntile) ||
         !make_tmap_bf16(&tx_h, ctx->h, N, F, pd.ntile))
         return fail(ctx, DLLM_ECUDA, "tensor map encode failed");
-    const AttnPlan ap = attn_plan(B, T, c.n_heads, c.head_dim, ctx->kv_len + T, ctx->sms);
+    AttnPlan ap = attn_plan(B, T, c.n_heads, c.head_dim, ctx->kv_len + Tw, ctx->sms);
+    ap.qx = R;
     EpiArgs ep{};
     ep.seq_kv = ctx->seq_kv;
     ep.n_seq = B;
     ep.theta = ctx->theta;
     ep.T = T;
+    ep.Tw = Tw;
+    ep.R = R;
+    ep.trk = ctx->trk;
     ep.H = c.n_heads;
     ep.hd = c.head_dim;
     ep.cap = c.max_ctx;
@@ -294,6 +310,8 @@ static int forward(dllm_ctx* ctx, int B, int T, bool head) {
         EpiArgs e = ep;
         e.kc = ctx->kv + static_cast<size_t>(2 * l) * L.kv_half;
         e.vc = ctx->kv + static_cast<size_t>(2 * l + 1) * L.kv_half;
+        e.kside = ctx->scr_side + static_cast<size_t>(2 * l) * qd * R;  // [L][2][H][R][hd]
+        e.vside = e.kside + static_cast<size_t>(qd) * R;
         return e;
     };
     // phase slot i of a chain uses scratch slot i; consecutive chains are ordered by the stream
@@ -360,7 +378,12 @@ static int step_kernels(dllm_ctx* ctx, int T) {
     ctx->trace_launch = 0;
     ctx->in_step = true;
     mark(ctx, -1);
-    int rc = forward(ctx, ctx->B, T, true);
+    const int R = ctx->sched.use_prefix_cache ? ctx->sched.scr_rows : 0;
+    if (R > 0) {  // the visible prefix positions this step refreshes
+        CK(launch_scr_select(ctx->st, ctx->seq_kv, ctx->trk, R, ctx->stream));
+        mark(ctx, DLLM_K_COMMIT);
+    }
+    int rc = forward(ctx, ctx->B, T, true, R);
     if (rc) {
         ctx->in_step = false;
         return rc;
@@ -377,6 +400,10 @@ static int step_kernels(dllm_ctx* ctx, int T) {
     a.outs = ctx->outs;
     a.B = ctx->B;
     a.T = T;
+    a.Tq = T + R;
+    a.R = R;
+    a.trk = ctx->trk;
+    a.merge = ctx->scr_merge;
     a.mask_id = ctx->cfg.mask_id;
     a.use_cache = ctx->sched.use_prefix_cache;
     a.S = ctx->sched.steps_per_block;
@@ -389,6 +416,11 @@ static int step_kernels(dllm_ctx* ctx, int T) {
     a.theta_visible = ctx->sched.theta_visible;
     cudaError_t ce = launch_commit(a, ctx->stream);
     mark(ctx, DLLM_K_COMMIT);
+    if (ce == cudaSuccess && R > 0) {  // the refreshed K/V merged at the step boundary
+        ce = launch_scr_merge(ctx->scr_side, ctx->kv, ctx->trk, ctx->scr_merge, ctx->cfg.n_layers, ctx->cfg.n_heads,
+                              ctx->cfg.head_dim, ctx->cfg.max_ctx, R, ctx->stream);
+        mark(ctx, DLLM_K_COMMIT);
+    }
     ctx->in_step = false;
     CK(ce);
     return DLLM_OK;
@@ -507,6 +539,9 @@ int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void*
     ctx->plan = reinterpret_cast<int*>(A + L.off_plan);
     ctx->outs = reinterpret_cast<int*>(A + L.off_outs);
     ctx->status = reinterpret_cast<int*>(A + L.off_status);
+    ctx->trk = reinterpret_cast<int*>(A + L.off_trk);
+    ctx->scr_merge = reinterpret_cast<int*>(A + L.off_smerge);
+    ctx->scr_side = reinterpret_cast<__nv_bfloat16*>(A + L.off_side);
     cudaStream_t s = ctx->stream;
     // zero everything that is read before it is written (counters, state, status)
     if (cudaMemsetAsync(A + L.off_sq, 0, L.total - L.off_sq, s) != cudaSuccess ||
@@ -574,8 +609,13 @@ static int start_request(dllm_ctx* ctx, const dllm_sched* sched, int batch, int 
     if (!sched || batch < 1 || Lp < 0 || gen_len < 1) return fail(ctx, DLLM_EINVAL, "bad request arguments");
     if (sched->steps_per_block < 1 || sched->remask_max < 0 || sched->spec_blocks < 0 ||
         (sched->commit_mode != DLLM_COMMIT_SCHEDULE && sched->commit_mode != DLLM_COMMIT_THRESHOLD) ||
-        !(sched->theta_visible == sched->theta_visible))
+        !(sched->theta_visible == sched->theta_visible) || sched->scr_rows < 0 ||
+        sched->scr_rows > DLLM_MAX_SCR_ROWS)
         return fail(ctx, DLLM_EINVAL, "bad schedule");
+    if (sched->scr_rows > 0 && (!sched->use_prefix_cache || batch != 1))
+        return fail(ctx, DLLM_EINVAL, "sparse cache refresh needs one sequence and the prefix cache");
+    if (sched->use_prefix_cache && c.block_len * (1 + sched->spec_blocks) + sched->scr_rows > c.max_window)
+        return fail(ctx, DLLM_ECAPACITY, "window plus refresh rows > max_window %d", c.max_window);
     if (batch > c.max_batch) return fail(ctx, DLLM_ECAPACITY, "batch %d > max_batch %d", batch, c.max_batch);
     const int n_pos = Lp + gen_len;
     if (n_pos > c.max_ctx) return fail(ctx, DLLM_ECAPACITY, "Lp + gen_len = %d > max_ctx %d", n_pos, c.max_ctx);
@@ -728,7 +768,9 @@ int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out) {
     ctx->last_spec = spec;
     const bool use_graph = !(ctx->debug & 2);
     if (use_graph) {
-        const int key_dbg = ctx->debug | (ctx->profiling ? 256 : 0);  // trace pointers are baked in too
+        // trace pointers and the refresh rows are baked in too
+        const int key_dbg = ctx->debug | (ctx->profiling ? 256 : 0) |
+                            ((s.use_prefix_cache ? s.scr_rows : 0) << 10);
         if (!ctx->gexec || ctx->g_T != T || ctx->g_B != ctx->B || ctx->g_kv != ctx->kv_len || ctx->g_dbg != key_dbg) {
             if (ctx->gexec) {
                 cudaGraphExecDestroy(ctx->gexec);
@@ -778,6 +820,8 @@ int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out) {
             out->n_drafts += r[3];
             out->block_done &= r[4];
             out->masked_after += r[5];
+            out->n_refreshed += r[6];
+            out->n_revised += r[7];
         }
     }
     return DLLM_OK;
@@ -918,6 +962,20 @@ int dllm_get_step_debug(dllm_ctx* ctx, float* logits, int32_t* argmax, float* co
     if (argmax) CK(cudaMemcpyAsync(argmax, ctx->x0, n * 4, cudaMemcpyDeviceToHost, ctx->stream));
     if (conf) CK(cudaMemcpyAsync(conf, ctx->conf, n * 4, cudaMemcpyDeviceToHost, ctx->stream));
     if (tokconf) CK(cudaMemcpyAsync(tokconf, ctx->tokconf, n * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    return sync_check(ctx);
+}
+
+int dllm_get_scr_debug(dllm_ctx* ctx, int32_t* pos, int32_t* argmax, float* conf, float* tokconf, int* n) {
+    GUARD(ctx);
+    const int R = ctx->sched.use_prefix_cache ? ctx->sched.scr_rows : 0;
+    if (n) *n = R;
+    if (R == 0) return DLLM_OK;
+    const size_t off = static_cast<size_t>(ctx->last_T);  // one sequence: rows T .. T + R - 1
+    if (pos) CK(cudaMemcpyAsync(pos, ctx->trk, static_cast<size_t>(R) * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    if (argmax) CK(cudaMemcpyAsync(argmax, ctx->x0 + off, static_cast<size_t>(R) * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    if (conf) CK(cudaMemcpyAsync(conf, ctx->conf + off, static_cast<size_t>(R) * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    if (tokconf)
+        CK(cudaMemcpyAsync(tokconf, ctx->tokconf + off, static_cast<size_t>(R) * 4, cudaMemcpyDeviceToHost, ctx->stream));
     return sync_check(ctx);
 }
 

@@ -104,7 +104,7 @@ struct TcMaps {
 template <int NB>
 __global__ void __launch_bounds__(kTcThreads, 1)
     k_attn_tc(const __grid_constant__ TcMaps maps, const int* __restrict__ seq_kv, __nv_bfloat16* __restrict__ out,
-              int T, int H, int cap, int qtiles, int csize, int* status, unsigned long long* trace) {
+              int T, int H, int cap, int qtiles, int csize, int qx, int* status, unsigned long long* trace) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sQ = smem;                       // 32 KB
@@ -126,7 +126,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     pdl_launch_dependents();
     const int split = blockIdx.x, h = blockIdx.y;
     const int b = blockIdx.z / qtiles, qt = blockIdx.z - b * qtiles;
-    const int NK = seq_kv[b] + T;
+    const int NK = seq_kv[b] + T - qx;  // the last qx rows are queries only
     const int nblk = (NK + kTcKeys - 1) / kTcKeys;
     const int blk0 = split * nblk / csize, blk1 = (split + 1) * nblk / csize;
     const int kbeg = blk0 * kTcKeys, kend = min(NK, blk1 * kTcKeys);
@@ -446,7 +446,8 @@ cudaError_t tc_go(cudaLaunchConfig_t& cfg, const TcMaps& maps, const int* seq_kv
                   int cap, const AttnPlan& a, int* status, unsigned long long* trace) {
     cfg.blockDim = dim3(kTcThreads);
     cfg.dynamicSmemBytes = tc_smem<NB>();
-    return cudaLaunchKernelEx(&cfg, k_attn_tc<NB>, maps, seq_kv, out, T, H, cap, a.qtiles, a.csize, status, trace);
+    return cudaLaunchKernelEx(&cfg, k_attn_tc<NB>, maps, seq_kv, out, T, H, cap, a.qtiles, a.csize, a.qx, status,
+                              trace);
 }
 
 }  // namespace

@@ -186,7 +186,8 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
         fi = (pp >> 1) + (pp & 1) * (ep.hd >> 1);
         theta = sm.theta[rt];
         bl = col0 / ep.T;
-        run = min(col0 + 31, p.N - 1) / ep.T == bl;  // all 32 columns in one sequence
+        // all 32 columns in one sequence's window (consecutive positions)
+        run = min(col0 + 31, p.N - 1) / ep.T == bl && min(col0 + 31, p.N - 1) - bl * ep.T < ep.Tw;
         qkv_dst = part == 0 ? ep.q : (part == 1 ? ep.kc : ep.vc);
         if (part < 2 && run) {
             const float2 a = rot_cs(static_cast<float>(sm.kvs[bl] + (col0 + GW * half - bl * ep.T)) * theta);
@@ -277,7 +278,9 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                     const int b = min((cg + u) / ep.T, ep.n_seq - 1);
                     bs[u] = b;
                     ts[u] = cg + u - b * ep.T;
-                    const float2 r = rot_cs(static_cast<float>(sm.kvs[b] + ts[u]) * theta);
+                    // a window row, or (sparse cache refresh) a tracked prefix position
+                    const int ps = ts[u] < ep.Tw ? sm.kvs[b] + ts[u] : max(ep.trk[ts[u] - ep.Tw], 0);
+                    const float2 r = rot_cs(static_cast<float>(ps) * theta);
                     cs[u] = r.x;
                     ss[u] = r.y;
                 }
@@ -357,10 +360,21 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
         if (col < p.N) {
             const int b = min(col / ep.T, ep.n_seq - 1);
             const int ts = col - b * ep.T;
-            const int pos = sm.kvs[b] + ts;
+            const bool tracked = ts >= ep.Tw;  // sparse cache refresh: K/V to the side buffers
+            const int pos = tracked ? ep.trk[ts - ep.Tw] : sm.kvs[b] + ts;
             const int head = (mt * kBM - part * ep.H * ep.hd + f0) / ep.hd;
             const int fi0 = f0 % ep.hd;
-            if (pos >= 0 && pos < ep.cap) {
+            if (tracked && part > 0) {
+                if (pos >= 0) {
+                    const uint4* src = reinterpret_cast<const uint4*>(
+                        reinterpret_cast<const __nv_bfloat16*>(sm.stg) + tok * kBM + f0);
+                    __nv_bfloat16* side = part == 1 ? ep.kside : ep.vside;
+                    uint4* dst = reinterpret_cast<uint4*>(
+                        side + (static_cast<size_t>(head) * ep.R + (ts - ep.Tw)) * ep.hd + fi0);
+#pragma unroll
+                    for (int i = 0; i < 2; ++i) dst[i] = src[i];
+                }
+            } else if (tracked || (pos >= 0 && pos < ep.cap)) {
                 const size_t plane = part == 0 ? static_cast<size_t>(ep.T) : static_cast<size_t>(ep.cap);
                 const size_t r = (static_cast<size_t>(b) * ep.H + head) * plane + (part == 0 ? ts : pos);
                 const uint4* src = reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(sm.stg) +

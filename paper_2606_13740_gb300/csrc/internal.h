@@ -57,6 +57,13 @@ struct EpiArgs {
     // EPI_SWIGLU: tile k row 2f is gate feature 64k+f, row 2f+1 the matching up row
     __nv_bfloat16* h;    // [N][F]
     int F;
+    // EPI_QKV with sparse cache refresh (one sequence): of the T rows the first Tw are the
+    // window, row Tw + r is the prefix position trk[r] (< 0: an unused row, no K/V written),
+    // whose K and V go to kside / vside [H][R][hd] instead of the cache
+    int Tw, R;
+    const int* trk;
+    __nv_bfloat16* kside;
+    __nv_bfloat16* vside;
     // EPI_LMHEAD
     float* lm_part;      // [N][m_tiles][3]: max, sum exp(z - max), argmax (as float bits)
     float* zcur;         // [N]: logit of the current token id
@@ -172,8 +179,17 @@ cudaError_t launch_init_kv_random(__nv_bfloat16* cache, int B, int H, int hd, in
                                   int which, int L, uint64_t seed, cudaStream_t st);
 // x = embedding rows of the window's ids (fp32), xb = bf16(x), sq[d/128][N] = per-128-feature
 // sums of x^2, cur[N] = the ids (for the LM head's current-token probability).
+// T rows per sequence: the first Tw at the window positions seq_kv[b] + t, the rest (one
+// sequence) at the prefix positions trk[t - Tw] (< 0: id 0).
 cudaError_t launch_embed(const int* tok, int tok_ld, const int* seq_kv, const __nv_bfloat16* emb, float* x,
-                         __nv_bfloat16* xb, float* sq, int* cur, int* epoch, int B, int T, int d, cudaStream_t st);
+                         __nv_bfloat16* xb, float* sq, int* cur, int* epoch, int B, int T, int d, cudaStream_t st,
+                         int Tw = -1, const int* trk = nullptr);
+// Sparse cache refresh (one sequence): trk[r] = the r-th COMMITTED position below seq_kv[0]
+// (ascending), -1 past the last; merge: the K/V rows of the refreshed positions (merge[r] != 0)
+// from the side buffers [L][2][H][R][hd] into the cache [L][2][1][H][cap][hd].
+cudaError_t launch_scr_select(const uint8_t* st, const int* seq_kv, int* trk, int R, cudaStream_t stream);
+cudaError_t launch_scr_merge(const __nv_bfloat16* side, __nv_bfloat16* cache, const int* trk, const int* merge, int L,
+                             int H, int hd, int cap, int R, cudaStream_t stream);
 // The kernels below are launched with PDL when `pdl` (inside the context's step chain); the
 // single-kernel entry points pass false because their inputs may come from foreign kernels.
 // Attention plan: CTAs (split, head, sequence x query tile of 16*nw rows); the csize
@@ -184,6 +200,7 @@ struct AttnPlan {
     int nb;     // K/V sub-blocks in flight per CTA (1 or 2)
     int pairs;  // warp groups per CTA, each on its own share of the CTA's sub-blocks (1 or 2)
     bool tc;    // head dim 128: the tcgen05 kernel (128-row query tiles, 64-key sub-blocks)
+    int qx;     // the last qx of a sequence's T rows are queries only: keys = kv_len + T - qx
 };
 // head dim 128 and at least kTcMinKeys keys: the tcgen05 kernel's plan; otherwise the
 // mma.sync kernel's
@@ -221,6 +238,11 @@ struct CommitArgs {
     float theta_remask, theta_stable;
     int commit_mode;     // DLLM_COMMIT_SCHEDULE / DLLM_COMMIT_THRESHOLD (dllm.h)
     float theta_visible;
+    // rows per sequence of x0 / conf / tokconf (T, or T + R with sparse cache refresh: rows
+    // T + r are the prefix positions trk[r]; one sequence); merge[r]: its K/V are merged
+    int Tq, R;
+    const int* trk;
+    int* merge;
 };
 cudaError_t launch_commit(const CommitArgs& a, cudaStream_t st, bool pdl = true);
 

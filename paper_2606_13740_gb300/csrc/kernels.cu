@@ -130,13 +130,15 @@ cudaError_t launch_init_kv_random(__nv_bfloat16* cache, int B, int H, int hd, in
 // cur[token] = the id (for the LM head's current-token probability).
 __global__ void __launch_bounds__(256) k_embed(const int* tok, int tok_ld, const int* seq_kv,
                                                const __nv_bfloat16* emb, float* x, __nv_bfloat16* xb, float* sq,
-                                               int* cur, int* epoch, int T, int N, int d) {
+                                               int* cur, int* epoch, int T, int N, int d, int Tw, const int* trk) {
     pdl_wait();
     pdl_launch_dependents();
     const int j = blockIdx.x;
     if (j == 0 && threadIdx.x == 0) *epoch += 1;  // one forward pass: a new tag for the chained projections
     const int b = j / T, t = j - b * T;
-    const int id = tok[static_cast<size_t>(b) * tok_ld + seq_kv[b] + t];
+    // window rows, then (sparse cache refresh, one sequence) the tracked prefix positions
+    const int pos = t < Tw ? seq_kv[b] + t : trk[t - Tw];
+    const int id = pos >= 0 ? tok[static_cast<size_t>(b) * tok_ld + pos] : 0;
     if (threadIdx.x == 0) cur[j] = id;
     const __nv_bfloat16* e = emb + static_cast<size_t>(id) * d;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -158,9 +160,12 @@ __global__ void __launch_bounds__(256) k_embed(const int* tok, int tok_ld, const
 }
 
 cudaError_t launch_embed(const int* tok, int tok_ld, const int* seq_kv, const __nv_bfloat16* emb, float* x,
-                         __nv_bfloat16* xb, float* sq, int* cur, int* epoch, int B, int T, int d, cudaStream_t st) {
+                         __nv_bfloat16* xb, float* sq, int* cur, int* epoch, int B, int T, int d, cudaStream_t st,
+                         int Tw, const int* trk) {
+    if (Tw < 0) Tw = T;
+    if (Tw < T && (!trk || B != 1)) return cudaErrorInvalidValue;
     return launch_k(k_embed, dim3(B * T), dim3(256), 0, st, true, tok, tok_ld, seq_kv, emb, x, xb, sq, cur, epoch, T,
-                    B * T, d);
+                    B * T, d, Tw, trk);
 }
 
 // ------------------------------------------------------------------ attention
@@ -221,7 +226,7 @@ __global__ void __launch_bounds__(PR * NW * 32) k_attn(const __nv_bfloat16* __re
                                                        const __nv_bfloat16* __restrict__ kc,
                                                        const __nv_bfloat16* __restrict__ vc,
                                                        const int* __restrict__ seq_kv, __nv_bfloat16* __restrict__ out,
-                                                       int T, int H, int cap, int qtiles, int csize,
+                                                       int T, int H, int cap, int qtiles, int csize, int qx,
                                                        unsigned long long* trace) {
     constexpr int AQ = NW * 16;  // query rows per CTA
     constexpr int NT = NW * 32;  // threads of one warp group
@@ -248,7 +253,7 @@ __global__ void __launch_bounds__(PR * NW * 32) k_attn(const __nv_bfloat16* __re
     const int split = blockIdx.x, h = blockIdx.y;  // split = rank in the cluster
     const int b = blockIdx.z / qtiles, qt = blockIdx.z - b * qtiles;
     const int kv = seq_kv[b];
-    const int NK = kv + T;
+    const int NK = kv + T - qx;  // the last qx rows are queries only
     const int nblk = (NK + kAK - 1) / kAK;
     const int blk0 = split * nblk / csize, blk1 = (split + 1) * nblk / csize;  // the CTA's sub-blocks
     const int kbeg = (blk0 + grp * (blk1 - blk0) / PR) * kAK;
@@ -471,7 +476,7 @@ static cudaError_t attn_go(cudaLaunchConfig_t& cfg, const __nv_bfloat16* q, cons
     cfg.blockDim = dim3(PR * NW * 32);
     cfg.dynamicSmemBytes = attn_smem(NW, NB, PR, HD);
     return cudaLaunchKernelEx(&cfg, k_attn<HD, NW, NB, PR>, q, kc, vc, seq_kv, out, T, H, cap, a.qtiles, a.csize,
-                              trace);
+                              a.qx, trace);
 }
 
 cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
@@ -608,9 +613,9 @@ __global__ void __launch_bounds__(256) k_commit(CommitArgs a) {
     const int c0 = plan[0], c1 = plan[1], step = plan[2];
     const int n = c1 - c0;  // <= kMaxBlock (checked by the host)
     const int w0 = a.use_cache ? a.seq_kv[b] : 0;
-    const int* x0 = a.x0 + static_cast<size_t>(b) * a.T;
-    const float* conf = a.conf + static_cast<size_t>(b) * a.T;
-    const float* tc = a.tokconf + static_cast<size_t>(b) * a.T;
+    const int* x0 = a.x0 + static_cast<size_t>(b) * a.Tq;
+    const float* conf = a.conf + static_cast<size_t>(b) * a.Tq;
+    const float* tc = a.tokconf + static_cast<size_t>(b) * a.Tq;
     __shared__ int s_cnt[8];
     __shared__ uint8_t s_sel[kMaxBlock];
     if (threadIdx.x < 8) s_cnt[threadIdx.x] = 0;
@@ -758,6 +763,28 @@ __global__ void __launch_bounds__(256) k_commit(CommitArgs a) {
         }
     }
     __syncthreads();
+    // sparse cache refresh (one sequence): the tracked prefix positions, rows Tw + r, re-scored;
+    // those that keep their id have their refreshed K/V merged after this kernel
+    for (int r = threadIdx.x; r < a.R; r += blockDim.x) {
+        const int p = a.trk[r];
+        int merge = 0;
+        if (p >= 0) {
+            const float v = tc[a.T + r];
+            const int x = x0[a.T + r];
+            merge = 1;
+            if (v >= a.theta_stable) {
+                st[p] = 3;
+                atomicAdd(&s_cnt[2], 1);
+            } else if (a.theta_remask > 0.0f && v < a.theta_remask && x != tok[p]) {
+                tok[p] = x;
+                merge = 0;
+                atomicAdd(&s_cnt[7], 1);
+            }
+            if (merge) atomicAdd(&s_cnt[6], 1);
+        }
+        a.merge[r] = merge;
+    }
+    __syncthreads();
     if (threadIdx.x == 0) {
         int* o = a.outs + b * 8;
         o[0] = s_cnt[0];
@@ -766,8 +793,77 @@ __global__ void __launch_bounds__(256) k_commit(CommitArgs a) {
         o[3] = s_cnt[3];
         o[5] = m - s_cnt[0];
         o[4] = o[5] == 0;
+        o[6] = s_cnt[6];
+        o[7] = s_cnt[7];
         plan[2] = step + 1;
     }
+}
+
+// ------------------------------------------------------------------ sparse cache refresh
+// One CTA: trk[r] = the r-th position p < seq_kv[0] whose state is COMMITTED (ascending), -1
+// past the last.  Positions are scanned 256 at a time with a block-wide prefix count.
+__global__ void __launch_bounds__(256) k_scr_select(const uint8_t* st, const int* seq_kv, int* trk, int R) {
+    pdl_wait();
+    pdl_launch_dependents();
+    __shared__ int s_warp[8];
+    __shared__ int s_base;
+    const int kv = seq_kv[0];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) s_base = 0;
+    for (int r = threadIdx.x; r < R; r += blockDim.x) trk[r] = -1;
+    __syncthreads();
+    for (int p0 = 0; p0 < kv; p0 += blockDim.x) {
+        const int p = p0 + static_cast<int>(threadIdx.x);
+        const bool hit = p < kv && st[p] == 2;
+        const unsigned bal = __ballot_sync(0xffffffffu, hit);
+        if (lane == 0) s_warp[warp] = __popc(bal);
+        __syncthreads();
+        int before = s_base;
+        for (int w = 0; w < warp; ++w) before += s_warp[w];
+        const int idx = before + __popc(bal & ((1u << lane) - 1u));
+        if (hit && idx < R) trk[idx] = p;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            int tot = 0;
+            for (int w = 0; w < 8; ++w) tot += s_warp[w];
+            s_base += tot;
+        }
+        __syncthreads();
+        if (s_base >= R) break;
+    }
+}
+
+cudaError_t launch_scr_select(const uint8_t* st, const int* seq_kv, int* trk, int R, cudaStream_t stream) {
+    return launch_k(k_scr_select, dim3(1), dim3(256), 0, stream, true, st, seq_kv, trk, R);
+}
+
+// Grid (R, L): row r of layer l, when merged, copies its K and V rows of every head (hd
+// elements each) from the side buffers into the cache at position trk[r].
+__global__ void __launch_bounds__(128) k_scr_merge(const __nv_bfloat16* side, __nv_bfloat16* cache, const int* trk,
+                                                   const int* merge, int H, int hd, int cap, int R) {
+    pdl_wait();
+    pdl_launch_dependents();
+    const int r = blockIdx.x, l = blockIdx.y;
+    const int p = trk[r];
+    if (p < 0 || !merge[r]) return;
+    const size_t side_layer = static_cast<size_t>(2) * H * R * hd;
+    const size_t cache_half = static_cast<size_t>(H) * cap * hd;
+    const int n4 = hd / 8;  // 16-byte pieces per head row
+    for (int e = threadIdx.x; e < 2 * H * n4; e += blockDim.x) {
+        const int which = e / (H * n4), rem = e - which * H * n4;
+        const int h = rem / n4, i = rem - h * n4;
+        const uint4* src = reinterpret_cast<const uint4*>(side + l * side_layer + (static_cast<size_t>(which) * H + h) *
+                                                                                    R * hd + static_cast<size_t>(r) * hd) + i;
+        uint4* dst = reinterpret_cast<uint4*>(cache + (static_cast<size_t>(2 * l + which)) * cache_half +
+                                              (static_cast<size_t>(h) * cap + p) * hd) + i;
+        *dst = *src;
+    }
+}
+
+cudaError_t launch_scr_merge(const __nv_bfloat16* side, __nv_bfloat16* cache, const int* trk, const int* merge, int L,
+                             int H, int hd, int cap, int R, cudaStream_t stream) {
+    if (R < 1 || hd % 8) return cudaErrorInvalidValue;
+    return launch_k(k_scr_merge, dim3(R, L), dim3(128), 0, stream, true, side, cache, trk, merge, H, hd, cap, R);
 }
 
 cudaError_t launch_commit(const CommitArgs& a, cudaStream_t st, bool pdl) {

@@ -241,6 +241,7 @@ int dllm_op_commit(int32_t* tok, uint8_t* status, int n_pos, int w0, int T, int 
     a.theta_stable = theta_stable;
     a.commit_mode = commit_mode;
     a.theta_visible = theta_visible;
+    a.Tq = T;  // window rows only (no sparse cache refresh rows)
     cudaError_t e = launch_commit(a, nullptr, false);
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) return op_fail(DLLM_ECUDA, "commit: %s", cudaGetErrorString(e));

@@ -38,12 +38,13 @@ class dllm_config(C.Structure):
 class dllm_sched(C.Structure):
     _fields_ = [("steps_per_block", C.c_int), ("theta_remask", C.c_float), ("theta_stable", C.c_float),
                 ("remask_max", C.c_int), ("spec_trigger", C.c_int), ("spec_blocks", C.c_int),
-                ("use_prefix_cache", C.c_int), ("commit_mode", C.c_int), ("theta_visible", C.c_float)]
+                ("use_prefix_cache", C.c_int), ("commit_mode", C.c_int), ("theta_visible", C.c_float),
+                ("scr_rows", C.c_int)]
 
 
 class dllm_step_out(C.Structure):
     _fields_ = [("n_committed", C.c_int), ("n_remasked", C.c_int), ("n_stable", C.c_int), ("n_drafts", C.c_int),
-                ("block_done", C.c_int), ("masked_after", C.c_int)]
+                ("block_done", C.c_int), ("masked_after", C.c_int), ("n_refreshed", C.c_int), ("n_revised", C.c_int)]
 
     def as_dict(self):
         return {k: getattr(self, k) for k, _ in self._fields_}
@@ -71,6 +72,7 @@ SIGNATURES = {
     "dllm_get_state": (_I, [_P, _P, _P, _P]),
     "dllm_set_state": (_I, [_P, _P, _P]),
     "dllm_get_step_debug": (_I, [_P, _P, _P, _P, _P]),
+    "dllm_get_scr_debug": (_I, [_P, _P, _P, _P, _P, _P]),
     "dllm_set_debug": (_I, [_P, _I]),
     "dllm_get_weight": (_I, [_P, _I, _I, _P, _SZ]),
     "dllm_get_kv": (_I, [_P, _I, _I, _I, _I, _I, _P]),
@@ -157,11 +159,12 @@ class Sched:
     use_prefix_cache: int = 1
     commit_mode: int = COMMIT_SCHEDULE
     theta_visible: float = 0.7
+    scr_rows: int = 0  # sparse cache refresh: visible prefix positions re-scored per step (one sequence)
 
     def c(self):
         return dllm_sched(self.steps_per_block, self.theta_remask, self.theta_stable, self.remask_max,
                           self.spec_trigger, self.spec_blocks, self.use_prefix_cache, self.commit_mode,
-                          self.theta_visible)
+                          self.theta_visible, self.scr_rows)
 
 
 def dllm_arena_bytes(cfg: Config) -> int:
@@ -265,6 +268,18 @@ class Context:
         if logits:
             r["logits"] = lg.reshape(self.B, T, self.cfg.vocab)
         return r
+
+    def dllm_get_scr_debug(self):
+        """The last step's sparse-cache-refresh rows: positions (-1 unused), argmax, conf, tokconf."""
+        R = 64
+        pos = np.empty(R, np.int32)
+        x0 = np.empty(R, np.int32)
+        conf = np.empty(R, np.float32)
+        tc = np.empty(R, np.float32)
+        n = C.c_int()
+        _check(lib().dllm_get_scr_debug(self.h, _p(pos), _p(x0), _p(conf), _p(tc), C.byref(n)), self.h)
+        k = n.value
+        return {"pos": pos[:k], "x0": x0[:k], "conf": conf[:k], "tokconf": tc[:k]}
 
     def dllm_get_weight(self, layer, which):
         c = self.cfg

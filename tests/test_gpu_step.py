@@ -51,7 +51,7 @@ def _unambiguous_commits(od, o_tok_before, o_st_before, c0, c1, w0, k):
     return (c[k - 1] - c[k]) > 0.02 * c[k - 1]
 
 
-def _run_teacher_forced(model, osched, gsched, prompt, gen_len, ctx):
+def _run_teacher_forced(model, osched, gsched, prompt, gen_len, ctx, check=None):
     sess = O.Session(model, osched, prompt, gen_len)
     sess.prefill()
     ctx.dllm_prefill(gsched, prompt, gen_len)
@@ -87,6 +87,8 @@ def _run_teacher_forced(model, osched, gsched, prompt, gen_len, ctx):
                 assert go[key] == oo[key], (key, go, oo)
             g_tok, g_st, _ = ctx.dllm_get_state()
             o_tok, o_st, _ = sess.state()
+            if check is not None:
+                check(sess, ctx, oo, go, (o_tok0, o_st0), (o_tok, o_st), (g_tok[0], g_st[0]))
             if _unambiguous_commits(od, o_tok0, o_st0, ow["c0"], ow["c1"], ow["w0"], oo["n_committed"]):
                 newly_o = (o_st == O.COMMITTED) & (o_st0 == O.MASKED)
                 newly_g = (g_st[0] == O.COMMITTED) & (g_st0[0] == O.MASKED)
@@ -182,6 +184,47 @@ def test_threshold_commit_generation_mid_thresholds(model):
     assert stable_direct == int((st[0, 32:96] == STABLE).sum())
     again, _ = ctx.dllm_generate(sched, prompt, 64)
     assert np.array_equal(again[0], tok[0, 32:96])
+    ctx.close()
+
+
+@pytest.mark.parametrize("theta_stable", [2.0, 0.0])
+def test_sparse_cache_refresh_teacher_forced(model, theta_stable):
+    """Sparse cache refresh of 8 visible prefix positions per step (Sec. 3.3).  Every step: the
+    same tracked positions as the oracle, their decisions within tolerance, the same refresh and
+    stabilization counts, and the same prefix states after the step; at the end the prefix K/V
+    (refreshed in place by the merges) against the oracle's.  theta_stable 2: the rows only
+    refresh; 0: every tracked row also becomes STABLE."""
+    from paper_2606_13740_gb300 import Sched
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=61)
+    osched = O.OracleSched(steps_per_block=4, scr_rows=8, theta_stable=theta_stable)
+    gsched = Sched(steps_per_block=4, scr_rows=8, theta_stable=theta_stable)
+    counts = {"steps_with_rows": 0}
+
+    def check(sess, ctx, oo, go, before, o_after, g_after):
+        od, gd = sess.scr_decisions(), ctx.dllm_get_scr_debug()
+        n = len(od["pos"])
+        assert np.array_equal(gd["pos"][:n], od["pos"]) and (gd["pos"][n:] == -1).all()
+        if n:
+            counts["steps_with_rows"] += 1
+            assert np.allclose(gd["conf"][:n], od["conf"], rtol=0.05)
+            assert np.allclose(gd["tokconf"][:n], od["tokconf"], rtol=0.05)
+            safe = od["margin"] > 0.05
+            assert np.array_equal(gd["x0"][:n][safe], od["x0"][safe])
+        for key in ("n_refreshed", "n_revised", "n_stable"):
+            assert go[key] == oo[key], (key, go, oo)
+        kv = sess.window()["kv_len"]
+        assert np.array_equal(g_after[1][:kv], o_after[1][:kv])  # the prefix states
+        assert np.array_equal(g_after[0][:kv], o_after[0][:kv])
+
+    ctx = _gpu_ctx()
+    sess, steps, worst = _run_teacher_forced(model, osched, gsched, prompt, 96, ctx, check)
+    assert steps == 12 and counts["steps_with_rows"] >= 4
+    kv_len = sess.state()[2]
+    for layer in range(TINY.n_layers):
+        for which in (0, 1):
+            ref = sess.prefix_kv(layer, which)
+            got = ctx.dllm_get_kv(layer, which, 0, 0, kv_len)
+            assert np.linalg.norm(got - ref) / np.linalg.norm(ref) <= 1e-2
     ctx.close()
 
 
