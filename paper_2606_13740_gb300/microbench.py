@@ -223,7 +223,9 @@ def generate(a):
     the threshold commit rule (staged token stabilization) on the 256-token prompt with the
     paper's thresholds (0.7 visible, 0.9 stable; a random-weight model's confidences stay near
     1/V, so every step takes the single-position fallback) and with theta_visible 0 (a whole
-    block per step: the rule's fastest case)."""
+    block per step: the rule's fastest case); and sparse cache refresh of 32 visible prefix
+    positions per step (random weights never reach theta_stable, so from the second block on
+    every step carries 32 refresh rows besides its 32-token window)."""
     import time
 
     import numpy as np
@@ -240,8 +242,10 @@ def generate(a):
             ("threshold_0.7_0.9_p256_g128", 256, 128,
              Sched(steps_per_block=32, commit_mode=COMMIT_THRESHOLD, theta_visible=0.7, theta_stable=0.9)),
             ("threshold_0_p256_g128", 256, 128,
-             Sched(steps_per_block=32, commit_mode=COMMIT_THRESHOLD, theta_visible=0.0, theta_stable=0.9))):
-        cfg = Config(max_batch=1, max_ctx=Lp + gen, max_window=max(Lp, 96), n_layers=a.layers, **SHAPE_8B)
+             Sched(steps_per_block=32, commit_mode=COMMIT_THRESHOLD, theta_visible=0.0, theta_stable=0.9)),
+            ("scr32_p256_g128", 256, 128, Sched(steps_per_block=32, scr_rows=32))):
+        cfg = Config(max_batch=1, max_ctx=Lp + gen, max_window=max(Lp, 96 + sched.scr_rows), n_layers=a.layers,
+                     **SHAPE_8B)
         ctx = Context(cfg)
         prompt = I.uniform_prompt(Lp, cfg.vocab, cfg.mask_id)
         ctx.dllm_generate(sched, prompt, gen)  # warm-up: graphs for every window shape
