@@ -649,9 +649,23 @@ int orc_denoise_step(orc_session* x, orc_step_out* out, int keep_logits) {
         w0 = x->kv_len;
         w1 = x->c1;
         if (x->s.spec_blocks > 0 && masked <= x->s.spec_trigger && x->c1 < x->n_pos) {
-            spec = 1;
-            w1 = x->c1 + x->s.spec_blocks * x->s.block_len;
-            if (w1 > x->n_pos) w1 = x->n_pos;
+            int k = x->s.spec_blocks;
+            if (x->s.spec_allowance >= 0.0f && x->s.spec_lat_n > 0) {
+                /* greedy: one more future block while the step stays within the allowance */
+                int i0 = (x->c1 - w0 + x->s.block_len - 1) / x->s.block_len - 1;
+                k = 0;
+                for (int j = 1; j <= x->s.spec_blocks; ++j) {
+                    int i = i0 + j;
+                    if (i0 < 0 || i >= x->s.spec_lat_n || i0 >= x->s.spec_lat_n) break;
+                    if (x->s.spec_lat[i] > (1.0f + x->s.spec_allowance) * x->s.spec_lat[i0]) break;
+                    k = j;
+                }
+            }
+            if (k > 0) {
+                spec = 1;
+                w1 = x->c1 + k * x->s.block_len;
+                if (w1 > x->n_pos) w1 = x->n_pos;
+            }
         }
     } else {
         w0 = 0;

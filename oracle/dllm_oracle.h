@@ -49,6 +49,13 @@ typedef struct {
     int commit_mode;       /* ORC_COMMIT_SCHEDULE or ORC_COMMIT_THRESHOLD */
     float theta_visible;   /* threshold mode: promotion of a masked position to visible */
     int scr_rows;          /* sparse cache refresh: prefix positions re-scored per step (0 = off) */
+    /* Adaptive lookahead (Sec. 3.2): with spec_allowance >= 0 and a latency table, the window
+     * takes the largest k <= spec_blocks future blocks for which every step up to k stays
+     * within (1 + spec_allowance) times the latency without lookahead: spec_lat[i] = the step
+     * latency with a window of i + 1 blocks.  spec_allowance < 0: all spec_blocks (fixed). */
+    float spec_allowance;
+    int spec_lat_n;
+    float spec_lat[8];
 } orc_sched;
 
 /* Commit rules.  SCHEDULE: LLaDA's fixed schedule, ceil(m / (S - step)) of the m masked

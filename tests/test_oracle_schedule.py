@@ -412,3 +412,40 @@ def test_scr_revision_replaces_ids_and_skips_their_merge(tiny_model):
         assert tok1[p] == x and st1[p] == O.COMMITTED
     moved = set(np.flatnonzero(np.abs(k1 - k0).max(axis=1) > 0).tolist())
     assert moved == set(kept)
+
+
+# ------------------------------------------------------------ adaptive lookahead (Sec. 3.2)
+def _lookahead_windows(model, **kw):
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=71)
+    sess = O.Session(model, O.OracleSched(steps_per_block=8, spec_blocks=3, spec_trigger=4, **kw), prompt, 160)
+    sess.prefill()
+    windows = []
+    while sess.begin_block():
+        while True:
+            out = sess.step()
+            windows.append(sess.window()["T"])
+            if out["block_done"]:
+                break
+    return windows, sess.state()[0]
+
+
+def test_adaptive_lookahead_takes_the_blocks_within_the_allowance(tiny_model):
+    lat = (1.0, 1.05, 1.1, 2.0)  # step latency with 1, 2, 3, 4 blocks of window
+    w, _ = _lookahead_windows(tiny_model, spec_allowance=0.12, spec_lat=lat)
+    assert set(w) <= {32, 64, 96} and 96 in w  # two future blocks at most: 1.1 <= 1.12 < 2.0
+    w5, _ = _lookahead_windows(tiny_model, spec_allowance=0.06, spec_lat=lat)
+    assert set(w5) <= {32, 64} and 64 in w5
+
+
+def test_adaptive_lookahead_reduces_to_fixed_and_to_none(tiny_model):
+    # an allowance no table entry exceeds: every spec block, the fixed form; 0 with a rising
+    # table: none, the plain block-wise decoding
+    lat = (1.0, 1.05, 1.1, 2.0)
+    fixed_w, fixed_tok = _lookahead_windows(tiny_model)
+    wide_w, wide_tok = _lookahead_windows(tiny_model, spec_allowance=10.0, spec_lat=lat)
+    assert wide_w == fixed_w and np.array_equal(wide_tok, fixed_tok)
+    none_w, none_tok = _lookahead_windows(tiny_model, spec_allowance=0.0, spec_lat=lat)
+    assert set(none_w) == {32}
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=71)
+    plain = O.Session(tiny_model, O.OracleSched(steps_per_block=8), prompt, 160).generate()
+    assert np.array_equal(none_tok[32:], plain)
