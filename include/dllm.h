@@ -106,6 +106,14 @@ typedef struct {
      * step (the merge is not visible inside the step).  The window then counts scr_rows more
      * rows against max_window. */
     int scr_rows;
+    /* Adaptive lookahead (Sec. 3.2): with spec_allowance >= 0 and spec_lat_n > 0, once the
+     * lookahead triggers the window takes the largest k <= spec_blocks future blocks for which
+     * every step up to k stays within (1 + spec_allowance) times the latency without lookahead;
+     * spec_lat[i] = the measured step latency with a window of i + 1 blocks (the window-size
+     * sweep).  k = 0 runs the plain window.  spec_allowance < 0: all spec_blocks (fixed). */
+    float spec_allowance;
+    int spec_lat_n;
+    float spec_lat[8];
 } dllm_sched;
 #define DLLM_MAX_SCR_ROWS 32
 

@@ -610,7 +610,7 @@ static int start_request(dllm_ctx* ctx, const dllm_sched* sched, int batch, int 
     if (sched->steps_per_block < 1 || sched->remask_max < 0 || sched->spec_blocks < 0 ||
         (sched->commit_mode != DLLM_COMMIT_SCHEDULE && sched->commit_mode != DLLM_COMMIT_THRESHOLD) ||
         !(sched->theta_visible == sched->theta_visible) || sched->scr_rows < 0 ||
-        sched->scr_rows > DLLM_MAX_SCR_ROWS)
+        sched->scr_rows > DLLM_MAX_SCR_ROWS || sched->spec_lat_n < 0 || sched->spec_lat_n > 8)
         return fail(ctx, DLLM_EINVAL, "bad schedule");
     if (sched->scr_rows > 0 && (!sched->use_prefix_cache || batch != 1))
         return fail(ctx, DLLM_EINVAL, "sparse cache refresh needs one sequence and the prefix cache");
@@ -754,8 +754,22 @@ int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out) {
             int rc = count_masked_max(ctx, ctx->c0, ctx->c1, &m);
             if (rc) return rc;
             if (m <= s.spec_trigger) {
-                spec = 1;
-                w1 = std::min(ctx->c1 + s.spec_blocks * bl, ctx->n_pos);
+                int k = s.spec_blocks;
+                if (s.spec_allowance >= 0.0f && s.spec_lat_n > 0) {
+                    // greedy: one more future block while the step stays within the allowance
+                    const int i0 = (ctx->c1 - w0 + bl - 1) / bl - 1;
+                    k = 0;
+                    for (int j = 1; j <= s.spec_blocks; ++j) {
+                        const int i = i0 + j;
+                        if (i0 < 0 || i >= s.spec_lat_n || i0 >= s.spec_lat_n) break;
+                        if (s.spec_lat[i] > (1.0f + s.spec_allowance) * s.spec_lat[i0]) break;
+                        k = j;
+                    }
+                }
+                if (k > 0) {
+                    spec = 1;
+                    w1 = std::min(ctx->c1 + k * bl, ctx->n_pos);
+                }
             }
         }
         T = w1 - w0;

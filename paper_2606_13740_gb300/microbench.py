@@ -33,6 +33,9 @@ def main(argv=None):
     ap.add_argument("--dump", default="", help="gemm-trace: write every CTA's timeline to this JSON file")
     ap.add_argument("--no-pdl", action="store_true")
     ap.add_argument("--debug", type=int, default=0, help="step-trace: extra dllm_set_debug flags")
+    ap.add_argument("--lat", type=float, nargs="*", default=[3.37, 3.97, 4.14],
+                    help="generate: step ms with a window of 1, 2, 3 blocks (the window sweep at batch 1)")
+    ap.add_argument("--allowance", type=float, default=0.2, help="generate: adaptive lookahead allowance")
     a = ap.parse_args(argv)
     lib()
     dev = torch.device("cuda:0")
@@ -225,7 +228,8 @@ def generate(a):
     1/V, so every step takes the single-position fallback) and with theta_visible 0 (a whole
     block per step: the rule's fastest case); and sparse cache refresh of 32 visible prefix
     positions per step (random weights never reach theta_stable, so from the second block on
-    every step carries 32 refresh rows besides its 32-token window)."""
+    every step carries 32 refresh rows besides its 32-token window); and the 1024-token workload
+    with adaptive lookahead from the window sweep's step times (--lat, --allowance)."""
     import time
 
     import numpy as np
@@ -243,7 +247,10 @@ def generate(a):
              Sched(steps_per_block=32, commit_mode=COMMIT_THRESHOLD, theta_visible=0.7, theta_stable=0.9)),
             ("threshold_0_p256_g128", 256, 128,
              Sched(steps_per_block=32, commit_mode=COMMIT_THRESHOLD, theta_visible=0.0, theta_stable=0.9)),
-            ("scr32_p256_g128", 256, 128, Sched(steps_per_block=32, scr_rows=32))):
+            ("scr32_p256_g128", 256, 128, Sched(steps_per_block=32, scr_rows=32)),
+            ("adaptive_lookahead_p1024_g256", 1024, 256,
+             Sched(steps_per_block=32, spec_trigger=8, spec_blocks=2, theta_remask=0.5, remask_max=1,
+                   spec_allowance=a.allowance, spec_lat=tuple(a.lat)))):
         cfg = Config(max_batch=1, max_ctx=Lp + gen, max_window=max(Lp, 96 + sched.scr_rows), n_layers=a.layers,
                      **SHAPE_8B)
         ctx = Context(cfg)

@@ -228,6 +228,25 @@ def test_sparse_cache_refresh_teacher_forced(model, theta_stable):
     ctx.close()
 
 
+def test_adaptive_lookahead_teacher_forced(model):
+    """Adaptive lookahead (Sec. 3.2) from a latency table: every step's window equals the
+    oracle's (the harness compares them), and the table admits two future blocks, not three."""
+    from paper_2606_13740_gb300 import Sched
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=71)
+    lat = (1.0, 1.05, 1.1, 2.0)
+    osched = O.OracleSched(steps_per_block=8, spec_blocks=3, spec_trigger=4, spec_allowance=0.12, spec_lat=lat)
+    gsched = Sched(steps_per_block=8, spec_blocks=3, spec_trigger=4, spec_allowance=0.12, spec_lat=lat)
+    ctx = _gpu_ctx(max_window=160)
+    windows = []
+
+    def check(sess, ctx, oo, go, before, o_after, g_after):
+        windows.append(sess.window()["T"])
+
+    _run_teacher_forced(model, osched, gsched, prompt, 160, ctx, check)
+    assert 96 in windows and 128 not in windows
+    ctx.close()
+
+
 def test_generate_matches_stepwise_and_is_deterministic(model):
     from paper_2606_13740_gb300 import Sched
     prompt = I.uniform_prompt(64, TINY.vocab, TINY.mask_id)
