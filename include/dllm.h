@@ -96,8 +96,8 @@ typedef struct {
     int use_prefix_cache;
     int commit_mode;      /* DLLM_COMMIT_SCHEDULE or DLLM_COMMIT_THRESHOLD */
     float theta_visible;  /* threshold mode only */
-    /* Sparse cache refresh (Sec. 3.3; one sequence with the prefix cache on; 0 = off, at most
-     * DLLM_MAX_SCR_ROWS): each step the first scr_rows prefix positions that are COMMITTED
+    /* Sparse cache refresh (Sec. 3.3; with the prefix cache on; 0 = off, at most
+     * DLLM_MAX_SCR_ROWS): each step, per sequence, the first scr_rows prefix positions that are COMMITTED
      * (visible, not stable) run with the window as extra query rows at their own positions,
      * attending to the prefix as cached and to the window and adding no keys.  After the
      * commit pass each is re-scored: STABLE at tokconf >= theta_stable; below theta_remask
@@ -202,8 +202,8 @@ int dllm_set_state(dllm_ctx* ctx, const int32_t* tokens, const uint8_t* status);
  * Synchronises. */
 int dllm_get_step_debug(dllm_ctx* ctx, float* logits, int32_t* argmax, float* conf, float* tokconf);
 
-/* The last step's sparse-cache-refresh rows: pos, argmax, conf, tokconf (host arrays of
- * scr_rows entries, nullable; pos -1 = an unused row); *n = scr_rows.  Synchronises. */
+/* The last step's sparse-cache-refresh rows: pos, argmax, conf, tokconf (host arrays
+ * [batch][scr_rows], nullable; pos -1 = an unused row); *n = scr_rows.  Synchronises. */
 int dllm_get_scr_debug(dllm_ctx* ctx, int32_t* pos, int32_t* argmax, float* conf, float* tokconf, int* n);
 
 /* flags bit 0: materialise logits; bit 1: disable CUDA graphs; bit 2: launch

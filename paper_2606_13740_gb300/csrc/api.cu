@@ -105,11 +105,11 @@ Layout make_layout(const dllm_config& c) {
     L.off_plan = take(static_cast<size_t>(c.max_batch) * 16);
     L.off_outs = take(static_cast<size_t>(c.max_batch) * 32);
     L.off_status = take(16);
-    // sparse cache refresh (one sequence): tracked positions, merge flags, side K/V
-    // [L][2][H][DLLM_MAX_SCR_ROWS][hd]
-    L.off_trk = take(DLLM_MAX_SCR_ROWS * 4);
-    L.off_smerge = take(DLLM_MAX_SCR_ROWS * 4);
-    L.off_side = take(static_cast<size_t>(c.n_layers) * 2 * L.qd * DLLM_MAX_SCR_ROWS * 2);
+    // sparse cache refresh: tracked positions and merge flags [B][R], side K/V
+    // [L][2][B][H][R][hd] (R <= DLLM_MAX_SCR_ROWS)
+    L.off_trk = take(static_cast<size_t>(c.max_batch) * DLLM_MAX_SCR_ROWS * 4);
+    L.off_smerge = take(static_cast<size_t>(c.max_batch) * DLLM_MAX_SCR_ROWS * 4);
+    L.off_side = take(static_cast<size_t>(c.n_layers) * 2 * c.max_batch * L.qd * DLLM_MAX_SCR_ROWS * 2);
     L.total = o;
     return L;
 }
@@ -251,7 +251,7 @@ static int sync_check(dllm_ctx* ctx) {
 // ------------------------------------------------------------------ forward
 // Layers (and optionally the LM head) over T window tokens of each of the B
 // sequences; token ids come from the state at seq_kv[b] + t.
-// T window rows per sequence, then (sparse cache refresh, one sequence) R tracked prefix rows:
+// T window rows per sequence, then (sparse cache refresh) R tracked prefix rows:
 // they run through every projection and the head, attend as queries only, and their K/V go to
 // the side buffers.
 static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0) {
@@ -310,8 +310,8 @@ static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0) {
         EpiArgs e = ep;
         e.kc = ctx->kv + static_cast<size_t>(2 * l) * L.kv_half;
         e.vc = ctx->kv + static_cast<size_t>(2 * l + 1) * L.kv_half;
-        e.kside = ctx->scr_side + static_cast<size_t>(2 * l) * qd * R;  // [L][2][H][R][hd]
-        e.vside = e.kside + static_cast<size_t>(qd) * R;
+        e.kside = ctx->scr_side + static_cast<size_t>(2 * l) * B * qd * R;  // [L][2][B][H][R][hd]
+        e.vside = e.kside + static_cast<size_t>(B) * qd * R;
         return e;
     };
     // phase slot i of a chain uses scratch slot i; consecutive chains are ordered by the stream
@@ -380,7 +380,7 @@ static int step_kernels(dllm_ctx* ctx, int T) {
     mark(ctx, -1);
     const int R = ctx->sched.use_prefix_cache ? ctx->sched.scr_rows : 0;
     if (R > 0) {  // the visible prefix positions this step refreshes
-        CK(launch_scr_select(ctx->st, ctx->seq_kv, ctx->trk, R, ctx->stream));
+        CK(launch_scr_select(ctx->st, ctx->cfg.max_ctx, ctx->seq_kv, ctx->trk, ctx->B, R, ctx->stream));
         mark(ctx, DLLM_K_COMMIT);
     }
     int rc = forward(ctx, ctx->B, T, true, R);
@@ -417,8 +417,9 @@ static int step_kernels(dllm_ctx* ctx, int T) {
     cudaError_t ce = launch_commit(a, ctx->stream);
     mark(ctx, DLLM_K_COMMIT);
     if (ce == cudaSuccess && R > 0) {  // the refreshed K/V merged at the step boundary
-        ce = launch_scr_merge(ctx->scr_side, ctx->kv, ctx->trk, ctx->scr_merge, ctx->cfg.n_layers, ctx->cfg.n_heads,
-                              ctx->cfg.head_dim, ctx->cfg.max_ctx, R, ctx->stream);
+        ce = launch_scr_merge(ctx->scr_side, ctx->kv, ctx->trk, ctx->scr_merge, ctx->cfg.n_layers, ctx->B,
+                              ctx->cfg.max_batch, ctx->cfg.n_heads, ctx->cfg.head_dim, ctx->cfg.max_ctx, R,
+                              ctx->stream);
         mark(ctx, DLLM_K_COMMIT);
     }
     ctx->in_step = false;
@@ -612,8 +613,8 @@ static int start_request(dllm_ctx* ctx, const dllm_sched* sched, int batch, int 
         !(sched->theta_visible == sched->theta_visible) || sched->scr_rows < 0 ||
         sched->scr_rows > DLLM_MAX_SCR_ROWS || sched->spec_lat_n < 0 || sched->spec_lat_n > 8)
         return fail(ctx, DLLM_EINVAL, "bad schedule");
-    if (sched->scr_rows > 0 && (!sched->use_prefix_cache || batch != 1))
-        return fail(ctx, DLLM_EINVAL, "sparse cache refresh needs one sequence and the prefix cache");
+    if (sched->scr_rows > 0 && !sched->use_prefix_cache)
+        return fail(ctx, DLLM_EINVAL, "sparse cache refresh needs the prefix cache");
     if (sched->use_prefix_cache && c.block_len * (1 + sched->spec_blocks) + sched->scr_rows > c.max_window)
         return fail(ctx, DLLM_ECAPACITY, "window plus refresh rows > max_window %d", c.max_window);
     if (batch > c.max_batch) return fail(ctx, DLLM_ECAPACITY, "batch %d > max_batch %d", batch, c.max_batch);
@@ -968,14 +969,19 @@ int dllm_set_state(dllm_ctx* ctx, const int32_t* tokens, const uint8_t* status) 
 
 int dllm_get_step_debug(dllm_ctx* ctx, float* logits, int32_t* argmax, float* conf, float* tokconf) {
     GUARD(ctx);
-    const size_t n = static_cast<size_t>(ctx->B) * ctx->last_T;
+    // a sequence's rows: its T window rows (then, with sparse cache refresh, its refresh rows)
+    const size_t T = static_cast<size_t>(ctx->last_T), B = static_cast<size_t>(ctx->B);
+    const size_t Tq = T + (ctx->sched.use_prefix_cache ? ctx->sched.scr_rows : 0);
+    const size_t V = static_cast<size_t>(ctx->cfg.vocab);
     if (logits) {
         if (!(ctx->debug & 1) || !ctx->logits) return fail(ctx, DLLM_EINVAL, "logits need dllm_set_debug(1)");
-        CK(cudaMemcpyAsync(logits, ctx->logits, n * ctx->cfg.vocab * 4, cudaMemcpyDeviceToHost, ctx->stream));
+        CK(cudaMemcpy2DAsync(logits, T * V * 4, ctx->logits, Tq * V * 4, T * V * 4, B, cudaMemcpyDeviceToHost,
+                             ctx->stream));
     }
-    if (argmax) CK(cudaMemcpyAsync(argmax, ctx->x0, n * 4, cudaMemcpyDeviceToHost, ctx->stream));
-    if (conf) CK(cudaMemcpyAsync(conf, ctx->conf, n * 4, cudaMemcpyDeviceToHost, ctx->stream));
-    if (tokconf) CK(cudaMemcpyAsync(tokconf, ctx->tokconf, n * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    if (argmax) CK(cudaMemcpy2DAsync(argmax, T * 4, ctx->x0, Tq * 4, T * 4, B, cudaMemcpyDeviceToHost, ctx->stream));
+    if (conf) CK(cudaMemcpy2DAsync(conf, T * 4, ctx->conf, Tq * 4, T * 4, B, cudaMemcpyDeviceToHost, ctx->stream));
+    if (tokconf)
+        CK(cudaMemcpy2DAsync(tokconf, T * 4, ctx->tokconf, Tq * 4, T * 4, B, cudaMemcpyDeviceToHost, ctx->stream));
     return sync_check(ctx);
 }
 
@@ -984,12 +990,13 @@ int dllm_get_scr_debug(dllm_ctx* ctx, int32_t* pos, int32_t* argmax, float* conf
     const int R = ctx->sched.use_prefix_cache ? ctx->sched.scr_rows : 0;
     if (n) *n = R;
     if (R == 0) return DLLM_OK;
-    const size_t off = static_cast<size_t>(ctx->last_T);  // one sequence: rows T .. T + R - 1
-    if (pos) CK(cudaMemcpyAsync(pos, ctx->trk, static_cast<size_t>(R) * 4, cudaMemcpyDeviceToHost, ctx->stream));
-    if (argmax) CK(cudaMemcpyAsync(argmax, ctx->x0 + off, static_cast<size_t>(R) * 4, cudaMemcpyDeviceToHost, ctx->stream));
-    if (conf) CK(cudaMemcpyAsync(conf, ctx->conf + off, static_cast<size_t>(R) * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    // sequence b's rows T .. T + R - 1 of its T + R
+    const size_t T = static_cast<size_t>(ctx->last_T), Tq = T + R, B = static_cast<size_t>(ctx->B);
+    if (pos) CK(cudaMemcpyAsync(pos, ctx->trk, B * R * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    if (argmax) CK(cudaMemcpy2DAsync(argmax, R * 4, ctx->x0 + T, Tq * 4, R * 4, B, cudaMemcpyDeviceToHost, ctx->stream));
+    if (conf) CK(cudaMemcpy2DAsync(conf, R * 4, ctx->conf + T, Tq * 4, R * 4, B, cudaMemcpyDeviceToHost, ctx->stream));
     if (tokconf)
-        CK(cudaMemcpyAsync(tokconf, ctx->tokconf + off, static_cast<size_t>(R) * 4, cudaMemcpyDeviceToHost, ctx->stream));
+        CK(cudaMemcpy2DAsync(tokconf, R * 4, ctx->tokconf + T, Tq * 4, R * 4, B, cudaMemcpyDeviceToHost, ctx->stream));
     return sync_check(ctx);
 }
 

@@ -279,7 +279,7 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                     bs[u] = b;
                     ts[u] = cg + u - b * ep.T;
                     // a window row, or (sparse cache refresh) a tracked prefix position
-                    const int ps = ts[u] < ep.Tw ? sm.kvs[b] + ts[u] : max(ep.trk[ts[u] - ep.Tw], 0);
+                    const int ps = ts[u] < ep.Tw ? sm.kvs[b] + ts[u] : max(ep.trk[b * ep.R + ts[u] - ep.Tw], 0);
                     const float2 r = rot_cs(static_cast<float>(ps) * theta);
                     cs[u] = r.x;
                     ss[u] = r.y;
@@ -361,7 +361,7 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
             const int b = min(col / ep.T, ep.n_seq - 1);
             const int ts = col - b * ep.T;
             const bool tracked = ts >= ep.Tw;  // sparse cache refresh: K/V to the side buffers
-            const int pos = tracked ? ep.trk[ts - ep.Tw] : sm.kvs[b] + ts;
+            const int pos = tracked ? ep.trk[b * ep.R + ts - ep.Tw] : sm.kvs[b] + ts;
             const int head = (mt * kBM - part * ep.H * ep.hd + f0) / ep.hd;
             const int fi0 = f0 % ep.hd;
             if (tracked && part > 0) {
@@ -370,7 +370,7 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                         reinterpret_cast<const __nv_bfloat16*>(sm.stg) + tok * kBM + f0);
                     __nv_bfloat16* side = part == 1 ? ep.kside : ep.vside;
                     uint4* dst = reinterpret_cast<uint4*>(
-                        side + (static_cast<size_t>(head) * ep.R + (ts - ep.Tw)) * ep.hd + fi0);
+                        side + ((static_cast<size_t>(b) * ep.H + head) * ep.R + (ts - ep.Tw)) * ep.hd + fi0);
 #pragma unroll
                     for (int i = 0; i < 2; ++i) dst[i] = src[i];
                 }

@@ -57,9 +57,9 @@ struct EpiArgs {
     // EPI_SWIGLU: tile k row 2f is gate feature 64k+f, row 2f+1 the matching up row
     __nv_bfloat16* h;    // [N][F]
     int F;
-    // EPI_QKV with sparse cache refresh (one sequence): of the T rows the first Tw are the
-    // window, row Tw + r is the prefix position trk[r] (< 0: an unused row, no K/V written),
-    // whose K and V go to kside / vside [H][R][hd] instead of the cache
+    // EPI_QKV with sparse cache refresh: of a sequence's T rows the first Tw are the window,
+    // row Tw + r of sequence b is the prefix position trk[b R + r] (< 0: an unused row, no K/V
+    // written), whose K and V go to kside / vside [B][H][R][hd] instead of the cache
     int Tw, R;
     const int* trk;
     __nv_bfloat16* kside;
@@ -179,17 +179,19 @@ cudaError_t launch_init_kv_random(__nv_bfloat16* cache, int B, int H, int hd, in
                                   int which, int L, uint64_t seed, cudaStream_t st);
 // x = embedding rows of the window's ids (fp32), xb = bf16(x), sq[d/128][N] = per-128-feature
 // sums of x^2, cur[N] = the ids (for the LM head's current-token probability).
-// T rows per sequence: the first Tw at the window positions seq_kv[b] + t, the rest (one
-// sequence) at the prefix positions trk[t - Tw] (< 0: id 0).
+// T rows per sequence: the first Tw at the window positions seq_kv[b] + t, the rest at the
+// prefix positions trk[b (T - Tw) + t - Tw] (< 0: id 0).
 cudaError_t launch_embed(const int* tok, int tok_ld, const int* seq_kv, const __nv_bfloat16* emb, float* x,
                          __nv_bfloat16* xb, float* sq, int* cur, int* epoch, int B, int T, int d, cudaStream_t st,
                          int Tw = -1, const int* trk = nullptr);
-// Sparse cache refresh (one sequence): trk[r] = the r-th COMMITTED position below seq_kv[0]
-// (ascending), -1 past the last; merge: the K/V rows of the refreshed positions (merge[r] != 0)
-// from the side buffers [L][2][H][R][hd] into the cache [L][2][1][H][cap][hd].
-cudaError_t launch_scr_select(const uint8_t* st, const int* seq_kv, int* trk, int R, cudaStream_t stream);
+// Sparse cache refresh: trk[b R + r] = the r-th COMMITTED position of sequence b below
+// seq_kv[b] (ascending), -1 past the last (state rows st + b ld); merge: the K/V rows of the
+// refreshed positions (merge[b R + r] != 0) from the side buffers [L][2][B][H][R][hd] into the
+// cache [L][2][kv_B][H][cap][hd].
+cudaError_t launch_scr_select(const uint8_t* st, int ld, const int* seq_kv, int* trk, int B, int R,
+                              cudaStream_t stream);
 cudaError_t launch_scr_merge(const __nv_bfloat16* side, __nv_bfloat16* cache, const int* trk, const int* merge, int L,
-                             int H, int hd, int cap, int R, cudaStream_t stream);
+                             int B, int kv_B, int H, int hd, int cap, int R, cudaStream_t stream);
 // The kernels below are launched with PDL when `pdl` (inside the context's step chain); the
 // single-kernel entry points pass false because their inputs may come from foreign kernels.
 // Attention plan: CTAs (split, head, sequence x query tile of 16*nw rows); the csize
@@ -238,8 +240,8 @@ struct CommitArgs {
     float theta_remask, theta_stable;
     int commit_mode;     // DLLM_COMMIT_SCHEDULE / DLLM_COMMIT_THRESHOLD (dllm.h)
     float theta_visible;
-    // rows per sequence of x0 / conf / tokconf (T, or T + R with sparse cache refresh: rows
-    // T + r are the prefix positions trk[r]; one sequence); merge[r]: its K/V are merged
+    // rows per sequence of x0 / conf / tokconf (T, or T + R with sparse cache refresh: row
+    // T + r of sequence b is the prefix position trk[b R + r]); merge[b R + r]: its K/V are merged
     int Tq, R;
     const int* trk;
     int* merge;

@@ -137,7 +137,7 @@ __global__ void __launch_bounds__(256) k_embed(const int* tok, int tok_ld, const
     if (j == 0 && threadIdx.x == 0) *epoch += 1;  // one forward pass: a new tag for the chained projections
     const int b = j / T, t = j - b * T;
     // window rows, then (sparse cache refresh, one sequence) the tracked prefix positions
-    const int pos = t < Tw ? seq_kv[b] + t : trk[t - Tw];
+    const int pos = t < Tw ? seq_kv[b] + t : trk[b * (T - Tw) + t - Tw];
     const int id = pos >= 0 ? tok[static_cast<size_t>(b) * tok_ld + pos] : 0;
     if (threadIdx.x == 0) cur[j] = id;
     const __nv_bfloat16* e = emb + static_cast<size_t>(id) * d;
@@ -163,7 +163,7 @@ cudaError_t launch_embed(const int* tok, int tok_ld, const int* seq_kv, const __
                          __nv_bfloat16* xb, float* sq, int* cur, int* epoch, int B, int T, int d, cudaStream_t st,
                          int Tw, const int* trk) {
     if (Tw < 0) Tw = T;
-    if (Tw < T && (!trk || B != 1)) return cudaErrorInvalidValue;
+    if (Tw < T && !trk) return cudaErrorInvalidValue;
     return launch_k(k_embed, dim3(B * T), dim3(256), 0, st, true, tok, tok_ld, seq_kv, emb, x, xb, sq, cur, epoch, T,
                     B * T, d, Tw, trk);
 }
@@ -763,10 +763,10 @@ __global__ void __launch_bounds__(256) k_commit(CommitArgs a) {
         }
     }
     __syncthreads();
-    // sparse cache refresh (one sequence): the tracked prefix positions, rows Tw + r, re-scored;
-    // those that keep their id have their refreshed K/V merged after this kernel
+    // sparse cache refresh: the tracked prefix positions, rows Tw + r, re-scored; those that
+    // keep their id have their refreshed K/V merged after this kernel
     for (int r = threadIdx.x; r < a.R; r += blockDim.x) {
-        const int p = a.trk[r];
+        const int p = a.trk[b * a.R + r];
         int merge = 0;
         if (p >= 0) {
             const float v = tc[a.T + r];
@@ -782,7 +782,7 @@ __global__ void __launch_bounds__(256) k_commit(CommitArgs a) {
             }
             if (merge) atomicAdd(&s_cnt[6], 1);
         }
-        a.merge[r] = merge;
+        a.merge[b * a.R + r] = merge;
     }
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -800,14 +800,19 @@ __global__ void __launch_bounds__(256) k_commit(CommitArgs a) {
 }
 
 // ------------------------------------------------------------------ sparse cache refresh
-// One CTA: trk[r] = the r-th position p < seq_kv[0] whose state is COMMITTED (ascending), -1
-// past the last.  Positions are scanned 256 at a time with a block-wide prefix count.
-__global__ void __launch_bounds__(256) k_scr_select(const uint8_t* st, const int* seq_kv, int* trk, int R) {
+// One CTA per sequence b: trk[b R + r] = the r-th position p < seq_kv[b] whose state is
+// COMMITTED (ascending), -1 past the last.  Positions are scanned 256 at a time with a
+// block-wide prefix count.
+__global__ void __launch_bounds__(256) k_scr_select(const uint8_t* st_all, int ld, const int* seq_kv, int* trk_all,
+                                                    int R) {
     pdl_wait();
     pdl_launch_dependents();
     __shared__ int s_warp[8];
     __shared__ int s_base;
-    const int kv = seq_kv[0];
+    const int b = blockIdx.x;
+    const uint8_t* st = st_all + static_cast<size_t>(b) * ld;
+    int* trk = trk_all + b * R;
+    const int kv = seq_kv[b];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) s_base = 0;
     for (int r = threadIdx.x; r < R; r += blockDim.x) trk[r] = -1;
@@ -833,37 +838,40 @@ __global__ void __launch_bounds__(256) k_scr_select(const uint8_t* st, const int
     }
 }
 
-cudaError_t launch_scr_select(const uint8_t* st, const int* seq_kv, int* trk, int R, cudaStream_t stream) {
-    return launch_k(k_scr_select, dim3(1), dim3(256), 0, stream, true, st, seq_kv, trk, R);
+cudaError_t launch_scr_select(const uint8_t* st, int ld, const int* seq_kv, int* trk, int B, int R,
+                              cudaStream_t stream) {
+    return launch_k(k_scr_select, dim3(B), dim3(256), 0, stream, true, st, ld, seq_kv, trk, R);
 }
 
-// Grid (R, L): row r of layer l, when merged, copies its K and V rows of every head (hd
-// elements each) from the side buffers into the cache at position trk[r].
+// Grid (R, L, B): row r of sequence b in layer l, when merged, copies its K and V rows of every
+// head (hd elements each) from the side buffers into the cache at position trk[b R + r].
 __global__ void __launch_bounds__(128) k_scr_merge(const __nv_bfloat16* side, __nv_bfloat16* cache, const int* trk,
-                                                   const int* merge, int H, int hd, int cap, int R) {
+                                                   const int* merge, int B, int kv_B, int H, int hd, int cap, int R) {
     pdl_wait();
     pdl_launch_dependents();
-    const int r = blockIdx.x, l = blockIdx.y;
-    const int p = trk[r];
-    if (p < 0 || !merge[r]) return;
-    const size_t side_layer = static_cast<size_t>(2) * H * R * hd;
-    const size_t cache_half = static_cast<size_t>(H) * cap * hd;
+    const int r = blockIdx.x, l = blockIdx.y, b = blockIdx.z;
+    const int p = trk[b * R + r];
+    if (p < 0 || !merge[b * R + r]) return;
+    const size_t side_layer = static_cast<size_t>(2) * B * H * R * hd;
+    const size_t cache_half = static_cast<size_t>(kv_B) * H * cap * hd;
     const int n4 = hd / 8;  // 16-byte pieces per head row
     for (int e = threadIdx.x; e < 2 * H * n4; e += blockDim.x) {
         const int which = e / (H * n4), rem = e - which * H * n4;
         const int h = rem / n4, i = rem - h * n4;
-        const uint4* src = reinterpret_cast<const uint4*>(side + l * side_layer + (static_cast<size_t>(which) * H + h) *
-                                                                                    R * hd + static_cast<size_t>(r) * hd) + i;
+        const uint4* src = reinterpret_cast<const uint4*>(
+                               side + l * side_layer + ((static_cast<size_t>(which) * B + b) * H + h) * R * hd +
+                               static_cast<size_t>(r) * hd) + i;
         uint4* dst = reinterpret_cast<uint4*>(cache + (static_cast<size_t>(2 * l + which)) * cache_half +
-                                              (static_cast<size_t>(h) * cap + p) * hd) + i;
+                                              ((static_cast<size_t>(b) * H + h) * cap + p) * hd) + i;
         *dst = *src;
     }
 }
 
 cudaError_t launch_scr_merge(const __nv_bfloat16* side, __nv_bfloat16* cache, const int* trk, const int* merge, int L,
-                             int H, int hd, int cap, int R, cudaStream_t stream) {
-    if (R < 1 || hd % 8) return cudaErrorInvalidValue;
-    return launch_k(k_scr_merge, dim3(R, L), dim3(128), 0, stream, true, side, cache, trk, merge, H, hd, cap, R);
+                             int B, int kv_B, int H, int hd, int cap, int R, cudaStream_t stream) {
+    if (R < 1 || hd % 8 || B < 1 || B > kv_B) return cudaErrorInvalidValue;
+    return launch_k(k_scr_merge, dim3(R, L, B), dim3(128), 0, stream, true, side, cache, trk, merge, B, kv_B, H, hd,
+                    cap, R);
 }
 
 cudaError_t launch_commit(const CommitArgs& a, cudaStream_t st, bool pdl) {

@@ -273,17 +273,19 @@ class Context:
             r["logits"] = lg.reshape(self.B, T, self.cfg.vocab)
         return r
 
-    def dllm_get_scr_debug(self):
-        """The last step's sparse-cache-refresh rows: positions (-1 unused), argmax, conf, tokconf."""
-        R = 64
-        pos = np.empty(R, np.int32)
-        x0 = np.empty(R, np.int32)
-        conf = np.empty(R, np.float32)
-        tc = np.empty(R, np.float32)
+    def dllm_get_scr_debug(self, seq=0):
+        """The last step's sparse-cache-refresh rows of sequence seq: positions (-1 unused),
+        argmax, conf, tokconf."""
         n = C.c_int()
+        _check(lib().dllm_get_scr_debug(self.h, None, None, None, None, C.byref(n)), self.h)
+        k = max(1, n.value)
+        pos = np.empty((self.B, k), np.int32)
+        x0 = np.empty((self.B, k), np.int32)
+        conf = np.empty((self.B, k), np.float32)
+        tc = np.empty((self.B, k), np.float32)
         _check(lib().dllm_get_scr_debug(self.h, _p(pos), _p(x0), _p(conf), _p(tc), C.byref(n)), self.h)
         k = n.value
-        return {"pos": pos[:k], "x0": x0[:k], "conf": conf[:k], "tokconf": tc[:k]}
+        return {"pos": pos[seq, :k], "x0": x0[seq, :k], "conf": conf[seq, :k], "tokconf": tc[seq, :k]}
 
     def dllm_get_weight(self, layer, which):
         c = self.cfg
