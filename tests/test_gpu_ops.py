@@ -84,6 +84,8 @@ def _attn_ref(q, k, v, kv_len, T):
     # the tensor-core kernel (head dim 128, >= 1024 keys): two 128-row query tiles (the second
     # ragged), eight key splits per cluster, a sequence whose keys fill no split but the first
     (1, 192, 2, 128, [1100], 1300), (1, 32, 1, 128, [2000], 2048), (2, 40, 3, 128, [1, 1500], 1600),
+    # more units than one wave (12 x 32 = 384 > 2 per SM), mixed prefix lengths
+    (12, 64, 32, 128, [1000, 1200, 2000, 964, 1100, 1500, 1960, 1024, 1300, 999, 1700, 1800], 2100),
 ])
 def test_attention_matches_numpy(dev, B, T, H, hd, kv, cap):
     from paper_2606_13740_gb300 import dllm_op_attention
