@@ -114,6 +114,12 @@ typedef struct {
     float spec_allowance;
     int spec_lat_n;
     float spec_lat[8];
+    /* Selective logits skipping (Sec. 3.3; 0 = off, 1 = on): the LM head, its softmax
+     * statistics and the decision run only for the rows that still need one (positions that
+     * are MASKED, COMMITTED or DRAFT, and refresh rows); FIXED and STABLE rows are skipped and
+     * their step decisions read x0 = -1, conf = tokconf = 0.  Ignored while the logits are
+     * captured for debugging. */
+    int sls;
 } dllm_sched;
 #define DLLM_MAX_SCR_ROWS 32
 

@@ -38,6 +38,7 @@ struct Layout {
     int n_sq;
     size_t off_lmp, off_zcur, off_cur, off_x0, off_conf, off_tokconf;
     size_t off_part, part_floats, off_cnt, off_done, off_epoch, off_trk, off_smerge, off_side;
+    size_t off_xc, off_sqc, off_curc, off_rmap, off_nrows;
     int cnt_len, done_len;  // per phase slot
     size_t off_tok, off_st, off_stok, off_sst, off_seqkv, off_plan, off_outs, off_status;
     size_t total;
@@ -110,6 +111,13 @@ Layout make_layout(const dllm_config& c) {
     L.off_trk = take(static_cast<size_t>(c.max_batch) * DLLM_MAX_SCR_ROWS * 4);
     L.off_smerge = take(static_cast<size_t>(c.max_batch) * DLLM_MAX_SCR_ROWS * 4);
     L.off_side = take(static_cast<size_t>(c.n_layers) * 2 * c.max_batch * L.qd * DLLM_MAX_SCR_ROWS * 2);
+    // selective logits skipping: the compacted LM-head operand (bf16 rows, RMSNorm statistics,
+    // current ids), the row map and the row count
+    L.off_xc = take(T * d * 2);
+    L.off_sqc = take(static_cast<size_t>(L.n_sq) * T * 4);
+    L.off_curc = take(T * 4);
+    L.off_rmap = take(T * 4);
+    L.off_nrows = take(16);
     L.total = o;
     return L;
 }
@@ -155,6 +163,9 @@ struct dllm_ctx {
     int* trk = nullptr;
     int* scr_merge = nullptr;
     __nv_bfloat16* scr_side = nullptr;
+    __nv_bfloat16* sls_x = nullptr;  // compacted LM-head rows
+    float* sls_sq = nullptr;
+    int *sls_cur = nullptr, *sls_map = nullptr, *sls_n = nullptr;
     int *chain_cnt = nullptr, *chain_done = nullptr, *epoch = nullptr;
     int *tok = nullptr, *stok = nullptr, *seq_kv = nullptr, *plan = nullptr, *outs = nullptr, *status = nullptr;
     uint8_t *st = nullptr, *sst = nullptr;
@@ -253,8 +264,9 @@ static int sync_check(dllm_ctx* ctx) {
 // sequences; token ids come from the state at seq_kv[b] + t.
 // T window rows per sequence, then (sparse cache refresh) R tracked prefix rows:
 // they run through every projection and the head, attend as queries only, and their K/V go to
-// the side buffers.
-static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0) {
+// the side buffers.  With `sls` (selective logits skipping) the LM head runs as its own launch
+// over the compacted rows that need a decision; the other rows get x0 = -1, conf = tokconf = 0.
+static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0, bool sls = false) {
     const int T = Tw + R;  // rows per sequence
     const dllm_config& c = ctx->cfg;
     const Layout& L = ctx->L;
@@ -270,10 +282,11 @@ static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0) {
     const GemmPlan pg = gemm_plan(L.gu_rows, N, d, ctx->sms, EPI_SWIGLU);
     const GemmPlan pd = gemm_plan(L.d_rows, N, F, ctx->sms, EPI_RESID);
     const GemmPlan ph = gemm_plan(L.head_rows, N, d, ctx->sms, EPI_LMHEAD);
-    CUtensorMap tx_xn, tx_attn, tx_h;
+    CUtensorMap tx_xn, tx_attn, tx_h, tx_c;
     if (!make_tmap_bf16(&tx_xn, ctx->xn, N, d, pq.ntile) || !make_tmap_bf16(&tx_attn, ctx->attn, N, qd, po.ntile) ||
-        !make_tmap_bf16(&tx_h, ctx->h, N, F, pd.ntile))
+        !make_tmap_bf16(&tx_h, ctx->h, N, F, pd.ntile) || !make_tmap_bf16(&tx_c, ctx->sls_x, N, d, ph.ntile))
         return fail(ctx, DLLM_ECUDA, "tensor map encode failed");
+    sls = sls && head;
     AttnPlan ap = attn_plan(B, T, c.n_heads, c.head_dim, ctx->kv_len + Tw, ctx->sms);
     ap.qx = R;
     EpiArgs ep{};
@@ -361,12 +374,30 @@ static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0) {
         add_phase(ca, m, pg, EPI_SWIGLU, ep, 128, w + L.w_gu, tx_xn);
         add_phase(ca, m, pd, EPI_RESID, er, 64, w + L.w_d, tx_h);
         if (l + 1 < c.n_layers) add_phase(ca, m, pq, EPI_QKV, qkv_args(l + 1), 128, ctx->wl[l + 1] + L.w_qkv, tx_xn);
-        else if (head) add_phase(ca, m, ph, EPI_LMHEAD, eh, 128, ctx->head, tx_xn);
+        else if (head && !sls) add_phase(ca, m, ph, EPI_LMHEAD, eh, 128, ctx->head, tx_xn);
         if (int rc = run_chain(ca, m, l + 2, DLLM_K_LAYER)) return rc;
     }
+    if (sls) {
+        CK(launch_sls_map(ctx->st, c.max_ctx, ctx->seq_kv, ctx->sched.use_prefix_cache, B, Tw, T, ctx->sls_map,
+                          ctx->sls_n, ctx->x0, ctx->conf, ctx->tokconf, s));
+        mark(ctx, DLLM_K_HEAD);
+        CK(launch_sls_gather(ctx->sls_map, ctx->sls_n, N, ph.ntile, d, ctx->xn, ctx->sq, L.n_sq, ctx->cur, ctx->sls_x,
+                             ctx->sls_sq, ctx->sls_cur, s));
+        mark(ctx, DLLM_K_HEAD);
+        EpiArgs ec = eh;
+        ec.sq_in = ctx->sls_sq;
+        ec.cur_tok = ctx->sls_cur;
+        ec.logits = nullptr;
+        ChainArgs ca{};
+        ChainMaps m{};
+        add_phase(ca, m, ph, EPI_LMHEAD, ec, 0, ctx->head, tx_c);
+        ca.dyn_rows = ctx->sls_n;  // the head covers only the token tiles holding the listed rows
+        if (int rc = run_chain(ca, m, c.n_layers + 2, DLLM_K_HEAD)) return rc;
+    }
     if (head) {
-        CK(launch_lmhead_reduce(ctx->lmp, ctx->zcur, ctx->cur, L.head_tiles, N, c.mask_id, ctx->x0, ctx->conf,
-                                ctx->tokconf, s));
+        CK(launch_lmhead_reduce(ctx->lmp, ctx->zcur, sls ? ctx->sls_cur : ctx->cur, L.head_tiles, N, c.mask_id,
+                                ctx->x0, ctx->conf, ctx->tokconf, s, true, sls ? ctx->sls_map : nullptr,
+                                sls ? ctx->sls_n : nullptr));
         mark(ctx, DLLM_K_HEAD_REDUCE);
     }
     return DLLM_OK;
@@ -383,7 +414,7 @@ static int step_kernels(dllm_ctx* ctx, int T) {
         CK(launch_scr_select(ctx->st, ctx->cfg.max_ctx, ctx->seq_kv, ctx->trk, ctx->B, R, ctx->stream));
         mark(ctx, DLLM_K_COMMIT);
     }
-    int rc = forward(ctx, ctx->B, T, true, R);
+    int rc = forward(ctx, ctx->B, T, true, R, ctx->sched.sls && !(ctx->debug & 1));
     if (rc) {
         ctx->in_step = false;
         return rc;
@@ -543,6 +574,11 @@ int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void*
     ctx->trk = reinterpret_cast<int*>(A + L.off_trk);
     ctx->scr_merge = reinterpret_cast<int*>(A + L.off_smerge);
     ctx->scr_side = reinterpret_cast<__nv_bfloat16*>(A + L.off_side);
+    ctx->sls_x = reinterpret_cast<__nv_bfloat16*>(A + L.off_xc);
+    ctx->sls_sq = reinterpret_cast<float*>(A + L.off_sqc);
+    ctx->sls_cur = reinterpret_cast<int*>(A + L.off_curc);
+    ctx->sls_map = reinterpret_cast<int*>(A + L.off_rmap);
+    ctx->sls_n = reinterpret_cast<int*>(A + L.off_nrows);
     cudaStream_t s = ctx->stream;
     // zero everything that is read before it is written (counters, state, status)
     if (cudaMemsetAsync(A + L.off_sq, 0, L.total - L.off_sq, s) != cudaSuccess ||
@@ -611,7 +647,8 @@ static int start_request(dllm_ctx* ctx, const dllm_sched* sched, int batch, int 
     if (sched->steps_per_block < 1 || sched->remask_max < 0 || sched->spec_blocks < 0 ||
         (sched->commit_mode != DLLM_COMMIT_SCHEDULE && sched->commit_mode != DLLM_COMMIT_THRESHOLD) ||
         !(sched->theta_visible == sched->theta_visible) || sched->scr_rows < 0 ||
-        sched->scr_rows > DLLM_MAX_SCR_ROWS || sched->spec_lat_n < 0 || sched->spec_lat_n > 8)
+        sched->scr_rows > DLLM_MAX_SCR_ROWS || sched->spec_lat_n < 0 || sched->spec_lat_n > 8 ||
+        (sched->sls != 0 && sched->sls != 1))
         return fail(ctx, DLLM_EINVAL, "bad schedule");
     if (sched->scr_rows > 0 && !sched->use_prefix_cache)
         return fail(ctx, DLLM_EINVAL, "sparse cache refresh needs the prefix cache");
@@ -624,6 +661,11 @@ static int start_request(dllm_ctx* ctx, const dllm_sched* sched, int batch, int 
     if (maxT > c.max_window) return fail(ctx, DLLM_ECAPACITY, "window of %d tokens > max_window %d", maxT, c.max_window);
     if (!sched->use_prefix_cache && gen_len > kMaxBlock) return fail(ctx, DLLM_ECAPACITY, "block too long");
     ctx->sched = *sched;
+    if (ctx->gexec) {  // the captured step bakes in the schedule's thresholds and counts
+        cudaGraphExecDestroy(ctx->gexec);
+        ctx->gexec = nullptr;
+        ctx->g_T = -1;
+    }
     ctx->B = batch;
     ctx->Lp = Lp;
     ctx->gen_len = gen_len;
@@ -785,7 +827,7 @@ int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out) {
     if (use_graph) {
         // trace pointers and the refresh rows are baked in too
         const int key_dbg = ctx->debug | (ctx->profiling ? 256 : 0) |
-                            ((s.use_prefix_cache ? s.scr_rows : 0) << 10);
+                            ((s.use_prefix_cache ? s.scr_rows : 0) << 10) | (s.sls << 16);
         if (!ctx->gexec || ctx->g_T != T || ctx->g_B != ctx->B || ctx->g_kv != ctx->kv_len || ctx->g_dbg != key_dbg) {
             if (ctx->gexec) {
                 cudaGraphExecDestroy(ctx->gexec);

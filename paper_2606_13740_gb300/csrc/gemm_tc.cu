@@ -82,7 +82,23 @@ struct EpiSmem {
                    // own memory: the next chunk's partial slices arrive meanwhile)
     uint8_t* stg2; // staging of a chunk's fp32 residual (second pass), 16 KB: the partial staging memory
     float* xs;    // [2][32][128] the old fp32 residual of a wide tile's chunks (nullptr: none), see xs_offset
+    const int* rows;  // the launch's device-resolved row count (-1: the plans as given)
 };
+
+// The plan of a phase in a launch whose rows are resolved on the device (rows >= 0): only the
+// token tiles that hold rows [0, rows), their iterations split anew over the CTAs (a phase with
+// no rows gets grid 0: every role skips it).
+__device__ __forceinline__ GemmPlan phase_plan(const ChainPhase& P, int rows) {
+    GemmPlan p = P.p;
+    if (rows >= 0) {
+        const int nt = min(p.n_tiles, (rows + p.ntile - 1) / p.ntile);
+        p.n_tiles = nt;
+        p.total = static_cast<long long>(p.m_tiles) * nt * p.kb;
+        const long long min_iters = (p.kb + 29) / 30;  // at most 31 parts per tile, as on the host
+        if (p.grid > p.total / min_iters) p.grid = static_cast<int>(p.total / min_iters);
+    }
+    return p;
+}
 
 // Word offset of (token j, tile row f) in a 32-token chunk of staged residual: [token][128 rows],
 // the 16-byte pieces of a token's row rotated so that neither the copies (thread = token, 8
@@ -513,7 +529,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                                                   volatile int* s_abort, uint32_t tmem_base, const EpiSmem& esm,
                                                   ChainEpiState& es) {
     const ChainPhase& P = ca.ph[ph];
-    const GemmPlan& p = P.p;
+    const GemmPlan p = phase_plan(P, *esm.rows);
     const EpiArgs& ep = P.ep;
     int* status = ca.status;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -856,6 +872,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     uint64_t* redbar = drain + 1;  // two partial staging slots
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(redbar + 2);
     volatile int* s_abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    int* s_rows = reinterpret_cast<int*>(tmem_slot + 2);
+    esm.rows = s_rows;
     int* status = ca.status;
 
     const int warp = threadIdx.x >> 5;
@@ -874,6 +892,12 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         mbar_init(&redbar[0], 1);
         mbar_init(&redbar[1], 1);
         *s_abort = 0;
+        int rows = -1;
+        if (ca.dyn_rows) {
+            pdl_wait();  // the count is written by the preceding launch
+            rows = max(*ca.dyn_rows, 0);
+        }
+        *s_rows = rows;
         mbar_fence_init();
     }
     if (warp == 0 && lane == 0) {
@@ -892,6 +916,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
     const int acc_cols = ca.acc_cols;
+    const int rows = *s_rows;
 
     if (warp == 0) {
         // ---------------------------------------------------------- weight producer
@@ -901,7 +926,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             uint32_t par = 0;
             uint32_t pending = 0, pend_par = 0;
             for (int ph = 0; ph < ca.n_phases && !*s_abort; ++ph) {
-                const GemmPlan& p = ca.ph[ph].p;
+                const GemmPlan p = phase_plan(ca.ph[ph], rows);
                 if (static_cast<int>(blockIdx.x) >= p.grid) continue;
                 const int it0 = static_cast<int>(range_begin(blockIdx.x, p.total, p.grid));
                 const int it1 = static_cast<int>(range_begin(blockIdx.x + 1, p.total, p.grid));
@@ -961,7 +986,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         bool stop = false;
         for (int ph = 0; ph < ca.n_phases && !stop; ++ph) {
             const ChainPhase& P = ca.ph[ph];
-            const GemmPlan& p = P.p;
+            const GemmPlan p = phase_plan(P, rows);
             if (static_cast<int>(blockIdx.x) >= p.grid) continue;
             const int it0 = static_cast<int>(range_begin(blockIdx.x, p.total, p.grid));
             const int it1 = static_cast<int>(range_begin(blockIdx.x + 1, p.total, p.grid));
@@ -1042,7 +1067,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             uint32_t acc_phase = 0;
             bool issued = false;
             for (int ph = 0; ph < ca.n_phases && !*s_abort; ++ph) {
-                const GemmPlan& p = ca.ph[ph].p;
+                const GemmPlan p = phase_plan(ca.ph[ph], rows);
                 if (static_cast<int>(blockIdx.x) >= p.grid) continue;
                 const long long it0 = range_begin(blockIdx.x, p.total, p.grid);
                 const long long it1 = range_begin(blockIdx.x + 1, p.total, p.grid);
@@ -1271,6 +1296,8 @@ cudaError_t chain_launch(const ChainMaps& maps, const ChainArgs& ca, cudaStream_
         if (p.grid > ca.grid || !ca.ph[i].partials || !ca.ph[i].tickets || (i > 0 && ca.ph[i].dep_rows < 0))
             return cudaErrorInvalidValue;
     }
+    // a device-resolved row count changes a phase's tiling: no later phase may wait on its flags
+    if (ca.dyn_rows && ca.n_phases != 1) return cudaErrorInvalidValue;
     return launch_k(k_chain, dim3(ca.grid), dim3(kChainThreads), ca.smem, st, pdl, maps, ca);
 }
 

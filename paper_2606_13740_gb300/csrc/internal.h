@@ -123,6 +123,11 @@ struct ChainArgs {
     const int* epoch;    // device step counter; tag = *epoch * tag_mul + tag_add (null: tag = tag_add)
     int tag_mul, tag_add;
     int* status;
+    // Rows resolved on the device (null: every phase's plan as given).  With it, the launch
+    // reads the token count from here once its predecessor has finished, and every phase
+    // covers only the token tiles that hold those rows (the rest of the iteration space is
+    // re-split over the CTAs).  Used by the LM head over compacted rows.
+    const int* dyn_rows;
     ChainPhase ph[kMaxPhases];
 };
 struct ChainMaps {
@@ -220,7 +225,18 @@ cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, co
                              unsigned long long* trace = nullptr, int* status = nullptr);
 cudaError_t launch_lmhead_reduce(const float* lm_part, const float* zcur, const int* cur_tok, int m_tiles,
                                  int N, int mask_id, int* x0, float* conf, float* tokconf, cudaStream_t st,
-                                 bool pdl = true);
+                                 bool pdl = true, const int* row_map = nullptr, const int* n_rows = nullptr);
+// Selective logits skipping (Sec. 3.3): the rows of the step that need a decision are those whose
+// position is MASKED, COMMITTED or DRAFT (tracked refresh rows always); FIXED and STABLE rows
+// skip the LM head.  launch_sls_map (one CTA) lists the needed rows in ascending order
+// (row_map[0..*n_rows)) and gives every skipped row the decision x0 = -1, conf = tokconf = 0;
+// launch_sls_gather copies the listed rows' bf16 activations, RMSNorm statistics and current
+// ids into compact buffers and zero-fills the rest of the last token tile (pad_to rows).
+cudaError_t launch_sls_map(const uint8_t* st, int ld, const int* seq_kv, int use_cache, int B, int Tw, int T,
+                           int* row_map, int* n_rows, int* x0, float* conf, float* tokconf, cudaStream_t stream);
+cudaError_t launch_sls_gather(const int* row_map, const int* n_rows, int N, int pad_to, int d,
+                              const __nv_bfloat16* xn, const float* sq, int n_sq, const int* cur,
+                              __nv_bfloat16* xc, float* sqc, int* curc, cudaStream_t stream);
 
 // Commit pass.  Per sequence b: state arrays at tok + b*ld, st + b*ld; the
 // window starts at seq_kv[b] (prefix cache on) or 0 (off); plan[b] holds

@@ -546,12 +546,15 @@ __device__ __forceinline__ void lse_merge(float& m, float& s, int& i, float m2, 
 
 __global__ void __launch_bounds__(256) k_lmhead_reduce(const float* __restrict__ part, const float* __restrict__ zcur,
                                                         const int* __restrict__ cur_tok, int m_tiles, int mask_id,
-                                                        int* x0, float* conf, float* tokconf) {
+                                                        int* x0, float* conf, float* tokconf, const int* row_map,
+                                                        const int* n_rows) {
     pdl_wait();
     pdl_launch_dependents();
     __shared__ float sm_m[8], sm_s[8];
     __shared__ int sm_i[8];
-    const int col = blockIdx.x;
+    const int col = blockIdx.x;  // the head's token column (a compacted row with a row map)
+    if (row_map && col >= *n_rows) return;
+    const int out = row_map ? row_map[col] : col;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     float m = -INFINITY, s = 0.0f;
     int idx = INT_MAX;
@@ -576,17 +579,112 @@ __global__ void __launch_bounds__(256) k_lmhead_reduce(const float* __restrict__
         s = sm_s[0];
         idx = sm_i[0];
         for (int w = 1; w < static_cast<int>(blockDim.x >> 5); ++w) lse_merge(m, s, idx, sm_m[w], sm_s[w], sm_i[w]);
-        x0[col] = idx;
-        conf[col] = 1.0f / s;
+        x0[out] = idx;
+        conf[out] = 1.0f / s;
         const int cur = cur_tok[col];
-        tokconf[col] = (cur >= 0 && cur != mask_id) ? expf(zcur[col] - m) / s : 0.0f;
+        tokconf[out] = (cur >= 0 && cur != mask_id) ? expf(zcur[col] - m) / s : 0.0f;
     }
 }
 
 cudaError_t launch_lmhead_reduce(const float* lm_part, const float* zcur, const int* cur_tok, int m_tiles, int N,
-                                 int mask_id, int* x0, float* conf, float* tokconf, cudaStream_t st, bool pdl) {
+                                 int mask_id, int* x0, float* conf, float* tokconf, cudaStream_t st, bool pdl,
+                                 const int* row_map, const int* n_rows) {
     return launch_k(k_lmhead_reduce, dim3(N), dim3(256), 0, st, pdl, lm_part, zcur, cur_tok, m_tiles, mask_id, x0, conf,
-                    tokconf);
+                    tokconf, row_map, n_rows);
+}
+
+// ------------------------------------------------------------------ selective logits skipping
+// One CTA lists the rows (b T + t) that need a decision, in ascending order: window row t < Tw
+// is needed when its position's state is MASKED (1), COMMITTED (2) or DRAFT (4); rows t >= Tw
+// (tracked refresh rows) always.  Skipped rows get x0 = -1, conf = tokconf = 0.
+__global__ void __launch_bounds__(1024) k_sls_map(const uint8_t* st, int ld, const int* seq_kv, int use_cache, int B,
+                                                  int Tw, int T, int* row_map, int* n_rows, int* x0, float* conf,
+                                                  float* tokconf) {
+    pdl_wait();
+    pdl_launch_dependents();
+    __shared__ int s_warp[32];
+    __shared__ int s_base;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    if (threadIdx.x == 0) s_base = 0;
+    __syncthreads();
+    const int N = B * T;
+    for (int base = 0; base < N; base += blockDim.x) {
+        const int row = base + static_cast<int>(threadIdx.x);
+        bool need = false;
+        if (row < N) {
+            const int b = row / T, t = row - b * T;
+            if (t >= Tw) {
+                need = true;
+            } else {
+                const int w0 = use_cache ? seq_kv[b] : 0;
+                const uint8_t s = st[static_cast<size_t>(b) * ld + w0 + t];
+                need = s == 1 || s == 2 || s == 4;
+            }
+        }
+        const uint32_t bal = __ballot_sync(0xffffffffu, need);
+        if (lane == 0) s_warp[warp] = __popc(bal);
+        __syncthreads();
+        int before = s_base, tot = 0;
+        for (int w = 0; w < nw; ++w) {
+            const int c = s_warp[w];
+            if (w < warp) before += c;
+            tot += c;
+        }
+        before += __popc(bal & ((1u << lane) - 1u));
+        if (need) {
+            row_map[before] = row;
+        } else if (row < N) {
+            x0[row] = -1;
+            conf[row] = 0.0f;
+            tokconf[row] = 0.0f;
+        }
+        __syncthreads();  // every thread has read s_base and s_warp
+        if (threadIdx.x == 0) s_base += tot;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) *n_rows = s_base;
+}
+
+cudaError_t launch_sls_map(const uint8_t* st, int ld, const int* seq_kv, int use_cache, int B, int Tw, int T,
+                           int* row_map, int* n_rows, int* x0, float* conf, float* tokconf, cudaStream_t stream) {
+    return launch_k(k_sls_map, dim3(1), dim3(1024), 0, stream, true, st, ld, seq_kv, use_cache, B, Tw, T, row_map,
+                    n_rows, x0, conf, tokconf);
+}
+
+// One warp per compact row j < pad_to: rows j < n copy activation row row_map[j] (d bf16, 16-byte
+// pieces), its n_sq RMSNorm statistics (stride N) and current id; rows n <= j < pad_to become
+// zero activations with unit statistics and id -1 (finite, and never reduced).
+__global__ void __launch_bounds__(256) k_sls_gather(const int* row_map, const int* n_rows, int N, int pad_to, int d,
+                                                    const __nv_bfloat16* xn, const float* sq, int n_sq,
+                                                    const int* cur, __nv_bfloat16* xc, float* sqc, int* curc) {
+    pdl_wait();
+    pdl_launch_dependents();
+    const int lane = threadIdx.x & 31;
+    const int j = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    const int n = *n_rows;
+    const int pad_end = (n + pad_to - 1) / pad_to * pad_to;  // the end of the last token tile in use
+    if (j >= pad_end || j >= N) return;
+    const int n16 = d / 8;
+    uint4* dst = reinterpret_cast<uint4*>(xc + static_cast<size_t>(j) * d);
+    if (j < n) {
+        const int row = row_map[j];
+        const uint4* src = reinterpret_cast<const uint4*>(xn + static_cast<size_t>(row) * d);
+        for (int i = lane; i < n16; i += 32) dst[i] = src[i];
+        for (int t = lane; t < n_sq; t += 32) sqc[static_cast<size_t>(t) * N + j] = sq[static_cast<size_t>(t) * N + row];
+        if (lane == 0) curc[j] = cur[row];
+    } else {
+        for (int i = lane; i < n16; i += 32) dst[i] = make_uint4(0u, 0u, 0u, 0u);
+        for (int t = lane; t < n_sq; t += 32) sqc[static_cast<size_t>(t) * N + j] = 1.0f;
+        if (lane == 0) curc[j] = -1;
+    }
+}
+
+cudaError_t launch_sls_gather(const int* row_map, const int* n_rows, int N, int pad_to, int d,
+                              const __nv_bfloat16* xn, const float* sq, int n_sq, const int* cur,
+                              __nv_bfloat16* xc, float* sqc, int* curc, cudaStream_t stream) {
+    if (N < 1 || pad_to < 1 || d % 8) return cudaErrorInvalidValue;
+    return launch_k(k_sls_gather, dim3((N + 7) / 8), dim3(256), 0, stream, true, row_map, n_rows, N, pad_to, d, xn,
+                    sq, n_sq, cur, xc, sqc, curc);
 }
 
 // ------------------------------------------------------------------ commit pass

@@ -36,6 +36,8 @@ def main(argv=None):
     ap.add_argument("--lat", type=float, nargs="*", default=[3.37, 3.97, 4.14],
                     help="generate: step ms with a window of 1, 2, 3 blocks (the window sweep at batch 1)")
     ap.add_argument("--allowance", type=float, default=0.2, help="generate: adaptive lookahead allowance")
+    ap.add_argument("--sls", type=int, default=0, help="step-b16: selective logits skipping (0/1)")
+    ap.add_argument("--stable", action="store_true", help="step-b16: the window's visible positions are STABLE")
     a = ap.parse_args(argv)
     lib()
     dev = torch.device("cuda:0")
@@ -141,29 +143,31 @@ def _timed_steps(ctx, step, n, warm=3):
 
 def step_b16(a):
     """Batch-16 denoising step: synthetic prefix KV of 4096 positions per sequence, a 64-token
-    window (current block + one speculative block) with 32 masked, Zipf(1.1) ids.  Prints
-    ms/step and the projections' achieved bf16 TFLOP/s (events around each launch)."""
+    window (current block + one speculative block) with 32 masked, Zipf(1.1) ids; the other 32
+    visible (COMMITTED, or STABLE with --stable).  Prints ms/step and the projections' achieved
+    bf16 TFLOP/s (events around each launch; the LM head counted over the rows it decides)."""
     import numpy as np
 
     import dllm_inputs as I
 
-    from .dllm import COMMITTED, MASKED, Config, Context, Sched
+    from .dllm import COMMITTED, MASKED, STABLE, Config, Context, Sched
 
     B, P, T, L = 16, 4096, 64, a.layers
     cfg = Config(max_batch=B, max_ctx=P + T, max_window=T, n_layers=L, **SHAPE_8B)
     ctx = Context(cfg)
-    sched = Sched(steps_per_block=32, spec_trigger=32, spec_blocks=1)
+    sched = Sched(steps_per_block=32, spec_trigger=32, spec_blocks=1, sls=a.sls)
     ctx.dllm_set_prefix_kv_random(sched, B, P, T, I.SEED_KV)
     ctx.dllm_begin_block()
     tok, st, _ = ctx.dllm_get_state()
     win = np.arange(P, P + T)
     tok[:, win] = I.zipf_ids((B, T), cfg.vocab, cfg.mask_id)
-    st[:, win] = COMMITTED
+    st[:, win] = STABLE if a.stable else COMMITTED
     for b in range(B):
         m = win[I.masked_positions(T, 32, seed=I.SEED_PROMPT + 100 + b)]
         tok[b, m], st[b, m] = cfg.mask_id, MASKED
     ctx.dllm_set_state(tok, st)
     w = ctx.dllm_window()
+    head_rows = B * T if not (a.sls and a.stable) else int((st[:, win] != STABLE).sum())
 
     def step():
         ctx.dllm_rewind_block()
@@ -178,11 +182,12 @@ def step_b16(a):
     N = B * T
     d, F, V = cfg.d_model, cfg.ffn, cfg.vocab
     layer_flops = 2 * N * (4 * d * d + 3 * d * F)
-    head_flops = 2 * N * V * d
+    head_flops = 2 * head_rows * V * d
     attn_flops = B * L * 4 * T * (P + T) * d
-    chain_ms = (prof["qkv"]["ms_total"] + prof["layer"]["ms_total"]) / psteps
+    chain_ms = (prof["qkv"]["ms_total"] + prof["layer"]["ms_total"] + prof["head"]["ms_total"]) / psteps
     gemm_flops = L * layer_flops + head_flops
-    print(json.dumps({"op": "step-b16", "window": w, "ms_per_step": ms, "steps_per_s": 1e3 / ms,
+    print(json.dumps({"op": "step-b16", "sls": a.sls, "stable": a.stable, "head_rows": head_rows,
+                      "window": w, "ms_per_step": ms, "steps_per_s": 1e3 / ms,
                       "kernel_ms_per_step": {k: v["ms_total"] / psteps for k, v in prof.items()},
                       "gemm_tflops": gemm_flops / (chain_ms * 1e-3) / 1e12,
                       "attn_kv_GBps": B * L * 2 * (P + T) * d * 2 / (prof["attn"]["ms_total"] / psteps * 1e-3) / 1e9,

@@ -338,3 +338,113 @@ def test_errors_poison_context(model):
     with pytest.raises(DllmError):  # block unfinished
         ctx.dllm_begin_block()
     ctx.close()
+
+
+def test_selective_logits_skipping_teacher_forced(model):
+    """Selective logits skipping (Sec. 3.3) against the oracle, which decides every row: each
+    step, the rows whose position is MASKED, COMMITTED or DRAFT carry the oracle's decisions,
+    STABLE rows carry none (x0 -1, conf and tokconf 0), and the commit bookkeeping is that of
+    the oracle.  Revision and one lookahead block run; between steps, teacher forcing makes
+    every other visible position STABLE in both (the thresholds stay out of the tiny model's
+    confidence range, so no decision sits on one of them)."""
+    from paper_2606_13740_gb300 import Sched
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=43)
+    kw = dict(steps_per_block=8, theta_remask=0.5, remask_max=1, spec_blocks=1, spec_trigger=16)
+    sess = O.Session(model, O.OracleSched(**kw), prompt, 96)
+    sess.prefill()
+    ctx = _gpu_ctx()
+    ctx.dllm_prefill(Sched(sls=1, **kw), prompt, 96)
+    skipped, needed, states = 0, 0, set()
+    while True:
+        more = sess.begin_block()
+        assert more == ctx.dllm_begin_block()
+        if not more:
+            break
+        while True:
+            o_tok0, o_st0, _ = sess.state()
+            g_tok0, g_st0, _ = ctx.dllm_get_state()
+            assert np.array_equal(g_tok0[0], o_tok0) and np.array_equal(g_st0[0], o_st0)
+            oo = sess.step()
+            go = ctx.dllm_denoise_step()
+            ow, gw = sess.window(), ctx.dllm_window()
+            for key in ("w0", "T", "c0", "c1", "kv_len", "spec_on", "step"):
+                assert ow[key] == gw[key], (key, ow, gw)
+            od = sess.decisions()
+            gd = ctx.dllm_get_step_debug()
+            w0, T = ow["w0"], ow["T"]
+            win = o_st0[w0:w0 + T]
+            states.update(int(s) for s in win)
+            need = np.isin(win, (O.MASKED, O.COMMITTED, O.DRAFT))
+            gx, gc, gt = gd["x0"][0], gd["conf"][0], gd["tokconf"][0]
+            assert (gx[~need] == -1).all() and (gc[~need] == 0).all() and (gt[~need] == 0).all()
+            safe = need & (od["margin"] > 0.05)
+            assert np.array_equal(gx[safe], od["x0"][safe])
+            assert np.allclose(gc[need], od["conf"][need], rtol=0.05)
+            assert np.allclose(gt[need], od["tokconf"][need], rtol=0.05, atol=1e-7)
+            for key in ("n_committed", "n_remasked", "n_stable", "n_drafts", "block_done", "masked_after"):
+                assert go[key] == oo[key], (key, go, oo)
+            skipped += int((~need).sum())
+            needed += int(need.sum())
+            o_tok, o_st, _ = sess.state()
+            vis = np.flatnonzero(o_st == O.COMMITTED)
+            o_st[vis[::2]] = O.STABLE
+            sess.set_state(o_tok, o_st)
+            ctx.dllm_set_state(o_tok[None], o_st[None])  # teacher forcing
+            if oo["block_done"]:
+                break
+    assert skipped > 0 and needed > 0
+    assert {O.MASKED, O.COMMITTED, O.STABLE, O.DRAFT} <= states
+    ctx.close()
+
+
+@pytest.mark.parametrize("n_stable", [0, 24, 32])
+def test_selective_logits_skipping_batch_one_step(model, n_stable):
+    """Sixteen sequences, one step over their 32-token blocks (two 256-token head tiles without
+    skipping): sequence b has max(0, n_stable - 2 b) of its block positions STABLE and a third
+    of the rest visible.  With n_stable = 32 sequence 0 needs no row and the needed rows fit
+    one token tile; with 24 they end inside the second tile.  Every needed row's decision
+    matches the oracle's for that sequence and state; every other row carries none."""
+    from paper_2606_13740_gb300 import Sched
+    B, gen = 16, 64
+    prompts = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, batch=B, seed=90)
+    kw = dict(steps_per_block=8, theta_remask=0.5, remask_max=1)
+    ctx = _gpu_ctx(max_batch=B, max_window=64)
+    ctx.dllm_prefill(Sched(sls=1, **kw), prompts, gen)
+    assert ctx.dllm_begin_block()
+    tok, st, kv = ctx.dllm_get_state()
+    rng = np.random.default_rng(91)
+    for b in range(B):
+        w0 = int(kv[b])
+        k = max(0, n_stable - 2 * b)
+        pos = w0 + rng.permutation(32)
+        tok[b, pos[:k]] = rng.integers(0, TINY.mask_id, k)
+        st[b, pos[:k]] = O.STABLE
+        vis = pos[k:k + (32 - k) // 3]
+        tok[b, vis] = rng.integers(0, TINY.mask_id, len(vis))
+        st[b, vis] = O.COMMITTED
+    ctx.dllm_set_state(tok, st)
+    ctx.dllm_denoise_step()
+    assert ctx.dllm_window()["T"] == 32
+    gd = ctx.dllm_get_step_debug()
+    n_need = []
+    for b in range(B):
+        sess = O.Session(model, O.OracleSched(**kw), prompts[b], gen)
+        sess.prefill()
+        assert sess.begin_block()
+        sess.set_state(tok[b], st[b])
+        sess.step()
+        assert sess.window()["T"] == 32
+        od = sess.decisions()
+        win = st[b, int(kv[b]):int(kv[b]) + 32]
+        need = np.isin(win, (O.MASKED, O.COMMITTED, O.DRAFT))
+        n_need.append(int(need.sum()))
+        gx, gc = gd["x0"][b], gd["conf"][b]
+        assert (gx[~need] == -1).all() and (gc[~need] == 0).all()
+        safe = need & (od["margin"] > 0.05)
+        assert np.array_equal(gx[safe], od["x0"][safe])
+        assert np.allclose(gc[need], od["conf"][need], rtol=0.05)
+    if n_stable == 32:
+        assert n_need[0] == 0 and sum(n_need) <= 256
+    elif n_stable == 24:
+        assert 256 < sum(n_need) < 512
+    ctx.close()
