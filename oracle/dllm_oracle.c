@@ -412,9 +412,13 @@ int orc_commit(const orc_sched* s, int mask_id, int n_pos, int32_t* tok, uint8_t
     orc_step_out r;
     memset(&r, 0, sizeof(r));
     int S = s->steps_per_block;
-    if (c0 < w0 || c1 > w0 + T || c1 > n_pos || c0 > c1) return -1;
+    if (c1 > w0 + T || c1 > n_pos || c0 > c1 || w0 > c1) return -1;
+    /* block positions left of the window (continuous sliding) are settled */
+    for (int p = c0; p < w0 && p < c1; ++p)
+        if (st[p] == ORC_MASKED || st[p] == ORC_DRAFT) return -1;
     if (s->theta_remask > 0.0f && step < S - 1) {
-        for (int p = c0; p < c1; ++p)
+        int r0 = c0 > w0 ? c0 : w0; /* the revision reaches only the block positions in the window */
+        for (int p = r0; p < c1; ++p)
             if (st[p] == ORC_COMMITTED && tokconf[p - w0] >= s->theta_stable) {
                 st[p] = ORC_STABLE;
                 r.n_stable++;
@@ -422,10 +426,10 @@ int orc_commit(const orc_sched* s, int mask_id, int n_pos, int32_t* tok, uint8_t
         /* candidates ranked by (tokconf ascending, position ascending) */
         int* sel = (int*)malloc(sizeof(int) * (size_t)(c1 - c0 + 1));
         int nsel = 0;
-        for (int p = c0; p < c1; ++p) {
+        for (int p = r0; p < c1; ++p) {
             if (st[p] != ORC_COMMITTED || !(tokconf[p - w0] < s->theta_remask)) continue;
             int rank = 0;
-            for (int q = c0; q < c1; ++q) {
+            for (int q = r0; q < c1; ++q) {
                 if (q == p || st[q] != ORC_COMMITTED || !(tokconf[q - w0] < s->theta_remask)) continue;
                 float a = tokconf[q - w0], b = tokconf[p - w0];
                 if (a < b || (a == b && q < p)) rank++;
@@ -487,7 +491,7 @@ int orc_commit(const orc_sched* s, int mask_id, int n_pos, int32_t* tok, uint8_t
         free(committed);
     }
     r.n_committed = nc;
-    if (s->use_prefix_cache && s->spec_blocks > 0) {
+    if (s->use_prefix_cache && (s->spec_blocks > 0 || s->slide)) { /* future blocks in the window */
         int w1 = w0 + T;
         for (int b0 = c1; b0 < w1; b0 += s->block_len) {
             int b1 = b0 + s->block_len < w1 ? b0 + s->block_len : w1;
@@ -620,7 +624,7 @@ int orc_begin_block(orc_session* x) {
         for (int p = x->c0; p < x->c1; ++p)
             if (x->st[p] == ORC_MASKED) return -3; /* block not finished */
         if (x->s.use_prefix_cache) {
-            int rc = append_kv(x, x->c0, x->c1);
+            int rc = append_kv(x, x->kv_len, x->c1); /* what has not slid into the cache yet */
             if (rc) return rc;
         }
     }
@@ -647,12 +651,16 @@ int orc_denoise_step(orc_session* x, orc_step_out* out, int keep_logits) {
     int w0, w1, spec = 0;
     if (x->s.use_prefix_cache) {
         w0 = x->kv_len;
-        w1 = x->c1;
-        if (x->s.spec_blocks > 0 && masked <= x->s.spec_trigger && x->c1 < x->n_pos) {
+        /* the window without lookahead: the current block, or with sliding one block's length
+         * from the frontier */
+        int base = x->s.slide ? w0 + x->s.block_len : x->c1;
+        if (base > x->n_pos) base = x->n_pos;
+        w1 = base;
+        if (x->s.spec_blocks > 0 && masked <= x->s.spec_trigger && base < x->n_pos) {
             int k = x->s.spec_blocks;
             if (x->s.spec_allowance >= 0.0f && x->s.spec_lat_n > 0) {
                 /* greedy: one more future block while the step stays within the allowance */
-                int i0 = (x->c1 - w0 + x->s.block_len - 1) / x->s.block_len - 1;
+                int i0 = (base - w0 + x->s.block_len - 1) / x->s.block_len - 1;
                 k = 0;
                 for (int j = 1; j <= x->s.spec_blocks; ++j) {
                     int i = i0 + j;
@@ -663,7 +671,7 @@ int orc_denoise_step(orc_session* x, orc_step_out* out, int keep_logits) {
             }
             if (k > 0) {
                 spec = 1;
-                w1 = x->c1 + k * x->s.block_len;
+                w1 = base + k * x->s.block_len;
                 if (w1 > x->n_pos) w1 = x->n_pos;
             }
         }
@@ -703,8 +711,9 @@ int orc_denoise_step(orc_session* x, orc_step_out* out, int keep_logits) {
     }
     free(x->logits);
     x->logits = (float*)malloc(sizeof(float) * (size_t)Tq * V);
-    float* nk = nt ? (float*)malloc(sizeof(float) * (size_t)L * Tq * qd) : NULL;
-    float* nv = nt ? (float*)malloc(sizeof(float) * (size_t)L * Tq * qd) : NULL;
+    int keep_kv = nt > 0 || x->s.slide;
+    float* nk = keep_kv ? (float*)malloc(sizeof(float) * (size_t)L * Tq * qd) : NULL;
+    float* nv = keep_kv ? (float*)malloc(sizeof(float) * (size_t)L * Tq * qd) : NULL;
     int rc = orc_forward_ex(x->m, Tq, T, rows, pos, P, pk, pv, NULL, nk, nv, x->logits, -1);
     free(pos); free(rows); free(pk); free(pv);
     if (rc) { free(nk); free(nv); return rc; }
@@ -715,6 +724,10 @@ int orc_denoise_step(orc_session* x, orc_step_out* out, int keep_logits) {
         orc_decide(V, c->mask_id, x->logits + (size_t)(T + r) * V, x->tok[x->scr_pos[r]], x->scr_x0 + r,
                    x->scr_conf + r, x->scr_tokconf + r, x->scr_margin + r);
     if (!keep_logits) { free(x->logits); x->logits = NULL; }
+    /* continuous sliding: the block positions visible when the forward ran */
+    int nb_win = x->c1 - w0 > 0 ? x->c1 - w0 : 0;
+    uint8_t* vis0 = (uint8_t*)malloc((size_t)nb_win + 1);
+    for (int t = 0; t < nb_win; ++t) vis0[t] = x->st[w0 + t] == ORC_COMMITTED || x->st[w0 + t] == ORC_STABLE;
     orc_step_out so;
     rc = orc_commit(&x->s, c->mask_id, x->n_pos, x->tok, x->st, w0, T, x->c0, x->c1, x->step, x->x0, x->conf,
                     x->tokconf, &so);
@@ -736,6 +749,21 @@ int orc_denoise_step(orc_session* x, orc_step_out* out, int keep_logits) {
         }
         so.n_refreshed++;
     }
+    /* continuous sliding: the leading run of positions visible before and after the commit pass
+     * takes the K/V this forward computed (from those same ids) into the cache */
+    if (x->s.slide && !rc) {
+        int adv = 0;
+        while (adv < nb_win && vis0[adv] &&
+               (x->st[w0 + adv] == ORC_COMMITTED || x->st[w0 + adv] == ORC_STABLE))
+            adv++;
+        for (int l = 0; l < L; ++l)
+            for (int t = 0; t < adv; ++t) {
+                memcpy(x->pk + ((size_t)l * x->n_pos + w0 + t) * qd, nk + ((size_t)l * Tq + t) * qd, sizeof(float) * qd);
+                memcpy(x->pv + ((size_t)l * x->n_pos + w0 + t) * qd, nv + ((size_t)l * Tq + t) * qd, sizeof(float) * qd);
+            }
+        x->kv_len += adv;
+    }
+    free(vis0);
     free(nk); free(nv);
     if (out) *out = so;
     x->step++;

@@ -56,6 +56,13 @@ typedef struct {
     float spec_allowance;
     int spec_lat_n;
     float spec_lat[8];
+    /* Continuous sliding (Sec. 3.2, with the prefix cache): the window keeps the size of a block
+     * (plus lookahead blocks) and starts at the cache frontier kv_len.  After the commit pass the
+     * longest leading run of window positions that were visible (COMMITTED or STABLE) when the
+     * forward ran and still are joins the prefix cache with the K/V that forward computed for
+     * them, so the window slides right into the next block, whose positions it drafts like
+     * lookahead blocks.  Positions that left the window are no longer revised. */
+    int slide;
 } orc_sched;
 
 /* Commit rules.  SCHEDULE: LLaDA's fixed schedule, ceil(m / (S - step)) of the m masked

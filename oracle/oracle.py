@@ -48,7 +48,7 @@ class _Sched(C.Structure):
                 ("theta_stable", C.c_float), ("remask_max", C.c_int), ("spec_trigger", C.c_int),
                 ("spec_blocks", C.c_int), ("use_prefix_cache", C.c_int), ("commit_mode", C.c_int),
                 ("theta_visible", C.c_float), ("scr_rows", C.c_int), ("spec_allowance", C.c_float),
-                ("spec_lat_n", C.c_int), ("spec_lat", C.c_float * 8)]
+                ("spec_lat_n", C.c_int), ("spec_lat", C.c_float * 8), ("slide", C.c_int)]
 
 
 class _StepOut(C.Structure):
@@ -151,13 +151,14 @@ class OracleSched:
     scr_rows: int = 0             # sparse cache refresh: visible prefix positions re-scored per step
     spec_allowance: float = -1.0  # adaptive lookahead allowance (< 0: fixed, all spec_blocks)
     spec_lat: tuple = ()          # step latency with a window of 1, 2, ... blocks (at most 8)
+    slide: int = 0                # continuous sliding of the window along the commit frontier
 
     def c(self):
         lat = (C.c_float * 8)(*self.spec_lat[:8])
         return _Sched(self.steps_per_block, self.block_len, self.theta_remask, self.theta_stable,
                       self.remask_max, self.spec_trigger, self.spec_blocks, self.use_prefix_cache,
                       self.commit_mode, self.theta_visible, self.scr_rows, self.spec_allowance,
-                      len(self.spec_lat[:8]), lat)
+                      len(self.spec_lat[:8]), lat, self.slide)
 
 
 def gen_f32(seed, tensor_id, first, n, sigma):

@@ -449,3 +449,74 @@ def test_adaptive_lookahead_reduces_to_fixed_and_to_none(tiny_model):
     prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=71)
     plain = O.Session(tiny_model, O.OracleSched(steps_per_block=8), prompt, 160).generate()
     assert np.array_equal(none_tok[32:], plain)
+
+
+def test_continuous_sliding_frontier_and_cache(tiny_model):
+    """Continuous sliding (Sec. 3.2): a window of one block's length starting at the cache
+    frontier; after a step, the leading run of positions that were visible at the forward and
+    still are joins the cache with exactly the K/V that forward computed (all layers; at layer
+    0 also those of the id alone at its position); the window then reaches into the next block
+    and drafts there; positions left of the window are never revised; the block end appends
+    only what has not slid."""
+    Lp, bl = 32, 32
+    prompt = I.uniform_prompt(Lp, TINY.vocab, TINY.mask_id, seed=61)
+    sched = O.OracleSched(steps_per_block=8, slide=1)
+    sess = O.Session(tiny_model, sched, prompt, 2 * bl)
+    sess.prefill()
+    assert sess.begin_block()
+    sess.step()
+    assert sess.window()["kv_len"] == Lp  # nothing was visible at the forward
+    tok, st, kv = sess.state()
+    assert kv == Lp
+    # teacher forcing: the first 5 block positions visible (and the 6th masked)
+    tok[Lp:Lp + bl] = TINY.mask_id
+    st[Lp:Lp + bl] = O.MASKED
+    tok[Lp:Lp + 5] = [3, 14, 15, 92, 65]
+    st[Lp:Lp + 5] = O.COMMITTED
+    sess.set_state(tok, st)
+    L = TINY.n_layers
+    pk = np.stack([sess.prefix_kv(l, 0) for l in range(L)])
+    pv = np.stack([sess.prefix_kv(l, 1) for l in range(L)])
+    win_tok, win_pos = tok[Lp:Lp + bl].copy(), np.arange(Lp, Lp + bl, dtype=np.int32)
+    ref = O.forward(tiny_model, win_tok, win_pos, prefix_k=pk, prefix_v=pv, want_kv=True, logits=False)
+    out = sess.step()
+    w = sess.window()
+    assert w["w0"] == Lp and w["T"] == bl and w["kv_len"] == Lp + 5
+    for l in range(L):
+        for which, r in ((0, ref["k"]), (1, ref["v"])):
+            got = sess.prefix_kv(l, which)[Lp:Lp + 5]
+            assert np.array_equal(got, r[l][:5])
+    alone = O.forward(tiny_model, win_tok[:5], win_pos[:5], want_kv=True, logits=False, n_layers_run=1)
+    assert np.allclose(sess.prefix_kv(0, 0)[Lp:Lp + 5], alone["k"][0], rtol=1e-6, atol=1e-7)
+    assert out["n_drafts"] == 0  # the window still ended at the block end
+    # the next window: one block's length from the frontier, 5 positions into the next block
+    out = sess.step()
+    w = sess.window()
+    assert w["w0"] == Lp + 5 and w["T"] == bl
+    assert out["n_drafts"] == 1
+    tok2, st2, _ = sess.state()
+    assert (st2[2 * Lp:2 * Lp + 5] == O.DRAFT).sum() == 1 and (st2[2 * Lp + 5:] != O.DRAFT).all()
+    kept = sess.prefix_kv(1, 0)[Lp:Lp + 5].copy()
+    # the commit pass with the window 5 positions into its block and every visible position a
+    # revision candidate: those left of the window are untouched, one inside is re-masked
+    n, c0, c1, w0 = 96, 32, 64, 37
+    st_c = np.full(n, O.MASKED, np.uint8)
+    st_c[c0:c0 + 8] = O.COMMITTED
+    tok_c = np.where(st_c == O.MASKED, TINY.mask_id, 5).astype(np.int32)
+    T = 32
+    tc = np.linspace(0.01, 0.3, T).astype(np.float32)
+    s_rev = O.OracleSched(steps_per_block=8, theta_remask=0.5, remask_max=32, slide=1)
+    tok_r, st_r, out_r = O.commit(s_rev, TINY.mask_id, tok_c, st_c, w0, T, c0, c1, 0,
+                                  np.arange(T, dtype=np.int32), np.full(T, 0.5, np.float32), tc)
+    assert (st_r[c0:w0] == O.COMMITTED).all() and (tok_r[c0:w0] == 5).all()
+    assert out_r["n_remasked"] == 3  # positions 37..39, the visible ones inside the window
+    # finish the block in the first session: the append covers only [kv_len, c1)
+    tok, st, kv = sess.state()
+    m = np.flatnonzero(st[Lp:Lp + bl] == O.MASKED) + Lp
+    tok[m], st[m] = 7, O.COMMITTED
+    sess.set_state(tok, st)
+    front = sess.state()[2]
+    assert sess.begin_block()
+    assert sess.state()[2] == Lp + bl
+    assert np.array_equal(sess.prefix_kv(1, 0)[Lp:Lp + 5], kept)
+    assert front >= Lp + 5
