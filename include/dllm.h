@@ -120,6 +120,13 @@ typedef struct {
      * their step decisions read x0 = -1, conf = tokconf = 0.  Ignored while the logits are
      * captured for debugging. */
     int sls;
+    /* Continuous sliding (Sec. 3.2; 0 = off, 1 = on; prefix cache on, batch 1): the window
+     * keeps one block's length (plus lookahead blocks) and starts at the cache frontier; after
+     * each step the leading run of window positions that were visible (COMMITTED or STABLE) at
+     * the forward and still are joins the prefix cache with the K/V that forward computed, so
+     * the window slides into the next block, drafting there as lookahead does.  Positions that
+     * left the window are not revised; the block end appends only what has not slid. */
+    int slide;
 } dllm_sched;
 #define DLLM_MAX_SCR_ROWS 32
 

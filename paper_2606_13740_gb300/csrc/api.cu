@@ -266,6 +266,13 @@ static int sync_check(dllm_ctx* ctx) {
 // they run through every projection and the head, attend as queries only, and their K/V go to
 // the side buffers.  With `sls` (selective logits skipping) the LM head runs as its own launch
 // over the compacted rows that need a decision; the other rows get x0 = -1, conf = tokconf = 0.
+// The cache length the step's attention is planned for: with sliding the frontier moves every
+// few steps, so the plan (and the captured step) covers it rounded up to 64 positions; the
+// kernels read each sequence's own length at run time and leave the rest of a split empty.
+static int plan_kv(const dllm_ctx* ctx) {
+    return ctx->sched.slide && ctx->sched.use_prefix_cache ? rup(ctx->kv_len, 64) : ctx->kv_len;
+}
+
 static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0, bool sls = false) {
     const int T = Tw + R;  // rows per sequence
     const dllm_config& c = ctx->cfg;
@@ -287,7 +294,7 @@ static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0, bool sls 
         !make_tmap_bf16(&tx_h, ctx->h, N, F, pd.ntile) || !make_tmap_bf16(&tx_c, ctx->sls_x, N, d, ph.ntile))
         return fail(ctx, DLLM_ECUDA, "tensor map encode failed");
     sls = sls && head;
-    AttnPlan ap = attn_plan(B, T, c.n_heads, c.head_dim, ctx->kv_len + Tw, ctx->sms);
+    AttnPlan ap = attn_plan(B, T, c.n_heads, c.head_dim, (ctx->in_step ? plan_kv(ctx) : ctx->kv_len) + Tw, ctx->sms);
     ap.qx = R;
     EpiArgs ep{};
     ep.seq_kv = ctx->seq_kv;
@@ -444,6 +451,7 @@ static int step_kernels(dllm_ctx* ctx, int T) {
     a.theta_remask = ctx->sched.theta_remask;
     a.theta_stable = ctx->sched.theta_stable;
     a.commit_mode = ctx->sched.commit_mode;
+    a.slide_kv = ctx->sched.slide && ctx->sched.use_prefix_cache ? ctx->seq_kv : nullptr;
     a.theta_visible = ctx->sched.theta_visible;
     cudaError_t ce = launch_commit(a, ctx->stream);
     mark(ctx, DLLM_K_COMMIT);
@@ -648,10 +656,12 @@ static int start_request(dllm_ctx* ctx, const dllm_sched* sched, int batch, int 
         (sched->commit_mode != DLLM_COMMIT_SCHEDULE && sched->commit_mode != DLLM_COMMIT_THRESHOLD) ||
         !(sched->theta_visible == sched->theta_visible) || sched->scr_rows < 0 ||
         sched->scr_rows > DLLM_MAX_SCR_ROWS || sched->spec_lat_n < 0 || sched->spec_lat_n > 8 ||
-        (sched->sls != 0 && sched->sls != 1))
+        (sched->sls != 0 && sched->sls != 1) || (sched->slide != 0 && sched->slide != 1))
         return fail(ctx, DLLM_EINVAL, "bad schedule");
     if (sched->scr_rows > 0 && !sched->use_prefix_cache)
         return fail(ctx, DLLM_EINVAL, "sparse cache refresh needs the prefix cache");
+    if (sched->slide && (!sched->use_prefix_cache || batch != 1))
+        return fail(ctx, DLLM_EINVAL, "continuous sliding needs the prefix cache and batch 1");
     if (sched->use_prefix_cache && c.block_len * (1 + sched->spec_blocks) + sched->scr_rows > c.max_window)
         return fail(ctx, DLLM_ECAPACITY, "window plus refresh rows > max_window %d", c.max_window);
     if (batch > c.max_batch) return fail(ctx, DLLM_ECAPACITY, "batch %d > max_batch %d", batch, c.max_batch);
@@ -748,10 +758,14 @@ int dllm_begin_block(dllm_ctx* ctx) {
         if (rc) return rc;
         if (m) return fail(ctx, DLLM_EINVAL, "current block still has %d masked positions", m);
         if (ctx->sched.use_prefix_cache) {
-            // recompute the finished block's K/V from its final ids and append them
-            rc = forward(ctx, ctx->B, ctx->c1 - ctx->c0, false);
-            if (rc) return rc;
-            ctx->kv_len += ctx->c1 - ctx->c0;
+            // recompute the finished block's K/V from its final ids and append them (with
+            // sliding: the part that has not slid into the cache yet)
+            const int rem = ctx->c1 - ctx->kv_len;
+            if (rem > 0) {
+                rc = forward(ctx, ctx->B, rem, false);
+                if (rc) return rc;
+            }
+            ctx->kv_len = ctx->c1;
             CK(launch_set_kv_len(ctx->seq_kv, ctx->B, ctx->kv_len, ctx->stream));
         }
         ctx->have_block = false;
@@ -779,6 +793,10 @@ int dllm_rewind_block(dllm_ctx* ctx) {
     if (!ctx->have_block) return fail(ctx, DLLM_EINVAL, "no current block");
     CK(launch_rewind(ctx->tok, ctx->st, ctx->stok, ctx->sst, ctx->cfg.max_ctx, ctx->n_pos, ctx->plan, ctx->B,
                      ctx->stream));
+    if (ctx->sched.slide && ctx->sched.use_prefix_cache && ctx->kv_len != ctx->c0) {  // the frontier goes back too
+        ctx->kv_len = ctx->c0;
+        CK(launch_set_kv_len(ctx->seq_kv, ctx->B, ctx->kv_len, ctx->stream));
+    }
     ctx->step = 0;
     return DLLM_OK;
 }
@@ -791,8 +809,11 @@ int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out) {
     int w0, T, spec = 0;
     if (s.use_prefix_cache) {
         w0 = ctx->kv_len;
-        int w1 = ctx->c1;
-        if (s.spec_blocks > 0 && ctx->c1 < ctx->n_pos) {
+        // the window without lookahead: the current block, or with sliding one block's length
+        // from the frontier
+        const int base = s.slide ? std::min(w0 + bl, ctx->n_pos) : ctx->c1;
+        int w1 = base;
+        if (s.spec_blocks > 0 && base < ctx->n_pos) {
             int m = 0;
             int rc = count_masked_max(ctx, ctx->c0, ctx->c1, &m);
             if (rc) return rc;
@@ -800,7 +821,7 @@ int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out) {
                 int k = s.spec_blocks;
                 if (s.spec_allowance >= 0.0f && s.spec_lat_n > 0) {
                     // greedy: one more future block while the step stays within the allowance
-                    const int i0 = (ctx->c1 - w0 + bl - 1) / bl - 1;
+                    const int i0 = (base - w0 + bl - 1) / bl - 1;
                     k = 0;
                     for (int j = 1; j <= s.spec_blocks; ++j) {
                         const int i = i0 + j;
@@ -811,7 +832,7 @@ int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out) {
                 }
                 if (k > 0) {
                     spec = 1;
-                    w1 = std::min(ctx->c1 + k * bl, ctx->n_pos);
+                    w1 = std::min(base + k * bl, ctx->n_pos);
                 }
             }
         }
@@ -828,7 +849,7 @@ int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out) {
         // trace pointers and the refresh rows are baked in too
         const int key_dbg = ctx->debug | (ctx->profiling ? 256 : 0) |
                             ((s.use_prefix_cache ? s.scr_rows : 0) << 10) | (s.sls << 16);
-        if (!ctx->gexec || ctx->g_T != T || ctx->g_B != ctx->B || ctx->g_kv != ctx->kv_len || ctx->g_dbg != key_dbg) {
+        if (!ctx->gexec || ctx->g_T != T || ctx->g_B != ctx->B || ctx->g_kv != plan_kv(ctx) || ctx->g_dbg != key_dbg) {
             if (ctx->gexec) {
                 cudaGraphExecDestroy(ctx->gexec);
                 ctx->gexec = nullptr;
@@ -849,7 +870,7 @@ int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out) {
             if (ee != cudaSuccess) return fail(ctx, DLLM_ECUDA, "graph instantiate: %s", cudaGetErrorString(ee));
             ctx->g_T = T;
             ctx->g_B = ctx->B;
-            ctx->g_kv = ctx->kv_len;
+            ctx->g_kv = plan_kv(ctx);
             ctx->g_dbg = key_dbg;
         }
         CK(cudaGraphLaunch(ctx->gexec, ctx->stream));
@@ -862,6 +883,13 @@ int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out) {
         if (rc) return rc;
     }
     ctx->step++;
+    if (s.slide && s.use_prefix_cache) {  // the frontier the commit pass moved
+        int kv = 0;
+        CK(cudaMemcpyAsync(&kv, ctx->seq_kv, 4, cudaMemcpyDeviceToHost, ctx->stream));
+        int rc = sync_check(ctx);
+        if (rc) return rc;
+        ctx->kv_len = kv;
+    }
     if (out) {
         std::vector<int> o(static_cast<size_t>(ctx->B) * 8);
         CK(cudaMemcpyAsync(o.data(), ctx->outs, o.size() * 4, cudaMemcpyDeviceToHost, ctx->stream));

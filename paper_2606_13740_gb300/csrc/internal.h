@@ -251,6 +251,7 @@ struct CommitArgs {
     const float* conf;
     const float* tokconf;
     int* outs;           // [B][8]: committed, remasked, stable, drafts, done, masked_after
+    int* slide_kv;       // continuous sliding: the per-sequence cache frontier to advance (null: off)
     int B, T, mask_id, use_cache;
     int S, remask_max, spec_blocks, block_len;
     float theta_remask, theta_stable;

@@ -716,12 +716,18 @@ __global__ void __launch_bounds__(256) k_commit(CommitArgs a) {
     const float* tc = a.tokconf + static_cast<size_t>(b) * a.Tq;
     __shared__ int s_cnt[8];
     __shared__ uint8_t s_sel[kMaxBlock];
+    __shared__ uint8_t s_vis[kMaxBlock];  // continuous sliding: block positions visible at the forward
     if (threadIdx.x < 8) s_cnt[threadIdx.x] = 0;
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+        const int p = c0 + i;
+        s_vis[i] = p >= w0 && (st[p] == 2 || st[p] == 3);
+    }
     __syncthreads();
+    // the revision reaches only the block positions inside the window (sliding moves w0 past c0)
     if (a.theta_remask > 0.0f && step < a.S - 1) {
         for (int i = threadIdx.x; i < n; i += blockDim.x) {
             const int p = c0 + i;
-            if (st[p] == 2 && tc[p - w0] >= a.theta_stable) {
+            if (p >= w0 && st[p] == 2 && tc[p - w0] >= a.theta_stable) {
                 st[p] = 3;
                 atomicAdd(&s_cnt[2], 1);
             }
@@ -731,10 +737,10 @@ __global__ void __launch_bounds__(256) k_commit(CommitArgs a) {
         for (int i = threadIdx.x; i < n; i += blockDim.x) {
             const int p = c0 + i;
             uint8_t sel = 0;
-            if (st[p] == 2 && tc[p - w0] < a.theta_remask) {
+            if (p >= w0 && st[p] == 2 && tc[p - w0] < a.theta_remask) {
                 const float vp = tc[p - w0];
                 int rank = 0;
-                for (int qq = c0; qq < c1; ++qq) {
+                for (int qq = max(c0, w0); qq < c1; ++qq) {
                     if (qq == p || st[qq] != 2) continue;
                     const float vq = tc[qq - w0];
                     if (!(vq < a.theta_remask)) continue;
@@ -829,7 +835,7 @@ __global__ void __launch_bounds__(256) k_commit(CommitArgs a) {
     }
     __syncthreads();
     // drafts for the future blocks inside the window
-    if (a.use_cache && a.spec_blocks > 0 && threadIdx.x < 32) {
+    if (a.use_cache && (a.spec_blocks > 0 || a.slide_kv) && threadIdx.x < 32) {
         const int w1 = w0 + a.T;
         for (int d0 = c1; d0 < w1; d0 += a.block_len) {
             const int d1 = min(d0 + a.block_len, w1);
@@ -894,6 +900,13 @@ __global__ void __launch_bounds__(256) k_commit(CommitArgs a) {
         o[6] = s_cnt[6];
         o[7] = s_cnt[7];
         plan[2] = step + 1;
+        if (a.slide_kv && w0 >= c0) {
+            // continuous sliding: the leading run of block positions visible at the forward and
+            // still visible joins the cache (its K/V were written there by this step's forward)
+            int adv = 0;
+            while (w0 + adv < c1 && s_vis[w0 + adv - c0] && (st[w0 + adv] == 2 || st[w0 + adv] == 3)) ++adv;
+            a.slide_kv[b] = w0 + adv;
+        }
     }
 }
 

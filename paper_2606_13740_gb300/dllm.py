@@ -40,7 +40,7 @@ class dllm_sched(C.Structure):
                 ("remask_max", C.c_int), ("spec_trigger", C.c_int), ("spec_blocks", C.c_int),
                 ("use_prefix_cache", C.c_int), ("commit_mode", C.c_int), ("theta_visible", C.c_float),
                 ("scr_rows", C.c_int), ("spec_allowance", C.c_float), ("spec_lat_n", C.c_int),
-                ("spec_lat", C.c_float * 8), ("sls", C.c_int)]
+                ("spec_lat", C.c_float * 8), ("sls", C.c_int), ("slide", C.c_int)]
 
 
 class dllm_step_out(C.Structure):
@@ -164,13 +164,14 @@ class Sched:
     spec_allowance: float = -1.0  # adaptive lookahead allowance (< 0: fixed, all spec_blocks)
     spec_lat: tuple = ()          # step latency with a window of 1, 2, ... blocks (at most 8)
     sls: int = 0                  # selective logits skipping: the LM head only for rows needing a decision
+    slide: int = 0                # continuous sliding of the window along the commit frontier (batch 1)
 
     def c(self):
         lat = (C.c_float * 8)(*self.spec_lat[:8])
         return dllm_sched(self.steps_per_block, self.theta_remask, self.theta_stable, self.remask_max,
                           self.spec_trigger, self.spec_blocks, self.use_prefix_cache, self.commit_mode,
                           self.theta_visible, self.scr_rows, self.spec_allowance, len(self.spec_lat[:8]), lat,
-                          self.sls)
+                          self.sls, self.slide)
 
 
 def dllm_arena_bytes(cfg: Config) -> int:

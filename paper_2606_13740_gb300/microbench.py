@@ -253,6 +253,9 @@ def generate(a):
             ("threshold_0_p256_g128", 256, 128,
              Sched(steps_per_block=32, commit_mode=COMMIT_THRESHOLD, theta_visible=0.0, theta_stable=0.9)),
             ("scr32_p256_g128", 256, 128, Sched(steps_per_block=32, scr_rows=32)),
+            ("slide_p256_g128", 256, 128, Sched(steps_per_block=32, slide=1)),
+            ("slide_lookahead_p1024_g256", 1024, 256,
+             Sched(steps_per_block=32, slide=1, spec_trigger=8, spec_blocks=2, theta_remask=0.5, remask_max=1)),
             ("adaptive_lookahead_p1024_g256", 1024, 256,
              Sched(steps_per_block=32, spec_trigger=8, spec_blocks=2, theta_remask=0.5, remask_max=1,
                    spec_allowance=a.allowance, spec_lat=tuple(a.lat)))):

@@ -448,3 +448,29 @@ def test_selective_logits_skipping_batch_one_step(model, n_stable):
     elif n_stable == 24:
         assert 256 < sum(n_need) < 512
     ctx.close()
+
+
+@pytest.mark.parametrize("spec", [0, 1])
+def test_continuous_sliding_teacher_forced(model, spec):
+    """Continuous sliding (Sec. 3.2) against the oracle: every step's window (start, size, cache
+    frontier), decisions and bookkeeping, the final ids, states and cache; the window does move
+    past its block start, with and without a lookahead block."""
+    from paper_2606_13740_gb300 import Sched
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=62)
+    kw = dict(steps_per_block=8, slide=1, spec_blocks=spec, spec_trigger=8)
+    ctx = _gpu_ctx()
+    moved = []
+
+    def check(sess, ctx_, oo, go, pre_o, post_o, post_g):
+        w = sess.window()
+        moved.append(w["kv_len"] > w["c0"])
+
+    sess, steps, _ = _run_teacher_forced(model, O.OracleSched(**kw), Sched(**kw), prompt, 96, ctx, check=check)
+    assert any(moved)
+    kv_len = sess.state()[2]
+    for layer in range(TINY.n_layers):
+        for which in (0, 1):
+            ref = sess.prefix_kv(layer, which)
+            got = ctx.dllm_get_kv(layer, which, 0, 0, kv_len)
+            assert np.linalg.norm(got - ref) / np.linalg.norm(ref) <= 1e-2
+    ctx.close()
