@@ -340,7 +340,8 @@ def test_errors_poison_context(model):
     ctx.close()
 
 
-def test_selective_logits_skipping_teacher_forced(model):
+@pytest.mark.parametrize("slide", [0, 1])
+def test_selective_logits_skipping_teacher_forced(model, slide):
     """Selective logits skipping (Sec. 3.3) against the oracle, which decides every row: each
     step, the rows whose position is MASKED, COMMITTED or DRAFT carry the oracle's decisions,
     STABLE rows carry none (x0 -1, conf and tokconf 0), and the commit bookkeeping is that of
@@ -349,7 +350,7 @@ def test_selective_logits_skipping_teacher_forced(model):
     confidence range, so no decision sits on one of them)."""
     from paper_2606_13740_gb300 import Sched
     prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=43)
-    kw = dict(steps_per_block=8, theta_remask=0.5, remask_max=1, spec_blocks=1, spec_trigger=16)
+    kw = dict(steps_per_block=8, theta_remask=0.5, remask_max=1, spec_blocks=1, spec_trigger=16, slide=slide)
     sess = O.Session(model, O.OracleSched(**kw), prompt, 96)
     sess.prefill()
     ctx = _gpu_ctx()
@@ -473,4 +474,29 @@ def test_continuous_sliding_teacher_forced(model, spec):
             ref = sess.prefix_kv(layer, which)
             got = ctx.dllm_get_kv(layer, which, 0, 0, kv_len)
             assert np.linalg.norm(got - ref) / np.linalg.norm(ref) <= 1e-2
+    ctx.close()
+
+
+@pytest.mark.parametrize("case", ["refresh", "threshold_fallback"])
+def test_continuous_sliding_with_other_rows(model, case):
+    """Continuous sliding combined with sparse cache refresh (slid positions are COMMITTED
+    prefix positions, so they become refresh rows) and with the threshold commit's one-position
+    fallback, teacher-forced against the oracle."""
+    from paper_2606_13740_gb300 import COMMIT_THRESHOLD, Sched
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=63)
+    if case == "refresh":
+        okw = gkw = dict(steps_per_block=8, slide=1, scr_rows=8, theta_stable=2.0)
+    else:
+        okw = dict(steps_per_block=8, slide=1, commit_mode=1, theta_visible=2.0, theta_stable=2.0)
+        gkw = dict(okw, commit_mode=COMMIT_THRESHOLD)
+    ctx = _gpu_ctx()
+    moved = []
+
+    def check(sess, ctx_, oo, go, pre_o, post_o, post_g):
+        w = sess.window()
+        moved.append(w["kv_len"] > w["c0"])
+        assert go["n_refreshed"] == oo["n_refreshed"] and go["n_revised"] == oo["n_revised"]
+
+    _run_teacher_forced(model, O.OracleSched(**okw), Sched(**gkw), prompt, 64, ctx, check=check)
+    assert any(moved)
     ctx.close()
