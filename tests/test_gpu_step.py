@@ -500,3 +500,18 @@ def test_continuous_sliding_with_other_rows(model, case):
     _run_teacher_forced(model, O.OracleSched(**okw), Sched(**gkw), prompt, 64, ctx, check=check)
     assert any(moved)
     ctx.close()
+
+
+def test_new_request_takes_its_own_schedule(model):
+    """The captured step bakes in the schedule's commit rule: a new request on the same context
+    (same window, batch and cache length) must run under its own schedule, not replay the last
+    one's step."""
+    from paper_2606_13740_gb300 import COMMIT_THRESHOLD, Sched
+    prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id, seed=64)
+    ctx = _gpu_ctx()
+    _, s1 = ctx.dllm_generate(Sched(steps_per_block=8), prompt, 64)
+    _, s2 = ctx.dllm_generate(Sched(steps_per_block=8, commit_mode=COMMIT_THRESHOLD, theta_visible=0.0), prompt, 64)
+    _, s3 = ctx.dllm_generate(Sched(steps_per_block=8), prompt, 64)
+    assert s1["steps"] == s3["steps"] == 16
+    assert s2["steps"] == 2  # a whole block per step
+    ctx.close()
