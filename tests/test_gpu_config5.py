@@ -32,31 +32,31 @@ def gpu():
     return pkg
 
 
-def _window_state(cfg, tok, st, seqs, id_seed=I.SEED_ZIPF):
+def _window_state(cfg, tok, st, seqs, id_seed=I.SEED_ZIPF, visible=O.COMMITTED):
     win = np.arange(P, P + T)
     ids = I.zipf_ids((B, T), cfg.vocab, cfg.mask_id, seed=id_seed)
     ids[0] = I.zipf_ids((B, T), cfg.vocab, cfg.mask_id)[0]  # sequence 0 keeps its ids
     for k, b in enumerate(seqs):
         tok[k, win] = ids[b]
-        st[k, win] = O.COMMITTED
+        st[k, win] = visible
         m = win[I.masked_positions(T, 32, seed=I.SEED_PROMPT + 100 + b)]
         tok[k, m], st[k, m] = cfg.mask_id, O.MASKED
     return tok, st
 
 
-def _step(gpu, seqs, id_seed=I.SEED_ZIPF):
+def _step(gpu, seqs, id_seed=I.SEED_ZIPF, visible=O.COMMITTED, sls=0):
     cfg = gpu.Config(n_layers=L, max_batch=len(seqs), max_ctx=P + T, max_window=T, **SHAPE)
     ctx = gpu.Context(cfg)
-    sched = gpu.Sched(steps_per_block=32, spec_trigger=32, spec_blocks=1)
+    sched = gpu.Sched(steps_per_block=32, spec_trigger=32, spec_blocks=1, sls=sls)
     ctx.dllm_set_prefix_kv_random(sched, len(seqs), P, T, I.SEED_KV)
     ctx.dllm_begin_block()
     tok, st, _ = ctx.dllm_get_state()
-    tok, st = _window_state(cfg, tok, st, seqs, id_seed)
+    tok, st = _window_state(cfg, tok, st, seqs, id_seed, visible)
     ctx.dllm_set_state(tok, st)
-    ctx.dllm_set_debug(1)
+    ctx.dllm_set_debug(0 if sls else 1)  # captured logits would switch the skipping off
     out = ctx.dllm_denoise_step()
     w = ctx.dllm_window()
-    d = ctx.dllm_get_step_debug(logits=True)
+    d = ctx.dllm_get_step_debug(logits=not sls)
     ctx.close()
     return tok, st, out, w, d
 
@@ -96,3 +96,26 @@ def test_batch16_sequences_independent(gpu):
     assert not np.array_equal(da["x0"][1:], db["x0"][1:])  # the others did change
     assert np.array_equal(da["logits"][0], db["logits"][0])
     assert np.array_equal(da["x0"][0], db["x0"][0]) and np.array_equal(da["conf"][0], db["conf"][0])
+
+
+def test_batch16_selective_logits_skipping_matches_oracle(gpu):
+    """The same full-width batch-16 step with the visible half of every window STABLE and
+    selective logits skipping on: the head runs over the 512 masked rows only; those rows'
+    decisions match the oracle's for the sampled sequences, the STABLE rows carry none."""
+    seqs = list(range(B))
+    tok, st, out, w, d = _step(gpu, seqs, visible=O.STABLE, sls=1)
+    model = O.Model(O.OracleConfig(n_layers=L, **SHAPE))
+    for b in (0, 13):
+        need = st[b, P:P + T] == O.MASKED
+        assert need.sum() == 32
+        assert (d["x0"][b][~need] == -1).all() and (d["conf"][b][~need] == 0).all()
+        pk = np.stack([_oracle_prefix(b, l, 0) for l in range(L)])
+        pv = np.stack([_oracle_prefix(b, l, 1) for l in range(L)])
+        ref = O.forward(model, tok[b, P:P + T], np.arange(P, P + T), prefix_k=pk, prefix_v=pv)["logits"]
+        dec = [O.decide(ref[t], SHAPE["mask_id"], int(tok[b, P + t])) for t in range(T)]
+        x0 = np.array([v[0] for v in dec])
+        conf = np.array([v[1] for v in dec])
+        safe = need & (np.array([v[3] for v in dec]) > 0.05)
+        assert safe.sum() > 0
+        assert np.array_equal(d["x0"][b][safe], x0[safe]), b
+        assert np.allclose(d["conf"][b][need], conf[need], rtol=0.05), b
