@@ -13,8 +13,12 @@
  * Conventions for every entry point:
  *   - Return 0 (DLLM_OK) or a negative DLLM_E* code (DLLM_DONE = 1 is a
  *     non-error status of dllm_begin_block).  No C++ exception crosses the ABI.
- *   - After an error the context is poisoned: later calls return
- *     DLLM_ESTATE until dllm_free.  dllm_last_error gives the message.
+ *   - Argument and capacity errors (DLLM_EINVAL, DLLM_ECAPACITY) are
+ *     detected on the host; they leave the context usable (a request whose
+ *     start failed is not started: call dllm_prefill again).  Every other error (DLLM_ENOMEM, DLLM_ECUDA,
+ *     DLLM_ETIMEOUT, DLLM_ESTATE from a failed generation) poisons the
+ *     context: later calls return DLLM_ESTATE until dllm_free.
+ *     dllm_last_error gives the message of the last error.
  *   - Host pointers belong to the caller and are only read/written during the
  *     call.  Device memory belongs to the context (or to the caller's arena,
  *     which the context never frees).
@@ -175,15 +179,22 @@ int dllm_prefill(dllm_ctx* ctx, const dllm_sched* sched, int batch, const int32_
  * state FIXED, followed by gen_len masked positions. */
 int dllm_set_prefix_kv_random(dllm_ctx* ctx, const dllm_sched* sched, int batch, int P, int gen_len, uint64_t seed);
 
-/* Advance to the next block.  If a block is current it must be finished (no
+/* Advance to the next block (Sec. 2.1 "Block-Wise Decoding": blocks are
+ * decoded left to right and a finished block's KV joins the reusable prefix;
+ * Sec. 3.2: drafts a future block already holds are re-checked once it becomes
+ * current).  If a block is current it must be finished (no
  * MASKED position, else DLLM_EINVAL); with the prefix cache on its K/V are
  * recomputed from its final ids (attending to prefix + block) and appended.
  * Drafts of the new block become COMMITTED (re-checked by the revision
  * pass).  Returns DLLM_DONE when no block is left. */
 int dllm_begin_block(dllm_ctx* ctx);
 
-/* One denoising step on the current window: forward, decisions, commit /
- * re-mask / drafts.  out (nullable, host): filled after a stream sync; with
+/* One denoising step on the current window (Sec. 2.1 "Diffusion Large
+ * Language Model": every unresolved position is predicted in parallel and a
+ * confidence-selected subset is committed; Sec. 3.2: the window may extend
+ * over future blocks, whose predictions become drafts; Sec. 3.3: committed
+ * tokens are revised until stable): forward, decisions, commit / re-mask /
+ * drafts.  out (nullable, host): filled after a stream sync; with
  * NULL the call stays asynchronous unless lookahead needs the masked count. */
 int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out);
 
@@ -192,7 +203,9 @@ int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out);
  * steps). */
 int dllm_rewind_block(dllm_ctx* ctx);
 
-/* Whole request: prefill, then blocks until done.  out_tokens: host int32
+/* Whole request (Sec. 2.1, the block-wise decoding loop with prefix KV
+ * reuse; Sec. 3.2 / 3.3 as selected by sched): prefill, then blocks until
+ * done.  out_tokens: host int32
  * [batch][gen_len].  stats nullable. */
 int dllm_generate(dllm_ctx* ctx, const dllm_sched* sched, int batch, const int32_t* prompt, int Lp, int gen_len,
                   int32_t* out_tokens, dllm_stats* stats);
@@ -224,7 +237,10 @@ int dllm_get_scr_debug(dllm_ctx* ctx, int32_t* pos, int32_t* argmax, float* conf
  * projections 227 KB of shared memory (one CTA per SM, the deepest weight
  * ring) instead of leaving room beside them for the attention kernel's CTAs
  * (146 KB for the chained projections, 113 KB for dllm_op_gemm_*); bit 4:
- * record GEMM and attention timelines (dllm_get_trace).  Bits 2 and 3 apply
+ * record GEMM and attention timelines (dllm_get_trace); bit 5: the bounded-
+ * wait test: the next denoising step's first projection waits for a device
+ * word that nothing writes, so that wait runs out (after about 2 s) and the
+ * step reports DLLM_ETIMEOUT, which poisons the context.  Bits 2 and 3 apply
  * process-wide (for A/B measurements). */
 int dllm_set_debug(dllm_ctx* ctx, int flags);
 

@@ -29,7 +29,10 @@ int dllm_op_gemm(const void* W, const void* X, float* D, int M, int N, int K, in
  * allocation; *ms_per_launch = average kernel time by CUDA events on the
  * stream (micro-benchmark hook).  flags bit 0: chain the timed launches with
  * programmatic dependent launch; bit 1: plan 227 KB of shared memory instead
- * of 113 KB (one CTA per SM) for <= 96 tokens. */
+ * of 113 KB (one CTA per SM) for <= 96 tokens; bit 2: the bounded-wait test:
+ * a single launch whose operand producer waits for a device word that nothing
+ * writes, so the wait runs out after about 2 s, every role of the kernel
+ * unwinds and the call returns DLLM_ETIMEOUT (ms_per_launch is not set). */
 int dllm_op_gemm_timed(const void* W, const void* X, float* D, int M, int N, int K, int grid, int reps, int flags,
                        float* ms_per_launch, void* stream);
 
@@ -45,23 +48,29 @@ int dllm_op_gemm_timed(const void* W, const void* X, float* D, int M, int N, int
 int dllm_op_gemm_trace(const void* W, const void* X, float* D, int M, int N, int K, int grid, int reps,
                        float* ms_per_launch, unsigned long long* trace, int* grid_used, void* stream);
 
-/* dllm_op_gemm for callers that cannot allocate device memory, for example
- * code that runs while a stream is being captured into a CUDA graph (a
- * cudaMalloc there breaks the capture), or an embedding application whose
- * memory is owned by its own pool and forbids allocations behind its back.
- * The paper has no counterpart: this is a property of this library's API.
- * It computes the same D[n][m] = sum_k W[m][k] * X[n][k] as dllm_op_gemm but
- * keeps its scratch (split partials, tile tickets, status word) in one
- * statically sized device array of 8 MiB that every GPU loading the library
- * holds until the process exits; it calls no cudaMalloc, cudaFree or other
- * allocating routine.  Limits: at most 2046 output tiles (ceil(M/128) x
- * token tiles); the grid (0 = one CTA per SM, at most the SM count) is
- * shrunk to fit the array when chosen automatically, and an explicit grid
- * that does not fit is rejected with DLLM_ECAPACITY.  The first call on a device looks up the array's
- * device address (cudaGetSymbolAddress) with that device current; make that
- * first call before any stream capture.  All calls share the one array: two
+/* dllm_op_gemm for callers that cannot allocate device memory.  Such callers
+ * exist: an application (a serving engine, a game, a plugin host) often hands
+ * nearly all of a GPU's memory to its own pool allocator at start-up, so a
+ * cudaMalloc from a library it calls fails or breaks its accounting, and a
+ * latency-critical loop cannot afford the implicit device synchronisation
+ * that cudaMalloc and cudaFree may cause.  The paper has no counterpart: this
+ * is a property of this library's API.
+ * It computes the same D[n][m] = sum_k W[m][k] * X[n][k] as dllm_op_gemm
+ * (same arguments, same layouts) but keeps its scratch (split partials, tile
+ * tickets, status word) in one statically sized device array of 8 MiB that
+ * every GPU loading the library holds until the process exits; it calls no
+ * cudaMalloc, cudaFree or other allocating routine.
+ * Limits: at most 2046 output tiles (ceil(M/128) x token tiles of <= 256
+ * tokens), else DLLM_ECAPACITY; the grid (0 = one CTA per SM, at most the SM
+ * count) is shrunk to fit the array when chosen automatically (for 256-token
+ * tiles: 62 CTAs), and an explicit grid that does not fit is rejected with
+ * DLLM_ECAPACITY.
+ * The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress) with that device current.  Every call shares the
+ * one array and clears its tickets and status word before its launch: two
  * calls that overlap on the GPU (other streams, other host threads) race and
- * corrupt each other's results.  Synchronises the stream. */
+ * corrupt each other's results.  Synchronises the stream.
+ * Errors: DLLM_EINVAL, DLLM_ECAPACITY, DLLM_ECUDA, DLLM_ETIMEOUT. */
 int dllm_op_gemm_noalloc(const void* W, const void* X, float* D, int M, int N, int K, int grid, void* stream);
 
 /* Bidirectional attention of the window's queries over cached + window keys

@@ -366,6 +366,8 @@ static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0, bool sls 
         ChainArgs ca{};
         ChainMaps m{};
         add_phase(ca, m, pq, EPI_QKV, qkv_args(0), 0, ctx->wl[0] + L.w_qkv, tx_xn);
+        // debug flag 32 (the bounded-wait test): this launch waits for a word nobody writes
+        if ((ctx->debug & 32) && ctx->in_step) ca.gate = ctx->status + 2;
         if (int rc = run_chain(ca, m, 1, DLLM_K_QKV)) return rc;
     }
     for (int l = 0; l < c.n_layers; ++l) {
@@ -670,6 +672,12 @@ static int start_request(dllm_ctx* ctx, const dllm_sched* sched, int batch, int 
     int maxT = sched->use_prefix_cache ? std::max(P_random ? 0 : Lp, c.block_len * (1 + sched->spec_blocks)) : n_pos;
     if (maxT > c.max_window) return fail(ctx, DLLM_ECAPACITY, "window of %d tokens > max_window %d", maxT, c.max_window);
     if (!sched->use_prefix_cache && gen_len > kMaxBlock) return fail(ctx, DLLM_ECAPACITY, "block too long");
+    if (prompt)
+        for (int b = 0; b < batch; ++b)
+            for (int p = 0; p < Lp; ++p) {
+                int v = prompt[static_cast<size_t>(b) * Lp + p];
+                if (v < 0 || v >= c.vocab) return fail(ctx, DLLM_EINVAL, "prompt id %d out of range", v);
+            }
     ctx->sched = *sched;
     if (ctx->gexec) {  // the captured step bakes in the schedule's thresholds and counts
         cudaGraphExecDestroy(ctx->gexec);
@@ -693,12 +701,6 @@ static int start_request(dllm_ctx* ctx, const dllm_sched* sched, int batch, int 
             tok[static_cast<size_t>(b) * c.max_ctx + p] = prompt ? prompt[static_cast<size_t>(b) * Lp + p] : 0;
             st[static_cast<size_t>(b) * c.max_ctx + p] = DLLM_FIXED;
         }
-    if (prompt)
-        for (int b = 0; b < batch; ++b)
-            for (int p = 0; p < Lp; ++p) {
-                int v = prompt[static_cast<size_t>(b) * Lp + p];
-                if (v < 0 || v >= c.vocab) return fail(ctx, DLLM_EINVAL, "prompt id %d out of range", v);
-            }
     CK(cudaMemcpyAsync(ctx->tok, tok.data(), tok.size() * 4, cudaMemcpyHostToDevice, ctx->stream));
     CK(cudaMemcpyAsync(ctx->st, st.data(), st.size(), cudaMemcpyHostToDevice, ctx->stream));
     CK(launch_set_kv_len(ctx->seq_kv, batch, 0, ctx->stream));

@@ -1,6 +1,6 @@
-// Attention split shared by the attention kernel and the chained projections' in-chain
-// attention phase: the online-softmax pass of one query tile (16 rows per warp) over the keys
-// [kbeg, kend) of one (sequence, head), on bf16 mma.sync tiles.
+// One split of the mma.sync attention kernel (k_attn, kernels.cu): the online-softmax pass of
+// one query tile (16 rows per warp) over the keys [kbeg, kend) of one (sequence, head), on bf16
+// mma.sync tiles.
 #pragma once
 
 #include "common.cuh"

@@ -984,6 +984,11 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         int stage = 0;
         uint32_t par = 0;
         bool stop = false;
+        if (ca.gate) {  // the bounded-wait test hook (see ChainArgs::gate)
+            int open = 1;
+            if (lane == 0) open = wait_flag(ca.gate, tag, s_abort, status) ? 1 : 0;
+            stop = __shfl_sync(0xffffffffu, open, 0) == 0;  // warp-uniform decision
+        }
         for (int ph = 0; ph < ca.n_phases && !stop; ++ph) {
             const ChainPhase& P = ca.ph[ph];
             const GemmPlan p = phase_plan(P, rows);
@@ -1218,14 +1223,15 @@ cudaError_t gemm_init_attrs() { return chain_init_attrs(); }
 
 // One projection = a chain of one phase.
 cudaError_t gemm_launch(int epi, const GemmPlan& p, const CUtensorMap& tmW, const CUtensorMap& tmX,
-                        const EpiArgs& ep, const Scratch& scr, int* status, cudaStream_t st) {
-    if (static_cast<size_t>(p.grid) * p.ntile * kBM > scr.partial_floats ||
+                        const EpiArgs& ep, const Scratch& scr, int* status, cudaStream_t st, const int* gate) {
+    if (gemm_partial_floats(p) > scr.partial_floats ||
         static_cast<long long>(p.m_tiles) * p.n_tiles * kTicketStride > scr.counter_len)
         return cudaErrorInvalidValue;
     ChainArgs ca{};
     ca.n_phases = 1;
     ca.status = status;
     ca.tag_add = 1;
+    ca.gate = gate;
     ChainPhase& P = ca.ph[0];
     P.p = p;
     P.ep = ep;

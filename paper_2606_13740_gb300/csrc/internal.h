@@ -84,7 +84,7 @@ struct GemmPlan {
 };
 
 struct Scratch {
-    float* partials;     // [grid][2][ntile*128]
+    float* partials;     // [grid][ntile*128]: one split partial per CTA (gemm_partial_floats)
     int* counters;       // tile tickets, one per 128-byte line ([m_tiles*n_tiles][32]), zero between launches
     size_t partial_floats;
     int counter_len;
@@ -128,6 +128,10 @@ struct ChainArgs {
     // covers only the token tiles that hold those rows (the rest of the iteration space is
     // re-split over the CTAs).  Used by the LM head over compacted rows.
     const int* dyn_rows;
+    // Test hook for the bounded waits (null: off): the operand producer waits for *gate == the
+    // launch's tag before its first load.  Given a word nobody writes, that wait runs out after
+    // kWaitLimitCycles and the launch unwinds with kStatusTimeout, as any stalled wait would.
+    const int* gate;
     ChainPhase ph[kMaxPhases];
 };
 struct ChainMaps {
@@ -146,9 +150,15 @@ cudaError_t chain_init_attrs();
 // Tiling of one projection: token tiles of at most 256 (multiples of 32), 128 weight rows
 // per tile, 64-wide k-blocks, grid = min(iterations, grid_max).
 GemmPlan gemm_plan(int M, int N, int K, int grid_max, int epi);
+// Split-partial floats a single-projection launch of plan p needs (a CTA contributes to at most
+// one split tile, so one ntile x 128 slot per CTA); gemm_launch rejects a smaller Scratch.
+inline size_t gemm_partial_floats(const GemmPlan& p) {
+    return static_cast<size_t>(p.grid) * static_cast<size_t>(p.ntile) * 128;
+}
 bool make_tmap_bf16(CUtensorMap* tm, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows);
 cudaError_t gemm_launch(int epi, const GemmPlan& p, const CUtensorMap& tmW, const CUtensorMap& tmX,
-                        const EpiArgs& ep, const Scratch& scr, int* status, cudaStream_t st);
+                        const EpiArgs& ep, const Scratch& scr, int* status, cudaStream_t st,
+                        const int* gate = nullptr);
 
 // ---------------------------------------------------------------- launches
 // Every kernel is launched with programmatic stream serialisation (PDL): it may start

@@ -7,6 +7,8 @@
 // cannot use the array's name as a device address (in host code the symbol is
 // a host-side stand-in), so the first call on each device looks up the real
 // address with cudaGetSymbolAddress while that device is current, and keeps it.
+// The mutex below covers only that one-time lookup: the calls themselves share
+// the array without any ordering, so two calls that overlap on the GPU race.
 #include "../../include/dllm.h"
 #include "../../include/dllm_ops.h"
 #include "internal.h"
@@ -65,8 +67,11 @@ extern "C" int dllm_op_gemm_noalloc(const void* W, const void* X, float* D, int 
         return noalloc_fail(DLLM_ECUDA, "device query failed");
     GemmPlan p = gemm_plan(M, N, K, (grid > 0 && grid < sms) ? grid : sms, EPI_F32);
     p.pdl = false;
-    // the split partials take [grid][ntile x 128] floats behind the tickets
-    const size_t per_cta = static_cast<size_t>(p.ntile) * 128 * sizeof(float);
+    // the split partials sit behind the tickets; gemm_partial_floats is the bound gemm_launch
+    // checks, so the grid that fits is the one whose partials fit the rest of the array
+    GemmPlan one = p;
+    one.grid = 1;
+    const size_t per_cta = gemm_partial_floats(one) * sizeof(float);
     const size_t cap_ctas = (kNoAllocScratchBytes - kTicketBytes) / per_cta;
     if (static_cast<long long>(p.m_tiles) * p.n_tiles > kMaxTickets)
         return noalloc_fail(DLLM_ECAPACITY, "too many output tiles for the static scratch (M x N too large)");

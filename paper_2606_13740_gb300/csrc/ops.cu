@@ -73,7 +73,7 @@ static int gemm_impl(const void* W, const void* X, float* D, int M, int N, int K
     if (!make_tmap_bf16(&tw, W, M, K, 128) || !make_tmap_bf16(&tx, X, N, K, p.ntile))
         return op_fail(DLLM_EINVAL, "tensor map encode failed (alignment?)");
     DevBuf part, cnt, status;
-    const size_t pf = static_cast<size_t>(p.grid) * 2 * p.ntile * 128;
+    const size_t pf = gemm_partial_floats(p);
     const int cl = p.m_tiles * p.n_tiles * 32;
     if (!part.alloc(pf * 4) || !cnt.alloc(static_cast<size_t>(cl) * 4) || !status.alloc(16))
         return op_fail(DLLM_ENOMEM, "scratch allocation failed");
@@ -90,6 +90,14 @@ static int gemm_impl(const void* W, const void* X, float* D, int M, int N, int K
         ep.trace = static_cast<unsigned long long*>(tr.p);
     }
     if (grid_out) *grid_out = p.grid;
+    if (flags & 4) {
+        // the bounded-wait test: one launch whose operand producer waits for a word nobody
+        // writes (the zeroed third int of the status allocation; the launch's tag is 1)
+        cudaError_t e = gemm_launch(EPI_F32, p, tw, tx, ep, scr, static_cast<int*>(status.p), st,
+                                    static_cast<int*>(status.p) + 2);
+        if (e != cudaSuccess) return op_fail(DLLM_ECUDA, "gemm launch: %s", cudaGetErrorString(e));
+        return finish(st, static_cast<int*>(status.p));
+    }
     cudaEvent_t e0 = nullptr, e1 = nullptr;
     if (ms && (cudaEventCreate(&e0) != cudaSuccess || cudaEventCreate(&e1) != cudaSuccess))
         return op_fail(DLLM_ECUDA, "event creation failed");
@@ -172,7 +180,7 @@ int dllm_op_lmhead(const void* W, const void* X, const int32_t* cur, int32_t* x0
     if (!make_tmap_bf16(&tw, W, V, d, 128) || !make_tmap_bf16(&tx, X, N, d, p.ntile))
         return op_fail(DLLM_EINVAL, "tensor map encode failed (alignment?)");
     DevBuf part, cnt, status, lmp, zc;
-    const size_t pf = static_cast<size_t>(p.grid) * 2 * p.ntile * 128;
+    const size_t pf = gemm_partial_floats(p);
     const int cl = p.m_tiles * p.n_tiles * 32;
     if (!part.alloc(pf * 4) || !cnt.alloc(static_cast<size_t>(cl) * 4) || !status.alloc(16) ||
         !lmp.alloc(static_cast<size_t>(p.m_tiles) * N * 3 * 4) || !zc.alloc(static_cast<size_t>(N) * 4))

@@ -63,6 +63,23 @@ def test_gemm_llada_shapes_sampled(dev, M, N, K):
     assert np.array_equal(D, D2)
 
 
+def test_gemm_bounded_wait_times_out(dev):
+    """A launch whose operand wait can never be satisfied (a flag nothing writes) gives up after
+    its bounded wait, unwinds every role and reports DLLM_ETIMEOUT; the next launch is normal."""
+    from paper_2606_13740_gb300 import DllmError, dllm_op_gemm, dllm_op_gemm_timed
+    M, N, K = 1024, 32, 1024
+    rng = np.random.default_rng(5)
+    W = _bf16(rng, (M, K), 0.05)
+    X = _bf16(rng, (N, K))
+    with pytest.raises(DllmError) as e:
+        dllm_op_gemm_timed(W.to(dev), X.to(dev), M, N, K, 1, flags=4)
+    assert e.value.code == -4
+    D = dllm_op_gemm(W.to(dev), X.to(dev), M, N, K).cpu().numpy()
+    ref = _f64(X) @ _f64(W).T
+    scale = np.sqrt((_f64(X) ** 2).sum(1))[:, None] * np.sqrt((_f64(W) ** 2).sum(1))[None, :]
+    assert np.all(np.abs(D - ref) <= 1e-5 * scale + 1e-6)
+
+
 # ------------------------------------------------------------------ attention
 def _attn_ref(q, k, v, kv_len, T):
     B, H, _, hd = q.shape

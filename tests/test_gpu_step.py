@@ -325,19 +325,45 @@ def test_rewind_repeats_identical_step(model):
 
 
 def test_errors_poison_context(model):
+    """Argument and capacity errors leave the context usable; a device-side failure (here a
+    bounded wait that runs out) poisons it: the call reports DLLM_ETIMEOUT, every later call
+    DLLM_ESTATE, and a fresh context works."""
     from paper_2606_13740_gb300 import DllmError, Sched
     ctx = _gpu_ctx(max_ctx=96)
-    with pytest.raises(DllmError):  # capacity
+    with pytest.raises(DllmError) as e:  # capacity
         ctx.dllm_prefill(Sched(), I.uniform_prompt(64, TINY.vocab, TINY.mask_id), 64)
-    with pytest.raises(DllmError):  # no request yet
+    assert e.value.code == -6
+    with pytest.raises(DllmError) as e:  # no request yet
         ctx.dllm_begin_block()
+    assert e.value.code == -1
+    bad = I.uniform_prompt(32, TINY.vocab, TINY.mask_id)
+    bad[5] = TINY.vocab  # an id out of range: rejected before the request starts
+    with pytest.raises(DllmError) as e:
+        ctx.dllm_prefill(Sched(steps_per_block=8), bad, 32)
+    assert e.value.code == -1
     prompt = I.uniform_prompt(32, TINY.vocab, TINY.mask_id)
     ctx.dllm_prefill(Sched(steps_per_block=8), prompt, 32)
     ctx.dllm_begin_block()
     ctx.dllm_denoise_step()
-    with pytest.raises(DllmError):  # block unfinished
+    with pytest.raises(DllmError) as e:  # block unfinished
         ctx.dllm_begin_block()
+    assert e.value.code == -1
+    out = ctx.dllm_denoise_step()  # still usable
+    assert out["n_committed"] == 4
+    ctx.dllm_set_debug(32)  # the next step's first projection waits for a word nothing writes
+    with pytest.raises(DllmError) as e:
+        ctx.dllm_denoise_step()
+    assert e.value.code == -4  # DLLM_ETIMEOUT
+    for call in (ctx.dllm_denoise_step, ctx.dllm_begin_block, ctx.dllm_get_state, ctx.dllm_sync):
+        with pytest.raises(DllmError) as e:
+            call()
+        assert e.value.code == -5  # DLLM_ESTATE: poisoned
     ctx.close()
+    fresh = _gpu_ctx(max_ctx=96)
+    fresh.dllm_prefill(Sched(steps_per_block=8), prompt, 32)
+    fresh.dllm_begin_block()
+    assert fresh.dllm_denoise_step()["n_committed"] == 4
+    fresh.close()
 
 
 @pytest.mark.parametrize("slide", [0, 1])
