@@ -178,9 +178,17 @@ struct dllm_ctx {
     int blk = -1, c0 = 0, c1 = 0, step = 0;
     int last_w0 = 0, last_T = 0, last_spec = 0;
     int debug = 0;
-    // graph cache for the step
-    cudaGraphExec_t gexec = nullptr;
-    int g_T = -1, g_B = -1, g_kv = -1, g_dbg = -1;
+    // captured steps, one per (window rows, batch, planned cache length, debug key); all of them
+    // bake in the request's schedule, so a request with another schedule drops them
+    struct StepGraph {
+        cudaGraphExec_t exec = nullptr;
+        int T = -1, B = -1, kv = -1, dbg = -1;
+        unsigned long long used = 0;  // last use, for eviction
+        int n_marks = 0, launches = 0, trace_launches = 0;
+        std::vector<int> ev_kind;     // the profiling events' kinds as recorded at capture
+    };
+    std::vector<StepGraph> graphs;
+    unsigned long long graph_clock = 0;
     // per-kernel timing (events recorded after every launch of the step)
     bool profiling = false;
     std::vector<cudaEvent_t> ev;
@@ -211,6 +219,7 @@ static void mark(dllm_ctx* ctx, int kind) {
 }
 
 constexpr int kTraceLaunches = 512;
+constexpr size_t kMaxStepGraphs = 32;  // captured steps kept per context (LRU)
 constexpr size_t kTraceStride = 256 * 16;  // per launch: 256 CTAs x 16 slots
 
 // Trace buffer for the GEMM launch about to be made in a step (null when off).
@@ -501,7 +510,7 @@ const char* dllm_last_error(const dllm_ctx* ctx) { return ctx ? ctx->err.c_str()
 void dllm_free(dllm_ctx* ctx) {
     if (!ctx) return;
     if (ctx->stream) cudaStreamSynchronize(ctx->stream);
-    if (ctx->gexec) cudaGraphExecDestroy(ctx->gexec);
+    for (auto& g : ctx->graphs) cudaGraphExecDestroy(g.exec);
     for (cudaEvent_t e : ctx->ev) cudaEventDestroy(e);
     if (ctx->logits) cudaFree(ctx->logits);
     if (ctx->trace) cudaFree(ctx->trace);
@@ -678,12 +687,12 @@ static int start_request(dllm_ctx* ctx, const dllm_sched* sched, int batch, int 
                 int v = prompt[static_cast<size_t>(b) * Lp + p];
                 if (v < 0 || v >= c.vocab) return fail(ctx, DLLM_EINVAL, "prompt id %d out of range", v);
             }
-    ctx->sched = *sched;
-    if (ctx->gexec) {  // the captured step bakes in the schedule's thresholds and counts
-        cudaGraphExecDestroy(ctx->gexec);
-        ctx->gexec = nullptr;
-        ctx->g_T = -1;
+    if (memcmp(&ctx->sched, sched, sizeof(dllm_sched)) != 0) {
+        // the captured steps bake in the schedule's thresholds and counts
+        for (auto& g : ctx->graphs) cudaGraphExecDestroy(g.exec);
+        ctx->graphs.clear();
     }
+    ctx->sched = *sched;
     ctx->B = batch;
     ctx->Lp = Lp;
     ctx->gen_len = gen_len;
@@ -851,11 +860,11 @@ int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out) {
         // trace pointers and the refresh rows are baked in too
         const int key_dbg = ctx->debug | (ctx->profiling ? 256 : 0) |
                             ((s.use_prefix_cache ? s.scr_rows : 0) << 10) | (s.sls << 16);
-        if (!ctx->gexec || ctx->g_T != T || ctx->g_B != ctx->B || ctx->g_kv != plan_kv(ctx) || ctx->g_dbg != key_dbg) {
-            if (ctx->gexec) {
-                cudaGraphExecDestroy(ctx->gexec);
-                ctx->gexec = nullptr;
-            }
+        const int kv = plan_kv(ctx);
+        dllm_ctx::StepGraph* hit = nullptr;
+        for (auto& g : ctx->graphs)
+            if (g.T == T && g.B == ctx->B && g.kv == kv && g.dbg == key_dbg) hit = &g;
+        if (!hit) {
             cudaGraph_t g = nullptr;
             CK(cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal));
             ctx->capturing = true;
@@ -867,15 +876,37 @@ int dllm_denoise_step(dllm_ctx* ctx, dllm_step_out* out) {
                 return rc;
             }
             if (ee != cudaSuccess) return fail(ctx, DLLM_ECUDA, "graph capture: %s", cudaGetErrorString(ee));
-            ee = cudaGraphInstantiate(&ctx->gexec, g, 0);
+            cudaGraphExec_t exec = nullptr;
+            ee = cudaGraphInstantiate(&exec, g, 0);
             cudaGraphDestroy(g);
             if (ee != cudaSuccess) return fail(ctx, DLLM_ECUDA, "graph instantiate: %s", cudaGetErrorString(ee));
-            ctx->g_T = T;
-            ctx->g_B = ctx->B;
-            ctx->g_kv = plan_kv(ctx);
-            ctx->g_dbg = key_dbg;
+            if (ctx->graphs.size() >= kMaxStepGraphs) {  // evict the least recently used
+                size_t lru = 0;
+                for (size_t i = 1; i < ctx->graphs.size(); ++i)
+                    if (ctx->graphs[i].used < ctx->graphs[lru].used) lru = i;
+                cudaGraphExecDestroy(ctx->graphs[lru].exec);
+                ctx->graphs.erase(ctx->graphs.begin() + static_cast<long>(lru));
+            }
+            dllm_ctx::StepGraph sg;
+            sg.exec = exec;
+            sg.T = T;
+            sg.B = ctx->B;
+            sg.kv = kv;
+            sg.dbg = key_dbg;
+            sg.n_marks = ctx->n_marks;
+            sg.launches = ctx->launches_per_step;
+            sg.trace_launches = ctx->trace_launch;
+            sg.ev_kind = ctx->ev_kind;
+            ctx->graphs.push_back(sg);
+            hit = &ctx->graphs.back();
         }
-        CK(cudaGraphLaunch(ctx->gexec, ctx->stream));
+        hit->used = ++ctx->graph_clock;
+        // what the replayed graph records: its own events' kinds, launch and trace counts
+        ctx->n_marks = hit->n_marks;
+        ctx->launches_per_step = hit->launches;
+        ctx->trace_launch = hit->trace_launches;
+        if (!hit->ev_kind.empty()) ctx->ev_kind = hit->ev_kind;
+        CK(cudaGraphLaunch(hit->exec, ctx->stream));
     } else {
         int rc = step_kernels(ctx, T);
         if (rc) return rc;
@@ -920,8 +951,19 @@ int dllm_generate(dllm_ctx* ctx, const dllm_sched* sched, int batch, const int32
     int rc = dllm_prefill(ctx, sched, batch, prompt, Lp, gen_len);
     if (rc) return rc;
     dllm_stats stt{};
+    // LLaDA's fixed schedule without lookahead or sliding finishes a block of at least S
+    // positions in exactly S = steps_per_block steps (every step commits at least one position
+    // and leaves at least one per remaining step; re-masks only add to the count; the last step
+    // commits what is left): those steps are queued without a read-back, the last one reports
+    const bool fixed_len = sched->commit_mode == DLLM_COMMIT_SCHEDULE && sched->spec_blocks == 0 && !sched->slide;
     while ((rc = dllm_begin_block(ctx)) == DLLM_OK) {
         dllm_step_out o{};
+        if (fixed_len && sched->steps_per_block <= ctx->c1 - ctx->c0)
+            for (int i = 0; i + 1 < sched->steps_per_block; ++i) {
+                rc = dllm_denoise_step(ctx, nullptr);
+                if (rc) return rc;
+                stt.steps++;
+            }
         // a block finishes within S steps (schedule), or within the revision horizon S plus one
         // step per position (threshold: every step commits at least one)
         for (int guard = 0; guard < 4 * sched->steps_per_block + 4 + ctx->cfg.block_len; ++guard) {
