@@ -59,8 +59,13 @@ typedef struct dllm_ctx dllm_ctx;
  * causal mask, rotate-half RoPE, SwiGLU MLP, untied LM head.  Weights are
  * bf16, drawn on the device from weight_seed (N(0, 0.02) by a counter-based
  * SplitMix64/Irwin-Hall generator); RMSNorm gains are one.
+ * n_kv_heads < n_heads gives grouped-query attention (the Dream-7B model the
+ * paper also runs, Sec. 5.1): query head h reads K/V head h / (n_heads /
+ * n_kv_heads), and the KV cache holds n_kv_heads heads.
  * Constraints: head_dim in {64, 128}; d_model, n_heads*head_dim multiples of
- * 128; vocab, ffn multiples of 8; max_window * max_batch <= 4096. */
+ * 128; n_kv_heads 0 (= n_heads) or a divisor of n_heads with
+ * n_kv_heads*head_dim a multiple of 128; vocab, ffn multiples of 8;
+ * max_window * max_batch <= 4096. */
 typedef struct {
     int n_layers, d_model, n_heads, head_dim, ffn, vocab, mask_id;
     float rope_base, rms_eps;
@@ -69,6 +74,7 @@ typedef struct {
     int max_window;  /* query tokens per sequence per forward (window or prompt) */
     int block_len;   /* tokens per block (32) */
     uint64_t weight_seed;
+    int n_kv_heads;  /* K/V heads; 0 = n_heads (multi-head attention, LLaDA) */
 } dllm_config;
 
 /* Commit rules (dllm_sched.commit_mode). */
@@ -250,7 +256,7 @@ int dllm_set_debug(dllm_ctx* ctx, int flags);
 int dllm_get_weight(dllm_ctx* ctx, int layer, int which, uint16_t* out, size_t n_elems);
 
 /* Copy a slice of the K or V cache (which 0/1) of one layer and sequence:
- * out fp32 [n][n_heads*head_dim] for positions [p0, p0+n).  Synchronises. */
+ * out fp32 [n][n_kv_heads*head_dim] for positions [p0, p0+n).  Synchronises. */
 int dllm_get_kv(dllm_ctx* ctx, int layer, int which, int seq, int p0, int n, float* out);
 
 /* Kernel kinds of one denoising step, for dllm_get_profile. */

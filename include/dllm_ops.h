@@ -75,11 +75,13 @@ int dllm_op_gemm_noalloc(const void* W, const void* X, float* D, int M, int N, i
 
 /* Bidirectional attention of the window's queries over cached + window keys
  * (Sec. 2.1, block-wise decoding with prefix KV reuse; no causal mask).
- * q dev bf16 [B][H][T][hd]; kc, vc dev bf16 [B][H][cap][hd] (keys of
+ * q dev bf16 [B][H][T][hd]; kc, vc dev bf16 [B][Hkv][cap][hd] (keys of
  * sequence b: positions [0, kv_len[b] + T)); kv_len dev int32 [B];
- * out dev bf16 [B*T][H*hd].  hd in {64, 128}. */
+ * out dev bf16 [B*T][H*hd].  hd in {64, 128}.  Hkv = H is multi-head
+ * attention; Hkv < H (dividing H) is grouped-query attention (the Dream-7B
+ * model of Sec. 5.1): query head h reads K/V head h / (H / Hkv). */
 int dllm_op_attention(const void* q, const void* kc, const void* vc, const int32_t* kv_len, void* out, int B, int T,
-                      int H, int hd, int cap, int max_kv_len, void* stream);
+                      int H, int Hkv, int hd, int cap, int max_kv_len, void* stream);
 
 /* LM head with decision (Sec. 2.1 confidence-selected commits; Sec. 3.3
  * selective logits): per token n, z = W X[n]^T over the vocab; x0 = argmax

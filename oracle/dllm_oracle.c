@@ -109,11 +109,18 @@ struct orc_model {
     float* norm_final; /* [d] */
 };
 
+/* Width of the K and V projections: K/V heads x head_dim (grouped-query attention has fewer
+ * K/V heads than query heads; n_kv_heads = 0 means as many as query heads). */
+static int kv_width(const orc_config* c) {
+    return (c->n_kv_heads > 0 ? c->n_kv_heads : c->n_heads) * c->head_dim;
+}
+
 static size_t wsize(const orc_config* c, int which, int* rows, int* cols) {
     int d = c->d_model, qd = c->n_heads * c->head_dim, F = c->ffn;
     int r = 0, k = 0;
     switch (which) {
-        case ORC_W_Q: case ORC_W_K: case ORC_W_V: r = qd; k = d; break;
+        case ORC_W_Q: r = qd; k = d; break;
+        case ORC_W_K: case ORC_W_V: r = kv_width(c); k = d; break;
         case ORC_W_O: r = d; k = qd; break;
         case ORC_W_GATE: case ORC_W_UP: r = F; k = d; break;
         case ORC_W_DOWN: r = d; k = F; break;
@@ -291,6 +298,9 @@ int orc_forward_ex(const orc_model* m, int T, int Tk, const int32_t* tok, const 
     const orc_config* c = &m->c;
     int d = c->d_model, H = c->n_heads, hd = c->head_dim, F = c->ffn, V = c->vocab;
     int qd = H * hd;
+    /* grouped-query attention: query head hh reads K/V head hh / grp */
+    int kvd = kv_width(c), Hkv = kvd / hd, grp = H / Hkv;
+    if (Hkv < 1 || H % Hkv) return -1;
     int L = n_layers_run < 0 || n_layers_run > c->n_layers ? c->n_layers : n_layers_run;
     if (L > m->n_gen_layers) return -1;
     if (T <= 0) return 0;
@@ -299,8 +309,8 @@ int orc_forward_ex(const orc_model* m, int T, int Tk, const int32_t* tok, const 
     float* x = (float*)malloc(sizeof(float) * Td);
     float* h = (float*)malloc(sizeof(float) * Td);
     float* q = (float*)malloc(sizeof(float) * (size_t)T * qd);
-    float* k = (float*)malloc(sizeof(float) * (size_t)T * qd);
-    float* v = (float*)malloc(sizeof(float) * (size_t)T * qd);
+    float* k = (float*)malloc(sizeof(float) * (size_t)T * kvd);
+    float* v = (float*)malloc(sizeof(float) * (size_t)T * kvd);
     float* att = (float*)malloc(sizeof(float) * (size_t)T * qd);
     float* o = (float*)malloc(sizeof(float) * Td);
     float* g = (float*)malloc(sizeof(float) * (size_t)T * F);
@@ -315,17 +325,16 @@ int orc_forward_ex(const orc_model* m, int T, int Tk, const int32_t* tok, const 
         for (int t = 0; t < T; ++t)
             orc_rmsnorm(d, x + (size_t)t * d, m->norm_attn + (size_t)l * d, c->rms_eps, h + (size_t)t * d);
         linear(W[ORC_W_Q], qd, d, h, T, q);
-        linear(W[ORC_W_K], qd, d, h, T, k);
-        linear(W[ORC_W_V], qd, d, h, T, v);
-        for (int t = 0; t < T; ++t)
-            for (int hh = 0; hh < H; ++hh) {
-                orc_rope(hd, c->rope_base, pos[t], q + (size_t)t * qd + (size_t)hh * hd);
-                orc_rope(hd, c->rope_base, pos[t], k + (size_t)t * qd + (size_t)hh * hd);
-            }
-        if (out_k) memcpy(out_k + (size_t)l * T * qd, k, sizeof(float) * (size_t)T * qd);
-        if (out_v) memcpy(out_v + (size_t)l * T * qd, v, sizeof(float) * (size_t)T * qd);
-        const float* lk = P > 0 ? pk + (size_t)l * P * qd : NULL;
-        const float* lv = P > 0 ? pv + (size_t)l * P * qd : NULL;
+        linear(W[ORC_W_K], kvd, d, h, T, k);
+        linear(W[ORC_W_V], kvd, d, h, T, v);
+        for (int t = 0; t < T; ++t) {
+            for (int hh = 0; hh < H; ++hh) orc_rope(hd, c->rope_base, pos[t], q + (size_t)t * qd + (size_t)hh * hd);
+            for (int hh = 0; hh < Hkv; ++hh) orc_rope(hd, c->rope_base, pos[t], k + (size_t)t * kvd + (size_t)hh * hd);
+        }
+        if (out_k) memcpy(out_k + (size_t)l * T * kvd, k, sizeof(float) * (size_t)T * kvd);
+        if (out_v) memcpy(out_v + (size_t)l * T * kvd, v, sizeof(float) * (size_t)T * kvd);
+        const float* lk = P > 0 ? pk + (size_t)l * P * kvd : NULL;
+        const float* lv = P > 0 ? pv + (size_t)l * P * kvd : NULL;
         int NK = P + Tk; /* rows from Tk on are queries only */
 #pragma omp parallel
         {
@@ -335,16 +344,17 @@ int orc_forward_ex(const orc_model* m, int T, int Tk, const int32_t* tok, const 
             for (int hh = 0; hh < H; ++hh)
                 for (int t = 0; t < T; ++t) {
                     const float* qt = q + (size_t)t * qd + (size_t)hh * hd;
+                    const size_t kh = (size_t)(hh / grp) * hd; /* its K/V head */
                     double mx = -INFINITY;
                     /* keys in position order: cached prefix, then the window */
                     for (int j = 0; j < NK; ++j) {
                         const float* kj;
                         if (j < P) {
-                            kj = lk + (size_t)j * qd + (size_t)hh * hd;
+                            kj = lk + (size_t)j * kvd + kh;
                         } else {
                             int w = j - P;
                             if (group && group[w] > group[t]) { sc[j] = -INFINITY; continue; }
-                            kj = k + (size_t)w * qd + (size_t)hh * hd;
+                            kj = k + (size_t)w * kvd + kh;
                         }
                         double s = 0.0;
                         for (int i = 0; i < hd; ++i) s += (double)qt[i] * (double)kj[i];
@@ -359,8 +369,7 @@ int orc_forward_ex(const orc_model* m, int T, int Tk, const int32_t* tok, const 
                     for (int i = 0; i < hd; ++i) acc[i] = 0.0;
                     for (int j = 0; j < NK; ++j) {
                         if (sc[j] == 0.0) continue;
-                        const float* vj = j < P ? lv + (size_t)j * qd + (size_t)hh * hd
-                                                : v + (size_t)(j - P) * qd + (size_t)hh * hd;
+                        const float* vj = j < P ? lv + (size_t)j * kvd + kh : v + (size_t)(j - P) * kvd + kh;
                         double p = sc[j] / sum;
                         for (int i = 0; i < hd; ++i) acc[i] += p * (double)vj[i];
                     }
@@ -522,7 +531,7 @@ struct orc_session {
     int Lp, G, n_pos;
     int32_t* tok;
     uint8_t* st;
-    float* pk; /* [L][n_pos][qd] */
+    float* pk; /* [L][n_pos][kvd]: K/V heads x head_dim */
     float* pv;
     int kv_len;
     int cb, c0, c1, step; /* current block */
@@ -548,7 +557,7 @@ orc_session* orc_session_new(const orc_model* m, const orc_sched* s, int Lp, con
     x->st = (uint8_t*)malloc((size_t)x->n_pos);
     for (int i = 0; i < Lp; ++i) { x->tok[i] = prompt[i]; x->st[i] = ORC_FIXED; }
     for (int i = Lp; i < x->n_pos; ++i) { x->tok[i] = c->mask_id; x->st[i] = ORC_MASKED; }
-    size_t kvn = (size_t)c->n_layers * x->n_pos * c->n_heads * c->head_dim;
+    size_t kvn = (size_t)c->n_layers * x->n_pos * kv_width(c);
     x->pk = (float*)calloc(kvn, sizeof(float));
     x->pv = (float*)calloc(kvn, sizeof(float));
     x->cb = -1;
@@ -585,27 +594,27 @@ int orc_n_pos(const orc_session* x) { return x->n_pos; }
  * append use the same rule: attend to prefix plus the new positions). */
 static int append_kv(orc_session* x, int a, int b) {
     const orc_config* c = &x->m->c;
-    int T = b - a, qd = c->n_heads * c->head_dim, L = c->n_layers;
+    int T = b - a, kvd = kv_width(c), L = c->n_layers;
     if (T <= 0) return 0;
     int P = x->kv_len;
     int32_t* pos = (int32_t*)malloc(sizeof(int32_t) * (size_t)T);
     for (int t = 0; t < T; ++t) pos[t] = a + t;
     float* pk = NULL;
     float* pv = NULL;
-    if (P > 0) { /* contiguous [L][P][qd] view of the cache */
-        pk = (float*)malloc(sizeof(float) * (size_t)L * P * qd);
-        pv = (float*)malloc(sizeof(float) * (size_t)L * P * qd);
+    if (P > 0) { /* contiguous [L][P][kvd] view of the cache */
+        pk = (float*)malloc(sizeof(float) * (size_t)L * P * kvd);
+        pv = (float*)malloc(sizeof(float) * (size_t)L * P * kvd);
         for (int l = 0; l < L; ++l) {
-            memcpy(pk + (size_t)l * P * qd, x->pk + (size_t)l * x->n_pos * qd, sizeof(float) * (size_t)P * qd);
-            memcpy(pv + (size_t)l * P * qd, x->pv + (size_t)l * x->n_pos * qd, sizeof(float) * (size_t)P * qd);
+            memcpy(pk + (size_t)l * P * kvd, x->pk + (size_t)l * x->n_pos * kvd, sizeof(float) * (size_t)P * kvd);
+            memcpy(pv + (size_t)l * P * kvd, x->pv + (size_t)l * x->n_pos * kvd, sizeof(float) * (size_t)P * kvd);
         }
     }
-    float* ok = (float*)malloc(sizeof(float) * (size_t)L * T * qd);
-    float* ov = (float*)malloc(sizeof(float) * (size_t)L * T * qd);
+    float* ok = (float*)malloc(sizeof(float) * (size_t)L * T * kvd);
+    float* ov = (float*)malloc(sizeof(float) * (size_t)L * T * kvd);
     int rc = orc_forward(x->m, T, x->tok + a, pos, P, pk, pv, NULL, ok, ov, NULL, -1);
     for (int l = 0; l < L; ++l) {
-        memcpy(x->pk + ((size_t)l * x->n_pos + P) * qd, ok + (size_t)l * T * qd, sizeof(float) * (size_t)T * qd);
-        memcpy(x->pv + ((size_t)l * x->n_pos + P) * qd, ov + (size_t)l * T * qd, sizeof(float) * (size_t)T * qd);
+        memcpy(x->pk + ((size_t)l * x->n_pos + P) * kvd, ok + (size_t)l * T * kvd, sizeof(float) * (size_t)T * kvd);
+        memcpy(x->pv + ((size_t)l * x->n_pos + P) * kvd, ov + (size_t)l * T * kvd, sizeof(float) * (size_t)T * kvd);
     }
     x->kv_len = P + T;
     free(pos); free(pk); free(pv); free(ok); free(ov);
@@ -644,7 +653,7 @@ int orc_begin_block(orc_session* x) {
 
 int orc_denoise_step(orc_session* x, orc_step_out* out, int keep_logits) {
     const orc_config* c = &x->m->c;
-    int V = c->vocab, qd = c->n_heads * c->head_dim, L = c->n_layers;
+    int V = c->vocab, kvd = kv_width(c), L = c->n_layers;
     if (x->cb < 0 || x->c0 >= x->n_pos) return -3;
     int masked = 0;
     for (int p = x->c0; p < x->c1; ++p) masked += x->st[p] == ORC_MASKED;
@@ -702,18 +711,18 @@ int orc_denoise_step(orc_session* x, orc_step_out* out, int keep_logits) {
     float* pk = NULL;
     float* pv = NULL;
     if (P > 0) {
-        pk = (float*)malloc(sizeof(float) * (size_t)L * P * qd);
-        pv = (float*)malloc(sizeof(float) * (size_t)L * P * qd);
+        pk = (float*)malloc(sizeof(float) * (size_t)L * P * kvd);
+        pv = (float*)malloc(sizeof(float) * (size_t)L * P * kvd);
         for (int l = 0; l < L; ++l) {
-            memcpy(pk + (size_t)l * P * qd, x->pk + (size_t)l * x->n_pos * qd, sizeof(float) * (size_t)P * qd);
-            memcpy(pv + (size_t)l * P * qd, x->pv + (size_t)l * x->n_pos * qd, sizeof(float) * (size_t)P * qd);
+            memcpy(pk + (size_t)l * P * kvd, x->pk + (size_t)l * x->n_pos * kvd, sizeof(float) * (size_t)P * kvd);
+            memcpy(pv + (size_t)l * P * kvd, x->pv + (size_t)l * x->n_pos * kvd, sizeof(float) * (size_t)P * kvd);
         }
     }
     free(x->logits);
     x->logits = (float*)malloc(sizeof(float) * (size_t)Tq * V);
     int keep_kv = nt > 0 || x->s.slide;
-    float* nk = keep_kv ? (float*)malloc(sizeof(float) * (size_t)L * Tq * qd) : NULL;
-    float* nv = keep_kv ? (float*)malloc(sizeof(float) * (size_t)L * Tq * qd) : NULL;
+    float* nk = keep_kv ? (float*)malloc(sizeof(float) * (size_t)L * Tq * kvd) : NULL;
+    float* nv = keep_kv ? (float*)malloc(sizeof(float) * (size_t)L * Tq * kvd) : NULL;
     int rc = orc_forward_ex(x->m, Tq, T, rows, pos, P, pk, pv, NULL, nk, nv, x->logits, -1);
     free(pos); free(rows); free(pk); free(pv);
     if (rc) { free(nk); free(nv); return rc; }
@@ -744,8 +753,8 @@ int orc_denoise_step(orc_session* x, orc_step_out* out, int keep_logits) {
             continue;
         }
         for (int l = 0; l < L; ++l) {
-            memcpy(x->pk + ((size_t)l * x->n_pos + p) * qd, nk + ((size_t)l * Tq + T + r) * qd, sizeof(float) * qd);
-            memcpy(x->pv + ((size_t)l * x->n_pos + p) * qd, nv + ((size_t)l * Tq + T + r) * qd, sizeof(float) * qd);
+            memcpy(x->pk + ((size_t)l * x->n_pos + p) * kvd, nk + ((size_t)l * Tq + T + r) * kvd, sizeof(float) * kvd);
+            memcpy(x->pv + ((size_t)l * x->n_pos + p) * kvd, nv + ((size_t)l * Tq + T + r) * kvd, sizeof(float) * kvd);
         }
         so.n_refreshed++;
     }
@@ -758,8 +767,8 @@ int orc_denoise_step(orc_session* x, orc_step_out* out, int keep_logits) {
             adv++;
         for (int l = 0; l < L; ++l)
             for (int t = 0; t < adv; ++t) {
-                memcpy(x->pk + ((size_t)l * x->n_pos + w0 + t) * qd, nk + ((size_t)l * Tq + t) * qd, sizeof(float) * qd);
-                memcpy(x->pv + ((size_t)l * x->n_pos + w0 + t) * qd, nv + ((size_t)l * Tq + t) * qd, sizeof(float) * qd);
+                memcpy(x->pk + ((size_t)l * x->n_pos + w0 + t) * kvd, nk + ((size_t)l * Tq + t) * kvd, sizeof(float) * kvd);
+                memcpy(x->pv + ((size_t)l * x->n_pos + w0 + t) * kvd, nv + ((size_t)l * Tq + t) * kvd, sizeof(float) * kvd);
             }
         x->kv_len += adv;
     }
@@ -804,6 +813,6 @@ int orc_set_state(orc_session* x, const int32_t* tok, const uint8_t* st) {
 
 const float* orc_prefix_kv(const orc_session* x, int layer, int which) {
     const orc_config* c = &x->m->c;
-    size_t off = (size_t)layer * x->n_pos * c->n_heads * c->head_dim;
+    size_t off = (size_t)layer * x->n_pos * kv_width(c);
     return (which == 0 ? x->pk : x->pv) + off;
 }

@@ -35,6 +35,10 @@ typedef struct {
     int n_layers, d_model, n_heads, head_dim, ffn, vocab, mask_id;
     double rope_base, rms_eps;
     uint64_t weight_seed;
+    /* K/V heads (grouped-query attention, as in the Dream-7B model of Sec. 5.1); 0 = n_heads
+     * (multi-head attention, LLaDA).  Must divide n_heads: query head h reads K/V head
+     * h / (n_heads / n_kv_heads). */
+    int n_kv_heads;
 } orc_config;
 
 typedef struct {

@@ -40,7 +40,8 @@ def build(force: bool = False) -> str:
 class _Cfg(C.Structure):
     _fields_ = [("n_layers", C.c_int), ("d_model", C.c_int), ("n_heads", C.c_int),
                 ("head_dim", C.c_int), ("ffn", C.c_int), ("vocab", C.c_int), ("mask_id", C.c_int),
-                ("rope_base", C.c_double), ("rms_eps", C.c_double), ("weight_seed", C.c_uint64)]
+                ("rope_base", C.c_double), ("rms_eps", C.c_double), ("weight_seed", C.c_uint64),
+                ("n_kv_heads", C.c_int)]
 
 
 class _Sched(C.Structure):
@@ -130,10 +131,15 @@ class OracleConfig:
     rope_base: float = 10000.0
     rms_eps: float = 1e-5
     weight_seed: int = 0x11ADA8B
+    n_kv_heads: int = 0  # grouped-query attention (Dream-7B style); 0 = n_heads (LLaDA's multi-head)
+
+    @property
+    def kv_dim(self):
+        return (self.n_kv_heads or self.n_heads) * self.head_dim
 
     def c(self):
         return _Cfg(self.n_layers, self.d_model, self.n_heads, self.head_dim, self.ffn, self.vocab,
-                    self.mask_id, self.rope_base, self.rms_eps, self.weight_seed)
+                    self.mask_id, self.rope_base, self.rms_eps, self.weight_seed, self.n_kv_heads)
 
 
 @dataclass
@@ -239,7 +245,8 @@ class Model:
         if not ptr:
             raise KeyError((layer, which))
         qd = c.n_heads * c.head_dim
-        shapes = {W_Q: (qd, c.d_model), W_K: (qd, c.d_model), W_V: (qd, c.d_model), W_O: (c.d_model, qd),
+        kvd = c.kv_dim
+        shapes = {W_Q: (qd, c.d_model), W_K: (kvd, c.d_model), W_V: (kvd, c.d_model), W_O: (c.d_model, qd),
                   W_GATE: (c.ffn, c.d_model), W_UP: (c.ffn, c.d_model), W_DOWN: (c.d_model, c.ffn)}
         shape = (c.vocab, c.d_model) if layer < 0 else shapes[which]
         buf = (C.c_uint16 * n.value).from_address(ptr)
@@ -258,19 +265,19 @@ class Model:
 
 def forward(model: Model, tok, pos, prefix_k=None, prefix_v=None, group=None, want_kv=False, logits=True,
             n_layers_run=-1):
-    """orc_forward; returns dict(logits [T][V], k [L][T][qd], v [L][T][qd])."""
+    """orc_forward; returns dict(logits [T][V], k [L][T][kvd], v [L][T][kvd]) (kvd: K/V heads x head_dim)."""
     c = model.cfg
     tok = np.ascontiguousarray(tok, np.int32)
     pos = np.ascontiguousarray(pos, np.int32)
     T = tok.size
-    qd = c.n_heads * c.head_dim
+    kvd = c.kv_dim
     P = 0 if prefix_k is None else prefix_k.shape[1]
     pk = None if prefix_k is None else np.ascontiguousarray(prefix_k, np.float32)
     pv = None if prefix_v is None else np.ascontiguousarray(prefix_v, np.float32)
     grp = None if group is None else np.ascontiguousarray(group, np.int32)
     L = c.n_layers if n_layers_run < 0 else n_layers_run
-    ok = np.empty((L, T, qd), np.float32) if want_kv else None
-    ov = np.empty((L, T, qd), np.float32) if want_kv else None
+    ok = np.empty((L, T, kvd), np.float32) if want_kv else None
+    ov = np.empty((L, T, kvd), np.float32) if want_kv else None
     lg = np.empty((T, c.vocab), np.float32) if logits else None
     rc = lib().orc_forward(model.h, T, _p(tok), _p(pos), P, _p(pk), _p(pv), _p(grp), _p(ok), _p(ov), _p(lg),
                            n_layers_run)
@@ -354,10 +361,10 @@ class Session:
     def prefix_kv(self, layer, which):
         c = self.model.cfg
         kv_len = self.state()[2]
-        qd = c.n_heads * c.head_dim
+        kvd = c.kv_dim
         ptr = lib().orc_prefix_kv(self.h, layer, which)
-        buf = (C.c_float * (kv_len * qd)).from_address(ptr)
-        return np.frombuffer(buf, np.float32).reshape(kv_len, qd).copy()
+        buf = (C.c_float * (kv_len * kvd)).from_address(ptr)
+        return np.frombuffer(buf, np.float32).reshape(kv_len, kvd).copy()
 
     def generate(self):
         """Whole block loop; returns the generated ids."""

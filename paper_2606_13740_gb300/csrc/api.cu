@@ -32,7 +32,7 @@ size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
 int rup(int x, int m) { return (x + m - 1) / m * m; }
 
 struct Layout {
-    int qd, qkv_rows, gu_rows, d_rows, o_rows, head_rows, head_tiles, max_tok;
+    int qd, kvd, Hkv, qkv_rows, gu_rows, d_rows, o_rows, head_rows, head_tiles, max_tok;
     size_t off_w, per_layer, off_emb, off_head, off_kv, kv_half;
     size_t off_x, off_xn, off_q, off_attn, off_h, off_sq, off_theta;
     int n_sq;
@@ -49,7 +49,9 @@ Layout make_layout(const dllm_config& c) {
     Layout L{};
     const int d = c.d_model, H = c.n_heads, hd = c.head_dim, F = c.ffn, V = c.vocab;
     L.qd = H * hd;
-    L.qkv_rows = rup(3 * L.qd, 128);
+    L.Hkv = c.n_kv_heads > 0 ? c.n_kv_heads : H;  // grouped-query attention: fewer K/V heads
+    L.kvd = L.Hkv * hd;
+    L.qkv_rows = rup(L.qd + 2 * L.kvd, 128);
     L.o_rows = rup(d, 128);
     L.gu_rows = (F + 63) / 64 * 128;
     L.d_rows = rup(d, 128);
@@ -70,7 +72,7 @@ Layout make_layout(const dllm_config& c) {
     L.off_w = take(L.per_layer * 2 * c.n_layers);
     L.off_emb = take(static_cast<size_t>(V) * d * 2);
     L.off_head = take(static_cast<size_t>(L.head_rows) * d * 2);
-    L.kv_half = static_cast<size_t>(c.max_batch) * H * c.max_ctx * hd;
+    L.kv_half = static_cast<size_t>(c.max_batch) * L.Hkv * c.max_ctx * hd;
     L.off_kv = take(L.kv_half * 2 * 2 * c.n_layers);
     const size_t T = L.max_tok;
     L.off_x = take(T * d * 4);
@@ -107,10 +109,10 @@ Layout make_layout(const dllm_config& c) {
     L.off_outs = take(static_cast<size_t>(c.max_batch) * 32);
     L.off_status = take(16);
     // sparse cache refresh: tracked positions and merge flags [B][R], side K/V
-    // [L][2][B][H][R][hd] (R <= DLLM_MAX_SCR_ROWS)
+    // [L][2][B][Hkv][R][hd] (R <= DLLM_MAX_SCR_ROWS)
     L.off_trk = take(static_cast<size_t>(c.max_batch) * DLLM_MAX_SCR_ROWS * 4);
     L.off_smerge = take(static_cast<size_t>(c.max_batch) * DLLM_MAX_SCR_ROWS * 4);
-    L.off_side = take(static_cast<size_t>(c.n_layers) * 2 * c.max_batch * L.qd * DLLM_MAX_SCR_ROWS * 2);
+    L.off_side = take(static_cast<size_t>(c.n_layers) * 2 * c.max_batch * L.kvd * DLLM_MAX_SCR_ROWS * 2);
     // selective logits skipping: the compacted LM-head operand (bf16 rows, RMSNorm statistics,
     // current ids), the row map and the row count
     L.off_xc = take(T * d * 2);
@@ -127,6 +129,8 @@ const char* check_cfg(const dllm_config& c) {
     if (c.head_dim != 64 && c.head_dim != 128) return "head_dim must be 64 or 128";
     if (c.d_model % 128 || (c.n_heads * c.head_dim) % 128)
         return "d_model and n_heads*head_dim must be multiples of 128";
+    if (c.n_kv_heads < 0 || (c.n_kv_heads > 0 && (c.n_heads % c.n_kv_heads || (c.n_kv_heads * c.head_dim) % 128)))
+        return "n_kv_heads must divide n_heads, with n_kv_heads*head_dim a multiple of 128";
     if (c.ffn % 8 || c.vocab % 8) return "ffn and vocab must be multiples of 8";
     if (c.mask_id < 0 || c.mask_id >= c.vocab) return "mask_id out of range";
     if (c.max_batch < 1 || c.max_ctx < 1 || c.max_window < 1 || c.block_len < 1) return "bad capacities";
@@ -314,6 +318,7 @@ static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0, bool sls 
     ep.R = R;
     ep.trk = ctx->trk;
     ep.H = c.n_heads;
+    ep.Hkv = L.Hkv;
     ep.hd = c.head_dim;
     ep.cap = c.max_ctx;
     ep.q = ctx->q;
@@ -339,8 +344,8 @@ static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0, bool sls 
         EpiArgs e = ep;
         e.kc = ctx->kv + static_cast<size_t>(2 * l) * L.kv_half;
         e.vc = ctx->kv + static_cast<size_t>(2 * l + 1) * L.kv_half;
-        e.kside = ctx->scr_side + static_cast<size_t>(2 * l) * B * qd * R;  // [L][2][B][H][R][hd]
-        e.vside = e.kside + static_cast<size_t>(B) * qd * R;
+        e.kside = ctx->scr_side + static_cast<size_t>(2 * l) * B * L.kvd * R;  // [L][2][B][Hkv][R][hd]
+        e.vside = e.kside + static_cast<size_t>(B) * L.kvd * R;
         return e;
     };
     // phase slot i of a chain uses scratch slot i; consecutive chains are ordered by the stream
@@ -381,8 +386,8 @@ static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0, bool sls 
     }
     for (int l = 0; l < c.n_layers; ++l) {
         const EpiArgs el = qkv_args(l);
-        CK(launch_attention(ctx->q, el.kc, el.vc, ctx->seq_kv, ctx->attn, B, T, c.n_heads, c.head_dim, c.max_ctx, ap, s,
-                            true, next_trace(ctx), ctx->status));
+        CK(launch_attention(ctx->q, el.kc, el.vc, ctx->seq_kv, ctx->attn, B, T, c.n_heads, L.Hkv, c.head_dim, c.max_ctx,
+                            ap, s, true, next_trace(ctx), ctx->status));
         mark(ctx, DLLM_K_ATTN);
         // output projection (+ residual) -> gate/up (+ SwiGLU) -> down (+ residual) -> next QKV or LM head
         ChainArgs ca{};
@@ -468,7 +473,7 @@ static int step_kernels(dllm_ctx* ctx, int T) {
     mark(ctx, DLLM_K_COMMIT);
     if (ce == cudaSuccess && R > 0) {  // the refreshed K/V merged at the step boundary
         ce = launch_scr_merge(ctx->scr_side, ctx->kv, ctx->trk, ctx->scr_merge, ctx->cfg.n_layers, ctx->B,
-                              ctx->cfg.max_batch, ctx->cfg.n_heads, ctx->cfg.head_dim, ctx->cfg.max_ctx, R,
+                              ctx->cfg.max_batch, ctx->L.Hkv, ctx->cfg.head_dim, ctx->cfg.max_ctx, R,
                               ctx->stream);
         mark(ctx, DLLM_K_COMMIT);
     }
@@ -607,17 +612,22 @@ int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void*
     const uint64_t seed = c.weight_seed;
     const int hd = c.head_dim;
     // (the embedding is gathered by rows: row-major; the projections are streamed: tile-major)
-    cudaError_t ie = launch_init_weight(ctx->emb, 0, c.vocab, d, c.vocab, seed, 1, qd, hd, false, s);
-    if (ie == cudaSuccess) ie = launch_init_weight(ctx->head, 0, L.head_rows, d, c.vocab, seed, 2, qd, hd, true, s);
+    const int kvd = L.kvd;
+    cudaError_t ie = launch_init_weight(ctx->emb, 0, c.vocab, d, c.vocab, seed, 1, qd, kvd, hd, false, s);
+    if (ie == cudaSuccess)
+        ie = launch_init_weight(ctx->head, 0, L.head_rows, d, c.vocab, seed, 2, qd, kvd, hd, true, s);
     ctx->wl.resize(c.n_layers);
     for (int l = 0; l < c.n_layers && ie == cudaSuccess; ++l) {
         __nv_bfloat16* w = reinterpret_cast<__nv_bfloat16*>(A + L.off_w) + static_cast<size_t>(l) * L.per_layer;
         ctx->wl[l] = w;
         const uint64_t t0 = 16 + 8ull * l;
-        ie = launch_init_weight(w + L.w_qkv, 1, L.qkv_rows, d, qd, seed, t0 + 0, qd, hd, true, s);
-        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_o, 0, L.o_rows, qd, d, seed, t0 + 3, qd, hd, true, s);
-        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_gu, 2, L.gu_rows, d, F, seed, t0 + 4, qd, hd, true, s);
-        if (ie == cudaSuccess) ie = launch_init_weight(w + L.w_d, 0, L.d_rows, F, d, seed, t0 + 6, qd, hd, true, s);
+        ie = launch_init_weight(w + L.w_qkv, 1, L.qkv_rows, d, qd, seed, t0 + 0, qd, kvd, hd, true, s);
+        if (ie == cudaSuccess)
+            ie = launch_init_weight(w + L.w_o, 0, L.o_rows, qd, d, seed, t0 + 3, qd, kvd, hd, true, s);
+        if (ie == cudaSuccess)
+            ie = launch_init_weight(w + L.w_gu, 2, L.gu_rows, d, F, seed, t0 + 4, qd, kvd, hd, true, s);
+        if (ie == cudaSuccess)
+            ie = launch_init_weight(w + L.w_d, 0, L.d_rows, F, d, seed, t0 + 6, qd, kvd, hd, true, s);
     }
     // RoPE frequencies base^(-2j/hd), in double on the host
     std::vector<float> th(c.head_dim / 2);
@@ -717,7 +727,7 @@ static int start_request(dllm_ctx* ctx, const dllm_sched* sched, int batch, int 
     if (P_random) {
         for (int l = 0; l < c.n_layers; ++l)
             for (int w = 0; w < 2; ++w)
-                CK(launch_init_kv_random(ctx->kv + static_cast<size_t>(2 * l + w) * ctx->L.kv_half, batch, c.n_heads,
+                CK(launch_init_kv_random(ctx->kv + static_cast<size_t>(2 * l + w) * ctx->L.kv_half, batch, ctx->L.Hkv,
                                          c.head_dim, c.max_ctx, Lp, l, w, c.n_layers, kv_seed, ctx->stream));
         ctx->kv_len = Lp;
         CK(launch_set_kv_len(ctx->seq_kv, batch, Lp, ctx->stream));
@@ -1133,7 +1143,7 @@ int dllm_get_weight(dllm_ctx* ctx, int layer, int which, uint16_t* out, size_t n
         return fail(ctx, DLLM_EINVAL, "bad tensor");
     }
     // a projection: copy its tile-major matrix, then gather the logical rows
-    const int rows = layer < 0 ? c.vocab : (which <= 2) ? qd : (which == 3 || which == 6) ? d : F;
+    const int rows = layer < 0 ? c.vocab : (which == 0) ? qd : (which <= 2) ? L.kvd : (which == 3 || which == 6) ? d : F;
     const int cols = layer < 0 ? d : (which == 3) ? qd : (which == 6) ? F : d;
     if (n_elems < static_cast<size_t>(rows) * cols) return fail(ctx, DLLM_EINVAL, "buffer too small");
     const __nv_bfloat16* src;
@@ -1156,7 +1166,7 @@ int dllm_get_weight(dllm_ctx* ctx, int layer, int which, uint16_t* out, size_t n
         int pr = r;
         if (layer >= 0 && which <= 2) {  // q/k/v rows are interleaved inside each head
             const int hh = r / hd, i = r % hd;
-            pr = which * qd + hh * hd + 2 * (i % half) + i / half;
+            pr = (which == 0 ? 0 : qd + (which - 1) * L.kvd) + hh * hd + 2 * (i % half) + i / half;
         } else if (layer >= 0 && (which == 4 || which == 5)) {  // gate/up rows alternate in each tile
             pr = (r / 64) * 128 + 2 * (r % 64) + (which == 5 ? 1 : 0);
         }
@@ -1172,7 +1182,7 @@ int dllm_get_kv(dllm_ctx* ctx, int layer, int which, int seq, int p0, int n, flo
     if (!out || layer < 0 || layer >= c.n_layers || which < 0 || which > 1 || seq < 0 || seq >= c.max_batch || p0 < 0 ||
         n < 0 || p0 + n > c.max_ctx)
         return fail(ctx, DLLM_EINVAL, "bad KV slice");
-    const int H = c.n_heads, hd = c.head_dim, qd = H * hd;
+    const int H = ctx->L.Hkv, hd = c.head_dim, qd = H * hd;  // the cache's K/V heads
     std::vector<uint16_t> buf(static_cast<size_t>(H) * n * hd);
     const __nv_bfloat16* base = ctx->kv + static_cast<size_t>(2 * layer + which) * ctx->L.kv_half;
     for (int h = 0; h < H; ++h)

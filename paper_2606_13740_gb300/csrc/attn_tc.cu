@@ -97,14 +97,15 @@ __device__ __forceinline__ unsigned smid_tc() {
 
 struct TcMaps {
     CUtensorMap q;  // [B*H*T][128]: box 64 x 128 rows
-    CUtensorMap k;  // [B*H*cap][128]: box 64 x 64 keys
+    CUtensorMap k;  // [B*Hkv*cap][128]: box 64 x 64 keys (Hkv: the cache's K/V heads)
     CUtensorMap v;
 };
 
 template <int NB>
 __global__ void __launch_bounds__(kTcThreads, 1)
     k_attn_tc(const __grid_constant__ TcMaps maps, const int* __restrict__ seq_kv, __nv_bfloat16* __restrict__ out,
-              int T, int H, int cap, int qtiles, int csize, int qx, int* status, unsigned long long* trace) {
+              int T, int H, int Hkv, int cap, int qtiles, int csize, int qx, int* status,
+              unsigned long long* trace) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sQ = smem;                       // 32 KB
@@ -174,7 +175,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             mbar_arrive_expect_tx(&qbar, kTcQBytes);
             tma_load_2d(sQ, &maps.q, 0, qrow, &qbar, pol_q);
             tma_load_2d(sQ + kTcQBytes / 2, &maps.q, 64, qrow, &qbar, pol_q);
-            const int krow0 = (b * H + h) * cap + kbeg;
+            const int krow0 = (b * Hkv + h / (H / Hkv)) * cap + kbeg;  // K/V head of query head h
             int kiss = 0, viss = 0;  // sub-blocks whose K, V copies were issued
             for (int j = 0; j < nsub && !s_abort; ++j) {
                 const int st = j % NB;
@@ -443,10 +444,10 @@ size_t tc_smem() {
 
 template <int NB>
 cudaError_t tc_go(cudaLaunchConfig_t& cfg, const TcMaps& maps, const int* seq_kv, __nv_bfloat16* out, int T, int H,
-                  int cap, const AttnPlan& a, int* status, unsigned long long* trace) {
+                  int Hkv, int cap, const AttnPlan& a, int* status, unsigned long long* trace) {
     cfg.blockDim = dim3(kTcThreads);
     cfg.dynamicSmemBytes = tc_smem<NB>();
-    return cudaLaunchKernelEx(&cfg, k_attn_tc<NB>, maps, seq_kv, out, T, H, cap, a.qtiles, a.csize, a.qx, status,
+    return cudaLaunchKernelEx(&cfg, k_attn_tc<NB>, maps, seq_kv, out, T, H, Hkv, cap, a.qtiles, a.csize, a.qx, status,
                               trace);
 }
 
@@ -478,14 +479,15 @@ AttnPlan attn_plan_tc(int B, int T, int H, int max_keys, int sms) {
 }
 
 cudaError_t launch_attention_tc(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
-                                const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int cap,
+                                const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int Hkv, int cap,
                                 const AttnPlan& a, cudaStream_t st, bool pdl, unsigned long long* trace,
                                 int* status) {
-    if (a.csize < 1 || a.csize > kTcMaxCluster || (a.nb != 1 && a.nb != 2)) return cudaErrorInvalidValue;
+    if (a.csize < 1 || a.csize > kTcMaxCluster || (a.nb != 1 && a.nb != 2) || Hkv < 1 || H % Hkv)
+        return cudaErrorInvalidValue;
     TcMaps maps;
     if (!make_tmap_bf16(&maps.q, q, static_cast<uint64_t>(B) * H * T, 128, kTcRows) ||
-        !make_tmap_bf16(&maps.k, kc, static_cast<uint64_t>(B) * H * cap, 128, kTcKeys) ||
-        !make_tmap_bf16(&maps.v, vc, static_cast<uint64_t>(B) * H * cap, 128, kTcKeys))
+        !make_tmap_bf16(&maps.k, kc, static_cast<uint64_t>(B) * Hkv * cap, 128, kTcKeys) ||
+        !make_tmap_bf16(&maps.v, vc, static_cast<uint64_t>(B) * Hkv * cap, 128, kTcKeys))
         return cudaErrorInvalidValue;
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3(a.csize, H, B * a.qtiles);
@@ -504,8 +506,8 @@ cudaError_t launch_attention_tc(const __nv_bfloat16* q, const __nv_bfloat16* kc,
     }
     cfg.attrs = at;
     cfg.numAttrs = n;
-    return a.nb == 2 ? tc_go<2>(cfg, maps, seq_kv, out, T, H, cap, a, status, trace)
-                     : tc_go<1>(cfg, maps, seq_kv, out, T, H, cap, a, status, trace);
+    return a.nb == 2 ? tc_go<2>(cfg, maps, seq_kv, out, T, H, Hkv, cap, a, status, trace)
+                     : tc_go<1>(cfg, maps, seq_kv, out, T, H, Hkv, cap, a, status, trace);
 }
 
 }  // namespace dllm

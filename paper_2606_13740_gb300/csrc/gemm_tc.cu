@@ -194,9 +194,11 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
     float cn = 1.0f, sn = 0.0f, cd = 1.0f, sd = 0.0f, theta = 0.0f;
     __nv_bfloat16* qkv_dst = nullptr;
     if constexpr (EPI == EPI_QKV) {
-        const int qd = ep.H * ep.hd;
-        part = row / qd;  // the same for the whole warp (qd is a multiple of 128)
-        const int f = row - part * qd;
+        // q rows [0, qd), k rows [qd, qd + kvd), v rows [qd + kvd, qd + 2 kvd): the same part for
+        // the whole warp (qd and kvd are multiples of 128)
+        const int qd = ep.H * ep.hd, kvd = ep.Hkv * ep.hd;
+        part = row < qd ? 0 : (row < qd + kvd ? 1 : 2);
+        const int f = row - (part == 0 ? 0 : qd + (part - 1) * kvd);
         hh = f / ep.hd;
         pp = f - hh * ep.hd;
         fi = (pp >> 1) + (pp & 1) * (ep.hd >> 1);
@@ -378,7 +380,9 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
             const int ts = col - b * ep.T;
             const bool tracked = ts >= ep.Tw;  // sparse cache refresh: K/V to the side buffers
             const int pos = tracked ? ep.trk[b * ep.R + ts - ep.Tw] : sm.kvs[b] + ts;
-            const int head = (mt * kBM - part * ep.H * ep.hd + f0) / ep.hd;
+            const int base = part == 0 ? 0 : ep.H * ep.hd + (part - 1) * ep.Hkv * ep.hd;  // the part's first row
+            const int head = (mt * kBM - base + f0) / ep.hd;
+            const int heads = part == 0 ? ep.H : ep.Hkv;  // q: query heads; K/V: the cache's heads
             const int fi0 = f0 % ep.hd;
             if (tracked && part > 0) {
                 if (pos >= 0) {
@@ -386,13 +390,13 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                         reinterpret_cast<const __nv_bfloat16*>(sm.stg) + tok * kBM + f0);
                     __nv_bfloat16* side = part == 1 ? ep.kside : ep.vside;
                     uint4* dst = reinterpret_cast<uint4*>(
-                        side + ((static_cast<size_t>(b) * ep.H + head) * ep.R + (ts - ep.Tw)) * ep.hd + fi0);
+                        side + ((static_cast<size_t>(b) * heads + head) * ep.R + (ts - ep.Tw)) * ep.hd + fi0);
 #pragma unroll
                     for (int i = 0; i < 2; ++i) dst[i] = src[i];
                 }
             } else if (tracked || (pos >= 0 && pos < ep.cap)) {
                 const size_t plane = part == 0 ? static_cast<size_t>(ep.T) : static_cast<size_t>(ep.cap);
-                const size_t r = (static_cast<size_t>(b) * ep.H + head) * plane + (part == 0 ? ts : pos);
+                const size_t r = (static_cast<size_t>(b) * heads + head) * plane + (part == 0 ? ts : pos);
                 const uint4* src = reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(sm.stg) +
                                                                   tok * kBM + f0);
                 uint4* dst = reinterpret_cast<uint4*>(qkv_dst + r * ep.hd + fi0);
@@ -495,7 +499,7 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
 // TMEM accumulators and their barriers are shared by all phases; a running iteration counter
 // gives every stage its use parity.
 constexpr int kChainThreads = 64 + 32 + 32 * kEpiWarps;
-constexpr int kMaxDepTiles = 256;  // the operand producer keeps a readiness bit per producing tile: 8 per lane
+constexpr int kMaxDepTiles = 1024;  // the operand producer keeps a readiness bit per producing tile: 32 per lane
 
 struct ChainEpiState {
     int acc;

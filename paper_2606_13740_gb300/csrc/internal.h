@@ -45,13 +45,15 @@ struct EpiArgs {
     const float* sq_in;
     int n_sq, norm_dim;
     float eps;
-    // EPI_QKV: rows [0,qd) q, [qd,2qd) k, [2qd,3qd) v; rotate-half RoPE on q, k.  Inside
-    // each head the rows are interleaved: row 2j is feature j, row 2j+1 feature j + hd/2
+    // EPI_QKV: rows [0,qd) q, [qd,qd+kvd) k, [qd+kvd,qd+2kvd) v (qd = H*hd, kvd = Hkv*hd: under
+    // grouped-query attention fewer K/V heads than query heads); rotate-half RoPE on q, k.
+    // Inside each head the rows are interleaved: row 2j is feature j, row 2j+1 feature j + hd/2
     __nv_bfloat16* q;    // [B][H][T][hd]
-    __nv_bfloat16* kc;   // layer's K cache base: [B][H][cap][hd]
+    __nv_bfloat16* kc;   // layer's K cache base: [B][Hkv][cap][hd]
     __nv_bfloat16* vc;
     const int* seq_kv;   // per-sequence first window position (kv_len)
     int T, H, hd, cap;
+    int Hkv;             // K/V heads (a multiple of 128 / hd rows each part: Hkv * hd % 128 == 0)
     int n_seq;           // sequences (B), <= 256
     const float* theta;  // [hd/2]: rotation of feature pair j at position p is p * theta[j]
     // EPI_SWIGLU: tile k row 2f is gate feature 64k+f, row 2f+1 the matching up row
@@ -59,7 +61,7 @@ struct EpiArgs {
     int F;
     // EPI_QKV with sparse cache refresh: of a sequence's T rows the first Tw are the window,
     // row Tw + r of sequence b is the prefix position trk[b R + r] (< 0: an unused row, no K/V
-    // written), whose K and V go to kside / vside [B][H][R][hd] instead of the cache
+    // written), whose K and V go to kside / vside [B][Hkv][R][hd] instead of the cache
     int Tw, R;
     const int* trk;
     __nv_bfloat16* kside;
@@ -189,7 +191,7 @@ inline cudaError_t launch_k(void (*k)(KArgs...), dim3 grid, dim3 block, size_t s
 // Seeded weights (rows_phys x cols, see k_init_weight for the row orders), stored tile-major
 // (tiled_index; rows_phys a multiple of 128) when `tiled`, else row-major.
 cudaError_t launch_init_weight(__nv_bfloat16* dst, int mode, int rows_phys, int cols, int logical_rows,
-                               uint64_t seed, uint64_t tid0, int qd, int hd, bool tiled, cudaStream_t st);
+                               uint64_t seed, uint64_t tid0, int qd, int kvd, int hd, bool tiled, cudaStream_t st);
 cudaError_t launch_init_kv_random(__nv_bfloat16* cache, int B, int H, int hd, int cap, int P, int layer,
                                   int which, int L, uint64_t seed, cudaStream_t st);
 // x = embedding rows of the window's ids (fp32), xb = bf16(x), sq[d/128][N] = per-128-feature
@@ -202,7 +204,7 @@ cudaError_t launch_embed(const int* tok, int tok_ld, const int* seq_kv, const __
 // Sparse cache refresh: trk[b R + r] = the r-th COMMITTED position of sequence b below
 // seq_kv[b] (ascending), -1 past the last (state rows st + b ld); merge: the K/V rows of the
 // refreshed positions (merge[b R + r] != 0) from the side buffers [L][2][B][H][R][hd] into the
-// cache [L][2][kv_B][H][cap][hd].
+// cache [L][2][kv_B][H][cap][hd] (H: the K/V heads).
 cudaError_t launch_scr_select(const uint8_t* st, int ld, const int* seq_kv, int* trk, int B, int R,
                               cudaStream_t stream);
 cudaError_t launch_scr_merge(const __nv_bfloat16* side, __nv_bfloat16* cache, const int* trk, const int* merge, int L,
@@ -225,12 +227,13 @@ constexpr int kTcMinKeys = 1024;
 AttnPlan attn_plan(int B, int T, int H, int hd, int max_keys, int sms);
 AttnPlan attn_plan_tc(int B, int T, int H, int max_keys, int sms);
 cudaError_t attn_tc_init_attrs();
+// Grouped-query attention: query head h reads K/V head h / (H / Hkv) of the cache [B][Hkv][cap][hd].
 cudaError_t launch_attention_tc(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
-                                const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int cap,
+                                const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int Hkv, int cap,
                                 const AttnPlan& a, cudaStream_t st, bool pdl, unsigned long long* trace,
                                 int* status);
 cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
-                             const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int hd, int cap,
+                             const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int Hkv, int hd, int cap,
                              const AttnPlan& a, cudaStream_t st, bool pdl = true,
                              unsigned long long* trace = nullptr, int* status = nullptr);
 cudaError_t launch_lmhead_reduce(const float* lm_part, const float* zcur, const int* cur_tok, int m_tiles,

@@ -33,15 +33,16 @@ __device__ __forceinline__ float gen_value(uint64_t key, uint64_t i, double sigm
 
 // mode 0: plain (physical row = logical row of tensor tid0, zero rows past
 //         logical_rows);
-// mode 1: fused QKV: rows [0,qd) tensor tid0 (q), [qd,2qd) tid0+1 (k), [2qd,3qd) tid0+2 (v);
-//         inside each head of hd rows, physical row 2j holds feature j and row 2j+1 feature
-//         j + hd/2 (the rotate-half RoPE pair sits in adjacent TMEM lanes);
+// mode 1: fused QKV: rows [0,qd) tensor tid0 (q), [qd,qd+kvd) tid0+1 (k), [qd+kvd,qd+2kvd)
+//         tid0+2 (v) (kvd = K/V heads x hd: fewer K/V heads than query heads under grouped-query
+//         attention); inside each head of hd rows, physical row 2j holds feature j and row 2j+1
+//         feature j + hd/2 (the rotate-half RoPE pair sits in adjacent TMEM lanes);
 // mode 2: fused gate/up: 128-row tile k, physical row 2f = gate row 64k+f (tensor tid0),
 //         row 2f+1 = up row 64k+f (tensor tid0+1); zero past logical_rows.
 // Storage: row-major, or tile-major (tiled_index) when tiled; the loop walks the destination in
 // storage order.
 __global__ void k_init_weight(__nv_bfloat16* dst, int mode, int rows, int cols, int logical_rows, uint64_t seed,
-                              uint64_t tid0, int qd, int hd, int tiled) {
+                              uint64_t tid0, int qd, int kvd, int hd, int tiled) {
     const int kb = (cols + 63) / 64;
     const size_t n = tiled ? static_cast<size_t>(rows) * kb * 64 : static_cast<size_t>(rows) * cols;
     for (size_t e = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; e < n;
@@ -64,11 +65,12 @@ __global__ void k_init_weight(__nv_bfloat16* dst, int mode, int rows, int cols, 
         uint64_t tid = tid0;
         int lr = r;
         if (mode == 1) {
-            const int part = r / qd, f = r % qd;
+            const int part = r < qd ? 0 : (r < qd + kvd ? 1 : (r < qd + 2 * kvd ? 2 : 3));
+            const int f = r - (part == 0 ? 0 : qd + (part - 1) * kvd);
             const int hh = f / hd, pp = f % hd;
             tid = tid0 + part;
             lr = hh * hd + (pp >> 1) + (pp & 1) * (hd >> 1);
-            if (part > 2) lr = logical_rows;  // padding rows
+            if (part > 2 || lr >= (part == 0 ? qd : kvd)) lr = logical_rows;  // padding rows
         } else if (mode == 2) {
             const int tile = r >> 7, w = r & 127;
             tid = tid0 + (w & 1);
@@ -84,17 +86,17 @@ __global__ void k_init_weight(__nv_bfloat16* dst, int mode, int rows, int cols, 
 }
 
 cudaError_t launch_init_weight(__nv_bfloat16* dst, int mode, int rows_phys, int cols, int logical_rows,
-                               uint64_t seed, uint64_t tid0, int qd, int hd, bool tiled, cudaStream_t st) {
+                               uint64_t seed, uint64_t tid0, int qd, int kvd, int hd, bool tiled, cudaStream_t st) {
     if (tiled && (rows_phys & 127)) return cudaErrorInvalidValue;
     size_t n = static_cast<size_t>(rows_phys) * (tiled ? (cols + 63) / 64 * 64 : cols);
     int blocks = static_cast<int>((n + 255) / 256 < 65536 ? (n + 255) / 256 : 65536);
-    k_init_weight<<<blocks, 256, 0, st>>>(dst, mode, rows_phys, cols, logical_rows, seed, tid0, qd, hd,
+    k_init_weight<<<blocks, 256, 0, st>>>(dst, mode, rows_phys, cols, logical_rows, seed, tid0, qd, kvd, hd,
                                           tiled ? 1 : 0);
     return cudaGetLastError();
 }
 
-// Synthetic prefix KV: cache[b][h][pos][i] for pos < P is element pos*qd + h*hd + i
-// of tensor 2^32 + ((b*L + layer)*2 + which), sigma 1.
+// Synthetic prefix KV: cache[b][h][pos][i] for pos < P is element pos*(H*hd) + h*hd + i
+// of tensor 2^32 + ((b*L + layer)*2 + which), sigma 1 (H: the cache's K/V heads).
 __global__ void k_init_kv(__nv_bfloat16* cache, int B, int H, int hd, int cap, int P, int layer, int which, int L,
                           uint64_t seed) {
     const size_t n = static_cast<size_t>(B) * H * P * hd;
@@ -226,8 +228,8 @@ __global__ void __launch_bounds__(PR * NW * 32) k_attn(const __nv_bfloat16* __re
                                                        const __nv_bfloat16* __restrict__ kc,
                                                        const __nv_bfloat16* __restrict__ vc,
                                                        const int* __restrict__ seq_kv, __nv_bfloat16* __restrict__ out,
-                                                       int T, int H, int cap, int qtiles, int csize, int qx,
-                                                       unsigned long long* trace) {
+                                                       int T, int H, int Hkv, int cap, int qtiles, int csize,
+                                                       int qx, unsigned long long* trace) {
     constexpr int AQ = NW * 16;  // query rows per CTA
     constexpr int NT = NW * 32;  // threads of one warp group
     constexpr int PART = (AQ + 2 * NB * kAK) * HD * 2;  // one group's Q, K, V tiles
@@ -264,8 +266,10 @@ __global__ void __launch_bounds__(PR * NW * 32) k_attn(const __nv_bfloat16* __re
     const int g = lane >> 2, c4 = lane & 3;
 
     const __nv_bfloat16* qbase = q + ((static_cast<size_t>(b) * H + h) * T + q0) * HD;
-    const __nv_bfloat16* kbase = kc + (static_cast<size_t>(b) * H + h) * cap * HD;
-    const __nv_bfloat16* vbase = vc + (static_cast<size_t>(b) * H + h) * cap * HD;
+    // grouped-query attention: query head h reads K/V head h / (H / Hkv)
+    const int hk = h / (H / Hkv);
+    const __nv_bfloat16* kbase = kc + (static_cast<size_t>(b) * Hkv + hk) * cap * HD;
+    const __nv_bfloat16* vbase = vc + (static_cast<size_t>(b) * Hkv + hk) * cap * HD;
 
     auto sync = [grp]() {
         if constexpr (PR == 1) __syncthreads();
@@ -471,20 +475,21 @@ AttnPlan attn_plan(int B, int T, int H, int hd, int max_keys, int sms) {
 
 template <int HD, int NW, int NB, int PR>
 static cudaError_t attn_go(cudaLaunchConfig_t& cfg, const __nv_bfloat16* q, const __nv_bfloat16* kc,
-                           const __nv_bfloat16* vc, const int* seq_kv, __nv_bfloat16* out, int T, int H, int cap,
-                           const AttnPlan& a, unsigned long long* trace) {
+                           const __nv_bfloat16* vc, const int* seq_kv, __nv_bfloat16* out, int T, int H, int Hkv,
+                           int cap, const AttnPlan& a, unsigned long long* trace) {
     cfg.blockDim = dim3(PR * NW * 32);
     cfg.dynamicSmemBytes = attn_smem(NW, NB, PR, HD);
-    return cudaLaunchKernelEx(&cfg, k_attn<HD, NW, NB, PR>, q, kc, vc, seq_kv, out, T, H, cap, a.qtiles, a.csize,
+    return cudaLaunchKernelEx(&cfg, k_attn<HD, NW, NB, PR>, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a.qtiles, a.csize,
                               a.qx, trace);
 }
 
 cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
-                             const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int hd, int cap,
+                             const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int Hkv, int hd, int cap,
                              const AttnPlan& a, cudaStream_t st, bool pdl, unsigned long long* trace, int* status) {
+    if (Hkv < 1 || H % Hkv) return cudaErrorInvalidValue;
     if (a.tc) {
         if (hd != 128) return cudaErrorInvalidValue;
-        return launch_attention_tc(q, kc, vc, seq_kv, out, B, T, H, cap, a, st, pdl, trace, status);
+        return launch_attention_tc(q, kc, vc, seq_kv, out, B, T, H, Hkv, cap, a, st, pdl, trace, status);
     }
     if (a.csize < 1 || a.csize > kMaxCluster || (a.nw != 2 && a.nw != 4) || (a.nb != 1 && a.nb != 2) ||
         (a.pairs != 1 && a.pairs != 2) || (a.pairs == 2 && (a.nw != 2 || a.nb != 1)) || (hd != 64 && hd != 128))
@@ -507,18 +512,18 @@ cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, co
     cfg.attrs = at;
     cfg.numAttrs = n;
     if (a.pairs == 2)
-        return hd == 128 ? attn_go<128, 2, 1, 2>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace)
-                         : attn_go<64, 2, 1, 2>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        return hd == 128 ? attn_go<128, 2, 1, 2>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace)
+                         : attn_go<64, 2, 1, 2>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
     const int key = (hd == 128 ? 4 : 0) + (a.nw == 4 ? 2 : 0) + (a.nb == 2 ? 1 : 0);
     switch (key) {
-        case 0: return attn_go<64, 2, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
-        case 1: return attn_go<64, 2, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
-        case 2: return attn_go<64, 4, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
-        case 3: return attn_go<64, 4, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
-        case 4: return attn_go<128, 2, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
-        case 5: return attn_go<128, 2, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
-        case 6: return attn_go<128, 4, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
-        default: return attn_go<128, 4, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, cap, a, trace);
+        case 0: return attn_go<64, 2, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
+        case 1: return attn_go<64, 2, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
+        case 2: return attn_go<64, 4, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
+        case 3: return attn_go<64, 4, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
+        case 4: return attn_go<128, 2, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
+        case 5: return attn_go<128, 2, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
+        case 6: return attn_go<128, 4, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
+        default: return attn_go<128, 4, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
     }
 }
 

@@ -149,9 +149,9 @@ int dllm_op_gemm_trace(const void* W, const void* X, float* D, int M, int N, int
 }
 
 int dllm_op_attention(const void* q, const void* kc, const void* vc, const int32_t* kv_len, void* out, int B, int T,
-                      int H, int hd, int cap, int max_kv_len, void* stream) {
-    if (!q || !kc || !vc || !kv_len || !out || B < 1 || T < 1 || H < 1 || (hd != 64 && hd != 128) ||
-        max_kv_len < 0 || max_kv_len + T > cap)
+                      int H, int Hkv, int hd, int cap, int max_kv_len, void* stream) {
+    if (!q || !kc || !vc || !kv_len || !out || B < 1 || T < 1 || H < 1 || Hkv < 1 || H % Hkv ||
+        (hd != 64 && hd != 128) || max_kv_len < 0 || max_kv_len + T > cap)
         return op_fail(DLLM_EINVAL, "bad attention arguments");
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     int sms = sm_count();
@@ -160,7 +160,7 @@ int dllm_op_attention(const void* q, const void* kc, const void* vc, const int32
     AttnPlan a = attn_plan(B, T, H, hd, max_kv_len + T, sms);
     cudaError_t e = launch_attention(static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(kc),
                                      static_cast<const __nv_bfloat16*>(vc), kv_len, static_cast<__nv_bfloat16*>(out),
-                                     B, T, H, hd, cap, a, st, false);
+                                     B, T, H, Hkv, hd, cap, a, st, false);
     if (e != cudaSuccess) return op_fail(DLLM_ECUDA, "attention launch: %s", cudaGetErrorString(e));
     return finish(st, nullptr);
 }

@@ -32,7 +32,7 @@ class dllm_config(C.Structure):
     _fields_ = [("n_layers", C.c_int), ("d_model", C.c_int), ("n_heads", C.c_int), ("head_dim", C.c_int),
                 ("ffn", C.c_int), ("vocab", C.c_int), ("mask_id", C.c_int), ("rope_base", C.c_float),
                 ("rms_eps", C.c_float), ("max_batch", C.c_int), ("max_ctx", C.c_int), ("max_window", C.c_int),
-                ("block_len", C.c_int), ("weight_seed", C.c_uint64)]
+                ("block_len", C.c_int), ("weight_seed", C.c_uint64), ("n_kv_heads", C.c_int)]
 
 
 class dllm_sched(C.Structure):
@@ -85,7 +85,7 @@ SIGNATURES = {
     "dllm_op_gemm_noalloc": (_I, [_P, _P, _P, _I, _I, _I, _I, _P]),
     "dllm_op_gemm_trace": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P]),
     "dllm_op_gemm_timed": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P]),
-    "dllm_op_attention": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P]),
+    "dllm_op_attention": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
     "dllm_op_lmhead": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _P]),
     "dllm_op_commit": (_I, [_P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _I, _F, _F, _I, _I, _I, _I, _I, _I, _F, _P]),
 }
@@ -142,11 +142,16 @@ class Config:
     max_window: int = 128
     block_len: int = 32
     weight_seed: int = 0x11ADA8B
+    n_kv_heads: int = 0  # grouped-query attention: K/V heads (0 = n_heads)
+
+    @property
+    def kv_dim(self):
+        return (self.n_kv_heads or self.n_heads) * self.head_dim
 
     def c(self):
         return dllm_config(self.n_layers, self.d_model, self.n_heads, self.head_dim, self.ffn, self.vocab,
                            self.mask_id, self.rope_base, self.rms_eps, self.max_batch, self.max_ctx, self.max_window,
-                           self.block_len, self.weight_seed)
+                           self.block_len, self.weight_seed, self.n_kv_heads)
 
 
 @dataclass
@@ -293,7 +298,7 @@ class Context:
     def dllm_get_weight(self, layer, which):
         c = self.cfg
         qd = c.n_heads * c.head_dim
-        shapes = {0: (qd, c.d_model), 1: (qd, c.d_model), 2: (qd, c.d_model), 3: (c.d_model, qd),
+        shapes = {0: (qd, c.d_model), 1: (c.kv_dim, c.d_model), 2: (c.kv_dim, c.d_model), 3: (c.d_model, qd),
                   4: (c.ffn, c.d_model), 5: (c.ffn, c.d_model), 6: (c.d_model, c.ffn)}
         shape = (c.vocab, c.d_model) if layer < 0 else shapes[which]
         out = np.empty(shape, np.uint16)
@@ -301,8 +306,7 @@ class Context:
         return out
 
     def dllm_get_kv(self, layer, which, seq, p0, n):
-        qd = self.cfg.n_heads * self.cfg.head_dim
-        out = np.empty((n, qd), np.float32)
+        out = np.empty((n, self.cfg.kv_dim), np.float32)
         _check(lib().dllm_get_kv(self.h, layer, which, seq, p0, n, _p(out)), self.h)
         return out
 
@@ -391,12 +395,14 @@ def dllm_op_gemm_trace(W, X, M, N, K, reps, grid=0, stream=None):
     return ms.value, tr[:used.value]
 
 
-def dllm_op_attention(q, kc, vc, kv_len, B, T, H, hd, cap, max_kv_len, stream=None):
+def dllm_op_attention(q, kc, vc, kv_len, B, T, H, hd, cap, max_kv_len, stream=None, Hkv=None):
+    """q bf16 [B][H][T][hd], kc/vc bf16 [B][Hkv][cap][hd] (Hkv defaults to H); returns bf16 [B*T][H*hd]."""
     import torch
 
     out = torch.empty((B * T, H * hd), dtype=torch.bfloat16, device=q.device)
     _check(lib().dllm_op_attention(_p(q.data_ptr()), _p(kc.data_ptr()), _p(vc.data_ptr()), _p(kv_len.data_ptr()),
-                                   _p(out.data_ptr()), B, T, H, hd, cap, max_kv_len, _p(_stream_ptr(stream))))
+                                   _p(out.data_ptr()), B, T, H, H if Hkv is None else Hkv, hd, cap, max_kv_len,
+                                   _p(_stream_ptr(stream))))
     return out
 
 

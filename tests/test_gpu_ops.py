@@ -66,7 +66,7 @@ def test_gemm_llada_shapes_sampled(dev, M, N, K):
 def test_gemm_bounded_wait_times_out(dev):
     """A launch whose operand wait can never be satisfied (a flag nothing writes) gives up after
     its bounded wait, unwinds every role and reports DLLM_ETIMEOUT; the next launch is normal."""
-    from paper_2606_13740_gb300 import DllmError, dllm_op_gemm, dllm_op_gemm_timed
+    from paper_2606_13740_gb300.dllm import DllmError, dllm_op_gemm, dllm_op_gemm_timed
     M, N, K = 1024, 32, 1024
     rng = np.random.default_rng(5)
     W = _bf16(rng, (M, K), 0.05)
