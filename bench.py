@@ -10,6 +10,8 @@ commit).  Weights are random N(0, 0.02) drawn on the device; the data are
 synthetic.
 
 Other workloads (`--workload`, one JSON line each, same schema):
+  llada8b_step_b1_p512_t32_q4      the default step with the projections and the LM head in
+                                   the 4-bit block format of the paper's Q4_0 weights
   llada8b_step_b16_p4096_t64       batched serving step: 16 sequences, synthetic
                                    4096-position prefix KV each, 64-token window
                                    (current block + one speculative block), 32
@@ -82,8 +84,9 @@ GENERATIONS = {
         "adaptive lookahead from the window sweep's step latencies, allowance 0.2 (Sec. 3.2)"),
 }
 STEP_B16 = "llada8b_step_b16_p4096_t64"
+STEP_Q4 = "llada8b_step_b1_p512_t32_q4"
 SWEEP = "llada8b_window_sweep_b1_p512"
-ALL = [WORKLOAD["workload"], STEP_B16, SWEEP, *GENERATIONS]
+ALL = [WORKLOAD["workload"], STEP_Q4, STEP_B16, SWEEP, *GENERATIONS]
 
 
 def _peaks():
@@ -97,24 +100,28 @@ def _peaks():
         return 6800.0, 1900.0, 1700.0, "fallback"
 
 
-def _algorithmic_bytes(N):
-    """Bytes each kind of launch must move at minimum (weights once, activations once)."""
+def _algorithmic_bytes(N, wb=2.0):
+    """Bytes each kind of launch must move at minimum (weights once at wb bytes per weight,
+    activations once)."""
     d, qd, F, V = 4096, 4096, 12288, 126464
     return {
-        "qkv": 3 * qd * d * 2 + N * d * 2 + 3 * N * qd * 2,
-        "oproj": d * qd * 2 + N * qd * 2 + 2 * N * d * 4,
-        "gateup": 2 * F * d * 2 + N * d * 2 + N * F * 2,
-        "down": d * F * 2 + N * F * 2 + 2 * N * d * 4,
-        "head": V * d * 2 + N * d * 2 + (V // 128) * N * 12,
+        "qkv": 3 * qd * d * wb + N * d * 2 + 3 * N * qd * 2,
+        "oproj": d * qd * wb + N * qd * 2 + 2 * N * d * 4,
+        "gateup": 2 * F * d * wb + N * d * 2 + N * F * 2,
+        "down": d * F * wb + N * F * 2 + 2 * N * d * 4,
+        "head": V * d * wb + N * d * 2 + (V // 128) * N * 12,
     }
+
+
+Q4_BYTES = 0.5 + 2.0 / 32  # 4-bit code plus a bf16 scale per block of 32: 4.5 bits per weight
 
 
 def _attn_bytes(P, T_):
     return 2 * (P + T_) * 4096 * 2  # K and V rows of one layer (prefix + window), read once
 
 
-def _step_bytes(P, T_):
-    a = _algorithmic_bytes(T_)
+def _step_bytes(P, T_, wb=2.0):
+    a = _algorithmic_bytes(T_, wb)
     return 32 * (a["qkv"] + a["oproj"] + a["gateup"] + a["down"] + _attn_bytes(P, T_)) + a["head"]
 
 
@@ -210,7 +217,7 @@ class OracleSample:
     1/`head_div` of the vocabulary rows for `head_rows` of the window's rows, all scaled to the
     full step (32 layers, `batch` sequences, every row of the head)."""
 
-    def __init__(self, layers, head_div, P=LP, T_=T, batch=1, head_rows=None):
+    def __init__(self, layers, head_div, P=LP, T_=T, batch=1, head_rows=None, weight_bits=16):
         import numpy as np
         import oracle as O
 
@@ -218,10 +225,11 @@ class OracleSample:
         self.O = O
         self.layers, self.head_div, self.batch = layers, head_div, batch
         self.head_rows = T_ if head_rows is None else head_rows
-        self.lmodel = O.Model(O.OracleConfig(**dict(SHAPE, n_layers=layers)), gen_layers=layers, gen_head=False)
+        self.lmodel = O.Model(O.OracleConfig(**dict(SHAPE, n_layers=layers, weight_bits=weight_bits)),
+                              gen_layers=layers, gen_head=False)
         hv = SHAPE["vocab"] // head_div
-        self.hmodel = O.Model(O.OracleConfig(**dict(SHAPE, n_layers=1, vocab=hv, mask_id=hv - 1)), gen_layers=0,
-                              gen_head=True)
+        self.hmodel = O.Model(O.OracleConfig(**dict(SHAPE, n_layers=1, vocab=hv, mask_id=hv - 1,
+                                                    weight_bits=weight_bits)), gen_layers=0, gen_head=True)
         rng = np.random.default_rng(I.SEED_KV)
         self.pk = rng.standard_normal((layers, P, 4096), dtype=np.float32)
         self.pv = rng.standard_normal((layers, P, 4096), dtype=np.float32)
@@ -333,12 +341,13 @@ def _chain_roofline(prof, psteps, per_launch_units, unit, peak, peak_source, bou
             "avg_launch_ms": chain_ms}
 
 
-def run_step_b1(args, env):
+def run_step_b1(args, env, q4=False):
     import numpy as np
     torch, device, world, rank, pg = env["torch"], env["device"], env["world"], env["rank"], env["pg"]
     from paper_2606_13740_gb300 import COMMITTED, MASKED, Config, Context, Sched
 
-    cfg = Config(max_batch=1, max_ctx=LP + T, max_window=LP, **SHAPE)
+    cfg = Config(max_batch=1, max_ctx=LP + T, max_window=LP, weight_bits=4 if q4 else 16, **SHAPE)
+    wb = Q4_BYTES if q4 else 2.0
     ctx = Context(cfg)
     if args.no_pdl or args.full_smem:
         ctx.dllm_set_debug((4 if args.no_pdl else 0) | (8 if args.full_smem else 0))
@@ -398,27 +407,31 @@ def run_step_b1(args, env):
     n_pos = LP + T
 
     hbm, bf16, bf16_sus, peak_src = env["peaks"]
-    algo = _algorithmic_bytes(T)
+    algo = _algorithmic_bytes(T, wb)
     per_layer = algo["oproj"] + algo["gateup"] + algo["down"]
     chain_bytes = (31 * (per_layer + algo["qkv"]) + per_layer + algo["head"]) / 32  # average launch
     roof = _chain_roofline(prof, psteps, chain_bytes, "GB/s", hbm, peak_src, "hbm",
                            "k_chain (one layer: output, gate/up, down and next-QKV projections, "
-                           "436 MB of weights per launch)")
-    try:  # DRAM bytes of one layer-chain launch from an ncu capture of this exact source
-        with open(os.path.join(ROOT, "profiles", "chain_layer_traffic.json")) as f:
-            tr = json.load(f)
-        if tr.get("source_hash") == _kernel_hash():
-            roof["traffic"] = tr["dram_bytes_per_launch"]
-    except Exception:
-        pass
-    step_bytes = _step_bytes(LP, T)
+                           + ("123 MB of 4-bit weights per launch, expanded to bf16 in shared memory)"
+                              if q4 else "436 MB of weights per launch)"))
+    if not q4:
+        try:  # DRAM bytes of one layer-chain launch from an ncu capture of this exact source
+            with open(os.path.join(ROOT, "profiles", "chain_layer_traffic.json")) as f:
+                tr = json.load(f)
+            if tr.get("source_hash") == _kernel_hash():
+                roof["traffic"] = tr["dram_bytes_per_launch"]
+        except Exception:
+            pass
+    step_bytes = _step_bytes(LP, T, wb)
     step_ach = step_bytes / (ms_per_step * 1e-3) / 1e9
     gemm_ms = (prof["qkv"]["ms_total"] + prof["layer"]["ms_total"]) / max(1, psteps)
     gemm_bytes = 32 * (algo["qkv"] + algo["oproj"] + algo["gateup"] + algo["down"]) + algo["head"]
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": max(args.warmup, 3), "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": WORKLOAD,
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": dict(WORKLOAD, workload=STEP_Q4, weights="4-bit block format (Q4_0-style: 32 weights per "
+                       "bf16 scale, codes 0..15 for d*(q-8)), 4.5 bits per weight; bf16 arithmetic") if q4 else WORKLOAD,
         "parallelism": "replicas" if world > 1 else "single-gpu",
         "gen_tokens_per_s": value * WORKLOAD["commits_per_step"],
         "roofline": roof,
@@ -432,7 +445,8 @@ def run_step_b1(args, env):
         "clocks": tm.clocks,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = _cpu_baseline(OracleSample(4, 8), UNIT, lambda s: 1.0 / s)
+        line["cpu_baseline"] = _cpu_baseline(OracleSample(4, 8, weight_bits=4 if q4 else 16), UNIT,
+                                             lambda s: 1.0 / s)
     ctx.close()
     return line
 
@@ -456,7 +470,6 @@ def run_step_b16(args, env):
         m = win[I.masked_positions(Tw, M, seed=I.SEED_PROMPT + 100 + b)]
         tok[b, m], st[b, m] = cfg.mask_id, MASKED
     ctx.dllm_set_state(tok, st)
-    window = ctx.dllm_window()
 
     def step():
         ctx.dllm_rewind_block()
@@ -466,6 +479,7 @@ def run_step_b16(args, env):
         step()
     torch.cuda.synchronize()
     launches = ctx.dllm_launches_per_step()
+    window = ctx.dllm_window()
     steps = max(3, min(args.steps, 40))
     with Timed(torch, device, ctx.stream, pg) as tm:
         for _ in range(steps):
@@ -653,6 +667,8 @@ def run_ours(args):
     for name in names:
         if name == WORKLOAD["workload"]:
             line = run_step_b1(args, env)
+        elif name == STEP_Q4:
+            line = run_step_b1(args, env, q4=True)
         elif name == STEP_B16:
             line = run_step_b16(args, env)
         elif name == SWEEP:

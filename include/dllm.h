@@ -75,6 +75,13 @@ typedef struct {
     int block_len;   /* tokens per block (32) */
     uint64_t weight_seed;
     int n_kv_heads;  /* K/V heads; 0 = n_heads (multi-head attention, LLaDA) */
+    /* Projection weights (the seven per layer and the LM head; the embedding is always bf16):
+     * 16 (or 0): bf16; 4: the 4-bit block format of the Q4_0 weights the paper runs (Sec. 5.1):
+     * 32 consecutive weights of a row (along the input dimension) share one bf16 scale d, each
+     * weight is a 4-bit code q standing for d * (q - 8), and the tensor cores multiply the bf16
+     * value of d * (q - 8) (rounded once); 4.5 bits per weight in HBM.  Drawn from weight_seed:
+     * codes uniform over 0..15, scales (1 + m/128) * 2^-8. */
+    int weight_bits;
 } dllm_config;
 
 /* Commit rules (dllm_sched.commit_mode). */

@@ -8,5 +8,6 @@ from .oracle import (  # noqa: F401
     MASKED, COMMITTED, STABLE, DRAFT, FIXED,
     OracleConfig, OracleSched, Model, Session, build, lib, commit, decide,
     gen_bf16, gen_f32, bf16_to_f32, f32_to_bf16_bits, rmsnorm, rope, forward,
+    q4_dequant, q4_code, q4_scale, gen_q4,
     W_Q, W_K, W_V, W_O, W_GATE, W_UP, W_DOWN, T_EMBED, T_HEAD,
 )

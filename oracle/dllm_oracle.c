@@ -95,6 +95,32 @@ void orc_gen_bf16(uint64_t seed, uint64_t tid, uint64_t first, uint64_t n, doubl
     for (long long i = 0; i < (long long)n; ++i) out[i] = orc_f32_to_bf16(gen_one(key, first + (uint64_t)i, sigma));
 }
 
+/* 4-bit block format (see dllm_oracle.h): weight = bf16(d * (q - 8)). */
+uint16_t orc_q4_dequant(int code, uint16_t scale_bits) {
+    float d = orc_bf16_to_f32(scale_bits);
+    float w = d * (float)(code - 8); /* exact: an 8-bit significand times a 4-bit integer */
+    return orc_f32_to_bf16(w);
+}
+
+int orc_q4_code(uint64_t seed, uint64_t tid, int cols, int r, int c) {
+    uint64_t key = orc_splitmix_at(seed, ORC_Q4_CODES + tid);
+    return (int)(orc_splitmix_at(key, (uint64_t)r * (uint64_t)cols + (uint64_t)c) >> 60);
+}
+
+uint16_t orc_q4_scale(uint64_t seed, uint64_t tid, int cols, int r, int b) {
+    uint64_t key = orc_splitmix_at(seed, ORC_Q4_SCALES + tid);
+    uint64_t nblk = (uint64_t)(cols + 31) / 32;
+    return (uint16_t)(0x3B80u | (uint32_t)(orc_splitmix_at(key, (uint64_t)r * nblk + (uint64_t)b) >> 57));
+}
+
+void orc_gen_q4(uint64_t seed, uint64_t tid, int rows, int cols, uint16_t* out) {
+#pragma omp parallel for schedule(static)
+    for (int r = 0; r < rows; ++r)
+        for (int c = 0; c < cols; ++c)
+            out[(size_t)r * cols + c] =
+                orc_q4_dequant(orc_q4_code(seed, tid, cols, r, c), orc_q4_scale(seed, tid, cols, r, c / 32));
+}
+
 /* ------------------------------------------------------------------ */
 /* Model                                                                */
 /* ------------------------------------------------------------------ */
@@ -152,15 +178,23 @@ orc_model* orc_model_new(const orc_config* c, int gen_layers, int gen_head) {
         m->embed = (uint16_t*)malloc(Vd * 2);
         orc_gen_bf16(c->weight_seed, ORC_T_EMBED, 0, Vd, 0.02, m->embed);
     }
+    const int q4 = c->weight_bits == 4; /* the projections in the 4-bit block format */
     if (gen_head) {
         m->head = (uint16_t*)malloc(Vd * 2);
-        orc_gen_bf16(c->weight_seed, ORC_T_HEAD, 0, Vd, 0.02, m->head);
+        if (q4)
+            orc_gen_q4(c->weight_seed, ORC_T_HEAD, c->vocab, c->d_model, m->head);
+        else
+            orc_gen_bf16(c->weight_seed, ORC_T_HEAD, 0, Vd, 0.02, m->head);
     }
     for (int l = 0; l < L; ++l)
         for (int w = 0; w < 7; ++w) {
-            size_t n = wsize(c, w, NULL, NULL);
+            int rows = 0, cols = 0;
+            size_t n = wsize(c, w, &rows, &cols);
             m->w[l * 7 + w] = (uint16_t*)malloc(n * 2);
-            orc_gen_bf16(c->weight_seed, ORC_LAYER_TENSOR(l, w), 0, n, 0.02, m->w[l * 7 + w]);
+            if (q4)
+                orc_gen_q4(c->weight_seed, ORC_LAYER_TENSOR(l, w), rows, cols, m->w[l * 7 + w]);
+            else
+                orc_gen_bf16(c->weight_seed, ORC_LAYER_TENSOR(l, w), 0, n, 0.02, m->w[l * 7 + w]);
         }
     return m;
 }

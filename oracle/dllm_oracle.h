@@ -39,6 +39,11 @@ typedef struct {
      * (multi-head attention, LLaDA).  Must divide n_heads: query head h reads K/V head
      * h / (n_heads / n_kv_heads). */
     int n_kv_heads;
+    /* Storage of the projection weights (the seven per layer and the LM head; the embedding is
+     * always bf16): 16 (or 0) = bf16 drawn N(0, 0.02); 4 = the 4-bit block format of the Q4_0
+     * weights the paper runs (Sec. 5.1), see orc_q4_dequant.  The oracle keeps every weight as
+     * the bf16 value it dequantizes to, so the arithmetic after it is the same for both. */
+    int weight_bits;
 } orc_config;
 
 typedef struct {
@@ -96,6 +101,23 @@ void orc_gen_f32(uint64_t seed, uint64_t tensor_id, uint64_t first, uint64_t n, 
 void orc_gen_bf16(uint64_t seed, uint64_t tensor_id, uint64_t first, uint64_t n, double sigma, uint16_t* out);
 uint16_t orc_f32_to_bf16(float f);
 float orc_bf16_to_f32(uint16_t h);
+
+/* ---- 4-bit block-quantised weights (Q4_0, Sec. 5.1) ----
+ * Along the input dimension every 32 consecutive weights of a row form a block with one scale
+ * d; each weight is a 4-bit code q in 0..15 and stands for d * (q - 8).  The paper's Q4_0 keeps
+ * d in fp16; here d is a bf16 value (reading: the GPU multiplies in bf16), and the weight the
+ * arithmetic uses is d * (q - 8) rounded once to bf16 (the product itself is exact in fp32).
+ * Synthetic draws (no trained weights): for tensor tid, q of element (r, c) = the top 4 bits
+ * of SplitMix64 output r*cols + c of the stream keyed by (seed, ORC_Q4_CODES + tid); d of
+ * block (r, b) = the bf16 with bits 0x3B80 | (top 7 bits of output r*ceil(cols/32) + b of the
+ * stream keyed by (seed, ORC_Q4_SCALES + tid)), i.e. (1 + m/128) * 2^-8, m in 0..127. */
+#define ORC_Q4_CODES (3ull << 40)
+#define ORC_Q4_SCALES (4ull << 40)
+uint16_t orc_q4_dequant(int code, uint16_t scale_bits);
+int orc_q4_code(uint64_t seed, uint64_t tid, int cols, int r, int c);
+uint16_t orc_q4_scale(uint64_t seed, uint64_t tid, int cols, int r, int b);
+/* rows x cols weights of tensor tid in the 4-bit format, dequantised to bf16 bits. */
+void orc_gen_q4(uint64_t seed, uint64_t tid, int rows, int cols, uint16_t* out);
 
 /* ---- model ---- */
 typedef struct orc_model orc_model;

@@ -41,7 +41,7 @@ class _Cfg(C.Structure):
     _fields_ = [("n_layers", C.c_int), ("d_model", C.c_int), ("n_heads", C.c_int),
                 ("head_dim", C.c_int), ("ffn", C.c_int), ("vocab", C.c_int), ("mask_id", C.c_int),
                 ("rope_base", C.c_double), ("rms_eps", C.c_double), ("weight_seed", C.c_uint64),
-                ("n_kv_heads", C.c_int)]
+                ("n_kv_heads", C.c_int), ("weight_bits", C.c_int)]
 
 
 class _Sched(C.Structure):
@@ -76,6 +76,13 @@ def lib():
         L.orc_gen_bf16.argtypes = [U64, U64, U64, U64, D, P]
         L.orc_f32_to_bf16.restype = C.c_uint16
         L.orc_f32_to_bf16.argtypes = [F]
+        L.orc_q4_dequant.restype = C.c_uint16
+        L.orc_q4_dequant.argtypes = [I, C.c_uint16]
+        L.orc_q4_code.restype = I
+        L.orc_q4_code.argtypes = [U64, U64, I, I, I]
+        L.orc_q4_scale.restype = C.c_uint16
+        L.orc_q4_scale.argtypes = [U64, U64, I, I, I]
+        L.orc_gen_q4.argtypes = [U64, U64, I, I, P]
         L.orc_model_new.restype = P
         L.orc_model_new.argtypes = [P, I, I]
         L.orc_model_new_zero.restype = P
@@ -132,6 +139,7 @@ class OracleConfig:
     rms_eps: float = 1e-5
     weight_seed: int = 0x11ADA8B
     n_kv_heads: int = 0  # grouped-query attention (Dream-7B style); 0 = n_heads (LLaDA's multi-head)
+    weight_bits: int = 16  # 4: the projections in the 4-bit block format (Q4_0, Sec. 5.1)
 
     @property
     def kv_dim(self):
@@ -139,7 +147,8 @@ class OracleConfig:
 
     def c(self):
         return _Cfg(self.n_layers, self.d_model, self.n_heads, self.head_dim, self.ffn, self.vocab,
-                    self.mask_id, self.rope_base, self.rms_eps, self.weight_seed, self.n_kv_heads)
+                    self.mask_id, self.rope_base, self.rms_eps, self.weight_seed, self.n_kv_heads,
+                    self.weight_bits)
 
 
 @dataclass
@@ -176,6 +185,26 @@ def gen_f32(seed, tensor_id, first, n, sigma):
 def gen_bf16(seed, tensor_id, first, n, sigma):
     out = np.empty(n, np.uint16)
     lib().orc_gen_bf16(seed, tensor_id, first, n, sigma, _p(out))
+    return out
+
+
+def q4_dequant(code, scale_bits):
+    """bf16 bits of the 4-bit block format's weight d * (code - 8) (orc_q4_dequant)."""
+    return int(lib().orc_q4_dequant(int(code), int(scale_bits)))
+
+
+def q4_code(seed, tid, cols, r, c):
+    return int(lib().orc_q4_code(seed, tid, cols, r, c))
+
+
+def q4_scale(seed, tid, cols, r, b):
+    return int(lib().orc_q4_scale(seed, tid, cols, r, b))
+
+
+def gen_q4(seed, tid, rows, cols):
+    """rows x cols weights of tensor tid in the 4-bit format, as dequantised bf16 bits."""
+    out = np.empty((rows, cols), np.uint16)
+    lib().orc_gen_q4(seed, tid, rows, cols, _p(out))
     return out
 
 

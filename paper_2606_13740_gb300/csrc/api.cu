@@ -42,7 +42,8 @@ struct Layout {
     int cnt_len, done_len;  // per phase slot
     size_t off_tok, off_st, off_stok, off_sst, off_seqkv, off_plan, off_outs, off_status;
     size_t total;
-    size_t w_qkv, w_o, w_gu, w_d;  // element offsets inside a layer
+    size_t w_qkv, w_o, w_gu, w_d;  // element offsets inside a layer (bf16) or byte offsets (4-bit)
+    bool q4;                       // projections in the 4-bit block format (kQ4TileBytes tiles)
 };
 
 Layout make_layout(const dllm_config& c) {
@@ -58,20 +59,31 @@ Layout make_layout(const dllm_config& c) {
     L.head_rows = rup(V, 128);
     L.head_tiles = L.head_rows / 128;
     L.max_tok = c.max_batch * c.max_window;
-    L.w_qkv = 0;
-    L.w_o = L.w_qkv + static_cast<size_t>(L.qkv_rows) * d;
-    L.w_gu = L.w_o + static_cast<size_t>(L.o_rows) * L.qd;
-    L.w_d = L.w_gu + static_cast<size_t>(L.gu_rows) * d;
-    L.per_layer = L.w_d + static_cast<size_t>(L.d_rows) * rup(F, 64);  // tile-major: K padded to 64
+    L.q4 = c.weight_bits == 4;
+    if (L.q4) {  // byte offsets of tile-major 4-bit matrices: (rows / 128) x (K / 64) tiles each
+        auto tiles = [](int rows, int k) { return static_cast<size_t>(rows / 128) * ((k + 63) / 64) * kQ4TileBytes; };
+        L.w_qkv = 0;
+        L.w_o = L.w_qkv + tiles(L.qkv_rows, d);
+        L.w_gu = L.w_o + tiles(L.o_rows, L.qd);
+        L.w_d = L.w_gu + tiles(L.gu_rows, d);
+        L.per_layer = L.w_d + tiles(L.d_rows, F);
+    } else {
+        L.w_qkv = 0;
+        L.w_o = L.w_qkv + static_cast<size_t>(L.qkv_rows) * d;
+        L.w_gu = L.w_o + static_cast<size_t>(L.o_rows) * L.qd;
+        L.w_d = L.w_gu + static_cast<size_t>(L.gu_rows) * d;
+        L.per_layer = L.w_d + static_cast<size_t>(L.d_rows) * rup(F, 64);  // tile-major: K padded to 64
+    }
     size_t o = 0;
     auto take = [&](size_t bytes) {
         size_t r = o;
         o = al256(o + bytes);
         return r;
     };
-    L.off_w = take(L.per_layer * 2 * c.n_layers);
+    L.off_w = take(L.per_layer * (L.q4 ? 1 : 2) * c.n_layers);
     L.off_emb = take(static_cast<size_t>(V) * d * 2);
-    L.off_head = take(static_cast<size_t>(L.head_rows) * d * 2);
+    L.off_head = take(L.q4 ? static_cast<size_t>(L.head_tiles) * ((d + 63) / 64) * kQ4TileBytes
+                           : static_cast<size_t>(L.head_rows) * d * 2);
     L.kv_half = static_cast<size_t>(c.max_batch) * L.Hkv * c.max_ctx * hd;
     L.off_kv = take(L.kv_half * 2 * 2 * c.n_layers);
     const size_t T = L.max_tok;
@@ -138,6 +150,7 @@ const char* check_cfg(const dllm_config& c) {
     if (c.max_batch > 256) return "max_batch must be <= 256";
     if (c.block_len > kMaxBlock) return "block_len too large";
     if (c.rms_eps <= 0.0f || c.rope_base <= 1.0f) return "bad rope_base / rms_eps";
+    if (c.weight_bits != 0 && c.weight_bits != 16 && c.weight_bits != 4) return "weight_bits must be 16 or 4";
     return nullptr;
 }
 
@@ -153,8 +166,8 @@ struct dllm_ctx {
     bool own_arena = false;
     // views
     __nv_bfloat16* emb = nullptr;
-    __nv_bfloat16* head = nullptr;
-    std::vector<__nv_bfloat16*> wl;
+    uint8_t* head = nullptr;         // LM head: bf16 or 4-bit tiles
+    std::vector<uint8_t*> wl;        // per layer: the four projection matrices (bf16 or 4-bit tiles)
 
     __nv_bfloat16* kv = nullptr;
     float* x = nullptr;
@@ -210,6 +223,12 @@ struct dllm_ctx {
     bool poisoned = false;
     std::string err;
 };
+
+// Start of a projection matrix of layer l at offset off (elements of bf16 weights, bytes of
+// 4-bit tiles).
+static const void* wmat(const dllm_ctx* ctx, int l, size_t off) {
+    return ctx->wl[l] + off * (ctx->L.q4 ? 1 : 2);
+}
 
 // Record a timing event after a launch of the given kind (or the start mark).
 static void mark(dllm_ctx* ctx, int kind) {
@@ -350,7 +369,7 @@ static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0, bool sls 
     };
     // phase slot i of a chain uses scratch slot i; consecutive chains are ordered by the stream
     auto add_phase = [&](ChainArgs& ca, ChainMaps& m, const GemmPlan& p, int epi, EpiArgs e, int dep_rows,
-                         const __nv_bfloat16* w_tiles, const CUtensorMap& x) {
+                         const void* w_tiles, const CUtensorMap& x) {
         const int i = ca.n_phases++;
         ChainPhase& P = ca.ph[i];
         P.p = p;
@@ -367,6 +386,7 @@ static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0, bool sls 
     };
     const int smem_budget = (ctx->debug & 8) ? kChainSmemFull : kChainSmemShared;
     auto run_chain = [&](ChainArgs& ca, const ChainMaps& m, int tag_add, int kind) -> int {
+        ca.q4 = L.q4 ? 1 : 0;
         ca.epoch = ctx->epoch;
         ca.tag_mul = c.n_layers + 2;
         ca.tag_add = tag_add;
@@ -379,7 +399,7 @@ static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0, bool sls 
     {
         ChainArgs ca{};
         ChainMaps m{};
-        add_phase(ca, m, pq, EPI_QKV, qkv_args(0), 0, ctx->wl[0] + L.w_qkv, tx_xn);
+        add_phase(ca, m, pq, EPI_QKV, qkv_args(0), 0, wmat(ctx, 0, L.w_qkv), tx_xn);
         // debug flag 32 (the bounded-wait test): this launch waits for a word nobody writes
         if ((ctx->debug & 32) && ctx->in_step) ca.gate = ctx->status + 2;
         if (int rc = run_chain(ca, m, 1, DLLM_K_QKV)) return rc;
@@ -392,11 +412,10 @@ static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0, bool sls 
         // output projection (+ residual) -> gate/up (+ SwiGLU) -> down (+ residual) -> next QKV or LM head
         ChainArgs ca{};
         ChainMaps m{};
-        const __nv_bfloat16* w = ctx->wl[l];
-        add_phase(ca, m, po, EPI_RESID, er, 0, w + L.w_o, tx_attn);
-        add_phase(ca, m, pg, EPI_SWIGLU, ep, 128, w + L.w_gu, tx_xn);
-        add_phase(ca, m, pd, EPI_RESID, er, 64, w + L.w_d, tx_h);
-        if (l + 1 < c.n_layers) add_phase(ca, m, pq, EPI_QKV, qkv_args(l + 1), 128, ctx->wl[l + 1] + L.w_qkv, tx_xn);
+        add_phase(ca, m, po, EPI_RESID, er, 0, wmat(ctx, l, L.w_o), tx_attn);
+        add_phase(ca, m, pg, EPI_SWIGLU, ep, 128, wmat(ctx, l, L.w_gu), tx_xn);
+        add_phase(ca, m, pd, EPI_RESID, er, 64, wmat(ctx, l, L.w_d), tx_h);
+        if (l + 1 < c.n_layers) add_phase(ca, m, pq, EPI_QKV, qkv_args(l + 1), 128, wmat(ctx, l + 1, L.w_qkv), tx_xn);
         else if (head && !sls) add_phase(ca, m, ph, EPI_LMHEAD, eh, 128, ctx->head, tx_xn);
         if (int rc = run_chain(ca, m, l + 2, DLLM_K_LAYER)) return rc;
     }
@@ -568,7 +587,7 @@ int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void*
     uint8_t* A = ctx->arena;
     const int d = c.d_model, F = c.ffn, qd = L.qd;
     ctx->emb = reinterpret_cast<__nv_bfloat16*>(A + L.off_emb);
-    ctx->head = reinterpret_cast<__nv_bfloat16*>(A + L.off_head);
+    ctx->head = A + L.off_head;
     ctx->kv = reinterpret_cast<__nv_bfloat16*>(A + L.off_kv);
     ctx->x = reinterpret_cast<float*>(A + L.off_x);
     ctx->xn = reinterpret_cast<__nv_bfloat16*>(A + L.off_xn);
@@ -613,21 +632,24 @@ int dllm_init(const dllm_config* cfg, void* dev_arena, size_t arena_bytes, void*
     const int hd = c.head_dim;
     // (the embedding is gathered by rows: row-major; the projections are streamed: tile-major)
     const int kvd = L.kvd;
+    // a projection matrix (rows_phys x cols, row order `mode`) of tensors tid.. in the context's format
+    auto init_w = [&](uint8_t* dst, int mode, int rows_phys, int cols, int logical_rows, uint64_t tid) {
+        return L.q4 ? launch_init_weight_q4(dst, mode, rows_phys, cols, logical_rows, seed, tid, qd, kvd, hd, s)
+                    : launch_init_weight(reinterpret_cast<__nv_bfloat16*>(dst), mode, rows_phys, cols, logical_rows,
+                                         seed, tid, qd, kvd, hd, true, s);
+    };
     cudaError_t ie = launch_init_weight(ctx->emb, 0, c.vocab, d, c.vocab, seed, 1, qd, kvd, hd, false, s);
-    if (ie == cudaSuccess)
-        ie = launch_init_weight(ctx->head, 0, L.head_rows, d, c.vocab, seed, 2, qd, kvd, hd, true, s);
+    if (ie == cudaSuccess) ie = init_w(ctx->head, 0, L.head_rows, d, c.vocab, 2);
     ctx->wl.resize(c.n_layers);
+    const size_t unit = L.q4 ? 1 : 2;  // bytes per layout offset unit
     for (int l = 0; l < c.n_layers && ie == cudaSuccess; ++l) {
-        __nv_bfloat16* w = reinterpret_cast<__nv_bfloat16*>(A + L.off_w) + static_cast<size_t>(l) * L.per_layer;
+        uint8_t* w = A + L.off_w + static_cast<size_t>(l) * L.per_layer * unit;
         ctx->wl[l] = w;
         const uint64_t t0 = 16 + 8ull * l;
-        ie = launch_init_weight(w + L.w_qkv, 1, L.qkv_rows, d, qd, seed, t0 + 0, qd, kvd, hd, true, s);
-        if (ie == cudaSuccess)
-            ie = launch_init_weight(w + L.w_o, 0, L.o_rows, qd, d, seed, t0 + 3, qd, kvd, hd, true, s);
-        if (ie == cudaSuccess)
-            ie = launch_init_weight(w + L.w_gu, 2, L.gu_rows, d, F, seed, t0 + 4, qd, kvd, hd, true, s);
-        if (ie == cudaSuccess)
-            ie = launch_init_weight(w + L.w_d, 0, L.d_rows, F, d, seed, t0 + 6, qd, kvd, hd, true, s);
+        ie = init_w(w + L.w_qkv * unit, 1, L.qkv_rows, d, qd, t0 + 0);
+        if (ie == cudaSuccess) ie = init_w(w + L.w_o * unit, 0, L.o_rows, qd, d, t0 + 3);
+        if (ie == cudaSuccess) ie = init_w(w + L.w_gu * unit, 2, L.gu_rows, d, F, t0 + 4);
+        if (ie == cudaSuccess) ie = init_w(w + L.w_d * unit, 0, L.d_rows, F, d, t0 + 6);
     }
     // RoPE frequencies base^(-2j/hd), in double on the host
     std::vector<float> th(c.head_dim / 2);
@@ -1146,21 +1168,43 @@ int dllm_get_weight(dllm_ctx* ctx, int layer, int which, uint16_t* out, size_t n
     const int rows = layer < 0 ? c.vocab : (which == 0) ? qd : (which <= 2) ? L.kvd : (which == 3 || which == 6) ? d : F;
     const int cols = layer < 0 ? d : (which == 3) ? qd : (which == 6) ? F : d;
     if (n_elems < static_cast<size_t>(rows) * cols) return fail(ctx, DLLM_EINVAL, "buffer too small");
-    const __nv_bfloat16* src;
+    const uint8_t* src;
     int phys_rows;
+    const size_t unit = L.q4 ? 1 : 2;
     if (layer < 0) {
         src = ctx->head;
         phys_rows = L.head_rows;
     } else {
-        const __nv_bfloat16* w = ctx->wl[layer];
-        src = w + (which <= 2 ? L.w_qkv : which == 3 ? L.w_o : which == 6 ? L.w_d : L.w_gu);
+        src = ctx->wl[layer] + unit * (which <= 2 ? L.w_qkv : which == 3 ? L.w_o : which == 6 ? L.w_d : L.w_gu);
         phys_rows = which <= 2 ? L.qkv_rows : which == 3 ? L.o_rows : which == 6 ? L.d_rows : L.gu_rows;
     }
     const int kb = (cols + 63) / 64;
-    std::vector<uint16_t> phys(static_cast<size_t>(phys_rows) * kb * 64);
-    CK(cudaMemcpyAsync(phys.data(), src, phys.size() * 2, cudaMemcpyDeviceToHost, ctx->stream));
+    const size_t bytes = L.q4 ? static_cast<size_t>(phys_rows / 128) * kb * kQ4TileBytes
+                              : static_cast<size_t>(phys_rows) * kb * 64 * 2;
+    std::vector<uint8_t> phys(bytes);
+    CK(cudaMemcpyAsync(phys.data(), src, bytes, cudaMemcpyDeviceToHost, ctx->stream));
     rc = sync_check(ctx);
     if (rc) return rc;
+    // element (physical row pr, column col) as bf16 bits; 4-bit tiles: bf16(d * (q - 8)), the
+    // product exact in fp32 and rounded once to nearest even, as the kernel's expansion does
+    auto element = [&](int pr, int col) -> uint16_t {
+        if (!L.q4) return reinterpret_cast<const uint16_t*>(phys.data())[tiled_index(pr, col, kb)];
+        const uint8_t* tile = phys.data() + (static_cast<size_t>(pr >> 7) * kb + (col >> 6)) * kQ4TileBytes;
+        const int rr = pr & 127, cc = col & 63;
+        uint32_t word;
+        memcpy(&word, tile + ((cc >> 3) * 128 + rr) * 4, 4);
+        const int q = static_cast<int>((word >> q4_code_shift(cc & 7)) & 15u);
+        uint16_t sb;
+        memcpy(&sb, tile + 4096 + ((cc >> 5) * 128 + rr) * 2, 2);
+        uint32_t sbits = static_cast<uint32_t>(sb) << 16;
+        float dsc;
+        memcpy(&dsc, &sbits, 4);
+        const float w = dsc * static_cast<float>(q - 8);
+        uint32_t b;
+        memcpy(&b, &w, 4);
+        b += 0x7FFFu + ((b >> 16) & 1u);  // round to nearest, ties to even (finite values)
+        return static_cast<uint16_t>(b >> 16);
+    };
     const int hd = c.head_dim, half = hd / 2;
     for (int r = 0; r < rows; ++r) {
         int pr = r;
@@ -1171,7 +1215,7 @@ int dllm_get_weight(dllm_ctx* ctx, int layer, int which, uint16_t* out, size_t n
             pr = (r / 64) * 128 + 2 * (r % 64) + (which == 5 ? 1 : 0);
         }
         uint16_t* o = out + static_cast<size_t>(r) * cols;
-        for (int col = 0; col < cols; ++col) o[col] = phys[tiled_index(pr, col, kb)];
+        for (int col = 0; col < cols; ++col) o[col] = element(pr, col);
     }
     return DLLM_OK;
 }

@@ -499,6 +499,9 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
 // TMEM accumulators and their barriers are shared by all phases; a running iteration counter
 // gives every stage its use parity.
 constexpr int kChainThreads = 64 + 32 + 32 * kEpiWarps;
+// 4-bit weights: warps 11..14 expand each raw tile into the bf16 A stage
+constexpr int kDeqWarp0 = 11, kDeqWarps = 4;
+constexpr int kChainThreadsQ4 = kChainThreads + 32 * kDeqWarps;
 constexpr int kMaxDepTiles = 1024;  // the operand producer keeps a readiness bit per producing tile: 32 per lane
 
 struct ChainEpiState {
@@ -849,15 +852,45 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
     if (tr && threadIdx.x == 64) tr[kTrEpiDone] = global_ns();
 }
 
-__global__ void __launch_bounds__(kChainThreads, 1)
+// Expand one 4-bit weight tile (see kQ4TileBytes) into the 128-byte-swizzled K-major bf16 image
+// the UMMA descriptor reads: thread t of the 128 writes row t, each weight bf16(d * (q - 8)).
+// 128 + q is built as a bf16 bit pattern (exponent of 128, q in the low mantissa bits), 136 is
+// subtracted exactly and the scale applied with one correctly rounded bf16 multiply.
+__device__ __forceinline__ void q4_expand_row(const uint8_t* raw, uint8_t* dst_tile, int t) {
+    const uint32_t* codes = reinterpret_cast<const uint32_t*>(raw);
+    const uint16_t* sc = reinterpret_cast<const uint16_t*>(raw + 4096);
+    const uint32_t s0 = sc[t], s1 = sc[128 + t];
+    const __nv_bfloat162 off = __floats2bfloat162_rn(136.0f, 136.0f);
+    uint8_t* row = dst_tile + t * 128;
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+        const uint32_t w = codes[c * 128 + t];
+        const uint32_t sb = c < 4 ? s0 : s1;
+        const uint32_t sbb = sb | (sb << 16);
+        const __nv_bfloat162 d2 = *reinterpret_cast<const __nv_bfloat162*>(&sbb);
+        uint32_t o[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const uint32_t v = ((w >> (4 * j)) & 0x000F000Fu) | 0x43004300u;
+            const __nv_bfloat162 x = __hmul2(__hsub2(*reinterpret_cast<const __nv_bfloat162*>(&v), off), d2);
+            o[j] = *reinterpret_cast<const uint32_t*>(&x);
+        }
+        *reinterpret_cast<uint4*>(row + ((c ^ (t & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+}
+
+template <bool Q4>
+__global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
     k_chain(const __grid_constant__ ChainMaps maps, const __grid_constant__ ChainArgs ca) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int S = ca.stages;
+    const int R = Q4 ? ca.raw_stages : 0;
     const uint32_t b_bytes = static_cast<uint32_t>(ca.ntile) * kBK * 2;
     uint8_t* sA = smem;
     uint8_t* sB = sA + static_cast<size_t>(S) * kABytes;
-    uint8_t* red_stage = sB + static_cast<size_t>(S) * b_bytes;
+    uint8_t* sRaw = sB + static_cast<size_t>(S) * b_bytes;  // 4-bit weight tiles (Q4)
+    uint8_t* red_stage = sRaw + static_cast<size_t>(R) * kQ4TileBytes;
     float* tail = reinterpret_cast<float*>(red_stage + ca.red_bytes + ca.xs_bytes + ca.stg_bytes);
     EpiSmem esm;
     esm.xs = ca.xs_bytes ? reinterpret_cast<float*>(red_stage + ca.red_bytes) : nullptr;
@@ -874,7 +907,9 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     uint64_t* tempty = tfull + 2;
     uint64_t* drain = tempty + 2;
     uint64_t* redbar = drain + 1;  // two partial staging slots
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(redbar + 2);
+    uint64_t* rfull = redbar + 2;  // raw 4-bit tiles (Q4): arrived / read
+    uint64_t* rempty = rfull + R;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(rempty + R);
     volatile int* s_abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
     int* s_rows = reinterpret_cast<int*>(tmem_slot + 2);
     esm.rows = s_rows;
@@ -885,8 +920,13 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     if (threadIdx.x == 0) {
         pdl_launch_dependents();
         for (int s = 0; s < S; ++s) {
-            mbar_init(&full[s], 1);
+            // Q4: the operand producer's expect-tx arrival plus one arrival per dequantizing warp
+            mbar_init(&full[s], Q4 ? 1 + kDeqWarps : 1);
             mbar_init(&empty[s], 1);
+        }
+        for (int r = 0; r < R; ++r) {
+            mbar_init(&rfull[r], 1);
+            mbar_init(&rempty[r], kDeqWarps);
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&tfull[a], 1);
@@ -929,6 +969,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             int stage = 0;
             uint32_t par = 0;
             uint32_t pending = 0, pend_par = 0;
+            constexpr uint32_t tile_bytes = Q4 ? kQ4TileBytes : kABytes;
             for (int ph = 0; ph < ca.n_phases && !*s_abort; ++ph) {
                 const GemmPlan p = phase_plan(ca.ph[ph], rows);
                 if (static_cast<int>(blockIdx.x) >= p.grid) continue;
@@ -940,23 +981,31 @@ __global__ void __launch_bounds__(kChainThreads, 1)
                 int tile = it0 / p.kb, k = it0 - tile * p.kb;
                 int nt = tile / p.m_tiles, mt = tile - nt * p.m_tiles;
                 const char* wt = reinterpret_cast<const char*>(ca.ph[ph].w_tiles);
-                size_t woff = (static_cast<size_t>(mt) * p.kb + k) * kABytes;  // tile-major: (mt*kb + k) tiles
+                size_t woff = (static_cast<size_t>(mt) * p.kb + k) * tile_bytes;  // tile-major: (mt*kb + k) tiles
                 for (int it = it0; it < it1; ++it) {
-                    if (!mbar_wait(&empty[stage], par ^ 1u, s_abort, status)) break;
-                    mbar_arrive_expect_tx(&full[stage], kABytes + b_bytes);
-                    if (wt)
-                        bulk_load_hint(sA + static_cast<size_t>(stage) * kABytes, wt + woff, kABytes, &full[stage],
-                                       pol_w);
-                    else
-                        tma_load_2d(sA + static_cast<size_t>(stage) * kABytes, &maps.w[ph], k * kBK, mt * kBM,
-                                    &full[stage], pol_w);
+                    if constexpr (Q4) {
+                        // the raw tile goes to its own ring; the dequantizing warps fill the A stage
+                        if (!mbar_wait(&rempty[stage], par ^ 1u, s_abort, status)) break;
+                        mbar_arrive_expect_tx(&rfull[stage], kQ4TileBytes);
+                        bulk_load_hint(sRaw + static_cast<size_t>(stage) * kQ4TileBytes, wt + woff, kQ4TileBytes,
+                                       &rfull[stage], pol_w);
+                    } else {
+                        if (!mbar_wait(&empty[stage], par ^ 1u, s_abort, status)) break;
+                        mbar_arrive_expect_tx(&full[stage], kABytes + b_bytes);
+                        if (wt)
+                            bulk_load_hint(sA + static_cast<size_t>(stage) * kABytes, wt + woff, kABytes,
+                                           &full[stage], pol_w);
+                        else
+                            tma_load_2d(sA + static_cast<size_t>(stage) * kABytes, &maps.w[ph], k * kBK, mt * kBM,
+                                        &full[stage], pol_w);
+                    }
                     pending |= 1u << stage;
                     pend_par = (pend_par & ~(1u << stage)) | (par << stage);
-                    if (++stage == S) {
+                    if (++stage == (Q4 ? R : S)) {
                         stage = 0;
                         par ^= 1u;
                     }
-                    woff += kABytes;
+                    woff += tile_bytes;
                     if (++k == p.kb) {
                         k = 0;
                         if (++mt == p.m_tiles) {
@@ -971,9 +1020,10 @@ __global__ void __launch_bounds__(kChainThreads, 1)
                 // let the copies in flight land before the CTA's shared memory is released (a
                 // stage whose operand was never issued does not complete: one deadline for all)
                 const long long t0 = spin_clock();
-                for (int s = 0; s < S; ++s) {
+                for (int s = 0; s < (Q4 ? R : S); ++s) {
                     if (!(pending >> s & 1u)) continue;
-                    while (!mbar_try_wait(&full[s], (pend_par >> s) & 1u) && spin_clock() - t0 < kWaitLimitCycles) {
+                    uint64_t* bar = Q4 ? &rfull[s] : &full[s];
+                    while (!mbar_try_wait(bar, (pend_par >> s) & 1u) && spin_clock() - t0 < kWaitLimitCycles) {
                     }
                 }
             }
@@ -1049,9 +1099,11 @@ __global__ void __launch_bounds__(kChainThreads, 1)
                         if (stop) break;
                     }
                 }
-                if (lane == 0)
+                if (lane == 0) {
+                    if constexpr (Q4) mbar_arrive_expect_tx(&full[stage], b_bytes);  // the A part arrives by warps
                     tma_load_2d(sB + static_cast<size_t>(stage) * b_bytes, &maps.x[ph], k * kBK, nt * ca.ntile,
                                 &full[stage], pol_x);
+                }
                 __syncwarp();
                 if (++stage == S) {
                     stage = 0;
@@ -1063,6 +1115,44 @@ __global__ void __launch_bounds__(kChainThreads, 1)
                         mt = 0;
                         ++nt;
                     }
+                }
+            }
+        }
+    } else if (Q4 && warp >= kDeqWarp0) {
+        // ---------------------------------------------------------- dequantizers (4-bit weights)
+        // Every iteration: wait for its raw tile and for its A stage to be free (the MMAs that
+        // read the stage's previous tile are done), expand the tile (thread t: row t), make the
+        // writes visible to the tensor core's proxy, and arrive (one arrival per warp) on the
+        // stage's full barrier and on the raw slot's empty barrier.
+        const int t = threadIdx.x - kDeqWarp0 * 32;
+        int stage = 0, rs = 0;
+        uint32_t par = 0, rpar = 0;
+        bool stop = false;
+        for (int ph = 0; ph < ca.n_phases && !stop; ++ph) {
+            const GemmPlan p = phase_plan(ca.ph[ph], rows);
+            if (static_cast<int>(blockIdx.x) >= p.grid) continue;
+            const int it0 = static_cast<int>(range_begin(blockIdx.x, p.total, p.grid));
+            const int it1 = static_cast<int>(range_begin(blockIdx.x + 1, p.total, p.grid));
+            for (int it = it0; it < it1; ++it) {
+                if (!mbar_wait(&rfull[rs], rpar, s_abort, status) || !mbar_wait(&empty[stage], par ^ 1u, s_abort, status)) {
+                    stop = true;
+                    break;
+                }
+                q4_expand_row(sRaw + static_cast<size_t>(rs) * kQ4TileBytes, sA + static_cast<size_t>(stage) * kABytes,
+                              t);
+                fence_proxy_async_smem();  // generic writes (and the raw reads) -> async-proxy accesses
+                __syncwarp();
+                if (lane == 0) {
+                    mbar_arrive(&full[stage]);
+                    mbar_arrive(&rempty[rs]);
+                }
+                if (++stage == S) {
+                    stage = 0;
+                    par ^= 1u;
+                }
+                if (++rs == R) {
+                    rs = 0;
+                    rpar ^= 1u;
                 }
             }
         }
@@ -1283,7 +1373,11 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
     // the ring at least 3 stages
     ca.stg_bytes = c32 ? 0 : 32 * kBM * 2;
     ca.xs_bytes = 0;
-    const int fixed0 = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + ca.stg_bytes + 7 * 8 + 16;
+    // 4-bit weights: a ring of 8 raw tiles (4.5 KB each and two barriers) in front of the stages
+    const int raw = ca.q4 ? 8 : 0;
+    ca.raw_stages = raw;
+    const int raw_bytes = raw * (kQ4TileBytes + 16);
+    const int fixed0 = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + ca.stg_bytes + 7 * 8 + 16 + raw_bytes;
     if (ca.x_cols == 0 && (smem_budget - fixed0 - 2 * 32 * kBM * 4) / (stage_bytes + 16) >= 3)
         ca.xs_bytes = 2 * 32 * kBM * 4;
     const int fixed = fixed0 + ca.xs_bytes;
@@ -1296,8 +1390,12 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
 }
 
 cudaError_t chain_init_attrs() {
-    return cudaFuncSetAttribute(reinterpret_cast<const void*>(k_chain), cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                kFullSmem);
+    cudaError_t e = cudaFuncSetAttribute(reinterpret_cast<const void*>(k_chain<false>),
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kFullSmem);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(reinterpret_cast<const void*>(k_chain<true>),
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, kFullSmem);
+    return e;
 }
 
 cudaError_t chain_launch(const ChainMaps& maps, const ChainArgs& ca, cudaStream_t st, bool pdl) {
@@ -1308,7 +1406,13 @@ cudaError_t chain_launch(const ChainMaps& maps, const ChainArgs& ca, cudaStream_
     }
     // a device-resolved row count changes a phase's tiling: no later phase may wait on its flags
     if (ca.dyn_rows && ca.n_phases != 1) return cudaErrorInvalidValue;
-    return launch_k(k_chain, dim3(ca.grid), dim3(kChainThreads), ca.smem, st, pdl, maps, ca);
+    if (ca.q4) {  // every phase's weights in the 4-bit tile format
+        for (int i = 0; i < ca.n_phases; ++i)
+            if (!ca.ph[i].w_tiles) return cudaErrorInvalidValue;
+        if (ca.raw_stages < 2 || ca.raw_stages > 32) return cudaErrorInvalidValue;
+        return launch_k(k_chain<true>, dim3(ca.grid), dim3(kChainThreadsQ4), ca.smem, st, pdl, maps, ca);
+    }
+    return launch_k(k_chain<false>, dim3(ca.grid), dim3(kChainThreads), ca.smem, st, pdl, maps, ca);
 }
 
 }  // namespace dllm

@@ -28,6 +28,17 @@ __host__ __device__ inline size_t tiled_index(int r, int c, int kb) {
            ((((c & 63) >> 3) ^ (r & 7)) << 3) + (c & 7);
 }
 
+// ---------------------------------------------------------------- 4-bit weight storage
+// A 128-row x 64-column tile of 4-bit block-quantised weights (32 weights of a row share one
+// bf16 scale d; a weight is a 4-bit code q standing for d * (q - 8)) is kQ4TileBytes: first the
+// codes, 32-bit word (c16, r) = the 8 codes of row r, columns 8 c16 .. 8 c16 + 7, at word
+// c16 * 128 + r, column 8 c16 + j in bits 4 (j / 2) + 16 (j % 2) .. +3 (so that one mask and
+// one OR turn a shifted word into the bf16 pair 128 + q of two neighbouring columns); then the
+// scales, bf16 (b, r) for columns 32 b .. 32 b + 31 of row r at 4096 + 2 (b * 128 + r).
+// Tiles are stored tile-major as for bf16 ((m-tile * kb + k-block) * kQ4TileBytes).
+constexpr int kQ4TileBytes = 4096 + 512;
+__host__ __device__ inline int q4_code_shift(int j) { return 4 * (j >> 1) + 16 * (j & 1); }
+
 // ---------------------------------------------------------------- GEMM
 // D = W * X^T on tensor cores: W bf16 [M][K] (weights, rows padded to 128),
 // X bf16 [N][K] (tokens).  Row m of D is an output feature, column n a token.
@@ -111,8 +122,10 @@ struct ChainPhase {
     float* partials;     // [grid][ntile*128] split partials (a CTA contributes to at most one tile per phase)
     int* tickets;        // [m_tiles*n_tiles][32], zero between launches
     // non-null: the weights are stored tile-major (tiled_index) and each 16 KB tile arrives with
-    // one contiguous bulk copy; null: row-major [M][K] through the chain's tensor map
-    const __nv_bfloat16* w_tiles;
+    // one contiguous bulk copy; null: row-major [M][K] through the chain's tensor map.  In a
+    // 4-bit chain (ChainArgs::q4) the tiles are kQ4TileBytes each, laid out as q4_tile_word /
+    // q4_tile_scale describe.
+    const void* w_tiles;
 };
 struct ChainArgs {
     int n_phases;
@@ -134,6 +147,10 @@ struct ChainArgs {
     // launch's tag before its first load.  Given a word nobody writes, that wait runs out after
     // kWaitLimitCycles and the launch unwinds with kStatusTimeout, as any stalled wait would.
     const int* gate;
+    // 4-bit weights (the block format of Q4_0, see q4_tile_word): the weight producer streams
+    // raw 4.5 KB tiles into raw_stages slots, and four more warps expand each into the bf16
+    // A stage the tensor cores read
+    int q4, raw_stages;
     ChainPhase ph[kMaxPhases];
 };
 struct ChainMaps {
@@ -192,6 +209,9 @@ inline cudaError_t launch_k(void (*k)(KArgs...), dim3 grid, dim3 block, size_t s
 // (tiled_index; rows_phys a multiple of 128) when `tiled`, else row-major.
 cudaError_t launch_init_weight(__nv_bfloat16* dst, int mode, int rows_phys, int cols, int logical_rows,
                                uint64_t seed, uint64_t tid0, int qd, int kvd, int hd, bool tiled, cudaStream_t st);
+// The same weights in the 4-bit block format (kQ4TileBytes tiles, tile-major).
+cudaError_t launch_init_weight_q4(uint8_t* dst, int mode, int rows_phys, int cols, int logical_rows, uint64_t seed,
+                                  uint64_t tid0, int qd, int kvd, int hd, cudaStream_t st);
 cudaError_t launch_init_kv_random(__nv_bfloat16* cache, int B, int H, int hd, int cap, int P, int layer,
                                   int which, int L, uint64_t seed, cudaStream_t st);
 // x = embedding rows of the window's ids (fp32), xb = bf16(x), sq[d/128][N] = per-128-feature

@@ -31,6 +31,26 @@ __device__ __forceinline__ float gen_value(uint64_t key, uint64_t i, double sigm
     return __double2float_rn(scaled);
 }
 
+// Row map shared by the bf16 and 4-bit generators: physical row r of a fused matrix -> the
+// tensor (tid0 + part) and logical row it holds (logical_rows: a padding row).
+__device__ __forceinline__ void weight_row(int mode, int r, int qd, int kvd, int hd, int logical_rows, uint64_t tid0,
+                                           uint64_t* tid, int* lr) {
+    *tid = tid0;
+    *lr = r;
+    if (mode == 1) {
+        const int part = r < qd ? 0 : (r < qd + kvd ? 1 : (r < qd + 2 * kvd ? 2 : 3));
+        const int f = r - (part == 0 ? 0 : qd + (part - 1) * kvd);
+        const int hh = f / hd, pp = f % hd;
+        *tid = tid0 + part;
+        *lr = hh * hd + (pp >> 1) + (pp & 1) * (hd >> 1);
+        if (part > 2 || *lr >= (part == 0 ? qd : kvd)) *lr = logical_rows;
+    } else if (mode == 2) {
+        const int tile = r >> 7, w = r & 127;
+        *tid = tid0 + (w & 1);
+        *lr = tile * 64 + (w >> 1);
+    }
+}
+
 // mode 0: plain (physical row = logical row of tensor tid0, zero rows past
 //         logical_rows);
 // mode 1: fused QKV: rows [0,qd) tensor tid0 (q), [qd,qd+kvd) tid0+1 (k), [qd+kvd,qd+2kvd)
@@ -62,20 +82,9 @@ __global__ void k_init_weight(__nv_bfloat16* dst, int mode, int rows, int cols, 
             r = static_cast<int>(e / cols);
             c = static_cast<int>(e - static_cast<size_t>(r) * cols);
         }
-        uint64_t tid = tid0;
-        int lr = r;
-        if (mode == 1) {
-            const int part = r < qd ? 0 : (r < qd + kvd ? 1 : (r < qd + 2 * kvd ? 2 : 3));
-            const int f = r - (part == 0 ? 0 : qd + (part - 1) * kvd);
-            const int hh = f / hd, pp = f % hd;
-            tid = tid0 + part;
-            lr = hh * hd + (pp >> 1) + (pp & 1) * (hd >> 1);
-            if (part > 2 || lr >= (part == 0 ? qd : kvd)) lr = logical_rows;  // padding rows
-        } else if (mode == 2) {
-            const int tile = r >> 7, w = r & 127;
-            tid = tid0 + (w & 1);
-            lr = tile * 64 + (w >> 1);
-        }
+        uint64_t tid;
+        int lr;
+        weight_row(mode, r, qd, kvd, hd, logical_rows, tid0, &tid, &lr);
         float v = 0.0f;
         if (lr < logical_rows) {
             uint64_t key = sm64_at_hd(seed, tid);
@@ -92,6 +101,62 @@ cudaError_t launch_init_weight(__nv_bfloat16* dst, int mode, int rows_phys, int 
     int blocks = static_cast<int>((n + 255) / 256 < 65536 ? (n + 255) / 256 : 65536);
     k_init_weight<<<blocks, 256, 0, st>>>(dst, mode, rows_phys, cols, logical_rows, seed, tid0, qd, kvd, hd,
                                           tiled ? 1 : 0);
+    return cudaGetLastError();
+}
+
+// Seeded 4-bit block-quantised weights (the Q4_0 format of the paper's runs) in the tile layout
+// of kQ4TileBytes (internal.h).  Code of logical element (lr, c) of tensor tid: the top 4 bits
+// of SplitMix64 output lr * cols + c of the stream keyed by (seed, 3 * 2^40 + tid); scale of
+// block (lr, b): bf16 bits 0x3B80 | the top 7 bits of output lr * ceil(cols / 32) + b of the
+// stream keyed by (seed, 4 * 2^40 + tid).  Padding rows: scale 0; columns past cols: code 8.
+// One thread per (tile, row, code word or scale).
+__global__ void k_init_weight_q4(uint8_t* dst, int mode, int rows, int cols, int logical_rows, uint64_t seed,
+                                 uint64_t tid0, int qd, int kvd, int hd) {
+    const int kb = (cols + 63) / 64;
+    const int nblk = (cols + 31) / 32;
+    const size_t n = static_cast<size_t>(rows / 128) * kb * 128 * 10;
+    for (size_t e = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; e < n;
+         e += static_cast<size_t>(gridDim.x) * blockDim.x) {
+        const size_t tile = e / 1280;
+        const int w = static_cast<int>(e - tile * 1280), rr = w & 127, item = w >> 7;
+        const int mt = static_cast<int>(tile / kb), kt = static_cast<int>(tile - static_cast<size_t>(mt) * kb);
+        uint64_t tid;
+        int lr;
+        weight_row(mode, mt * 128 + rr, qd, kvd, hd, logical_rows, tid0, &tid, &lr);
+        const bool valid = lr < logical_rows;
+        uint8_t* tb = dst + tile * kQ4TileBytes;
+        if (item < 8) {
+            const uint64_t key = sm64_at_hd(seed, (3ull << 40) + tid);
+            uint32_t word = 0;
+            for (int j = 0; j < 8; ++j) {
+                const int c = kt * 64 + item * 8 + j;
+                const uint32_t code =
+                    (valid && c < cols)
+                        ? static_cast<uint32_t>(sm64_at_hd(key, static_cast<uint64_t>(lr) * cols + c) >> 60)
+                        : 8u;
+                word |= code << q4_code_shift(j);
+            }
+            reinterpret_cast<uint32_t*>(tb)[item * 128 + rr] = word;
+        } else {
+            const int b = item - 8;
+            const uint64_t key = sm64_at_hd(seed, (4ull << 40) + tid);
+            const int blk = 2 * kt + b;
+            const uint16_t bits =
+                (valid && blk < nblk)
+                    ? static_cast<uint16_t>(0x3B80u | static_cast<uint32_t>(
+                                                          sm64_at_hd(key, static_cast<uint64_t>(lr) * nblk + blk) >> 57))
+                    : static_cast<uint16_t>(0);
+            reinterpret_cast<uint16_t*>(tb + 4096)[b * 128 + rr] = bits;
+        }
+    }
+}
+
+cudaError_t launch_init_weight_q4(uint8_t* dst, int mode, int rows_phys, int cols, int logical_rows, uint64_t seed,
+                                  uint64_t tid0, int qd, int kvd, int hd, cudaStream_t st) {
+    if (rows_phys & 127) return cudaErrorInvalidValue;
+    const size_t n = static_cast<size_t>(rows_phys / 128) * ((cols + 63) / 64) * 1280;
+    const int blocks = static_cast<int>((n + 255) / 256 < 65536 ? (n + 255) / 256 : 65536);
+    k_init_weight_q4<<<blocks, 256, 0, st>>>(dst, mode, rows_phys, cols, logical_rows, seed, tid0, qd, kvd, hd);
     return cudaGetLastError();
 }
 

@@ -32,7 +32,8 @@ class dllm_config(C.Structure):
     _fields_ = [("n_layers", C.c_int), ("d_model", C.c_int), ("n_heads", C.c_int), ("head_dim", C.c_int),
                 ("ffn", C.c_int), ("vocab", C.c_int), ("mask_id", C.c_int), ("rope_base", C.c_float),
                 ("rms_eps", C.c_float), ("max_batch", C.c_int), ("max_ctx", C.c_int), ("max_window", C.c_int),
-                ("block_len", C.c_int), ("weight_seed", C.c_uint64), ("n_kv_heads", C.c_int)]
+                ("block_len", C.c_int), ("weight_seed", C.c_uint64), ("n_kv_heads", C.c_int),
+                ("weight_bits", C.c_int)]
 
 
 class dllm_sched(C.Structure):
@@ -143,6 +144,7 @@ class Config:
     block_len: int = 32
     weight_seed: int = 0x11ADA8B
     n_kv_heads: int = 0  # grouped-query attention: K/V heads (0 = n_heads)
+    weight_bits: int = 16  # 4: projections in the 4-bit block format (Q4_0 weights, Sec. 5.1)
 
     @property
     def kv_dim(self):
@@ -151,7 +153,7 @@ class Config:
     def c(self):
         return dllm_config(self.n_layers, self.d_model, self.n_heads, self.head_dim, self.ffn, self.vocab,
                            self.mask_id, self.rope_base, self.rms_eps, self.max_batch, self.max_ctx, self.max_window,
-                           self.block_len, self.weight_seed, self.n_kv_heads)
+                           self.block_len, self.weight_seed, self.n_kv_heads, self.weight_bits)
 
 
 @dataclass

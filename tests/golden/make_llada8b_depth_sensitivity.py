@@ -91,7 +91,7 @@ def main():
                 "seed 0x11ADA8B weights, 512-token uniform prompt (seed 1), one step on a 32-token window with "
                 "24 masked; written by tests/golden/make_llada8b_depth_sensitivity.py from the oracle only",
         "citation": "Sec. 5.1 (16-bit activations on the NPU; read as bf16 operands with fp32 accumulation)",
-        "u_bf16": 2.0 ** -9,
+        "u_bf16": 2.0 ** -8,
         "delta_in": d_in,
         "A_K": [rel(k0[l], k1[l]) / d_in for l in range(SHAPE["n_layers"])],
         "A_V": [rel(v0[l], v1[l]) / d_in for l in range(SHAPE["n_layers"])],
