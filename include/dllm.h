@@ -80,7 +80,8 @@ typedef struct {
      * 32 consecutive weights of a row (along the input dimension) share one bf16 scale d, each
      * weight is a 4-bit code q standing for d * (q - 8), and the tensor cores multiply the bf16
      * value of d * (q - 8) (rounded once); 4.5 bits per weight in HBM.  Drawn from weight_seed:
-     * codes uniform over 0..15, scales (1 + m/128) * 2^-8. */
+     * codes uniform over 0..15, scales (1 + m/128) * 2^-8 with m in 0..31 (standard deviation
+     * of the weights about 0.02, as for the bf16 draws). */
     int weight_bits;
 } dllm_config;
 

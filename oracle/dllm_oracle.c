@@ -110,7 +110,7 @@ int orc_q4_code(uint64_t seed, uint64_t tid, int cols, int r, int c) {
 uint16_t orc_q4_scale(uint64_t seed, uint64_t tid, int cols, int r, int b) {
     uint64_t key = orc_splitmix_at(seed, ORC_Q4_SCALES + tid);
     uint64_t nblk = (uint64_t)(cols + 31) / 32;
-    return (uint16_t)(0x3B80u | (uint32_t)(orc_splitmix_at(key, (uint64_t)r * nblk + (uint64_t)b) >> 57));
+    return (uint16_t)(0x3B80u | (uint32_t)(orc_splitmix_at(key, (uint64_t)r * nblk + (uint64_t)b) >> 59));
 }
 
 void orc_gen_q4(uint64_t seed, uint64_t tid, int rows, int cols, uint16_t* out) {

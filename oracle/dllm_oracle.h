@@ -109,8 +109,9 @@ float orc_bf16_to_f32(uint16_t h);
  * arithmetic uses is d * (q - 8) rounded once to bf16 (the product itself is exact in fp32).
  * Synthetic draws (no trained weights): for tensor tid, q of element (r, c) = the top 4 bits
  * of SplitMix64 output r*cols + c of the stream keyed by (seed, ORC_Q4_CODES + tid); d of
- * block (r, b) = the bf16 with bits 0x3B80 | (top 7 bits of output r*ceil(cols/32) + b of the
- * stream keyed by (seed, ORC_Q4_SCALES + tid)), i.e. (1 + m/128) * 2^-8, m in 0..127. */
+ * block (r, b) = the bf16 with bits 0x3B80 | (top 5 bits of output r*ceil(cols/32) + b of the
+ * stream keyed by (seed, ORC_Q4_SCALES + tid)), i.e. (1 + m/128) * 2^-8, m in 0..31: the
+ * weights' standard deviation is then about 0.02, that of the bf16 weights N(0, 0.02). */
 #define ORC_Q4_CODES (3ull << 40)
 #define ORC_Q4_SCALES (4ull << 40)
 uint16_t orc_q4_dequant(int code, uint16_t scale_bits);

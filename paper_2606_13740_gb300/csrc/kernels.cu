@@ -107,8 +107,9 @@ cudaError_t launch_init_weight(__nv_bfloat16* dst, int mode, int rows_phys, int 
 // Seeded 4-bit block-quantised weights (the Q4_0 format of the paper's runs) in the tile layout
 // of kQ4TileBytes (internal.h).  Code of logical element (lr, c) of tensor tid: the top 4 bits
 // of SplitMix64 output lr * cols + c of the stream keyed by (seed, 3 * 2^40 + tid); scale of
-// block (lr, b): bf16 bits 0x3B80 | the top 7 bits of output lr * ceil(cols / 32) + b of the
-// stream keyed by (seed, 4 * 2^40 + tid).  Padding rows: scale 0; columns past cols: code 8.
+// block (lr, b): bf16 bits 0x3B80 | the top 5 bits of output lr * ceil(cols / 32) + b of the
+// stream keyed by (seed, 4 * 2^40 + tid), i.e. (1 + m/128) * 2^-8 with m < 32 (weights of
+// standard deviation about 0.02).  Padding rows: scale 0; columns past cols: code 8.
 // One thread per (tile, row, code word or scale).
 __global__ void k_init_weight_q4(uint8_t* dst, int mode, int rows, int cols, int logical_rows, uint64_t seed,
                                  uint64_t tid0, int qd, int kvd, int hd) {
@@ -144,7 +145,7 @@ __global__ void k_init_weight_q4(uint8_t* dst, int mode, int rows, int cols, int
             const uint16_t bits =
                 (valid && blk < nblk)
                     ? static_cast<uint16_t>(0x3B80u | static_cast<uint32_t>(
-                                                          sm64_at_hd(key, static_cast<uint64_t>(lr) * nblk + blk) >> 57))
+                                                          sm64_at_hd(key, static_cast<uint64_t>(lr) * nblk + blk) >> 59))
                     : static_cast<uint16_t>(0);
             reinterpret_cast<uint16_t*>(tb + 4096)[b * 128 + rr] = bits;
         }

@@ -6,8 +6,9 @@ d * (q - 8), which the arithmetic uses rounded once to bf16.
 - With power-of-two scales the format is exact (no rounding): d * (q - 8) itself.
 - Otherwise the rounding stays within half a bf16 ulp of d * (q - 8): 2^-8 relative (8 significant
   bits).
-- The synthetic draws: codes uniform over 0..15, scales in [2^-8, 2^-7), one scale per block of
-  32, and a model in the format holds exactly those dequantised weights.
+- The synthetic draws: codes uniform over 0..15, scales (1 + m/128) 2^-8 with m < 32 (weights of
+  standard deviation 0.02, like the bf16 draws), one scale per block of 32, and a model in the
+  format holds exactly those dequantised weights.
 """
 from fractions import Fraction
 
@@ -96,8 +97,11 @@ def test_synthetic_draws(lib):
     assert chi2 < 45.0  # 15 degrees of freedom: p < 1e-4 above this
     nblk = (cols + 31) // 32
     scales = np.array([[O.q4_scale(seed, tid, cols, r, b) for b in range(nblk)] for r in range(rows)])
-    assert scales.min() >= 0x3B80 and scales.max() <= 0x3BFF  # [2^-8, 2^-7)
-    assert len(np.unique(scales)) > 100
+    assert scales.min() >= 0x3B80 and scales.max() <= 0x3B9F  # (1 + m/128) 2^-8, m < 32
+    assert len(np.unique(scales)) == 32
+    # the weights' spread is that of the bf16 draws, N(0, 0.02)
+    wf = (O.gen_q4(seed, tid, 512, 256).astype(np.uint32) << 16).view(np.float32)
+    assert abs(float(wf.std()) - 0.02) < 0.001
     w = O.gen_q4(seed, tid, rows, cols)
     for r in (0, 17, 63):
         for c in (0, 31, 32, 199):
