@@ -338,6 +338,7 @@ static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0, bool sls 
     ep.trk = ctx->trk;
     ep.H = c.n_heads;
     ep.Hkv = L.Hkv;
+    ep.v_row0 = qd + L.kvd;
     ep.hd = c.head_dim;
     ep.cap = c.max_ctx;
     ep.q = ctx->q;

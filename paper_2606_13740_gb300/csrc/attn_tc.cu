@@ -175,7 +175,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             mbar_arrive_expect_tx(&qbar, kTcQBytes);
             tma_load_2d(sQ, &maps.q, 0, qrow, &qbar, pol_q);
             tma_load_2d(sQ + kTcQBytes / 2, &maps.q, 64, qrow, &qbar, pol_q);
-            const int krow0 = (b * Hkv + h / (H / Hkv)) * cap + kbeg;  // K/V head of query head h
+            const int krow0 = (b * Hkv + (Hkv == H ? h : h / (H / Hkv))) * cap + kbeg;  // K/V head of query head h
             int kiss = 0, viss = 0;  // sub-blocks whose K, V copies were issued
             for (int j = 0; j < nsub && !s_abort; ++j) {
                 const int st = j % NB;

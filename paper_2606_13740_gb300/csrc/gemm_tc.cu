@@ -196,9 +196,9 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
     if constexpr (EPI == EPI_QKV) {
         // q rows [0, qd), k rows [qd, qd + kvd), v rows [qd + kvd, qd + 2 kvd): the same part for
         // the whole warp (qd and kvd are multiples of 128)
-        const int qd = ep.H * ep.hd, kvd = ep.Hkv * ep.hd;
-        part = row < qd ? 0 : (row < qd + kvd ? 1 : 2);
-        const int f = row - (part == 0 ? 0 : qd + (part - 1) * kvd);
+        const int qd = ep.H * ep.hd;
+        part = row < qd ? 0 : (row < ep.v_row0 ? 1 : 2);
+        const int f = row - (part == 0 ? 0 : (part == 1 ? qd : ep.v_row0));
         hh = f / ep.hd;
         pp = f - hh * ep.hd;
         fi = (pp >> 1) + (pp & 1) * (ep.hd >> 1);
@@ -380,7 +380,7 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
             const int ts = col - b * ep.T;
             const bool tracked = ts >= ep.Tw;  // sparse cache refresh: K/V to the side buffers
             const int pos = tracked ? ep.trk[b * ep.R + ts - ep.Tw] : sm.kvs[b] + ts;
-            const int base = part == 0 ? 0 : ep.H * ep.hd + (part - 1) * ep.Hkv * ep.hd;  // the part's first row
+            const int base = part == 0 ? 0 : (part == 1 ? ep.H * ep.hd : ep.v_row0);  // the part's first row
             const int head = (mt * kBM - base + f0) / ep.hd;
             const int heads = part == 0 ? ep.H : ep.Hkv;  // q: query heads; K/V: the cache's heads
             const int fi0 = f0 % ep.hd;
@@ -856,27 +856,32 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
 // the UMMA descriptor reads: thread t of the 128 writes row t, each weight bf16(d * (q - 8)).
 // 128 + q is built as a bf16 bit pattern (exponent of 128, q in the low mantissa bits), 136 is
 // subtracted exactly and the scale applied with one correctly rounded bf16 multiply.
-__device__ __forceinline__ void q4_expand_row(const uint8_t* raw, uint8_t* dst_tile, int t) {
+__device__ __forceinline__ void q4_expand_row(const uint8_t* __restrict__ raw, uint8_t* __restrict__ dst_tile, int t) {
     const uint32_t* codes = reinterpret_cast<const uint32_t*>(raw);
     const uint16_t* sc = reinterpret_cast<const uint16_t*>(raw + 4096);
+    // every load first (the raw slot and the A stage are both shared memory: loads issued after
+    // a store could not be moved above it), then the arithmetic of all eight chunks, then stores
+    uint32_t w[8];
+#pragma unroll
+    for (int c = 0; c < 8; ++c) w[c] = codes[c * 128 + t];
     const uint32_t s0 = sc[t], s1 = sc[128 + t];
-    const __nv_bfloat162 off = __floats2bfloat162_rn(136.0f, 136.0f);
-    uint8_t* row = dst_tile + t * 128;
+    const uint32_t d0 = s0 | (s0 << 16), d1 = s1 | (s1 << 16);  // (d, d) as bf16x2, per block of 32
+    uint32_t o[8][4];
 #pragma unroll
     for (int c = 0; c < 8; ++c) {
-        const uint32_t w = codes[c * 128 + t];
-        const uint32_t sb = c < 4 ? s0 : s1;
-        const uint32_t sbb = sb | (sb << 16);
-        const __nv_bfloat162 d2 = *reinterpret_cast<const __nv_bfloat162*>(&sbb);
-        uint32_t o[4];
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-            const uint32_t v = ((w >> (4 * j)) & 0x000F000Fu) | 0x43004300u;
-            const __nv_bfloat162 x = __hmul2(__hsub2(*reinterpret_cast<const __nv_bfloat162*>(&v), off), d2);
-            o[j] = *reinterpret_cast<const uint32_t*>(&x);
+            uint32_t v, x;
+            // (w >> 4j) & 0x000F000F | 0x43004300: the bf16 pair (128 + q, 128 + q') of two columns
+            asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(v) : "r"(w[c] >> (4 * j)), "r"(0x000F000Fu), "r"(0x43004300u));
+            asm("sub.rn.bf16x2 %0, %1, %2;" : "=r"(x) : "r"(v), "r"(0x43084308u));           // - (136, 136): exact
+            asm("mul.rn.bf16x2 %0, %1, %2;" : "=r"(o[c][j]) : "r"(x), "r"(c < 4 ? d0 : d1));  // * d: one rounding
         }
-        *reinterpret_cast<uint4*>(row + ((c ^ (t & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
     }
+    uint8_t* row = dst_tile + t * 128;
+#pragma unroll
+    for (int c = 0; c < 8; ++c)
+        *reinterpret_cast<uint4*>(row + ((c ^ (t & 7)) << 4)) = make_uint4(o[c][0], o[c][1], o[c][2], o[c][3]);
 }
 
 template <bool Q4>
@@ -886,10 +891,12 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int S = ca.stages;
     const int R = Q4 ? ca.raw_stages : 0;
+    // 4-bit weights: the operand (B) tiles have a ring of their own, deeper than the A stages
+    const int SB = Q4 ? ca.b_stages : S;
     const uint32_t b_bytes = static_cast<uint32_t>(ca.ntile) * kBK * 2;
     uint8_t* sA = smem;
     uint8_t* sB = sA + static_cast<size_t>(S) * kABytes;
-    uint8_t* sRaw = sB + static_cast<size_t>(S) * b_bytes;  // 4-bit weight tiles (Q4)
+    uint8_t* sRaw = sB + static_cast<size_t>(SB) * b_bytes;  // 4-bit weight tiles (Q4)
     uint8_t* red_stage = sRaw + static_cast<size_t>(R) * kQ4TileBytes;
     float* tail = reinterpret_cast<float*>(red_stage + ca.red_bytes + ca.xs_bytes + ca.stg_bytes);
     EpiSmem esm;
@@ -909,7 +916,9 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
     uint64_t* redbar = drain + 1;  // two partial staging slots
     uint64_t* rfull = redbar + 2;  // raw 4-bit tiles (Q4): arrived / read
     uint64_t* rempty = rfull + R;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(rempty + R);
+    uint64_t* bfull = rempty + R;  // operand tiles of the 4-bit kernel: arrived / consumed
+    uint64_t* bempty = bfull + (Q4 ? SB : 0);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bempty + (Q4 ? SB : 0));
     volatile int* s_abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
     int* s_rows = reinterpret_cast<int*>(tmem_slot + 2);
     esm.rows = s_rows;
@@ -920,14 +929,19 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
     if (threadIdx.x == 0) {
         pdl_launch_dependents();
         for (int s = 0; s < S; ++s) {
-            // Q4: the operand producer's expect-tx arrival plus one arrival per dequantizing warp
-            mbar_init(&full[s], Q4 ? 1 + kDeqWarps : 1);
+            // Q4: one arrival per dequantizing warp (the operand has barriers of its own)
+            mbar_init(&full[s], Q4 ? kDeqWarps : 1);
             mbar_init(&empty[s], 1);
         }
         for (int r = 0; r < R; ++r) {
             mbar_init(&rfull[r], 1);
             mbar_init(&rempty[r], kDeqWarps);
         }
+        if (Q4)
+            for (int b = 0; b < SB; ++b) {
+                mbar_init(&bfull[b], 1);
+                mbar_init(&bempty[b], 1);
+            }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&tfull[a], 1);
             mbar_init(&tempty[a], kEpiThreads);
@@ -1037,6 +1051,7 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
         const int tag = chain_tag(ca);
         int stage = 0;
         uint32_t par = 0;
+        uint32_t bpend = 0, bpend_par = 0;  // Q4: operand copies issued (for the drain on abort)
         bool stop = false;
         if (ca.gate) {  // the bounded-wait test hook (see ChainArgs::gate)
             int open = 1;
@@ -1059,7 +1074,7 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
             int nt = tile / p.m_tiles, mt = tile - nt * p.m_tiles;
             for (int it = it0; it < it1; ++it) {
                 int free_stage = 1;
-                if (lane == 0) free_stage = mbar_wait(&empty[stage], par ^ 1u, s_abort, status) ? 1 : 0;
+                if (lane == 0) free_stage = mbar_wait(Q4 ? &bempty[stage] : &empty[stage], par ^ 1u, s_abort, status) ? 1 : 0;
                 if (!__shfl_sync(0xffffffffu, free_stage, 0)) {  // warp-uniform decision
                     stop = true;
                     break;
@@ -1100,12 +1115,17 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                     }
                 }
                 if (lane == 0) {
-                    if constexpr (Q4) mbar_arrive_expect_tx(&full[stage], b_bytes);  // the A part arrives by warps
-                    tma_load_2d(sB + static_cast<size_t>(stage) * b_bytes, &maps.x[ph], k * kBK, nt * ca.ntile,
-                                &full[stage], pol_x);
+                    uint64_t* fb = Q4 ? &bfull[stage] : &full[stage];
+                    if constexpr (Q4) {  // its own barrier; the A part of the stage arrives by the dequantizers
+                        mbar_arrive_expect_tx(fb, b_bytes);
+                        bpend |= 1u << stage;
+                        bpend_par = (bpend_par & ~(1u << stage)) | (par << stage);
+                    }
+                    tma_load_2d(sB + static_cast<size_t>(stage) * b_bytes, &maps.x[ph], k * kBK, nt * ca.ntile, fb,
+                                pol_x);
                 }
                 __syncwarp();
-                if (++stage == S) {
+                if (++stage == SB) {
                     stage = 0;
                     par ^= 1u;
                 }
@@ -1116,6 +1136,17 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                         ++nt;
                     }
                 }
+            }
+        }
+        if constexpr (Q4) {
+            // the operand ring is this warp's alone: on an abort, let its copies in flight land
+            // before the CTA's shared memory is released (one deadline for all)
+            if (lane == 0 && *s_abort) {
+                const long long t0 = spin_clock();
+                for (int b = 0; b < SB; ++b)
+                    while ((bpend >> b & 1u) && !mbar_try_wait(&bfull[b], (bpend_par >> b) & 1u) &&
+                           spin_clock() - t0 < kWaitLimitCycles) {
+                    }
             }
         }
     } else if (Q4 && warp >= kDeqWarp0) {
@@ -1160,8 +1191,8 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
         // ---------------------------------------------------------- MMA issuer
         if (lane == 0) {
             const uint32_t idesc = umma_idesc_bf16(kBM, ca.ntile);
-            int stage = 0;
-            uint32_t par = 0;
+            int stage = 0, bstage = 0;  // A stage; Q4: the operand's own ring
+            uint32_t par = 0, bpar = 0;
             int acc = 0;
             uint32_t acc_phase = 0;
             bool issued = false;
@@ -1182,7 +1213,8 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                     const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * acc_cols);
                     bool ok = true;
                     for (int k = k_lo; k < k_hi; ++k) {
-                        if (!mbar_wait(&full[stage], par, s_abort, status)) {
+                        if (!mbar_wait(&full[stage], par, s_abort, status) ||
+                            (Q4 && !mbar_wait(&bfull[bstage], bpar, s_abort, status))) {
                             ok = false;
                             break;
                         }
@@ -1190,7 +1222,8 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                         first = false;
                         tc_fence_after();
                         const uint64_t adesc = sw128_kmajor_desc(smem_u32(sA + static_cast<size_t>(stage) * kABytes));
-                        const uint64_t bdesc = sw128_kmajor_desc(smem_u32(sB + static_cast<size_t>(stage) * b_bytes));
+                        const uint64_t bdesc =
+                            sw128_kmajor_desc(smem_u32(sB + static_cast<size_t>(Q4 ? bstage : stage) * b_bytes));
 #pragma unroll
                         for (int kk = 0; kk < kBK / 16; ++kk)
                             umma_bf16(d_tmem, adesc + 2ull * kk, bdesc + 2ull * kk, idesc,
@@ -1200,6 +1233,13 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                         if (++stage == S) {
                             stage = 0;
                             par ^= 1u;
+                        }
+                        if constexpr (Q4) {
+                            umma_commit(&bempty[bstage]);
+                            if (++bstage == SB) {
+                                bstage = 0;
+                                bpar ^= 1u;
+                            }
                         }
                     }
                     if (!ok) break;
@@ -1373,11 +1413,28 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
     // the ring at least 3 stages
     ca.stg_bytes = c32 ? 0 : 32 * kBM * 2;
     ca.xs_bytes = 0;
-    // 4-bit weights: a ring of 8 raw tiles (4.5 KB each and two barriers) in front of the stages
-    const int raw = ca.q4 ? 8 : 0;
-    ca.raw_stages = raw;
-    const int raw_bytes = raw * (kQ4TileBytes + 16);
-    const int fixed0 = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + ca.stg_bytes + 7 * 8 + 16 + raw_bytes;
+    const int fixed0 = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + ca.stg_bytes + 7 * 8 + 16;
+    if (ca.q4) {
+        // 4-bit weights (480 threads: no room beside the CTA for another one, so all of shared
+        // memory): raw 4.5 KB tiles, a few bf16 A stages the dequantizers fill, and a ring of
+        // operand tiles of its own, as deep as what is left allows (2 .. 24)
+        static const int kRaw[3] = {12, 8, 6}, kA[3] = {4, 3, 2};
+        const int b_stage = ntile * kBK * 2 + 16;
+        for (int i = 0; i < 3; ++i) {
+            const int fixed = fixed0 + kRaw[i] * (kQ4TileBytes + 16) + kA[i] * (static_cast<int>(kABytes) + 16);
+            const int sb = (kFullSmem - fixed) / b_stage;
+            if (sb >= 2 || i == 2) {
+                ca.raw_stages = kRaw[i];
+                ca.stages = kA[i];
+                ca.b_stages = sb > 24 ? 24 : sb;
+                ca.smem = static_cast<size_t>(fixed) + static_cast<size_t>(ca.b_stages) * b_stage;
+                break;
+            }
+        }
+        return ca.b_stages >= 2 && ca.smem <= static_cast<size_t>(kFullSmem);
+    }
+    ca.raw_stages = 0;
+    ca.b_stages = 0;
     if (ca.x_cols == 0 && (smem_budget - fixed0 - 2 * 32 * kBM * 4) / (stage_bytes + 16) >= 3)
         ca.xs_bytes = 2 * 32 * kBM * 4;
     const int fixed = fixed0 + ca.xs_bytes;
@@ -1409,7 +1466,7 @@ cudaError_t chain_launch(const ChainMaps& maps, const ChainArgs& ca, cudaStream_
     if (ca.q4) {  // every phase's weights in the 4-bit tile format
         for (int i = 0; i < ca.n_phases; ++i)
             if (!ca.ph[i].w_tiles) return cudaErrorInvalidValue;
-        if (ca.raw_stages < 2 || ca.raw_stages > 32) return cudaErrorInvalidValue;
+        if (ca.raw_stages < 2 || ca.raw_stages > 32 || ca.b_stages < 2 || ca.b_stages > 32) return cudaErrorInvalidValue;
         return launch_k(k_chain<true>, dim3(ca.grid), dim3(kChainThreadsQ4), ca.smem, st, pdl, maps, ca);
     }
     return launch_k(k_chain<false>, dim3(ca.grid), dim3(kChainThreads), ca.smem, st, pdl, maps, ca);

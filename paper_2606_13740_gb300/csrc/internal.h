@@ -65,6 +65,7 @@ struct EpiArgs {
     const int* seq_kv;   // per-sequence first window position (kv_len)
     int T, H, hd, cap;
     int Hkv;             // K/V heads (a multiple of 128 / hd rows each part: Hkv * hd % 128 == 0)
+    int v_row0;          // first v row: qd + Hkv * hd
     int n_seq;           // sequences (B), <= 256
     const float* theta;  // [hd/2]: rotation of feature pair j at position p is p * theta[j]
     // EPI_SWIGLU: tile k row 2f is gate feature 64k+f, row 2f+1 the matching up row
@@ -123,8 +124,8 @@ struct ChainPhase {
     int* tickets;        // [m_tiles*n_tiles][32], zero between launches
     // non-null: the weights are stored tile-major (tiled_index) and each 16 KB tile arrives with
     // one contiguous bulk copy; null: row-major [M][K] through the chain's tensor map.  In a
-    // 4-bit chain (ChainArgs::q4) the tiles are kQ4TileBytes each, laid out as q4_tile_word /
-    // q4_tile_scale describe.
+    // 4-bit chain (ChainArgs::q4) the tiles are kQ4TileBytes each, laid out as described at
+    // kQ4TileBytes.
     const void* w_tiles;
 };
 struct ChainArgs {
@@ -147,10 +148,10 @@ struct ChainArgs {
     // launch's tag before its first load.  Given a word nobody writes, that wait runs out after
     // kWaitLimitCycles and the launch unwinds with kStatusTimeout, as any stalled wait would.
     const int* gate;
-    // 4-bit weights (the block format of Q4_0, see q4_tile_word): the weight producer streams
-    // raw 4.5 KB tiles into raw_stages slots, and four more warps expand each into the bf16
-    // A stage the tensor cores read
-    int q4, raw_stages;
+    // 4-bit weights (the block format of Q4_0, see kQ4TileBytes): the weight producer streams
+    // raw 4.5 KB tiles into raw_stages slots, four more warps expand each into the bf16 A stage
+    // the tensor cores read, and the operand tiles go through a ring of b_stages of their own
+    int q4, raw_stages, b_stages;  // b_stages: the operand ring of the 4-bit kernel
     ChainPhase ph[kMaxPhases];
 };
 struct ChainMaps {

@@ -333,7 +333,7 @@ __global__ void __launch_bounds__(PR * NW * 32) k_attn(const __nv_bfloat16* __re
 
     const __nv_bfloat16* qbase = q + ((static_cast<size_t>(b) * H + h) * T + q0) * HD;
     // grouped-query attention: query head h reads K/V head h / (H / Hkv)
-    const int hk = h / (H / Hkv);
+    const int hk = Hkv == H ? h : h / (H / Hkv);
     const __nv_bfloat16* kbase = kc + (static_cast<size_t>(b) * Hkv + hk) * cap * HD;
     const __nv_bfloat16* vbase = vc + (static_cast<size_t>(b) * Hkv + hk) * cap * HD;
 
