@@ -28,6 +28,7 @@ def main(argv=None):
     ap.add_argument("--H", type=int, default=32)
     ap.add_argument("--P", type=int, default=4096)
     ap.add_argument("--reps", type=int, default=3)
+    ap.add_argument("--weight-bits", type=int, default=16, help="step-small: 16 (bf16) or 4 (4-bit block format)")
     a = ap.parse_args(argv)
     lib()
     if a.op == "step-small":
@@ -64,14 +65,15 @@ def main(argv=None):
 
 def step_small(a):
     """A few denoising steps of a 2-layer model at the LLaDA-8B width (about 3 GB on the device):
-    the small case for ncu captures of the step's kernels."""
+    the small case for ncu captures of the step's kernels (--weight-bits 4: the projections in
+    the 4-bit block format)."""
     import numpy as np
 
     from .dllm import Config, Context, Sched
 
     shape = dict(n_layers=2, d_model=4096, n_heads=32, head_dim=128, ffn=12288, vocab=126464, mask_id=126463,
                  rope_base=500000.0)
-    ctx = Context(Config(max_batch=1, max_ctx=544, max_window=512, **shape))
+    ctx = Context(Config(max_batch=1, max_ctx=544, max_window=512, weight_bits=a.weight_bits, **shape))
     rng = np.random.default_rng(1)
     ctx.dllm_prefill(Sched(steps_per_block=24), rng.integers(0, 126463, 512).astype(np.int32), 32)
     ctx.dllm_begin_block()
