@@ -530,7 +530,7 @@ __device__ __forceinline__ bool wait_flag(const int* flag, int tag, volatile int
 }
 
 // The epilogue warps' share of one phase: every tile of this CTA's range.
-template <int EPI>
+template <int EPI, int DP>
 __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph, int tag, uint8_t* red_stage,
                                                   uint64_t* tfull, uint64_t* tempty, uint64_t* redbar,
                                                   volatile int* s_abort, uint32_t tmem_base, const EpiSmem& esm,
@@ -759,8 +759,13 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                     inflight |= 1u << sl;
                 }
             };
+            // A 32-token tile (one chunk) skips the staging: each thread's 16 columns of its row of
+            // every part come straight into registers, up to DP parts at a time once
+            // their flags are seen, so the parts cost one round trip to L2 instead of a copy each
+            // (the same sum, in the same order, bit for bit).
+            const bool direct = nchunks == 1;
             if (tr && threadIdx.x == 64) tr[kTrPartStored] = global_ns();
-            if (ew == 0) {
+            if (ew == 0 && !direct) {
                 if (nslices > 0) issue(0);
                 if (nslices > 1) issue(1);
             }
@@ -768,7 +773,53 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             int si = 0;
             for (int c = 0; c < nchunks && !stop; ++c) {
                 tmem_ld_32x16(t_acc + static_cast<uint32_t>(c * 32 + half * 16), v);  // own (first) k-range
-                for (int q = 1; q < nparts; ++q, ++si) {
+                for (int q0 = 1; direct && q0 < nparts; q0 += DP) {
+                    const int qn = min(DP, nparts - q0);
+                    if (ew == 0) {  // lane i polls part i's flag: one round trip covers the group
+                        const long long t0 = spin_clock();
+                        for (;;) {
+                            const bool ok = lane < q0 || lane >= q0 + qn || ld_acquire(flags + lane) == tag;
+                            if (__all_sync(0xffffffffu, ok)) break;
+                            int give_up = 0;
+                            if (lane == 0) give_up = (*s_abort || spin_clock() - t0 > kWaitLimitCycles) ? 1 : 0;
+                            if (__shfl_sync(0xffffffffu, give_up, 0)) {  // warp-uniform decision
+                                if (lane == 0 && !*s_abort) {
+                                    *s_abort = 1;
+                                    atomicOr(status, kStatusTimeout);
+                                }
+                                break;
+                            }
+                            __nanosleep(32);
+                        }
+                    }
+                    if (named_bar_any(1, kEpiThreads, *s_abort != 0)) {
+                        stop = true;
+                        break;
+                    }
+                    // L2 only (.cg): other CTAs wrote these lines, and the next launch writes the
+                    // same slots again.  A group's loads go out unconditionally (the slot index held
+                    // at the last part), its adds stop at the group's last part.
+                    float4 a[DP][4];
+#pragma unroll
+                    for (int g = 0; g < DP; ++g) {
+                        const float4* src = reinterpret_cast<const float4*>(
+                            P.partials + static_cast<size_t>(min(c_first + q0 + g, c_last)) * slot_floats);
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) a[g][j] = __ldcg(src + static_cast<size_t>(half * 4 + j) * kBM + rt);
+                    }
+#pragma unroll
+                    for (int g = 0; g < DP; ++g)
+                        if (g < qn) {
+#pragma unroll
+                            for (int j = 0; j < 4; ++j) {
+                                v[4 * j] += a[g][j].x;
+                                v[4 * j + 1] += a[g][j].y;
+                                v[4 * j + 2] += a[g][j].z;
+                                v[4 * j + 3] += a[g][j].w;
+                            }
+                        }
+                }
+                for (int q = 1; !direct && q < nparts; ++q, ++si) {
                     const int sl = si & 1;
                     mbar_wait(redbar + sl, (es.red_phase >> sl) & 1u, s_abort, status);
                     es.red_phase ^= 1u << sl;
@@ -1264,22 +1315,25 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
         pdl_wait();
         const int tag = chain_tag(ca);
         ChainEpiState es{0, 0u, 0u};
+        // split 32-token tiles: parts whose rows are loaded into registers at once (the 4-bit
+        // kernel's smaller register budget takes two)
+        constexpr int kDP = Q4 ? 2 : 4;
         for (int ph = 0; ph < ca.n_phases; ++ph) {  // on abort every phase returns at its first barrier
             switch (ca.ph[ph].epi) {
                 case EPI_F32:
-                    chain_phase_epilogue<EPI_F32>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    chain_phase_epilogue<EPI_F32, kDP>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
                     break;
                 case EPI_RESID:
-                    chain_phase_epilogue<EPI_RESID>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    chain_phase_epilogue<EPI_RESID, kDP>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
                     break;
                 case EPI_QKV:
-                    chain_phase_epilogue<EPI_QKV>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    chain_phase_epilogue<EPI_QKV, kDP>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
                     break;
                 case EPI_SWIGLU:
-                    chain_phase_epilogue<EPI_SWIGLU>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    chain_phase_epilogue<EPI_SWIGLU, kDP>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
                     break;
                 default:
-                    chain_phase_epilogue<EPI_LMHEAD>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+                    chain_phase_epilogue<EPI_LMHEAD, kDP>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
                     break;
             }
         }
