@@ -407,8 +407,22 @@ static int forward(dllm_ctx* ctx, int B, int Tw, bool head, int R = 0, bool sls 
     }
     for (int l = 0; l < c.n_layers; ++l) {
         const EpiArgs el = qkv_args(l);
+        // The mma.sync attention starts per (sequence, head) on the QKV tiles it reads: layer 0's
+        // come from the QKV chain (phase slot 0, tag 1), layer l's from phase slot 3 of layer
+        // l-1's chain (tag l + 1).
+        AttnSync sy{};
+        if (!ap.tc) {
+            sy.qkv_done = ctx->chain_done + static_cast<size_t>(l == 0 ? 0 : 3) * L.done_len;
+            sy.qkv_ntile = pq.ntile;
+            sy.qkv_ntiles = pq.n_tiles;
+            sy.k_row0 = qd;
+            sy.v_row0 = qd + L.kvd;
+            sy.epoch = ctx->epoch;
+            sy.tag_mul = c.n_layers + 2;
+            sy.tag_add = l + 1;
+        }
         CK(launch_attention(ctx->q, el.kc, el.vc, ctx->seq_kv, ctx->attn, B, T, c.n_heads, L.Hkv, c.head_dim, c.max_ctx,
-                            ap, s, true, next_trace(ctx), ctx->status));
+                            ap, s, true, next_trace(ctx), ctx->status, &sy));
         mark(ctx, DLLM_K_ATTN);
         // output projection (+ residual) -> gate/up (+ SwiGLU) -> down (+ residual) -> next QKV or LM head
         ChainArgs ca{};

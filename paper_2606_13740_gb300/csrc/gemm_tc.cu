@@ -166,6 +166,77 @@ __device__ __forceinline__ void warp_reduce_scatter(float* v, int lane) {
     for (int w = 16 / N; w >= 1; w >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], w);
 }
 
+// What a QKV epilogue thread needs besides the accumulator, from the tile and chunk alone: its
+// row's part (q, K or V) and position in the head, the rotation at its first column and the
+// per-column step (angle addition along the positions, when all 32 columns are consecutive
+// positions of one sequence's window), and the 32-byte store it makes after the staging (token
+// t/8, tile features 16 (t%8) .. +15: part of one head's run at the token's row of the q
+// tensor, the K/V cache or, for tracked prefix rows, the side buffers).  A finisher that waits
+// for other parts of its tile builds it before the wait.
+struct QkvPlan {
+    int part, pp, fi, bl;
+    bool run;
+    float cn, sn, cd, sd, theta;
+    uint4* dst;  // null: no store
+    bool bad;    // a window position outside the cache
+};
+__device__ __forceinline__ QkvPlan qkv_plan(const EpiArgs& ep, const GemmPlan& p, int mt, int col0, int rt,
+                                            const EpiSmem& sm, int e, int half) {
+    QkvPlan q;
+    const int row = mt * kBM + rt;
+    // q rows [0, qd), k rows [qd, qd + kvd), v rows [qd + kvd, qd + 2 kvd): the same part for
+    // the whole tile (qd and kvd are multiples of 128)
+    const int qd = ep.H * ep.hd;
+    q.part = row < qd ? 0 : (row < ep.v_row0 ? 1 : 2);
+    const int f = row - (q.part == 0 ? 0 : (q.part == 1 ? qd : ep.v_row0));
+    q.pp = f % ep.hd;
+    q.fi = (q.pp >> 1) + (q.pp & 1) * (ep.hd >> 1);
+    q.theta = sm.theta[rt];
+    q.bl = col0 / ep.T;
+    q.run = min(col0 + 31, p.N - 1) / ep.T == q.bl && min(col0 + 31, p.N - 1) - q.bl * ep.T < ep.Tw;
+    q.cn = 1.0f;
+    q.sn = 0.0f;
+    q.cd = 1.0f;
+    q.sd = 0.0f;
+    if (q.part < 2 && q.run) {
+        const float2 a = rot_cs(static_cast<float>(sm.kvs[q.bl] + (col0 + kEpiGroup * half - q.bl * ep.T)) * q.theta);
+        const float2 d = rot_cs(q.theta);
+        q.cn = a.x;
+        q.sn = a.y;
+        q.cd = d.x;
+        q.sd = d.y;
+    }
+    const int tok = e >> 3, f0 = (e & 7) * 16;
+    const int col = col0 + tok;
+    q.dst = nullptr;
+    q.bad = false;
+    if (col < p.N) {
+        const int b = min(col / ep.T, ep.n_seq - 1);
+        const int ts = col - b * ep.T;
+        const bool tracked = ts >= ep.Tw;  // sparse cache refresh: K/V to the side buffers
+        const int pos = tracked ? ep.trk[b * ep.R + ts - ep.Tw] : sm.kvs[b] + ts;
+        const int base = q.part == 0 ? 0 : (q.part == 1 ? qd : ep.v_row0);  // the part's first row
+        const int head = (mt * kBM - base + f0) / ep.hd;
+        const int heads = q.part == 0 ? ep.H : ep.Hkv;  // q: query heads; K/V: the cache's heads
+        const int fi0 = f0 % ep.hd;
+        if (tracked && q.part > 0) {
+            if (pos >= 0) {
+                __nv_bfloat16* side = q.part == 1 ? ep.kside : ep.vside;
+                q.dst = reinterpret_cast<uint4*>(
+                    side + ((static_cast<size_t>(b) * heads + head) * ep.R + (ts - ep.Tw)) * ep.hd + fi0);
+            }
+        } else if (tracked || (pos >= 0 && pos < ep.cap)) {
+            const size_t plane = q.part == 0 ? static_cast<size_t>(ep.T) : static_cast<size_t>(ep.cap);
+            const size_t r = (static_cast<size_t>(b) * heads + head) * plane + (q.part == 0 ? ts : pos);
+            __nv_bfloat16* base_ptr = q.part == 0 ? ep.q : (q.part == 1 ? ep.kc : ep.vc);
+            q.dst = reinterpret_cast<uint4*>(base_ptr + r * ep.hd + fi0);
+        } else {
+            q.bad = true;
+        }
+    }
+    return q;
+}
+
 // Epilogue of a 32-token chunk, compact: each epilogue thread takes its TMEM lane (tile row)
 // and one half of the chunk, 16 columns read from TMEM (t_src; for the residual, the old x of
 // a narrow tile was staged at t_x before the accumulator was ready), so its code stays small
@@ -178,43 +249,36 @@ __device__ __forceinline__ void warp_reduce_scatter(float* v, int lane) {
 template <int EPI, int PASS = 0>
 __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& p, int mt, int col0, int c_in,
                                              int rt, uint32_t t_src, uint32_t t_x, const float* xs, const EpiSmem& sm,
-                                             int e, int half, int quarter, int lane, int* status) {
+                                             int e, int half, int quarter, int lane, int* status,
+                                             const float* a_in = nullptr, const QkvPlan* qkv_pre = nullptr) {
     // col0: the chunk's first token column; c_in: its offset inside the token tile (index into
-    // the tile's RMSNorm scales and staged ids).  The old residual (pass 1) comes from TMEM
-    // (t_x), else from shared memory (xs, the chunk's staged copy), else from global; pass 1
-    // leaves the new residual in the accumulator, where pass 2 reads it.  e: the epilogue
-    // thread (0 .. kEpiThreads-1), half: which 16 columns of the chunk.
+    // the tile's RMSNorm scales and staged ids).  The thread's 16 accumulator columns come from
+    // a_in (a finisher's sum of the parts, in registers), else from TMEM at t_src.  The old
+    // residual (pass 1) comes from TMEM (t_x), else from shared memory (xs, the chunk's staged
+    // copy), else from global; pass 1 leaves the new residual in the accumulator, where pass 2
+    // reads it.  e: the epilogue thread (0 .. kEpiThreads-1), half: which 16 columns of the
+    // chunk.  qkv_pre: the QKV plan, built ahead (null: built here).
     constexpr int GW = kEpiGroup;  // columns per group
     constexpr int LS = 32 / GW;    // lanes sharing one column's sum after the scatter
     const int row = mt * kBM + rt;
     const bool scale = (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) && ep.sq_in != nullptr;
-    // QKV state: feature, head, rotation (angle-addition recurrence along the positions)
-    int part = 0, hh = 0, pp = 0, fi = 0, bl = 0;
+    QkvPlan qp;
+    if constexpr (EPI == EPI_QKV) qp = qkv_pre ? *qkv_pre : qkv_plan(ep, p, mt, col0, rt, sm, e, half);
+    // QKV state: feature, rotation (angle-addition recurrence along the positions)
+    int part = 0, pp = 0, fi = 0, bl = 0;
     bool run = true;
     float cn = 1.0f, sn = 0.0f, cd = 1.0f, sd = 0.0f, theta = 0.0f;
-    __nv_bfloat16* qkv_dst = nullptr;
     if constexpr (EPI == EPI_QKV) {
-        // q rows [0, qd), k rows [qd, qd + kvd), v rows [qd + kvd, qd + 2 kvd): the same part for
-        // the whole warp (qd and kvd are multiples of 128)
-        const int qd = ep.H * ep.hd;
-        part = row < qd ? 0 : (row < ep.v_row0 ? 1 : 2);
-        const int f = row - (part == 0 ? 0 : (part == 1 ? qd : ep.v_row0));
-        hh = f / ep.hd;
-        pp = f - hh * ep.hd;
-        fi = (pp >> 1) + (pp & 1) * (ep.hd >> 1);
-        theta = sm.theta[rt];
-        bl = col0 / ep.T;
-        // all 32 columns in one sequence's window (consecutive positions)
-        run = min(col0 + 31, p.N - 1) / ep.T == bl && min(col0 + 31, p.N - 1) - bl * ep.T < ep.Tw;
-        qkv_dst = part == 0 ? ep.q : (part == 1 ? ep.kc : ep.vc);
-        if (part < 2 && run) {
-            const float2 a = rot_cs(static_cast<float>(sm.kvs[bl] + (col0 + GW * half - bl * ep.T)) * theta);
-            const float2 d = rot_cs(theta);
-            cn = a.x;
-            sn = a.y;
-            cd = d.x;
-            sd = d.y;
-        }
+        part = qp.part;
+        pp = qp.pp;
+        fi = qp.fi;
+        bl = qp.bl;
+        run = qp.run;
+        cn = qp.cn;
+        sn = qp.sn;
+        cd = qp.cd;
+        sd = qp.sd;
+        theta = qp.theta;
     }
     bool lm_ok = false;
     if constexpr (EPI == EPI_LMHEAD) lm_ok = row < ep.V && row != ep.mask_id;
@@ -224,7 +288,12 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
 
         const int cg = col0 + GW * g;  // first column of the group
         float a[GW];
-        tmem_ld_32xn<GW>(t_src + static_cast<uint32_t>(GW * g), a);
+        if (a_in) {
+#pragma unroll
+            for (int u = 0; u < GW; ++u) a[u] = a_in[u];
+        } else {
+            tmem_ld_32xn<GW>(t_src + static_cast<uint32_t>(GW * g), a);
+        }
         if (scale) {
 #pragma unroll
             for (int u = 0; u < GW; ++u) a[u] *= sm.rs[c_in + GW * g + u];
@@ -369,44 +438,16 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
         }
     }
     if constexpr (EPI == EPI_QKV) {
-        // thread t stores token t/8, tile features 16 (t%8) .. +15: part of one head's
-        // contiguous run at the token's row of the q tensor or of the K/V cache
+        // thread t stores token t/8, tile features 16 (t%8) .. +15 (the plan's destination)
         named_bar(1, kEpiThreads);
-        const int t = e, tok = t >> 3, f0 = (t & 7) * 16;
-        const int col = col0 + tok;
-        bool bad = false;
-        if (col < p.N) {
-            const int b = min(col / ep.T, ep.n_seq - 1);
-            const int ts = col - b * ep.T;
-            const bool tracked = ts >= ep.Tw;  // sparse cache refresh: K/V to the side buffers
-            const int pos = tracked ? ep.trk[b * ep.R + ts - ep.Tw] : sm.kvs[b] + ts;
-            const int base = part == 0 ? 0 : (part == 1 ? ep.H * ep.hd : ep.v_row0);  // the part's first row
-            const int head = (mt * kBM - base + f0) / ep.hd;
-            const int heads = part == 0 ? ep.H : ep.Hkv;  // q: query heads; K/V: the cache's heads
-            const int fi0 = f0 % ep.hd;
-            if (tracked && part > 0) {
-                if (pos >= 0) {
-                    const uint4* src = reinterpret_cast<const uint4*>(
-                        reinterpret_cast<const __nv_bfloat16*>(sm.stg) + tok * kBM + f0);
-                    __nv_bfloat16* side = part == 1 ? ep.kside : ep.vside;
-                    uint4* dst = reinterpret_cast<uint4*>(
-                        side + ((static_cast<size_t>(b) * heads + head) * ep.R + (ts - ep.Tw)) * ep.hd + fi0);
+        if (qp.dst) {
+            const int t = e, tok = t >> 3, f0 = (t & 7) * 16;
+            const uint4* src =
+                reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(sm.stg) + tok * kBM + f0);
 #pragma unroll
-                    for (int i = 0; i < 2; ++i) dst[i] = src[i];
-                }
-            } else if (tracked || (pos >= 0 && pos < ep.cap)) {
-                const size_t plane = part == 0 ? static_cast<size_t>(ep.T) : static_cast<size_t>(ep.cap);
-                const size_t r = (static_cast<size_t>(b) * heads + head) * plane + (part == 0 ? ts : pos);
-                const uint4* src = reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(sm.stg) +
-                                                                  tok * kBM + f0);
-                uint4* dst = reinterpret_cast<uint4*>(qkv_dst + r * ep.hd + fi0);
-#pragma unroll
-                for (int i = 0; i < 2; ++i) dst[i] = src[i];
-            } else {
-                bad = true;
-            }
+            for (int i = 0; i < 2; ++i) qp.dst[i] = src[i];
         }
-        if (bad) atomicOr(status, kStatusBadIndex);
+        if (qp.bad) atomicOr(status, kStatusBadIndex);
         named_bar(1, kEpiThreads);  // the staging memory is free again
     } else if constexpr (EPI == EPI_SWIGLU) {
         // thread t stores token t/8, features 8 (t%8) .. +7 of the tile's 64
@@ -765,6 +806,11 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             // (the same sum, in the same order, bit for bit).
             const bool direct = nchunks == 1;
             if (tr && threadIdx.x == 64) tr[kTrPartStored] = global_ns();
+            // the QKV plan of a one-chunk tile does not need the sum: built while the parts arrive
+            QkvPlan qpre;
+            if constexpr (EPI == EPI_QKV) {
+                if (direct) qpre = qkv_plan(ep, p, mt, nt * p.ntile, rt, esm, e, half);
+            }
             if (ew == 0 && !direct) {
                 if (nslices > 0) issue(0);
                 if (nslices > 1) issue(1);
@@ -845,13 +891,13 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                     tr[kTrReduced] = global_ns();
                     tr[kTrIsLast] = 1;
                 }
-                // the sum goes back into the (still owned) accumulator, then the compact epilogue
-                tmem_st_32x16(t_acc + static_cast<uint32_t>(c * 32 + half * 16), v);
+                // the compact epilogue on the sum in registers (the residual's first pass leaves the
+                // new residual in the still owned accumulator, for the second)
                 const float* xs = x_chunk(mt, nt, c);
                 epilogue_c32<EPI, kPass1>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt,
                                           t_acc + static_cast<uint32_t>(c * 32),
                                           t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, xs, esm, e, half, quarter,
-                                          lane, status);
+                                          lane, status, v, (EPI == EPI_QKV && direct) ? &qpre : nullptr);
             }
             if (threadIdx.x == 64) {
                 if (stop) {  // let copies in flight land before the shared memory is released

@@ -242,6 +242,20 @@ struct AttnPlan {
     bool tc;    // head dim 128: the tcgen05 kernel (128-row query tiles, 64-key sub-blocks)
     int qx;     // the last qx of a sequence's T rows are queries only: keys = kv_len + T - qx
 };
+// Finer ordering of the mma.sync attention after the chained projections that computed its
+// q/K/V (null: the whole preceding grid, by griddepcontrol.wait).  The attention of a
+// (sequence, head) starts once the QKV phase has published the tiles holding query head h's
+// rows, K head hk's and V head hk's for the sequence's token columns; before it exits, the
+// CTA still waits for the whole preceding grid, so a kernel ordered after the attention by
+// griddepcontrol.wait stays ordered after that grid too.
+struct AttnSync {
+    const int* qkv_done;  // the QKV phase's tile flags, [m-tile][token tile]
+    int qkv_ntile;        // token columns per token tile
+    int qkv_ntiles;       // token tiles
+    int k_row0, v_row0;   // first K row, first V row of the fused QKV output
+    const int* epoch;     // the flags' tag: *epoch * tag_mul + tag_add (the chain's tagging)
+    int tag_mul, tag_add;
+};
 // head dim 128 and at least kTcMinKeys keys: the tcgen05 kernel's plan; otherwise the
 // mma.sync kernel's
 constexpr int kTcMinKeys = 1024;
@@ -256,7 +270,8 @@ cudaError_t launch_attention_tc(const __nv_bfloat16* q, const __nv_bfloat16* kc,
 cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
                              const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int Hkv, int hd, int cap,
                              const AttnPlan& a, cudaStream_t st, bool pdl = true,
-                             unsigned long long* trace = nullptr, int* status = nullptr);
+                             unsigned long long* trace = nullptr, int* status = nullptr,
+                             const AttnSync* sync = nullptr);
 cudaError_t launch_lmhead_reduce(const float* lm_part, const float* zcur, const int* cur_tok, int m_tiles,
                                  int N, int mask_id, int* x0, float* conf, float* tokconf, cudaStream_t st,
                                  bool pdl = true, const int* row_map = nullptr, const int* n_rows = nullptr);

@@ -295,7 +295,8 @@ __global__ void __launch_bounds__(PR * NW * 32) k_attn(const __nv_bfloat16* __re
                                                        const __nv_bfloat16* __restrict__ vc,
                                                        const int* __restrict__ seq_kv, __nv_bfloat16* __restrict__ out,
                                                        int T, int H, int Hkv, int cap, int qtiles, int csize,
-                                                       int qx, unsigned long long* trace) {
+                                                       int qx, unsigned long long* trace, const AttnSync sy,
+                                                       int* status) {
     constexpr int AQ = NW * 16;  // query rows per CTA
     constexpr int NT = NW * 32;  // threads of one warp group
     constexpr int PART = (AQ + 2 * NB * kAK) * HD * 2;  // one group's Q, K, V tiles
@@ -342,7 +343,39 @@ __global__ void __launch_bounds__(PR * NW * 32) k_attn(const __nv_bfloat16* __re
         else named_bar(1 + grp, NT);
     };
     const bool prefix_first = attn_prefetch_prefix<HD, NT>(kbase, vbase, kv, kbeg, kend, sK, sV, tid);
-    pdl_wait();
+    if (sy.qkv_done) {
+        // the QKV tiles holding this sequence's window rows of q head h, K head hk and V head hk.
+        // On a timeout the status word records it and the CTA goes on (its cluster peers wait
+        // for it at the merge); the launch's result is then discarded.
+        // Warp 0 polls them side by side, one flag per lane (q, K, V for each token tile).
+        if (threadIdx.x < 32) {
+            const int tag = *reinterpret_cast<const volatile int*>(sy.epoch) * sy.tag_mul + sy.tag_add;
+            const int nt0 = (b * T) / sy.qkv_ntile, nts = (b * T + T - 1) / sy.qkv_ntile - nt0 + 1;
+            const int lane = threadIdx.x;
+            for (int f0 = 0; f0 < 3 * nts; f0 += 32) {
+                const int fi = f0 + lane;
+                const int* f = nullptr;
+                if (fi < 3 * nts) {
+                    const int which = fi / nts, nt = nt0 + fi - which * nts;
+                    const int row = which == 0 ? h * HD : (which == 1 ? sy.k_row0 : sy.v_row0) + hk * HD;
+                    f = sy.qkv_done + static_cast<size_t>(row / 128) * sy.qkv_ntiles + nt;
+                }
+                const long long t0 = spin_clock();
+                for (;;) {
+                    const bool ok = !f || ld_acquire(f) == tag;
+                    if (__all_sync(0xffffffffu, ok)) break;
+                    if (spin_clock() - t0 > kWaitLimitCycles) {  // warp-uniform (one clock read)
+                        if (!ok && status) atomicOr(status, kStatusTimeout);
+                        break;
+                    }
+                    __nanosleep(32);
+                }
+            }
+        }
+        __syncthreads();
+    } else {
+        pdl_wait();
+    }
     if (tr) tr[kAtDepWait] = global_ns();
     constexpr int DN = HD / 8;  // output n-blocks
     float o[DN][4];
@@ -402,6 +435,7 @@ __global__ void __launch_bounds__(PR * NW * 32) k_attn(const __nv_bfloat16* __re
                         __floats2bfloat162_rn(o[dn][2] * i1, o[dn][3] * i1);
             }
         }
+        if (sy.qkv_done && threadIdx.x == 0) pdl_wait();  // see AttnSync
         return;
     }
     // the CTA's partial into the first group's shared memory (its Q/K/V tiles are done)
@@ -480,6 +514,7 @@ __global__ void __launch_bounds__(PR * NW * 32) k_attn(const __nv_bfloat16* __re
     if (tr) tr[kAtMergeLoop] = global_ns();
     cluster_sync_all();  // no CTA leaves while its partials may still be read
     if (tr) tr[kAtMerged] = global_ns();
+    if (sy.qkv_done && threadIdx.x == 0) pdl_wait();  // see AttnSync
 }
 
 static size_t attn_smem(int nw, int nb, int pr, int hd) {
@@ -542,17 +577,23 @@ AttnPlan attn_plan(int B, int T, int H, int hd, int max_keys, int sms) {
 template <int HD, int NW, int NB, int PR>
 static cudaError_t attn_go(cudaLaunchConfig_t& cfg, const __nv_bfloat16* q, const __nv_bfloat16* kc,
                            const __nv_bfloat16* vc, const int* seq_kv, __nv_bfloat16* out, int T, int H, int Hkv,
-                           int cap, const AttnPlan& a, unsigned long long* trace) {
+                           int cap, const AttnPlan& a, unsigned long long* trace, const AttnSync& sy, int* status) {
     cfg.blockDim = dim3(PR * NW * 32);
     cfg.dynamicSmemBytes = attn_smem(NW, NB, PR, HD);
     return cudaLaunchKernelEx(&cfg, k_attn<HD, NW, NB, PR>, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a.qtiles, a.csize,
-                              a.qx, trace);
+                              a.qx, trace, sy, status);
 }
 
 cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, const __nv_bfloat16* vc,
                              const int* seq_kv, __nv_bfloat16* out, int B, int T, int H, int Hkv, int hd, int cap,
-                             const AttnPlan& a, cudaStream_t st, bool pdl, unsigned long long* trace, int* status) {
+                             const AttnPlan& a, cudaStream_t st, bool pdl, unsigned long long* trace, int* status,
+                             const AttnSync* sync) {
     if (Hkv < 1 || H % Hkv) return cudaErrorInvalidValue;
+    AttnSync sy{};
+    if (sync && sync->qkv_done) {
+        if (!sync->epoch || sync->qkv_ntile < 1 || sync->qkv_ntiles < 1) return cudaErrorInvalidValue;
+        sy = *sync;
+    }
     if (a.tc) {
         if (hd != 128) return cudaErrorInvalidValue;
         return launch_attention_tc(q, kc, vc, seq_kv, out, B, T, H, Hkv, cap, a, st, pdl, trace, status);
@@ -578,18 +619,18 @@ cudaError_t launch_attention(const __nv_bfloat16* q, const __nv_bfloat16* kc, co
     cfg.attrs = at;
     cfg.numAttrs = n;
     if (a.pairs == 2)
-        return hd == 128 ? attn_go<128, 2, 1, 2>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace)
-                         : attn_go<64, 2, 1, 2>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
+        return hd == 128 ? attn_go<128, 2, 1, 2>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace, sy, status)
+                         : attn_go<64, 2, 1, 2>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace, sy, status);
     const int key = (hd == 128 ? 4 : 0) + (a.nw == 4 ? 2 : 0) + (a.nb == 2 ? 1 : 0);
     switch (key) {
-        case 0: return attn_go<64, 2, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
-        case 1: return attn_go<64, 2, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
-        case 2: return attn_go<64, 4, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
-        case 3: return attn_go<64, 4, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
-        case 4: return attn_go<128, 2, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
-        case 5: return attn_go<128, 2, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
-        case 6: return attn_go<128, 4, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
-        default: return attn_go<128, 4, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace);
+        case 0: return attn_go<64, 2, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace, sy, status);
+        case 1: return attn_go<64, 2, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace, sy, status);
+        case 2: return attn_go<64, 4, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace, sy, status);
+        case 3: return attn_go<64, 4, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace, sy, status);
+        case 4: return attn_go<128, 2, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace, sy, status);
+        case 5: return attn_go<128, 2, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace, sy, status);
+        case 6: return attn_go<128, 4, 1, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace, sy, status);
+        default: return attn_go<128, 4, 2, 1>(cfg, q, kc, vc, seq_kv, out, T, H, Hkv, cap, a, trace, sy, status);
     }
 }
 
