@@ -570,6 +570,32 @@ __device__ __forceinline__ bool wait_flag(const int* flag, int tag, volatile int
     return true;
 }
 
+// A finisher's wait for parts q0 .. q0+qn-1 of its tile (flag q == tag): warp ew 0 polls them,
+// lane q reading flag q, so one round trip covers the group; then every epilogue thread passes
+// a barrier.  False when the launch is unwinding (a stalled wait sets the abort flag and the
+// status word).
+__device__ __forceinline__ bool wait_parts(const int* flags, int q0, int qn, int tag, int ew, int lane,
+                                           volatile int* s_abort, int* status) {
+    if (ew == 0) {
+        const long long t0 = spin_clock();
+        for (;;) {
+            const bool ok = lane < q0 || lane >= q0 + qn || ld_acquire(flags + lane) == tag;
+            if (__all_sync(0xffffffffu, ok)) break;
+            int give_up = 0;
+            if (lane == 0) give_up = (*s_abort || spin_clock() - t0 > kWaitLimitCycles) ? 1 : 0;
+            if (__shfl_sync(0xffffffffu, give_up, 0)) {  // warp-uniform decision
+                if (lane == 0 && !*s_abort) {
+                    *s_abort = 1;
+                    atomicOr(status, kStatusTimeout);
+                }
+                break;
+            }
+            __nanosleep(32);
+        }
+    }
+    return !named_bar_any(1, kEpiThreads, *s_abort != 0);
+}
+
 // The epilogue warps' share of one phase: every tile of this CTA's range.
 template <int EPI, int DP>
 __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph, int tag, uint8_t* red_stage,
@@ -710,16 +736,21 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         // a contributor's range goes on into a tile whose first k-blocks it holds: a finisher
         if (finisher) prepare(tile);
         else if (tend < it1) prepare(tile + 1);
-        mbar_wait(&tfull[es.acc], es.acc_phase, s_abort, status);
-        if (named_bar_any(1, kEpiThreads, *s_abort != 0)) {
-            cp_async_wait<0>();  // no copy lands in shared memory after the launch has ended
-            return;
+        // the accumulator (a one-chunk split tile's finisher waits for it after fetching its
+        // second part, below)
+        const bool late_acc = reducer && nchunks == 1;
+        if (!late_acc) {
+            mbar_wait(&tfull[es.acc], es.acc_phase, s_abort, status);
+            if (named_bar_any(1, kEpiThreads, *s_abort != 0)) {
+                cp_async_wait<0>();  // no copy lands in shared memory after the launch has ended
+                return;
+            }
+            if (tr && threadIdx.x == 64) {
+                tr[kTrAccReady] = global_ns();
+                tr[kTrTile] = static_cast<unsigned long long>(tile);
+            }
+            tc_fence_after();
         }
-        if (tr && threadIdx.x == 64) {
-            tr[kTrAccReady] = global_ns();
-            tr[kTrTile] = static_cast<unsigned long long>(tile);
-        }
-        tc_fence_after();
         const uint32_t t_acc = tmem_base + static_cast<uint32_t>(es.acc * ca.acc_cols) +
                                (static_cast<uint32_t>(quarter * 32) << 16);
         if (whole) {
@@ -818,27 +849,41 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             bool stop = false;
             int si = 0;
             for (int c = 0; c < nchunks && !stop; ++c) {
-                tmem_ld_32x16(t_acc + static_cast<uint32_t>(c * 32 + half * 16), v);  // own (first) k-range
-                for (int q0 = 1; direct && q0 < nparts; q0 += DP) {
-                    const int qn = min(DP, nparts - q0);
-                    if (ew == 0) {  // lane i polls part i's flag: one round trip covers the group
-                        const long long t0 = spin_clock();
-                        for (;;) {
-                            const bool ok = lane < q0 || lane >= q0 + qn || ld_acquire(flags + lane) == tag;
-                            if (__all_sync(0xffffffffu, ok)) break;
-                            int give_up = 0;
-                            if (lane == 0) give_up = (*s_abort || spin_clock() - t0 > kWaitLimitCycles) ? 1 : 0;
-                            if (__shfl_sync(0xffffffffu, give_up, 0)) {  // warp-uniform decision
-                                if (lane == 0 && !*s_abort) {
-                                    *s_abort = 1;
-                                    atomicOr(status, kStatusTimeout);
-                                }
-                                break;
-                            }
-                            __nanosleep(32);
-                        }
+                if (direct) {
+                    // part 1 is fetched before the own accumulator is waited for: a part that
+                    // finished earlier than the finisher's own range costs nothing then
+                    if (!wait_parts(flags, 1, 1, tag, ew, lane, s_abort, status)) {
+                        stop = true;
+                        break;
                     }
+                    const float4* src1 = reinterpret_cast<const float4*>(P.partials + static_cast<size_t>(c_first + 1) * slot_floats);
+                    float4 a1[4];
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) a1[j] = __ldcg(src1 + static_cast<size_t>(half * 4 + j) * kBM + rt);
+                    mbar_wait(&tfull[es.acc], es.acc_phase, s_abort, status);
                     if (named_bar_any(1, kEpiThreads, *s_abort != 0)) {
+                        stop = true;
+                        break;
+                    }
+                    if (tr && threadIdx.x == 64) {
+                        tr[kTrAccReady] = global_ns();
+                        tr[kTrTile] = static_cast<unsigned long long>(tile);
+                    }
+                    tc_fence_after();
+                    tmem_ld_32x16(t_acc + static_cast<uint32_t>(half * 16), v);  // own (first) k-range
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        v[4 * j] += a1[j].x;
+                        v[4 * j + 1] += a1[j].y;
+                        v[4 * j + 2] += a1[j].z;
+                        v[4 * j + 3] += a1[j].w;
+                    }
+                } else {
+                    tmem_ld_32x16(t_acc + static_cast<uint32_t>(c * 32 + half * 16), v);  // own (first) k-range
+                }
+                for (int q0 = 2; direct && q0 < nparts; q0 += DP) {
+                    const int qn = min(DP, nparts - q0);
+                    if (!wait_parts(flags, q0, qn, tag, ew, lane, s_abort, status)) {
                         stop = true;
                         break;
                     }
