@@ -850,16 +850,18 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             int si = 0;
             for (int c = 0; c < nchunks && !stop; ++c) {
                 if (direct) {
-                    // part 1 is fetched before the own accumulator is waited for: a part that
-                    // finished earlier than the finisher's own range costs nothing then
-                    if (!wait_parts(flags, 1, 1, tag, ew, lane, s_abort, status)) {
+                    // The last part holds the tile's last k-blocks at the start of its CTA's range:
+                    // it is fetched before the own accumulator is waited for (it usually finished
+                    // earlier, and then costs nothing) and added after the middle parts, which
+                    // follow in groups (the sum in part order).
+                    if (!wait_parts(flags, nparts - 1, 1, tag, ew, lane, s_abort, status)) {
                         stop = true;
                         break;
                     }
-                    const float4* src1 = reinterpret_cast<const float4*>(P.partials + static_cast<size_t>(c_first + 1) * slot_floats);
-                    float4 a1[4];
+                    const float4* srcl = reinterpret_cast<const float4*>(P.partials + static_cast<size_t>(c_last) * slot_floats);
+                    float4 al[4];
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) a1[j] = __ldcg(src1 + static_cast<size_t>(half * 4 + j) * kBM + rt);
+                    for (int j = 0; j < 4; ++j) al[j] = __ldcg(srcl + static_cast<size_t>(half * 4 + j) * kBM + rt);
                     mbar_wait(&tfull[es.acc], es.acc_phase, s_abort, status);
                     if (named_bar_any(1, kEpiThreads, *s_abort != 0)) {
                         stop = true;
@@ -871,44 +873,45 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                     }
                     tc_fence_after();
                     tmem_ld_32x16(t_acc + static_cast<uint32_t>(half * 16), v);  // own (first) k-range
+                    for (int q0 = 1; q0 < nparts - 1; q0 += DP) {
+                        const int qn = min(DP, nparts - 1 - q0);
+                        if (!wait_parts(flags, q0, qn, tag, ew, lane, s_abort, status)) {
+                            stop = true;
+                            break;
+                        }
+                        // L2 only (.cg): other CTAs wrote these lines, and the next launch writes
+                        // the same slots again.  A group's loads go out unconditionally (the slot
+                        // index held at the last part), its adds stop at the group's last part.
+                        float4 a[DP][4];
+#pragma unroll
+                        for (int g = 0; g < DP; ++g) {
+                            const float4* src = reinterpret_cast<const float4*>(
+                                P.partials + static_cast<size_t>(min(c_first + q0 + g, c_last)) * slot_floats);
+#pragma unroll
+                            for (int j = 0; j < 4; ++j) a[g][j] = __ldcg(src + static_cast<size_t>(half * 4 + j) * kBM + rt);
+                        }
+#pragma unroll
+                        for (int g = 0; g < DP; ++g)
+                            if (g < qn) {
+#pragma unroll
+                                for (int j = 0; j < 4; ++j) {
+                                    v[4 * j] += a[g][j].x;
+                                    v[4 * j + 1] += a[g][j].y;
+                                    v[4 * j + 2] += a[g][j].z;
+                                    v[4 * j + 3] += a[g][j].w;
+                                }
+                            }
+                    }
+                    if (stop) break;
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
-                        v[4 * j] += a1[j].x;
-                        v[4 * j + 1] += a1[j].y;
-                        v[4 * j + 2] += a1[j].z;
-                        v[4 * j + 3] += a1[j].w;
+                        v[4 * j] += al[j].x;
+                        v[4 * j + 1] += al[j].y;
+                        v[4 * j + 2] += al[j].z;
+                        v[4 * j + 3] += al[j].w;
                     }
                 } else {
                     tmem_ld_32x16(t_acc + static_cast<uint32_t>(c * 32 + half * 16), v);  // own (first) k-range
-                }
-                for (int q0 = 2; direct && q0 < nparts; q0 += DP) {
-                    const int qn = min(DP, nparts - q0);
-                    if (!wait_parts(flags, q0, qn, tag, ew, lane, s_abort, status)) {
-                        stop = true;
-                        break;
-                    }
-                    // L2 only (.cg): other CTAs wrote these lines, and the next launch writes the
-                    // same slots again.  A group's loads go out unconditionally (the slot index held
-                    // at the last part), its adds stop at the group's last part.
-                    float4 a[DP][4];
-#pragma unroll
-                    for (int g = 0; g < DP; ++g) {
-                        const float4* src = reinterpret_cast<const float4*>(
-                            P.partials + static_cast<size_t>(min(c_first + q0 + g, c_last)) * slot_floats);
-#pragma unroll
-                        for (int j = 0; j < 4; ++j) a[g][j] = __ldcg(src + static_cast<size_t>(half * 4 + j) * kBM + rt);
-                    }
-#pragma unroll
-                    for (int g = 0; g < DP; ++g)
-                        if (g < qn) {
-#pragma unroll
-                            for (int j = 0; j < 4; ++j) {
-                                v[4 * j] += a[g][j].x;
-                                v[4 * j + 1] += a[g][j].y;
-                                v[4 * j + 2] += a[g][j].z;
-                                v[4 * j + 3] += a[g][j].w;
-                            }
-                        }
                 }
                 for (int q = 1; !direct && q < nparts; ++q, ++si) {
                     const int sl = si & 1;
