@@ -335,8 +335,8 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                     }
                 } else if constexpr (PASS == 1) {  // token-major staging, stored below in 16-byte pieces
                     reinterpret_cast<__nv_bfloat16*>(sm.stg)[(GW * g + u) * kBM + rt] = __float2bfloat16_rn(xo[u]);
-                } else {
-                    reinterpret_cast<float*>(sm.stg2)[(GW * g + u) * kBM + rt] = xo[u];
+                } else {  // fp32: a warp's 32 rows of one token are one 128-byte line
+                    if (ok) ep.out[static_cast<size_t>(cg + u) * ep.ld_out + row] = xo[u];
                 }
             }
             if constexpr (PASS != 2) {
@@ -462,29 +462,21 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
         }
         named_bar(1, kEpiThreads);
     }
-    if constexpr (EPI == EPI_RESID && PASS != 0) {
+    if constexpr (EPI == EPI_RESID && PASS == 1) {
         // the staged chunk: thread t stores token t/8, features 16 (t%8) .. +15 of the tile
         named_bar(1, kEpiThreads);
         const int t = e, tok = t >> 3, f0 = (t & 7) * 16;
         const int col = col0 + tok;
         if (col < p.N) {
-            if constexpr (PASS == 1) {
-                const uint4* src =
-                    reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(sm.stg) + tok * kBM + f0);
-                uint4* dst = reinterpret_cast<uint4*>(ep.xb + static_cast<size_t>(col) * ep.ld_out + mt * kBM + f0);
+            const uint4* src =
+                reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(sm.stg) + tok * kBM + f0);
+            uint4* dst = reinterpret_cast<uint4*>(ep.xb + static_cast<size_t>(col) * ep.ld_out + mt * kBM + f0);
 #pragma unroll
-                for (int i = 0; i < 2; ++i) dst[i] = src[i];
-            } else {
-                const float4* src =
-                    reinterpret_cast<const float4*>(reinterpret_cast<const float*>(sm.stg2) + tok * kBM + f0);
-                float4* dst = reinterpret_cast<float4*>(ep.out + static_cast<size_t>(col) * ep.ld_out + mt * kBM + f0);
-#pragma unroll
-                for (int i = 0; i < 4; ++i) dst[i] = src[i];
-            }
+            for (int i = 0; i < 2; ++i) dst[i] = src[i];
         }
         named_bar(1, kEpiThreads);  // the staging memory is free again
     }
-    if constexpr (EPI == EPI_RESID && PASS != 1) {
+    if constexpr (EPI == EPI_RESID && PASS == 0) {
         named_bar(1, kEpiThreads);
         if (e < 32) {
             const int col = col0 + lane;
@@ -493,6 +485,15 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
                 ep.sq_out[static_cast<size_t>(mt) * p.N + col] = ((rd[lane] + rd[32 + lane]) + rd[64 + lane]) + rd[96 + lane];
         }
         named_bar(1, kEpiThreads);
+    } else if constexpr (EPI == EPI_RESID && PASS == 2) {
+        // the chunk's four quarter sums, written by its first pass (the barriers since then order
+        // them; the next writer of these words comes after the tile's next barrier)
+        if (e < 32) {
+            const int col = col0 + lane;
+            const float* rd = sm.red + (c_in / 32) * 128;
+            if (col < p.N)
+                ep.sq_out[static_cast<size_t>(mt) * p.N + col] = ((rd[lane] + rd[32 + lane]) + rd[64 + lane]) + rd[96 + lane];
+        }
     } else if constexpr (EPI == EPI_LMHEAD) {
         named_bar(1, kEpiThreads);
         if (e < 32) {  // merge the four row quarters in a fixed order
