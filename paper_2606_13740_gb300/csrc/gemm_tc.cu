@@ -80,7 +80,6 @@ struct EpiSmem {
     float* theta; // [128] rotation frequency of each tile row's feature pair (QKV)
     uint8_t* stg;  // staging of a 32-token chunk's bf16 outputs, 8 KB (for tiles of more than one chunk its
                    // own memory: the next chunk's partial slices arrive meanwhile)
-    uint8_t* stg2; // staging of a chunk's fp32 residual (second pass), 16 KB: the partial staging memory
     float* xs;    // [2][32][128] the old fp32 residual of a wide tile's chunks (nullptr: none), see xs_offset
     const int* rows;  // the launch's device-resolved row count (-1: the plans as given)
 };
@@ -784,19 +783,19 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         }
         if (reducer) {
             // Part q's partial, chunk c (32 columns), is the contiguous 16 KB slice [c*8 + j][row]
-            // float4.  The slices go through the two staging slots in one stream, chunk-major
-            // (slice s = chunk s / (nparts-1), part s % (nparts-1) + 1, slot s % 2), two in flight:
-            // each copy is issued as soon as its part has published (flag q == tag) and its slot's
-            // previous slice is added, so the next chunk's slices arrive during this chunk's
-            // epilogue and the early parts' while the late ones still compute.  The sum runs over
-            // q in order, so it does not depend on the arrival order.
+            // float4.  The slices go through the staging slot in one stream, chunk-major (slice
+            // s = chunk s / (nparts-1), part s % (nparts-1) + 1): each copy is issued as soon as
+            // its part has published (flag q == tag) and the previous slice is added, so a
+            // chunk's slice arrives during the previous chunk's epilogue.  The sum runs over q in
+            // order, so it does not depend on the arrival order.  (Tiles of one 32-token chunk
+            // take the direct path below instead.)
             const int nparts = c_last - c_first + 1;
             const int np1 = nparts - 1;
             const int nslices = nchunks * np1;
             int* flags = &P.tickets[tile * kTicketStride];
             constexpr uint32_t slice_bytes = 32 * kBM * 4;
             uint32_t ready = 0;     // warp 2: parts seen published (bit q)
-            uint32_t inflight = 0;  // thread 64: slots with a copy not yet waited for
+            uint32_t inflight = 0;  // thread 64: a copy not yet waited for
             // warp 2, warp-uniform: make sure slice s's part has published, polling every part's
             // flag at once (lane i reads flag i, so one round trip covers them all), then thread
             // 64 issues the copy
@@ -821,15 +820,14 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                     }
                 }
                 if (lane == 0) {
-                    const int sl = si & 1;
                     fence_proxy_async_global();
                     fence_proxy_async_smem();  // the slot was last touched by generic accesses
-                    mbar_arrive_expect_tx(redbar + sl, slice_bytes);
-                    bulk_load(red_stage + static_cast<size_t>(sl) * slice_bytes,
+                    mbar_arrive_expect_tx(redbar, slice_bytes);
+                    bulk_load(red_stage,
                               P.partials + static_cast<size_t>(c_first + q) * slot_floats +
                                   static_cast<size_t>(c) * 32 * kBM,
-                              slice_bytes, redbar + sl);
-                    inflight |= 1u << sl;
+                              slice_bytes, redbar);
+                    inflight = 1;
                 }
             };
             // A 32-token tile (one chunk) skips the staging: each thread's 16 columns of its row of
@@ -845,7 +843,6 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             }
             if (ew == 0 && !direct) {
                 if (nslices > 0) issue(0);
-                if (nslices > 1) issue(1);
             }
             bool stop = false;
             int si = 0;
@@ -915,11 +912,10 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                     tmem_ld_32x16(t_acc + static_cast<uint32_t>(c * 32 + half * 16), v);  // own (first) k-range
                 }
                 for (int q = 1; !direct && q < nparts; ++q, ++si) {
-                    const int sl = si & 1;
-                    mbar_wait(redbar + sl, (es.red_phase >> sl) & 1u, s_abort, status);
-                    es.red_phase ^= 1u << sl;
-                    if (threadIdx.x == 64) inflight &= ~(1u << sl);
-                    const float4* src = reinterpret_cast<const float4*>(red_stage + static_cast<size_t>(sl) * slice_bytes);
+                    mbar_wait(redbar, es.red_phase & 1u, s_abort, status);
+                    es.red_phase ^= 1u;
+                    if (threadIdx.x == 64) inflight = 0;
+                    const float4* src = reinterpret_cast<const float4*>(red_stage);
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
                         const float4 a = src[(half * 4 + j) * kBM + rt];
@@ -932,7 +928,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                         stop = true;
                         break;
                     }
-                    if (ew == 0 && si + 2 < nslices) issue(si + 2);
+                    if (ew == 0 && si + 1 < nslices) issue(si + 1);
                 }
                 if (stop) break;
                 if (tr && threadIdx.x == 64 && c == 0) {
@@ -951,10 +947,8 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             if (threadIdx.x == 64) {
                 if (stop) {  // let copies in flight land before the shared memory is released
                     const long long t0 = spin_clock();
-                    for (int sl = 0; sl < 2; ++sl)
-                        while ((inflight >> sl & 1u) && !mbar_try_wait(redbar + sl, (es.red_phase >> sl) & 1u) &&
-                               spin_clock() - t0 < kWaitLimitCycles) {
-                        }
+                    while (inflight && !mbar_try_wait(redbar, es.red_phase & 1u) && spin_clock() - t0 < kWaitLimitCycles) {
+                    }
                 } else {
                     for (int q = 1; q < nparts; ++q) flags[q] = 0;  // ready for the next launch
                 }
@@ -1052,15 +1046,14 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
     esm.kvs = reinterpret_cast<int*>(tail + 256 + 1024);
     esm.theta = tail + 256 + 1024 + 256;
     esm.stg = ca.stg_bytes ? red_stage + ca.red_bytes + ca.xs_bytes : red_stage;
-    esm.stg2 = red_stage;
     float* after = tail + 256 + 1024 + 256 + 128;
     uint64_t* full = reinterpret_cast<uint64_t*>(after);
     uint64_t* empty = full + S;
     uint64_t* tfull = empty + S;
     uint64_t* tempty = tfull + 2;
     uint64_t* drain = tempty + 2;
-    uint64_t* redbar = drain + 1;  // two partial staging slots
-    uint64_t* rfull = redbar + 2;  // raw 4-bit tiles (Q4): arrived / read
+    uint64_t* redbar = drain + 1;  // the partial staging slot
+    uint64_t* rfull = redbar + 1;  // raw 4-bit tiles (Q4): arrived / read
     uint64_t* rempty = rfull + R;
     uint64_t* bfull = rempty + R;  // operand tiles of the 4-bit kernel: arrived / consumed
     uint64_t* bempty = bfull + (Q4 ? SB : 0);
@@ -1093,8 +1086,7 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
             mbar_init(&tempty[a], kEpiThreads);
         }
         mbar_init(drain, 1);
-        mbar_init(&redbar[0], 1);
-        mbar_init(&redbar[1], 1);
+        mbar_init(redbar, 1);
         *s_abort = 0;
         int rows = -1;
         if (ca.dyn_rows) {
@@ -1555,11 +1547,13 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
     ca.acc_cols = c32 ? 32 : pow2ceil(ntile);
     ca.x_cols = ntile <= 128 ? ntile : 0;  // staged residual (none for 256-token tiles: TMEM is full)
     ca.tmem_cols = pow2ceil(2 * ca.acc_cols + ca.x_cols);
-    ca.red_bytes = 2 * 32 * kBM * 4;  // two 32-column partial slices per bulk-copy round
+    // One partial slice staged for the finisher of a split tile of several 32-token chunks (the
+    // ring of 256-token stages needs the room: the tensor cores keep busy with 4 stages, not
+    // with 3); for 32-token chains, whose finishers load the parts straight into registers, it
+    // is the output staging.
+    ca.red_bytes = 32 * kBM * 4;
     const int stage_bytes = static_cast<int>(kABytes) + ntile * kBK * 2;
-    // tiles of more than one 32-token chunk: their own 8 KB for the bf16 output staging; wide
-    // tiles: the old residual staged in shared memory two chunks at a time, where that leaves
-    // the ring at least 3 stages
+    // tiles of more than one 32-token chunk: their own 8 KB for the bf16 output staging
     ca.stg_bytes = c32 ? 0 : 32 * kBM * 2;
     ca.xs_bytes = 0;
     const int fixed0 = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + ca.stg_bytes + 7 * 8 + 16;
@@ -1584,9 +1578,9 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
     }
     ca.raw_stages = 0;
     ca.b_stages = 0;
-    if (ca.x_cols == 0 && (smem_budget - fixed0 - 2 * 32 * kBM * 4) / (stage_bytes + 16) >= 3)
-        ca.xs_bytes = 2 * 32 * kBM * 4;
-    const int fixed = fixed0 + ca.xs_bytes;
+    // wide residual tiles read the old residual from global memory (a warp's 32 rows of a token
+    // are one 128-byte line), not from a staged copy: the ring keeps the room
+    const int fixed = fixed0;
     int st = (smem_budget - fixed) / (stage_bytes + 16);
     if (st > 32) st = 32;
     if (st < 2) return false;
