@@ -597,7 +597,9 @@ __device__ __forceinline__ bool wait_parts(const int* flags, int q0, int qn, int
 }
 
 // The epilogue warps' share of one phase: every tile of this CTA's range.
-template <int EPI, int DP>
+// WIDE: token tiles of several 32-token chunks (split tiles reduced through the staging
+// slots); else one chunk (split tiles reduced in registers): each its own code.
+template <int EPI, int DP, bool WIDE>
 __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph, int tag, uint8_t* red_stage,
                                                   uint64_t* tfull, uint64_t* tempty, uint64_t* redbar,
                                                   volatile int* s_abort, uint32_t tmem_base, const EpiSmem& esm,
@@ -738,7 +740,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         else if (tend < it1) prepare(tile + 1);
         // the accumulator (a one-chunk split tile's finisher waits for it after fetching its
         // second part, below)
-        const bool late_acc = reducer && nchunks == 1;
+        const bool late_acc = reducer && !WIDE;
         if (!late_acc) {
             mbar_wait(&tfull[es.acc], es.acc_phase, s_abort, status);
             if (named_bar_any(1, kEpiThreads, *s_abort != 0)) {
@@ -783,19 +785,20 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         }
         if (reducer) {
             // Part q's partial, chunk c (32 columns), is the contiguous 16 KB slice [c*8 + j][row]
-            // float4.  The slices go through the staging slot in one stream, chunk-major (slice
-            // s = chunk s / (nparts-1), part s % (nparts-1) + 1): each copy is issued as soon as
-            // its part has published (flag q == tag) and the previous slice is added, so a
-            // chunk's slice arrives during the previous chunk's epilogue.  The sum runs over q in
-            // order, so it does not depend on the arrival order.  (Tiles of one 32-token chunk
-            // take the direct path below instead.)
+            // float4.  The slices go through the nsl staging slots (one or two) in one stream,
+            // chunk-major (slice s = chunk s / (nparts-1), part s % (nparts-1) + 1, slot s % nsl):
+            // each copy is issued as soon as its part has published (flag q == tag) and its
+            // slot's previous slice is added, so a chunk's slices arrive during the previous
+            // chunk's epilogue.  The sum runs over q in order, so it does not depend on the arrival
+            // order.  (Tiles of one 32-token chunk take the direct path below instead.)
             const int nparts = c_last - c_first + 1;
             const int np1 = nparts - 1;
             const int nslices = nchunks * np1;
             int* flags = &P.tickets[tile * kTicketStride];
             constexpr uint32_t slice_bytes = 32 * kBM * 4;
+            const int nsl = ca.red_bytes >= 2 * static_cast<int>(slice_bytes) ? 2 : 1;
             uint32_t ready = 0;     // warp 2: parts seen published (bit q)
-            uint32_t inflight = 0;  // thread 64: a copy not yet waited for
+            uint32_t inflight = 0;  // thread 64: slots with a copy not yet waited for
             // warp 2, warp-uniform: make sure slice s's part has published, polling every part's
             // flag at once (lane i reads flag i, so one round trip covers them all), then thread
             // 64 issues the copy
@@ -822,19 +825,20 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                 if (lane == 0) {
                     fence_proxy_async_global();
                     fence_proxy_async_smem();  // the slot was last touched by generic accesses
-                    mbar_arrive_expect_tx(redbar, slice_bytes);
-                    bulk_load(red_stage,
+                    const int sl = si & (nsl - 1);
+                    mbar_arrive_expect_tx(redbar + sl, slice_bytes);
+                    bulk_load(red_stage + static_cast<size_t>(sl) * slice_bytes,
                               P.partials + static_cast<size_t>(c_first + q) * slot_floats +
                                   static_cast<size_t>(c) * 32 * kBM,
-                              slice_bytes, redbar);
-                    inflight = 1;
+                              slice_bytes, redbar + sl);
+                    inflight |= 1u << sl;
                 }
             };
             // A 32-token tile (one chunk) skips the staging: each thread's 16 columns of its row of
             // every part come straight into registers, up to DP parts at a time once
             // their flags are seen, so the parts cost one round trip to L2 instead of a copy each
             // (the same sum, in the same order, bit for bit).
-            const bool direct = nchunks == 1;
+            constexpr bool direct = !WIDE;
             if (tr && threadIdx.x == 64) tr[kTrPartStored] = global_ns();
             // the QKV plan of a one-chunk tile does not need the sum: built while the parts arrive
             QkvPlan qpre;
@@ -843,6 +847,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             }
             if (ew == 0 && !direct) {
                 if (nslices > 0) issue(0);
+                if (nslices > 1 && nsl > 1) issue(1);
             }
             bool stop = false;
             int si = 0;
@@ -912,10 +917,11 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                     tmem_ld_32x16(t_acc + static_cast<uint32_t>(c * 32 + half * 16), v);  // own (first) k-range
                 }
                 for (int q = 1; !direct && q < nparts; ++q, ++si) {
-                    mbar_wait(redbar, es.red_phase & 1u, s_abort, status);
-                    es.red_phase ^= 1u;
-                    if (threadIdx.x == 64) inflight = 0;
-                    const float4* src = reinterpret_cast<const float4*>(red_stage);
+                    const int sl = si & (nsl - 1);
+                    mbar_wait(redbar + sl, (es.red_phase >> sl) & 1u, s_abort, status);
+                    es.red_phase ^= 1u << sl;
+                    if (threadIdx.x == 64) inflight &= ~(1u << sl);
+                    const float4* src = reinterpret_cast<const float4*>(red_stage + static_cast<size_t>(sl) * slice_bytes);
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
                         const float4 a = src[(half * 4 + j) * kBM + rt];
@@ -928,7 +934,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                         stop = true;
                         break;
                     }
-                    if (ew == 0 && si + 1 < nslices) issue(si + 1);
+                    if (ew == 0 && si + nsl < nslices) issue(si + nsl);
                 }
                 if (stop) break;
                 if (tr && threadIdx.x == 64 && c == 0) {
@@ -947,8 +953,10 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             if (threadIdx.x == 64) {
                 if (stop) {  // let copies in flight land before the shared memory is released
                     const long long t0 = spin_clock();
-                    while (inflight && !mbar_try_wait(redbar, es.red_phase & 1u) && spin_clock() - t0 < kWaitLimitCycles) {
-                    }
+                    for (int sl = 0; sl < nsl; ++sl)
+                        while ((inflight >> sl & 1u) && !mbar_try_wait(redbar + sl, (es.red_phase >> sl) & 1u) &&
+                               spin_clock() - t0 < kWaitLimitCycles) {
+                        }
                 } else {
                     for (int q = 1; q < nparts; ++q) flags[q] = 0;  // ready for the next launch
                 }
@@ -990,6 +998,30 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
     }
     cp_async_wait<0>();
     if (tr && threadIdx.x == 64) tr[kTrEpiDone] = global_ns();
+}
+
+template <int DP, bool WIDE>
+__device__ __forceinline__ void chain_epilogue_dispatch(const ChainArgs& ca, int ph, int tag, uint8_t* red_stage,
+                                                        uint64_t* tfull, uint64_t* tempty, uint64_t* redbar,
+                                                        volatile int* s_abort, uint32_t tmem_base, const EpiSmem& esm,
+                                                        ChainEpiState& es) {
+    switch (ca.ph[ph].epi) {
+        case EPI_F32:
+            chain_phase_epilogue<EPI_F32, DP, WIDE>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+            break;
+        case EPI_RESID:
+            chain_phase_epilogue<EPI_RESID, DP, WIDE>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+            break;
+        case EPI_QKV:
+            chain_phase_epilogue<EPI_QKV, DP, WIDE>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+            break;
+        case EPI_SWIGLU:
+            chain_phase_epilogue<EPI_SWIGLU, DP, WIDE>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+            break;
+        default:
+            chain_phase_epilogue<EPI_LMHEAD, DP, WIDE>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
+            break;
+    }
 }
 
 // Expand one 4-bit weight tile (see kQ4TileBytes) into the 128-byte-swizzled K-major bf16 image
@@ -1052,8 +1084,8 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
     uint64_t* tfull = empty + S;
     uint64_t* tempty = tfull + 2;
     uint64_t* drain = tempty + 2;
-    uint64_t* redbar = drain + 1;  // the partial staging slot
-    uint64_t* rfull = redbar + 1;  // raw 4-bit tiles (Q4): arrived / read
+    uint64_t* redbar = drain + 1;  // the partial staging slots (one or two)
+    uint64_t* rfull = redbar + 2;  // raw 4-bit tiles (Q4): arrived / read
     uint64_t* rempty = rfull + R;
     uint64_t* bfull = rempty + R;  // operand tiles of the 4-bit kernel: arrived / consumed
     uint64_t* bempty = bfull + (Q4 ? SB : 0);
@@ -1086,7 +1118,8 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
             mbar_init(&tempty[a], kEpiThreads);
         }
         mbar_init(drain, 1);
-        mbar_init(redbar, 1);
+        mbar_init(&redbar[0], 1);
+        mbar_init(&redbar[1], 1);
         *s_abort = 0;
         int rows = -1;
         if (ca.dyn_rows) {
@@ -1406,23 +1439,12 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
         // kernel's smaller register budget takes two)
         constexpr int kDP = Q4 ? 2 : 4;
         for (int ph = 0; ph < ca.n_phases; ++ph) {  // on abort every phase returns at its first barrier
-            switch (ca.ph[ph].epi) {
-                case EPI_F32:
-                    chain_phase_epilogue<EPI_F32, kDP>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
-                    break;
-                case EPI_RESID:
-                    chain_phase_epilogue<EPI_RESID, kDP>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
-                    break;
-                case EPI_QKV:
-                    chain_phase_epilogue<EPI_QKV, kDP>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
-                    break;
-                case EPI_SWIGLU:
-                    chain_phase_epilogue<EPI_SWIGLU, kDP>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
-                    break;
-                default:
-                    chain_phase_epilogue<EPI_LMHEAD, kDP>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base, esm, es);
-                    break;
-            }
+            if (ca.ntile == 32)
+                chain_epilogue_dispatch<kDP, false>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base,
+                                                    esm, es);
+            else
+                chain_epilogue_dispatch<kDP, true>(ca, ph, tag, red_stage, tfull, tempty, redbar, s_abort, tmem_base,
+                                                   esm, es);
         }
     }
 
@@ -1547,11 +1569,11 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
     ca.acc_cols = c32 ? 32 : pow2ceil(ntile);
     ca.x_cols = ntile <= 128 ? ntile : 0;  // staged residual (none for 256-token tiles: TMEM is full)
     ca.tmem_cols = pow2ceil(2 * ca.acc_cols + ca.x_cols);
-    // One partial slice staged for the finisher of a split tile of several 32-token chunks (the
-    // ring of 256-token stages needs the room: the tensor cores keep busy with 4 stages, not
-    // with 3); for 32-token chains, whose finishers load the parts straight into registers, it
-    // is the output staging.
-    ca.red_bytes = 32 * kBM * 4;
+    // Partial slices staged for the finisher of a split tile of several 32-token chunks: two in
+    // flight, one for 256-token tiles (their ring needs the room: the tensor cores keep busy
+    // with 4 stages of 256 tokens, not with 3); for 32-token chains, whose finishers load the
+    // parts straight into registers, one slot that is the output staging.
+    ca.red_bytes = (c32 || ntile > 128 ? 1 : 2) * 32 * kBM * 4;
     const int stage_bytes = static_cast<int>(kABytes) + ntile * kBK * 2;
     // tiles of more than one 32-token chunk: their own 8 KB for the bf16 output staging
     ca.stg_bytes = c32 ? 0 : 32 * kBM * 2;
