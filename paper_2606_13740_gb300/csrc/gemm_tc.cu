@@ -80,7 +80,6 @@ struct EpiSmem {
     float* theta; // [128] rotation frequency of each tile row's feature pair (QKV)
     uint8_t* stg;  // staging of a 32-token chunk's bf16 outputs, 8 KB (for tiles of more than one chunk its
                    // own memory: the next chunk's partial slices arrive meanwhile)
-    float* xs;    // [2][32][128] the old fp32 residual of a wide tile's chunks (nullptr: none), see xs_offset
     const int* rows;  // the launch's device-resolved row count (-1: the plans as given)
 };
 
@@ -97,15 +96,6 @@ __device__ __forceinline__ GemmPlan phase_plan(const ChainPhase& P, int rows) {
         if (p.grid > p.total / min_iters) p.grid = static_cast<int>(p.total / min_iters);
     }
     return p;
-}
-
-// Word offset of (token j, tile row f) in a 32-token chunk of staged residual: [token][128 rows],
-// the 16-byte pieces of a token's row rotated so that neither the copies (thread = token, 8
-// pieces) nor the epilogue's reads (lane = row) meet bank conflicts.
-__device__ __forceinline__ int xs_offset(int j, int f) {
-    const int c16 = f >> 2;
-    const int key = (j + 2 * (c16 >> 3)) & 7;
-    return j * kBM + (((c16 & ~7) | ((c16 & 7) ^ key)) << 2) + (f & 3);
 }
 
 // RMSNorm scale of every column of token tile nt: rs[c] = rsqrt(sum_t sq[t][col] / dim + eps).
@@ -247,15 +237,15 @@ __device__ __forceinline__ QkvPlan qkv_plan(const EpiArgs& ep, const GemmPlan& p
 // published to the next phase's operand producer between them; PASS 0: both at once.
 template <int EPI, int PASS = 0>
 __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& p, int mt, int col0, int c_in,
-                                             int rt, uint32_t t_src, uint32_t t_x, const float* xs, const EpiSmem& sm,
+                                             int rt, uint32_t t_src, uint32_t t_x, const EpiSmem& sm,
                                              int e, int half, int quarter, int lane, int* status,
                                              const float* a_in = nullptr, const QkvPlan* qkv_pre = nullptr) {
     // col0: the chunk's first token column; c_in: its offset inside the token tile (index into
     // the tile's RMSNorm scales and staged ids).  The thread's 16 accumulator columns come from
     // a_in (a finisher's sum of the parts, in registers), else from TMEM at t_src.  The old
-    // residual (pass 1) comes from TMEM (t_x), else from shared memory (xs, the chunk's staged
-    // copy), else from global; pass 1 leaves the new residual in the accumulator, where pass 2
-    // reads it.  e: the epilogue thread (0 .. kEpiThreads-1), half: which 16 columns of the
+    // residual (pass 1) comes from TMEM (t_x), else from global memory (a warp's 32 rows of a
+    // token are one 128-byte line; L2 only: other CTAs wrote them in earlier phases); pass 1
+    // leaves the new residual in the accumulator, where pass 2 reads it.  e: the epilogue thread (0 .. kEpiThreads-1), half: which 16 columns of the
     // chunk.  qkv_pre: the QKV plan, built ahead (null: built here).
     constexpr int GW = kEpiGroup;  // columns per group
     constexpr int LS = 32 / GW;    // lanes sharing one column's sum after the scatter
@@ -309,13 +299,10 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
             } else {
                 if (t_x) {
                     tmem_ld_32xn<GW>(t_x + static_cast<uint32_t>(GW * g), xo);
-                } else if (xs) {
-#pragma unroll
-                    for (int u = 0; u < GW; ++u) xo[u] = xs[xs_offset(GW * g + u, rt)];
                 } else {
 #pragma unroll
                     for (int u = 0; u < GW; ++u)
-                        xo[u] = (row < p.M && cg + u < p.N) ? ep.out[static_cast<size_t>(cg + u) * ep.ld_out + row]
+                        xo[u] = (row < p.M && cg + u < p.N) ? __ldcg(ep.out + static_cast<size_t>(cg + u) * ep.ld_out + row)
                                                             : 0.0f;
                 }
 #pragma unroll
@@ -649,33 +636,6 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
     const uint32_t t_x =
         ca.x_cols ? tmem_base + static_cast<uint32_t>(2 * ca.acc_cols) + (static_cast<uint32_t>(quarter * 32) << 16)
                   : 0u;
-    // Wide residual tiles (no TMEM room for the old x): each 32-token chunk of the old fp32
-    // residual is copied into shared memory (two buffers, chunk c in buffer c % 2) by cp.async,
-    // 16 bytes a copy, epilogue thread t < 128 taking token t/4's rows 32 (t%4) .. +31, one
-    // chunk ahead of its use; x_chunk starts the next chunk's copies, then waits for this chunk's.
-    const bool use_xs = EPI == EPI_RESID && esm.xs != nullptr && (ep.ld_out & 3) == 0 &&
-                        (reinterpret_cast<uintptr_t>(ep.out) & 15) == 0;
-    auto x_fetch = [&](int fmt, int fnt, int c) {
-        const int t = e, tok = t >> 2, q = t & 3;
-        const int col = fnt * p.ntile + c * 32 + tok;
-        float* buf = esm.xs + (c & 1) * (32 * kBM);
-        if (t < 128 && col < p.N) {
-            const int f0 = fmt * kBM + q * 32;
-            const float* src = ep.out + static_cast<size_t>(col) * ep.ld_out + f0;
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-                if (f0 + 4 * i < p.M) cp_async16(buf + xs_offset(tok, q * 32 + 4 * i), src + 4 * i);
-        }
-        cp_async_commit();
-    };
-    auto x_chunk = [&](int cmt, int cnt, int c) -> const float* {
-        if (!use_xs) return nullptr;
-        if (c + 1 < nchunks) x_fetch(cmt, cnt, c + 1);
-        else cp_async_commit();
-        cp_async_wait<1>();
-        named_bar(1, kEpiThreads);
-        return esm.xs + (c & 1) * (32 * kBM);
-    };
     int rs_nt = -1, ids_nt = -1;
     long long prepared = -1;
     float v[16];
@@ -705,7 +665,6 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             }
         }
         if constexpr (EPI == EPI_RESID) {
-            if (use_xs) x_fetch(pmt, pnt, 0);
             if (t_x) {
                 const int row = pmt * kBM + rt;
                 for (int c = 0; c < nchunks; ++c) {
@@ -758,11 +717,10 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
         if (whole) {
             // the compact epilogue per 32-column chunk, straight from the accumulator in TMEM
             for (int c = 0; c < nchunks; ++c) {
-                const float* xs = x_chunk(mt, nt, c);
                 epilogue_c32<EPI, kPass1>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt,
                                           t_acc + static_cast<uint32_t>(c * 32),
-                                          t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, xs, esm, e, half, quarter,
-                                          lane, status);
+                                          t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, esm, e, half, quarter, lane,
+                                          status);
             }
         } else if (!reducer) {
             float* my_part = P.partials + static_cast<size_t>(blockIdx.x) * slot_floats;
@@ -944,11 +902,10 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                 }
                 // the compact epilogue on the sum in registers (the residual's first pass leaves the
                 // new residual in the still owned accumulator, for the second)
-                const float* xs = x_chunk(mt, nt, c);
                 epilogue_c32<EPI, kPass1>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt,
                                           t_acc + static_cast<uint32_t>(c * 32),
-                                          t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, xs, esm, e, half, quarter,
-                                          lane, status, v, (EPI == EPI_QKV && direct) ? &qpre : nullptr);
+                                          t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, esm, e, half, quarter, lane,
+                                          status, v, (EPI == EPI_QKV && direct) ? &qpre : nullptr);
             }
             if (threadIdx.x == 64) {
                 if (stop) {  // let copies in flight land before the shared memory is released
@@ -978,7 +935,7 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
             if (finisher) {  // then the fp32 residual and the RMSNorm sums, for the later phases' epilogues
                 for (int c = 0; c < nchunks; ++c)
                     epilogue_c32<EPI, 2>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt,
-                                         t_acc + static_cast<uint32_t>(c * 32), 0u, nullptr, esm, e, half, quarter,
+                                         t_acc + static_cast<uint32_t>(c * 32), 0u, esm, e, half, quarter,
                                          lane, status);
                 if (P.done2) {
                     named_bar(1, kEpiThreads);
@@ -1070,14 +1027,13 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
     uint8_t* sB = sA + static_cast<size_t>(S) * kABytes;
     uint8_t* sRaw = sB + static_cast<size_t>(SB) * b_bytes;  // 4-bit weight tiles (Q4)
     uint8_t* red_stage = sRaw + static_cast<size_t>(R) * kQ4TileBytes;
-    float* tail = reinterpret_cast<float*>(red_stage + ca.red_bytes + ca.xs_bytes + ca.stg_bytes);
+    float* tail = reinterpret_cast<float*>(red_stage + ca.red_bytes + ca.stg_bytes);
     EpiSmem esm;
-    esm.xs = ca.xs_bytes ? reinterpret_cast<float*>(red_stage + ca.red_bytes) : nullptr;
     esm.rs = tail;
     esm.red = tail + 256;
     esm.kvs = reinterpret_cast<int*>(tail + 256 + 1024);
     esm.theta = tail + 256 + 1024 + 256;
-    esm.stg = ca.stg_bytes ? red_stage + ca.red_bytes + ca.xs_bytes : red_stage;
+    esm.stg = ca.stg_bytes ? red_stage + ca.red_bytes : red_stage;
     float* after = tail + 256 + 1024 + 256 + 128;
     uint64_t* full = reinterpret_cast<uint64_t*>(after);
     uint64_t* empty = full + S;
@@ -1577,7 +1533,6 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
     const int stage_bytes = static_cast<int>(kABytes) + ntile * kBK * 2;
     // tiles of more than one 32-token chunk: their own 8 KB for the bf16 output staging
     ca.stg_bytes = c32 ? 0 : 32 * kBM * 2;
-    ca.xs_bytes = 0;
     const int fixed0 = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + ca.stg_bytes + 7 * 8 + 16;
     if (ca.q4) {
         // 4-bit weights (480 threads: no room beside the CTA for another one, so all of shared

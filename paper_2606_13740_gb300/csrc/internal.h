@@ -133,7 +133,6 @@ struct ChainArgs {
     int grid, stages, ntile, acc_cols, tmem_cols;
     int red_bytes;       // shared staging for split partials
     int x_cols;          // TMEM columns for the staged old residual (0: none)
-    int xs_bytes;        // shared staging of the old residual when x_cols == 0 (0: read from global)
     int stg_bytes;       // the epilogue's own output staging (0: it shares the partial staging)
     size_t smem;
     const int* epoch;    // device step counter; tag = *epoch * tag_mul + tag_add (null: tag = tag_add)
@@ -158,7 +157,7 @@ struct ChainMaps {
     CUtensorMap w[kMaxPhases];
     CUtensorMap x[kMaxPhases];
 };
-// Fills grid, stages, ntile, acc_cols, x_cols, xs_bytes, stg_bytes, tmem_cols, red_bytes and
+// Fills grid, stages, ntile, acc_cols, x_cols, stg_bytes, tmem_cols, red_bytes and
 // smem from the phases' plans for a shared-memory budget (bytes, <= 227 KB).  False if the
 // phases do not share one token tiling.
 bool chain_plan(ChainArgs& ca, int smem_budget);
