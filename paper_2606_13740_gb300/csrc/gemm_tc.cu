@@ -239,7 +239,8 @@ template <int EPI, int PASS = 0>
 __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& p, int mt, int col0, int c_in,
                                              int rt, uint32_t t_src, uint32_t t_x, const EpiSmem& sm,
                                              int e, int half, int quarter, int lane, int* status,
-                                             const float* a_in = nullptr, const QkvPlan* qkv_pre = nullptr) {
+                                             const float* a_in = nullptr, const QkvPlan* qkv_pre = nullptr,
+                                             const float* x_in = nullptr) {
     // col0: the chunk's first token column; c_in: its offset inside the token tile (index into
     // the tile's RMSNorm scales and staged ids).  The thread's 16 accumulator columns come from
     // a_in (a finisher's sum of the parts, in registers), else from TMEM at t_src.  The old
@@ -299,6 +300,9 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
             } else {
                 if (t_x) {
                     tmem_ld_32xn<GW>(t_x + static_cast<uint32_t>(GW * g), xo);
+                } else if (x_in) {
+#pragma unroll
+                    for (int u = 0; u < GW; ++u) xo[u] = x_in[u];
                 } else {
 #pragma unroll
                     for (int u = 0; u < GW; ++u)
@@ -874,6 +878,17 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                 } else {
                     tmem_ld_32x16(t_acc + static_cast<uint32_t>(c * 32 + half * 16), v);  // own (first) k-range
                 }
+                // a wide residual tile's old rows of this chunk, loaded while its parts arrive
+                float xw[kEpiGroup];
+                if constexpr (EPI == EPI_RESID && WIDE) {
+                    const int xrow = mt * kBM + rt;
+#pragma unroll
+                    for (int u = 0; u < kEpiGroup; ++u) {
+                        const int xcol = nt * p.ntile + c * 32 + half * kEpiGroup + u;
+                        xw[u] = (xrow < p.M && xcol < p.N) ? __ldcg(ep.out + static_cast<size_t>(xcol) * ep.ld_out + xrow)
+                                                           : 0.0f;
+                    }
+                }
                 for (int q = 1; !direct && q < nparts; ++q, ++si) {
                     const int sl = si & (nsl - 1);
                     mbar_wait(redbar + sl, (es.red_phase >> sl) & 1u, s_abort, status);
@@ -905,7 +920,8 @@ __device__ __forceinline__ void chain_phase_epilogue(const ChainArgs& ca, int ph
                 epilogue_c32<EPI, kPass1>(ep, p, mt, nt * p.ntile + c * 32, c * 32, rt,
                                           t_acc + static_cast<uint32_t>(c * 32),
                                           t_x ? t_x + static_cast<uint32_t>(c * 32) : 0u, esm, e, half, quarter, lane,
-                                          status, v, (EPI == EPI_QKV && direct) ? &qpre : nullptr);
+                                          status, v, (EPI == EPI_QKV && direct) ? &qpre : nullptr,
+                                          EPI == EPI_RESID && WIDE ? xw : nullptr);
             }
             if (threadIdx.x == 64) {
                 if (stop) {  // let copies in flight land before the shared memory is released
