@@ -262,10 +262,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         float m = -INFINITY, l = 0.0f;
         float v[64];
         bool ok = true;
+        // a warp whose rows are all past the window's queries (the tile's padding) keeps step with
+        // the sub-blocks but computes nothing: its rows of P and O are never read
+        const bool live = warp * 32 < nq;
         for (int j = 0; j < nsub && ok; ++j) {
             const int sb = j % 2;
             ok = __all_sync(0xffffffffu, mbar_wait(&sfull[sb], static_cast<uint32_t>((j / 2) & 1), &s_abort, status));
             if (!ok) break;
+            if (!live) {
+                mbar_arrive(&pfull[sb]);
+                continue;
+            }
             tc_fence_after();
             const uint32_t ts = tS0 + static_cast<uint32_t>(sb * 64) + lane_off;
             tmem_ld_32x32(ts, v);
