@@ -997,21 +997,20 @@ __device__ __forceinline__ void chain_epilogue_dispatch(const ChainArgs& ca, int
     }
 }
 
-// Expand one 4-bit weight tile (see kQ4TileBytes) into the 128-byte-swizzled K-major bf16 image
-// the UMMA descriptor reads: thread t of the 128 writes row t, each weight bf16(d * (q - 8)).
-// 128 + q is built as a bf16 bit pattern (exponent of 128, q in the low mantissa bits), 136 is
-// subtracted exactly and the scale applied with one correctly rounded bf16 multiply.
-__device__ __forceinline__ void q4_expand_row(const uint8_t* __restrict__ raw, uint8_t* __restrict__ dst_tile, int t) {
+// Expand row t of one 4-bit weight tile (see kQ4TileBytes) into its 64 bf16 weights, as 32
+// pairs o[c][j] = (k = 8c + 2j, 8c + 2j + 1), each weight bf16(d * (q - 8)).  128 + q is built as
+// a bf16 bit pattern (exponent of 128, q in the low mantissa bits), 136 is subtracted exactly
+// and the scale applied with one correctly rounded bf16 multiply.
+__device__ __forceinline__ void q4_expand(const uint8_t* __restrict__ raw, int t, uint32_t (&o)[8][4]) {
     const uint32_t* codes = reinterpret_cast<const uint32_t*>(raw);
     const uint16_t* sc = reinterpret_cast<const uint16_t*>(raw + 4096);
-    // every load first (the raw slot and the A stage are both shared memory: loads issued after
-    // a store could not be moved above it), then the arithmetic of all eight chunks, then stores
+    // every load first (the raw slot and the A stage may both be shared memory: loads issued
+    // after a store could not be moved above it), then the arithmetic of all eight chunks
     uint32_t w[8];
 #pragma unroll
     for (int c = 0; c < 8; ++c) w[c] = codes[c * 128 + t];
     const uint32_t s0 = sc[t], s1 = sc[128 + t];
     const uint32_t d0 = s0 | (s0 << 16), d1 = s1 | (s1 << 16);  // (d, d) as bf16x2, per block of 32
-    uint32_t o[8][4];
 #pragma unroll
     for (int c = 0; c < 8; ++c) {
 #pragma unroll
@@ -1023,10 +1022,34 @@ __device__ __forceinline__ void q4_expand_row(const uint8_t* __restrict__ raw, u
             asm("mul.rn.bf16x2 %0, %1, %2;" : "=r"(o[c][j]) : "r"(x), "r"(c < 4 ? d0 : d1));  // * d: one rounding
         }
     }
+}
+
+// ... into the 128-byte-swizzled K-major bf16 image in shared memory the UMMA descriptor reads
+// (thread t of the 128 writes row t)
+__device__ __forceinline__ void q4_expand_row(const uint8_t* __restrict__ raw, uint8_t* __restrict__ dst_tile, int t) {
+    uint32_t o[8][4];
+    q4_expand(raw, t, o);
     uint8_t* row = dst_tile + t * 128;
 #pragma unroll
     for (int c = 0; c < 8; ++c)
         *reinterpret_cast<uint4*>(row + ((c ^ (t & 7)) << 4)) = make_uint4(o[c][0], o[c][1], o[c][2], o[c][3]);
+}
+
+// ... or into tensor memory, row r at lane r: 64 weights in 32 columns from taddr, the pair of
+// k = 2i, 2i + 1 in column i (the layout of an MMA's A operand read from tensor memory); the
+// calling warp's lanes are rows 32 (warp % 4) .. +31
+__device__ __forceinline__ void q4_expand_tmem(const uint8_t* __restrict__ raw, int r, uint32_t taddr) {
+    uint32_t o[8][4];
+    q4_expand(raw, r, o);
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, "
+        "%14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+        "r"(o[0][0]), "r"(o[0][1]), "r"(o[0][2]), "r"(o[0][3]), "r"(o[1][0]), "r"(o[1][1]), "r"(o[1][2]), "r"(o[1][3]),
+        "r"(o[2][0]), "r"(o[2][1]), "r"(o[2][2]), "r"(o[2][3]), "r"(o[3][0]), "r"(o[3][1]), "r"(o[3][2]), "r"(o[3][3]),
+        "r"(o[4][0]), "r"(o[4][1]), "r"(o[4][2]), "r"(o[4][3]), "r"(o[5][0]), "r"(o[5][1]), "r"(o[5][2]), "r"(o[5][3]),
+        "r"(o[6][0]), "r"(o[6][1]), "r"(o[6][2]), "r"(o[6][3]), "r"(o[7][0]), "r"(o[7][1]), "r"(o[7][2]), "r"(o[7][3])
+        : "memory");
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
 template <bool Q4>
@@ -1039,8 +1062,10 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
     // 4-bit weights: the operand (B) tiles have a ring of their own, deeper than the A stages
     const int SB = Q4 ? ca.b_stages : S;
     const uint32_t b_bytes = static_cast<uint32_t>(ca.ntile) * kBK * 2;
+    // 4-bit weights with the A stages in tensor memory (ca.a_tmem): no shared A stages
+    const bool a_tm = Q4 && ca.a_tmem;
     uint8_t* sA = smem;
-    uint8_t* sB = sA + static_cast<size_t>(S) * kABytes;
+    uint8_t* sB = sA + (a_tm ? 0 : static_cast<size_t>(S) * kABytes);
     uint8_t* sRaw = sB + static_cast<size_t>(SB) * b_bytes;  // 4-bit weight tiles (Q4)
     uint8_t* red_stage = sRaw + static_cast<size_t>(R) * kQ4TileBytes;
     float* tail = reinterpret_cast<float*>(red_stage + ca.red_bytes + ca.stg_bytes);
@@ -1295,10 +1320,12 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
     } else if (Q4 && warp >= kDeqWarp0) {
         // ---------------------------------------------------------- dequantizers (4-bit weights)
         // Every iteration: wait for its raw tile and for its A stage to be free (the MMAs that
-        // read the stage's previous tile are done), expand the tile (thread t: row t), make the
-        // writes visible to the tensor core's proxy, and arrive (one arrival per warp) on the
-        // stage's full barrier and on the raw slot's empty barrier.
-        const int t = threadIdx.x - kDeqWarp0 * 32;
+        // read the stage's previous tile are done), expand the tile, make the writes visible to
+        // the tensor cores, and arrive (one arrival per warp) on the stage's full barrier and on
+        // the raw slot's empty barrier.  Shared A stages: thread t writes row t; A stages in
+        // tensor memory: a warp writes the rows of its TMEM lane quarter, 32 (warp % 4) + lane.
+        const int t = a_tm ? (warp & 3) * 32 + lane : threadIdx.x - kDeqWarp0 * 32;
+        const uint32_t a_lane = static_cast<uint32_t>((warp & 3) * 32) << 16;
         int stage = 0, rs = 0;
         uint32_t par = 0, rpar = 0;
         bool stop = false;
@@ -1312,9 +1339,15 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                     stop = true;
                     break;
                 }
-                q4_expand_row(sRaw + static_cast<size_t>(rs) * kQ4TileBytes, sA + static_cast<size_t>(stage) * kABytes,
-                              t);
-                fence_proxy_async_smem();  // generic writes (and the raw reads) -> async-proxy accesses
+                if (a_tm) {
+                    q4_expand_tmem(sRaw + static_cast<size_t>(rs) * kQ4TileBytes, t,
+                                   tmem_base + a_lane + static_cast<uint32_t>(ca.a_col0 + stage * (kBK / 2)));
+                    tc_fence_before();  // the tensor-memory writes -> the MMA issuer's wait
+                } else {
+                    q4_expand_row(sRaw + static_cast<size_t>(rs) * kQ4TileBytes, sA + static_cast<size_t>(stage) * kABytes,
+                                  t);
+                    fence_proxy_async_smem();  // generic writes (and the raw reads) -> async-proxy accesses
+                }
                 __syncwarp();
                 if (lane == 0) {
                     mbar_arrive(&full[stage]);
@@ -1364,13 +1397,21 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                         if (tr && first) tr[kTrFirstData] = global_ns();
                         first = false;
                         tc_fence_after();
-                        const uint64_t adesc = sw128_kmajor_desc(smem_u32(sA + static_cast<size_t>(stage) * kABytes));
                         const uint64_t bdesc =
                             sw128_kmajor_desc(smem_u32(sB + static_cast<size_t>(Q4 ? bstage : stage) * b_bytes));
+                        if (a_tm) {  // A: 8 tensor-memory columns per 16-wide K step
+                            const uint32_t a_t = tmem_base + static_cast<uint32_t>(ca.a_col0 + stage * (kBK / 2));
 #pragma unroll
-                        for (int kk = 0; kk < kBK / 16; ++kk)
-                            umma_bf16(d_tmem, adesc + 2ull * kk, bdesc + 2ull * kk, idesc,
-                                      (k > k_lo || kk > 0) ? 1u : 0u);
+                            for (int kk = 0; kk < kBK / 16; ++kk)
+                                umma_bf16_tmem_a(d_tmem, a_t + static_cast<uint32_t>(kk * 8), bdesc + 2ull * kk, idesc,
+                                                 (k > k_lo || kk > 0) ? 1u : 0u);
+                        } else {
+                            const uint64_t adesc = sw128_kmajor_desc(smem_u32(sA + static_cast<size_t>(stage) * kABytes));
+#pragma unroll
+                            for (int kk = 0; kk < kBK / 16; ++kk)
+                                umma_bf16(d_tmem, adesc + 2ull * kk, bdesc + 2ull * kk, idesc,
+                                          (k > k_lo || kk > 0) ? 1u : 0u);
+                        }
                         issued = true;
                         umma_commit(&empty[stage]);
                         if (++stage == S) {
@@ -1552,12 +1593,18 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
     const int fixed0 = 1024 + (256 + 1024 + 256 + 128) * 4 + ca.red_bytes + ca.stg_bytes + 7 * 8 + 16;
     if (ca.q4) {
         // 4-bit weights (480 threads: no room beside the CTA for another one, so all of shared
-        // memory): raw 4.5 KB tiles, a few bf16 A stages the dequantizers fill, and a ring of
-        // operand tiles of its own, as deep as what is left allows (2 .. 24)
+        // memory): raw 4.5 KB tiles, a few bf16 A stages the dequantizers fill (in tensor memory
+        // where it has the room, else shared), and a ring of operand tiles of its own, as deep as
+        // what is left allows (2 .. 24)
         static const int kRaw[3] = {12, 8, 6}, kA[3] = {4, 3, 2};
         const int b_stage = ntile * kBK * 2 + 16;
+        const int a_col0 = 2 * ca.acc_cols + ca.x_cols;
+        ca.a_tmem = a_col0 + kA[0] * (kBK / 2) <= 512 ? 1 : 0;
+        ca.a_col0 = ca.a_tmem ? a_col0 : 0;
+        if (ca.a_tmem) ca.tmem_cols = pow2ceil(a_col0 + kA[0] * (kBK / 2));
         for (int i = 0; i < 3; ++i) {
-            const int fixed = fixed0 + kRaw[i] * (kQ4TileBytes + 16) + kA[i] * (static_cast<int>(kABytes) + 16);
+            const int a_bytes = ca.a_tmem ? 0 : static_cast<int>(kABytes);
+            const int fixed = fixed0 + kRaw[i] * (kQ4TileBytes + 16) + kA[i] * (a_bytes + 16);
             const int sb = (kFullSmem - fixed) / b_stage;
             if (sb >= 2 || i == 2) {
                 ca.raw_stages = kRaw[i];
@@ -1571,6 +1618,8 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
     }
     ca.raw_stages = 0;
     ca.b_stages = 0;
+    ca.a_tmem = 0;
+    ca.a_col0 = 0;
     // wide residual tiles read the old residual from global memory (a warp's 32 rows of a token
     // are one 128-byte line), not from a staged copy: the ring keeps the room
     const int fixed = fixed0;

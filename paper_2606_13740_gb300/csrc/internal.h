@@ -151,6 +151,9 @@ struct ChainArgs {
     // raw 4.5 KB tiles into raw_stages slots, four more warps expand each into the bf16 A stage
     // the tensor cores read, and the operand tiles go through a ring of b_stages of their own
     int q4, raw_stages, b_stages;  // b_stages: the operand ring of the 4-bit kernel
+    // 4-bit kernel: the expanded A stages in tensor memory from column a_col0 (32 columns per
+    // stage, the MMA reading A from there) instead of shared memory, where TMEM has the room
+    int a_tmem, a_col0;
     ChainPhase ph[kMaxPhases];
 };
 struct ChainMaps {
