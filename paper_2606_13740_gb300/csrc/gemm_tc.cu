@@ -1365,42 +1365,53 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
         }
     } else if (warp == 1) {
         // ---------------------------------------------------------- MMA issuer
-        if (lane == 0) {
-            const uint32_t idesc = umma_idesc_bf16(kBM, ca.ntile);
-            int stage = 0, bstage = 0;  // A stage; Q4: the operand's own ring
-            uint32_t par = 0, bpar = 0;
-            int acc = 0;
-            uint32_t acc_phase = 0;
-            bool issued = false;
-            for (int ph = 0; ph < ca.n_phases && !*s_abort; ++ph) {
-                const GemmPlan p = phase_plan(ca.ph[ph], rows);
-                if (static_cast<int>(blockIdx.x) >= p.grid) continue;
-                const long long it0 = range_begin(blockIdx.x, p.total, p.grid);
-                const long long it1 = range_begin(blockIdx.x + 1, p.total, p.grid);
-                unsigned long long* tr = ca.ph[ph].ep.trace ? ca.ph[ph].ep.trace + static_cast<size_t>(blockIdx.x) * kTrSlots : nullptr;
-                bool first = true;
-                for (long long it = it0; it < it1 && !*s_abort;) {
-                    const long long tile = it / p.kb;
-                    const int k_lo = static_cast<int>(it - tile * p.kb);
-                    const long long tend = (tile + 1) * p.kb;
-                    const int k_hi = static_cast<int>((it1 < tend ? it1 : tend) - tile * p.kb);
-                    if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, s_abort, status)) break;
+        // The whole warp runs the loop (its waits and their outcomes voted warp-wide), so that
+        // the tensor-memory addresses and shared-memory descriptors are warp-uniform values;
+        // one elected lane issues the MMAs and the commits.
+        const bool leader = elect_one();
+        const uint32_t tbase = __shfl_sync(0xffffffffu, tmem_base, 0);
+        const int urows = __shfl_sync(0xffffffffu, rows, 0);
+        const uint32_t idesc = umma_idesc_bf16(kBM, ca.ntile);
+        int stage = 0, bstage = 0;  // A stage; Q4: the operand's own ring
+        uint32_t par = 0, bpar = 0;
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        bool issued = false, stop = false;
+        for (int ph = 0; ph < ca.n_phases && !stop; ++ph) {
+            const GemmPlan p = phase_plan(ca.ph[ph], urows);
+            if (static_cast<int>(blockIdx.x) >= p.grid) continue;
+            const long long it0 = range_begin(blockIdx.x, p.total, p.grid);
+            const long long it1 = range_begin(blockIdx.x + 1, p.total, p.grid);
+            unsigned long long* tr =
+                (leader && ca.ph[ph].ep.trace) ? ca.ph[ph].ep.trace + static_cast<size_t>(blockIdx.x) * kTrSlots : nullptr;
+            bool first = true;
+            for (long long it = it0; it < it1;) {
+                const long long tile = it / p.kb;
+                const int k_lo = static_cast<int>(it - tile * p.kb);
+                const long long tend = (tile + 1) * p.kb;
+                const int k_hi = static_cast<int>((it1 < tend ? it1 : tend) - tile * p.kb);
+                if (__any_sync(0xffffffffu, *s_abort != 0) ||
+                    !__all_sync(0xffffffffu, mbar_wait(&tempty[acc], acc_phase ^ 1u, s_abort, status))) {
+                    stop = true;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d_tmem = tbase + static_cast<uint32_t>(acc * acc_cols);
+                for (int k = k_lo; k < k_hi; ++k) {
+                    const bool got = mbar_wait(&full[stage], par, s_abort, status) &&
+                                     (!Q4 || mbar_wait(&bfull[bstage], bpar, s_abort, status));
+                    if (!__all_sync(0xffffffffu, got)) {
+                        stop = true;
+                        break;
+                    }
+                    if (tr && first) tr[kTrFirstData] = global_ns();
+                    first = false;
                     tc_fence_after();
-                    const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * acc_cols);
-                    bool ok = true;
-                    for (int k = k_lo; k < k_hi; ++k) {
-                        if (!mbar_wait(&full[stage], par, s_abort, status) ||
-                            (Q4 && !mbar_wait(&bfull[bstage], bpar, s_abort, status))) {
-                            ok = false;
-                            break;
-                        }
-                        if (tr && first) tr[kTrFirstData] = global_ns();
-                        first = false;
-                        tc_fence_after();
-                        const uint64_t bdesc =
-                            sw128_kmajor_desc(smem_u32(sB + static_cast<size_t>(Q4 ? bstage : stage) * b_bytes));
+                    const uint64_t bdesc =
+                        sw128_kmajor_desc(smem_u32(sB + static_cast<size_t>(Q4 ? bstage : stage) * b_bytes));
+                    if (leader) {
                         if (a_tm) {  // A: 8 tensor-memory columns per 16-wide K step
-                            const uint32_t a_t = tmem_base + static_cast<uint32_t>(ca.a_col0 + stage * (kBK / 2));
+                            const uint32_t a_t = tbase + static_cast<uint32_t>(ca.a_col0 + stage * (kBK / 2));
 #pragma unroll
                             for (int kk = 0; kk < kBK / 16; ++kk)
                                 umma_bf16_tmem_a(d_tmem, a_t + static_cast<uint32_t>(kk * 8), bdesc + 2ull * kk, idesc,
@@ -1412,36 +1423,41 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                                 umma_bf16(d_tmem, adesc + 2ull * kk, bdesc + 2ull * kk, idesc,
                                           (k > k_lo || kk > 0) ? 1u : 0u);
                         }
-                        issued = true;
                         umma_commit(&empty[stage]);
-                        if (++stage == S) {
-                            stage = 0;
-                            par ^= 1u;
-                        }
-                        if constexpr (Q4) {
-                            umma_commit(&bempty[bstage]);
-                            if (++bstage == SB) {
-                                bstage = 0;
-                                bpar ^= 1u;
-                            }
+                        if constexpr (Q4) umma_commit(&bempty[bstage]);
+                    }
+                    __syncwarp();
+                    issued = true;
+                    if (++stage == S) {
+                        stage = 0;
+                        par ^= 1u;
+                    }
+                    if constexpr (Q4) {
+                        if (++bstage == SB) {
+                            bstage = 0;
+                            bpar ^= 1u;
                         }
                     }
-                    if (!ok) break;
-                    umma_commit(&tfull[acc]);
-                    if (++acc == 2) {
-                        acc = 0;
-                        acc_phase ^= 1u;
-                    }
-                    it = tile * p.kb + k_hi;
                 }
-                if (tr) tr[kTrLastData] = global_ns();
+                if (stop) break;
+                if (leader) umma_commit(&tfull[acc]);
+                __syncwarp();
+                if (++acc == 2) {
+                    acc = 0;
+                    acc_phase ^= 1u;
+                }
+                it = tile * p.kb + k_hi;
             }
-            if (*s_abort && issued) {
+            if (tr) tr[kTrLastData] = global_ns();
+        }
+        if (__any_sync(0xffffffffu, *s_abort != 0) && issued) {
+            if (leader) {  // the MMAs in flight finish before tensor memory is released
                 umma_commit(drain);
                 const long long t0 = spin_clock();
                 while (!mbar_try_wait(drain, 0) && spin_clock() - t0 < kWaitLimitCycles) {
                 }
             }
+            __syncwarp();
         }
     } else {
         // ---------------------------------------------------------- epilogue
