@@ -1166,8 +1166,10 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                 size_t woff = (static_cast<size_t>(mt) * p.kb + k) * tile_bytes;  // tile-major: (mt*kb + k) tiles
                 for (int it = it0; it < it1; ++it) {
                     if constexpr (Q4) {
-                        // the raw tile goes to its own ring; the dequantizing warps fill the A stage
-                        if (!mbar_wait(&rempty[stage], par ^ 1u, s_abort, status)) break;
+                        // the raw tile goes to its own ring; the dequantizing warps fill the A stage.
+                        // A stages in tensor memory: raw slot s belongs to A stage s, and is free
+                        // again once the MMAs that read that stage are done
+                        if (!mbar_wait(a_tm ? &empty[stage] : &rempty[stage], par ^ 1u, s_abort, status)) break;
                         mbar_arrive_expect_tx(&rfull[stage], kQ4TileBytes);
                         bulk_load_hint(sRaw + static_cast<size_t>(stage) * kQ4TileBytes, wt + woff, kQ4TileBytes,
                                        &rfull[stage], pol_w);
@@ -1334,20 +1336,35 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
             if (static_cast<int>(blockIdx.x) >= p.grid) continue;
             const int it0 = static_cast<int>(range_begin(blockIdx.x, p.total, p.grid));
             const int it1 = static_cast<int>(range_begin(blockIdx.x + 1, p.total, p.grid));
+            if (a_tm) {
+                // raw slot and A stage share one index: the raw tile's arrival implies that the
+                // MMAs which read the stage's previous tile are done (the producer loaded it only
+                // after their commit), so one wait and one arrival per tile
+                for (int it = it0; it < it1; ++it) {
+                    if (!mbar_wait(&rfull[stage], par, s_abort, status)) {
+                        stop = true;
+                        break;
+                    }
+                    tc_fence_after();
+                    q4_expand_tmem(sRaw + static_cast<size_t>(stage) * kQ4TileBytes, t,
+                                   tmem_base + a_lane + static_cast<uint32_t>(ca.a_col0 + stage * (kBK / 2)));
+                    tc_fence_before();  // the tensor-memory writes -> the MMA issuer's wait
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&full[stage]);
+                    if (++stage == S) {
+                        stage = 0;
+                        par ^= 1u;
+                    }
+                }
+                continue;
+            }
             for (int it = it0; it < it1; ++it) {
                 if (!mbar_wait(&rfull[rs], rpar, s_abort, status) || !mbar_wait(&empty[stage], par ^ 1u, s_abort, status)) {
                     stop = true;
                     break;
                 }
-                if (a_tm) {
-                    q4_expand_tmem(sRaw + static_cast<size_t>(rs) * kQ4TileBytes, t,
-                                   tmem_base + a_lane + static_cast<uint32_t>(ca.a_col0 + stage * (kBK / 2)));
-                    tc_fence_before();  // the tensor-memory writes -> the MMA issuer's wait
-                } else {
-                    q4_expand_row(sRaw + static_cast<size_t>(rs) * kQ4TileBytes, sA + static_cast<size_t>(stage) * kABytes,
-                                  t);
-                    fence_proxy_async_smem();  // generic writes (and the raw reads) -> async-proxy accesses
-                }
+                q4_expand_row(sRaw + static_cast<size_t>(rs) * kQ4TileBytes, sA + static_cast<size_t>(stage) * kABytes, t);
+                fence_proxy_async_smem();  // generic writes (and the raw reads) -> async-proxy accesses
                 __syncwarp();
                 if (lane == 0) {
                     mbar_arrive(&full[stage]);
@@ -1612,12 +1629,19 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
         // memory): raw 4.5 KB tiles, a few bf16 A stages the dequantizers fill (in tensor memory
         // where it has the room, else shared), and a ring of operand tiles of its own, as deep as
         // what is left allows (2 .. 24)
-        static const int kRaw[3] = {12, 8, 6}, kA[3] = {4, 3, 2};
+        int kRaw[3] = {12, 8, 6}, kA[3] = {4, 3, 2};
         const int b_stage = ntile * kBK * 2 + 16;
         const int a_col0 = 2 * ca.acc_cols + ca.x_cols;
-        ca.a_tmem = a_col0 + kA[0] * (kBK / 2) <= 512 ? 1 : 0;
+        // A stages in tensor memory where it holds at least 8 of them (then raw slots and A stages
+        // are one ring), else in shared memory beside a deeper raw ring
+        const int tm_stages = (512 - a_col0) / (kBK / 2);
+        ca.a_tmem = tm_stages >= 8 ? 1 : 0;
         ca.a_col0 = ca.a_tmem ? a_col0 : 0;
-        if (ca.a_tmem) ca.tmem_cols = pow2ceil(a_col0 + kA[0] * (kBK / 2));
+        if (ca.a_tmem) {
+            const int n = tm_stages < 12 ? tm_stages : 12;
+            for (int i = 0; i < 3; ++i) kRaw[i] = kA[i] = n - 2 * i;
+            ca.tmem_cols = pow2ceil(a_col0 + n * (kBK / 2));
+        }
         for (int i = 0; i < 3; ++i) {
             const int a_bytes = ca.a_tmem ? 0 : static_cast<int>(kABytes);
             const int fixed = fixed0 + kRaw[i] * (kQ4TileBytes + 16) + kA[i] * (a_bytes + 16);
