@@ -1037,10 +1037,9 @@ __device__ __forceinline__ void q4_expand_row(const uint8_t* __restrict__ raw, u
 
 // ... or into tensor memory, row r at lane r: 64 weights in 32 columns from taddr, the pair of
 // k = 2i, 2i + 1 in column i (the layout of an MMA's A operand read from tensor memory); the
-// calling warp's lanes are rows 32 (warp % 4) .. +31
-__device__ __forceinline__ void q4_expand_tmem(const uint8_t* __restrict__ raw, int r, uint32_t taddr) {
-    uint32_t o[8][4];
-    q4_expand(raw, r, o);
+// calling warp's lanes are rows 32 (warp % 4) .. +31.  The caller waits for the store
+// (tcgen05.wait::st) before it publishes the stage.
+__device__ __forceinline__ void tmem_st_row64(uint32_t taddr, const uint32_t (&o)[8][4]) {
     asm volatile(
         "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, "
         "%14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
@@ -1049,6 +1048,17 @@ __device__ __forceinline__ void q4_expand_tmem(const uint8_t* __restrict__ raw, 
         "r"(o[4][0]), "r"(o[4][1]), "r"(o[4][2]), "r"(o[4][3]), "r"(o[5][0]), "r"(o[5][1]), "r"(o[5][2]), "r"(o[5][3]),
         "r"(o[6][0]), "r"(o[6][1]), "r"(o[6][2]), "r"(o[6][3]), "r"(o[7][0]), "r"(o[7][1]), "r"(o[7][2]), "r"(o[7][3])
         : "memory");
+}
+
+// n (1 or 2) consecutive tiles of one raw slot into consecutive 32-column groups from taddr
+__device__ __forceinline__ void q4_expand_tmem(const uint8_t* __restrict__ raw, int r, uint32_t taddr, int n) {
+    uint32_t o[8][4];
+    q4_expand(raw, r, o);
+    tmem_st_row64(taddr, o);
+    if (n == 2) {
+        q4_expand(raw + kQ4TileBytes, r, o);
+        tmem_st_row64(taddr + 32, o);
+    }
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
@@ -1062,12 +1072,18 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
     // 4-bit weights: the operand (B) tiles have a ring of their own, deeper than the A stages
     const int SB = Q4 ? ca.b_stages : S;
     const uint32_t b_bytes = static_cast<uint32_t>(ca.ntile) * kBK * 2;
-    // 4-bit weights with the A stages in tensor memory (ca.a_tmem): no shared A stages
+    // 4-bit weights with the A stages in tensor memory (ca.a_tmem): no shared A stages, and a
+    // pipeline stage holds up to two consecutive k-blocks of one tile (kper): one wait, one
+    // arrival and one commit per role for both.  A tile's run of k-blocks in this CTA's range
+    // is cut into pairs from its start; an odd run ends with a stage of one.
     const bool a_tm = Q4 && ca.a_tmem;
+    const int kper = a_tm ? 2 : 1;
+    const uint32_t b_slot = b_bytes * static_cast<uint32_t>(kper);
+    const uint32_t raw_slot = kQ4TileBytes * static_cast<uint32_t>(kper);
     uint8_t* sA = smem;
     uint8_t* sB = sA + (a_tm ? 0 : static_cast<size_t>(S) * kABytes);
-    uint8_t* sRaw = sB + static_cast<size_t>(SB) * b_bytes;  // 4-bit weight tiles (Q4)
-    uint8_t* red_stage = sRaw + static_cast<size_t>(R) * kQ4TileBytes;
+    uint8_t* sRaw = sB + static_cast<size_t>(SB) * b_slot;  // 4-bit weight tiles (Q4)
+    uint8_t* red_stage = sRaw + static_cast<size_t>(R) * raw_slot;
     float* tail = reinterpret_cast<float*>(red_stage + ca.red_bytes + ca.stg_bytes);
     EpiSmem esm;
     esm.rs = tail;
@@ -1164,14 +1180,16 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                 int nt = tile / p.m_tiles, mt = tile - nt * p.m_tiles;
                 const char* wt = reinterpret_cast<const char*>(ca.ph[ph].w_tiles);
                 size_t woff = (static_cast<size_t>(mt) * p.kb + k) * tile_bytes;  // tile-major: (mt*kb + k) tiles
-                for (int it = it0; it < it1; ++it) {
+                for (int it = it0; it < it1;) {
+                    const int n = (a_tm && k + 1 < p.kb && it + 1 < it1) ? 2 : 1;  // k-blocks of this stage
                     if constexpr (Q4) {
                         // the raw tile goes to its own ring; the dequantizing warps fill the A stage.
                         // A stages in tensor memory: raw slot s belongs to A stage s, and is free
-                        // again once the MMAs that read that stage are done
+                        // again once the MMAs that read that stage are done; a pair of tiles of
+                        // one row block is one contiguous copy
                         if (!mbar_wait(a_tm ? &empty[stage] : &rempty[stage], par ^ 1u, s_abort, status)) break;
-                        mbar_arrive_expect_tx(&rfull[stage], kQ4TileBytes);
-                        bulk_load_hint(sRaw + static_cast<size_t>(stage) * kQ4TileBytes, wt + woff, kQ4TileBytes,
+                        mbar_arrive_expect_tx(&rfull[stage], n * kQ4TileBytes);
+                        bulk_load_hint(sRaw + static_cast<size_t>(stage) * raw_slot, wt + woff, n * kQ4TileBytes,
                                        &rfull[stage], pol_w);
                     } else {
                         if (!mbar_wait(&empty[stage], par ^ 1u, s_abort, status)) break;
@@ -1189,8 +1207,10 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                         stage = 0;
                         par ^= 1u;
                     }
-                    woff += tile_bytes;
-                    if (++k == p.kb) {
+                    it += n;
+                    woff += static_cast<size_t>(n) * tile_bytes;
+                    k += n;
+                    if (k == p.kb) {
                         k = 0;
                         if (++mt == p.m_tiles) {
                             mt = 0;
@@ -1242,15 +1262,16 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
             int mine_nt = -1;
             int tile = it0 / p.kb, k = it0 - tile * p.kb;
             int nt = tile / p.m_tiles, mt = tile - nt * p.m_tiles;
-            for (int it = it0; it < it1; ++it) {
+            for (int it = it0; it < it1;) {
+                const int n = (a_tm && k + 1 < p.kb && it + 1 < it1) ? 2 : 1;  // k-blocks of this stage
                 int free_stage = 1;
                 if (lane == 0) free_stage = mbar_wait(Q4 ? &bempty[stage] : &empty[stage], par ^ 1u, s_abort, status) ? 1 : 0;
                 if (!__shfl_sync(0xffffffffu, free_stage, 0)) {  // warp-uniform decision
                     stop = true;
                     break;
                 }
-                if (dep) {
-                    const int pmt = (k * kBK) / P.dep_rows;
+                for (int j = 0; dep && j < n; ++j) {
+                    const int pmt = ((k + j) * kBK) / P.dep_rows;
                     if (nt != mine_nt) {
                         mine = 0;
                         mine_nt = nt;
@@ -1284,22 +1305,26 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                         if (stop) break;
                     }
                 }
+                if (stop) break;
                 if (lane == 0) {
                     uint64_t* fb = Q4 ? &bfull[stage] : &full[stage];
                     if constexpr (Q4) {  // its own barrier; the A part of the stage arrives by the dequantizers
-                        mbar_arrive_expect_tx(fb, b_bytes);
+                        mbar_arrive_expect_tx(fb, n * b_bytes);
                         bpend |= 1u << stage;
                         bpend_par = (bpend_par & ~(1u << stage)) | (par << stage);
                     }
-                    tma_load_2d(sB + static_cast<size_t>(stage) * b_bytes, &maps.x[ph], k * kBK, nt * ca.ntile, fb,
-                                pol_x);
+                    for (int j = 0; j < n; ++j)
+                        tma_load_2d(sB + static_cast<size_t>(stage) * b_slot + static_cast<size_t>(j) * b_bytes, &maps.x[ph],
+                                    (k + j) * kBK, nt * ca.ntile, fb, pol_x);
                 }
                 __syncwarp();
                 if (++stage == SB) {
                     stage = 0;
                     par ^= 1u;
                 }
-                if (++k == p.kb) {
+                it += n;
+                k += n;
+                if (k == p.kb) {
                     k = 0;
                     if (++mt == p.m_tiles) {
                         mt = 0;
@@ -1337,17 +1362,19 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
             const int it0 = static_cast<int>(range_begin(blockIdx.x, p.total, p.grid));
             const int it1 = static_cast<int>(range_begin(blockIdx.x + 1, p.total, p.grid));
             if (a_tm) {
-                // raw slot and A stage share one index: the raw tile's arrival implies that the
-                // MMAs which read the stage's previous tile are done (the producer loaded it only
-                // after their commit), so one wait and one arrival per tile
-                for (int it = it0; it < it1; ++it) {
+                // raw slot and A stage share one index: the raw tiles' arrival implies that the
+                // MMAs which read the stage's previous tiles are done (the producer loaded them
+                // only after their commit), so one wait and one arrival per stage
+                int k = it0 - (it0 / p.kb) * p.kb;
+                for (int it = it0; it < it1;) {
+                    const int n = (k + 1 < p.kb && it + 1 < it1) ? 2 : 1;  // k-blocks of this stage
                     if (!mbar_wait(&rfull[stage], par, s_abort, status)) {
                         stop = true;
                         break;
                     }
                     tc_fence_after();
-                    q4_expand_tmem(sRaw + static_cast<size_t>(stage) * kQ4TileBytes, t,
-                                   tmem_base + a_lane + static_cast<uint32_t>(ca.a_col0 + stage * (kBK / 2)));
+                    q4_expand_tmem(sRaw + static_cast<size_t>(stage) * raw_slot, t,
+                                   tmem_base + a_lane + static_cast<uint32_t>(ca.a_col0 + stage * kBK), n);
                     tc_fence_before();  // the tensor-memory writes -> the MMA issuer's wait
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&full[stage]);
@@ -1355,6 +1382,9 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                         stage = 0;
                         par ^= 1u;
                     }
+                    it += n;
+                    k += n;
+                    if (k == p.kb) k = 0;
                 }
                 continue;
             }
@@ -1414,7 +1444,8 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                 }
                 tc_fence_after();
                 const uint32_t d_tmem = tbase + static_cast<uint32_t>(acc * acc_cols);
-                for (int k = k_lo; k < k_hi; ++k) {
+                for (int k = k_lo; k < k_hi;) {
+                    const int n = (a_tm && k + 1 < k_hi) ? 2 : 1;  // k-blocks of this stage
                     const bool got = mbar_wait(&full[stage], par, s_abort, status) &&
                                      (!Q4 || mbar_wait(&bfull[bstage], bpar, s_abort, status));
                     if (!__all_sync(0xffffffffu, got)) {
@@ -1424,15 +1455,22 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                     if (tr && first) tr[kTrFirstData] = global_ns();
                     first = false;
                     tc_fence_after();
-                    const uint64_t bdesc =
-                        sw128_kmajor_desc(smem_u32(sB + static_cast<size_t>(Q4 ? bstage : stage) * b_bytes));
+                    const uint8_t* b_st = sB + static_cast<size_t>(Q4 ? bstage : stage) * b_slot;
+                    const uint64_t bdesc = sw128_kmajor_desc(smem_u32(b_st));
                     if (leader) {
-                        if (a_tm) {  // A: 8 tensor-memory columns per 16-wide K step
-                            const uint32_t a_t = tbase + static_cast<uint32_t>(ca.a_col0 + stage * (kBK / 2));
+                        if (a_tm) {  // A: 8 tensor-memory columns per 16-wide K step, 32 per k-block
+                            const uint32_t a_t = tbase + static_cast<uint32_t>(ca.a_col0 + stage * kBK);
 #pragma unroll
                             for (int kk = 0; kk < kBK / 16; ++kk)
                                 umma_bf16_tmem_a(d_tmem, a_t + static_cast<uint32_t>(kk * 8), bdesc + 2ull * kk, idesc,
                                                  (k > k_lo || kk > 0) ? 1u : 0u);
+                            if (n == 2) {
+                                const uint64_t bdesc1 = sw128_kmajor_desc(smem_u32(b_st + b_bytes));
+#pragma unroll
+                                for (int kk = 0; kk < kBK / 16; ++kk)
+                                    umma_bf16_tmem_a(d_tmem, a_t + static_cast<uint32_t>(32 + kk * 8), bdesc1 + 2ull * kk,
+                                                     idesc, 1u);
+                            }
                         } else {
                             const uint64_t adesc = sw128_kmajor_desc(smem_u32(sA + static_cast<size_t>(stage) * kABytes));
 #pragma unroll
@@ -1455,6 +1493,7 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                             bpar ^= 1u;
                         }
                     }
+                    k += n;
                 }
                 if (stop) break;
                 if (leader) umma_commit(&tfull[acc]);
@@ -1629,22 +1668,29 @@ bool chain_plan(ChainArgs& ca, int smem_budget) {
         // memory): raw 4.5 KB tiles, a few bf16 A stages the dequantizers fill (in tensor memory
         // where it has the room, else shared), and a ring of operand tiles of its own, as deep as
         // what is left allows (2 .. 24)
-        int kRaw[3] = {12, 8, 6}, kA[3] = {4, 3, 2};
+        const int kRaw[3] = {12, 8, 6}, kA[3] = {4, 3, 2};
         const int b_stage = ntile * kBK * 2 + 16;
         const int a_col0 = 2 * ca.acc_cols + ca.x_cols;
-        // A stages in tensor memory where it holds at least 8 of them (then raw slots and A stages
-        // are one ring), else in shared memory beside a deeper raw ring
-        const int tm_stages = (512 - a_col0) / (kBK / 2);
-        ca.a_tmem = tm_stages >= 8 ? 1 : 0;
+        // A stages in tensor memory where it holds at least 4 stages of two k-blocks (64 columns
+        // each): then raw slots (two tiles each) and A stages are one ring of up to 6 stages, and
+        // the operand ring holds up to 12 stages of two k-blocks
+        const int tm_stages = (512 - a_col0) / kBK;
+        ca.a_tmem = tm_stages >= 4 ? 1 : 0;
         ca.a_col0 = ca.a_tmem ? a_col0 : 0;
         if (ca.a_tmem) {
-            const int n = tm_stages < 12 ? tm_stages : 12;
-            for (int i = 0; i < 3; ++i) kRaw[i] = kA[i] = n - 2 * i;
-            ca.tmem_cols = pow2ceil(a_col0 + n * (kBK / 2));
+            const int n = tm_stages < 6 ? tm_stages : 6;
+            const int per_raw = 2 * kQ4TileBytes + 16 + 16;
+            const int per_b = 2 * ntile * kBK * 2 + 16;
+            int sb = (kFullSmem - fixed0 - n * per_raw) / per_b;
+            if (sb > 12) sb = 12;
+            ca.tmem_cols = pow2ceil(a_col0 + n * kBK);
+            ca.raw_stages = ca.stages = n;
+            ca.b_stages = sb;
+            ca.smem = static_cast<size_t>(fixed0) + static_cast<size_t>(n) * per_raw + static_cast<size_t>(sb) * per_b;
+            return sb >= 2 && ca.smem <= static_cast<size_t>(kFullSmem);
         }
         for (int i = 0; i < 3; ++i) {
-            const int a_bytes = ca.a_tmem ? 0 : static_cast<int>(kABytes);
-            const int fixed = fixed0 + kRaw[i] * (kQ4TileBytes + 16) + kA[i] * (a_bytes + 16);
+            const int fixed = fixed0 + kRaw[i] * (kQ4TileBytes + 16) + kA[i] * (static_cast<int>(kABytes) + 16);
             const int sb = (kFullSmem - fixed) / b_stage;
             if (sb >= 2 || i == 2) {
                 ca.raw_stages = kRaw[i];

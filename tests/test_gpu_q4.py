@@ -42,11 +42,14 @@ def test_q4_weights_dequantise_to_the_oracles(pkg):
     ctx.close()
 
 
-def test_q4_blockwise_teacher_forced(pkg):
+@pytest.mark.parametrize("n_prompt", [64, 192])
+def test_q4_blockwise_teacher_forced(pkg, n_prompt):
+    """The 4-bit block loop against the oracle; a 192-token prompt puts the prefill on token
+    tiles too wide for tensor-memory A stages (the shared-memory stages and their own rings)."""
     from test_gpu_step import _run_teacher_forced
     model = O.Model(O.OracleConfig(weight_bits=4))
-    prompt = I.uniform_prompt(64, 1024, 1023, seed=31)
-    ctx = pkg.Context(pkg.Config(max_ctx=256, max_window=160, weight_bits=4))
+    prompt = I.uniform_prompt(n_prompt, 1024, 1023, seed=31)
+    ctx = pkg.Context(pkg.Config(max_ctx=n_prompt + 192, max_window=192, weight_bits=4))
     kw = dict(steps_per_block=8, theta_remask=0.5, remask_max=1, spec_blocks=1, spec_trigger=16)
     sess, steps, worst = _run_teacher_forced(model, O.OracleSched(**kw), pkg.Sched(**kw), prompt, 96, ctx)
     assert steps >= 24
