@@ -1256,6 +1256,7 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
             const int it1 = static_cast<int>(range_begin(blockIdx.x + 1, p.total, p.grid));
             const int* dep = (ph > 0 && P.dep_rows > 0) ? ca.ph[ph - 1].done : nullptr;
             const int dep_tiles = dep ? ca.ph[ph - 1].p.m_tiles : 0;
+            const int dep_shift = dep ? 31 - __clz(P.dep_rows) : 0;  // dep_rows is a power of two
             // completion of the previous phase's tiles for token tile mine_nt, as far as seen:
             // lane l, bit w = tile 32w + l (a flag, once complete, stays so for the launch)
             uint32_t mine = 0;
@@ -1271,7 +1272,7 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                     break;
                 }
                 for (int j = 0; dep && j < n; ++j) {
-                    const int pmt = ((k + j) * kBK) / P.dep_rows;
+                    const int pmt = ((k + j) * kBK) >> dep_shift;
                     if (nt != mine_nt) {
                         mine = 0;
                         mine_nt = nt;
@@ -1729,7 +1730,8 @@ cudaError_t chain_init_attrs() {
 cudaError_t chain_launch(const ChainMaps& maps, const ChainArgs& ca, cudaStream_t st, bool pdl) {
     for (int i = 0; i < ca.n_phases; ++i) {
         const GemmPlan& p = ca.ph[i].p;
-        if (p.grid > ca.grid || !ca.ph[i].partials || !ca.ph[i].tickets || (i > 0 && ca.ph[i].dep_rows < 0))
+        const int dr = ca.ph[i].dep_rows;
+        if (p.grid > ca.grid || !ca.ph[i].partials || !ca.ph[i].tickets || (i > 0 && (dr < 0 || (dr & (dr - 1)) != 0)))
             return cudaErrorInvalidValue;
     }
     // a device-resolved row count changes a phase's tiling: no later phase may wait on its flags

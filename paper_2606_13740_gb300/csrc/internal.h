@@ -115,7 +115,7 @@ struct ChainPhase {
     GemmPlan p;          // from gemm_plan (grid <= the chain's grid)
     EpiArgs ep;
     int epi;             // EpiKind
-    int dep_rows;        // X k-block k comes from tile (64k)/dep_rows of the previous phase; 0: ready at launch
+    int dep_rows;        // X k-block k comes from tile (64k)/dep_rows of the previous phase (a power of two); 0: ready at launch
     int* done;           // [m_tiles][n_tiles] completion flags (value: the launch's tag); may be null
     // residual phases: done = the bf16 operand is written, done2 = also the fp32 residual and
     // the RMSNorm sums (what the later phases' epilogues read); null: done covers both
