@@ -151,8 +151,10 @@ struct ChainArgs {
     // raw 4.5 KB tiles into raw_stages slots, four more warps expand each into the bf16 A stage
     // the tensor cores read, and the operand tiles go through a ring of b_stages of their own
     int q4, raw_stages, b_stages;  // b_stages: the operand ring of the 4-bit kernel
-    // 4-bit kernel: the expanded A stages in tensor memory from column a_col0 (32 columns per
-    // stage, the MMA reading A from there) instead of shared memory, where TMEM has the room
+    // 4-bit kernel: the expanded A stages in tensor memory from column a_col0 instead of shared
+    // memory, where TMEM has the room; a stage there holds two consecutive k-blocks of a tile
+    // (64 columns, the MMA reading A from there; raw slots of two tiles, raw_stages ==
+    // stages, and operand stages of two k-blocks)
     int a_tmem, a_col0;
     ChainPhase ph[kMaxPhases];
 };
