@@ -1234,11 +1234,15 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
         }
     } else if (warp == 6) {
         // ---------------------------------------------------------- operand producer
-        // The whole warp runs the loop: lane 0 issues the copies, and the completion flags of
-        // the producing tiles are polled 32 at a time (one round trip covers the next 32).
+        // The whole warp runs the loop: its slot waits are voted warp-wide, so that the copy
+        // coordinates stay warp-uniform values, one elected lane issues the copies, and the
+        // completion flags of the producing tiles are polled 32 at a time (one round trip
+        // covers the next 32).
         const uint64_t pol_x = policy_evict_last();
         pdl_wait();
         const int tag = chain_tag(ca);
+        const bool leader = elect_one();
+        const int urows = __shfl_sync(0xffffffffu, rows, 0);
         int stage = 0;
         uint32_t par = 0;
         uint32_t bpend = 0, bpend_par = 0;  // Q4: operand copies issued (for the drain on abort)
@@ -1250,7 +1254,7 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
         }
         for (int ph = 0; ph < ca.n_phases && !stop; ++ph) {
             const ChainPhase& P = ca.ph[ph];
-            const GemmPlan p = phase_plan(P, rows);
+            const GemmPlan p = phase_plan(P, urows);
             if (static_cast<int>(blockIdx.x) >= p.grid) continue;
             const int it0 = static_cast<int>(range_begin(blockIdx.x, p.total, p.grid));
             const int it1 = static_cast<int>(range_begin(blockIdx.x + 1, p.total, p.grid));
@@ -1265,9 +1269,7 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
             int nt = tile / p.m_tiles, mt = tile - nt * p.m_tiles;
             for (int it = it0; it < it1;) {
                 const int n = (a_tm && k + 1 < p.kb && it + 1 < it1) ? 2 : 1;  // k-blocks of this stage
-                int free_stage = 1;
-                if (lane == 0) free_stage = mbar_wait(Q4 ? &bempty[stage] : &empty[stage], par ^ 1u, s_abort, status) ? 1 : 0;
-                if (!__shfl_sync(0xffffffffu, free_stage, 0)) {  // warp-uniform decision
+                if (!__all_sync(0xffffffffu, mbar_wait(Q4 ? &bempty[stage] : &empty[stage], par ^ 1u, s_abort, status))) {
                     stop = true;
                     break;
                 }
@@ -1307,7 +1309,7 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
                     }
                 }
                 if (stop) break;
-                if (lane == 0) {
+                if (leader) {
                     uint64_t* fb = Q4 ? &bfull[stage] : &full[stage];
                     if constexpr (Q4) {  // its own barrier; the A part of the stage arrives by the dequantizers
                         mbar_arrive_expect_tx(fb, n * b_bytes);
@@ -1337,7 +1339,7 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
         if constexpr (Q4) {
             // the operand ring is this warp's alone: on an abort, let its copies in flight land
             // before the CTA's shared memory is released (one deadline for all)
-            if (lane == 0 && *s_abort) {
+            if (leader && *s_abort) {
                 const long long t0 = spin_clock();
                 for (int b = 0; b < SB; ++b)
                     while ((bpend >> b & 1u) && !mbar_try_wait(&bfull[b], (bpend_par >> b) & 1u) &&
