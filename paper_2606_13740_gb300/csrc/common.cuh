@@ -371,10 +371,10 @@ __device__ __forceinline__ bool elect_lane0() { return (threadIdx.x & 31) == 0; 
 // One lane of the converged warp, chosen by elect.sync: the issuing thread of a loop the whole
 // warp runs, so that the addresses and descriptors it passes stay warp-uniform values.
 __device__ __forceinline__ bool elect_one() {
-    uint32_t lane_id, is_leader;
+    [[maybe_unused]] uint32_t lane_id;
+    uint32_t is_leader;
     asm volatile("{\n .reg .pred p;\n elect.sync %0|p, 0xffffffff;\n selp.u32 %1, 1, 0, p;\n}\n"
                  : "=r"(lane_id), "=r"(is_leader));
-    (void)lane_id;
     return is_leader != 0;
 }
 

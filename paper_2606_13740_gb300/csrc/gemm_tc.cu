@@ -527,11 +527,12 @@ __device__ __forceinline__ void epilogue_c32(const EpiArgs& ep, const GemmPlan& 
 // threads): warp 0 = weight producer (never waits on data: weights are constant, so it runs
 // ahead by the whole ring, across phase boundaries), warp 6 = operand producer (waits for
 // the completion flag of the tile that writes each X k-block), warp 1 = TMEM owner and MMA
-// issuer, warps 2..5 and 7..10 = epilogue (two warps per TMEM lane quarter).  Ring stages,
+// issuer, warps 2..5 and 7..10 = epilogue (two warps per TMEM lane quarter).  The operand
+// producer's and the MMA issuer's loops run warp-wide, one elected lane issuing.  Ring stages,
 // TMEM accumulators and their barriers are shared by all phases; a running iteration counter
 // gives every stage its use parity.
 constexpr int kChainThreads = 64 + 32 + 32 * kEpiWarps;
-// 4-bit weights: warps 11..14 expand each raw tile into the bf16 A stage
+// 4-bit weights: warps 11..14 expand the raw tiles into the bf16 A stages
 constexpr int kDeqWarp0 = 11, kDeqWarps = 4;
 constexpr int kChainThreadsQ4 = kChainThreads + 32 * kDeqWarps;
 constexpr int kMaxDepTiles = 1024;  // the operand producer keeps a readiness bit per producing tile: 32 per lane
@@ -1349,11 +1350,11 @@ __global__ void __launch_bounds__(Q4 ? kChainThreadsQ4 : kChainThreads, 1)
         }
     } else if (Q4 && warp >= kDeqWarp0) {
         // ---------------------------------------------------------- dequantizers (4-bit weights)
-        // Every iteration: wait for its raw tile and for its A stage to be free (the MMAs that
-        // read the stage's previous tile are done), expand the tile, make the writes visible to
-        // the tensor cores, and arrive (one arrival per warp) on the stage's full barrier and on
-        // the raw slot's empty barrier.  Shared A stages: thread t writes row t; A stages in
-        // tensor memory: a warp writes the rows of its TMEM lane quarter, 32 (warp % 4) + lane.
+        // Every stage: wait for its raw tiles (shared A stages: and for the stage to be free),
+        // expand them, make the writes visible to the tensor cores, and arrive (one arrival per
+        // warp) on the stage's full barrier (shared A stages: and on the raw slot's empty
+        // barrier).  Shared A stages: thread t writes row t; A stages in tensor memory: a warp
+        // writes the rows of its TMEM lane quarter, 32 (warp % 4) + lane.
         const int t = a_tm ? (warp & 3) * 32 + lane : threadIdx.x - kDeqWarp0 * 32;
         const uint32_t a_lane = static_cast<uint32_t>((warp & 3) * 32) << 16;
         int stage = 0, rs = 0;
